@@ -1,0 +1,53 @@
+"""The pins must catch plausible mistakes in the oracle.
+
+Each case plants one mistake in a copy of oracle.cpp (on the CPU, in a
+temporary directory), builds it, and runs the pin suite against that build in
+a subprocess; the suite must fail.
+"""
+import os
+import subprocess
+import sys
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+MUTATIONS = {
+    "backoff weight dropped": ("double b = (j >= 0) ? bow[len - 1][(size_t)j] : 0.0;", "double b = 0.0;"),
+    "backoff to the wrong suffix": ("return b + score_ctx(h + 1, len - 1, v);",
+                                    "return b + score_ctx(h, len - 1, v);"),
+    "W_out read transposed": (
+        "const uint16_t* wk = m.W + (size_t)k * N;\n"
+        "    for (int32_t v = 0; v < N; ++v) logits[(size_t)v] += xk * (double)bf16_bits_to_float(wk[v]);",
+        "for (int32_t v = 0; v < N; ++v) logits[(size_t)v] += "
+        "xk * (double)bf16_bits_to_float(m.W[((size_t)v * H + k) % ((size_t)H * N)]);"),
+    "blank gets an LM score": ("fused[(size_t)V] = logits[(size_t)V] - lse;\n}",
+                               "fused[(size_t)V] = logits[(size_t)V] - lse + "
+                               "(lm ? lambda * lm->score(y, ylen, 0) : 0.0);\n}"),
+    "ReLU missing": ("if (s < 0.0f) s = 0.0f;", ""),
+    "no restart after a phrase": (
+        "if (l > 0 && b->is_phrase(g + (len - l), l)) h.rho = (int64_t)h.y.size();", "(void)l;"),
+    "log-softmax sign": ("double f = logits[(size_t)v] - lse;", "double f = logits[(size_t)v] + lse;"),
+    "beam without merging": ("if (o.y == h.y) {", "if (false) {"),
+    "LM state takes the shortest suffix": ("for (int64_t l = n; l >= 1; --l) {\n      if (find(hist",
+                                           "for (int64_t l = 1; l <= n; ++l) {\n      if (find(hist"),
+    "failed match not cancelled": (
+        "return bonus * (double)(match(gv.data(), len + 1) - match(g, len));",
+        "return bonus * (double)std::max(0, match(gv.data(), len + 1) - match(g, len));"),
+}
+
+
+@pytest.mark.parametrize("name", sorted(MUTATIONS))
+def test_pins_catch_planted_mistake(name, tmp_path):
+    src = open(os.path.join(ROOT, "oracle", "oracle.cpp")).read()
+    a, b = MUTATIONS[name]
+    assert a in src, "mutation anchor not found; update the mutation list"
+    cpp = tmp_path / "mutant.cpp"
+    cpp.write_text(src.replace(a, b))
+    so = tmp_path / "mutant.so"
+    subprocess.check_call(["g++", "-O1", "-std=c++17", "-ffp-contract=off", "-shared", "-fPIC", str(cpp), "-o",
+                           str(so)])
+    r = subprocess.run([sys.executable, "-m", "pytest", os.path.join(ROOT, "tests", "test_oracle_pins.py"), "-q",
+                        "-x", "-p", "no:cacheprovider"], cwd=ROOT, capture_output=True, text=True,
+                       env=dict(os.environ, TSD_ORACLE_LIB=str(so)), timeout=600)
+    assert r.returncode != 0, f"pins did not catch: {name}\n{r.stdout[-2000:]}"
