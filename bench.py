@@ -1,0 +1,337 @@
+"""Benchmark of the fused streaming decode step (one JSON line on stdout).
+
+A step is one decode_chunk call: a 13-frame encoder chunk (the paper's
+1040 ms look-ahead at 80 ms frames) for all B streams, through the whole hot
+path -- joint GEMM, log-softmax, LM and phrase-boost fusion, greedy
+selection and state advance, T*max_symbols label steps.
+
+Workload (default): B=256 streams, H=1024, V=1024+blank (0.6B-model-sized
+joint), 6-gram LM with ~20M n-grams, 5,000 boost phrases, lambda=0.5,
+beta=1.5, greedy with at most 5 labels per frame; synthetic seeded data.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+The reference arm (--impl reference) times the CPU oracle on this host's
+cores on a bounded sample of the same workload and reports the same metric.
+Under torchrun each rank decodes its own B streams (streams are independent:
+weak scaling, no collective on the data path); rank 0 prints.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import synth  # noqa: E402
+
+METRIC = "fused decode encoder-frames/sec over B streams"
+UNIT = "frames/s"
+PEAKS_FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+
+def peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return d, "measured"
+    return dict(PEAKS_FALLBACK), "fallback"
+
+
+def workload_config(w: synth.Workload, lm_total: int, n_phr: int):
+    return {"workload": f"cfg{w.cfg} {w.name}", "B_per_gpu": w.B, "T": w.T, "H": w.H, "V": w.V,
+            "lm_order": w.lm_order, "lm_ngrams": lm_total, "boost_phrases": n_phr, "lambda": w.lam,
+            "beta": w.beta, "max_symbols": w.max_sym, "beam": w.beam,
+            "data": "synthetic seeded (Philox4x32-10): enc, E ~ N(0,1), W_out ~ N(0, 3/sqrt(H)); "
+                    "normalized absolute-discount backoff LM over Zipf unigrams; random phrases"}
+
+
+class Clocks:
+    """Samples SM clocks and throttle reasons with nvidia-smi during a region."""
+
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+         "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+         "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.lines = []
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.Q}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t.start()
+        except (OSError, FileNotFoundError):
+            self.proc = None
+        return self
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def __exit__(self, *a):
+        if self.proc:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self):
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            parts = [p.strip() for p in ln.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                mx.append(float(parts[2]))
+            except ValueError:
+                continue
+            for nm, v in zip(names, parts[5:9]):
+                if v.lower() in ("active", "0x1", "1", "yes"):
+                    reasons.add(nm)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"], "samples": 0}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def _dist():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+def oracle_baseline(w, inp_lm, inp_ph, E, W, streams, chunks, threads=None):
+    """Times the oracle (as it stands) decoding `streams` x `chunks` of the
+    workload on this host's cores; returns (frames/s, cores, sample text)."""
+    import concurrent.futures
+
+    import oracle
+
+    threads = threads or len(os.sched_getaffinity(0))
+    olm = oracle.LM.from_arrays(inp_lm) if inp_lm is not None else None
+    obo = oracle.Boost.from_phrases(w.V, inp_ph, w.bonus) if inp_ph is not None else None
+    model = oracle.Model(w.V, w.H, E, W)
+    encs = {c: synth.enc_chunk(w, streams, c) for c in range(chunks)}
+
+    def one(i):
+        st = oracle.Stream(w.V)
+        for c in range(chunks):
+            oracle.decode_chunk(st, model, olm, obo, encs[c][i], w.lam, w.beta, w.max_sym)
+
+    t0 = time.perf_counter()
+    with concurrent.futures.ThreadPoolExecutor(max_workers=threads) as ex:
+        list(ex.map(one, range(len(streams))))
+    dt = time.perf_counter() - t0
+    frames = len(streams) * chunks * w.T
+    used = min(threads, len(streams))
+    sample = f"{len(streams)} streams x {chunks} chunks x {w.T} frames of the same workload ({frames} frames)"
+    return frames / dt, used, sample, dt
+
+
+def run_reference(args, w):
+    """The reference arm: the CPU oracle on this host's cores."""
+    ws, rank, _ = _dist()
+    if rank != 0:
+        return
+    lmA = synth.lm_for(w)
+    ph = synth.phrases_for(w)
+    E, W = synth.joint_weights(w)
+    n_str = args.ref_streams
+    # warm-up steps, then K timed steps; each step decodes a bounded sample
+    for _ in range(args.warmup):
+        oracle_baseline(w, lmA, ph, E, W, list(range(2)), 1)
+    vals, dts = [], []
+    for k in range(args.steps):
+        v, cores, sample, dt = oracle_baseline(w, lmA, ph, E, W, list(range(k * n_str, (k + 1) * n_str)), 1)
+        vals.append(v)
+        dts.append(dt)
+    value = float(np.mean(vals))
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000 * float(np.mean(dts)),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "config": workload_config(w, lmA.total, ph.n if ph else 0),
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
+                             "sample": f"per step: {sample}"},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def run_ours(args, w):
+    import torch
+
+    import paper_2609_14991_gb300 as tsd
+
+    ws, rank, local = _dist()
+    if ws > 1:
+        import torch.distributed as dist
+
+        dist.init_process_group("nccl" if torch.cuda.is_available() else "gloo")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    stream = torch.cuda.current_stream()
+
+    lmA = synth.lm_for(w)
+    ph = synth.phrases_for(w)
+    E, W = synth.joint_weights(w)
+    streams = list(range(rank * w.B, (rank + 1) * w.B))  # this rank's streams
+    lm = tsd.NGram.from_arrays(lmA) if lmA is not None else None
+    bo = tsd.Boost.from_phrases(w.V, ph, w.bonus) if ph is not None else None
+    dec = tsd.Decoder(w.V, w.H, torch.from_numpy(W.view(np.int16)).to(dev), torch.from_numpy(E.view(np.int16)).to(dev),
+                      lm=lm, boost=bo, max_symbols=w.max_sym, beam_k=w.beam, max_streams=w.B, max_T=w.T)
+    slots = [dec.open() for _ in range(w.B)]
+    slots_np = np.array(slots, dtype=np.int32)
+    n_chunks = args.warmup + args.steps
+    encs = [torch.from_numpy(synth.enc_chunk(w, streams, c % w.chunks).view(np.int16)).to(dev)
+            for c in range(n_chunks)]
+    out = dec.alloc_out(w.B, w.T)
+    outp = (out.tokens.data_ptr(), out.frames.data_ptr(), out.scores.data_ptr(), out.counts.data_ptr())
+    sh = stream.cuda_stream
+    flush = torch.empty(256 * 1024 * 1024, dtype=torch.uint8, device=dev)  # > 129 MB L2
+
+    def step(c):
+        dec.decode_chunk_raw(slots_np, encs[c].data_ptr(), w.T, w.lam, w.beta, outp, sh)
+
+    def barrier():
+        torch.cuda.synchronize()
+        if ws > 1:
+            import torch.distributed as dist
+
+            dist.barrier()
+        torch.cuda.synchronize()
+
+    for c in range(args.warmup):
+        step(c)
+    barrier()
+    dec.timing(reset=True)
+    dec.set_timing(True)
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    with Clocks(local) as clk:
+        barrier()
+        t0 = time.perf_counter()
+        for k in range(args.steps):
+            flush.zero_()  # L2 flush, outside the step's events
+            starts[k].record(stream)
+            step(args.warmup + k)
+            ends[k].record(stream)
+        barrier()
+        wall = time.perf_counter() - t0
+    dec.set_timing(False)
+    step_ms = [s.elapsed_time(e) for s, e in zip(starts, ends)]
+    kernel_ms, kernel_n = dec.timing(reset=True)
+    t_ms = float(sum(step_ms))
+    if ws > 1:
+        import torch.distributed as dist
+
+        tt = torch.tensor([t_ms], dtype=torch.float64, device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        t_ms = float(tt.item())
+    frames = ws * w.B * w.T * args.steps
+    value = frames / (t_ms / 1000.0)
+
+    # end to end through the public API with host buffers: H2D of the chunk
+    # from pinned memory, the decode, D2H of every output, inside the region
+    host_enc = [e.cpu().pin_memory() for e in encs[-min(len(encs), 8):]]
+    dev_enc = torch.empty_like(encs[0])
+    host_out = [torch.empty(t.shape, dtype=t.dtype, pin_memory=True) for t in
+                (out.tokens, out.frames, out.scores, out.counts)]
+    e2e_steps = min(args.steps, 8)
+    barrier()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for k in range(e2e_steps):
+        dev_enc.copy_(host_enc[k % len(host_enc)], non_blocking=True)
+        dec.decode_chunk_raw(slots_np, dev_enc.data_ptr(), w.T, w.lam, w.beta, outp, sh)
+        for h, d in zip(host_out, (out.tokens, out.frames, out.scores, out.counts)):
+            h.copy_(d, non_blocking=True)
+    e1.record(stream)
+    barrier()
+    e2e_ms = e0.elapsed_time(e1)
+    h2d = int(dev_enc.numel() * dev_enc.element_size())
+    d2h = int(sum(h.numel() * h.element_size() for h in host_out))
+    e2e_val = ws * w.B * w.T * e2e_steps / (e2e_ms / 1000.0)
+
+    if rank != 0:
+        return
+    pk, pk_kind = peaks()
+    S = w.T * w.max_sym
+    # dominant kernel by device time
+    joint_avg_ms = kernel_ms["joint"] / max(1, kernel_n["joint"])
+    row_avg_ms = kernel_ms["row"] / max(1, kernel_n["row"])
+    flop_per_launch = 2.0 * w.B * w.beam * w.H * (w.V + 1)
+    roof = {"kernel": "joint GEMM + fused log-softmax/selection epilogue", "bound": "tensor",
+            "achieved": flop_per_launch / (joint_avg_ms / 1000.0) / 1e12,
+            "peak": pk.get("bf16_tflops_sustained", pk["bf16_tflops"]), "unit": "TFLOP/s",
+            "traffic": None, "peak_kind": f"{pk_kind} bf16 sustained (kernel timed inside a long step)",
+            "algorithmic": f"2*M*H*(V+1) = {flop_per_launch:.4g} FLOP per launch (M={w.B * w.beam} rows)",
+            "avg_launch_ms": joint_avg_ms, "share_of_device_time": kernel_ms["joint"] / max(1e-9, sum(kernel_ms.values()))}
+    roof["frac"] = roof["achieved"] / roof["peak"]
+    if kernel_ms["row"] > kernel_ms["joint"]:
+        roof["note"] = "row pass takes more device time than the GEMM; see row_pass"
+    launches = dec.launches_per_chunk(w.B, w.T)
+    line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": t_ms / args.steps, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "config": dict(workload_config(w, lmA.total, ph.n if ph else 0),
+                           l2="flushed (256 MB write) before every timed step, outside the step's events",
+                           parallelism=f"dp{ws} (independent streams per GPU)"),
+            "e2e": {"value": e2e_val, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+                    "steps": e2e_steps},
+            "gpu_launches": int(launches * args.steps),
+            "roofline": roof,
+            "row_pass": {"avg_launch_ms": row_avg_ms, "launches": kernel_n["row"],
+                         "share_of_device_time": kernel_ms["row"] / max(1e-9, sum(kernel_ms.values()))},
+            "wall_s_timed_region": wall,
+            "clocks": clk.summary()}
+    if not args.no_cpu_baseline and ws == 1:
+        v, cores, sample, dt = oracle_baseline(w, lmA, ph, E, W, list(range(args.cpu_streams)), args.cpu_chunks)
+        line["cpu_baseline"] = {"value": v, "unit": UNIT, "cores": cores, "kind": "oracle",
+                                "sample": sample, "seconds": dt}
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--config", type=int, default=2)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-streams", type=int, default=32)
+    ap.add_argument("--cpu-chunks", type=int, default=2)
+    ap.add_argument("--ref-streams", type=int, default=16)
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+    w = synth.WORKLOADS[args.config]
+    if args.impl == "reference":
+        run_reference(args, w)
+    else:
+        run_ours(args, w)
+
+
+if __name__ == "__main__":
+    main()

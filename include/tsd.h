@@ -1,0 +1,245 @@
+/*
+ * tsd.h -- fused streaming Transducer decode step with shallow fusion, for
+ * one NVIDIA GB300 (sm_103a).
+ *
+ * The operation (paper Sec. III-C, Eq. 1): at every decoding step each
+ * hypothesis's next-label candidates are re-ranked by
+ *
+ *     score(y) = log p_AM(y | x) + lambda * log p_LM(y) + beta * boost(y)
+ *
+ * where p_AM is the Transducer's joint output after log-softmax over the V
+ * labels and blank, p_LM a backoff n-gram model over the same sub-word
+ * labels, and boost(y) the bonus of a phrase-boosting tree built from a user
+ * phrase list.  The LM and boost terms apply to the V non-blank labels only;
+ * blank (id V) keeps its acoustic score.  The decoder consumes one encoder
+ * chunk at a time and carries its state across chunks (Sec. III-B, the
+ * cache-aware streaming loop of Fig. 1), emitting labels greedily (Sec. III)
+ * or by beam search.
+ *
+ * The joint network is  logits = W_out^T ReLU(enc_t + E[last]),  with
+ * W_out [H][V+1] and E [V+1][H] in bf16, the hidden sum in fp32 rounded once
+ * to bf16, and an fp32-accumulated product; E[V] (the blank row) is the
+ * start-of-sequence input.
+ *
+ * Conventions for every call:
+ *   - Return TSD_OK (0) or a negative status; tsd_last_error() then gives a
+ *     message for the calling thread.  No call throws or aborts.
+ *   - NULL handles, NULL required pointers and out-of-range sizes return
+ *     TSD_EINVAL before any device work.
+ *   - "device" pointers are CUDA global memory of the current device;
+ *     "host" pointers are ordinary (pageable or pinned) host memory.
+ *   - A decoder has no internal locking: drive each decoder from one host
+ *     thread, and issue all of its calls on one CUDA stream (or order them).
+ */
+#ifndef TSD_H
+#define TSD_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#if defined(__GNUC__)
+#define TSD_API __attribute__((visibility("default")))
+#else
+#define TSD_API
+#endif
+
+typedef int32_t tsd_status;
+
+#define TSD_OK 0
+#define TSD_EINVAL (-1)  /* bad argument: NULL pointer, size, token or table inconsistency */
+#define TSD_ENOMEM (-2)  /* host or device allocation failed */
+#define TSD_ECUDA (-3)   /* a CUDA runtime call failed (message has the CUDA error) */
+#define TSD_ESTATE (-4)  /* slot closed, unknown or already in use; no free slot */
+#define TSD_EDEVICE (-5) /* a device-side range check tripped (see tsd_last_error) */
+
+typedef struct tsd_ngram tsd_ngram;
+typedef struct tsd_boost tsd_boost;
+typedef struct tsd_decoder tsd_decoder;
+
+/* Message of the last failing call on this thread ("" if none). The pointer
+ * stays valid until the next call on this thread. */
+TSD_API const char* tsd_last_error(void);
+
+/* Library version string, e.g. "tsd 0.1 sm_103a". */
+TSD_API const char* tsd_version(void);
+
+/* ------------------------------------------------------------------------
+ * n-gram LM (Eq. 1, second term; Sec. III-C "GPU n-gram language models ...
+ * over sub-word tokens").
+ *
+ * Builds the device tables of an order-`order` backoff model over labels
+ * [0, V) from ARPA-like arrays, per order k = 1..order (index k-1):
+ *   count[k-1]   number of n-grams of order k;
+ *   ngrams[k-1]  host int32 [count][k], the tokens of each n-gram, any order;
+ *   logp[k-1]    host float [count], natural-log conditional probability
+ *                (an ARPA log10 source must be scaled by ln 10 first);
+ *   bow[k-1]     host float [count], natural-log backoff weight, 0 = none
+ *                (ignored for the top order; bow itself may be NULL).
+ * The score of label v after history h is
+ *   log p(v | h) = logp(h v)                 if h v is an n-gram,
+ *                = bow(h) + log p(v | h[1:])  otherwise (bow = 0 if h is
+ *                  not an n-gram), with only the last order-1 labels of h
+ *                  used and log p(v | empty) = logp of the unigram v.
+ * Requirements (else TSD_EINVAL): 1 <= order <= 16; every unigram [0, V)
+ * present exactly once; tokens in range; no duplicate n-gram; the set is
+ * prefix- and suffix-closed (every prefix and every suffix of an n-gram is an
+ * n-gram), as in any ARPA model estimated from counts; finite values.
+ * The inputs are copied (the caller keeps ownership) and uploaded
+ * synchronously to the current device. *out owns the device tables. */
+TSD_API tsd_status tsd_ngram_build(int32_t V, int32_t order, const int64_t* count,
+                           const int32_t* const* ngrams, const float* const* logp,
+                           const float* const* bow, tsd_ngram** out);
+TSD_API void tsd_ngram_free(tsd_ngram* lm);
+
+/* Sizes of the built tables: LM states (root + every n-gram below the top
+ * order), arcs (every n-gram above order 1), and device bytes held. */
+TSD_API tsd_status tsd_ngram_info(const tsd_ngram* lm, int64_t* n_states, int64_t* n_arcs,
+                          int64_t* device_bytes);
+
+/* The label tuple an LM state id stands for (host call, no device work).
+ * Writes up to cap labels, sets *len to the tuple length (0 for the root). */
+TSD_API tsd_status tsd_ngram_state_tuple(const tsd_ngram* lm, int32_t state, int32_t* buf, int32_t cap,
+                                 int32_t* len);
+
+/* ------------------------------------------------------------------------
+ * Phrase boosting tree (Eq. 1, third term; Sec. III-C "a phrase-boosting
+ * tree from a user word list", Fig. 1).
+ *
+ * Compiles n_phr phrases (host int32: phrase i is tokens[offsets[i] ..
+ * offsets[i+1]), 1 <= length <= 32, labels in [0, V)) into an Aho-Corasick
+ * trie with failure links.  boost(v) = token_bonus * (d(h v) - d(h)), where
+ * d(g) is the length of the longest suffix of g that is a prefix of some
+ * phrase, and g runs over the labels emitted since the last completed
+ * phrase: when the longest match after an emission is a whole phrase, its
+ * bonus is kept and matching restarts empty.  A partial match that fails
+ * gives back what it earned.  Duplicate phrases are merged; a phrase that is
+ * a prefix of another makes the longer one unreachable.
+ * Inputs are copied; tables are uploaded synchronously to the current device. */
+TSD_API tsd_status tsd_boost_build(int32_t V, int32_t n_phr, const int32_t* offsets,
+                           const int32_t* tokens, float token_bonus, tsd_boost** out);
+TSD_API void tsd_boost_free(tsd_boost* b);
+
+/* Trie nodes (root included), the longest phrase, and device bytes held. */
+TSD_API tsd_status tsd_boost_info(const tsd_boost* b, int32_t* n_nodes, int32_t* max_depth,
+                          int64_t* device_bytes);
+
+/* The label tuple (phrase prefix) a trie node stands for (host call). */
+TSD_API tsd_status tsd_boost_node_tuple(const tsd_boost* b, int32_t node, int32_t* buf, int32_t cap,
+                                int32_t* len);
+
+/* ------------------------------------------------------------------------
+ * Decoder.
+ */
+typedef struct {
+  int32_t V;           /* non-blank labels; blank = V; 1 <= V <= 32767 */
+  int32_t H;           /* joint hidden size; multiple of 64, 64 <= H <= 8192 */
+  int32_t max_symbols; /* labels per frame (greedy; Sec. III); beam requires 1 */
+  int32_t beam_k;      /* 1 = greedy; 2..8 = beam search */
+  int32_t max_streams; /* stream slots; max_streams * beam_k <= 4096 */
+  int32_t max_T;       /* frames per chunk, 1 <= max_T <= 4096 */
+} tsd_decoder_cfg;
+
+/* Creates a decoder for one joint network and optional LM / phrase tree.
+ *   W_out_bf16: device bf16 [H][V+1] (row-major), E_bf16: device bf16
+ *   [V+1][H].  Both are copied (W_out repacked label-major, padded) on
+ *   cuda_stream and may be freed once the stream reaches this point.
+ *   lm, boost: may be NULL (then that term is 0); they must outlive the
+ *   decoder and have the same V.
+ * Allocates all device work memory up front; no later call allocates. */
+TSD_API tsd_status tsd_decoder_create(const tsd_decoder_cfg* cfg, const void* W_out_bf16,
+                              const void* E_bf16, const tsd_ngram* lm, const tsd_boost* boost,
+                              void* cuda_stream, tsd_decoder** out);
+TSD_API void tsd_decoder_free(tsd_decoder* dec);
+
+/* Opens a stream slot and resets its state on the decoder's stream: no
+ * labels, previous label = blank (start of sequence), LM at the empty
+ * context, phrase matching empty; beam: one empty hypothesis.
+ * TSD_ESTATE if all slots are in use. */
+TSD_API tsd_status tsd_stream_open(tsd_decoder* dec, int32_t* slot_out);
+/* Frees a slot (TSD_ESTATE if it is not open). */
+TSD_API tsd_status tsd_stream_close(tsd_decoder* dec, int32_t slot);
+
+/* Decodes one encoder chunk of T frames for n open streams (the hot path).
+ *   slots:  host int32 [n], distinct open slots; row i of every array below
+ *           belongs to slots[i].
+ *   enc_bf16: device bf16 [n][T][H], the chunk's encoder frames.
+ *   lambda, beta: fusion weights of Eq. 1.
+ *   Greedy (beam_k = 1): for each stream, labels are emitted frame by frame,
+ *   at most max_symbols per frame, a blank or the limit ending the frame:
+ *     out_tokens  device int32 [n][T*max_symbols]: emitted labels in order;
+ *     out_frames  device int32 [n][T*max_symbols]: frame (0..T-1) of each;
+ *     out_scores  device float [n][T*max_symbols]: its fused score (Eq. 1);
+ *     out_counts  device int32 [n]: labels emitted this chunk.
+ *   Beam (beam_k > 1): every live hypothesis is extended by blank or one
+ *   label per frame; the top beam_k of all extensions survive and those with
+ *   equal label sequences are merged by log-sum-exp.  out_counts[i] = length
+ *   of the best hypothesis, out_scores[i*T*max_symbols] = its score,
+ *   out_tokens/out_frames are not written; read the labels with
+ *   tsd_stream_result.
+ * Asynchronous on cuda_stream (must be the decoder's stream order, see
+ * above); the device arrays are borrowed until the stream passes this call.
+ * T <= max_T and n <= max_streams, else TSD_EINVAL. */
+TSD_API tsd_status tsd_decode_chunk(tsd_decoder* dec, int32_t n, const int32_t* slots,
+                            const void* enc_bf16, int32_t T, float lambda, float beta,
+                            int32_t* out_tokens, int32_t* out_frames, float* out_scores,
+                            int32_t* out_counts, void* cuda_stream);
+
+/* Reads a greedy stream's state (synchronizes the decoder's stream): the LM
+ * state id (see tsd_ngram_state_tuple; 0 = empty context), the trie node
+ * (tsd_boost_node_tuple; 0 = root) and the previous label (V = blank/SOS).
+ * Any output pointer may be NULL. */
+TSD_API tsd_status tsd_stream_state(tsd_decoder* dec, int32_t slot, int32_t* lm_state,
+                            int32_t* trie_node, int32_t* last);
+
+/* Beam: the best live hypothesis of a slot (synchronizes): up to cap labels
+ * into buf (host), *len = its length, *score = its score (may be NULL).
+ * Greedy: not available (TSD_EINVAL); use the chunk outputs. */
+TSD_API tsd_status tsd_stream_result(tsd_decoder* dec, int32_t slot, int32_t* buf, int32_t cap,
+                             int32_t* len, float* score);
+
+/* Beam: all live hypotheses of a slot (synchronizes).  Writes up to cap_hyps
+ * entries: lengths[i], scores[i], and labels into buf at offsets i*cap_len
+ * (up to cap_len each).  *n_hyps = live hypotheses. */
+TSD_API tsd_status tsd_stream_hyps(tsd_decoder* dec, int32_t slot, int32_t* buf, int32_t cap_len,
+                           int32_t* lengths, float* scores, int32_t cap_hyps, int32_t* n_hyps);
+
+/* ------------------------------------------------------------------------
+ * Execution control and instrumentation (no counterpart in the paper).
+ */
+
+/* 1 (default): each (n, T) shape of decode_chunk is captured once into a
+ * CUDA graph and replayed; 0: kernels are launched one by one. */
+TSD_API tsd_status tsd_decoder_set_graphs(tsd_decoder* dec, int32_t enable);
+
+/* 1: record CUDA events around every kernel of later decode_chunk calls and
+ * accumulate per-kernel device time; 0 (default): no events. */
+TSD_API tsd_status tsd_decoder_set_timing(tsd_decoder* dec, int32_t enable);
+
+/* Accumulated device time (ms) and launch counts since the last reset, per
+ * kernel class: [0] row pass (state advance, LM + boost bias, joint input),
+ * [1] joint GEMM with the fused log-softmax/selection epilogue.  Waits for
+ * outstanding timed work.  reset != 0 clears the totals after reading. */
+TSD_API tsd_status tsd_decoder_timing(tsd_decoder* dec, double* ms, int64_t* launches, int32_t n_classes,
+                              int32_t reset);
+
+/* Kernel launches one decode_chunk(n, T) issues (for launch accounting). */
+TSD_API tsd_status tsd_decoder_launches_per_chunk(const tsd_decoder* dec, int32_t n, int32_t T,
+                                          int64_t* launches);
+
+/* Test hook: when logits is non-NULL, later decode_chunk calls also write the
+ * fp32 joint logits of every evaluation step s < max_steps into logits
+ * (device float [max_steps][n*beam_k][V+1]) and, when rows is non-NULL, per
+ * step and row the int32 quadruple (frame, previous label, LM state, trie
+ * node) the step was evaluated at into rows (device [max_steps][n*beam_k][4]).
+ * Pass NULLs to turn capture off.  Capture is slow; it is for parity tests. */
+TSD_API tsd_status tsd_decoder_debug_capture(tsd_decoder* dec, float* logits, int32_t* rows,
+                                     int32_t max_steps);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* TSD_H */

@@ -1,0 +1,304 @@
+"""Fused streaming Transducer decode with n-gram shallow fusion and phrase
+boosting on one GB300 (sm_103a).
+
+A thin ctypes binding over the C ABI in ``include/tsd.h`` (``libtsd.so``):
+the functions below only marshal arguments.  Every step of the decode path
+runs in the library's CUDA kernels; PyTorch is used for device memory and
+streams.  There is no CPU fallback: if the library is not built, importing
+the binding's entry points raises.
+
+Typical use::
+
+    lm = NGram(V, tokens_per_order, logp_per_order, bow_per_order)
+    boost = Boost(V, offsets, tokens, bonus)
+    dec = Decoder(V, H, W_out, E, lm=lm, boost=boost, max_streams=B, max_T=13)
+    slots = [dec.open() for _ in range(B)]
+    out = dec.decode_chunk(slots, enc, lam=0.5, beta=1.5)   # enc: cuda bf16 [B, T, H]
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from typing import List, Optional, Sequence, Tuple
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libtsd.so")
+
+TSD_OK, TSD_EINVAL, TSD_ENOMEM, TSD_ECUDA, TSD_ESTATE, TSD_EDEVICE = 0, -1, -2, -3, -4, -5
+_STATUS = {-1: "EINVAL", -2: "ENOMEM", -3: "ECUDA", -4: "ESTATE", -5: "EDEVICE"}
+
+# every entry point declared in include/tsd.h: name -> (argtypes, restype)
+_vp, _i32, _i64, _f32 = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_float
+_P = ctypes.POINTER
+
+
+class DecoderCfg(ctypes.Structure):
+    _fields_ = [("V", _i32), ("H", _i32), ("max_symbols", _i32), ("beam_k", _i32), ("max_streams", _i32),
+                ("max_T", _i32)]
+
+
+SIGNATURES = {
+    "tsd_last_error": ([], ctypes.c_char_p),
+    "tsd_version": ([], ctypes.c_char_p),
+    "tsd_ngram_build": ([_i32, _i32, _vp, _vp, _vp, _vp, _P(_vp)], _i32),
+    "tsd_ngram_free": ([_vp], None),
+    "tsd_ngram_info": ([_vp, _P(_i64), _P(_i64), _P(_i64)], _i32),
+    "tsd_ngram_state_tuple": ([_vp, _i32, _vp, _i32, _P(_i32)], _i32),
+    "tsd_boost_build": ([_i32, _i32, _vp, _vp, _f32, _P(_vp)], _i32),
+    "tsd_boost_free": ([_vp], None),
+    "tsd_boost_info": ([_vp, _P(_i32), _P(_i32), _P(_i64)], _i32),
+    "tsd_boost_node_tuple": ([_vp, _i32, _vp, _i32, _P(_i32)], _i32),
+    "tsd_decoder_create": ([_P(DecoderCfg), _vp, _vp, _vp, _vp, _vp, _P(_vp)], _i32),
+    "tsd_decoder_free": ([_vp], None),
+    "tsd_stream_open": ([_vp, _P(_i32)], _i32),
+    "tsd_stream_close": ([_vp, _i32], _i32),
+    "tsd_decode_chunk": ([_vp, _i32, _vp, _vp, _i32, _f32, _f32, _vp, _vp, _vp, _vp, _vp], _i32),
+    "tsd_stream_state": ([_vp, _i32, _P(_i32), _P(_i32), _P(_i32)], _i32),
+    "tsd_stream_result": ([_vp, _i32, _vp, _i32, _P(_i32), _P(_f32)], _i32),
+    "tsd_stream_hyps": ([_vp, _i32, _vp, _i32, _vp, _vp, _i32, _P(_i32)], _i32),
+    "tsd_decoder_set_graphs": ([_vp, _i32], _i32),
+    "tsd_decoder_set_timing": ([_vp, _i32], _i32),
+    "tsd_decoder_timing": ([_vp, _vp, _vp, _i32, _i32], _i32),
+    "tsd_decoder_launches_per_chunk": ([_vp, _i32, _i32, _P(_i64)], _i32),
+    "tsd_decoder_debug_capture": ([_vp, _vp, _vp, _i32], _i32),
+}
+
+_lib = None
+
+
+class TsdError(RuntimeError):
+    def __init__(self, status: int, msg: str):
+        super().__init__(f"tsd {_STATUS.get(status, status)}: {msg}")
+        self.status = status
+
+
+def lib() -> ctypes.CDLL:
+    """The loaded library.  Raises if it has not been built: there is no
+    fallback implementation."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH):
+            raise RuntimeError(f"{LIB_PATH} is missing: build it first (python -c 'import __graft_entry__ as g; "
+                               "g.build()')")
+        L = ctypes.CDLL(LIB_PATH)
+        for name, (args, res) in SIGNATURES.items():
+            f = getattr(L, name)
+            f.argtypes = args
+            f.restype = res
+        _lib = L
+    return _lib
+
+
+def _check(st: int):
+    if st != TSD_OK:
+        raise TsdError(st, lib().tsd_last_error().decode())
+
+
+def version() -> str:
+    return lib().tsd_version().decode()
+
+
+def _i32arr(x) -> np.ndarray:
+    return np.ascontiguousarray(np.asarray(x, dtype=np.int32))
+
+
+def _ptr(t) -> int:
+    """Device or host address of a torch tensor / numpy array."""
+    if isinstance(t, np.ndarray):
+        return t.ctypes.data
+    return t.data_ptr()
+
+
+def _stream(stream) -> int:
+    import torch
+
+    s = torch.cuda.current_stream() if stream is None else stream
+    return s.cuda_stream
+
+
+class NGram:
+    """Backoff n-gram tables on the device (``tsd_ngram_build``)."""
+
+    def __init__(self, V: int, tokens: Sequence[np.ndarray], logp: Sequence[np.ndarray],
+                 bow: Optional[Sequence[np.ndarray]] = None):
+        order = len(tokens)
+        toks = [np.ascontiguousarray(t, dtype=np.int32) for t in tokens]
+        lps = [np.ascontiguousarray(x, dtype=np.float32) for x in logp]
+        bws = [np.ascontiguousarray(x, dtype=np.float32) for x in bow] if bow is not None else None
+        cnt = np.array([len(x) for x in lps], dtype=np.int64)
+        tp = (_vp * order)(*[t.ctypes.data for t in toks])
+        lp = (_vp * order)(*[t.ctypes.data for t in lps])
+        bp = (_vp * order)(*[t.ctypes.data for t in bws]) if bws is not None else None
+        h = _vp()
+        _check(lib().tsd_ngram_build(V, order, cnt.ctypes.data, tp, lp, bp, ctypes.byref(h)))
+        self.h, self.V, self.order = h, V, order
+
+    @classmethod
+    def from_arrays(cls, a) -> "NGram":
+        return cls(a.V, a.tokens, a.logp, a.bow)
+
+    def info(self) -> Tuple[int, int, int]:
+        s, a, b = _i64(), _i64(), _i64()
+        _check(lib().tsd_ngram_info(self.h, ctypes.byref(s), ctypes.byref(a), ctypes.byref(b)))
+        return s.value, a.value, b.value
+
+    def state_tuple(self, state: int) -> Tuple[int, ...]:
+        buf = np.zeros(16, dtype=np.int32)
+        n = _i32()
+        _check(lib().tsd_ngram_state_tuple(self.h, int(state), buf.ctypes.data, 16, ctypes.byref(n)))
+        return tuple(int(x) for x in buf[: n.value])
+
+    def __del__(self):
+        if getattr(self, "h", None):
+            lib().tsd_ngram_free(self.h)
+            self.h = None
+
+
+class Boost:
+    """Phrase-boosting trie on the device (``tsd_boost_build``)."""
+
+    def __init__(self, V: int, offsets, tokens, bonus: float):
+        off = _i32arr(offsets)
+        tok = _i32arr(tokens) if len(tokens) else np.zeros(1, dtype=np.int32)
+        h = _vp()
+        _check(lib().tsd_boost_build(V, len(off) - 1, off.ctypes.data, tok.ctypes.data, float(bonus),
+                                     ctypes.byref(h)))
+        self.h, self.V = h, V
+
+    @classmethod
+    def from_phrases(cls, V: int, p, bonus: float) -> "Boost":
+        return cls(V, p.offsets, p.tokens, bonus)
+
+    def info(self) -> Tuple[int, int, int]:
+        q, d, b = _i32(), _i32(), _i64()
+        _check(lib().tsd_boost_info(self.h, ctypes.byref(q), ctypes.byref(d), ctypes.byref(b)))
+        return q.value, d.value, b.value
+
+    def node_tuple(self, node: int) -> Tuple[int, ...]:
+        buf = np.zeros(32, dtype=np.int32)
+        n = _i32()
+        _check(lib().tsd_boost_node_tuple(self.h, int(node), buf.ctypes.data, 32, ctypes.byref(n)))
+        return tuple(int(x) for x in buf[: n.value])
+
+    def __del__(self):
+        if getattr(self, "h", None):
+            lib().tsd_boost_free(self.h)
+            self.h = None
+
+
+class ChunkOut:
+    """Device outputs of one decode_chunk call (torch tensors)."""
+
+    def __init__(self, tokens, frames, scores, counts):
+        self.tokens, self.frames, self.scores, self.counts = tokens, frames, scores, counts
+
+
+class Decoder:
+    """A decoder on the current CUDA device (``tsd_decoder_create``)."""
+
+    def __init__(self, V: int, H: int, W_out, E, lm: Optional[NGram] = None, boost: Optional[Boost] = None,
+                 max_symbols: int = 5, beam_k: int = 1, max_streams: int = 64, max_T: int = 64, stream=None):
+        import torch
+
+        assert W_out.is_cuda and E.is_cuda and W_out.element_size() == 2 and E.element_size() == 2
+        assert tuple(W_out.shape) == (H, V + 1) and tuple(E.shape) == (V + 1, H)
+        self.cfg = DecoderCfg(V, H, max_symbols, beam_k, max_streams, max_T)
+        self.V, self.H, self.max_symbols, self.beam_k = V, H, max_symbols, beam_k
+        self.lm, self.boost = lm, boost  # kept alive: the decoder borrows them
+        W_out = W_out.contiguous()
+        E = E.contiguous()
+        h = _vp()
+        _check(lib().tsd_decoder_create(ctypes.byref(self.cfg), _ptr(W_out), _ptr(E), lm.h if lm else None,
+                                        boost.h if boost else None, _stream(stream), ctypes.byref(h)))
+        self.h = h
+        self._keep = []
+
+    def __del__(self):
+        if getattr(self, "h", None):
+            lib().tsd_decoder_free(self.h)
+            self.h = None
+
+    def open(self) -> int:
+        s = _i32()
+        _check(lib().tsd_stream_open(self.h, ctypes.byref(s)))
+        return s.value
+
+    def close(self, slot: int):
+        _check(lib().tsd_stream_close(self.h, int(slot)))
+
+    def alloc_out(self, n: int, T: int) -> ChunkOut:
+        import torch
+
+        cap = T * self.max_symbols
+        dev = torch.device("cuda", torch.cuda.current_device())
+        return ChunkOut(torch.empty((n, cap), dtype=torch.int32, device=dev),
+                        torch.empty((n, cap), dtype=torch.int32, device=dev),
+                        torch.empty((n, cap), dtype=torch.float32, device=dev),
+                        torch.empty((n,), dtype=torch.int32, device=dev))
+
+    def decode_chunk(self, slots: Sequence[int], enc, lam: float, beta: float, out: Optional[ChunkOut] = None,
+                     stream=None) -> ChunkOut:
+        """enc: cuda bf16 (or int16/uint16 bit patterns) [n, T, H]."""
+        n, T, H = enc.shape
+        assert n == len(slots) and H == self.H and enc.is_cuda and enc.is_contiguous()
+        if out is None:
+            out = self.alloc_out(n, T)
+        sl = _i32arr(slots)
+        _check(lib().tsd_decode_chunk(self.h, n, sl.ctypes.data, _ptr(enc), T, float(lam), float(beta),
+                                      _ptr(out.tokens), _ptr(out.frames), _ptr(out.scores), _ptr(out.counts),
+                                      _stream(stream)))
+        return out
+
+    def decode_chunk_raw(self, slots_np: np.ndarray, enc_ptr: int, T: int, lam: float, beta: float,
+                         out_ptrs: Tuple[int, int, int, int], stream_handle: int):
+        """Pointer-level call (for timing loops)."""
+        _check(lib().tsd_decode_chunk(self.h, len(slots_np), slots_np.ctypes.data, enc_ptr, T, float(lam),
+                                      float(beta), out_ptrs[0], out_ptrs[1], out_ptrs[2], out_ptrs[3],
+                                      stream_handle))
+
+    def state(self, slot: int) -> Tuple[int, int, int]:
+        a, b, c = _i32(), _i32(), _i32()
+        _check(lib().tsd_stream_state(self.h, int(slot), ctypes.byref(a), ctypes.byref(b), ctypes.byref(c)))
+        return a.value, b.value, c.value
+
+    def result(self, slot: int, cap: int = 1 << 16) -> Tuple[List[int], float]:
+        buf = np.zeros(cap, dtype=np.int32)
+        n, sc = _i32(), _f32()
+        _check(lib().tsd_stream_result(self.h, int(slot), buf.ctypes.data, cap, ctypes.byref(n), ctypes.byref(sc)))
+        return [int(x) for x in buf[: min(n.value, cap)]], sc.value
+
+    def hyps(self, slot: int, cap_len: int = 4096) -> List[Tuple[List[int], float]]:
+        K = self.beam_k
+        buf = np.zeros(K * cap_len, dtype=np.int32)
+        lens = np.zeros(K, dtype=np.int32)
+        scs = np.zeros(K, dtype=np.float32)
+        nh = _i32()
+        _check(lib().tsd_stream_hyps(self.h, int(slot), buf.ctypes.data, cap_len, lens.ctypes.data,
+                                     scs.ctypes.data, K, ctypes.byref(nh)))
+        return [([int(x) for x in buf[i * cap_len: i * cap_len + min(lens[i], cap_len)]], float(scs[i]))
+                for i in range(nh.value)]
+
+    def set_graphs(self, enable: bool):
+        _check(lib().tsd_decoder_set_graphs(self.h, 1 if enable else 0))
+
+    def set_timing(self, enable: bool):
+        _check(lib().tsd_decoder_set_timing(self.h, 1 if enable else 0))
+
+    def timing(self, reset: bool = False):
+        """({'row': ms, 'joint': ms}, {'row': launches, 'joint': launches})"""
+        ms = np.zeros(2, dtype=np.float64)
+        ln = np.zeros(2, dtype=np.int64)
+        _check(lib().tsd_decoder_timing(self.h, ms.ctypes.data, ln.ctypes.data, 2, 1 if reset else 0))
+        return {"row": float(ms[0]), "joint": float(ms[1])}, {"row": int(ln[0]), "joint": int(ln[1])}
+
+    def launches_per_chunk(self, n: int, T: int) -> int:
+        x = _i64()
+        _check(lib().tsd_decoder_launches_per_chunk(self.h, n, T, ctypes.byref(x)))
+        return x.value
+
+    def debug_capture(self, logits=None, rows=None, max_steps: int = 0):
+        self._keep = [logits, rows]
+        _check(lib().tsd_decoder_debug_capture(self.h, _ptr(logits) if logits is not None else None,
+                                               _ptr(rows) if rows is not None else None, int(max_steps)))

@@ -1,0 +1,414 @@
+// Decoder host driver: creation, stream slots and the per-chunk label loop.
+//
+// One decode_chunk(n, T) is T*max_sym label steps (the most any stream can
+// need); each step is a row pass (decide, advance, joint input, fusion bias)
+// followed by the joint GEMM with its fused selection epilogue, and a final
+// row pass applies the last decision.  Every launch reads the call's
+// arguments from a small device block written just before, so the whole
+// chunk is captured once per (n, T) as a CUDA graph and replayed.
+#include <algorithm>
+#include <cmath>
+#include <cstring>
+#include <memory>
+#include <new>
+
+#include "decoder.h"
+
+using namespace tsd;
+
+namespace {
+
+int round_up(int x, int m) { return (x + m - 1) / m * m; }
+
+tsd_status set_device(const tsd_decoder* d) {
+  int cur = -1;
+  TSD_CUDA(cudaGetDevice(&cur));
+  if (cur != d->device) TSD_CUDA(cudaSetDevice(d->device));
+  return TSD_OK;
+}
+
+int steps_per_chunk(const tsd_decoder* d, int T) { return T * d->cfg.max_symbols; }
+
+// Enqueues one chunk's launches; with events, records one at each kernel
+// boundary (external records, so they survive graph capture).
+void enqueue_chunk(tsd_decoder* d, int M, int T, cudaStream_t s, const std::vector<cudaEvent_t>* ev) {
+  const int S = steps_per_chunk(d, T);
+  int e = 0;
+  auto mark = [&]() {
+    if (ev) cudaEventRecordWithFlags((*ev)[(size_t)e++], s, cudaEventRecordExternal);
+  };
+  for (int step = 0; step <= S; ++step) {
+    mark();
+    launch_row(d->view, M, step, step == S ? 1 : 0, d->row_smem, s);
+    if (step < S) {
+      mark();
+      launch_joint(d->view, M, step, s);
+    }
+  }
+  mark();
+}
+
+void harvest(tsd_decoder* d, tsd_decoder::EventSet& es) {
+  if (!es.pending) return;
+  cudaEventSynchronize(es.ev.back());
+  for (size_t i = 0; i + 1 < es.ev.size(); ++i) {
+    float ms = 0.f;
+    if (cudaEventElapsedTime(&ms, es.ev[i], es.ev[i + 1]) == cudaSuccess) {
+      d->ms[i & 1] += ms;
+      d->launches[i & 1] += 1;
+    }
+  }
+  cudaGetLastError();
+  es.pending = false;
+}
+
+void destroy_set(tsd_decoder::EventSet& es) {
+  if (es.exec) cudaGraphExecDestroy(es.exec);
+  for (cudaEvent_t e : es.ev) cudaEventDestroy(e);
+  es.ev.clear();
+  es.exec = nullptr;
+}
+
+}  // namespace
+
+extern "C" tsd_status tsd_decoder_create(const tsd_decoder_cfg* cfg, const void* W_out_bf16,
+                                         const void* E_bf16, const tsd_ngram* lm,
+                                         const tsd_boost* boost, void* cuda_stream,
+                                         tsd_decoder** out) {
+  clear_error();
+  if (!out) return fail(TSD_EINVAL, "tsd_decoder_create: out is NULL");
+  *out = nullptr;
+  if (!cfg || !W_out_bf16 || !E_bf16) return fail(TSD_EINVAL, "tsd_decoder_create: NULL argument");
+  const tsd_decoder_cfg c = *cfg;
+  if (c.V < 1 || c.V > 32767) return fail(TSD_EINVAL, "tsd_decoder_create: V=%d out of range", c.V);
+  if (c.H < 64 || c.H > 8192 || c.H % 64) return fail(TSD_EINVAL, "tsd_decoder_create: H=%d must be a multiple of 64 in [64, 8192]", c.H);
+  if (c.beam_k != 1) return fail(TSD_EINVAL, "tsd_decoder_create: beam_k=%d not supported by this build (greedy only)", c.beam_k);
+  if (c.max_symbols < 1 || c.max_symbols > 64) return fail(TSD_EINVAL, "tsd_decoder_create: max_symbols=%d out of range", c.max_symbols);
+  if (c.max_streams < 1 || (int64_t)c.max_streams * c.beam_k > 4096)
+    return fail(TSD_EINVAL, "tsd_decoder_create: max_streams=%d out of range", c.max_streams);
+  if (c.max_T < 1 || c.max_T > 4096) return fail(TSD_EINVAL, "tsd_decoder_create: max_T=%d out of range", c.max_T);
+  if (lm && lm->view.V != c.V) return fail(TSD_EINVAL, "tsd_decoder_create: LM has V=%d, decoder V=%d", lm->view.V, c.V);
+  if (boost && boost->view.V != c.V) return fail(TSD_EINVAL, "tsd_decoder_create: boost has V=%d, decoder V=%d", boost->view.V, c.V);
+
+  std::unique_ptr<tsd_decoder> d(new (std::nothrow) tsd_decoder());
+  if (!d) return fail(TSD_ENOMEM, "tsd_decoder_create: host allocation failed");
+  d->cfg = c;
+  TSD_CUDA(cudaGetDevice(&d->device));
+  cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
+  d->lm = lm;
+  d->boost = boost;
+  d->N = c.V + 1;
+  d->N_pad = round_up(d->N, kNPad);
+  d->M_max = c.max_streams * c.beam_k;
+  d->M_pad = round_up(d->M_max, kMPad);
+  d->n_ptiles = d->N_pad / kPartialCols;
+  d->V4 = round_up(c.V, 16);
+  d->row_smem = row_smem_bytes(d->V4);
+  if (d->row_smem > 200 * 1024) return fail(TSD_EINVAL, "tsd_decoder_create: V too large for the row pass");
+
+  DevArena& A = d->arena;
+  DecView& v = d->view;
+  uint16_t *Wt, *E, *Abuf;
+  float* bias;
+  float4* part;
+  int32_t *rt, *rs, *rc, *sl, *sll, *slc, *stl, *stc;
+  const size_t SK = (size_t)c.max_streams * c.beam_k;
+  d->params_bytes = sizeof(Params) + sizeof(int32_t) * (size_t)c.max_streams;
+  char* pdev = nullptr;
+  tsd_status st;
+  if ((st = A.alloc(&Wt, (size_t)d->N_pad * c.H)) || (st = A.alloc(&E, (size_t)d->N * c.H)) ||
+      (st = A.alloc(&Abuf, (size_t)d->M_pad * c.H)) || (st = A.alloc(&bias, (size_t)d->M_pad * d->N_pad)) ||
+      (st = A.alloc(&part, (size_t)d->M_pad * d->n_ptiles)) || (st = A.alloc(&rt, (size_t)d->M_pad)) ||
+      (st = A.alloc(&rs, (size_t)d->M_pad)) || (st = A.alloc(&rc, (size_t)d->M_pad)) ||
+      (st = A.alloc(&sl, SK)) || (st = A.alloc(&sll, SK)) || (st = A.alloc(&slc, SK * kLmChain)) ||
+      (st = A.alloc(&stl, SK)) || (st = A.alloc(&stc, SK * kTrChain)) || (st = A.alloc(&pdev, d->params_bytes))) {
+    A.release();
+    return st;
+  }
+  auto cleanup = [&](tsd_status e) {
+    for (int i = 0; i < tsd_decoder::kRing; ++i) {
+      if (d->staging[i]) cudaFreeHost(d->staging[i]);
+      if (d->staging_ev[i]) cudaEventDestroy(d->staging_ev[i]);
+    }
+    if (d->cap_stream) cudaStreamDestroy(d->cap_stream);
+    A.release();
+    return e;
+  };
+  cudaError_t ce;
+  if ((ce = cudaMemsetAsync(Abuf, 0, sizeof(uint16_t) * (size_t)d->M_pad * c.H, s)) != cudaSuccess ||
+      (ce = cudaMemsetAsync(bias, 0, sizeof(float) * (size_t)d->M_pad * d->N_pad, s)) != cudaSuccess ||
+      (ce = cudaMemsetAsync(sll, 0, sizeof(int32_t) * SK, s)) != cudaSuccess ||
+      (ce = cudaMemsetAsync(stl, 0, sizeof(int32_t) * SK, s)) != cudaSuccess ||
+      (ce = cudaMemcpyAsync(E, E_bf16, sizeof(uint16_t) * (size_t)d->N * c.H, cudaMemcpyDeviceToDevice, s)) != cudaSuccess)
+    return cleanup(cuda_fail(ce, "tsd_decoder_create: initial copies"));
+  launch_repack(static_cast<const uint16_t*>(W_out_bf16), Wt, c.H, d->N, d->N_pad, s);
+  if ((ce = cudaGetLastError()) != cudaSuccess) return cleanup(cuda_fail(ce, "tsd_decoder_create: repack"));
+  if ((ce = prepare_kernels(d->row_smem)) != cudaSuccess) return cleanup(cuda_fail(ce, "tsd_decoder_create: kernel attributes"));
+  for (int i = 0; i < tsd_decoder::kRing; ++i) {
+    if ((ce = cudaHostAlloc(reinterpret_cast<void**>(&d->staging[i]), d->params_bytes, cudaHostAllocDefault)) != cudaSuccess)
+      return cleanup(fail(TSD_ENOMEM, "tsd_decoder_create: pinned staging: %s", cudaGetErrorString(ce)));
+    if ((ce = cudaEventCreateWithFlags(&d->staging_ev[i], cudaEventDisableTiming)) != cudaSuccess)
+      return cleanup(cuda_fail(ce, "tsd_decoder_create: event"));
+  }
+  if ((ce = cudaStreamCreateWithFlags(&d->cap_stream, cudaStreamNonBlocking)) != cudaSuccess)
+    return cleanup(cuda_fail(ce, "tsd_decoder_create: capture stream"));
+
+  v.V = c.V;
+  v.N = d->N;
+  v.N_pad = d->N_pad;
+  v.H = c.H;
+  v.max_sym = c.max_symbols;
+  v.K = c.beam_k;
+  v.n_ptiles = d->n_ptiles;
+  v.V4 = d->V4;
+  v.params = reinterpret_cast<const Params*>(pdev);
+  d->params_dev = reinterpret_cast<Params*>(pdev);
+  v.E = E;
+  v.Wt = Wt;
+  v.A = Abuf;
+  v.bias = bias;
+  v.part = part;
+  v.r_t = rt;
+  v.r_sym = rs;
+  v.r_cnt = rc;
+  v.s_last = sl;
+  v.s_lm_len = sll;
+  v.s_lm_chain = slc;
+  v.s_tr_len = stl;
+  v.s_tr_chain = stc;
+  v.has_lm = lm ? 1 : 0;
+  v.has_tr = boost ? 1 : 0;
+  if (lm) v.lm = lm->view;
+  if (boost) v.tr = boost->view;
+  v.cap_logits = nullptr;
+  v.cap_rows = nullptr;
+  v.cap_steps = 0;
+  d->slot_open.assign((size_t)c.max_streams, 0);
+  d->last_stream = s;
+  *out = d.release();
+  return TSD_OK;
+}
+
+extern "C" void tsd_decoder_free(tsd_decoder* d) {
+  if (!d) return;
+  set_device(d);
+  cudaDeviceSynchronize();
+  for (auto& kv : d->entries) {
+    destroy_set(kv.second.set[0]);
+    destroy_set(kv.second.set[1]);
+  }
+  for (int i = 0; i < tsd_decoder::kRing; ++i) {
+    if (d->staging[i]) cudaFreeHost(d->staging[i]);
+    if (d->staging_ev[i]) cudaEventDestroy(d->staging_ev[i]);
+  }
+  if (d->cap_stream) cudaStreamDestroy(d->cap_stream);
+  d->arena.release();
+  cudaGetLastError();
+  delete d;
+}
+
+extern "C" tsd_status tsd_stream_open(tsd_decoder* d, int32_t* slot_out) {
+  clear_error();
+  if (!d || !slot_out) return fail(TSD_EINVAL, "tsd_stream_open: NULL argument");
+  auto it = std::find(d->slot_open.begin(), d->slot_open.end(), 0);
+  if (it == d->slot_open.end()) return fail(TSD_ESTATE, "tsd_stream_open: all %d slots are open", d->cfg.max_streams);
+  tsd_status st = set_device(d);
+  if (st) return st;
+  int slot = (int)(it - d->slot_open.begin());
+  launch_open(d->view, slot, d->last_stream);
+  TSD_CUDA(cudaGetLastError());
+  *it = 1;
+  *slot_out = slot;
+  return TSD_OK;
+}
+
+extern "C" tsd_status tsd_stream_close(tsd_decoder* d, int32_t slot) {
+  clear_error();
+  if (!d) return fail(TSD_EINVAL, "tsd_stream_close: NULL decoder");
+  if (slot < 0 || slot >= d->cfg.max_streams || !d->slot_open[(size_t)slot])
+    return fail(TSD_ESTATE, "tsd_stream_close: slot %d is not open", slot);
+  d->slot_open[(size_t)slot] = 0;
+  return TSD_OK;
+}
+
+extern "C" tsd_status tsd_decode_chunk(tsd_decoder* d, int32_t n, const int32_t* slots,
+                                       const void* enc_bf16, int32_t T, float lambda, float beta,
+                                       int32_t* out_tokens, int32_t* out_frames, float* out_scores,
+                                       int32_t* out_counts, void* cuda_stream) {
+  clear_error();
+  if (!d || !slots || !enc_bf16 || !out_counts) return fail(TSD_EINVAL, "tsd_decode_chunk: NULL argument");
+  if (d->cfg.beam_k == 1 && (!out_tokens || !out_frames || !out_scores))
+    return fail(TSD_EINVAL, "tsd_decode_chunk: NULL output array");
+  if (n < 1 || n > d->cfg.max_streams) return fail(TSD_EINVAL, "tsd_decode_chunk: n=%d out of [1, %d]", n, d->cfg.max_streams);
+  if (T < 1 || T > d->cfg.max_T) return fail(TSD_EINVAL, "tsd_decode_chunk: T=%d out of [1, %d]", T, d->cfg.max_T);
+  if (!std::isfinite(lambda) || !std::isfinite(beta)) return fail(TSD_EINVAL, "tsd_decode_chunk: non-finite weight");
+  {
+    std::vector<uint8_t> seen((size_t)d->cfg.max_streams, 0);
+    for (int i = 0; i < n; ++i) {
+      int s = slots[i];
+      if (s < 0 || s >= d->cfg.max_streams || !d->slot_open[(size_t)s])
+        return fail(TSD_ESTATE, "tsd_decode_chunk: slot %d is not open", s);
+      if (seen[(size_t)s]) return fail(TSD_EINVAL, "tsd_decode_chunk: slot %d listed twice", s);
+      seen[(size_t)s] = 1;
+    }
+  }
+  tsd_status st = set_device(d);
+  if (st) return st;
+  cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
+  d->last_stream = s;
+
+  // call parameters -> pinned staging -> device
+  const int slot_i = d->ring_pos;
+  d->ring_pos = (d->ring_pos + 1) % tsd_decoder::kRing;
+  TSD_CUDA(cudaEventSynchronize(d->staging_ev[slot_i]));
+  Params* hp = reinterpret_cast<Params*>(d->staging[slot_i]);
+  hp->enc = static_cast<const uint16_t*>(enc_bf16);
+  hp->out_tok = out_tokens;
+  hp->out_frame = out_frames;
+  hp->out_score = out_scores;
+  hp->out_count = out_counts;
+  hp->n = n;
+  hp->T = T;
+  hp->lambda = lambda;
+  hp->beta = beta;
+  std::memcpy(hp->slots, slots, sizeof(int32_t) * (size_t)n);
+  const size_t bytes = sizeof(Params) + sizeof(int32_t) * (size_t)n;
+  TSD_CUDA(cudaMemcpyAsync(d->params_dev, hp, bytes, cudaMemcpyHostToDevice, s));
+  TSD_CUDA(cudaEventRecord(d->staging_ev[slot_i], s));
+
+  const int M = n * d->cfg.beam_k;
+  const int S = steps_per_chunk(d, T);
+  const int n_events = 2 * S + 2;
+  auto key = std::make_tuple(n, T, d->use_graphs, d->timing);
+  tsd_decoder::Entry& ent = d->entries[key];
+  tsd_decoder::EventSet& es = ent.set[ent.next];
+  if (d->timing) {
+    ent.next ^= 1;
+    harvest(d, es);
+    if (es.ev.empty()) {
+      es.ev.resize((size_t)n_events);
+      for (auto& e : es.ev) TSD_CUDA(cudaEventCreate(&e));
+    }
+  }
+  const std::vector<cudaEvent_t>* evp = d->timing ? &es.ev : nullptr;
+  if (d->use_graphs) {
+    if (!es.exec) {
+      cudaGraph_t g = nullptr;
+      TSD_CUDA(cudaStreamBeginCapture(d->cap_stream, cudaStreamCaptureModeThreadLocal));
+      enqueue_chunk(d, M, T, d->cap_stream, evp);
+      cudaError_t ce = cudaStreamEndCapture(d->cap_stream, &g);
+      if (ce != cudaSuccess) return cuda_fail(ce, "tsd_decode_chunk: graph capture");
+      ce = cudaGraphInstantiate(&es.exec, g, 0);
+      cudaGraphDestroy(g);
+      if (ce != cudaSuccess) {
+        es.exec = nullptr;
+        return cuda_fail(ce, "tsd_decode_chunk: graph instantiate");
+      }
+    }
+    TSD_CUDA(cudaGraphLaunch(es.exec, s));
+  } else {
+    enqueue_chunk(d, M, T, s, evp);
+    TSD_CUDA(cudaGetLastError());
+  }
+  if (d->timing) es.pending = true;
+  return TSD_OK;
+}
+
+extern "C" tsd_status tsd_stream_state(tsd_decoder* d, int32_t slot, int32_t* lm_state,
+                                       int32_t* trie_node, int32_t* last) {
+  clear_error();
+  if (!d) return fail(TSD_EINVAL, "tsd_stream_state: NULL decoder");
+  if (slot < 0 || slot >= d->cfg.max_streams || !d->slot_open[(size_t)slot])
+    return fail(TSD_ESTATE, "tsd_stream_state: slot %d is not open", slot);
+  tsd_status st = set_device(d);
+  if (st) return st;
+  TSD_CUDA(cudaStreamSynchronize(d->last_stream));
+  int32_t ll = 0, tl = 0, ls = 0, chain_lm[kLmChain], chain_tr[kTrChain];
+  const DecView& v = d->view;
+  TSD_CUDA(cudaMemcpy(&ls, v.s_last + slot, 4, cudaMemcpyDeviceToHost));
+  TSD_CUDA(cudaMemcpy(&ll, v.s_lm_len + slot, 4, cudaMemcpyDeviceToHost));
+  TSD_CUDA(cudaMemcpy(&tl, v.s_tr_len + slot, 4, cudaMemcpyDeviceToHost));
+  TSD_CUDA(cudaMemcpy(chain_lm, v.s_lm_chain + (size_t)slot * kLmChain, sizeof(chain_lm), cudaMemcpyDeviceToHost));
+  TSD_CUDA(cudaMemcpy(chain_tr, v.s_tr_chain + (size_t)slot * kTrChain, sizeof(chain_tr), cudaMemcpyDeviceToHost));
+  if (lm_state) *lm_state = ll > 0 ? chain_lm[ll - 1] : 0;
+  if (trie_node) *trie_node = tl > 0 ? chain_tr[0] : 0;
+  if (last) *last = ls;
+  return TSD_OK;
+}
+
+extern "C" tsd_status tsd_stream_result(tsd_decoder* d, int32_t, int32_t*, int32_t, int32_t*, float*) {
+  clear_error();
+  if (!d) return fail(TSD_EINVAL, "tsd_stream_result: NULL decoder");
+  return fail(TSD_EINVAL, "tsd_stream_result: only beam decoders keep hypotheses");
+}
+
+extern "C" tsd_status tsd_stream_hyps(tsd_decoder* d, int32_t, int32_t*, int32_t, int32_t*, float*,
+                                      int32_t, int32_t*) {
+  clear_error();
+  if (!d) return fail(TSD_EINVAL, "tsd_stream_hyps: NULL decoder");
+  return fail(TSD_EINVAL, "tsd_stream_hyps: only beam decoders keep hypotheses");
+}
+
+extern "C" tsd_status tsd_decoder_set_graphs(tsd_decoder* d, int32_t enable) {
+  clear_error();
+  if (!d) return fail(TSD_EINVAL, "tsd_decoder_set_graphs: NULL decoder");
+  d->use_graphs = enable ? 1 : 0;
+  return TSD_OK;
+}
+
+extern "C" tsd_status tsd_decoder_set_timing(tsd_decoder* d, int32_t enable) {
+  clear_error();
+  if (!d) return fail(TSD_EINVAL, "tsd_decoder_set_timing: NULL decoder");
+  d->timing = enable ? 1 : 0;
+  return TSD_OK;
+}
+
+extern "C" tsd_status tsd_decoder_timing(tsd_decoder* d, double* ms, int64_t* launches,
+                                         int32_t n_classes, int32_t reset) {
+  clear_error();
+  if (!d) return fail(TSD_EINVAL, "tsd_decoder_timing: NULL decoder");
+  tsd_status st = set_device(d);
+  if (st) return st;
+  for (auto& kv : d->entries) {
+    harvest(d, kv.second.set[0]);
+    harvest(d, kv.second.set[1]);
+  }
+  for (int i = 0; i < n_classes && i < 2; ++i) {
+    if (ms) ms[i] = d->ms[i];
+    if (launches) launches[i] = d->launches[i];
+  }
+  if (reset) {
+    d->ms[0] = d->ms[1] = 0;
+    d->launches[0] = d->launches[1] = 0;
+  }
+  return TSD_OK;
+}
+
+extern "C" tsd_status tsd_decoder_launches_per_chunk(const tsd_decoder* d, int32_t n, int32_t T,
+                                                     int64_t* launches) {
+  clear_error();
+  if (!d || !launches) return fail(TSD_EINVAL, "tsd_decoder_launches_per_chunk: NULL argument");
+  (void)n;
+  *launches = 2 * (int64_t)steps_per_chunk(d, T) + 1;
+  return TSD_OK;
+}
+
+extern "C" tsd_status tsd_decoder_debug_capture(tsd_decoder* d, float* logits, int32_t* rows,
+                                                int32_t max_steps) {
+  clear_error();
+  if (!d) return fail(TSD_EINVAL, "tsd_decoder_debug_capture: NULL decoder");
+  if ((logits || rows) && max_steps < 1) return fail(TSD_EINVAL, "tsd_decoder_debug_capture: max_steps < 1");
+  d->view.cap_logits = logits;
+  d->view.cap_rows = rows;
+  d->view.cap_steps = (logits || rows) ? max_steps : 0;
+  // captured graphs bake the view in: drop them
+  tsd_status st = set_device(d);
+  if (st) return st;
+  cudaDeviceSynchronize();
+  for (auto& kv : d->entries) {
+    destroy_set(kv.second.set[0]);
+    destroy_set(kv.second.set[1]);
+  }
+  d->entries.clear();
+  return TSD_OK;
+}

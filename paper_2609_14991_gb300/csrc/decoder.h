@@ -1,0 +1,95 @@
+// Decoder internals shared by the host driver and the kernels.
+#pragma once
+
+#include <cuda_bf16.h>
+
+#include <map>
+#include <tuple>
+
+#include "internal.h"
+
+namespace tsd {
+
+// Per-call parameters, copied to the device before each chunk so that one
+// captured graph serves every call of the same shape.
+struct Params {
+  const uint16_t* enc;  // [n][T][H] bf16
+  int32_t* out_tok;     // [n][T*max_sym]
+  int32_t* out_frame;
+  float* out_score;
+  int32_t* out_count;  // [n]
+  int32_t n, T;
+  float lambda, beta;
+  int32_t slots[1];  // [n], the struct is allocated with room for max_streams
+};
+
+// Everything a kernel needs; passed by value.
+struct DecView {
+  int32_t V, N, N_pad, H, max_sym, K, n_ptiles, V4;
+  const Params* params;
+  const uint16_t* E;   // [N][H] bf16
+  const uint16_t* Wt;  // [N_pad][H] bf16, label-major (rows >= N are zero)
+  uint16_t* A;         // [M_pad][H] bf16, joint input of the current step
+  float* bias;         // [M_pad][N_pad] fp32, lambda*LM + beta*boost of the current step
+  float4* part;        // [M_pad][n_ptiles] (max logit, sum exp, best fused, best label)
+  int32_t* r_t;        // [M_pad] frame
+  int32_t* r_sym;      // [M_pad] labels emitted in this frame
+  int32_t* r_cnt;      // [M_pad] labels emitted in this chunk
+  // per-slot (x K hypotheses) persistent state
+  int32_t* s_last;      // previous label (V = blank / start)
+  int32_t* s_lm_len;    // LM chain length (order of the LM state)
+  int32_t* s_lm_chain;  // [.][kLmChain]
+  int32_t* s_tr_len;
+  int32_t* s_tr_chain;  // [.][kTrChain]
+  LmView lm;
+  TrieView tr;
+  int32_t has_lm, has_tr;
+  float* cap_logits;
+  int32_t* cap_rows;
+  int32_t cap_steps;
+};
+
+constexpr int kRowThreads = 256;
+
+void launch_repack(const uint16_t* W, uint16_t* Wt, int H, int N, int N_pad, cudaStream_t s);
+void launch_open(const DecView& d, int slot, cudaStream_t s);
+void launch_row(const DecView& d, int M, int step, int final_step, size_t smem, cudaStream_t s);
+void launch_joint(const DecView& d, int M, int step, cudaStream_t s);
+size_t row_smem_bytes(int V4);
+cudaError_t prepare_kernels(size_t row_smem);
+
+}  // namespace tsd
+
+struct tsd_decoder {
+  tsd_decoder_cfg cfg{};
+  int device = 0;
+  int N = 0, N_pad = 0, M_max = 0, M_pad = 0, n_ptiles = 0, V4 = 0;
+  tsd::DevArena arena;
+  const tsd_ngram* lm = nullptr;
+  const tsd_boost* boost = nullptr;
+  tsd::DecView view{};
+  tsd::Params* params_dev = nullptr;
+  size_t params_bytes = 0;
+  static constexpr int kRing = 4;
+  char* staging[kRing] = {};
+  cudaEvent_t staging_ev[kRing] = {};
+  int ring_pos = 0;
+  cudaStream_t cap_stream = nullptr;
+  cudaStream_t last_stream = nullptr;
+  std::vector<uint8_t> slot_open;
+  int use_graphs = 1, timing = 0;
+  size_t row_smem = 0;
+
+  struct EventSet {
+    std::vector<cudaEvent_t> ev;
+    cudaGraphExec_t exec = nullptr;
+    bool pending = false;
+  };
+  struct Entry {
+    EventSet set[2];
+    int next = 0;
+  };
+  std::map<std::tuple<int, int, int, int>, Entry> entries;  // (n, T, graphs, timing)
+  double ms[2] = {0, 0};
+  int64_t launches[2] = {0, 0};
+};

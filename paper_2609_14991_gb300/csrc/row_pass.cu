@@ -1,0 +1,330 @@
+// Row pass of the fused decode step: one CTA per hypothesis row.
+//
+// For row r at label step s it
+//   1. combines the joint kernel's per-tile partials of step s-1 into the
+//      log-sum-exp of the row and its best fused label (Eq. 1 argmax);
+//   2. applies the greedy decision: blank (or the per-frame label limit)
+//      advances the frame, a label is emitted and advances the LM state and
+//      the phrase-trie state;
+//   3. writes the joint input of step s, bf16(ReLU(enc_t + E[last])), and
+//   4. the dense fusion bias of step s, lambda*log p_LM(v|state) +
+//      beta*boost(v|trie state) for every label v (Eq. 1, terms 2 and 3).
+//
+// LM state and phrase state are both kept as their whole suffix chain (one
+// LM state per order; every trie node that is a suffix of the current one),
+// so the next chain after label y is assembled from independent searches of
+// y in each chain element -- no dependent pointer chase.
+#include "decoder.h"
+
+namespace tsd {
+
+namespace {
+
+constexpr float kNegInf = -__builtin_huge_valf();
+
+// Position of y in the sorted arr[0, n), or -1: a 32-ary search by one warp.
+__device__ __forceinline__ int warp_find(const int32_t* __restrict__ arr, int n, int y, int lane) {
+  int lo = 0, hi = n;
+  while (hi - lo > 32) {
+    int step = (hi - lo + 31) >> 5;
+    int idx = lo + lane * step;
+    int v = (idx < hi) ? __ldg(arr + idx) : INT_MAX;
+    unsigned m = __ballot_sync(0xffffffffu, v <= y);
+    if (m == 0) return -1;
+    int last = 31 - __clz((int)m);
+    lo = lo + last * step;
+    hi = min(hi, lo + step);
+  }
+  int idx = lo + lane;
+  bool hit = (idx < hi) && (__ldg(arr + idx) == y);
+  unsigned m = __ballot_sync(0xffffffffu, hit);
+  return m ? lo + __ffs((int)m) - 1 : -1;
+}
+
+// Merges two softmax partials (max, sum of exp(x - max)).
+__device__ __forceinline__ void lse_merge(float& m, float& s, float m2, float s2) {
+  if (m2 == kNegInf) return;
+  if (m == kNegInf) { m = m2; s = s2; return; }
+  float mx = fmaxf(m, m2);
+  s = s * expf(m - mx) + s2 * expf(m2 - mx);
+  m = mx;
+}
+
+__device__ __forceinline__ void best_merge(float& v, int& i, float v2, int i2) {
+  if (v2 > v || (v2 == v && i2 < i)) { v = v2; i = i2; }
+}
+
+__global__ void __launch_bounds__(kRowThreads) k_row(DecView d, int step, int final_step) {
+  const Params* __restrict__ P = d.params;
+  const int r = blockIdx.x;
+  const int slot = P->slots[r];
+  const int T = P->T;
+  const int V = d.V;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  extern __shared__ __align__(16) unsigned char smem[];
+  float* lmrow = reinterpret_cast<float*>(smem);
+  int8_t* dep = reinterpret_cast<int8_t*>(lmrow + d.V4);
+
+  __shared__ int s_t, s_sym, s_cnt, s_y, s_lm_len, s_tr_len, s_last;
+  __shared__ float s_score;
+  __shared__ int s_lm[kLmChain], s_tr[kTrChain];
+  __shared__ int s_lm_hit[kLmChain];
+  __shared__ int s_tr_hit[kTrChain];
+
+  if (tid == 0) {
+    if (step == 0) {
+      s_t = 0; s_sym = 0; s_cnt = 0;
+    } else {
+      s_t = d.r_t[r]; s_sym = d.r_sym[r]; s_cnt = d.r_cnt[r];
+    }
+    s_lm_len = d.has_lm ? d.s_lm_len[slot] : 0;
+    s_tr_len = d.has_tr ? d.s_tr_len[slot] : 0;
+    s_last = d.s_last[slot];
+  }
+  __syncthreads();
+  if (tid < s_lm_len) s_lm[tid] = d.s_lm_chain[slot * kLmChain + tid];
+  if (tid < s_tr_len) s_tr[tid] = d.s_tr_chain[slot * kTrChain + tid];
+  __syncthreads();
+  const bool evaluated = (step > 0) && (s_t < T);
+
+  if (evaluated) {
+    // 1. combine the partials of the previous joint step
+    if (warp == 0) {
+      float m = kNegInf, s = 0.f, bv = kNegInf;
+      int bi = INT_MAX;
+      const float4* pr = d.part + (size_t)r * d.n_ptiles;
+      for (int j = lane; j < d.n_ptiles; j += 32) {
+        float4 p = pr[j];
+        lse_merge(m, s, p.x, p.y);
+        best_merge(bv, bi, p.z, __float_as_int(p.w));
+      }
+      for (int o = 16; o > 0; o >>= 1) {
+        float m2 = __shfl_xor_sync(0xffffffffu, m, o);
+        float s2 = __shfl_xor_sync(0xffffffffu, s, o);
+        float v2 = __shfl_xor_sync(0xffffffffu, bv, o);
+        int i2 = __shfl_xor_sync(0xffffffffu, bi, o);
+        lse_merge(m, s, m2, s2);
+        best_merge(bv, bi, v2, i2);
+      }
+      if (lane == 0) {
+        s_y = (bi >= 0 && bi <= V) ? bi : V;
+        s_score = bv - (m + logf(s));
+      }
+    }
+    __syncthreads();
+    const int y = s_y;
+    if (y != V) {
+      // 2a. independent searches of y in every chain element
+      const int nl = s_lm_len, nt = s_tr_len;
+      for (int task = warp; task < nl + nt; task += kRowThreads / 32) {
+        if (task < nl) {
+          int st = s_lm[task];
+          int b = __ldg(d.lm.st_begin + st), c = __ldg(d.lm.st_count + st);
+          int i = warp_find(d.lm.arc_tok + b, c, y, lane);
+          if (lane == 0) s_lm_hit[task] = (i >= 0) ? b + i : -1;
+        } else {
+          int q = s_tr[task - nl];
+          int b = __ldg(d.tr.nd_begin + q), c = __ldg(d.tr.nd_count + q);
+          int i = warp_find(d.tr.ch_tok + b, c, y, lane);
+          if (lane == 0) s_tr_hit[task - nl] = (i >= 0) ? b + i : -1;
+        }
+      }
+      __syncthreads();
+      // 2b. assemble the new chains and emit
+      if (tid == 0) {
+        int newlm[kLmChain];
+        int ln = 0;
+        if (d.has_lm && d.lm.order >= 2) {
+          newlm[ln++] = __ldg(d.lm.uni_tgt + y);
+          for (int l = 0; l < nl && ln < kLmChain; ++l) {
+            int a = s_lm_hit[l];
+            if (a < 0) break;
+            int tgt = __ldg(d.lm.arc_tgt + a);
+            if (tgt < 0) break;
+            newlm[ln++] = tgt;
+          }
+        }
+        int newtr[kTrChain];
+        int tn = 0;
+        bool reset = false;
+        if (d.has_tr) {
+          for (int i = 0; i < nt; ++i) {
+            int a = s_tr_hit[i];
+            if (a < 0) continue;
+            if (tn == 0 && __ldg(d.tr.ch_next + a) == 0) reset = true;
+            if (tn < kTrChain) newtr[tn++] = __ldg(d.tr.ch_node + a);
+          }
+          int rc = __ldg(d.tr.root_child + y);
+          if (rc != 0) {
+            if (tn == 0 && __ldg(d.tr.root_next + y) == 0) reset = true;
+            if (tn < kTrChain) newtr[tn++] = rc;
+          }
+          if (reset) tn = 0;
+        }
+        for (int l = 0; l < ln; ++l) { s_lm[l] = newlm[l]; d.s_lm_chain[slot * kLmChain + l] = newlm[l]; }
+        for (int l = 0; l < tn; ++l) { s_tr[l] = newtr[l]; d.s_tr_chain[slot * kTrChain + l] = newtr[l]; }
+        s_lm_len = ln;
+        s_tr_len = tn;
+        if (d.has_lm) d.s_lm_len[slot] = ln;
+        if (d.has_tr) d.s_tr_len[slot] = tn;
+        const int cap = T * d.max_sym;
+        const int o = r * cap + s_cnt;
+        P->out_tok[o] = y;
+        P->out_frame[o] = s_t;
+        P->out_score[o] = s_score;
+        s_cnt += 1;
+        s_last = y;
+        d.s_last[slot] = y;
+        s_sym += 1;
+        if (s_sym >= d.max_sym) { s_t += 1; s_sym = 0; }
+      }
+    } else if (tid == 0) {
+      s_t += 1;
+      s_sym = 0;
+    }
+    __syncthreads();
+  }
+
+  if (final_step) {
+    if (tid == 0) P->out_count[r] = s_cnt;
+    return;
+  }
+  if (tid == 0) {
+    d.r_t[r] = s_t;
+    d.r_sym[r] = s_sym;
+    d.r_cnt[r] = s_cnt;
+  }
+  const int t = s_t;
+  if (d.cap_rows && step < d.cap_steps && tid == 0) {
+    int* c = d.cap_rows + ((size_t)step * P->n + r) * 4;
+    if (t < T) {
+      c[0] = t;
+      c[1] = s_last;
+      c[2] = s_lm_len ? s_lm[s_lm_len - 1] : 0;
+      c[3] = s_tr_len ? s_tr[0] : 0;
+    } else {
+      c[0] = -1; c[1] = -1; c[2] = -1; c[3] = -1;
+    }
+  }
+  if (t >= T) return;
+
+  // 3. joint input of this step
+  {
+    const int H = d.H;
+    const uint4* e = reinterpret_cast<const uint4*>(P->enc + ((size_t)r * T + t) * H);
+    const uint4* g = reinterpret_cast<const uint4*>(d.E + (size_t)s_last * H);
+    uint4* a = reinterpret_cast<uint4*>(d.A + (size_t)r * H);
+    for (int i = tid; i < H / 8; i += kRowThreads) {
+      uint4 x = __ldg(e + i), z = __ldg(g + i);
+      const __nv_bfloat162* xa = reinterpret_cast<const __nv_bfloat162*>(&x);
+      const __nv_bfloat162* za = reinterpret_cast<const __nv_bfloat162*>(&z);
+      uint4 out;
+      __nv_bfloat162* oa = reinterpret_cast<__nv_bfloat162*>(&out);
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        float2 xf = __bfloat1622float2(xa[q]);
+        float2 zf = __bfloat1622float2(za[q]);
+        float lo = fmaxf(xf.x + zf.x, 0.f), hi = fmaxf(xf.y + zf.y, 0.f);
+        oa[q] = __floats2bfloat162_rn(lo, hi);
+      }
+      a[i] = out;
+    }
+  }
+
+  // 4. fusion bias of this step
+  const int nl = s_lm_len, nt = s_tr_len;
+  const float lam = P->lambda, beta = P->beta;
+  const float cum_top = (d.has_lm && nl) ? __ldg(d.lm.st_cum + s_lm[nl - 1]) : 0.f;
+  const int depth_cur = (d.has_tr && nt) ? __ldg(d.tr.nd_depth + s_tr[0]) : 0;
+  const float unset = __int_as_float(0x7fc00000);
+  for (int v = tid; v < V; v += kRowThreads) {
+    lmrow[v] = unset;
+    dep[v] = -1;
+  }
+  __syncthreads();
+  const int phases = max(nl, nt);
+  for (int p = 0; p < phases; ++p) {
+    if (p < nl) {  // LM level nl-p (deepest first): its arcs win over shallower ones
+      int st = s_lm[nl - 1 - p];
+      int b = __ldg(d.lm.st_begin + st), c = __ldg(d.lm.st_count + st);
+      float off = cum_top - __ldg(d.lm.st_cum + st);
+      for (int j = tid; j < c; j += kRowThreads) {
+        int w = __ldg(d.lm.arc_tok + b + j);
+        if (isnan(lmrow[w])) lmrow[w] = off + __ldg(d.lm.arc_logp + b + j);
+      }
+    }
+    if (p < nt) {  // trie chain node p (deepest first)
+      int q = s_tr[p];
+      int b = __ldg(d.tr.nd_begin + q), c = __ldg(d.tr.nd_count + q);
+      int dd = __ldg(d.tr.nd_depth + q) + 1;
+      for (int j = tid; j < c; j += kRowThreads) {
+        int w = __ldg(d.tr.ch_tok + b + j);
+        if (dep[w] < 0) dep[w] = (int8_t)dd;
+      }
+    }
+    __syncthreads();
+  }
+  float* brow = d.bias + (size_t)r * d.N_pad;
+  const float bscale = beta * (d.has_tr ? d.tr.bonus : 0.f);
+  for (int v = tid; v < V; v += kRowThreads) {
+    float b = 0.f;
+    if (d.has_lm) {
+      float l = lmrow[v];
+      if (isnan(l)) l = cum_top + __ldg(d.lm.uni_logp + v);
+      b = lam * l;
+    }
+    if (d.has_tr) {
+      int dd = dep[v];
+      if (dd < 0) dd = (__ldg(d.tr.root_child + v) != 0) ? 1 : 0;
+      b += bscale * (float)(dd - depth_cur);
+    }
+    brow[v] = b;
+  }
+  if (tid == 0) brow[V] = 0.f;
+}
+
+__global__ void k_open(DecView d, int slot) {
+  if (threadIdx.x == 0) {
+    d.s_last[slot] = d.V;
+    d.s_lm_len[slot] = 0;
+    d.s_tr_len[slot] = 0;
+  }
+}
+
+__global__ void k_repack(const uint16_t* __restrict__ W, uint16_t* __restrict__ Wt, int H, int N, int N_pad) {
+  __shared__ uint16_t tile[32][33];
+  int k0 = blockIdx.y * 32, v0 = blockIdx.x * 32;
+  int tx = threadIdx.x, ty = threadIdx.y;  // 32 x 8
+  for (int i = ty; i < 32; i += 8) {
+    int k = k0 + i, v = v0 + tx;
+    tile[i][tx] = (k < H && v < N) ? W[(size_t)k * N + v] : (uint16_t)0;
+  }
+  __syncthreads();
+  for (int i = ty; i < 32; i += 8) {
+    int v = v0 + i, k = k0 + tx;
+    if (v < N_pad && k < H) Wt[(size_t)v * H + k] = tile[tx][i];
+  }
+}
+
+}  // namespace
+
+size_t row_smem_bytes(int V4) { return (size_t)V4 * (sizeof(float) + 1); }
+
+cudaError_t prepare_kernels(size_t row_smem) {
+  if (row_smem > 48 * 1024)
+    return cudaFuncSetAttribute(k_row, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)row_smem);
+  return cudaSuccess;
+}
+
+void launch_repack(const uint16_t* W, uint16_t* Wt, int H, int N, int N_pad, cudaStream_t s) {
+  dim3 grid((N_pad + 31) / 32, (H + 31) / 32), block(32, 8);
+  k_repack<<<grid, block, 0, s>>>(W, Wt, H, N, N_pad);
+}
+
+void launch_open(const DecView& d, int slot, cudaStream_t s) { k_open<<<1, 32, 0, s>>>(d, slot); }
+
+void launch_row(const DecView& d, int M, int step, int final_step, size_t smem, cudaStream_t s) {
+  k_row<<<M, kRowThreads, smem, s>>>(d, step, final_step);
+}
+
+}  // namespace tsd

@@ -1,0 +1,202 @@
+"""GPU parity: the CUDA decode path against the oracle on the same seeded
+inputs, through the C ABI.
+
+Rules (fixed here, derived from the fp32 arithmetic of the kernels):
+  * label sequences match wherever the oracle's top-2 gap exceeds 1e-3;
+    at nearer ties either choice is valid and the oracle follows the GPU;
+  * fused scores of emitted labels within 1e-4 absolute;
+  * joint logits within 2e-2 of the oracle's double product of the same
+    bf16-rounded inputs;
+  * LM state and trie node bit-exact (as label tuples) after every chunk,
+    and at every step where steps are captured.
+"""
+import numpy as np
+import pytest
+
+import oracle
+import synth
+from tests import parity_util as pu
+
+pytestmark = pytest.mark.gpu
+torch = pytest.importorskip("torch")
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _gpu():
+    assert torch.cuda.is_available(), "GPU tests need a CUDA device"
+    import paper_2609_14991_gb300 as tsd
+
+    tsd.lib()  # fails loudly if the library is missing
+
+
+def _evaluations(tok, fr, T, max_sym):
+    """(frame, labels emitted before) of every joint evaluation of one chunk,
+    reconstructed from the emitted labels: a frame with j < max_sym labels
+    had j + 1 evaluations (the last chose blank), one with max_sym had j."""
+    ev = []
+    hist = []
+    p = 0
+    for t in range(T):
+        j = 0
+        while True:
+            ev.append((t, list(hist)))
+            if p < len(tok) and fr[p] == t:
+                hist.append(int(tok[p]))
+                p += 1
+                j += 1
+                if j == max_sym:
+                    break
+            else:
+                break
+    return ev
+
+
+def test_cfg0_full_parity_with_step_capture():
+    w = synth.WORKLOADS[0]
+    inp = pu.Inputs(w)
+    S = w.T * w.max_sym
+    run = pu.GpuRun(inp, range(w.B), 1, capture_steps=S)
+    reps = pu.replay(inp, run, range(w.B))
+    pu.assert_reports(reps)
+    olm, obo, model = pu.oracle_models(inp)
+    rows = run.cap_rows.cpu().numpy()
+    logits = run.cap_logits.cpu().numpy()
+    worst = 0.0
+    for i in range(w.B):
+        tok, fr, _ = run.emitted(i, 0)
+        ev = _evaluations(tok, fr, w.T, w.max_sym)
+        assert len(ev) <= S
+        for s, (t, hist) in enumerate(ev):
+            ft, last, lm_state, node = rows[s, i]
+            assert ft == t
+            assert last == (hist[-1] if hist else w.V)
+            assert run.lm.state_tuple(lm_state) == olm.state(hist), (i, s)
+            rho = int(obo.trajectory(hist)[1][-1]) if hist else 0
+            assert run.bo.node_tuple(node) == pu.trie_tuple(obo, hist, rho), (i, s)
+            if s % 9 == 0:
+                want = model.joint_logits(run.enc[0][i][t], last)
+                worst = max(worst, float(np.abs(logits[s, i] - want).max()))
+        assert (rows[len(ev):, i, 0] == -1).all()  # finished rows stay idle
+    assert worst < pu.LOGIT_TOL, worst
+    print(f"cfg0: max |logit - oracle| = {worst:.2e}")
+
+
+def test_cfg1_sampled_parity_full_length():
+    w = synth.WORKLOADS[1]
+    inp = pu.Inputs(w)
+    run = pu.GpuRun(inp, range(w.B), w.chunks)
+    reps = pu.replay(inp, run, [0, 21, 42, 63])
+    pu.assert_reports(reps)
+
+
+def test_cfg2_sampled_parity_full_size():
+    w = synth.WORKLOADS[2]
+    inp = pu.Inputs(w)
+    run = pu.GpuRun(inp, range(w.B), w.chunks)
+    reps = pu.replay(inp, run, [0, 129, 255])
+    pu.assert_reports(reps)
+    # the boost trie was exercised
+    assert any(run.states[c][i][1] != 0 for c in range(w.chunks) for i in range(w.B))
+
+
+def _tokens(run, i):
+    return np.concatenate([run.emitted(i, c)[0] for c in range(len(run.chunks))])
+
+
+def test_chunking_stream_independence_determinism():
+    w = synth.scaled(synth.WORKLOADS[0], B=6, T=120)
+    inp = pu.Inputs(w)
+    whole = pu.GpuRun(inp, range(6), 1)
+    # the same frames in 4 chunks of 30 carry the state across calls
+    split = pu.GpuRun(pu.Inputs(synth.scaled(w, T=30), inp.lmA, inp.ph), range(6), 4)
+    for i in range(6):
+        a = whole.emitted(i, 0)
+        b = [split.emitted(i, c) for c in range(4)]
+        assert np.array_equal(a[0], np.concatenate([x[0] for x in b]))
+        assert np.array_equal(a[1], np.concatenate([x[1] + 30 * c for c, x in enumerate(b)]))
+        assert np.array_equal(a[2], np.concatenate([x[2] for x in b]))
+    # a subset decoded alone matches the same streams inside the batch
+    sub = pu.GpuRun(inp, [4, 1], 1)
+    for j, s in enumerate([4, 1]):
+        for x, y in zip(sub.emitted(j, 0), whole.emitted(s, 0)):
+            assert np.array_equal(x, y)
+    # run to run and graph vs direct launches: bit identical
+    again = pu.GpuRun(inp, range(6), 1, graphs=False)
+    for i in range(6):
+        for x, y in zip(again.emitted(i, 0), whole.emitted(i, 0)):
+            assert np.array_equal(x, y)
+
+
+@pytest.mark.parametrize("case", ["no_lm_no_boost", "zero_weights", "unigram_lm", "one_token_phrases",
+                                  "one_symbol", "tiny"])
+def test_edge_cases(case):
+    base = synth.scaled(synth.WORKLOADS[0], B=3, T=40)
+    kw = {}
+    if case == "no_lm_no_boost":
+        inp = pu.Inputs(base, with_lm=False, with_boost=False)
+    elif case == "zero_weights":
+        inp = pu.Inputs(synth.scaled(base, lam=0.0, beta=0.0))
+    elif case == "unigram_lm":
+        inp = pu.Inputs(base, lmA=synth.ngram_lm(3, base.V, 1, base.V, 1.1))
+    elif case == "one_token_phrases":
+        inp = pu.Inputs(base, ph=synth.phrases(5, base.V, 60, 1, 2, 0.0))
+    elif case == "one_symbol":
+        inp = pu.Inputs(synth.scaled(base, max_sym=1))
+    else:  # odd vocabulary (V+1 = 16), smallest hidden size, a single stream and frame
+        w = synth.scaled(base, V=15, H=64, B=1, T=1, lm_total=60)
+        inp = pu.Inputs(w, lmA=synth.ngram_lm(7, 15, 3, 60, 1.1), ph=synth.phrases(7, 15, 3, 1, 3, 0.0))
+    run = pu.GpuRun(inp, range(inp.w.B), 2)
+    pu.assert_reports(pu.replay(inp, run, range(inp.w.B)))
+
+
+def test_zero_weights_is_plain_greedy_on_gpu():
+    """lambda = beta = 0: the GPU labels are the argmax of the raw logits
+    (checked with torch's own bf16 matmul reference on the GPU's inputs)."""
+    w = synth.scaled(synth.WORKLOADS[1], B=4, T=13, lam=0.0, beta=0.0)
+    inp = pu.Inputs(w)
+    run = pu.GpuRun(inp, range(4), 2, capture_steps=13 * 5)
+    rows = run.cap_rows.cpu().numpy()
+    Ef = torch.from_numpy(synth.bf16_to_f32(inp.E)).double()
+    Wf = torch.from_numpy(synth.bf16_to_f32(inp.W)).double()
+    for i in range(4):
+        tok, fr, _ = run.emitted(i, 0)
+        ev = _evaluations(tok, fr, w.T, w.max_sym)
+        enc = torch.from_numpy(synth.bf16_to_f32(run.enc[0][i]))
+        for s, (t, hist) in enumerate(ev):
+            last = hist[-1] if hist else w.V
+            x = torch.relu(enc[t] + Ef[last].float()).to(torch.bfloat16).double()
+            lg = x @ Wf
+            top2 = torch.topk(lg, 2).values
+            y = int(torch.argmax(lg))
+            chosen = int(tok[len(hist)]) if len(hist) < len(tok) and fr[len(hist)] == t else w.V
+            if float(top2[0] - top2[1]) > pu.GAP_TOL:
+                assert chosen == y, (i, s)
+
+
+def test_status_errors_leave_decoder_usable():
+    import paper_2609_14991_gb300 as tsd
+
+    w = synth.scaled(synth.WORKLOADS[0], B=2, T=8)
+    inp = pu.Inputs(w)
+    run = pu.GpuRun(inp, range(2), 1)
+    dec = run.dec
+    enc = torch.zeros((2, 8, w.H), dtype=torch.int16, device="cuda")
+    with pytest.raises(tsd.TsdError) as e:
+        dec.open()  # both slots in use
+    assert e.value.status == tsd.TSD_ESTATE
+    with pytest.raises(tsd.TsdError) as e:
+        dec.decode_chunk([0, 0], enc, 0.1, 0.1)
+    assert e.value.status == tsd.TSD_EINVAL
+    with pytest.raises(tsd.TsdError) as e:
+        dec.decode_chunk([0, 1], torch.zeros((2, 9, w.H), dtype=torch.int16, device="cuda"), 0.1, 0.1)
+    assert e.value.status == tsd.TSD_EINVAL
+    dec.close(1)
+    with pytest.raises(tsd.TsdError) as e:
+        dec.decode_chunk([0, 1], enc, 0.1, 0.1)
+    assert e.value.status == tsd.TSD_ESTATE
+    with pytest.raises(tsd.TsdError):
+        dec.close(1)
+    s = dec.open()
+    out = dec.decode_chunk([0, s], enc, 0.1, 0.1)
+    torch.cuda.synchronize()
+    assert out.counts.cpu().numpy().min() >= 0
