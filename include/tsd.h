@@ -225,6 +225,16 @@ TSD_API tsd_status tsd_decoder_set_timing(tsd_decoder* dec, int32_t enable);
 TSD_API tsd_status tsd_decoder_timing(tsd_decoder* dec, double* ms, int64_t* launches, int32_t n_classes,
                               int32_t reset);
 
+/* Selects the joint GEMM kernel of later decode_chunk calls: 0 (default)
+ * the tcgen05 tensor-core kernel, 1 the CUDA-core kernel (a cross-check of
+ * the same contraction and epilogue).  Drops captured graphs. */
+TSD_API tsd_status tsd_decoder_set_joint_kernel(tsd_decoder* dec, int32_t kind);
+
+/* Waits for the decoder's stream and reports a device-side failure: every
+ * wait inside the kernels is bounded, and one that expires records a code
+ * that makes this call return TSD_EDEVICE (and clears it). */
+TSD_API tsd_status tsd_decoder_check(tsd_decoder* dec);
+
 /* Kernel launches one decode_chunk(n, T) issues (for launch accounting). */
 TSD_API tsd_status tsd_decoder_launches_per_chunk(const tsd_decoder* dec, int32_t n, int32_t T,
                                           int64_t* launches);

@@ -63,6 +63,8 @@ SIGNATURES = {
     "tsd_decoder_timing": ([_vp, _vp, _vp, _i32, _i32], _i32),
     "tsd_decoder_launches_per_chunk": ([_vp, _i32, _i32, _P(_i64)], _i32),
     "tsd_decoder_debug_capture": ([_vp, _vp, _vp, _i32], _i32),
+    "tsd_decoder_set_joint_kernel": ([_vp, _i32], _i32),
+    "tsd_decoder_check": ([_vp], _i32),
 }
 
 _lib = None
@@ -282,6 +284,14 @@ class Decoder:
 
     def set_graphs(self, enable: bool):
         _check(lib().tsd_decoder_set_graphs(self.h, 1 if enable else 0))
+
+    def set_joint_kernel(self, kind: int):
+        """0 = tcgen05 tensor-core GEMM (default), 1 = CUDA-core cross-check kernel."""
+        _check(lib().tsd_decoder_set_joint_kernel(self.h, int(kind)))
+
+    def check(self):
+        """Raises TsdError(EDEVICE) if a bounded device wait expired."""
+        _check(lib().tsd_decoder_check(self.h))
 
     def set_timing(self, enable: bool):
         _check(lib().tsd_decoder_set_timing(self.h, 1 if enable else 0))

@@ -13,6 +13,7 @@
 #include <new>
 
 #include "decoder.h"
+#include "joint_tc.h"
 
 using namespace tsd;
 
@@ -42,7 +43,8 @@ void enqueue_chunk(tsd_decoder* d, int M, int T, cudaStream_t s, const std::vect
     launch_row(d->view, M, step, step == S ? 1 : 0, d->row_smem, s);
     if (step < S) {
       mark();
-      launch_joint(d->view, M, step, s);
+      if (d->joint_kind == 0) launch_joint_tc(*d->jtc, d->view, M, step, s);
+      else launch_joint(d->view, M, step, s);
     }
   }
   mark();
@@ -111,14 +113,14 @@ extern "C" tsd_status tsd_decoder_create(const tsd_decoder_cfg* cfg, const void*
   uint16_t *Wt, *E, *Abuf;
   float* bias;
   float4* part;
-  int32_t *rt, *rs, *rc, *sl, *sll, *slc, *stl, *stc;
+  int32_t *rt, *rs, *rc, *sl, *sll, *slc, *stl, *stc, *err;
   const size_t SK = (size_t)c.max_streams * c.beam_k;
   d->params_bytes = sizeof(Params) + sizeof(int32_t) * (size_t)c.max_streams;
   char* pdev = nullptr;
   tsd_status st;
   if ((st = A.alloc(&Wt, (size_t)d->N_pad * c.H)) || (st = A.alloc(&E, (size_t)d->N * c.H)) ||
       (st = A.alloc(&Abuf, (size_t)d->M_pad * c.H)) || (st = A.alloc(&bias, (size_t)d->M_pad * d->N_pad)) ||
-      (st = A.alloc(&part, (size_t)d->M_pad * d->n_ptiles)) || (st = A.alloc(&rt, (size_t)d->M_pad)) ||
+      (st = A.alloc(&part, (size_t)d->M_pad * (d->N_pad / 64))) || (st = A.alloc(&err, 1)) || (st = A.alloc(&rt, (size_t)d->M_pad)) ||
       (st = A.alloc(&rs, (size_t)d->M_pad)) || (st = A.alloc(&rc, (size_t)d->M_pad)) ||
       (st = A.alloc(&sl, SK)) || (st = A.alloc(&sll, SK)) || (st = A.alloc(&slc, SK * kLmChain)) ||
       (st = A.alloc(&stl, SK)) || (st = A.alloc(&stc, SK * kTrChain)) || (st = A.alloc(&pdev, d->params_bytes))) {
@@ -126,6 +128,8 @@ extern "C" tsd_status tsd_decoder_create(const tsd_decoder_cfg* cfg, const void*
     return st;
   }
   auto cleanup = [&](tsd_status e) {
+    delete d->jtc;
+    d->jtc = nullptr;
     for (int i = 0; i < tsd_decoder::kRing; ++i) {
       if (d->staging[i]) cudaFreeHost(d->staging[i]);
       if (d->staging_ev[i]) cudaEventDestroy(d->staging_ev[i]);
@@ -139,11 +143,22 @@ extern "C" tsd_status tsd_decoder_create(const tsd_decoder_cfg* cfg, const void*
       (ce = cudaMemsetAsync(bias, 0, sizeof(float) * (size_t)d->M_pad * d->N_pad, s)) != cudaSuccess ||
       (ce = cudaMemsetAsync(sll, 0, sizeof(int32_t) * SK, s)) != cudaSuccess ||
       (ce = cudaMemsetAsync(stl, 0, sizeof(int32_t) * SK, s)) != cudaSuccess ||
+      (ce = cudaMemsetAsync(err, 0, sizeof(int32_t), s)) != cudaSuccess ||
       (ce = cudaMemcpyAsync(E, E_bf16, sizeof(uint16_t) * (size_t)d->N * c.H, cudaMemcpyDeviceToDevice, s)) != cudaSuccess)
     return cleanup(cuda_fail(ce, "tsd_decoder_create: initial copies"));
   launch_repack(static_cast<const uint16_t*>(W_out_bf16), Wt, c.H, d->N, d->N_pad, s);
   if ((ce = cudaGetLastError()) != cudaSuccess) return cleanup(cuda_fail(ce, "tsd_decoder_create: repack"));
   if ((ce = prepare_kernels(d->row_smem)) != cudaSuccess) return cleanup(cuda_fail(ce, "tsd_decoder_create: kernel attributes"));
+  {
+    int sms = 0;
+    if ((ce = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, d->device)) != cudaSuccess)
+      return cleanup(cuda_fail(ce, "tsd_decoder_create: SM count"));
+    d->jtc = new (std::nothrow) JointTc();
+    if (!d->jtc) return cleanup(fail(TSD_ENOMEM, "tsd_decoder_create: host allocation failed"));
+    const int bn = joint_tc_pick_bn(d->M_max, d->N_pad, sms);
+    if ((ce = joint_tc_prepare(d->jtc, Abuf, d->M_pad, Wt, d->N_pad, c.H, bn)) != cudaSuccess)
+      return cleanup(cuda_fail(ce, "tsd_decoder_create: tensor-core GEMM setup (TMA descriptors)"));
+  }
   for (int i = 0; i < tsd_decoder::kRing; ++i) {
     if ((ce = cudaHostAlloc(reinterpret_cast<void**>(&d->staging[i]), d->params_bytes, cudaHostAllocDefault)) != cudaSuccess)
       return cleanup(fail(TSD_ENOMEM, "tsd_decoder_create: pinned staging: %s", cudaGetErrorString(ce)));
@@ -159,6 +174,7 @@ extern "C" tsd_status tsd_decoder_create(const tsd_decoder_cfg* cfg, const void*
   v.H = c.H;
   v.max_sym = c.max_symbols;
   v.K = c.beam_k;
+  d->n_ptiles = d->N_pad / d->jtc->bn;
   v.n_ptiles = d->n_ptiles;
   v.V4 = d->V4;
   v.params = reinterpret_cast<const Params*>(pdev);
@@ -183,6 +199,7 @@ extern "C" tsd_status tsd_decoder_create(const tsd_decoder_cfg* cfg, const void*
   v.cap_logits = nullptr;
   v.cap_rows = nullptr;
   v.cap_steps = 0;
+  v.err = err;
   d->slot_open.assign((size_t)c.max_streams, 0);
   d->last_stream = s;
   *out = d.release();
@@ -203,6 +220,7 @@ extern "C" void tsd_decoder_free(tsd_decoder* d) {
   }
   if (d->cap_stream) cudaStreamDestroy(d->cap_stream);
   d->arena.release();
+  delete d->jtc;
   cudaGetLastError();
   delete d;
 }
@@ -393,6 +411,47 @@ extern "C" tsd_status tsd_decoder_launches_per_chunk(const tsd_decoder* d, int32
   return TSD_OK;
 }
 
+namespace {
+tsd_status drop_graphs(tsd_decoder* d) {
+  tsd_status st = set_device(d);
+  if (st) return st;
+  cudaDeviceSynchronize();
+  for (auto& kv : d->entries) {
+    harvest(d, kv.second.set[0]);
+    harvest(d, kv.second.set[1]);
+    destroy_set(kv.second.set[0]);
+    destroy_set(kv.second.set[1]);
+  }
+  d->entries.clear();
+  return TSD_OK;
+}
+}  // namespace
+
+extern "C" tsd_status tsd_decoder_set_joint_kernel(tsd_decoder* d, int32_t kind) {
+  clear_error();
+  if (!d) return fail(TSD_EINVAL, "tsd_decoder_set_joint_kernel: NULL decoder");
+  if (kind != 0 && kind != 1) return fail(TSD_EINVAL, "tsd_decoder_set_joint_kernel: kind must be 0 or 1");
+  d->joint_kind = kind;
+  d->n_ptiles = kind == 0 ? d->N_pad / d->jtc->bn : d->N_pad / kPartialCols;
+  d->view.n_ptiles = d->n_ptiles;
+  return drop_graphs(d);
+}
+
+extern "C" tsd_status tsd_decoder_check(tsd_decoder* d) {
+  clear_error();
+  if (!d) return fail(TSD_EINVAL, "tsd_decoder_check: NULL decoder");
+  tsd_status st = set_device(d);
+  if (st) return st;
+  TSD_CUDA(cudaStreamSynchronize(d->last_stream));
+  int32_t e = 0;
+  TSD_CUDA(cudaMemcpy(&e, d->view.err, sizeof(e), cudaMemcpyDeviceToHost));
+  if (e) {
+    TSD_CUDA(cudaMemset(d->view.err, 0, sizeof(e)));
+    return fail(TSD_EDEVICE, "tsd_decoder_check: a device wait expired (code 0x%x)", e);
+  }
+  return TSD_OK;
+}
+
 extern "C" tsd_status tsd_decoder_debug_capture(tsd_decoder* d, float* logits, int32_t* rows,
                                                 int32_t max_steps) {
   clear_error();
@@ -401,14 +460,5 @@ extern "C" tsd_status tsd_decoder_debug_capture(tsd_decoder* d, float* logits, i
   d->view.cap_logits = logits;
   d->view.cap_rows = rows;
   d->view.cap_steps = (logits || rows) ? max_steps : 0;
-  // captured graphs bake the view in: drop them
-  tsd_status st = set_device(d);
-  if (st) return st;
-  cudaDeviceSynchronize();
-  for (auto& kv : d->entries) {
-    destroy_set(kv.second.set[0]);
-    destroy_set(kv.second.set[1]);
-  }
-  d->entries.clear();
-  return TSD_OK;
+  return drop_graphs(d);  // captured graphs bake the view in
 }

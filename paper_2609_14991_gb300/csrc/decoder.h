@@ -9,6 +9,7 @@
 #include "internal.h"
 
 namespace tsd {
+struct JointTc;
 
 // Per-call parameters, copied to the device before each chunk so that one
 // captured graph serves every call of the same shape.
@@ -47,6 +48,7 @@ struct DecView {
   float* cap_logits;
   int32_t* cap_rows;
   int32_t cap_steps;
+  int32_t* err;  // device status word: nonzero after a bounded wait expired
 };
 
 constexpr int kRowThreads = 256;
@@ -90,6 +92,8 @@ struct tsd_decoder {
     int next = 0;
   };
   std::map<std::tuple<int, int, int, int>, Entry> entries;  // (n, T, graphs, timing)
+  tsd::JointTc* jtc = nullptr;  // tensor-core joint kernel state
+  int joint_kind = 0;           // 0 tensor cores, 1 CUDA cores
   double ms[2] = {0, 0};
   int64_t launches[2] = {0, 0};
 };

@@ -1,0 +1,347 @@
+// Joint GEMM on the 5th-generation tensor cores (tcgen05) with the fused
+// selection epilogue.
+//
+// logits[r][v] = sum_k A[r][k] * Wt[v][k]: A (joint input, bf16 [M][H]) and
+// Wt (W_out label-major, bf16 [N_pad][H]) are both K-major, loaded by TMA
+// into 128-byte-swizzled shared-memory stages; one elected thread issues
+// tcgen05.mma (kind::f16, bf16 x bf16 -> fp32) into a 128 x BN accumulator in
+// tensor memory.  Four epilogue warps read the accumulator back with
+// tcgen05.ld (thread = row) and reduce it on chip to the row's selection
+// partial for this tile: softmax max and sum over the real labels, and the
+// best fused value logit + bias (lambda*LM + beta*boost; blank gets 0), ties
+// to the lowest label.  Logits never leave the SM.
+//
+// Warp roles (192 threads): warp 0 TMA producer, warp 1 TMEM allocator and
+// MMA issuer, warps 2-5 epilogue.  Every wait on an mbarrier is bounded in
+// time; on expiry the kernel records an error in the decoder's status word,
+// drains its own copies and returns.
+#include <cuda.h>
+
+#include "decoder.h"
+#include "joint_tc.h"
+
+namespace tsd {
+
+namespace {
+
+constexpr int kBM = 128, kBK = 64;
+constexpr int kThreads = 192;
+constexpr float kNegInf = -__builtin_huge_valf();
+constexpr unsigned long long kWaitNs = 1000000000ull;  // 1 s bound on any barrier wait
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ unsigned long long global_ns() {
+  unsigned long long t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+
+__device__ __forceinline__ void mbar_init(uint64_t* b, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(b)), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void mbar_expect_tx(uint64_t* b, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(b)), "r"(bytes) : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try(uint64_t* b, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(smem_u32(b)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+// Waits for the phase of the given parity; false if it did not complete
+// within kWaitNs.
+__device__ __forceinline__ bool mbar_wait(uint64_t* b, uint32_t parity) {
+  if (mbar_try(b, parity)) return true;
+  const unsigned long long t0 = global_ns();
+  while (!mbar_try(b, parity)) {
+    if (global_ns() - t0 > kWaitNs) return false;
+  }
+  return true;
+}
+
+__device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, uint64_t* bar, int x, int y) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(
+          smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_u32(bar))
+      : "memory");
+}
+
+// Shared-memory matrix descriptor of a K-major tile stored with the 128-byte
+// swizzle: rows of 64 bf16 (128 B), 8-row groups 1024 B apart.
+__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
+  uint64_t d = 0;
+  d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);   // start address
+  d |= (uint64_t)1 << 16;                      // leading byte offset (unused for swizzled K-major)
+  d |= (uint64_t)(1024 >> 4) << 32;            // stride byte offset: next 8-row group
+  d |= (uint64_t)1 << 46;                      // descriptor version
+  d |= (uint64_t)2 << 61;                      // 128-byte swizzle
+  return d;
+}
+
+// Instruction descriptor: kind::f16, A = B = bf16, D = f32, both K-major.
+__host__ __device__ constexpr uint32_t idesc_bf16(int M, int N) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
+}
+
+__device__ __forceinline__ void mma_bf16(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
+                                         uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(tmem_d),
+      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+__device__ __forceinline__ void mma_commit(uint64_t* bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(bar))
+               : "memory");
+}
+
+__device__ __forceinline__ void fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+
+// 32 consecutive fp32 columns of this warp's 32 TMEM lanes (one per thread).
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float* v) {
+  uint32_t r[32];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+      "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, "
+      "%16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
+        "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
+        "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+template <int BN>
+struct Smem {
+  static constexpr int kStages = (BN == 256) ? 4 : 6;
+  static constexpr int kABytes = kBM * kBK * 2;
+  static constexpr int kBBytes = BN * kBK * 2;
+  static constexpr int kStageBytes = kABytes + kBBytes;
+  static constexpr int kBytes = kStages * kStageBytes + 1024 /*align*/ + 256 /*barriers*/;
+};
+
+template <int BN>
+__global__ void __launch_bounds__(kThreads, 1)
+    k_joint_tc(DecView d, int step, const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB) {
+  using S = Smem<BN>;
+  extern __shared__ __align__(1024) unsigned char smem_raw[];
+  unsigned char* smem = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + S::kStages * S::kStageBytes);
+  uint64_t* empty = full + S::kStages;
+  uint64_t* accum = empty + S::kStages;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(accum + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int n0 = blockIdx.x * BN, m0 = blockIdx.y * kBM;
+  const int M = d.params->n * d.K;
+  const int KB = d.H / kBK;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < S::kStages; ++s) {
+      mbar_init(full + s, 1);
+      mbar_init(empty + s, 1);
+    }
+    mbar_init(accum, 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
+                 "r"(BN)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  fence_before();
+  __syncthreads();
+  fence_after();
+  const uint32_t tmem = *tmem_slot;
+  bool ok = true;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      int issued = 0;
+      for (int kb = 0; kb < KB; ++kb) {
+        const int s = kb % S::kStages;
+        const uint32_t ph = (uint32_t)(kb / S::kStages) & 1u;
+        if (!mbar_wait(empty + s, ph ^ 1u)) { ok = false; break; }
+        unsigned char* sa = smem + s * S::kStageBytes;
+        mbar_expect_tx(full + s, S::kStageBytes);
+        tma_load_2d(sa, &tmA, full + s, kb * kBK, m0);
+        tma_load_2d(sa + S::kABytes, &tmB, full + s, kb * kBK, n0);
+        ++issued;
+      }
+      if (!ok) {
+        // drain the copies this CTA still has in flight before it exits
+        for (int kb = max(0, issued - S::kStages); kb < issued; ++kb)
+          mbar_wait(full + kb % S::kStages, (uint32_t)(kb / S::kStages) & 1u);
+        atomicOr(d.err, 1);
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      const uint32_t idesc = idesc_bf16(kBM, BN);
+      for (int kb = 0; kb < KB; ++kb) {
+        const int s = kb % S::kStages;
+        const uint32_t ph = (uint32_t)(kb / S::kStages) & 1u;
+        if (!mbar_wait(full + s, ph)) { ok = false; break; }
+        fence_after();
+        const uint32_t sa = smem_u32(smem + s * S::kStageBytes);
+        const uint64_t ad = sw128_desc(sa), bd = sw128_desc(sa + S::kABytes);
+#pragma unroll
+        for (int k = 0; k < kBK / 16; ++k)  // K = 16 per instruction: +32 bytes in the swizzle atom
+          mma_bf16(tmem, ad + (uint64_t)(2 * k), bd + (uint64_t)(2 * k), idesc, (kb | k) ? 1u : 0u);
+        mma_commit(empty + s);
+      }
+      // signals the epilogue once every issued MMA has completed (also after a
+      // timeout, so nothing is in flight when TMEM is released)
+      mma_commit(accum);
+      if (!ok) atomicOr(d.err, 2);
+    }
+    __syncwarp();
+  } else {
+    // epilogue: warps 2..5, thread = row of the tile
+    const int q = warp & 3;  // TMEM lane quadrant this warp may access
+    const int row = q * 32 + lane;
+    const int gr = m0 + row;
+    const bool live = gr < M;
+    const int N = d.N, V = d.V;
+    const float* brow = d.bias + (size_t)(live ? gr : 0) * d.N_pad + n0;
+    float mx = kNegInf, se = 0.f, bv = kNegInf;
+    int bi = INT_MAX;
+    ok = __all_sync(0xffffffffu, mbar_wait(accum, 0));  // warp-uniform: tcgen05.ld is .sync.aligned
+    if (!ok && lane == 0) atomicOr(d.err, 4);
+    fence_after();
+    if (ok) {
+      const uint32_t tbase = tmem + ((uint32_t)(q * 32) << 16);
+      float4 bnext[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) bnext[i] = live ? __ldg(reinterpret_cast<const float4*>(brow) + i) : make_float4(0, 0, 0, 0);
+#pragma unroll 1
+      for (int c = 0; c < BN / 32; ++c) {
+        float b[32];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          b[4 * i] = bnext[i].x; b[4 * i + 1] = bnext[i].y; b[4 * i + 2] = bnext[i].z; b[4 * i + 3] = bnext[i].w;
+        }
+        if (c + 1 < BN / 32) {
+#pragma unroll
+          for (int i = 0; i < 8; ++i)
+            bnext[i] = live ? __ldg(reinterpret_cast<const float4*>(brow + (c + 1) * 32) + i) : make_float4(0, 0, 0, 0);
+        }
+        float l[32];
+        tmem_ld32(tbase + (uint32_t)(c * 32), l);
+        const int c0 = n0 + c * 32;
+        float cm = kNegInf;
+#pragma unroll
+        for (int i = 0; i < 32; ++i) {
+          const int gc = c0 + i;
+          if (gc < N) {
+            cm = fmaxf(cm, l[i]);
+            const float f = l[i] + (gc < V ? b[i] : 0.f);
+            if (f > bv) { bv = f; bi = gc; }
+          }
+        }
+        if (cm != kNegInf) {
+          const float m2 = fmaxf(mx, cm);
+          float acc = (mx == kNegInf) ? 0.f : se * exp2f((mx - m2) * 1.4426950408889634f);
+#pragma unroll
+          for (int i = 0; i < 32; ++i)
+            if (c0 + i < N) acc += exp2f((l[i] - m2) * 1.4426950408889634f);
+          se = acc;
+          mx = m2;
+        }
+        if (d.cap_logits && step < d.cap_steps && live) {
+          float* cl = d.cap_logits + ((size_t)step * M + gr) * N;
+#pragma unroll
+          for (int i = 0; i < 32; ++i)
+            if (c0 + i < N) cl[c0 + i] = l[i];
+        }
+      }
+      if (live) d.part[(size_t)gr * d.n_ptiles + blockIdx.x] = make_float4(mx, se, bv, __int_as_float(bi));
+    }
+  }
+  fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(BN) : "memory");
+  }
+}
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  if (!fn) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+  }
+  return fn;
+}
+
+bool make_map(CUtensorMap* m, const void* base, int K, int rows, int box_rows) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {(cuuint64_t)K, (cuuint64_t)rows};
+  cuuint64_t strides[1] = {(cuuint64_t)K * 2};
+  cuuint32_t box[2] = {(cuuint32_t)kBK, (cuuint32_t)box_rows};
+  cuuint32_t es[2] = {1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, es,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+}  // namespace
+
+int joint_tc_pick_bn(int M_max, int N_pad, int sms) {
+  const int mt = (M_max + kBM - 1) / kBM;
+  if (mt * (N_pad / 256) >= sms) return 256;
+  if (mt * (N_pad / 128) >= sms / 2) return 128;
+  return 64;
+}
+
+cudaError_t joint_tc_prepare(JointTc* jt, const uint16_t* A, int M_pad, const uint16_t* Wt, int N_pad, int H, int bn) {
+  jt->bn = bn;
+  if (!make_map(&jt->mapA, A, H, M_pad, kBM)) return cudaErrorInvalidValue;
+  if (!make_map(&jt->mapB, Wt, H, N_pad, bn)) return cudaErrorInvalidValue;
+  cudaError_t e = cudaSuccess;
+  if (bn == 256) e = cudaFuncSetAttribute(k_joint_tc<256>, cudaFuncAttributeMaxDynamicSharedMemorySize, Smem<256>::kBytes);
+  else if (bn == 128) e = cudaFuncSetAttribute(k_joint_tc<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, Smem<128>::kBytes);
+  else e = cudaFuncSetAttribute(k_joint_tc<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, Smem<64>::kBytes);
+  return e;
+}
+
+void launch_joint_tc(const JointTc& jt, const DecView& d, int M, int step, cudaStream_t s) {
+  dim3 grid(d.N_pad / jt.bn, (M + kBM - 1) / kBM);
+  if (jt.bn == 256)
+    k_joint_tc<256><<<grid, kThreads, Smem<256>::kBytes, s>>>(d, step, jt.mapA, jt.mapB);
+  else if (jt.bn == 128)
+    k_joint_tc<128><<<grid, kThreads, Smem<128>::kBytes, s>>>(d, step, jt.mapA, jt.mapB);
+  else
+    k_joint_tc<64><<<grid, kThreads, Smem<64>::kBytes, s>>>(d, step, jt.mapA, jt.mapB);
+}
+
+}  // namespace tsd

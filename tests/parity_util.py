@@ -49,7 +49,7 @@ class GpuRun:
     """Decodes `streams` (stream ids of the workload) for `chunks` chunks."""
 
     def __init__(self, inp: Inputs, streams: Sequence[int], chunks: int, T: Optional[int] = None,
-                 capture_steps: int = 0, graphs: bool = True):
+                 capture_steps: int = 0, graphs: bool = True, joint_kind: int = 0):
         import torch
 
         import paper_2609_14991_gb300 as tsd
@@ -66,6 +66,8 @@ class GpuRun:
         self.dec = tsd.Decoder(w.V, w.H, Wt, Et, lm=self.lm, boost=self.bo, max_symbols=w.max_sym, beam_k=1,
                                max_streams=n, max_T=self.T)
         self.dec.set_graphs(graphs)
+        if joint_kind:
+            self.dec.set_joint_kernel(joint_kind)
         self.slots = [self.dec.open() for _ in range(n)]
         self.cap_logits = self.cap_rows = None
         if capture_steps:
@@ -85,6 +87,7 @@ class GpuRun:
             self.chunks.append({"count": cnt, "tok": tok, "frame": fr, "score": sc})
             self.enc.append(enc)
             self.states.append([self.dec.state(s) for s in self.slots])
+        self.dec.check()  # no bounded device wait expired
 
     def emitted(self, i: int, c: int):
         d = self.chunks[c]
