@@ -134,7 +134,7 @@ TSD_API tsd_status tsd_boost_node_tuple(const tsd_boost* b, int32_t node, int32_
  * Decoder.
  */
 typedef struct {
-  int32_t V;           /* non-blank labels; blank = V; 1 <= V <= 32767 */
+  int32_t V;           /* non-blank labels; blank = V; 1 <= V <= 16384 */
   int32_t H;           /* joint hidden size; multiple of 64, 64 <= H <= 8192 */
   int32_t max_symbols; /* labels per frame (greedy; Sec. III); beam requires 1 */
   int32_t beam_k;      /* 1 = greedy; 2..8 = beam search */
@@ -234,6 +234,29 @@ TSD_API tsd_status tsd_decoder_set_joint_kernel(tsd_decoder* dec, int32_t kind);
  * wait inside the kernels is bounded, and one that expires records a code
  * that makes this call return TSD_EDEVICE (and clears it). */
 TSD_API tsd_status tsd_decoder_check(tsd_decoder* dec);
+
+/* Tuning knobs, by name (drops captured graphs):
+ *   "pdl"      1 (default) / 0: programmatic dependent launch between the
+ *              row pass and the joint kernel, so each kernel's set-up
+ *              overlaps the tail of the one before;
+ *   "joint_bn" 64, 128 or 256: labels per tensor-core CTA tile (default:
+ *              chosen at create from the row count and the SM count).
+ * Unknown names return TSD_EINVAL. */
+TSD_API tsd_status tsd_decoder_set_option(tsd_decoder* dec, const char* name, int64_t value);
+
+/* Measurement hook: launches one kernel of the last decode_chunk's final
+ * label step reps times back to back on cuda_stream -- kernel 0 the row
+ * pass (in a mode that redoes the step's work but commits no state or
+ * output), kernel 1 the joint GEMM (idempotent) -- so a caller can time it
+ * with CUDA events in isolation.  Later decode_chunk calls are unaffected.
+ * If algo_bytes is non-NULL the call waits for the stream and stores the
+ * algorithmic bytes of one launch: for the row pass, counted by the kernel
+ * (partials, row state, label searches, joint input, every LM arc and trie
+ * child of the chains, plus the shared unigram/root rows once; not the
+ * dense bias it writes); for the joint kernel, its operands, bias rows and
+ * partials.  TSD_ESTATE before the first decode_chunk. */
+TSD_API tsd_status tsd_decoder_replay(tsd_decoder* dec, int32_t kernel, int32_t reps, void* cuda_stream,
+                                      int64_t* algo_bytes);
 
 /* Kernel launches one decode_chunk(n, T) issues (for launch accounting). */
 TSD_API tsd_status tsd_decoder_launches_per_chunk(const tsd_decoder* dec, int32_t n, int32_t T,

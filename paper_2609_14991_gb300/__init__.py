@@ -65,6 +65,8 @@ SIGNATURES = {
     "tsd_decoder_debug_capture": ([_vp, _vp, _vp, _i32], _i32),
     "tsd_decoder_set_joint_kernel": ([_vp, _i32], _i32),
     "tsd_decoder_check": ([_vp], _i32),
+    "tsd_decoder_set_option": ([_vp, ctypes.c_char_p, _i64], _i32),
+    "tsd_decoder_replay": ([_vp, _i32, _i32, _vp, _P(_i64)], _i32),
 }
 
 _lib = None
@@ -288,6 +290,18 @@ class Decoder:
     def set_joint_kernel(self, kind: int):
         """0 = tcgen05 tensor-core GEMM (default), 1 = CUDA-core cross-check kernel."""
         _check(lib().tsd_decoder_set_joint_kernel(self.h, int(kind)))
+
+    def set_option(self, name: str, value: int):
+        _check(lib().tsd_decoder_set_option(self.h, name.encode(), int(value)))
+
+    def replay(self, kernel: int, reps: int, stream=None, count_bytes: bool = False) -> int:
+        """Re-launch one kernel (0 row pass, 1 joint) of the last chunk's final
+        step reps times, for timing; with count_bytes, returns the algorithmic
+        bytes of one launch (and waits for the stream)."""
+        b = _i64(0)
+        _check(lib().tsd_decoder_replay(self.h, int(kernel), int(reps), _stream(stream),
+                                        ctypes.byref(b) if count_bytes else None))
+        return b.value
 
     def check(self):
         """Raises TsdError(EDEVICE) if a bounded device wait expired."""

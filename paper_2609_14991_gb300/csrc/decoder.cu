@@ -11,6 +11,7 @@
 #include <cstring>
 #include <memory>
 #include <new>
+#include <string>
 
 #include "decoder.h"
 #include "joint_tc.h"
@@ -39,11 +40,12 @@ void enqueue_chunk(tsd_decoder* d, int M, int T, cudaStream_t s, const std::vect
     if (ev) cudaEventRecordWithFlags((*ev)[(size_t)e++], s, cudaEventRecordExternal);
   };
   for (int step = 0; step <= S; ++step) {
+    const bool pdl = d->pdl && !ev && step > 0;  // the first launch follows the parameter copy
     mark();
-    launch_row(d->view, M, step, step == S ? 1 : 0, d->row_smem, s);
+    launch_row(d->view, M, step, step == S ? 1 : 0, d->row_smem, s, pdl);
     if (step < S) {
       mark();
-      if (d->joint_kind == 0) launch_joint_tc(*d->jtc, d->view, M, step, s);
+      if (d->joint_kind == 0) launch_joint_tc(*d->jtc, d->view, M, step, s, d->pdl && !ev);
       else launch_joint(d->view, M, step, s);
     }
   }
@@ -82,7 +84,7 @@ extern "C" tsd_status tsd_decoder_create(const tsd_decoder_cfg* cfg, const void*
   *out = nullptr;
   if (!cfg || !W_out_bf16 || !E_bf16) return fail(TSD_EINVAL, "tsd_decoder_create: NULL argument");
   const tsd_decoder_cfg c = *cfg;
-  if (c.V < 1 || c.V > 32767) return fail(TSD_EINVAL, "tsd_decoder_create: V=%d out of range", c.V);
+  if (c.V < 1 || c.V > 16384) return fail(TSD_EINVAL, "tsd_decoder_create: V=%d out of range [1, 16384]", c.V);
   if (c.H < 64 || c.H > 8192 || c.H % 64) return fail(TSD_EINVAL, "tsd_decoder_create: H=%d must be a multiple of 64 in [64, 8192]", c.H);
   if (c.beam_k != 1) return fail(TSD_EINVAL, "tsd_decoder_create: beam_k=%d not supported by this build (greedy only)", c.beam_k);
   if (c.max_symbols < 1 || c.max_symbols > 64) return fail(TSD_EINVAL, "tsd_decoder_create: max_symbols=%d out of range", c.max_symbols);
@@ -114,13 +116,14 @@ extern "C" tsd_status tsd_decoder_create(const tsd_decoder_cfg* cfg, const void*
   float* bias;
   float4* part;
   int32_t *rt, *rs, *rc, *sl, *sll, *slc, *stl, *stc, *err;
+  unsigned long long* ctr;
   const size_t SK = (size_t)c.max_streams * c.beam_k;
   d->params_bytes = sizeof(Params) + sizeof(int32_t) * (size_t)c.max_streams;
   char* pdev = nullptr;
   tsd_status st;
   if ((st = A.alloc(&Wt, (size_t)d->N_pad * c.H)) || (st = A.alloc(&E, (size_t)d->N * c.H)) ||
       (st = A.alloc(&Abuf, (size_t)d->M_pad * c.H)) || (st = A.alloc(&bias, (size_t)d->M_pad * d->N_pad)) ||
-      (st = A.alloc(&part, (size_t)d->M_pad * (d->N_pad / 64))) || (st = A.alloc(&err, 1)) || (st = A.alloc(&rt, (size_t)d->M_pad)) ||
+      (st = A.alloc(&part, (size_t)d->M_pad * (d->N_pad / 64))) || (st = A.alloc(&err, 1)) || (st = A.alloc(&ctr, 1)) || (st = A.alloc(&rt, (size_t)d->M_pad)) ||
       (st = A.alloc(&rs, (size_t)d->M_pad)) || (st = A.alloc(&rc, (size_t)d->M_pad)) ||
       (st = A.alloc(&sl, SK)) || (st = A.alloc(&sll, SK)) || (st = A.alloc(&slc, SK * kLmChain)) ||
       (st = A.alloc(&stl, SK)) || (st = A.alloc(&stc, SK * kTrChain)) || (st = A.alloc(&pdev, d->params_bytes))) {
@@ -144,6 +147,7 @@ extern "C" tsd_status tsd_decoder_create(const tsd_decoder_cfg* cfg, const void*
       (ce = cudaMemsetAsync(sll, 0, sizeof(int32_t) * SK, s)) != cudaSuccess ||
       (ce = cudaMemsetAsync(stl, 0, sizeof(int32_t) * SK, s)) != cudaSuccess ||
       (ce = cudaMemsetAsync(err, 0, sizeof(int32_t), s)) != cudaSuccess ||
+      (ce = cudaMemsetAsync(ctr, 0, sizeof(unsigned long long), s)) != cudaSuccess ||
       (ce = cudaMemcpyAsync(E, E_bf16, sizeof(uint16_t) * (size_t)d->N * c.H, cudaMemcpyDeviceToDevice, s)) != cudaSuccess)
     return cleanup(cuda_fail(ce, "tsd_decoder_create: initial copies"));
   launch_repack(static_cast<const uint16_t*>(W_out_bf16), Wt, c.H, d->N, d->N_pad, s);
@@ -155,6 +159,7 @@ extern "C" tsd_status tsd_decoder_create(const tsd_decoder_cfg* cfg, const void*
       return cleanup(cuda_fail(ce, "tsd_decoder_create: SM count"));
     d->jtc = new (std::nothrow) JointTc();
     if (!d->jtc) return cleanup(fail(TSD_ENOMEM, "tsd_decoder_create: host allocation failed"));
+    d->sms = sms;
     const int bn = joint_tc_pick_bn(d->M_max, d->N_pad, sms);
     if ((ce = joint_tc_prepare(d->jtc, Abuf, d->M_pad, Wt, d->N_pad, c.H, bn)) != cudaSuccess)
       return cleanup(cuda_fail(ce, "tsd_decoder_create: tensor-core GEMM setup (TMA descriptors)"));
@@ -200,6 +205,7 @@ extern "C" tsd_status tsd_decoder_create(const tsd_decoder_cfg* cfg, const void*
   v.cap_rows = nullptr;
   v.cap_steps = 0;
   v.err = err;
+  v.ctr = ctr;
   d->slot_open.assign((size_t)c.max_streams, 0);
   d->last_stream = s;
   *out = d.release();
@@ -296,6 +302,8 @@ extern "C" tsd_status tsd_decode_chunk(tsd_decoder* d, int32_t n, const int32_t*
 
   const int M = n * d->cfg.beam_k;
   const int S = steps_per_chunk(d, T);
+  d->last_n = n;
+  d->last_T = T;
   const int n_events = 2 * S + 2;
   auto key = std::make_tuple(n, T, d->use_graphs, d->timing);
   tsd_decoder::Entry& ent = d->entries[key];
@@ -435,6 +443,65 @@ extern "C" tsd_status tsd_decoder_set_joint_kernel(tsd_decoder* d, int32_t kind)
   d->n_ptiles = kind == 0 ? d->N_pad / d->jtc->bn : d->N_pad / kPartialCols;
   d->view.n_ptiles = d->n_ptiles;
   return drop_graphs(d);
+}
+
+extern "C" tsd_status tsd_decoder_set_option(tsd_decoder* d, const char* name, int64_t value) {
+  clear_error();
+  if (!d || !name) return fail(TSD_EINVAL, "tsd_decoder_set_option: NULL argument");
+  const std::string n(name);
+  if (n == "pdl") {
+    d->pdl = value ? 1 : 0;
+    return drop_graphs(d);
+  }
+  if (n == "joint_bn") {
+    if (value != 64 && value != 128 && value != 256) return fail(TSD_EINVAL, "tsd_decoder_set_option: joint_bn must be 64, 128 or 256");
+    tsd_status st = drop_graphs(d);
+    if (st) return st;
+    cudaError_t ce = joint_tc_prepare(d->jtc, d->view.A, d->M_pad, d->view.Wt, d->N_pad, d->cfg.H, (int)value);
+    if (ce != cudaSuccess) return cuda_fail(ce, "tsd_decoder_set_option: joint_bn");
+    if (d->joint_kind == 0) {
+      d->n_ptiles = d->N_pad / d->jtc->bn;
+      d->view.n_ptiles = d->n_ptiles;
+    }
+    return TSD_OK;
+  }
+  return fail(TSD_EINVAL, "tsd_decoder_set_option: unknown option '%s'", name);
+}
+
+extern "C" tsd_status tsd_decoder_replay(tsd_decoder* d, int32_t kernel, int32_t reps, void* cuda_stream,
+                                         int64_t* algo_bytes) {
+  clear_error();
+  if (!d) return fail(TSD_EINVAL, "tsd_decoder_replay: NULL decoder");
+  if (kernel != 0 && kernel != 1) return fail(TSD_EINVAL, "tsd_decoder_replay: kernel must be 0 (row pass) or 1 (joint)");
+  if (reps < 1) return fail(TSD_EINVAL, "tsd_decoder_replay: reps < 1");
+  if (d->last_n < 1) return fail(TSD_ESTATE, "tsd_decoder_replay: no chunk decoded yet");
+  tsd_status st = set_device(d);
+  if (st) return st;
+  cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
+  const int M = d->last_n * d->cfg.beam_k;
+  const int S = steps_per_chunk(d, d->last_T);
+  if (algo_bytes) TSD_CUDA(cudaMemsetAsync(d->view.ctr, 0, sizeof(unsigned long long), s));
+  for (int i = 0; i < reps; ++i) {
+    if (kernel == 0) launch_row(d->view, M, S - 1, 2, d->row_smem, s, false);
+    else if (d->joint_kind == 0) launch_joint_tc(*d->jtc, d->view, M, 1 << 30, s, false);
+    else launch_joint(d->view, M, 1 << 30, s);
+  }
+  TSD_CUDA(cudaGetLastError());
+  if (algo_bytes) {
+    unsigned long long b = 0;
+    TSD_CUDA(cudaMemcpyAsync(&b, d->view.ctr, sizeof(b), cudaMemcpyDeviceToHost, s));
+    TSD_CUDA(cudaStreamSynchronize(s));
+    if (kernel == 0) {
+      // per launch, plus the dense unigram and root rows every launch reads once
+      const int64_t shared = (int64_t)d->cfg.V * ((d->lm ? 4 : 0) + (d->boost ? 4 : 0));
+      *algo_bytes = (int64_t)(b / (unsigned long long)reps) + shared;
+    } else {
+      // joint: the operands once (A rows, W_out) and the bias rows read by the epilogue
+      *algo_bytes = (int64_t)M * d->cfg.H * 2 + (int64_t)d->N * d->cfg.H * 2 + (int64_t)M * d->N * 4 +
+                    (int64_t)M * d->n_ptiles * 16;
+    }
+  }
+  return TSD_OK;
 }
 
 extern "C" tsd_status tsd_decoder_check(tsd_decoder* d) {

@@ -49,13 +49,14 @@ struct DecView {
   int32_t* cap_rows;
   int32_t cap_steps;
   int32_t* err;  // device status word: nonzero after a bounded wait expired
+  unsigned long long* ctr;  // algorithmic bytes counted by replayed row passes
 };
 
 constexpr int kRowThreads = 256;
 
 void launch_repack(const uint16_t* W, uint16_t* Wt, int H, int N, int N_pad, cudaStream_t s);
 void launch_open(const DecView& d, int slot, cudaStream_t s);
-void launch_row(const DecView& d, int M, int step, int final_step, size_t smem, cudaStream_t s);
+void launch_row(const DecView& d, int M, int step, int mode, size_t smem, cudaStream_t s, bool pdl);
 void launch_joint(const DecView& d, int M, int step, cudaStream_t s);
 size_t row_smem_bytes(int V4);
 cudaError_t prepare_kernels(size_t row_smem);
@@ -94,6 +95,9 @@ struct tsd_decoder {
   std::map<std::tuple<int, int, int, int>, Entry> entries;  // (n, T, graphs, timing)
   tsd::JointTc* jtc = nullptr;  // tensor-core joint kernel state
   int joint_kind = 0;           // 0 tensor cores, 1 CUDA cores
+  int pdl = 1;                  // programmatic dependent launch between kernels
+  int sms = 0;
+  int last_n = 0, last_T = 0;   // shape of the last decode_chunk (for replay)
   double ms[2] = {0, 0};
   int64_t launches[2] = {0, 0};
 };

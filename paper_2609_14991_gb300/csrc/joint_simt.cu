@@ -31,6 +31,9 @@ __global__ void __launch_bounds__(256) k_joint_simt(DecView d, int step) {
   const int M = d.params->n * d.K;
   if (m0 >= M) return;
   const int H = d.H;
+  // launched without programmatic overlap; the wait is then a no-op
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   __shared__ __align__(16) float sm[kJM * (kJN + 4)];
   float* As = sm;                      // [kJK][kJM + 4]
   float* Bs = sm + kJK * (kJM + 4);    // [kJK][kJN + 4]

@@ -174,6 +174,11 @@ __global__ void __launch_bounds__(kThreads, 1)
   fence_after();
   const uint32_t tmem = *tmem_slot;
   bool ok = true;
+  // Programmatic dependent launch: the set-up above overlaps the row pass;
+  // its outputs (joint input, bias) are read only after the wait.  The next
+  // row pass may launch once every CTA is past this point.
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
   if (warp == 0) {
     if (lane == 0) {
@@ -233,7 +238,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint32_t tbase = tmem + ((uint32_t)(q * 32) << 16);
       float4 bnext[8];
 #pragma unroll
-      for (int i = 0; i < 8; ++i) bnext[i] = live ? __ldg(reinterpret_cast<const float4*>(brow) + i) : make_float4(0, 0, 0, 0);
+      for (int i = 0; i < 8; ++i) bnext[i] = live ? __ldcg(reinterpret_cast<const float4*>(brow) + i) : make_float4(0, 0, 0, 0);
 #pragma unroll 1
       for (int c = 0; c < BN / 32; ++c) {
         float b[32];
@@ -244,7 +249,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (c + 1 < BN / 32) {
 #pragma unroll
           for (int i = 0; i < 8; ++i)
-            bnext[i] = live ? __ldg(reinterpret_cast<const float4*>(brow + (c + 1) * 32) + i) : make_float4(0, 0, 0, 0);
+            bnext[i] = live ? __ldcg(reinterpret_cast<const float4*>(brow + (c + 1) * 32) + i) : make_float4(0, 0, 0, 0);
         }
         float l[32];
         tmem_ld32(tbase + (uint32_t)(c * 32), l);
@@ -334,14 +339,26 @@ cudaError_t joint_tc_prepare(JointTc* jt, const uint16_t* A, int M_pad, const ui
   return e;
 }
 
-void launch_joint_tc(const JointTc& jt, const DecView& d, int M, int step, cudaStream_t s) {
-  dim3 grid(d.N_pad / jt.bn, (M + kBM - 1) / kBM);
-  if (jt.bn == 256)
-    k_joint_tc<256><<<grid, kThreads, Smem<256>::kBytes, s>>>(d, step, jt.mapA, jt.mapB);
-  else if (jt.bn == 128)
-    k_joint_tc<128><<<grid, kThreads, Smem<128>::kBytes, s>>>(d, step, jt.mapA, jt.mapB);
-  else
-    k_joint_tc<64><<<grid, kThreads, Smem<64>::kBytes, s>>>(d, step, jt.mapA, jt.mapB);
+void launch_joint_tc(const JointTc& jt, const DecView& d, int M, int step, cudaStream_t s, bool pdl) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(d.N_pad / jt.bn, (M + kBM - 1) / kBM);
+  cfg.blockDim = dim3(kThreads);
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl ? 1 : 0;
+  if (jt.bn == 256) {
+    cfg.dynamicSmemBytes = Smem<256>::kBytes;
+    cudaLaunchKernelEx(&cfg, k_joint_tc<256>, d, step, jt.mapA, jt.mapB);
+  } else if (jt.bn == 128) {
+    cfg.dynamicSmemBytes = Smem<128>::kBytes;
+    cudaLaunchKernelEx(&cfg, k_joint_tc<128>, d, step, jt.mapA, jt.mapB);
+  } else {
+    cfg.dynamicSmemBytes = Smem<64>::kBytes;
+    cudaLaunchKernelEx(&cfg, k_joint_tc<64>, d, step, jt.mapA, jt.mapB);
+  }
 }
 
 }  // namespace tsd

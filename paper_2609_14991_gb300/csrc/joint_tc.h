@@ -17,6 +17,6 @@ struct JointTc {
 // Tile width for a row count: the widest whose tile count still fills the SMs.
 int joint_tc_pick_bn(int M_max, int N_pad, int sms);
 cudaError_t joint_tc_prepare(JointTc* jt, const uint16_t* A, int M_pad, const uint16_t* Wt, int N_pad, int H, int bn);
-void launch_joint_tc(const JointTc& jt, const DecView& d, int M, int step, cudaStream_t s);
+void launch_joint_tc(const JointTc& jt, const DecView& d, int M, int step, cudaStream_t s, bool pdl);
 
 }  // namespace tsd

@@ -54,38 +54,60 @@ __device__ __forceinline__ void best_merge(float& v, int& i, float v2, int i2) {
   if (v2 > v || (v2 == v && i2 < i)) { v = v2; i = i2; }
 }
 
-__global__ void __launch_bounds__(kRowThreads) k_row(DecView d, int step, int final_step) {
+// mode: 0 = label step, 1 = final step (apply the last decision only),
+// 2 = replay (redo the step's work without committing any state or output;
+// used only to time the kernel in isolation).
+__global__ void __launch_bounds__(kRowThreads) k_row(DecView d, int step, int mode) {
   const Params* __restrict__ P = d.params;
   const int r = blockIdx.x;
-  const int slot = P->slots[r];
-  const int T = P->T;
   const int V = d.V;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const bool commit = (mode != 2);
   extern __shared__ __align__(16) unsigned char smem[];
-  float* lmrow = reinterpret_cast<float*>(smem);
-  int8_t* dep = reinterpret_cast<int8_t*>(lmrow + d.V4);
+  // per-label scratch: LM (level << 32 | value bits), trie depth of the goto
+  unsigned long long* lmkey = reinterpret_cast<unsigned long long*>(smem);
+  int* dep = reinterpret_cast<int*>(lmkey + d.V4);
 
-  __shared__ int s_t, s_sym, s_cnt, s_y, s_lm_len, s_tr_len, s_last;
+  __shared__ int s_t, s_sym, s_cnt, s_y, s_lm_len, s_tr_len, s_last, s_slot, s_T;
   __shared__ float s_score;
   __shared__ int s_lm[kLmChain], s_tr[kTrChain];
-  __shared__ int s_lm_hit[kLmChain];
-  __shared__ int s_tr_hit[kTrChain];
+  __shared__ int s_lm_tgt[kLmChain];            // target state of y's arc at each LM level (-2 none)
+  __shared__ int s_tr_node[kTrChain], s_tr_nxt[kTrChain];  // child by y of each trie chain node (-1 none)
+  __shared__ int s_uni_tgt, s_root_child, s_root_next;
+  __shared__ int s_lb[kLmChain], s_lc[kLmChain];
+  __shared__ float s_lo[kLmChain];
+  __shared__ int s_tb[kTrChain], s_tc[kTrChain], s_td[kTrChain];
 
+  // The row state below was written by the previous row pass; under
+  // programmatic launch this grid may start before its own wait, so these
+  // loads go through L2 only (ld.global.cg), never a possibly stale L1 line.
   if (tid == 0) {
+    const int slot = __ldcg(P->slots + r);
+    s_slot = slot;
+    s_T = __ldcg(&P->T);
     if (step == 0) {
       s_t = 0; s_sym = 0; s_cnt = 0;
     } else {
-      s_t = d.r_t[r]; s_sym = d.r_sym[r]; s_cnt = d.r_cnt[r];
+      s_t = __ldcg(d.r_t + r); s_sym = __ldcg(d.r_sym + r); s_cnt = __ldcg(d.r_cnt + r);
     }
-    s_lm_len = d.has_lm ? d.s_lm_len[slot] : 0;
-    s_tr_len = d.has_tr ? d.s_tr_len[slot] : 0;
-    s_last = d.s_last[slot];
+    s_lm_len = d.has_lm ? __ldcg(d.s_lm_len + slot) : 0;
+    s_tr_len = d.has_tr ? __ldcg(d.s_tr_len + slot) : 0;
+    s_last = __ldcg(d.s_last + slot);
   }
   __syncthreads();
-  if (tid < s_lm_len) s_lm[tid] = d.s_lm_chain[slot * kLmChain + tid];
-  if (tid < s_tr_len) s_tr[tid] = d.s_tr_chain[slot * kTrChain + tid];
+  const int slot = s_slot, T = s_T;
+  if (tid < s_lm_len) s_lm[tid] = __ldcg(d.s_lm_chain + slot * kLmChain + tid);
+  if (tid >= 64 && tid - 64 < s_tr_len) s_tr[tid - 64] = __ldcg(d.s_tr_chain + slot * kTrChain + tid - 64);
   __syncthreads();
-  const bool evaluated = (step > 0) && (s_t < T);
+  // In replay mode every row redoes a full step (decision, advance, joint
+  // input, bias) even if it had finished the chunk, so the timing is that of
+  // a mid-chunk step.
+  const bool evaluated = (step > 0) && (s_t < T || !commit);
+  // Programmatic dependent launch: everything above reads only state the
+  // previous row pass wrote, which had completed before the joint kernel in
+  // between let this grid launch; the joint's partials need the wait.
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
   if (evaluated) {
     // 1. combine the partials of the previous joint step
@@ -94,7 +116,7 @@ __global__ void __launch_bounds__(kRowThreads) k_row(DecView d, int step, int fi
       int bi = INT_MAX;
       const float4* pr = d.part + (size_t)r * d.n_ptiles;
       for (int j = lane; j < d.n_ptiles; j += 32) {
-        float4 p = pr[j];
+        float4 p = __ldcg(pr + j);  // written by the joint kernel just before
         lse_merge(m, s, p.x, p.y);
         best_merge(bv, bi, p.z, __float_as_int(p.w));
       }
@@ -114,67 +136,75 @@ __global__ void __launch_bounds__(kRowThreads) k_row(DecView d, int step, int fi
     __syncthreads();
     const int y = s_y;
     if (y != V) {
-      // 2a. independent searches of y in every chain element
+      // 2a. independent searches of y in every chain element, each warp
+      //     also fetching what the new chain needs from the arc it found
       const int nl = s_lm_len, nt = s_tr_len;
+      if (tid == kRowThreads - 1) {
+        s_uni_tgt = (d.has_lm && d.lm.order >= 2) ? __ldg(d.lm.uni_tgt + y) : -1;
+        s_root_child = d.has_tr ? __ldg(d.tr.root_child + y) : 0;
+        s_root_next = d.has_tr ? __ldg(d.tr.root_next + y) : 0;
+      }
       for (int task = warp; task < nl + nt; task += kRowThreads / 32) {
         if (task < nl) {
           int st = s_lm[task];
           int b = __ldg(d.lm.st_begin + st), c = __ldg(d.lm.st_count + st);
           int i = warp_find(d.lm.arc_tok + b, c, y, lane);
-          if (lane == 0) s_lm_hit[task] = (i >= 0) ? b + i : -1;
+          if (lane == 0) s_lm_tgt[task] = (i >= 0) ? __ldg(d.lm.arc_tgt + b + i) : -2;
         } else {
-          int q = s_tr[task - nl];
+          int k = task - nl;
+          int q = s_tr[k];
           int b = __ldg(d.tr.nd_begin + q), c = __ldg(d.tr.nd_count + q);
           int i = warp_find(d.tr.ch_tok + b, c, y, lane);
-          if (lane == 0) s_tr_hit[task - nl] = (i >= 0) ? b + i : -1;
+          if (lane == 0) {
+            s_tr_node[k] = (i >= 0) ? __ldg(d.tr.ch_node + b + i) : -1;
+            s_tr_nxt[k] = (i >= 0) ? __ldg(d.tr.ch_next + b + i) : -1;
+          }
         }
       }
       __syncthreads();
-      // 2b. assemble the new chains and emit
+      // 2b. assemble the new chains (shared memory only) and emit
       if (tid == 0) {
         int newlm[kLmChain];
         int ln = 0;
-        if (d.has_lm && d.lm.order >= 2) {
-          newlm[ln++] = __ldg(d.lm.uni_tgt + y);
+        if (s_uni_tgt >= 0) {
+          newlm[ln++] = s_uni_tgt;
           for (int l = 0; l < nl && ln < kLmChain; ++l) {
-            int a = s_lm_hit[l];
-            if (a < 0) break;
-            int tgt = __ldg(d.lm.arc_tgt + a);
-            if (tgt < 0) break;
+            int tgt = s_lm_tgt[l];
+            if (tgt < 0) break;  // no arc at this level (-2) or the top order (-1)
             newlm[ln++] = tgt;
           }
         }
         int newtr[kTrChain];
         int tn = 0;
         bool reset = false;
-        if (d.has_tr) {
-          for (int i = 0; i < nt; ++i) {
-            int a = s_tr_hit[i];
-            if (a < 0) continue;
-            if (tn == 0 && __ldg(d.tr.ch_next + a) == 0) reset = true;
-            if (tn < kTrChain) newtr[tn++] = __ldg(d.tr.ch_node + a);
-          }
-          int rc = __ldg(d.tr.root_child + y);
-          if (rc != 0) {
-            if (tn == 0 && __ldg(d.tr.root_next + y) == 0) reset = true;
-            if (tn < kTrChain) newtr[tn++] = rc;
-          }
-          if (reset) tn = 0;
+        for (int i = 0; i < nt; ++i) {
+          if (s_tr_node[i] < 0) continue;
+          if (tn == 0 && s_tr_nxt[i] == 0) reset = true;
+          if (tn < kTrChain) newtr[tn++] = s_tr_node[i];
         }
-        for (int l = 0; l < ln; ++l) { s_lm[l] = newlm[l]; d.s_lm_chain[slot * kLmChain + l] = newlm[l]; }
-        for (int l = 0; l < tn; ++l) { s_tr[l] = newtr[l]; d.s_tr_chain[slot * kTrChain + l] = newtr[l]; }
+        if (s_root_child != 0) {
+          if (tn == 0 && s_root_next == 0) reset = true;
+          if (tn < kTrChain) newtr[tn++] = s_root_child;
+        }
+        if (reset) tn = 0;
+        for (int l = 0; l < ln; ++l) s_lm[l] = newlm[l];
+        for (int l = 0; l < tn; ++l) s_tr[l] = newtr[l];
         s_lm_len = ln;
         s_tr_len = tn;
-        if (d.has_lm) d.s_lm_len[slot] = ln;
-        if (d.has_tr) d.s_tr_len[slot] = tn;
-        const int cap = T * d.max_sym;
-        const int o = r * cap + s_cnt;
-        P->out_tok[o] = y;
-        P->out_frame[o] = s_t;
-        P->out_score[o] = s_score;
+        if (commit) {
+          for (int l = 0; l < ln; ++l) d.s_lm_chain[slot * kLmChain + l] = newlm[l];
+          for (int l = 0; l < tn; ++l) d.s_tr_chain[slot * kTrChain + l] = newtr[l];
+          if (d.has_lm) d.s_lm_len[slot] = ln;
+          if (d.has_tr) d.s_tr_len[slot] = tn;
+          const int cap = T * d.max_sym;
+          const int o = r * cap + s_cnt;
+          P->out_tok[o] = y;
+          P->out_frame[o] = s_t;
+          P->out_score[o] = s_score;
+          d.s_last[slot] = y;
+        }
         s_cnt += 1;
         s_last = y;
-        d.s_last[slot] = y;
         s_sym += 1;
         if (s_sym >= d.max_sym) { s_t += 1; s_sym = 0; }
       }
@@ -185,17 +215,17 @@ __global__ void __launch_bounds__(kRowThreads) k_row(DecView d, int step, int fi
     __syncthreads();
   }
 
-  if (final_step) {
+  if (mode == 1) {
     if (tid == 0) P->out_count[r] = s_cnt;
     return;
   }
-  if (tid == 0) {
+  if (tid == 0 && commit) {
     d.r_t[r] = s_t;
     d.r_sym[r] = s_sym;
     d.r_cnt[r] = s_cnt;
   }
-  const int t = s_t;
-  if (d.cap_rows && step < d.cap_steps && tid == 0) {
+  const int t = commit ? s_t : min(s_t, T - 1);
+  if (d.cap_rows && step < d.cap_steps && tid == 0 && commit) {
     int* c = d.cap_rows + ((size_t)step * P->n + r) * 4;
     if (t < T) {
       c[0] = t;
@@ -208,7 +238,25 @@ __global__ void __launch_bounds__(kRowThreads) k_row(DecView d, int step, int fi
   }
   if (t >= T) return;
 
-  // 3. joint input of this step
+  // 3. state records of the new chains (one thread each), scratch reset
+  const int nl = s_lm_len, nt = s_tr_len;
+  if (tid < nl) {
+    const int st = s_lm[tid];
+    s_lb[tid] = __ldg(d.lm.st_begin + st);
+    s_lc[tid] = __ldg(d.lm.st_count + st);
+    s_lo[tid] = __ldg(d.lm.st_cum + st);
+  } else if (tid >= 32 && tid - 32 < nt) {
+    const int q = s_tr[tid - 32];
+    s_tb[tid - 32] = __ldg(d.tr.nd_begin + q);
+    s_tc[tid - 32] = __ldg(d.tr.nd_count + q);
+    s_td[tid - 32] = __ldg(d.tr.nd_depth + q) + 1;
+  }
+  for (int v = tid; v < V; v += kRowThreads) {
+    lmkey[v] = 0ull;
+    dep[v] = 0;
+  }
+
+  // 4. joint input of this step (its loads overlap the records above)
   {
     const int H = d.H;
     const uint4* e = reinterpret_cast<const uint4*>(P->enc + ((size_t)r * T + t) * H);
@@ -230,57 +278,64 @@ __global__ void __launch_bounds__(kRowThreads) k_row(DecView d, int step, int fi
       a[i] = out;
     }
   }
+  __syncthreads();
 
-  // 4. fusion bias of this step
-  const int nl = s_lm_len, nt = s_tr_len;
-  const float lam = P->lambda, beta = P->beta;
-  const float cum_top = (d.has_lm && nl) ? __ldg(d.lm.st_cum + s_lm[nl - 1]) : 0.f;
-  const int depth_cur = (d.has_tr && nt) ? __ldg(d.tr.nd_depth + s_tr[0]) : 0;
-  const float unset = __int_as_float(0x7fc00000);
-  for (int v = tid; v < V; v += kRowThreads) {
-    lmrow[v] = unset;
-    dep[v] = -1;
+  // 5. fusion bias of this step: every chain level at once; a label's LM
+  //    score comes from the deepest level that continues with it (max of
+  //    level << 32 | value bits), its goto depth from the deepest trie node
+  //    that has it as a child (max of the child's depth)
+  const float cum_top = nl ? s_lo[nl - 1] : 0.f;
+  for (int l = 0; l < nl; ++l) {
+    const int b = s_lb[l], c = s_lc[l];
+    const float off = cum_top - s_lo[l];
+    const unsigned long long lev = (unsigned long long)(l + 1) << 32;
+    for (int j = tid; j < c; j += kRowThreads) {
+      const int w = __ldg(d.lm.arc_tok + b + j);
+      const float val = off + __ldg(d.lm.arc_logp + b + j);
+      atomicMax(lmkey + w, lev | (unsigned long long)__float_as_uint(val));
+    }
+  }
+  for (int k = 0; k < nt; ++k) {
+    const int b = s_tb[k], c = s_tc[k], dd = s_td[k];
+    for (int j = tid; j < c; j += kRowThreads) atomicMax(dep + __ldg(d.tr.ch_tok + b + j), dd);
   }
   __syncthreads();
-  const int phases = max(nl, nt);
-  for (int p = 0; p < phases; ++p) {
-    if (p < nl) {  // LM level nl-p (deepest first): its arcs win over shallower ones
-      int st = s_lm[nl - 1 - p];
-      int b = __ldg(d.lm.st_begin + st), c = __ldg(d.lm.st_count + st);
-      float off = cum_top - __ldg(d.lm.st_cum + st);
-      for (int j = tid; j < c; j += kRowThreads) {
-        int w = __ldg(d.lm.arc_tok + b + j);
-        if (isnan(lmrow[w])) lmrow[w] = off + __ldg(d.lm.arc_logp + b + j);
-      }
-    }
-    if (p < nt) {  // trie chain node p (deepest first)
-      int q = s_tr[p];
-      int b = __ldg(d.tr.nd_begin + q), c = __ldg(d.tr.nd_count + q);
-      int dd = __ldg(d.tr.nd_depth + q) + 1;
-      for (int j = tid; j < c; j += kRowThreads) {
-        int w = __ldg(d.tr.ch_tok + b + j);
-        if (dep[w] < 0) dep[w] = (int8_t)dd;
-      }
-    }
-    __syncthreads();
-  }
+  const int depth_cur = nt ? s_td[0] - 1 : 0;
+  const float lam = P->lambda, beta = P->beta;
   float* brow = d.bias + (size_t)r * d.N_pad;
   const float bscale = beta * (d.has_tr ? d.tr.bonus : 0.f);
   for (int v = tid; v < V; v += kRowThreads) {
     float b = 0.f;
     if (d.has_lm) {
-      float l = lmrow[v];
-      if (isnan(l)) l = cum_top + __ldg(d.lm.uni_logp + v);
+      const unsigned long long k = lmkey[v];
+      const float l = k ? __uint_as_float((unsigned)k) : cum_top + __ldg(d.lm.uni_logp + v);
       b = lam * l;
     }
     if (d.has_tr) {
       int dd = dep[v];
-      if (dd < 0) dd = (__ldg(d.tr.root_child + v) != 0) ? 1 : 0;
+      if (dd == 0) dd = (__ldg(d.tr.root_child + v) != 0) ? 1 : 0;
       b += bscale * (float)(dd - depth_cur);
     }
     brow[v] = b;
   }
   if (tid == 0) brow[V] = 0.f;
+  if (mode == 2 && tid == 0) {
+    // Algorithmic bytes of this row-step: selection partials, row state,
+    // the searches of the emitted label (one probe per halving plus the arc
+    // it found), the joint input (encoder frame and embedding row read, A
+    // row written), and every arc of every chain level and trie chain node
+    // with its state record.  The dense bias row written for the GEMM
+    // epilogue and the shared unigram/root rows are not counted here.
+    unsigned long long bytes = (unsigned long long)d.n_ptiles * 16 + 2ull * (24 + 4 * (nl + nt));
+    bytes += 6ull * d.H;
+    for (int l = 0; l < nl; ++l) bytes += 12 + 8ull * s_lc[l];
+    for (int k = 0; k < nt; ++k) bytes += 12 + 4ull * s_tc[k];
+    if (s_y != V && evaluated) {
+      for (int l = 0; l < nl; ++l) bytes += 8 + 4ull * (32 - __clz(s_lc[l] + 1)) + 4;
+      for (int k = 0; k < nt; ++k) bytes += 8 + 4ull * (32 - __clz(s_tc[k] + 1)) + 8;
+    }
+    atomicAdd(d.ctr, bytes);
+  }
 }
 
 __global__ void k_open(DecView d, int slot) {
@@ -308,7 +363,7 @@ __global__ void k_repack(const uint16_t* __restrict__ W, uint16_t* __restrict__ 
 
 }  // namespace
 
-size_t row_smem_bytes(int V4) { return (size_t)V4 * (sizeof(float) + 1); }
+size_t row_smem_bytes(int V4) { return (size_t)V4 * (sizeof(unsigned long long) + sizeof(int)); }
 
 cudaError_t prepare_kernels(size_t row_smem) {
   if (row_smem > 48 * 1024)
@@ -323,8 +378,18 @@ void launch_repack(const uint16_t* W, uint16_t* Wt, int H, int N, int N_pad, cud
 
 void launch_open(const DecView& d, int slot, cudaStream_t s) { k_open<<<1, 32, 0, s>>>(d, slot); }
 
-void launch_row(const DecView& d, int M, int step, int final_step, size_t smem, cudaStream_t s) {
-  k_row<<<M, kRowThreads, smem, s>>>(d, step, final_step);
+void launch_row(const DecView& d, int M, int step, int mode, size_t smem, cudaStream_t s, bool pdl) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(M);
+  cfg.blockDim = dim3(kRowThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl ? 1 : 0;
+  cudaLaunchKernelEx(&cfg, k_row, d, step, mode);
 }
 
 }  // namespace tsd

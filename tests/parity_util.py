@@ -49,7 +49,8 @@ class GpuRun:
     """Decodes `streams` (stream ids of the workload) for `chunks` chunks."""
 
     def __init__(self, inp: Inputs, streams: Sequence[int], chunks: int, T: Optional[int] = None,
-                 capture_steps: int = 0, graphs: bool = True, joint_kind: int = 0):
+                 capture_steps: int = 0, graphs: bool = True, joint_kind: int = 0, options=None,
+                 between_chunks=None):
         import torch
 
         import paper_2609_14991_gb300 as tsd
@@ -68,6 +69,8 @@ class GpuRun:
         self.dec.set_graphs(graphs)
         if joint_kind:
             self.dec.set_joint_kernel(joint_kind)
+        for k, v in (options or {}).items():
+            self.dec.set_option(k, v)
         self.slots = [self.dec.open() for _ in range(n)]
         self.cap_logits = self.cap_rows = None
         if capture_steps:
@@ -87,6 +90,8 @@ class GpuRun:
             self.chunks.append({"count": cnt, "tok": tok, "frame": fr, "score": sc})
             self.enc.append(enc)
             self.states.append([self.dec.state(s) for s in self.slots])
+            if between_chunks is not None:
+                between_chunks(self.dec)
         self.dec.check()  # no bounded device wait expired
 
     def emitted(self, i: int, c: int):

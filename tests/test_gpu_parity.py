@@ -192,6 +192,29 @@ def test_tensor_core_and_cuda_core_kernels_agree():
     pu.assert_reports(pu.replay(inp, a, [0, 64, 129]))
 
 
+def test_launch_options_and_replay_do_not_change_results():
+    """Programmatic dependent launch on/off and timing replays between chunks
+    give bit-identical decodes; every tensor-core tile width passes parity
+    (a different tile split only reorders the fp32 log-sum-exp)."""
+    w = synth.scaled(synth.WORKLOADS[1], B=150, chunks=3)
+    inp = pu.Inputs(w, lmA=synth.ngram_lm(13, w.V, 4, 300_000, 1.1), ph=synth.phrases(13, w.V, 300, 2, 6, 0.2))
+    base = pu.GpuRun(inp, range(w.B), 3)
+    exact = {"pdl off": pu.GpuRun(inp, range(w.B), 3, options={"pdl": 0}),
+             "replays": pu.GpuRun(inp, range(w.B), 3, between_chunks=lambda d: (d.replay(0, 3), d.replay(1, 3)))}
+    for name, r in exact.items():
+        for c in range(3):
+            for i in range(w.B):
+                for x, y in zip(r.emitted(i, c), base.emitted(i, c)):
+                    assert np.array_equal(x, y), (name, c, i)
+    for bn in (64, 128, 256):
+        r = pu.GpuRun(inp, range(w.B), 3, options={"joint_bn": bn})
+        pu.assert_reports(pu.replay(inp, r, [0, 77, 149]))
+        for c in range(3):
+            for i in range(0, w.B, 7):
+                np.testing.assert_allclose(r.emitted(i, c)[2][:5], base.emitted(i, c)[2][:5], atol=1e-5)
+    assert base.dec.replay(0, 1, count_bytes=True) > 0
+
+
 def test_status_errors_leave_decoder_usable():
     import paper_2609_14991_gb300 as tsd
 
