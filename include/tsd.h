@@ -258,6 +258,34 @@ TSD_API tsd_status tsd_decoder_set_option(tsd_decoder* dec, const char* name, in
 TSD_API tsd_status tsd_decoder_replay(tsd_decoder* dec, int32_t kernel, int32_t reps, void* cuda_stream,
                                       int64_t* algo_bytes);
 
+/* ------------------------------------------------------------------------
+ * Allocation-free joint selection (the paper has no counterpart; this is a
+ * service for callers that cannot allocate device memory: code that runs
+ * inside a memory pool or arena that owns all of the device's memory,
+ * plugins handed pre-allocated buffers by their host framework, and
+ * real-time paths that cannot afford cudaMalloc's implicit synchronization).
+ *
+ * For each of n rows: logits = A[r] . Wt^T (bf16 in, fp32 accumulate), the
+ * log-softmax over the V+1 labels, and the label maximizing the fused value
+ * logit + bias (bias 0 for blank = label V; ties to the lowest label):
+ *   A_bf16   device bf16 [n][H], the joint input rows (16-byte aligned);
+ *   Wt_bf16  device bf16 [V+1][H], W_out label-major (16-byte aligned);
+ *   bias     device fp32 [n][V] (lambda*LM + beta*boost), or NULL for 0;
+ *   out_label device int32 [n]; out_score device fp32 [n] = the fused value
+ *   of out_label minus the row's log-sum-exp.
+ * Limits: 1 <= n <= 1024, V + 1 <= 8192, H a multiple of 64 in [64, 8192];
+ * larger sizes return TSD_EINVAL.  The call allocates nothing: its working
+ * memory is a 1 MiB array compiled into the library, which every GPU that
+ * loads the library keeps until the process exits.  The first call on a
+ * device looks up that array's device address (cudaGetSymbolAddress); make
+ * that first call before any stream capture.  All calls share the array:
+ * calls that overlap on the GPU (different streams, or host threads on one
+ * device without ordering) race and must be serialized by the caller.
+ * Asynchronous on cuda_stream. */
+TSD_API tsd_status tsd_joint_select_noalloc(int32_t n, int32_t H, int32_t V, const void* A_bf16,
+                                            const void* Wt_bf16, const float* bias, int32_t* out_label,
+                                            float* out_score, void* cuda_stream);
+
 /* Kernel launches one decode_chunk(n, T) issues (for launch accounting). */
 TSD_API tsd_status tsd_decoder_launches_per_chunk(const tsd_decoder* dec, int32_t n, int32_t T,
                                           int64_t* launches);

@@ -67,6 +67,7 @@ SIGNATURES = {
     "tsd_decoder_check": ([_vp], _i32),
     "tsd_decoder_set_option": ([_vp, ctypes.c_char_p, _i64], _i32),
     "tsd_decoder_replay": ([_vp, _i32, _i32, _vp, _P(_i64)], _i32),
+    "tsd_joint_select_noalloc": ([_i32, _i32, _i32, _vp, _vp, _vp, _vp, _vp, _vp], _i32),
 }
 
 _lib = None
@@ -190,6 +191,17 @@ class Boost:
         if getattr(self, "h", None):
             lib().tsd_boost_free(self.h)
             self.h = None
+
+
+def joint_select_noalloc(A, Wt, bias, out_label, out_score, stream=None):
+    """Allocation-free joint selection (tsd_joint_select_noalloc): for callers
+    that cannot allocate device memory.  A: cuda bf16 [n, H]; Wt: cuda bf16
+    [V+1, H]; bias: cuda fp32 [n, V] or None; out_label: cuda int32 [n];
+    out_score: cuda fp32 [n].  Nothing is allocated by this call."""
+    n, H = A.shape
+    V = Wt.shape[0] - 1
+    _check(lib().tsd_joint_select_noalloc(n, H, V, _ptr(A), _ptr(Wt), _ptr(bias) if bias is not None else None,
+                                          _ptr(out_label), _ptr(out_score), _stream(stream)))
 
 
 class ChunkOut:
