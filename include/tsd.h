@@ -187,7 +187,8 @@ TSD_API tsd_status tsd_decode_chunk(tsd_decoder* dec, int32_t n, const int32_t* 
                             int32_t* out_tokens, int32_t* out_frames, float* out_scores,
                             int32_t* out_counts, void* cuda_stream);
 
-/* Reads a greedy stream's state (synchronizes the decoder's stream): the LM
+/* Reads a stream's state (synchronizes the decoder's stream; for a beam
+ * decoder, that of the stream's first live hypothesis): the LM
  * state id (see tsd_ngram_state_tuple; 0 = empty context), the trie node
  * (tsd_boost_node_tuple; 0 = root) and the previous label (V = blank/SOS).
  * Any output pointer may be NULL. */

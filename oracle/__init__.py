@@ -67,7 +67,9 @@ def lib() -> ctypes.CDLL:
             "oracle_decode_chunk": ([vp, vp, vp, i32, i32, vp, vp, vp, i32, dbl, dbl, i32, vp, vp, vp, i32, dbl,
                                      vp, vp, vp, i32, vp], i32),
             "oracle_beam_chunk": ([vp, vp, vp, i32, i32, vp, vp, vp, i32, dbl, dbl, i32], i32),
-            "oracle_beam_hyp": ([vp, i32, vp, i64, vp], i64),
+            "oracle_beam_hyp": ([vp, i32, vp, i64, vp, vp], i64),
+            "oracle_beam_chunk_follow": ([vp, vp, vp, i32, i32, vp, vp, vp, i32, dbl, dbl, i32, vp, vp, vp, dbl,
+                                          vp], i32),
             "oracle_joint_logits": ([i32, i32, vp, vp, vp, i32, vp], None),
             "oracle_fused_row": ([vp, vp, vp, i32, i32, vp, vp, vp, dbl, dbl, vp], None),
             "oracle_boost_trajectory": ([vp, vp, i64, vp, vp], None),
@@ -197,17 +199,20 @@ class Stream:
         y = _i32(y)
         lib().oracle_stream_set_history(self.h, _p(y), len(y), int(rho))
 
-    def beam_hyps(self) -> List[Tuple[List[int], float]]:
+    def beam_hyps(self, with_rho: bool = False):
+        """[(labels, score)] or, with_rho, [(labels, score, restart index)]."""
         out = []
         i = 0
         while True:
-            n = lib().oracle_beam_hyp(self.h, i, None, 0, None)
+            n = lib().oracle_beam_hyp(self.h, i, None, 0, None, None)
             if n < 0:
                 return out
             buf = np.zeros(max(1, n), dtype=np.int32)
             sc = ctypes.c_double()
-            lib().oracle_beam_hyp(self.h, i, _p(buf), n, ctypes.byref(sc))
-            out.append(([int(x) for x in buf[:n]], sc.value))
+            rho = ctypes.c_int64()
+            lib().oracle_beam_hyp(self.h, i, _p(buf), n, ctypes.byref(sc), ctypes.byref(rho))
+            labels = [int(x) for x in buf[:n]]
+            out.append((labels, sc.value, int(rho.value)) if with_rho else (labels, sc.value))
             i += 1
 
 
@@ -269,3 +274,18 @@ def beam_chunk(stream: Stream, model: Model, lm: Optional[LM], boost: Optional[B
     return lib().oracle_beam_chunk(stream.h, lm.h if lm else None, boost.h if boost else None, model.V, model.H,
                                    _p(model.E), _p(model.W), _p(enc), enc.shape[0], float(lam), float(beta),
                                    int(K))
+
+
+def beam_chunk_follow(stream: Stream, model: Model, lm: Optional[LM], boost: Optional[Boost], enc: np.ndarray,
+                      lam: float, beta: float, K: int, sel_hyp: np.ndarray, sel_tok: np.ndarray,
+                      sel_inc: np.ndarray, gap_tol: float = 1e-3) -> np.ndarray:
+    """Beam search over one chunk following kept candidates [T, K] under test;
+    returns the report (see oracle_beam_chunk_follow)."""
+    enc = np.ascontiguousarray(enc, dtype=np.uint16)
+    sh, st = _i32(sel_hyp).reshape(-1), _i32(sel_tok).reshape(-1)
+    si = np.ascontiguousarray(sel_inc, dtype=np.float32).reshape(-1)
+    rep = np.zeros(8, dtype=np.float64)
+    lib().oracle_beam_chunk_follow(stream.h, lm.h if lm else None, boost.h if boost else None, model.V, model.H,
+                                   _p(model.E), _p(model.W), _p(enc), enc.shape[0], float(lam), float(beta), int(K),
+                                   _p(sh), _p(st), _p(si), float(gap_tol), _p(rep))
+    return rep

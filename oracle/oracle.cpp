@@ -495,16 +495,104 @@ ORACLE_API int32_t oracle_beam_chunk(void* sp, const void* lmp, const void* boos
   return (int32_t)s->beam.size();
 }
 
-// Beam hypothesis i: copies up to cap labels to buf, writes its score,
-// returns the label count (-1 if i is out of range).
+// Beam hypothesis i: copies up to cap labels to buf, writes its score and
+// restart index, returns the label count (-1 if i is out of range).
 ORACLE_API int64_t oracle_beam_hyp(const void* sp, int32_t i, int32_t* buf, int64_t cap,
-                                   double* score) {
+                                   double* score, int64_t* rho) {
   const Stream* s = static_cast<const Stream*>(sp);
   if (i < 0 || i >= (int32_t)s->beam.size()) return -1;
   const Hyp& h = s->beam[(size_t)i];
   for (int64_t j = 0; j < (int64_t)h.y.size() && j < cap; ++j) buf[j] = h.y[(size_t)j];
   if (score) *score = h.score;
+  if (rho) *rho = h.rho;
   return (int64_t)h.y.size();
+}
+
+// Beam search over one chunk following the selections under test.  For
+// frame t, sel_hyp/sel_tok/sel_inc[t*K + i] (i < K) are the candidates that
+// were kept, in their order (hypothesis -1 = none): the hypothesis index,
+// the label (V = blank) and the score increment that was used.  The oracle
+// scores every candidate itself and checks that
+//   * each kept candidate's increment is its own fused value (largest
+//     difference reported),
+//   * no candidate left out beats a kept one by more than gap_tol, and the
+//     kept ones are in non-increasing order up to gap_tol,
+// then applies the selection in that order, merging equal label sequences
+// by log-sum-exp of its own scores.
+ORACLE_API int32_t oracle_beam_chunk_follow(void* sp, const void* lmp, const void* boostp, int32_t V,
+                                            int32_t H, const uint16_t* E, const uint16_t* W,
+                                            const uint16_t* enc, int32_t T, double lambda, double beta,
+                                            int32_t K, const int32_t* sel_hyp, const int32_t* sel_tok,
+                                            const float* sel_inc, double gap_tol, double* report) {
+  Stream* s = static_cast<Stream*>(sp);
+  const NGramDict* lm = static_cast<const NGramDict*>(lmp);
+  const PhraseSet* boost = static_cast<const PhraseSet*>(boostp);
+  Model m{V, H, E, W};
+  if (s->beam.empty()) s->beam.push_back(Hyp());
+  double rep[REP_N] = {0, 0, 0, 0, std::numeric_limits<double>::infinity(), -1, 0, 0};
+  std::vector<float> x;
+  std::vector<double> logits, fused;
+  for (int32_t t = 0; t < T; ++t) {
+    const size_t nh = s->beam.size();
+    std::vector<std::vector<double>> f(nh);
+    for (size_t i = 0; i < nh; ++i) {
+      fused_scores(m, enc + (size_t)t * H, s->beam[i], lm, boost, lambda, beta, x, logits, fused);
+      f[i] = fused;
+    }
+    std::vector<std::pair<int32_t, int32_t>> kept;
+    std::vector<char> is_kept(nh * (size_t)(V + 1), 0);
+    double min_kept = std::numeric_limits<double>::infinity(), prev = std::numeric_limits<double>::infinity();
+    for (int32_t i = 0; i < K; ++i) {
+      const int32_t h = sel_hyp[(size_t)t * K + i], v = sel_tok[(size_t)t * K + i];
+      if (h < 0) continue;
+      if (h >= (int32_t)nh || v < 0 || v > V) { rep[REP_INCONSISTENT] = 1; continue; }
+      const double sc = s->beam[(size_t)h].score + f[(size_t)h][(size_t)v];
+      rep[REP_MAX_SCORE_DIFF] = std::max(rep[REP_MAX_SCORE_DIFF],
+                                         std::fabs((double)sel_inc[(size_t)t * K + i] - f[(size_t)h][(size_t)v]));
+      if (sc > prev + gap_tol) rep[REP_MISMATCH] += 1;  // out of order
+      prev = sc;
+      min_kept = std::min(min_kept, sc);
+      is_kept[(size_t)h * (V + 1) + (size_t)v] = 1;
+      kept.push_back({h, v});
+    }
+    const size_t want = std::min((size_t)K, nh * (size_t)(V + 1));
+    if (kept.size() != want) rep[REP_INCONSISTENT] = 1;
+    double best_out = -std::numeric_limits<double>::infinity();
+    for (size_t h = 0; h < nh; ++h)
+      for (int32_t v = 0; v <= V; ++v)
+        if (!is_kept[h * (V + 1) + (size_t)v]) best_out = std::max(best_out, s->beam[h].score + f[h][(size_t)v]);
+    if (best_out > min_kept + gap_tol) {
+      rep[REP_MISMATCH] += 1;
+      if (rep[REP_FIRST_BAD] < 0) rep[REP_FIRST_BAD] = t;
+    } else if (best_out > min_kept) {
+      rep[REP_NEAR_TIE] += 1;
+    }
+    rep[REP_MIN_GAP] = std::min(rep[REP_MIN_GAP], min_kept - best_out);
+    std::vector<Hyp> next;
+    for (const auto& kv : kept) {
+      Hyp h = s->beam[(size_t)kv.first];
+      const double sc = h.score + f[(size_t)kv.first][(size_t)kv.second];
+      if (kv.second != V) {
+        h.y.push_back(kv.second);
+        advance_rho(boost, h);
+      }
+      h.score = sc;
+      bool merged = false;
+      for (Hyp& o : next) {
+        if (o.y == h.y) {
+          o.score = logaddexp(o.score, h.score);
+          merged = true;
+          break;
+        }
+      }
+      if (!merged) next.push_back(std::move(h));
+    }
+    s->beam = std::move(next);
+    rep[REP_STEPS] += 1;
+  }
+  if (report)
+    for (int i = 0; i < REP_N; ++i) report[i] = rep[i];
+  return (int32_t)s->beam.size();
 }
 
 // Joint logits of one frame for a given previous label, in double, for the

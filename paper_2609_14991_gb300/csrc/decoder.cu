@@ -42,7 +42,8 @@ void enqueue_chunk(tsd_decoder* d, int M, int T, cudaStream_t s, const std::vect
   for (int step = 0; step <= S; ++step) {
     const bool pdl = d->pdl && !ev && step > 0;  // the first launch follows the parameter copy
     mark();
-    launch_row(d->view, M, step, step == S ? 1 : 0, d->row_smem, s, pdl);
+    if (d->cfg.beam_k > 1) launch_row_beam(d->view, M / d->cfg.beam_k, step, step == S ? 1 : 0, d->row_smem, s, pdl);
+    else launch_row(d->view, M, step, step == S ? 1 : 0, d->row_smem, s, pdl);
     if (step < S) {
       mark();
       if (d->joint_kind == 0) launch_joint_tc(*d->jtc, d->view, M, step, s, d->pdl && !ev);
@@ -86,7 +87,11 @@ extern "C" tsd_status tsd_decoder_create(const tsd_decoder_cfg* cfg, const void*
   const tsd_decoder_cfg c = *cfg;
   if (c.V < 1 || c.V > 16384) return fail(TSD_EINVAL, "tsd_decoder_create: V=%d out of range [1, 16384]", c.V);
   if (c.H < 64 || c.H > 8192 || c.H % 64) return fail(TSD_EINVAL, "tsd_decoder_create: H=%d must be a multiple of 64 in [64, 8192]", c.H);
-  if (c.beam_k != 1) return fail(TSD_EINVAL, "tsd_decoder_create: beam_k=%d not supported by this build (greedy only)", c.beam_k);
+  if (c.beam_k < 1 || c.beam_k > 8) return fail(TSD_EINVAL, "tsd_decoder_create: beam_k=%d outside [1, 8]", c.beam_k);
+  if (c.beam_k > 1 && c.max_symbols != 1)
+    return fail(TSD_EINVAL, "tsd_decoder_create: beam search emits at most one label per frame (max_symbols must be 1)");
+  if (c.beam_k > 1 && ((c.V + 1 + kNPad - 1) / kNPad * kNPad / 64) * c.beam_k > 512)
+    return fail(TSD_EINVAL, "tsd_decoder_create: beam_k * (V+1)/64 must be <= 512");
   if (c.max_symbols < 1 || c.max_symbols > 64) return fail(TSD_EINVAL, "tsd_decoder_create: max_symbols=%d out of range", c.max_symbols);
   if (c.max_streams < 1 || (int64_t)c.max_streams * c.beam_k > 4096)
     return fail(TSD_EINVAL, "tsd_decoder_create: max_streams=%d out of range", c.max_streams);
@@ -117,6 +122,10 @@ extern "C" tsd_status tsd_decoder_create(const tsd_decoder_cfg* cfg, const void*
   float4* part;
   int32_t *rt, *rs, *rc, *sl, *sll, *slc, *stl, *stc, *err;
   unsigned long long* ctr;
+  float2* bpart = nullptr;
+  double* hscore = nullptr;
+  int32_t *hlive = nullptr, *hnode = nullptr, *hlen = nullptr, *ppar = nullptr, *ptok = nullptr, *pn = nullptr;
+  unsigned long long* hhash = nullptr;
   const size_t SK = (size_t)c.max_streams * c.beam_k;
   d->params_bytes = sizeof(Params) + sizeof(int32_t) * (size_t)c.max_streams;
   char* pdev = nullptr;
@@ -129,6 +138,20 @@ extern "C" tsd_status tsd_decoder_create(const tsd_decoder_cfg* cfg, const void*
       (st = A.alloc(&stl, SK)) || (st = A.alloc(&stc, SK * kTrChain)) || (st = A.alloc(&pdev, d->params_bytes))) {
     A.release();
     return st;
+  }
+  if (c.beam_k > 1) {
+    const size_t pool = (size_t)c.max_streams * kPoolCap;
+    if ((st = A.alloc(&bpart, (size_t)d->M_pad * (d->N_pad / 64) * (1 + c.beam_k))) || (st = A.alloc(&hscore, SK)) ||
+        (st = A.alloc(&hlive, SK)) || (st = A.alloc(&hnode, SK)) || (st = A.alloc(&hlen, SK)) ||
+        (st = A.alloc(&hhash, SK)) || (st = A.alloc(&ppar, pool)) || (st = A.alloc(&ptok, pool)) ||
+        (st = A.alloc(&pn, (size_t)c.max_streams))) {
+      A.release();
+      return st;
+    }
+    if (!bpart || !hscore || !hlive || !hnode || !hlen || !hhash || !ppar || !ptok || !pn) {
+      A.release();
+      return fail(TSD_ENOMEM, "tsd_decoder_create: beam state not allocated");
+    }
   }
   auto cleanup = [&](tsd_status e) {
     delete d->jtc;
@@ -153,6 +176,9 @@ extern "C" tsd_status tsd_decoder_create(const tsd_decoder_cfg* cfg, const void*
   launch_repack(static_cast<const uint16_t*>(W_out_bf16), Wt, c.H, d->N, d->N_pad, s);
   if ((ce = cudaGetLastError()) != cudaSuccess) return cleanup(cuda_fail(ce, "tsd_decoder_create: repack"));
   if ((ce = prepare_kernels(d->row_smem)) != cudaSuccess) return cleanup(cuda_fail(ce, "tsd_decoder_create: kernel attributes"));
+  if ((ce = prepare_beam_kernels(d->row_smem)) != cudaSuccess) return cleanup(cuda_fail(ce, "tsd_decoder_create: kernel attributes"));
+  if (hlive && (ce = cudaMemsetAsync(hlive, 0, sizeof(int32_t) * SK, s)) != cudaSuccess)
+    return cleanup(cuda_fail(ce, "tsd_decoder_create: initial copies"));
   {
     int sms = 0;
     if ((ce = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, d->device)) != cudaSuccess)
@@ -206,6 +232,16 @@ extern "C" tsd_status tsd_decoder_create(const tsd_decoder_cfg* cfg, const void*
   v.cap_steps = 0;
   v.err = err;
   v.ctr = ctr;
+  v.bpart = bpart;
+  v.h_score = hscore;
+  v.h_live = hlive;
+  v.h_node = hnode;
+  v.h_len = hlen;
+  v.h_hash = hhash;
+  v.pool_parent = ppar;
+  v.pool_tok = ptok;
+  v.pool_n = pn;
+  v.pool_cap = kPoolCap;
   d->slot_open.assign((size_t)c.max_streams, 0);
   d->last_stream = s;
   *out = d.release();
@@ -239,7 +275,10 @@ extern "C" tsd_status tsd_stream_open(tsd_decoder* d, int32_t* slot_out) {
   tsd_status st = set_device(d);
   if (st) return st;
   int slot = (int)(it - d->slot_open.begin());
-  launch_open(d->view, slot, d->last_stream);
+  if (d->cfg.beam_k > 1 && (!d->view.h_live || !d->view.pool_n))
+    return fail(TSD_ESTATE, "tsd_stream_open: beam state missing");
+  if (d->cfg.beam_k > 1) launch_open_beam(d->view, slot, d->last_stream);
+  else launch_open(d->view, slot, d->last_stream);
   TSD_CUDA(cudaGetLastError());
   *it = 1;
   *slot_out = slot;
@@ -263,6 +302,7 @@ extern "C" tsd_status tsd_decode_chunk(tsd_decoder* d, int32_t n, const int32_t*
   if (!d || !slots || !enc_bf16 || !out_counts) return fail(TSD_EINVAL, "tsd_decode_chunk: NULL argument");
   if (d->cfg.beam_k == 1 && (!out_tokens || !out_frames || !out_scores))
     return fail(TSD_EINVAL, "tsd_decode_chunk: NULL output array");
+  if (d->cfg.beam_k > 1 && !out_scores) return fail(TSD_EINVAL, "tsd_decode_chunk: NULL out_scores");
   if (n < 1 || n > d->cfg.max_streams) return fail(TSD_EINVAL, "tsd_decode_chunk: n=%d out of [1, %d]", n, d->cfg.max_streams);
   if (T < 1 || T > d->cfg.max_T) return fail(TSD_EINVAL, "tsd_decode_chunk: T=%d out of [1, %d]", T, d->cfg.max_T);
   if (!std::isfinite(lambda) || !std::isfinite(beta)) return fail(TSD_EINVAL, "tsd_decode_chunk: non-finite weight");
@@ -351,28 +391,105 @@ extern "C" tsd_status tsd_stream_state(tsd_decoder* d, int32_t slot, int32_t* lm
   TSD_CUDA(cudaStreamSynchronize(d->last_stream));
   int32_t ll = 0, tl = 0, ls = 0, chain_lm[kLmChain], chain_tr[kTrChain];
   const DecView& v = d->view;
-  TSD_CUDA(cudaMemcpy(&ls, v.s_last + slot, 4, cudaMemcpyDeviceToHost));
-  TSD_CUDA(cudaMemcpy(&ll, v.s_lm_len + slot, 4, cudaMemcpyDeviceToHost));
-  TSD_CUDA(cudaMemcpy(&tl, v.s_tr_len + slot, 4, cudaMemcpyDeviceToHost));
-  TSD_CUDA(cudaMemcpy(chain_lm, v.s_lm_chain + (size_t)slot * kLmChain, sizeof(chain_lm), cudaMemcpyDeviceToHost));
-  TSD_CUDA(cudaMemcpy(chain_tr, v.s_tr_chain + (size_t)slot * kTrChain, sizeof(chain_tr), cudaMemcpyDeviceToHost));
+  const size_t h = (size_t)slot * d->cfg.beam_k;  // beam: the slot's first hypothesis
+  TSD_CUDA(cudaMemcpy(&ls, v.s_last + h, 4, cudaMemcpyDeviceToHost));
+  TSD_CUDA(cudaMemcpy(&ll, v.s_lm_len + h, 4, cudaMemcpyDeviceToHost));
+  TSD_CUDA(cudaMemcpy(&tl, v.s_tr_len + h, 4, cudaMemcpyDeviceToHost));
+  TSD_CUDA(cudaMemcpy(chain_lm, v.s_lm_chain + h * kLmChain, sizeof(chain_lm), cudaMemcpyDeviceToHost));
+  TSD_CUDA(cudaMemcpy(chain_tr, v.s_tr_chain + h * kTrChain, sizeof(chain_tr), cudaMemcpyDeviceToHost));
   if (lm_state) *lm_state = ll > 0 ? chain_lm[ll - 1] : 0;
   if (trie_node) *trie_node = tl > 0 ? chain_tr[0] : 0;
   if (last) *last = ls;
   return TSD_OK;
 }
 
-extern "C" tsd_status tsd_stream_result(tsd_decoder* d, int32_t, int32_t*, int32_t, int32_t*, float*) {
-  clear_error();
-  if (!d) return fail(TSD_EINVAL, "tsd_stream_result: NULL decoder");
-  return fail(TSD_EINVAL, "tsd_stream_result: only beam decoders keep hypotheses");
+namespace {
+// Live hypotheses of a beam slot, read back from the device (synchronizes).
+struct HostHyp {
+  std::vector<int32_t> y;
+  double score;
+};
+
+tsd_status read_hyps(tsd_decoder* d, int32_t slot, std::vector<HostHyp>& out) {
+  const int K = d->cfg.beam_k;
+  tsd_status st = set_device(d);
+  if (st) return st;
+  TSD_CUDA(cudaStreamSynchronize(d->last_stream));
+  const DecView& v = d->view;
+  std::vector<int32_t> live(K), node(K), len(K);
+  std::vector<double> score(K);
+  const size_t h = (size_t)slot * K;
+  TSD_CUDA(cudaMemcpy(live.data(), v.h_live + h, sizeof(int32_t) * K, cudaMemcpyDeviceToHost));
+  TSD_CUDA(cudaMemcpy(node.data(), v.h_node + h, sizeof(int32_t) * K, cudaMemcpyDeviceToHost));
+  TSD_CUDA(cudaMemcpy(len.data(), v.h_len + h, sizeof(int32_t) * K, cudaMemcpyDeviceToHost));
+  TSD_CUDA(cudaMemcpy(score.data(), v.h_score + h, sizeof(double) * K, cudaMemcpyDeviceToHost));
+  int32_t used = 0;
+  TSD_CUDA(cudaMemcpy(&used, v.pool_n + slot, sizeof(int32_t), cudaMemcpyDeviceToHost));
+  std::vector<int32_t> par((size_t)std::max(used, 1)), tok((size_t)std::max(used, 1));
+  if (used > 0) {
+    TSD_CUDA(cudaMemcpy(par.data(), v.pool_parent + (size_t)slot * v.pool_cap, sizeof(int32_t) * used, cudaMemcpyDeviceToHost));
+    TSD_CUDA(cudaMemcpy(tok.data(), v.pool_tok + (size_t)slot * v.pool_cap, sizeof(int32_t) * used, cudaMemcpyDeviceToHost));
+  }
+  out.clear();
+  for (int k = 0; k < K; ++k) {
+    if (!live[k]) continue;
+    HostHyp hy;
+    hy.score = score[k];
+    for (int x = node[k], i = 0; x >= 0 && x < used && i <= used; x = par[x], ++i) hy.y.push_back(tok[x]);
+    std::reverse(hy.y.begin(), hy.y.end());
+    out.push_back(std::move(hy));
+  }
+  return TSD_OK;
 }
 
-extern "C" tsd_status tsd_stream_hyps(tsd_decoder* d, int32_t, int32_t*, int32_t, int32_t*, float*,
-                                      int32_t, int32_t*) {
+tsd_status check_beam_slot(tsd_decoder* d, int32_t slot, const char* fn) {
+  if (!d) return fail(TSD_EINVAL, "%s: NULL decoder", fn);
+  if (d->cfg.beam_k < 2) return fail(TSD_EINVAL, "%s: only beam decoders keep hypotheses", fn);
+  if (slot < 0 || slot >= d->cfg.max_streams || !d->slot_open[(size_t)slot])
+    return fail(TSD_ESTATE, "%s: slot %d is not open", fn, slot);
+  return TSD_OK;
+}
+}  // namespace
+
+extern "C" tsd_status tsd_stream_result(tsd_decoder* d, int32_t slot, int32_t* buf, int32_t cap, int32_t* len,
+                                        float* score) {
   clear_error();
-  if (!d) return fail(TSD_EINVAL, "tsd_stream_hyps: NULL decoder");
-  return fail(TSD_EINVAL, "tsd_stream_hyps: only beam decoders keep hypotheses");
+  tsd_status st = check_beam_slot(d, slot, "tsd_stream_result");
+  if (st) return st;
+  if (!len || (cap > 0 && !buf)) return fail(TSD_EINVAL, "tsd_stream_result: NULL output");
+  std::vector<HostHyp> hy;
+  if ((st = read_hyps(d, slot, hy))) return st;
+  size_t best = 0;
+  for (size_t i = 1; i < hy.size(); ++i)
+    if (hy[i].score > hy[best].score) best = i;
+  if (hy.empty()) {
+    *len = 0;
+    if (score) *score = 0.f;
+    return TSD_OK;
+  }
+  *len = (int32_t)hy[best].y.size();
+  for (int32_t i = 0; i < *len && i < cap; ++i) buf[i] = hy[best].y[(size_t)i];
+  if (score) *score = (float)hy[best].score;
+  return TSD_OK;
+}
+
+extern "C" tsd_status tsd_stream_hyps(tsd_decoder* d, int32_t slot, int32_t* buf, int32_t cap_len, int32_t* lengths,
+                                      float* scores, int32_t cap_hyps, int32_t* n_hyps) {
+  clear_error();
+  tsd_status st = check_beam_slot(d, slot, "tsd_stream_hyps");
+  if (st) return st;
+  if (!n_hyps) return fail(TSD_EINVAL, "tsd_stream_hyps: NULL output");
+  std::vector<HostHyp> hy;
+  if ((st = read_hyps(d, slot, hy))) return st;
+  *n_hyps = (int32_t)hy.size();
+  for (int32_t i = 0; i < (int32_t)hy.size() && i < cap_hyps; ++i) {
+    if (lengths) lengths[i] = (int32_t)hy[(size_t)i].y.size();
+    if (scores) scores[i] = (float)hy[(size_t)i].score;
+    if (buf)
+      for (int32_t j = 0; j < (int32_t)hy[(size_t)i].y.size() && j < cap_len; ++j)
+        buf[(size_t)i * cap_len + j] = hy[(size_t)i].y[(size_t)j];
+  }
+  return TSD_OK;
 }
 
 extern "C" tsd_status tsd_decoder_set_graphs(tsd_decoder* d, int32_t enable) {
@@ -482,7 +599,8 @@ extern "C" tsd_status tsd_decoder_replay(tsd_decoder* d, int32_t kernel, int32_t
   const int S = steps_per_chunk(d, d->last_T);
   if (algo_bytes) TSD_CUDA(cudaMemsetAsync(d->view.ctr, 0, sizeof(unsigned long long), s));
   for (int i = 0; i < reps; ++i) {
-    if (kernel == 0) launch_row(d->view, M, S - 1, 2, d->row_smem, s, false);
+    if (kernel == 0 && d->cfg.beam_k > 1) launch_row_beam(d->view, d->last_n, S - 1, 2, d->row_smem, s, false);
+    else if (kernel == 0) launch_row(d->view, M, S - 1, 2, d->row_smem, s, false);
     else if (d->joint_kind == 0) launch_joint_tc(*d->jtc, d->view, M, 1 << 30, s, false);
     else launch_joint(d->view, M, 1 << 30, s);
   }

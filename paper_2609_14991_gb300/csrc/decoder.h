@@ -48,6 +48,17 @@ struct DecView {
   float* cap_logits;
   int32_t* cap_rows;
   int32_t cap_steps;
+  // beam search (K > 1), per slot x K hypotheses
+  float2* bpart;        // [M_pad][n_ptiles][1 + K]: (max, sum exp), then top-K (value, label)
+  double* h_score;      // hypothesis score
+  int32_t* h_live;      // 1 if the hypothesis slot holds a live hypothesis
+  int32_t* h_node;      // label-sequence node (-1 = empty sequence)
+  int32_t* h_len;       // label-sequence length
+  unsigned long long* h_hash;  // rolling hash of the label sequence
+  int32_t* pool_parent; // [slots][pool_cap] label-sequence nodes: parent node
+  int32_t* pool_tok;    // [slots][pool_cap] label of the node
+  int32_t* pool_n;      // [slots] nodes used
+  int32_t pool_cap;
   int32_t* err;  // device status word: nonzero after a bounded wait expired
   unsigned long long* ctr;  // algorithmic bytes counted by replayed row passes
 };
@@ -60,6 +71,10 @@ void launch_row(const DecView& d, int M, int step, int mode, size_t smem, cudaSt
 void launch_joint(const DecView& d, int M, int step, cudaStream_t s);
 size_t row_smem_bytes(int V4);
 cudaError_t prepare_kernels(size_t row_smem);
+void launch_row_beam(const DecView& d, int n, int step, int mode, size_t smem, cudaStream_t s, bool pdl);
+void launch_open_beam(const DecView& d, int slot, cudaStream_t s);
+cudaError_t prepare_beam_kernels(size_t row_smem);
+constexpr int kPoolCap = 8192;  // label-sequence nodes per beam stream
 
 }  // namespace tsd
 

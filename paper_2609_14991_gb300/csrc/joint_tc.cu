@@ -139,7 +139,9 @@ struct Smem {
   static constexpr int kBytes = kStages * kStageBytes + 1024 /*align*/ + 256 /*barriers*/;
 };
 
-template <int BN>
+// BEAM: instead of the single best fused label, each row keeps the top-K
+// (K = beam width <= 8) fused values of the tile, ties to the lower label.
+template <int BN, bool BEAM>
 __global__ void __launch_bounds__(kThreads, 1)
     k_joint_tc(DecView d, int step, const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB) {
   using S = Smem<BN>;
@@ -231,6 +233,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     const float* brow = d.bias + (size_t)(live ? gr : 0) * d.N_pad + n0;
     float mx = kNegInf, se = 0.f, bv = kNegInf;
     int bi = INT_MAX;
+    const int K = d.K;
+    float tv[8];
+    int ti[8];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) { tv[j] = kNegInf; ti[j] = INT_MAX; }
+    float tmin = kNegInf;  // tv[K-1]
     ok = __all_sync(0xffffffffu, mbar_wait(accum, 0));  // warp-uniform: tcgen05.ld is .sync.aligned
     if (!ok && lane == 0) atomicOr(d.err, 4);
     fence_after();
@@ -261,7 +269,24 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (gc < N) {
             cm = fmaxf(cm, l[i]);
             const float f = l[i] + (gc < V ? b[i] : 0.f);
-            if (f > bv) { bv = f; bi = gc; }
+            if (!BEAM) {
+              if (f > bv) { bv = f; bi = gc; }
+            } else if (f > tmin) {
+              // bubble the new value into the sorted list (labels arrive in
+              // increasing order, so a later equal value stays behind)
+              float cv = f;
+              int ci = gc;
+#pragma unroll
+              for (int j = 0; j < 8; ++j) {
+                if (j < K && cv > tv[j]) {
+                  const float tf = tv[j]; tv[j] = cv; cv = tf;
+                  const int tk = ti[j]; ti[j] = ci; ci = tk;
+                }
+              }
+#pragma unroll
+              for (int j = 0; j < 8; ++j)
+                if (j == K - 1) tmin = tv[j];
+            }
           }
         }
         if (cm != kNegInf) {
@@ -280,7 +305,17 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (c0 + i < N) cl[c0 + i] = l[i];
         }
       }
-      if (live) d.part[(size_t)gr * d.n_ptiles + blockIdx.x] = make_float4(mx, se, bv, __int_as_float(bi));
+      if (live) {
+        if (!BEAM) {
+          d.part[(size_t)gr * d.n_ptiles + blockIdx.x] = make_float4(mx, se, bv, __int_as_float(bi));
+        } else {
+          float2* bp = d.bpart + ((size_t)gr * d.n_ptiles + blockIdx.x) * (1 + K);
+          bp[0] = make_float2(mx, se);
+#pragma unroll
+          for (int j = 0; j < 8; ++j)
+            if (j < K) bp[1 + j] = make_float2(tv[j], __int_as_float(ti[j]));
+        }
+      }
     }
   }
   fence_before();
@@ -333,9 +368,19 @@ cudaError_t joint_tc_prepare(JointTc* jt, const uint16_t* A, int M_pad, const ui
   if (!make_map(&jt->mapA, A, H, M_pad, kBM)) return cudaErrorInvalidValue;
   if (!make_map(&jt->mapB, Wt, H, N_pad, bn)) return cudaErrorInvalidValue;
   cudaError_t e = cudaSuccess;
-  if (bn == 256) e = cudaFuncSetAttribute(k_joint_tc<256>, cudaFuncAttributeMaxDynamicSharedMemorySize, Smem<256>::kBytes);
-  else if (bn == 128) e = cudaFuncSetAttribute(k_joint_tc<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, Smem<128>::kBytes);
-  else e = cudaFuncSetAttribute(k_joint_tc<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, Smem<64>::kBytes);
+  if (bn == 256) {
+    e = cudaFuncSetAttribute(k_joint_tc<256, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, Smem<256>::kBytes);
+    if (e == cudaSuccess)
+      e = cudaFuncSetAttribute(k_joint_tc<256, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, Smem<256>::kBytes);
+  } else if (bn == 128) {
+    e = cudaFuncSetAttribute(k_joint_tc<128, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, Smem<128>::kBytes);
+    if (e == cudaSuccess)
+      e = cudaFuncSetAttribute(k_joint_tc<128, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, Smem<128>::kBytes);
+  } else {
+    e = cudaFuncSetAttribute(k_joint_tc<64, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, Smem<64>::kBytes);
+    if (e == cudaSuccess)
+      e = cudaFuncSetAttribute(k_joint_tc<64, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, Smem<64>::kBytes);
+  }
   return e;
 }
 
@@ -349,15 +394,19 @@ void launch_joint_tc(const JointTc& jt, const DecView& d, int M, int step, cudaS
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = pdl ? 1 : 0;
+  const bool beam = d.K > 1;
   if (jt.bn == 256) {
     cfg.dynamicSmemBytes = Smem<256>::kBytes;
-    cudaLaunchKernelEx(&cfg, k_joint_tc<256>, d, step, jt.mapA, jt.mapB);
+    if (beam) cudaLaunchKernelEx(&cfg, k_joint_tc<256, true>, d, step, jt.mapA, jt.mapB);
+    else cudaLaunchKernelEx(&cfg, k_joint_tc<256, false>, d, step, jt.mapA, jt.mapB);
   } else if (jt.bn == 128) {
     cfg.dynamicSmemBytes = Smem<128>::kBytes;
-    cudaLaunchKernelEx(&cfg, k_joint_tc<128>, d, step, jt.mapA, jt.mapB);
+    if (beam) cudaLaunchKernelEx(&cfg, k_joint_tc<128, true>, d, step, jt.mapA, jt.mapB);
+    else cudaLaunchKernelEx(&cfg, k_joint_tc<128, false>, d, step, jt.mapA, jt.mapB);
   } else {
     cfg.dynamicSmemBytes = Smem<64>::kBytes;
-    cudaLaunchKernelEx(&cfg, k_joint_tc<64>, d, step, jt.mapA, jt.mapB);
+    if (beam) cudaLaunchKernelEx(&cfg, k_joint_tc<64, true>, d, step, jt.mapA, jt.mapB);
+    else cudaLaunchKernelEx(&cfg, k_joint_tc<64, false>, d, step, jt.mapA, jt.mapB);
   }
 }
 

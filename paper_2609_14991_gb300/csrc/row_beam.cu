@@ -1,0 +1,469 @@
+// Beam-search row pass: one CTA per stream, K hypotheses per stream.
+//
+// At label step s (frame s of the chunk; one label or blank per frame) it
+//   1. turns the joint kernel's per-tile partials of frame s-1 into each live
+//      hypothesis's log-sum-exp and its K best extensions (blank keeps the
+//      labels, label v appends v), scored hypothesis score + fused value -
+//      log-sum-exp (Eq. 1 summed along the hypothesis);
+//   2. keeps the global top K of those candidates by (score desc,
+//      hypothesis asc, label asc) and merges candidates with equal label
+//      sequences by log-sum-exp of their scores, in order of first appearance
+//      (so fewer than K may survive);
+//   3. advances each survivor's LM and phrase-trie suffix chains from its
+//      parent's (independent per-level searches, as in the greedy pass);
+//   4. writes the joint input and the fusion bias row of every survivor.
+// Label sequences live in a per-stream pool of (parent, label) nodes; two
+// candidates are the same sequence when their lengths and rolling hashes
+// agree and their node chains compare equal label by label.
+#include "row_common.cuh"
+
+namespace tsd {
+
+namespace {
+
+using row::kNegInf;
+using row::lse_merge;
+using row::warp_find;
+
+constexpr int kMaxK = 8;
+constexpr int kCandPerLane = 16;  // per-hypothesis candidates: n_tiles * K <= 512
+
+__device__ __forceinline__ unsigned long long hash_push(unsigned long long h, int v) {
+  return h * 0x100000001B3ull + (unsigned long long)(v + 1);
+}
+
+// The label sequences of pool nodes x and y are equal (-1 = empty sequence).
+__device__ bool nodes_equal(const int32_t* par, const int32_t* tok, int x, int y, int cap) {
+  for (int i = 0; i <= cap && x != y; ++i) {
+    if (x < 0 || y < 0) return false;
+    if (__ldcg(tok + x) != __ldcg(tok + y)) return false;
+    x = __ldcg(par + x);
+    y = __ldcg(par + y);
+  }
+  return x == y;
+}
+
+// seq(a) [+ label ea if ea >= 0] equals seq(b) [+ eb].
+__device__ bool seq_equal(const int32_t* par, const int32_t* tok, int a, int ea, int b, int eb, int cap) {
+  if (ea >= 0 && eb >= 0) return ea == eb && nodes_equal(par, tok, a, b, cap);
+  if (ea < 0 && eb < 0) return nodes_equal(par, tok, a, b, cap);
+  if (ea < 0) {
+    if (a < 0 || __ldcg(tok + a) != eb) return false;
+    return nodes_equal(par, tok, __ldcg(par + a), b, cap);
+  }
+  if (b < 0 || __ldcg(tok + b) != ea) return false;
+  return nodes_equal(par, tok, a, __ldcg(par + b), cap);
+}
+
+__device__ __forceinline__ double log_add(double a, double b) {
+  const double m = fmax(a, b);
+  return m + log(exp(a - m) + exp(b - m));
+}
+
+// candidate order: score desc, hypothesis asc, label asc
+__device__ __forceinline__ bool cand_before(double s1, int h1, int t1, double s2, int h2, int t2) {
+  if (s1 != s2) return s1 > s2;
+  if (h1 != h2) return h1 < h2;
+  return t1 < t2;
+}
+
+// mode: 0 = label step, 1 = final step (apply the last frame's selection),
+// 2 = replay (redo the step without committing anything; for timing).
+__global__ void __launch_bounds__(kRowThreads) k_row_beam(DecView d, int step, int mode) {
+  const Params* __restrict__ P = d.params;
+  const int b = blockIdx.x;
+  const int K = d.K, V = d.V;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const bool commit = (mode != 2);
+  extern __shared__ __align__(16) unsigned char smem[];
+  unsigned long long* lmkey = reinterpret_cast<unsigned long long*>(smem);
+  int* dep = reinterpret_cast<int*>(lmkey + d.V4);
+
+  __shared__ int s_slot, s_T;
+  __shared__ int o_live[kMaxK], o_last[kMaxK], o_node[kMaxK], o_len[kMaxK], o_lml[kMaxK], o_trl[kMaxK];
+  __shared__ double o_score[kMaxK];
+  __shared__ unsigned long long o_hash[kMaxK];
+  __shared__ int o_lm[kMaxK][kLmChain], o_tr[kMaxK][kTrChain];
+  __shared__ int n_cnt;
+  __shared__ int n_par[kMaxK], n_tok[kMaxK], n_node[kMaxK], n_len[kMaxK], n_lml[kMaxK], n_trl[kMaxK], n_last[kMaxK];
+  __shared__ double n_score[kMaxK];
+  __shared__ unsigned long long n_hash[kMaxK];
+  __shared__ int n_lm[kMaxK][kLmChain], n_tr[kMaxK][kTrChain];
+  __shared__ double c_score[kMaxK * kMaxK];
+  __shared__ float c_inc[kMaxK * kMaxK];
+  __shared__ int c_tok[kMaxK * kMaxK];
+  __shared__ int s_sel[kMaxK], s_into[kMaxK], s_nsel;
+  __shared__ int s_task0[kMaxK + 1];
+  __shared__ int sr_lm[kMaxK][kLmChain];
+  __shared__ int sr_trn[kMaxK][kTrChain], sr_trx[kMaxK][kTrChain];
+  __shared__ int sr_uni[kMaxK], sr_rc[kMaxK], sr_rn[kMaxK];
+  __shared__ row::ChainRecs rc;
+
+  // previous state of this stream's hypotheses (written by the previous row
+  // pass; L2-only loads, see the greedy pass)
+  if (tid == 0) {
+    s_slot = __ldcg(P->slots + b);
+    s_T = __ldcg(&P->T);
+  }
+  __syncthreads();
+  const int slot = s_slot, T = s_T;
+  const int hb = slot * K;
+  const int cap = d.pool_cap;
+  const int32_t* pool_par = d.pool_parent + (size_t)slot * cap;
+  const int32_t* pool_tok = d.pool_tok + (size_t)slot * cap;
+  if (tid < K) {
+    const int h = hb + tid;
+    o_live[tid] = __ldcg(d.h_live + h);
+    o_last[tid] = __ldcg(d.s_last + h);
+    o_node[tid] = __ldcg(d.h_node + h);
+    o_len[tid] = __ldcg(d.h_len + h);
+    o_score[tid] = __ldcg(d.h_score + h);
+    o_hash[tid] = __ldcg(d.h_hash + h);
+    o_lml[tid] = d.has_lm ? __ldcg(d.s_lm_len + h) : 0;
+    o_trl[tid] = d.has_tr ? __ldcg(d.s_tr_len + h) : 0;
+  }
+  __syncthreads();
+  for (int i = tid; i < K * kLmChain; i += kRowThreads) {
+    const int k = i / kLmChain, l = i % kLmChain;
+    if (l < o_lml[k]) o_lm[k][l] = __ldcg(d.s_lm_chain + (size_t)(hb + k) * kLmChain + l);
+  }
+  for (int i = tid; i < K * kTrChain; i += kRowThreads) {
+    const int k = i / kTrChain, l = i % kTrChain;
+    if (l < o_trl[k]) o_tr[k][l] = __ldcg(d.s_tr_chain + (size_t)(hb + k) * kTrChain + l);
+  }
+  __syncthreads();
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+
+  if (step > 0) {
+    // 1. per live hypothesis (warp k): log-sum-exp and its K best extensions
+    if (warp < K) {
+      const int k = warp;
+      const bool live = o_live[k] != 0;
+      const int r = b * K + k;
+      const float2* bp = d.bpart + (size_t)r * d.n_ptiles * (1 + K);
+      float m = kNegInf, s = 0.f;
+      if (live) {
+        for (int j = lane; j < d.n_ptiles; j += 32) {
+          const float2 p = __ldcg(bp + (size_t)j * (1 + K));
+          lse_merge(m, s, p.x, p.y);
+        }
+      }
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) {
+        const float m2 = __shfl_xor_sync(0xffffffffu, m, o), s2 = __shfl_xor_sync(0xffffffffu, s, o);
+        lse_merge(m, s, m2, s2);
+      }
+      const float lse = m + logf(s);
+      float cv[kCandPerLane];
+      int ct[kCandPerLane];
+      const int nc = live ? d.n_ptiles * K : 0;
+#pragma unroll
+      for (int q = 0; q < kCandPerLane; ++q) {
+        const int i = lane + 32 * q;
+        cv[q] = kNegInf;
+        ct[q] = INT_MAX;
+        if (i < nc) {
+          const float2 p = __ldcg(bp + (size_t)(i / K) * (1 + K) + 1 + (i % K));
+          cv[q] = p.x;
+          ct[q] = __float_as_int(p.y);
+        }
+      }
+      for (int round = 0; round < K; ++round) {
+        // this lane's best remaining (value desc, label asc)
+        float bv = kNegInf;
+        int bt = INT_MAX, bq = -1;
+#pragma unroll
+        for (int q = 0; q < kCandPerLane; ++q)
+          if (cv[q] > bv || (cv[q] == bv && cv[q] != kNegInf && ct[q] < bt)) { bv = cv[q]; bt = ct[q]; bq = q; }
+        float wv = bv;
+        int wt = bt, wl = lane;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+          const float v2 = __shfl_xor_sync(0xffffffffu, wv, o);
+          const int t2 = __shfl_xor_sync(0xffffffffu, wt, o), l2 = __shfl_xor_sync(0xffffffffu, wl, o);
+          if (v2 > wv || (v2 == wv && (t2 < wt || (t2 == wt && l2 < wl)))) { wv = v2; wt = t2; wl = l2; }
+        }
+        if (lane == wl && bq >= 0) {
+#pragma unroll
+          for (int q = 0; q < kCandPerLane; ++q)
+            if (q == bq) cv[q] = kNegInf;
+        }
+        if (lane == 0) {
+          const int c = k * K + round;
+          const bool valid = wv != kNegInf && wt >= 0 && wt <= V;
+          c_tok[c] = valid ? wt : -1;
+          c_inc[c] = valid ? wv - lse : 0.f;
+          c_score[c] = valid ? o_score[k] + (double)(wv - lse) : -1e300;
+        }
+      }
+    }
+    __syncthreads();
+    // 2. global top K, then merge equal label sequences
+    if (tid == 0) {
+      bool used[kMaxK * kMaxK];
+      for (int c = 0; c < K * K; ++c) used[c] = false;
+      int nsel = 0;
+      for (int round = 0; round < K; ++round) {
+        int best = -1;
+        for (int c = 0; c < K * K; ++c) {
+          if (used[c] || c_tok[c] < 0) continue;
+          if (best < 0 || cand_before(c_score[c], c / K, c_tok[c], c_score[best], best / K, c_tok[best])) best = c;
+        }
+        if (best < 0) break;
+        used[best] = true;
+        s_sel[nsel++] = best;
+      }
+      s_nsel = nsel;
+      int cnt = 0;
+      int pool_used = __ldcg(d.pool_n + slot);
+      for (int i = 0; i < nsel; ++i) {
+        const int c = s_sel[i], p = c / K, y = c_tok[c];
+        const int len = o_len[p] + (y != V ? 1 : 0);
+        const unsigned long long hsh = (y != V) ? hash_push(o_hash[p], y) : o_hash[p];
+        int into = -1;
+        for (int j = 0; j < cnt; ++j) {
+          if (n_len[j] != len || n_hash[j] != hsh) continue;
+          const int pj = n_par[j];
+          if (seq_equal(pool_par, pool_tok, o_node[p], y != V ? y : -1, o_node[pj], n_tok[j] != V ? n_tok[j] : -1, cap)) {
+            into = j;
+            break;
+          }
+        }
+        if (into >= 0) {
+          n_score[into] = log_add(n_score[into], c_score[c]);
+        } else {
+          into = cnt++;
+          n_par[into] = p;
+          n_tok[into] = y;
+          n_score[into] = c_score[c];
+          n_len[into] = len;
+          n_hash[into] = hsh;
+        }
+        s_into[i] = into;
+      }
+      // label-sequence nodes of the survivors that appended a label
+      for (int j = 0; j < cnt; ++j) {
+        const int p = n_par[j];
+        if (n_tok[j] == V) {
+          n_node[j] = o_node[p];
+        } else if (pool_used < cap) {
+          n_node[j] = pool_used;
+          if (commit) {
+            d.pool_parent[(size_t)slot * cap + pool_used] = o_node[p];
+            d.pool_tok[(size_t)slot * cap + pool_used] = n_tok[j];
+          }
+          ++pool_used;
+        } else {
+          n_node[j] = o_node[p];  // pool full: the label is not recorded
+          if (commit) atomicOr(d.err, 8);
+        }
+      }
+      if (commit) d.pool_n[slot] = pool_used;
+      n_cnt = cnt;
+      int tasks = 0;
+      for (int j = 0; j < cnt; ++j) {
+        s_task0[j] = tasks;
+        if (n_tok[j] != V) tasks += o_lml[n_par[j]] + o_trl[n_par[j]];
+      }
+      s_task0[cnt] = tasks;
+      if (d.cap_rows && step - 1 < d.cap_steps && commit) {
+        for (int i = 0; i < K; ++i) {
+          int* cr = d.cap_rows + ((size_t)(step - 1) * P->n * K + (size_t)b * K + i) * 4;
+          if (i < nsel) {
+            cr[0] = s_sel[i] / K;
+            cr[1] = c_tok[s_sel[i]];
+            cr[2] = __float_as_int(c_inc[s_sel[i]]);
+            cr[3] = s_into[i];
+          } else {
+            cr[0] = -1; cr[1] = -1; cr[2] = 0; cr[3] = -1;
+          }
+        }
+      }
+    }
+    __syncthreads();
+    // 3. searches of each survivor's label in its parent's chains
+    const int cnt = n_cnt;
+    if (tid >= kRowThreads - kMaxK) {
+      const int j = tid - (kRowThreads - kMaxK);
+      if (j < cnt && n_tok[j] != V) {
+        const int y = n_tok[j];
+        sr_uni[j] = (d.has_lm && d.lm.order >= 2) ? __ldg(d.lm.uni_tgt + y) : -1;
+        sr_rc[j] = d.has_tr ? __ldg(d.tr.root_child + y) : 0;
+        sr_rn[j] = d.has_tr ? __ldg(d.tr.root_next + y) : 0;
+      }
+    }
+    for (int task = warp; task < s_task0[cnt]; task += kRowThreads / 32) {
+      int j = 0;
+      while (j + 1 < cnt && s_task0[j + 1] <= task) ++j;
+      const int p = n_par[j], y = n_tok[j];
+      const int l = task - s_task0[j];
+      if (l < o_lml[p]) {
+        const int st = o_lm[p][l];
+        const int bb = __ldg(d.lm.st_begin + st), c = __ldg(d.lm.st_count + st);
+        const int i = warp_find(d.lm.arc_tok + bb, c, y, lane);
+        if (lane == 0) sr_lm[j][l] = (i >= 0) ? __ldg(d.lm.arc_tgt + bb + i) : -2;
+      } else {
+        const int k = l - o_lml[p];
+        const int q = o_tr[p][k];
+        const int bb = __ldg(d.tr.nd_begin + q), c = __ldg(d.tr.nd_count + q);
+        const int i = warp_find(d.tr.ch_tok + bb, c, y, lane);
+        if (lane == 0) {
+          sr_trn[j][k] = (i >= 0) ? __ldg(d.tr.ch_node + bb + i) : -1;
+          sr_trx[j][k] = (i >= 0) ? __ldg(d.tr.ch_next + bb + i) : -1;
+        }
+      }
+    }
+    __syncthreads();
+    // 4. survivors' chains (thread j for survivor j)
+    if (tid < cnt) {
+      const int j = tid, p = n_par[j], y = n_tok[j];
+      if (y == V) {
+        n_last[j] = o_last[p];
+        n_lml[j] = o_lml[p];
+        n_trl[j] = o_trl[p];
+        for (int l = 0; l < o_lml[p]; ++l) n_lm[j][l] = o_lm[p][l];
+        for (int l = 0; l < o_trl[p]; ++l) n_tr[j][l] = o_tr[p][l];
+      } else {
+        n_last[j] = y;
+        int ln = 0;
+        if (sr_uni[j] >= 0) {
+          n_lm[j][ln++] = sr_uni[j];
+          for (int l = 0; l < o_lml[p] && ln < kLmChain; ++l) {
+            const int tgt = sr_lm[j][l];
+            if (tgt < 0) break;
+            n_lm[j][ln++] = tgt;
+          }
+        }
+        n_lml[j] = ln;
+        int tn = 0;
+        bool reset = false;
+        if (d.has_tr) {
+          for (int k = 0; k < o_trl[p]; ++k) {
+            if (sr_trn[j][k] < 0) continue;
+            if (tn == 0 && sr_trx[j][k] == 0) reset = true;
+            if (tn < kTrChain) n_tr[j][tn++] = sr_trn[j][k];
+          }
+          if (sr_rc[j] != 0) {
+            if (tn == 0 && sr_rn[j] == 0) reset = true;
+            if (tn < kTrChain) n_tr[j][tn++] = sr_rc[j];
+          }
+          if (reset) tn = 0;
+        }
+        n_trl[j] = tn;
+      }
+    }
+    __syncthreads();
+  } else {
+    // frame 0 of the chunk: the hypotheses carried over from the last chunk
+    if (tid == 0) {
+      int cnt = 0;
+      for (int k = 0; k < K; ++k) cnt += o_live[k] ? 1 : 0;
+      n_cnt = cnt;
+    }
+    if (tid < K) {
+      const int k = tid;
+      n_par[k] = k;
+      n_tok[k] = V;
+      n_score[k] = o_score[k];
+      n_node[k] = o_node[k];
+      n_len[k] = o_len[k];
+      n_hash[k] = o_hash[k];
+      n_last[k] = o_last[k];
+      n_lml[k] = o_lml[k];
+      n_trl[k] = o_trl[k];
+      for (int l = 0; l < o_lml[k]; ++l) n_lm[k][l] = o_lm[k][l];
+      for (int l = 0; l < o_trl[k]; ++l) n_tr[k][l] = o_tr[k][l];
+    }
+    __syncthreads();
+  }
+  const int cnt = n_cnt;
+
+  // 5. commit the survivors (compact, first cnt slots) and retire the rest
+  if (commit && step > 0) {
+    if (tid < K) {
+      const int h = hb + tid;
+      const bool live = tid < cnt;
+      d.h_live[h] = live ? 1 : 0;
+      if (live) {
+        d.h_score[h] = n_score[tid];
+        d.h_node[h] = n_node[tid];
+        d.h_len[h] = n_len[tid];
+        d.h_hash[h] = n_hash[tid];
+        d.s_last[h] = n_last[tid];
+        if (d.has_lm) d.s_lm_len[h] = n_lml[tid];
+        if (d.has_tr) d.s_tr_len[h] = n_trl[tid];
+      }
+    }
+    for (int i = tid; i < cnt * kLmChain; i += kRowThreads) {
+      const int k = i / kLmChain, l = i % kLmChain;
+      if (l < n_lml[k]) d.s_lm_chain[(size_t)(hb + k) * kLmChain + l] = n_lm[k][l];
+    }
+    for (int i = tid; i < cnt * kTrChain; i += kRowThreads) {
+      const int k = i / kTrChain, l = i % kTrChain;
+      if (l < n_trl[k]) d.s_tr_chain[(size_t)(hb + k) * kTrChain + l] = n_tr[k][l];
+    }
+  }
+  if (mode == 1) {
+    if (tid == 0) {
+      int best = 0;
+      for (int j = 1; j < cnt; ++j)
+        if (n_score[j] > n_score[best]) best = j;
+      P->out_count[b] = cnt ? n_len[best] : 0;
+      P->out_score[(size_t)b * T * d.max_sym] = cnt ? (float)n_score[best] : 0.f;
+    }
+    return;
+  }
+
+  // 6. joint input and fusion bias of every survivor for frame `step`
+  const uint16_t* enc_row = P->enc + ((size_t)b * T + min(step, T - 1)) * d.H;
+  for (int j = 0; j < cnt; ++j) {
+    const int r = b * K + j;
+    row::bias_prepare(d, n_lm[j], n_lml[j], n_tr[j], n_trl[j], rc, lmkey, dep);
+    row::build_joint_input(d, enc_row, n_last[j], r);
+    row::bias_finish(d, n_lml[j], n_trl[j], rc, P->lambda, P->beta, d.bias + (size_t)r * d.N_pad, lmkey, dep);
+    __syncthreads();  // the scratch is reused by the next survivor
+  }
+}
+
+__global__ void k_open_beam(DecView d, int slot) {
+  const int k = threadIdx.x;
+  if (k < d.K) {
+    const int h = slot * d.K + k;
+    d.h_live[h] = (k == 0) ? 1 : 0;
+    d.h_score[h] = 0.0;
+    d.h_node[h] = -1;
+    d.h_len[h] = 0;
+    d.h_hash[h] = 0ull;
+    d.s_last[h] = d.V;
+    d.s_lm_len[h] = 0;
+    d.s_tr_len[h] = 0;
+  }
+  if (k == 0) d.pool_n[slot] = 0;
+}
+
+}  // namespace
+
+void launch_row_beam(const DecView& d, int n, int step, int mode, size_t smem, cudaStream_t s, bool pdl) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(n);
+  cfg.blockDim = dim3(kRowThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl ? 1 : 0;
+  cudaLaunchKernelEx(&cfg, k_row_beam, d, step, mode);
+}
+
+void launch_open_beam(const DecView& d, int slot, cudaStream_t s) { k_open_beam<<<1, 32, 0, s>>>(d, slot); }
+
+cudaError_t prepare_beam_kernels(size_t row_smem) {
+  if (row_smem > 48 * 1024)
+    return cudaFuncSetAttribute(k_row_beam, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)row_smem);
+  return cudaSuccess;
+}
+
+}  // namespace tsd

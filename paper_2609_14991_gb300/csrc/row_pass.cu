@@ -14,45 +14,16 @@
 // LM state per order; every trie node that is a suffix of the current one),
 // so the next chain after label y is assembled from independent searches of
 // y in each chain element -- no dependent pointer chase.
-#include "decoder.h"
+#include "row_common.cuh"
 
 namespace tsd {
 
 namespace {
 
-constexpr float kNegInf = -__builtin_huge_valf();
-
-// Position of y in the sorted arr[0, n), or -1: a 32-ary search by one warp.
-__device__ __forceinline__ int warp_find(const int32_t* __restrict__ arr, int n, int y, int lane) {
-  int lo = 0, hi = n;
-  while (hi - lo > 32) {
-    int step = (hi - lo + 31) >> 5;
-    int idx = lo + lane * step;
-    int v = (idx < hi) ? __ldg(arr + idx) : INT_MAX;
-    unsigned m = __ballot_sync(0xffffffffu, v <= y);
-    if (m == 0) return -1;
-    int last = 31 - __clz((int)m);
-    lo = lo + last * step;
-    hi = min(hi, lo + step);
-  }
-  int idx = lo + lane;
-  bool hit = (idx < hi) && (__ldg(arr + idx) == y);
-  unsigned m = __ballot_sync(0xffffffffu, hit);
-  return m ? lo + __ffs((int)m) - 1 : -1;
-}
-
-// Merges two softmax partials (max, sum of exp(x - max)).
-__device__ __forceinline__ void lse_merge(float& m, float& s, float m2, float s2) {
-  if (m2 == kNegInf) return;
-  if (m == kNegInf) { m = m2; s = s2; return; }
-  float mx = fmaxf(m, m2);
-  s = s * expf(m - mx) + s2 * expf(m2 - mx);
-  m = mx;
-}
-
-__device__ __forceinline__ void best_merge(float& v, int& i, float v2, int i2) {
-  if (v2 > v || (v2 == v && i2 < i)) { v = v2; i = i2; }
-}
+using row::best_merge;
+using row::kNegInf;
+using row::lse_merge;
+using row::warp_find;
 
 // mode: 0 = label step, 1 = final step (apply the last decision only),
 // 2 = replay (redo the step's work without committing any state or output;
@@ -74,9 +45,7 @@ __global__ void __launch_bounds__(kRowThreads) k_row(DecView d, int step, int mo
   __shared__ int s_lm_tgt[kLmChain];            // target state of y's arc at each LM level (-2 none)
   __shared__ int s_tr_node[kTrChain], s_tr_nxt[kTrChain];  // child by y of each trie chain node (-1 none)
   __shared__ int s_uni_tgt, s_root_child, s_root_next;
-  __shared__ int s_lb[kLmChain], s_lc[kLmChain];
-  __shared__ float s_lo[kLmChain];
-  __shared__ int s_tb[kTrChain], s_tc[kTrChain], s_td[kTrChain];
+  __shared__ row::ChainRecs rc;
 
   // The row state below was written by the previous row pass; under
   // programmatic launch this grid may start before its own wait, so these
@@ -238,87 +207,12 @@ __global__ void __launch_bounds__(kRowThreads) k_row(DecView d, int step, int mo
   }
   if (t >= T) return;
 
-  // 3. state records of the new chains (one thread each), scratch reset
+  // 3. records of the new chains, scratch reset; 4. joint input of this
+  // step (its loads overlap the records); 5. the fusion bias row
   const int nl = s_lm_len, nt = s_tr_len;
-  if (tid < nl) {
-    const int st = s_lm[tid];
-    s_lb[tid] = __ldg(d.lm.st_begin + st);
-    s_lc[tid] = __ldg(d.lm.st_count + st);
-    s_lo[tid] = __ldg(d.lm.st_cum + st);
-  } else if (tid >= 32 && tid - 32 < nt) {
-    const int q = s_tr[tid - 32];
-    s_tb[tid - 32] = __ldg(d.tr.nd_begin + q);
-    s_tc[tid - 32] = __ldg(d.tr.nd_count + q);
-    s_td[tid - 32] = __ldg(d.tr.nd_depth + q) + 1;
-  }
-  for (int v = tid; v < V; v += kRowThreads) {
-    lmkey[v] = 0ull;
-    dep[v] = 0;
-  }
-
-  // 4. joint input of this step (its loads overlap the records above)
-  {
-    const int H = d.H;
-    const uint4* e = reinterpret_cast<const uint4*>(P->enc + ((size_t)r * T + t) * H);
-    const uint4* g = reinterpret_cast<const uint4*>(d.E + (size_t)s_last * H);
-    uint4* a = reinterpret_cast<uint4*>(d.A + (size_t)r * H);
-    for (int i = tid; i < H / 8; i += kRowThreads) {
-      uint4 x = __ldg(e + i), z = __ldg(g + i);
-      const __nv_bfloat162* xa = reinterpret_cast<const __nv_bfloat162*>(&x);
-      const __nv_bfloat162* za = reinterpret_cast<const __nv_bfloat162*>(&z);
-      uint4 out;
-      __nv_bfloat162* oa = reinterpret_cast<__nv_bfloat162*>(&out);
-#pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        float2 xf = __bfloat1622float2(xa[q]);
-        float2 zf = __bfloat1622float2(za[q]);
-        float lo = fmaxf(xf.x + zf.x, 0.f), hi = fmaxf(xf.y + zf.y, 0.f);
-        oa[q] = __floats2bfloat162_rn(lo, hi);
-      }
-      a[i] = out;
-    }
-  }
-  __syncthreads();
-
-  // 5. fusion bias of this step: every chain level at once; a label's LM
-  //    score comes from the deepest level that continues with it (max of
-  //    level << 32 | value bits), its goto depth from the deepest trie node
-  //    that has it as a child (max of the child's depth)
-  const float cum_top = nl ? s_lo[nl - 1] : 0.f;
-  for (int l = 0; l < nl; ++l) {
-    const int b = s_lb[l], c = s_lc[l];
-    const float off = cum_top - s_lo[l];
-    const unsigned long long lev = (unsigned long long)(l + 1) << 32;
-    for (int j = tid; j < c; j += kRowThreads) {
-      const int w = __ldg(d.lm.arc_tok + b + j);
-      const float val = off + __ldg(d.lm.arc_logp + b + j);
-      atomicMax(lmkey + w, lev | (unsigned long long)__float_as_uint(val));
-    }
-  }
-  for (int k = 0; k < nt; ++k) {
-    const int b = s_tb[k], c = s_tc[k], dd = s_td[k];
-    for (int j = tid; j < c; j += kRowThreads) atomicMax(dep + __ldg(d.tr.ch_tok + b + j), dd);
-  }
-  __syncthreads();
-  const int depth_cur = nt ? s_td[0] - 1 : 0;
-  const float lam = P->lambda, beta = P->beta;
-  float* brow = d.bias + (size_t)r * d.N_pad;
-  const float bscale = beta * (d.has_tr ? d.tr.bonus : 0.f);
-  for (int v = tid; v < V; v += kRowThreads) {
-    float b = 0.f;
-    if (d.has_lm) {
-      const unsigned long long k = lmkey[v];
-      const float l = k ? __uint_as_float((unsigned)k) : cum_top + __ldg(d.lm.uni_logp + v);
-      b = lam * l;
-    }
-    if (d.has_tr) {
-      int dd = dep[v];
-      if (dd == 0) dd = (__ldg(d.tr.root_child + v) != 0) ? 1 : 0;
-      b += bscale * (float)(dd - depth_cur);
-    }
-    brow[v] = b;
-  }
-  if (tid == 0) brow[V] = 0.f;
+  row::bias_prepare(d, s_lm, nl, s_tr, nt, rc, lmkey, dep);
+  row::build_joint_input(d, P->enc + ((size_t)r * T + t) * d.H, s_last, r);
+  row::bias_finish(d, nl, nt, rc, P->lambda, P->beta, d.bias + (size_t)r * d.N_pad, lmkey, dep);
   if (mode == 2 && tid == 0) {
     // Algorithmic bytes of this row-step: selection partials, row state,
     // the searches of the emitted label (one probe per halving plus the arc
@@ -328,11 +222,11 @@ __global__ void __launch_bounds__(kRowThreads) k_row(DecView d, int step, int mo
     // epilogue and the shared unigram/root rows are not counted here.
     unsigned long long bytes = (unsigned long long)d.n_ptiles * 16 + 2ull * (24 + 4 * (nl + nt));
     bytes += 6ull * d.H;
-    for (int l = 0; l < nl; ++l) bytes += 12 + 8ull * s_lc[l];
-    for (int k = 0; k < nt; ++k) bytes += 12 + 4ull * s_tc[k];
+    for (int l = 0; l < nl; ++l) bytes += 12 + 8ull * rc.lc[l];
+    for (int k = 0; k < nt; ++k) bytes += 12 + 4ull * rc.tc[k];
     if (s_y != V && evaluated) {
-      for (int l = 0; l < nl; ++l) bytes += 8 + 4ull * (32 - __clz(s_lc[l] + 1)) + 4;
-      for (int k = 0; k < nt; ++k) bytes += 8 + 4ull * (32 - __clz(s_tc[k] + 1)) + 8;
+      for (int l = 0; l < nl; ++l) bytes += 8 + 4ull * (32 - __clz(rc.lc[l] + 1)) + 4;
+      for (int k = 0; k < nt; ++k) bytes += 8 + 4ull * (32 - __clz(rc.tc[k] + 1)) + 8;
     }
     atomicAdd(d.ctr, bytes);
   }

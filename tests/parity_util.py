@@ -64,7 +64,8 @@ class GpuRun:
         self.lm = tsd.NGram.from_arrays(inp.lmA) if inp.lmA is not None else None
         self.bo = tsd.Boost.from_phrases(w.V, inp.ph, w.bonus) if inp.ph is not None else None
         n = len(self.streams)
-        self.dec = tsd.Decoder(w.V, w.H, Wt, Et, lm=self.lm, boost=self.bo, max_symbols=w.max_sym, beam_k=1,
+        self.K = w.beam
+        self.dec = tsd.Decoder(w.V, w.H, Wt, Et, lm=self.lm, boost=self.bo, max_symbols=w.max_sym, beam_k=w.beam,
                                max_streams=n, max_T=self.T)
         self.dec.set_graphs(graphs)
         if joint_kind:
@@ -73,10 +74,13 @@ class GpuRun:
             self.dec.set_option(k, v)
         self.slots = [self.dec.open() for _ in range(n)]
         self.cap_logits = self.cap_rows = None
+        M = n * self.K
         if capture_steps:
-            self.cap_logits = torch.zeros((capture_steps, n, w.N), dtype=torch.float32, device=dev)
-            self.cap_rows = torch.full((capture_steps, n, 4), -7, dtype=torch.int32, device=dev)
+            self.cap_logits = torch.zeros((capture_steps, M, w.N), dtype=torch.float32, device=dev)
+            self.cap_rows = torch.full((capture_steps, M, 4), -7, dtype=torch.int32, device=dev)
             self.dec.debug_capture(self.cap_logits, self.cap_rows, capture_steps)
+        self.beam_sel: List[np.ndarray] = []   # per chunk: kept candidates [T, M, 4]
+        self.beam_hyps: List[List] = []        # per chunk: per stream [(labels, score)]
         self.chunks: List[Dict] = []
         self.enc: List[np.ndarray] = []
         self.states: List[List] = []
@@ -90,6 +94,10 @@ class GpuRun:
             self.chunks.append({"count": cnt, "tok": tok, "frame": fr, "score": sc})
             self.enc.append(enc)
             self.states.append([self.dec.state(s) for s in self.slots])
+            if self.K > 1:
+                if capture_steps:
+                    self.beam_sel.append(self.cap_rows.cpu().numpy().copy())
+                self.beam_hyps.append([self.dec.hyps(s) for s in self.slots])
             if between_chunks is not None:
                 between_chunks(self.dec)
         self.dec.check()  # no bounded device wait expired
@@ -156,3 +164,50 @@ def assert_reports(reps: List[Dict]):
         assert r["max_score_diff"] <= SCORE_TOL, r
         assert not r["state_errors"], r["state_errors"][:5]
         assert r["steps"] > 0
+
+
+def replay_beam_stream(inp: Inputs, run: GpuRun, i: int, olm, obo, model) -> Dict:
+    """Oracle replay of the i-th stream of a beam run: every frame's kept
+    candidates are checked and followed; after every chunk the surviving
+    label sequences must be the oracle's, in the same order, with scores
+    within SCORE_TOL per frame decoded so far."""
+    w = inp.w
+    K = w.beam
+    st = oracle.Stream(w.V)
+    out = {"steps": 0, "mismatch": 0, "near_tie": 0, "max_score_diff": 0.0, "inconsistent": 0, "state_errors": []}
+    frames = 0
+    for c in range(len(run.chunks)):
+        sel = run.beam_sel[c][:, i * K:(i + 1) * K, :]  # [T, K, 4]
+        rep = oracle.beam_chunk_follow(st, model, olm, obo, run.enc[c][i], inp.lam, inp.beta, K,
+                                       sel[:, :, 0], sel[:, :, 1], sel[:, :, 2].view(np.float32), GAP_TOL)
+        frames += run.T
+        out["steps"] += int(rep[oracle.REP_STEPS])
+        out["mismatch"] += int(rep[oracle.REP_MISMATCH])
+        out["near_tie"] += int(rep[oracle.REP_NEAR_TIE])
+        out["inconsistent"] += int(rep[oracle.REP_INCONSISTENT])
+        out["max_score_diff"] = max(out["max_score_diff"], float(rep[oracle.REP_MAX_SCORE_DIFF]))
+        want = st.beam_hyps(with_rho=True)
+        got = run.beam_hyps[c][i]
+        if [g[0] for g in got] != [h[0] for h in want]:
+            out["state_errors"].append((c, "hyp sequences", len(got), len(want)))
+            continue
+        for (gy, gs), (wy, ws, _) in zip(got, want):
+            if abs(gs - ws) > SCORE_TOL * frames:
+                out["state_errors"].append((c, "hyp score", gs, ws))
+        # the first hypothesis's LM state and trie node
+        lm_state, trie_node, last = run.states[c][i]
+        wy, _, wrho = want[0]
+        if last != (wy[-1] if wy else w.V):
+            out["state_errors"].append((c, "last", last))
+        if olm is not None and run.lm.state_tuple(lm_state) != olm.state(wy):
+            out["state_errors"].append((c, "lm"))
+        if obo is not None and run.bo.node_tuple(trie_node) != trie_tuple(obo, wy, wrho):
+            out["state_errors"].append((c, "trie"))
+    return out
+
+
+def replay_beam(inp: Inputs, run: GpuRun, sample: Sequence[int], threads: Optional[int] = None) -> List[Dict]:
+    olm, obo, model = oracle_models(inp)
+    threads = threads or min(len(sample), os.cpu_count() or 4)
+    with concurrent.futures.ThreadPoolExecutor(max_workers=threads) as ex:
+        return list(ex.map(lambda i: replay_beam_stream(inp, run, i, olm, obo, model), sample))

@@ -99,6 +99,35 @@ def test_cfg2_sampled_parity_full_size():
     assert any(run.states[c][i][1] != 0 for c in range(w.chunks) for i in range(w.B))
 
 
+def test_cfg3_beam_parity():
+    """Beam search, K=4, one label per frame: every frame's kept candidates
+    are the oracle's top K (up to near ties), each candidate's score
+    increment is within 1e-4, merges and surviving label sequences are the
+    oracle's, in order, over all 40 chunks of 3 sampled streams."""
+    w = synth.WORKLOADS[3]
+    inp = pu.Inputs(w)
+    run = pu.GpuRun(inp, range(w.B), w.chunks, capture_steps=w.T)
+    reps = pu.replay_beam(inp, run, [0, 63, 127])
+    pu.assert_reports(reps)
+    assert all(len(run.beam_hyps[-1][i]) >= 1 for i in range(w.B))
+    # merges happen: some frame keeps fewer than K hypotheses
+    assert any(len(h) < w.beam for c in run.beam_hyps for h in c)
+
+
+def test_beam_small_exhaustive_against_free_oracle():
+    """Tiny beam (V=15, H=64, K=3..8) against the free-running oracle's beam,
+    including the K = 8 limit and a stream with no LM or boost."""
+    for K in (3, 8):
+        w = synth.scaled(synth.WORKLOADS[0], V=15, H=64, B=5, T=9, beam=K, max_sym=1, lm_total=60)
+        inp = pu.Inputs(w, lmA=synth.ngram_lm(7, 15, 3, 60, 1.1), ph=synth.phrases(7, 15, 3, 1, 3, 0.0))
+        run = pu.GpuRun(inp, range(w.B), 3, capture_steps=w.T)
+        pu.assert_reports(pu.replay_beam(inp, run, range(w.B)))
+    w = synth.scaled(synth.WORKLOADS[0], V=15, H=64, B=2, T=6, beam=4, max_sym=1)
+    inp = pu.Inputs(w, with_lm=False, with_boost=False)
+    run = pu.GpuRun(inp, range(w.B), 2, capture_steps=w.T)
+    pu.assert_reports(pu.replay_beam(inp, run, range(w.B)))
+
+
 def _tokens(run, i):
     return np.concatenate([run.emitted(i, c)[0] for c in range(len(run.chunks))])
 

@@ -353,3 +353,66 @@ def test_beam_sums_alignments_exhaustively():
     assert set(got) == set(want)
     for k in want:
         assert abs(got[k] - want[k]) < 1e-9, k
+
+
+def _brute_selections(model, lm, bo, enc, lam, beta, K):
+    """Top-K kept candidates per frame by (score desc, hypothesis, label),
+    from fused rows of each hypothesis: an independent driver of the beam."""
+    V = model.V
+    hyps = [([], 0.0, 0)]
+    sels = []
+    for t in range(enc.shape[0]):
+        cands = []
+        for i, (y, sc, rho) in enumerate(hyps):
+            st = oracle.Stream(V)
+            st.set_history(y, rho)
+            f = oracle.fused_row(st, model, lm, bo, enc[t], lam, beta)
+            cands += [(sc + f[v], i, v) for v in range(V + 1)]
+        cands.sort(key=lambda c: (-c[0], c[1], c[2]))
+        kept = cands[:K]
+        sels.append(kept)
+        nxt = []
+        for sc, i, v in kept:
+            y, _, rho = hyps[i]
+            y2 = y + ([v] if v != V else [])
+            rho2 = int(bo.trajectory(y2)[1][-1]) if y2 else 0
+            for j, (yy, ss, rr) in enumerate(nxt):
+                if yy == y2:
+                    nxt[j] = (yy, float(np.logaddexp(ss, sc)), rr)
+                    break
+            else:
+                nxt.append((y2, sc, rho2))
+        hyps = nxt
+    return sels, hyps
+
+
+def test_beam_follow_mode():
+    """Following the brute-force selections reproduces the free-running beam
+    with no flagged frame; a selection that drops a clearly better candidate
+    is flagged."""
+    V, H, T, K = 6, 16, 5, 3
+    model, _ = _tiny_model(V=V, H=H, seed=12)
+    lm = oracle.LM.from_arrays(synth.ngram_lm(12, V, 3, 40, 1.1))
+    bo = oracle.Boost(V, np.array([0, 2, 3]), np.array([1, 2, 4]), 1.0)
+    enc = synth.normal_bf16(12, 1, 0, 0, T * H, 1.0).reshape(T, H)
+    sels, hyps = _brute_selections(model, lm, bo, enc, 0.4, 0.8, K)
+    free = oracle.Stream(V)
+    oracle.beam_chunk(free, model, lm, bo, enc, 0.4, 0.8, K)
+    got = free.beam_hyps()
+    assert [h[0] for h in got] == [h[0] for h in hyps]
+    for (ya, sa), (yb, sb, _) in zip(got, hyps):
+        assert abs(sa - sb) < 1e-9
+    sh = np.array([[c[1] for c in s] for s in sels], dtype=np.int32)
+    stok = np.array([[c[2] for c in s] for s in sels], dtype=np.int32)
+    sinc = np.zeros_like(sh, dtype=np.float32)
+    fol = oracle.Stream(V)
+    rep = oracle.beam_chunk_follow(fol, model, lm, bo, enc, 0.4, 0.8, K, sh, stok, sinc)
+    assert rep[oracle.REP_MISMATCH] == 0 and rep[oracle.REP_INCONSISTENT] == 0
+    assert [h[0] for h in fol.beam_hyps()] == [h[0] for h in got]
+    # keep the worst candidate of hypothesis 0 instead of the best one at frame 0
+    bad_tok = stok.copy()
+    st0 = oracle.Stream(V)
+    f0 = oracle.fused_row(st0, model, lm, bo, enc[0], 0.4, 0.8)
+    bad_tok[0, 0] = int(np.argmin(f0))
+    rep = oracle.beam_chunk_follow(oracle.Stream(V), model, lm, bo, enc, 0.4, 0.8, K, sh, bad_tok, sinc)
+    assert rep[oracle.REP_MISMATCH] >= 1
