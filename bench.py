@@ -379,13 +379,17 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--config", type=int, default=2)
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--cpu-streams", type=int, default=256)
-    ap.add_argument("--cpu-chunks", type=int, default=6)
+    ap.add_argument("--cpu-streams", type=int, default=None)
+    ap.add_argument("--cpu-chunks", type=int, default=None)
     ap.add_argument("--ref-streams", type=int, default=64)
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
     w = synth.WORKLOADS[args.config]
+    # bounded CPU samples (about 10-30 s of oracle work on 16 cores)
+    cpu_default = {0: (4, 1), 1: (64, 12), 2: (256, 6), 3: (64, 2), 4: (32, 1)}[args.config]
+    args.cpu_streams = args.cpu_streams or cpu_default[0]
+    args.cpu_chunks = args.cpu_chunks or cpu_default[1]
     if args.impl == "reference":
         run_reference(args, w)
     else:

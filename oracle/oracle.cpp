@@ -244,18 +244,25 @@ ORACLE_API void* oracle_lm_new(int32_t V, int32_t order, const int64_t* count,
   d->bow.resize((size_t)order);
   for (int k = 1; k <= order; ++k) {
     int64_t n = count[k - 1];
-    std::vector<int64_t> idx((size_t)n);
-    for (int64_t i = 0; i < n; ++i) idx[(size_t)i] = i;
     const int32_t* t = tokens[k - 1];
-    std::sort(idx.begin(), idx.end(), [&](int64_t a, int64_t b) {
-      return std::lexicographical_compare(t + a * k, t + a * k + k, t + b * k, t + b * k + k);
-    });
+    // sort the tuples (unless they already come sorted)
+    bool sorted = true;
+    for (int64_t i = 1; i < n && sorted; ++i)
+      sorted = std::lexicographical_compare(t + (i - 1) * k, t + i * k, t + i * k, t + i * k + k);
+    std::vector<int64_t> idx;
+    if (!sorted) {
+      idx.resize((size_t)n);
+      for (int64_t i = 0; i < n; ++i) idx[(size_t)i] = i;
+      std::sort(idx.begin(), idx.end(), [&](int64_t a, int64_t b) {
+        return std::lexicographical_compare(t + a * k, t + a * k + k, t + b * k, t + b * k + k);
+      });
+    }
     std::vector<int32_t>& dt = d->toks[(size_t)k - 1];
     dt.resize((size_t)n * k);
     d->logp[(size_t)k - 1].resize((size_t)n);
     d->bow[(size_t)k - 1].resize((size_t)n);
     for (int64_t j = 0; j < n; ++j) {
-      int64_t i = idx[(size_t)j];
+      int64_t i = sorted ? j : idx[(size_t)j];
       for (int q = 0; q < k; ++q) {
         int32_t tok = t[i * k + q];
         if (tok < 0 || tok >= V) { delete d; return nullptr; }

@@ -461,9 +461,9 @@ void launch_row_beam(const DecView& d, int n, int step, int mode, size_t smem, c
 void launch_open_beam(const DecView& d, int slot, cudaStream_t s) { k_open_beam<<<1, 32, 0, s>>>(d, slot); }
 
 cudaError_t prepare_beam_kernels(size_t row_smem) {
-  if (row_smem > 48 * 1024)
-    return cudaFuncSetAttribute(k_row_beam, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)row_smem);
-  return cudaSuccess;
+  // dynamic scratch plus the kernel's static shared memory may pass the
+  // 48 KB default even when the scratch alone does not
+  return cudaFuncSetAttribute(k_row_beam, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)row_smem);
 }
 
 }  // namespace tsd

@@ -260,9 +260,9 @@ __global__ void k_repack(const uint16_t* __restrict__ W, uint16_t* __restrict__ 
 size_t row_smem_bytes(int V4) { return (size_t)V4 * (sizeof(unsigned long long) + sizeof(int)); }
 
 cudaError_t prepare_kernels(size_t row_smem) {
-  if (row_smem > 48 * 1024)
-    return cudaFuncSetAttribute(k_row, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)row_smem);
-  return cudaSuccess;
+  // dynamic scratch plus the kernel's static shared memory may pass the
+  // 48 KB default even when the scratch alone does not
+  return cudaFuncSetAttribute(k_row, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)row_smem);
 }
 
 void launch_repack(const uint16_t* W, uint16_t* Wt, int H, int N, int N_pad, cudaStream_t s) {

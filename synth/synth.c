@@ -306,6 +306,49 @@ static int order_alloc(order_t* o, int64_t n) {
              : -1;
 }
 
+#include <pthread.h>
+#include <unistd.h>
+
+typedef void (*range_fn)(void* arg, int64_t b, int64_t e);
+typedef struct {
+  range_fn fn;
+  void* arg;
+  int64_t b, e;
+} range_task_t;
+
+static void* range_thread(void* p) {
+  range_task_t* t = (range_task_t*)p;
+  t->fn(t->arg, t->b, t->e);
+  return NULL;
+}
+
+/* fn over [0, n) split across the online cores (at most 32 threads). */
+static void run_parallel(int64_t n, range_fn fn, void* arg) {
+  long nt = sysconf(_SC_NPROCESSORS_ONLN);
+  if (nt < 1) nt = 1;
+  if (nt > 32) nt = 32;
+  if (n < 4096 || nt == 1) {
+    fn(arg, 0, n);
+    return;
+  }
+  pthread_t th[32];
+  range_task_t tk[32];
+  int64_t chunk = (n + nt - 1) / nt;
+  int started = 0;
+  for (long t = 0; t < nt; ++t) {
+    int64_t b = t * chunk, e = b + chunk < n ? b + chunk : n;
+    if (b >= e) break;
+    tk[t].fn = fn; tk[t].arg = arg; tk[t].b = b; tk[t].e = e;
+    if (pthread_create(&th[t], NULL, range_thread, &tk[t]) != 0) {
+      fn(arg, b, e);
+      tk[t].fn = NULL;
+    }
+    started = (int)t + 1;
+  }
+  for (int t = 0; t < started; ++t)
+    if (tk[t].fn) pthread_join(th[t], NULL);
+}
+
 /* candidate range of context i at order k (k>=2): the continuations of its
  * suffix g[1:], which live in the order-(k-1) list (all V unigrams at k=2) */
 static void cand_range(const synth_lm_t* m, int k, int64_t i, int64_t* b, int64_t* e) {
@@ -352,6 +395,34 @@ static int64_t total_for(double c, const double* pi, const int64_t* cap, int64_t
   return s;
 }
 
+typedef struct {
+  double c;
+  const double* pi;
+  const int64_t* cap;
+  int64_t part[64];
+  int64_t chunk;
+} total_job_t;
+
+static void total_range(void* arg, int64_t b, int64_t e) {
+  total_job_t* J = (total_job_t*)arg;
+  J->part[b / J->chunk] = total_for(J->c, J->pi + b, J->cap + b, e - b);
+}
+
+static int64_t total_par(double c, const double* pi, const int64_t* cap, int64_t nctx) {
+  if (nctx < 4096) return total_for(c, pi, cap, nctx);
+  long nt = sysconf(_SC_NPROCESSORS_ONLN);
+  if (nt < 1) nt = 1;
+  if (nt > 32) nt = 32;
+  total_job_t J;
+  memset(&J, 0, sizeof(J));
+  J.c = c; J.pi = pi; J.cap = cap;
+  J.chunk = (nctx + nt - 1) / nt;
+  run_parallel(nctx, total_range, &J);
+  int64_t s = 0;
+  for (int t = 0; t < 64; ++t) s += J.part[t];
+  return s;
+}
+
 /* Efraimidis-Spirakis weighted sampling without replacement: keys
  * ln(u)/w, keep the n largest.  Writes the chosen indices to out. */
 static void draw_es(const rng_t* r, uint32_t draw0, const double* p, int64_t b, int64_t e, int64_t n,
@@ -365,6 +436,140 @@ static void draw_es(const rng_t* r, uint32_t draw0, const double* p, int64_t b, 
   }
   qsort(es, (size_t)range, sizeof(es_t), cmp_es_desc);
   for (int64_t j = 0; j < n; ++j) out[j] = es[j].idx;
+}
+
+typedef struct {
+  synth_lm_t* m;
+  int k;
+} tuple_job_t;
+
+static void tuple_range(void* arg, int64_t x0, int64_t x1) {
+  tuple_job_t* J = (tuple_job_t*)arg;
+  const int k = J->k;
+  const order_t* o = &J->m->ord[k - 1];
+  for (int64_t x = x0; x < x1; ++x) {
+    int32_t* dst = J->m->tuples[k - 1] + (size_t)x * k;
+    if (k > 1) memcpy(dst, J->m->tuples[k - 2] + (size_t)o->ctx[x] * (k - 1), sizeof(int32_t) * (k - 1));
+    dst[k - 1] = o->tok[x];
+  }
+}
+
+typedef struct {
+  synth_lm_t* m;
+  int k;
+  uint64_t seed;
+  double discount, c;
+  const int64_t* caps;
+  const int64_t* start;
+  double z_root;
+  int failed;
+} gen_job_t;
+
+/* Draws the continuations of contexts [i0, i1) of order k-1. */
+static void gen_contexts(void* arg, int64_t i0, int64_t i1) {
+  gen_job_t* J = (gen_job_t*)arg;
+  synth_lm_t* m = J->m;
+  const int k = J->k;
+  const double discount = J->discount, c = J->c, z_root = J->z_root;
+  const uint64_t seed = J->seed;
+  const int32_t V = m->V;
+  order_t* ctxo = &m->ord[k - 2];
+  const order_t* lower = &m->ord[k - 2];
+  order_t* o = &m->ord[k - 1];
+  const int64_t* caps = J->caps;
+  int64_t* chosen = NULL;
+  es_t* es = NULL;
+  size_t chosen_cap = 0;
+  (void)V;
+  for (int64_t i = i0; i < i1; ++i) {
+    const int64_t pos = J->start[i];
+        int64_t b, e;
+        cand_range(m, k, i, &b, &e);
+        int64_t n = n_for(c, ctxo->pi[i], caps[i]);
+        ctxo->ch_begin[i] = pos;
+        ctxo->ch_count[i] = n;
+        /* total stored mass of the suffix context g[1:] */
+        double z_sfx = (k == 2) ? z_root : m->ord[k - 3].Z[ctxo->sfx[i]];
+        if (n == 0) {
+          ctxo->Z[i] = z_sfx; /* no continuations, no backoff weight */
+          continue;
+        }
+        int64_t range = e - b;
+        if ((size_t)range > chosen_cap) {
+          chosen_cap = (size_t)range;
+          free(chosen); free(es);
+          chosen = malloc(sizeof(int64_t) * chosen_cap);
+          es = malloc(sizeof(es_t) * chosen_cap);
+          if (!chosen || !es) { J->failed = 1; free(chosen); free(es); return; }
+        }
+        rng_t r = rng_make(seed, 0x6C6D0000u | (uint32_t)k, (uint32_t)i, (uint32_t)((uint64_t)i >> 32));
+        if (n == range) {
+          for (int64_t j = 0; j < range; ++j) chosen[j] = b + j;
+        } else if (n * 8 >= range) {
+          draw_es(&r, 0, lower->p, b, e, n, es, chosen);
+        } else {
+          /* successive sampling by inverse CDF over the candidates' running
+           * sum (which restarts at b), rejecting repeats */
+          const double* cum = lower->cum;
+          double tot = cum[e - 1];
+          uint32_t d = 0x10000u;
+          uint32_t tries = 0;
+          int64_t got = 0;
+          while (got < n && tries < (uint32_t)(n * 64 + 64)) {
+            uint32_t w4[4];
+            rng_draw(&r, d++, w4);
+            for (int q = 0; q < 4 && got < n; ++q) {
+              ++tries;
+              double tgt = u01(w4[q]) * tot;
+              int64_t lo = b, hi = e - 1;
+              while (lo < hi) {
+                int64_t mid = lo + (hi - lo) / 2;
+                if (cum[mid] < tgt) lo = mid + 1; else hi = mid;
+              }
+              int dup = 0;
+              for (int64_t j = 0; j < got; ++j)
+                if (chosen[j] == lo) { dup = 1; break; }
+              if (!dup) chosen[got++] = lo;
+            }
+          }
+          if (got < n) draw_es(&r, 0x20000u, lower->p, b, e, n, es, chosen);
+        }
+        qsort(chosen, (size_t)n, sizeof(int64_t), cmp_i64);
+        /* counts 1 + Geometric(1/2): trailing ones of a 64-bit word */
+        int64_t csum = 0;
+        uint32_t w4[4];
+        for (int64_t j = 0; j < n; ++j) {
+          if ((j & 1) == 0) rng_draw(&r, 0x40000u + (uint32_t)(j >> 1), w4);
+          uint64_t bits = ((uint64_t)w4[(j & 1) * 2] << 32) | w4[(j & 1) * 2 + 1];
+          int32_t g = 0;
+          while ((bits & 1u) && g < 63) { ++g; bits >>= 1; }
+          o->count[pos + j] = 1 + g;
+          csum += 1 + g;
+        }
+        double lower_mass = 0, kept = 0;
+        for (int64_t j = 0; j < n; ++j) {
+          int64_t cidx = chosen[j];
+          int64_t x = pos + j;
+          o->tok[x] = lower->tok[cidx];
+          o->ctx[x] = i;
+          o->sfx[x] = cidx; /* the suffix g[1:]·w is the candidate itself */
+          double p = ((double)o->count[x] - discount) / (double)csum;
+          o->logp[x] = (float)log(p);
+          o->p[x] = exp((double)o->logp[x]);
+          o->pi[x] = ctxo->pi[i] * o->p[x];
+          kept += o->p[x];
+          lower_mass += lower->p[cidx];
+        }
+        /* the backoff weight spreads 1 - kept over the tokens g does not
+         * continue, whose stored mass under g[1:] is z_sfx - lower_mass; the
+         * context's resulting total is recorded for the next order */
+        ctxo->bow[i] = (float)log((1.0 - kept) / (z_sfx - lower_mass));
+        ctxo->Z[i] = kept + exp((double)ctxo->bow[i]) * (z_sfx - lower_mass);
+        double acc = 0;
+        for (int64_t j = 0; j < n; ++j) { acc += o->p[pos + j]; o->cum[pos + j] = acc; }
+  }
+  free(chosen);
+  free(es);
 }
 
 SYNTH_API synth_lm_t* synth_lm_new(uint64_t seed, int32_t V, int32_t N, int64_t total,
@@ -424,18 +629,14 @@ SYNTH_API synth_lm_t* synth_lm_new(uint64_t seed, int32_t V, int32_t N, int64_t 
   /* Z of the empty context: the stored unigram mass */
   double z_root = o1->cum[V - 1];
 
-  int64_t* chosen = NULL;
-  es_t* es = NULL;
   int64_t* caps = NULL;
-  size_t chosen_cap = 0;
 
   for (int k = 2; k <= N; ++k) {
     order_t* ctxo = &m->ord[k - 2];      /* contexts: order k-1 */
-    const order_t* lower = &m->ord[k - 2]; /* candidates: order k-1 (children of g[1:]) */
     int64_t nctx = ctxo->n;
     free(caps);
     caps = malloc(sizeof(int64_t) * (size_t)(nctx > 0 ? nctx : 1));
-    if (!caps) { free(chosen); free(es); synth_lm_free(m); return NULL; }
+    if (!caps) { synth_lm_free(m); return NULL; }
     int64_t maxn = 0;
     for (int64_t i = 0; i < nctx; ++i) {
       int64_t b, e;
@@ -446,113 +647,34 @@ SYNTH_API synth_lm_t* synth_lm_new(uint64_t seed, int32_t V, int32_t N, int64_t 
     int64_t want = target[k] < maxn ? target[k] : maxn;
     /* bracket, then bisect the scale c so the order meets its budget (1%) */
     double lo_c = 0, hi_c = 1;
-    for (int it = 0; it < 200 && total_for(hi_c, ctxo->pi, caps, nctx) < want; ++it) {
+    for (int it = 0; it < 200 && total_par(hi_c, ctxo->pi, caps, nctx) < want; ++it) {
       lo_c = hi_c;
       hi_c *= 2;
     }
     double c = hi_c;
     for (int it = 0; it < 100; ++it) {
       double mid = 0.5 * (lo_c + hi_c);
-      int64_t s = total_for(mid, ctxo->pi, caps, nctx);
+      int64_t s = total_par(mid, ctxo->pi, caps, nctx);
       c = mid;
       if ((double)llabs(s - want) <= 0.01 * (double)want) break;
       if (s < want) lo_c = mid; else hi_c = mid;
     }
-    int64_t nk = total_for(c, ctxo->pi, caps, nctx);
+    int64_t nk = total_par(c, ctxo->pi, caps, nctx);
     order_t* o = &m->ord[k - 1];
-    if (order_alloc(o, nk)) { free(caps); free(chosen); free(es); synth_lm_free(m); return NULL; }
-    int64_t pos = 0;
-    for (int64_t i = 0; i < nctx; ++i) {
-      int64_t b, e;
-      cand_range(m, k, i, &b, &e);
-      int64_t n = n_for(c, ctxo->pi[i], caps[i]);
-      ctxo->ch_begin[i] = pos;
-      ctxo->ch_count[i] = n;
-      /* total stored mass of the suffix context g[1:] */
-      double z_sfx = (k == 2) ? z_root : m->ord[k - 3].Z[ctxo->sfx[i]];
-      if (n == 0) {
-        ctxo->Z[i] = z_sfx; /* no continuations, no backoff weight */
-        continue;
-      }
-      int64_t range = e - b;
-      if ((size_t)range > chosen_cap) {
-        chosen_cap = (size_t)range;
-        free(chosen); free(es);
-        chosen = malloc(sizeof(int64_t) * chosen_cap);
-        es = malloc(sizeof(es_t) * chosen_cap);
-        if (!chosen || !es) { free(caps); free(chosen); free(es); synth_lm_free(m); return NULL; }
-      }
-      rng_t r = rng_make(seed, 0x6C6D0000u | (uint32_t)k, (uint32_t)i, (uint32_t)((uint64_t)i >> 32));
-      if (n == range) {
-        for (int64_t j = 0; j < range; ++j) chosen[j] = b + j;
-      } else if (n * 8 >= range) {
-        draw_es(&r, 0, lower->p, b, e, n, es, chosen);
-      } else {
-        /* successive sampling by inverse CDF over the candidates' running
-         * sum (which restarts at b), rejecting repeats */
-        const double* cum = lower->cum;
-        double tot = cum[e - 1];
-        uint32_t d = 0x10000u;
-        uint32_t tries = 0;
-        int64_t got = 0;
-        while (got < n && tries < (uint32_t)(n * 64 + 64)) {
-          uint32_t w4[4];
-          rng_draw(&r, d++, w4);
-          for (int q = 0; q < 4 && got < n; ++q) {
-            ++tries;
-            double tgt = u01(w4[q]) * tot;
-            int64_t lo = b, hi = e - 1;
-            while (lo < hi) {
-              int64_t mid = lo + (hi - lo) / 2;
-              if (cum[mid] < tgt) lo = mid + 1; else hi = mid;
-            }
-            int dup = 0;
-            for (int64_t j = 0; j < got; ++j)
-              if (chosen[j] == lo) { dup = 1; break; }
-            if (!dup) chosen[got++] = lo;
-          }
-        }
-        if (got < n) draw_es(&r, 0x20000u, lower->p, b, e, n, es, chosen);
-      }
-      qsort(chosen, (size_t)n, sizeof(int64_t), cmp_i64);
-      /* counts 1 + Geometric(1/2): trailing ones of a 64-bit word */
-      int64_t csum = 0;
-      uint32_t w4[4];
-      for (int64_t j = 0; j < n; ++j) {
-        if ((j & 1) == 0) rng_draw(&r, 0x40000u + (uint32_t)(j >> 1), w4);
-        uint64_t bits = ((uint64_t)w4[(j & 1) * 2] << 32) | w4[(j & 1) * 2 + 1];
-        int32_t g = 0;
-        while ((bits & 1u) && g < 63) { ++g; bits >>= 1; }
-        o->count[pos + j] = 1 + g;
-        csum += 1 + g;
-      }
-      double lower_mass = 0, kept = 0;
-      for (int64_t j = 0; j < n; ++j) {
-        int64_t cidx = chosen[j];
-        int64_t x = pos + j;
-        o->tok[x] = lower->tok[cidx];
-        o->ctx[x] = i;
-        o->sfx[x] = cidx; /* the suffix g[1:]·w is the candidate itself */
-        double p = ((double)o->count[x] - discount) / (double)csum;
-        o->logp[x] = (float)log(p);
-        o->p[x] = exp((double)o->logp[x]);
-        o->pi[x] = ctxo->pi[i] * o->p[x];
-        kept += o->p[x];
-        lower_mass += lower->p[cidx];
-      }
-      /* the backoff weight spreads 1 - kept over the tokens g does not
-       * continue, whose stored mass under g[1:] is z_sfx - lower_mass; the
-       * context's resulting total is recorded for the next order */
-      ctxo->bow[i] = (float)log((1.0 - kept) / (z_sfx - lower_mass));
-      ctxo->Z[i] = kept + exp((double)ctxo->bow[i]) * (z_sfx - lower_mass);
-      double acc = 0;
-      for (int64_t j = 0; j < n; ++j) { acc += o->p[pos + j]; o->cum[pos + j] = acc; }
-      pos += n;
-    }
+    if (order_alloc(o, nk)) { free(caps); synth_lm_free(m); return NULL; }
+    /* output positions, then every context in parallel (each context's
+     * draws come from its own counter-based stream, so the result does not
+     * depend on the thread count) */
+    int64_t* start = malloc(sizeof(int64_t) * (size_t)(nctx + 1));
+    if (!start) { free(caps); synth_lm_free(m); return NULL; }
+    start[0] = 0;
+    for (int64_t i = 0; i < nctx; ++i) start[i + 1] = start[i] + n_for(c, ctxo->pi[i], caps[i]);
+    gen_job_t job = {m, k, seed, discount, c, caps, start, z_root, 0};
+    run_parallel(nctx, gen_contexts, &job);
+    free(start);
+    if (job.failed) { free(caps); synth_lm_free(m); return NULL; }
   }
   free(caps);
-  free(chosen);
-  free(es);
 
   /* materialize the tuples in lexicographic order */
   for (int k = 1; k <= N; ++k) {
@@ -560,11 +682,8 @@ SYNTH_API synth_lm_t* synth_lm_new(uint64_t seed, int32_t V, int32_t N, int64_t 
     size_t nn = (size_t)(o->n > 0 ? o->n : 1);
     m->tuples[k - 1] = malloc(sizeof(int32_t) * nn * (size_t)k);
     if (!m->tuples[k - 1]) { synth_lm_free(m); return NULL; }
-    for (int64_t x = 0; x < o->n; ++x) {
-      int32_t* dst = m->tuples[k - 1] + (size_t)x * k;
-      if (k > 1) memcpy(dst, m->tuples[k - 2] + (size_t)o->ctx[x] * (k - 1), sizeof(int32_t) * (k - 1));
-      dst[k - 1] = o->tok[x];
-    }
+    tuple_job_t tj = {m, k};
+    run_parallel(o->n, tuple_range, &tj);
   }
   return m;
 }

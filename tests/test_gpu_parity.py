@@ -99,6 +99,18 @@ def test_cfg2_sampled_parity_full_size():
     assert any(run.states[c][i][1] != 0 for c in range(w.chunks) for i in range(w.B))
 
 
+def test_cfg4_sampled_parity_full_size():
+    """The stress configuration at full size: V+1 = 4097, 1024 streams, a
+    10-gram LM with ~100M n-grams, 50,000 phrases; 3 streams replayed over all
+    20 chunks."""
+    w = synth.WORKLOADS[4]
+    inp = pu.Inputs(w)
+    run = pu.GpuRun(inp, range(w.B), w.chunks)
+    reps = pu.replay(inp, run, [0, 511, 1023])
+    pu.assert_reports(reps)
+    assert max(len(run.lm.state_tuple(run.states[-1][i][0])) for i in range(w.B)) >= 3
+
+
 def test_cfg3_beam_parity():
     """Beam search, K=4, one label per frame: every frame's kept candidates
     are the oracle's top K (up to near ties), each candidate's score

@@ -416,3 +416,18 @@ def test_beam_follow_mode():
     bad_tok[0, 0] = int(np.argmin(f0))
     rep = oracle.beam_chunk_follow(oracle.Stream(V), model, lm, bo, enc, 0.4, 0.8, K, sh, bad_tok, sinc)
     assert rep[oracle.REP_MISMATCH] >= 1
+
+
+def test_lm_order_of_input_does_not_matter():
+    """The dictionary is the same whether the n-grams arrive sorted or not."""
+    V = 9
+    lmA = synth.ngram_lm(41, V, 3, 120, 1.1)
+    a = oracle.LM.from_arrays(lmA)
+    rng = np.random.default_rng(3)
+    perms = [rng.permutation(len(x)) for x in lmA.logp]
+    b = oracle.LM(V, [t[p] for t, p in zip(lmA.tokens, perms)], [x[p] for x, p in zip(lmA.logp, perms)],
+                  [x[p] for x, p in zip(lmA.bow, perms)])
+    for h in [[], [1], [2, 3], [4, 0, 7]]:
+        for v in range(V):
+            assert a.score(h, v) == b.score(h, v)
+        assert a.state(h) == b.state(h)
