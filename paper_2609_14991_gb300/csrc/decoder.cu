@@ -187,7 +187,7 @@ extern "C" tsd_status tsd_decoder_create(const tsd_decoder_cfg* cfg, const void*
     if (!d->jtc) return cleanup(fail(TSD_ENOMEM, "tsd_decoder_create: host allocation failed"));
     d->sms = sms;
     const int bn = joint_tc_pick_bn(d->M_max, d->N_pad, sms);
-    if ((ce = joint_tc_prepare(d->jtc, Abuf, d->M_pad, Wt, d->N_pad, c.H, bn)) != cudaSuccess)
+    if ((ce = joint_tc_prepare(d->jtc, Abuf, d->M_pad, Wt, d->N_pad, c.H, bn, bias)) != cudaSuccess)
       return cleanup(cuda_fail(ce, "tsd_decoder_create: tensor-core GEMM setup (TMA descriptors)"));
   }
   for (int i = 0; i < tsd_decoder::kRing; ++i) {
@@ -574,7 +574,8 @@ extern "C" tsd_status tsd_decoder_set_option(tsd_decoder* d, const char* name, i
     if (value != 64 && value != 128 && value != 256) return fail(TSD_EINVAL, "tsd_decoder_set_option: joint_bn must be 64, 128 or 256");
     tsd_status st = drop_graphs(d);
     if (st) return st;
-    cudaError_t ce = joint_tc_prepare(d->jtc, d->view.A, d->M_pad, d->view.Wt, d->N_pad, d->cfg.H, (int)value);
+    cudaError_t ce = joint_tc_prepare(d->jtc, d->view.A, d->M_pad, d->view.Wt, d->N_pad, d->cfg.H, (int)value,
+                                      d->view.bias);
     if (ce != cudaSuccess) return cuda_fail(ce, "tsd_decoder_set_option: joint_bn");
     if (d->joint_kind == 0) {
       d->n_ptiles = d->N_pad / d->jtc->bn;

@@ -28,6 +28,14 @@ constexpr int kBM = 128, kBK = 64;
 constexpr int kThreads = 192;
 constexpr float kNegInf = -__builtin_huge_valf();
 constexpr unsigned long long kWaitNs = 1000000000ull;  // 1 s bound on any barrier wait
+constexpr float kLog2e = 1.4426950408889634f;
+
+// 2^x by the hardware approximation (relative error ~2^-22; 2^-inf = 0).
+__device__ __forceinline__ float ex2_approx(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
@@ -130,27 +138,39 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float* v) {
   for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
 }
 
+// Shared memory: [operand stages][bias boxes][barriers].  The fusion bias of
+// the tile (128 rows x BN fp32) arrives by TMA in 128 x 32 boxes with the
+// 128-byte swizzle while the mainloop runs; at BN = 256 only the first half
+// has its own buffer and the second half lands in the drained stages.
 template <int BN>
 struct Smem {
-  static constexpr int kStages = (BN == 256) ? 4 : 6;
+  static constexpr int kStages = (BN == 256) ? 3 : (BN == 128 ? 4 : 6);
   static constexpr int kABytes = kBM * kBK * 2;
   static constexpr int kBBytes = BN * kBK * 2;
   static constexpr int kStageBytes = kABytes + kBBytes;
-  static constexpr int kBytes = kStages * kStageBytes + 1024 /*align*/ + 256 /*barriers*/;
+  static constexpr int kBoxBytes = kBM * 32 * 4;
+  static constexpr int kBoxes = BN / 32;
+  static constexpr int kEarly = (BN == 256) ? 4 : kBoxes;
+  static constexpr int kBiasBytes = kEarly * kBoxBytes;
+  static constexpr int kBytes = kStages * kStageBytes + kBiasBytes + 1024 /*align*/ + 256 /*barriers*/;
+  static_assert((kBoxes - kEarly) * kBoxBytes <= kStages * kStageBytes, "late bias boxes fit the stages");
 };
 
 // BEAM: instead of the single best fused label, each row keeps the top-K
 // (K = beam width <= 8) fused values of the tile, ties to the lower label.
 template <int BN, bool BEAM>
 __global__ void __launch_bounds__(kThreads, 1)
-    k_joint_tc(DecView d, int step, const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB) {
+    k_joint_tc(DecView d, int step, const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+               const __grid_constant__ CUtensorMap tmBias) {
   using S = Smem<BN>;
   extern __shared__ __align__(1024) unsigned char smem_raw[];
   unsigned char* smem = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + S::kStages * S::kStageBytes);
+  unsigned char* bias_early = smem + S::kStages * S::kStageBytes;
+  uint64_t* full = reinterpret_cast<uint64_t*>(bias_early + S::kBiasBytes);
   uint64_t* empty = full + S::kStages;
   uint64_t* accum = empty + S::kStages;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(accum + 1);
+  uint64_t* biasbar = accum + 1;  // [0] early boxes, [1] late boxes
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(biasbar + 2);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int n0 = blockIdx.x * BN, m0 = blockIdx.y * kBM;
@@ -163,6 +183,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(empty + s, 1);
     }
     mbar_init(accum, 1);
+    mbar_init(biasbar, 1);
+    mbar_init(biasbar + 1, 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   if (warp == 1) {
@@ -184,6 +206,9 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (warp == 0) {
     if (lane == 0) {
+      // the bias tile first: the epilogue needs it as soon as the MMAs end
+      mbar_expect_tx(biasbar, S::kEarly * S::kBoxBytes);
+      for (int c = 0; c < S::kEarly; ++c) tma_load_2d(bias_early + c * S::kBoxBytes, &tmBias, biasbar, n0 + 32 * c, m0);
       int issued = 0;
       for (int kb = 0; kb < KB; ++kb) {
         const int s = kb % S::kStages;
@@ -202,6 +227,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         atomicOr(d.err, 1);
       }
     }
+    __syncwarp();  // reconverge before the CTA barrier below (bar.sync is warp-aligned)
   } else if (warp == 1) {
     if (lane == 0) {
       const uint32_t idesc = idesc_bf16(kBM, BN);
@@ -230,7 +256,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int gr = m0 + row;
     const bool live = gr < M;
     const int N = d.N, V = d.V;
-    const float* brow = d.bias + (size_t)(live ? gr : 0) * d.N_pad + n0;
     float mx = kNegInf, se = 0.f, bv = kNegInf;
     int bi = INT_MAX;
     const int K = d.K;
@@ -242,40 +267,79 @@ __global__ void __launch_bounds__(kThreads, 1)
     ok = __all_sync(0xffffffffu, mbar_wait(accum, 0));  // warp-uniform: tcgen05.ld is .sync.aligned
     if (!ok && lane == 0) atomicOr(d.err, 4);
     fence_after();
+    // the second half of a 256-wide bias tile goes into the drained stages
+    // (every MMA has completed, so nothing reads them any more)
+    const bool late = ok && S::kEarly < S::kBoxes;
+    if (late && warp == 2 && lane == 0) {
+      mbar_expect_tx(biasbar + 1, (S::kBoxes - S::kEarly) * S::kBoxBytes);
+      for (int c = S::kEarly; c < S::kBoxes; ++c)
+        tma_load_2d(smem + (c - S::kEarly) * S::kBoxBytes, &tmBias, biasbar + 1, n0 + 32 * c, m0);
+    }
+    const bool have_early = __all_sync(0xffffffffu, mbar_wait(biasbar, 0));
+    if (!have_early) {
+      ok = false;
+      if (lane == 0) atomicOr(d.err, 16);
+    }
+    bool late_done = !late;
     if (ok) {
       const uint32_t tbase = tmem + ((uint32_t)(q * 32) << 16);
-      float4 bnext[8];
-#pragma unroll
-      for (int i = 0; i < 8; ++i) bnext[i] = live ? __ldcg(reinterpret_cast<const float4*>(brow) + i) : make_float4(0, 0, 0, 0);
+      const int sw = row & 7;  // 128-byte swizzle: 16-byte chunk j of a row sits at j ^ (row % 8)
 #pragma unroll 1
       for (int c = 0; c < BN / 32; ++c) {
+        if (c == S::kEarly) {
+          late_done = true;
+          if (!__all_sync(0xffffffffu, mbar_wait(biasbar + 1, 0))) {
+            if (lane == 0) atomicOr(d.err, 32);
+            break;
+          }
+        }
+        const unsigned char* box = (c < S::kEarly) ? bias_early + c * S::kBoxBytes : smem + (c - S::kEarly) * S::kBoxBytes;
         float b[32];
 #pragma unroll
-        for (int i = 0; i < 8; ++i) {
-          b[4 * i] = bnext[i].x; b[4 * i + 1] = bnext[i].y; b[4 * i + 2] = bnext[i].z; b[4 * i + 3] = bnext[i].w;
-        }
-        if (c + 1 < BN / 32) {
-#pragma unroll
-          for (int i = 0; i < 8; ++i)
-            bnext[i] = live ? __ldcg(reinterpret_cast<const float4*>(brow + (c + 1) * 32) + i) : make_float4(0, 0, 0, 0);
+        for (int j = 0; j < 8; ++j) {
+          const float4 v = *reinterpret_cast<const float4*>(box + row * 128 + ((j ^ sw) << 4));
+          b[4 * j] = v.x; b[4 * j + 1] = v.y; b[4 * j + 2] = v.z; b[4 * j + 3] = v.w;
         }
         float l[32];
         tmem_ld32(tbase + (uint32_t)(c * 32), l);
         const int c0 = n0 + c * 32;
-        float cm = kNegInf;
+        // Labels at or past V+1 (padding of the last tile) take no part:
+        // their logit becomes -inf.  Blank (label V) has bias 0 in the row.
+        if (c0 + 32 > N) {
 #pragma unroll
-        for (int i = 0; i < 32; ++i) {
-          const int gc = c0 + i;
-          if (gc < N) {
-            cm = fmaxf(cm, l[i]);
-            const float f = l[i] + (gc < V ? b[i] : 0.f);
-            if (!BEAM) {
-              if (f > bv) { bv = f; bi = gc; }
-            } else if (f > tmin) {
+          for (int i = 0; i < 32; ++i)
+            if (c0 + i >= N) l[i] = kNegInf;
+        }
+        // fused values f = logit + bias (reuse b), chunk maxima by trees
+        float t[16], u[16];
+#pragma unroll
+        for (int i = 0; i < 32; ++i) b[i] += l[i];
+#pragma unroll
+        for (int i = 0; i < 16; ++i) { t[i] = fmaxf(l[i], l[i + 16]); u[i] = fmaxf(b[i], b[i + 16]); }
+#pragma unroll
+        for (int w = 8; w > 0; w >>= 1)
+#pragma unroll
+          for (int i = 0; i < w; ++i) { t[i] = fmaxf(t[i], t[i + w]); u[i] = fmaxf(u[i], u[i + w]); }
+        const float cm = t[0], fm = u[0];
+        if (!BEAM) {
+          // the first label of the chunk holding the chunk's best fused value
+          if (fm > bv) {
+            int j = 31;
+#pragma unroll
+            for (int i = 31; i >= 0; --i)
+              if (b[i] == fm) j = i;
+            bv = fm;
+            bi = c0 + j;
+          }
+        } else if (fm > tmin) {
+#pragma unroll
+          for (int i = 0; i < 32; ++i) {
+            const float f = b[i];
+            if (f > tmin) {
               // bubble the new value into the sorted list (labels arrive in
               // increasing order, so a later equal value stays behind)
               float cv = f;
-              int ci = gc;
+              int ci = c0 + i;
 #pragma unroll
               for (int j = 0; j < 8; ++j) {
                 if (j < K && cv > tv[j]) {
@@ -290,11 +354,12 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
         }
         if (cm != kNegInf) {
+          // online softmax partial: sum of 2^((logit - max) * log2 e)
           const float m2 = fmaxf(mx, cm);
-          float acc = (mx == kNegInf) ? 0.f : se * exp2f((mx - m2) * 1.4426950408889634f);
+          const float s2 = m2 * kLog2e;
+          float acc = (mx == kNegInf) ? 0.f : se * ex2_approx(mx * kLog2e - s2);
 #pragma unroll
-          for (int i = 0; i < 32; ++i)
-            if (c0 + i < N) acc += exp2f((l[i] - m2) * 1.4426950408889634f);
+          for (int i = 0; i < 32; ++i) acc += ex2_approx(fmaf(l[i], kLog2e, -s2));
           se = acc;
           mx = m2;
         }
@@ -317,6 +382,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
     }
+    // never leave with bias boxes still landing in shared memory
+    if (!late_done && warp == 2 && lane == 0) mbar_wait(biasbar + 1, 0);
   }
   fence_before();
   __syncthreads();
@@ -342,16 +409,19 @@ EncodeTiledFn encode_fn() {
   return fn;
 }
 
-bool make_map(CUtensorMap* m, const void* base, int K, int rows, int box_rows) {
+// 2-D row-major map with the 128-byte swizzle: `inner` elements per row,
+// boxes of box_inner x box_rows.
+bool make_map(CUtensorMap* m, const void* base, CUtensorMapDataType dtype, int elem_bytes, int inner, int rows,
+              int box_inner, int box_rows) {
   EncodeTiledFn fn = encode_fn();
   if (!fn) return false;
-  cuuint64_t dims[2] = {(cuuint64_t)K, (cuuint64_t)rows};
-  cuuint64_t strides[1] = {(cuuint64_t)K * 2};
-  cuuint32_t box[2] = {(cuuint32_t)kBK, (cuuint32_t)box_rows};
+  cuuint64_t dims[2] = {(cuuint64_t)inner, (cuuint64_t)rows};
+  cuuint64_t strides[1] = {(cuuint64_t)inner * elem_bytes};
+  cuuint32_t box[2] = {(cuuint32_t)box_inner, (cuuint32_t)box_rows};
   cuuint32_t es[2] = {1, 1};
-  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, es,
-            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+  return fn(m, dtype, 2, const_cast<void*>(base), dims, strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE,
+            CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) ==
+         CUDA_SUCCESS;
 }
 
 }  // namespace
@@ -363,10 +433,13 @@ int joint_tc_pick_bn(int M_max, int N_pad, int sms) {
   return 64;
 }
 
-cudaError_t joint_tc_prepare(JointTc* jt, const uint16_t* A, int M_pad, const uint16_t* Wt, int N_pad, int H, int bn) {
+cudaError_t joint_tc_prepare(JointTc* jt, const uint16_t* A, int M_pad, const uint16_t* Wt, int N_pad, int H, int bn,
+                             const float* bias) {
   jt->bn = bn;
-  if (!make_map(&jt->mapA, A, H, M_pad, kBM)) return cudaErrorInvalidValue;
-  if (!make_map(&jt->mapB, Wt, H, N_pad, bn)) return cudaErrorInvalidValue;
+  if (!make_map(&jt->mapA, A, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, H, M_pad, kBK, kBM)) return cudaErrorInvalidValue;
+  if (!make_map(&jt->mapB, Wt, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, H, N_pad, kBK, bn)) return cudaErrorInvalidValue;
+  if (!make_map(&jt->mapBias, bias, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, N_pad, M_pad, 32, kBM))
+    return cudaErrorInvalidValue;
   cudaError_t e = cudaSuccess;
   if (bn == 256) {
     e = cudaFuncSetAttribute(k_joint_tc<256, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, Smem<256>::kBytes);
@@ -397,16 +470,16 @@ void launch_joint_tc(const JointTc& jt, const DecView& d, int M, int step, cudaS
   const bool beam = d.K > 1;
   if (jt.bn == 256) {
     cfg.dynamicSmemBytes = Smem<256>::kBytes;
-    if (beam) cudaLaunchKernelEx(&cfg, k_joint_tc<256, true>, d, step, jt.mapA, jt.mapB);
-    else cudaLaunchKernelEx(&cfg, k_joint_tc<256, false>, d, step, jt.mapA, jt.mapB);
+    if (beam) cudaLaunchKernelEx(&cfg, k_joint_tc<256, true>, d, step, jt.mapA, jt.mapB, jt.mapBias);
+    else cudaLaunchKernelEx(&cfg, k_joint_tc<256, false>, d, step, jt.mapA, jt.mapB, jt.mapBias);
   } else if (jt.bn == 128) {
     cfg.dynamicSmemBytes = Smem<128>::kBytes;
-    if (beam) cudaLaunchKernelEx(&cfg, k_joint_tc<128, true>, d, step, jt.mapA, jt.mapB);
-    else cudaLaunchKernelEx(&cfg, k_joint_tc<128, false>, d, step, jt.mapA, jt.mapB);
+    if (beam) cudaLaunchKernelEx(&cfg, k_joint_tc<128, true>, d, step, jt.mapA, jt.mapB, jt.mapBias);
+    else cudaLaunchKernelEx(&cfg, k_joint_tc<128, false>, d, step, jt.mapA, jt.mapB, jt.mapBias);
   } else {
     cfg.dynamicSmemBytes = Smem<64>::kBytes;
-    if (beam) cudaLaunchKernelEx(&cfg, k_joint_tc<64, true>, d, step, jt.mapA, jt.mapB);
-    else cudaLaunchKernelEx(&cfg, k_joint_tc<64, false>, d, step, jt.mapA, jt.mapB);
+    if (beam) cudaLaunchKernelEx(&cfg, k_joint_tc<64, true>, d, step, jt.mapA, jt.mapB, jt.mapBias);
+    else cudaLaunchKernelEx(&cfg, k_joint_tc<64, false>, d, step, jt.mapA, jt.mapB, jt.mapBias);
   }
 }
 
