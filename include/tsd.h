@@ -84,7 +84,8 @@ TSD_API const char* tsd_version(void);
  *                  not an n-gram), with only the last order-1 labels of h
  *                  used and log p(v | empty) = logp of the unigram v.
  * Requirements (else TSD_EINVAL): 1 <= order <= 16; every unigram [0, V)
- * present exactly once; tokens in range; no duplicate n-gram; the set is
+ * present exactly once; fewer than 2^28 n-grams above order 1; tokens in
+ * range; no duplicate n-gram; the set is
  * prefix- and suffix-closed (every prefix and every suffix of an n-gram is an
  * n-gram), as in any ARPA model estimated from counts; finite values.
  * The inputs are copied (the caller keeps ownership) and uploaded

@@ -39,6 +39,7 @@ void enqueue_chunk(tsd_decoder* d, int M, int T, cudaStream_t s, const std::vect
   auto mark = [&]() {
     if (ev) cudaEventRecordWithFlags((*ev)[(size_t)e++], s, cudaEventRecordExternal);
   };
+  launch_defaults(d->view, s);
   for (int step = 0; step <= S; ++step) {
     const bool pdl = d->pdl && !ev && step > 0;  // the first launch follows the parameter copy
     mark();
@@ -123,6 +124,7 @@ extern "C" tsd_status tsd_decoder_create(const tsd_decoder_cfg* cfg, const void*
   int32_t *rt, *rs, *rc, *sl, *sll, *slc, *stl, *stc, *err;
   unsigned long long* ctr;
   float2* bpart = nullptr;
+  float2* dflt = nullptr;
   double* hscore = nullptr;
   int32_t *hlive = nullptr, *hnode = nullptr, *hlen = nullptr, *ppar = nullptr, *ptok = nullptr, *pn = nullptr;
   unsigned long long* hhash = nullptr;
@@ -132,7 +134,7 @@ extern "C" tsd_status tsd_decoder_create(const tsd_decoder_cfg* cfg, const void*
   tsd_status st;
   if ((st = A.alloc(&Wt, (size_t)d->N_pad * c.H)) || (st = A.alloc(&E, (size_t)d->N * c.H)) ||
       (st = A.alloc(&Abuf, (size_t)d->M_pad * c.H)) || (st = A.alloc(&bias, (size_t)d->M_pad * d->N_pad)) ||
-      (st = A.alloc(&part, (size_t)d->M_pad * (d->N_pad / 64))) || (st = A.alloc(&err, 1)) || (st = A.alloc(&ctr, 1)) || (st = A.alloc(&rt, (size_t)d->M_pad)) ||
+      (st = A.alloc(&part, (size_t)d->M_pad * (d->N_pad / 64))) || (st = A.alloc(&err, 1)) || (st = A.alloc(&ctr, 1)) || (st = A.alloc(&dflt, (size_t)c.V)) || (st = A.alloc(&rt, (size_t)d->M_pad)) ||
       (st = A.alloc(&rs, (size_t)d->M_pad)) || (st = A.alloc(&rc, (size_t)d->M_pad)) ||
       (st = A.alloc(&sl, SK)) || (st = A.alloc(&sll, SK)) || (st = A.alloc(&slc, SK * kLmChain)) ||
       (st = A.alloc(&stl, SK)) || (st = A.alloc(&stc, SK * kTrChain)) || (st = A.alloc(&pdev, d->params_bytes))) {
@@ -232,6 +234,7 @@ extern "C" tsd_status tsd_decoder_create(const tsd_decoder_cfg* cfg, const void*
   v.cap_steps = 0;
   v.err = err;
   v.ctr = ctr;
+  v.dflt = dflt;
   v.bpart = bpart;
   v.h_score = hscore;
   v.h_live = hlive;
@@ -532,7 +535,7 @@ extern "C" tsd_status tsd_decoder_launches_per_chunk(const tsd_decoder* d, int32
   clear_error();
   if (!d || !launches) return fail(TSD_EINVAL, "tsd_decoder_launches_per_chunk: NULL argument");
   (void)n;
-  *launches = 2 * (int64_t)steps_per_chunk(d, T) + 1;
+  *launches = 2 * (int64_t)steps_per_chunk(d, T) + 2;
   return TSD_OK;
 }
 

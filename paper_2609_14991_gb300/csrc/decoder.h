@@ -59,6 +59,7 @@ struct DecView {
   int32_t* pool_tok;    // [slots][pool_cap] label of the node
   int32_t* pool_n;      // [slots] nodes used
   int32_t pool_cap;
+  float2* dflt;  // [V] per-call bias defaults (lambda*log p(v), beta*bonus*[root child v])
   int32_t* err;  // device status word: nonzero after a bounded wait expired
   unsigned long long* ctr;  // algorithmic bytes counted by replayed row passes
 };
@@ -69,6 +70,7 @@ void launch_repack(const uint16_t* W, uint16_t* Wt, int H, int N, int N_pad, cud
 void launch_open(const DecView& d, int slot, cudaStream_t s);
 void launch_row(const DecView& d, int M, int step, int mode, size_t smem, cudaStream_t s, bool pdl);
 void launch_joint(const DecView& d, int M, int step, cudaStream_t s);
+void launch_defaults(const DecView& d, cudaStream_t s);
 size_t row_smem_bytes(int V4);
 cudaError_t prepare_kernels(size_t row_smem);
 void launch_row_beam(const DecView& d, int n, int step, int mode, size_t smem, cudaStream_t s, bool pdl);

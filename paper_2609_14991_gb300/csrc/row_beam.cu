@@ -76,8 +76,8 @@ __global__ void __launch_bounds__(kRowThreads) k_row_beam(DecView d, int step, i
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const bool commit = (mode != 2);
   extern __shared__ __align__(16) unsigned char smem[];
-  unsigned long long* lmkey = reinterpret_cast<unsigned long long*>(smem);
-  int* dep = reinterpret_cast<int*>(lmkey + d.V4);
+  float* lmv = reinterpret_cast<float*>(smem);
+  uint8_t* dep = reinterpret_cast<uint8_t*>(lmv + d.V4);
 
   __shared__ int s_slot, s_T;
   __shared__ int o_live[kMaxK], o_last[kMaxK], o_node[kMaxK], o_len[kMaxK], o_lml[kMaxK], o_trl[kMaxK];
@@ -419,9 +419,9 @@ __global__ void __launch_bounds__(kRowThreads) k_row_beam(DecView d, int step, i
   const uint16_t* enc_row = P->enc + ((size_t)b * T + min(step, T - 1)) * d.H;
   for (int j = 0; j < cnt; ++j) {
     const int r = b * K + j;
-    row::bias_prepare(d, n_lm[j], n_lml[j], n_tr[j], n_trl[j], rc, lmkey, dep);
+    row::bias_prepare(d, n_lm[j], n_lml[j], n_tr[j], n_trl[j], rc, lmv, dep);
     row::build_joint_input(d, enc_row, n_last[j], r);
-    row::bias_finish(d, n_lml[j], n_trl[j], rc, P->lambda, P->beta, d.bias + (size_t)r * d.N_pad, lmkey, dep);
+    row::bias_finish(d, n_lml[j], n_trl[j], rc, P->lambda, P->beta, d.bias + (size_t)r * d.N_pad, lmv, dep);
     __syncthreads();  // the scratch is reused by the next survivor
   }
 }

@@ -71,10 +71,16 @@ struct ChainRecs {
   int td[kTrChain];                // trie chain node: depth of its children
 };
 
+// Per-label scratch of a bias row in shared memory (5 bytes per label):
+//   lmv[v] = log p_LM(v | state) from the deepest LM chain level that
+//            continues with v, NaN if none does;
+//   dep[v] = depth of v's trie goto node from the chain, 0 if none.
+__device__ __forceinline__ float unset_value() { return __int_as_float(0x7fc00000); }
+
 // Step 1 of a bias row (no barrier): fetch the chains' records, clear the
 // per-label scratch.  All threads of the block call it.
 __device__ __forceinline__ void bias_prepare(const DecView& d, const int* lm_chain, int nl, const int* tr_chain,
-                                             int nt, ChainRecs& rc, unsigned long long* lmkey, int* dep) {
+                                             int nt, ChainRecs& rc, float* lmv, uint8_t* dep) {
   const int tid = threadIdx.x;
   if (tid < nl) {
     const int st = lm_chain[tid];
@@ -87,54 +93,87 @@ __device__ __forceinline__ void bias_prepare(const DecView& d, const int* lm_cha
     rc.tc[tid - 32] = __ldg(d.tr.nd_count + q);
     rc.td[tid - 32] = __ldg(d.tr.nd_depth + q) + 1;
   }
+  const float unset = unset_value();
   for (int v = tid; v < d.V; v += blockDim.x) {
-    lmkey[v] = 0ull;
+    lmv[v] = unset;
     dep[v] = 0;
   }
 }
 
 // Step 2: the dense fusion bias row lambda*log p_LM(v|state) +
 // beta*bonus*(goto depth - current depth) for every label v (blank: 0).
-// Every chain level is merged at once: a label's LM score comes from the
-// deepest level that continues with it (max of level << 32 | value bits),
-// its goto depth from the deepest trie node that has it as a child.
+// LM chain levels are applied deepest first, each label keeping the first
+// value it gets; trie chain nodes shallowest first, the deepest node's child
+// depth overwriting.  One barrier per level.  Labels no level touches take
+// the call's defaults dflt[v] = (lambda*log p(v), beta*bonus*[root has v]).
 __device__ __forceinline__ void bias_finish(const DecView& d, int nl, int nt, const ChainRecs& rc, float lam,
-                                            float beta, float* brow, unsigned long long* lmkey, int* dep) {
+                                            float beta, float* brow, float* lmv, uint8_t* dep) {
   const int tid = threadIdx.x;
   const int V = d.V;
+  const int step = blockDim.x;
   __syncthreads();
   const float cum_top = nl ? rc.lo[nl - 1] : 0.f;
-  for (int l = 0; l < nl; ++l) {
-    const int b = rc.lb[l], c = rc.lc[l];
-    const float off = cum_top - rc.lo[l];
-    const unsigned long long lev = (unsigned long long)(l + 1) << 32;
-    for (int j = tid; j < c; j += blockDim.x) {
-      const int w = __ldg(d.lm.arc_tok + b + j);
-      const float val = off + __ldg(d.lm.arc_logp + b + j);
-      atomicMax(lmkey + w, lev | (unsigned long long)__float_as_uint(val));
+  const int phases = max(nl, nt);
+  for (int p = 0; p < phases; ++p) {
+    if (p < nl) {
+      const int l = nl - 1 - p;
+      const int b = rc.lb[l], c = rc.lc[l];
+      const float off = cum_top - rc.lo[l];
+      int j = tid;
+      for (; j + 3 * step < c; j += 4 * step) {  // four arcs' loads in flight
+        int w[4];
+        float lp[4];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          w[q] = __ldg(d.lm.arc_tok + b + j + q * step);
+          lp[q] = __ldg(d.lm.arc_logp + b + j + q * step);
+        }
+#pragma unroll
+        for (int q = 0; q < 4; ++q)
+          if (isnan(lmv[w[q]])) lmv[w[q]] = off + lp[q];
+      }
+      for (; j < c; j += step) {
+        const int w = __ldg(d.lm.arc_tok + b + j);
+        const float lp = __ldg(d.lm.arc_logp + b + j);
+        if (isnan(lmv[w])) lmv[w] = off + lp;
+      }
     }
+    if (p < nt) {
+      const int k = nt - 1 - p;
+      const int b = rc.tb[k], c = rc.tc[k];
+      const uint8_t dd = (uint8_t)rc.td[k];
+      for (int j = tid; j < c; j += step) dep[__ldg(d.tr.ch_tok + b + j)] = dd;
+    }
+    __syncthreads();
   }
-  for (int k = 0; k < nt; ++k) {
-    const int b = rc.tb[k], c = rc.tc[k], dd = rc.td[k];
-    for (int j = tid; j < c; j += blockDim.x) atomicMax(dep + __ldg(d.tr.ch_tok + b + j), dd);
-  }
-  __syncthreads();
   const int depth_cur = nt ? rc.td[0] - 1 : 0;
   const float bscale = beta * (d.has_tr ? d.tr.bonus : 0.f);
-  for (int v = tid; v < V; v += blockDim.x) {
-    float b = 0.f;
-    if (d.has_lm) {
-      const unsigned long long k = lmkey[v];
-      const float l = k ? __uint_as_float((unsigned)k) : cum_top + __ldg(d.lm.uni_logp + v);
-      b = lam * l;
+  const float base = lam * cum_top - bscale * (float)depth_cur;
+  const float2* dflt = d.dflt;
+  int v = tid;
+  for (; v + 3 * step < V; v += 4 * step) {  // four labels' defaults in flight
+    float2 df[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) df[q] = __ldcg(dflt + v + q * step);
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const int u = v + q * step;
+      const float l = lmv[u];
+      const int dd = dep[u];
+      const float blm = isnan(l) ? df[q].x + lam * cum_top : lam * l;
+      const float btr = dd ? bscale * (float)(dd - depth_cur) : df[q].y - bscale * (float)depth_cur;
+      brow[u] = blm + btr;
     }
-    if (d.has_tr) {
-      int dd = dep[v];
-      if (dd == 0) dd = (__ldg(d.tr.root_child + v) != 0) ? 1 : 0;
-      b += bscale * (float)(dd - depth_cur);
-    }
-    brow[v] = b;
   }
+  for (; v < V; v += step) {
+    const float2 df = __ldcg(dflt + v);
+    const float l = lmv[v];
+    const int dd = dep[v];
+    const float blm = isnan(l) ? df.x + lam * cum_top : lam * l;
+    const float btr = dd ? bscale * (float)(dd - depth_cur) : df.y - bscale * (float)depth_cur;
+    brow[v] = blm + btr;
+  }
+  (void)base;
   if (tid == 0) brow[V] = 0.f;
 }
 

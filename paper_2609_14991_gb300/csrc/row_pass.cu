@@ -36,8 +36,8 @@ __global__ void __launch_bounds__(kRowThreads) k_row(DecView d, int step, int mo
   const bool commit = (mode != 2);
   extern __shared__ __align__(16) unsigned char smem[];
   // per-label scratch: LM (level << 32 | value bits), trie depth of the goto
-  unsigned long long* lmkey = reinterpret_cast<unsigned long long*>(smem);
-  int* dep = reinterpret_cast<int*>(lmkey + d.V4);
+  float* lmv = reinterpret_cast<float*>(smem);
+  uint8_t* dep = reinterpret_cast<uint8_t*>(lmv + d.V4);
 
   __shared__ int s_t, s_sym, s_cnt, s_y, s_lm_len, s_tr_len, s_last, s_slot, s_T;
   __shared__ float s_score;
@@ -210,9 +210,9 @@ __global__ void __launch_bounds__(kRowThreads) k_row(DecView d, int step, int mo
   // 3. records of the new chains, scratch reset; 4. joint input of this
   // step (its loads overlap the records); 5. the fusion bias row
   const int nl = s_lm_len, nt = s_tr_len;
-  row::bias_prepare(d, s_lm, nl, s_tr, nt, rc, lmkey, dep);
+  row::bias_prepare(d, s_lm, nl, s_tr, nt, rc, lmv, dep);
   row::build_joint_input(d, P->enc + ((size_t)r * T + t) * d.H, s_last, r);
-  row::bias_finish(d, nl, nt, rc, P->lambda, P->beta, d.bias + (size_t)r * d.N_pad, lmkey, dep);
+  row::bias_finish(d, nl, nt, rc, P->lambda, P->beta, d.bias + (size_t)r * d.N_pad, lmv, dep);
   if (mode == 2 && tid == 0) {
     // Algorithmic bytes of this row-step: selection partials, row state,
     // the searches of the emitted label (one probe per halving plus the arc
@@ -257,7 +257,24 @@ __global__ void k_repack(const uint16_t* __restrict__ W, uint16_t* __restrict__ 
 
 }  // namespace
 
-size_t row_smem_bytes(int V4) { return (size_t)V4 * (sizeof(unsigned long long) + sizeof(int)); }
+size_t row_smem_bytes(int V4) { return (size_t)V4 * (sizeof(float) + sizeof(uint8_t)); }
+
+namespace {
+// Per-call defaults of the fusion bias: (lambda * log p(v), beta * bonus *
+// [the trie root has a child v]) for every label; the row pass adds the
+// row's own terms.  One small launch at the start of every chunk.
+__global__ void k_defaults(DecView d) {
+  const Params* P = d.params;
+  const float lam = P->lambda, bscale = P->beta * (d.has_tr ? d.tr.bonus : 0.f);
+  for (int v = blockIdx.x * blockDim.x + threadIdx.x; v < d.V; v += gridDim.x * blockDim.x) {
+    const float lm = d.has_lm ? lam * __ldg(d.lm.uni_logp + v) : 0.f;
+    const float tr = (d.has_tr && __ldg(d.tr.root_child + v) != 0) ? bscale : 0.f;
+    d.dflt[v] = make_float2(lm, tr);
+  }
+}
+}  // namespace
+
+void launch_defaults(const DecView& d, cudaStream_t s) { k_defaults<<<(d.V + 255) / 256, 256, 0, s>>>(d); }
 
 cudaError_t prepare_kernels(size_t row_smem) {
   // dynamic scratch plus the kernel's static shared memory may pass the

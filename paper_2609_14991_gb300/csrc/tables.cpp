@@ -108,7 +108,8 @@ extern "C" tsd_status tsd_ngram_build(int32_t V, int32_t order, const int64_t* c
     if (k >= 2) total_arcs += o.n;
   }
   if (in[1].n != V) return fail(TSD_EINVAL, "tsd_ngram_build: %lld unigrams, need all %d", (long long)in[1].n, V);
-  if (total_arcs > INT32_MAX - 1) return fail(TSD_EINVAL, "tsd_ngram_build: too many n-grams");
+  // the row pass tags arc indices with their level in 32-bit keys
+  if (total_arcs >= (int64_t)1 << 28) return fail(TSD_EINVAL, "tsd_ngram_build: more than 2^28 n-grams above order 1");
 
   // range and value checks, then sort each order
   for (int k = 1; k <= order; ++k) {
