@@ -28,7 +28,7 @@ using row::warp_find;
 // mode: 0 = label step, 1 = final step (apply the last decision only),
 // 2 = replay (redo the step's work without committing any state or output;
 // used only to time the kernel in isolation).
-__global__ void __launch_bounds__(kRowThreads) k_row(DecView d, int step, int mode) {
+__global__ void __launch_bounds__(kRowThreads, 8) k_row(DecView d, int step, int mode) {
   const Params* __restrict__ P = d.params;
   const int r = blockIdx.x;
   const int V = d.V;
@@ -40,6 +40,14 @@ __global__ void __launch_bounds__(kRowThreads) k_row(DecView d, int step, int mo
   uint8_t* dep = reinterpret_cast<uint8_t*>(lmv + d.V4);
 
   __shared__ int s_t, s_sym, s_cnt, s_y, s_lm_len, s_tr_len, s_last, s_slot, s_T;
+  // the call's parameters, read once before the dependency wait
+  __shared__ int32_t* s_out_tok;
+  __shared__ int32_t* s_out_frame;
+  __shared__ float* s_out_score;
+  __shared__ int32_t* s_out_count;
+  __shared__ const uint16_t* s_enc;
+  __shared__ float s_lam, s_beta;
+  __shared__ int s_n;
   __shared__ float s_score;
   __shared__ int s_lm[kLmChain], s_tr[kTrChain];
   __shared__ int s_lm_tgt[kLmChain];            // target state of y's arc at each LM level (-2 none)
@@ -54,6 +62,14 @@ __global__ void __launch_bounds__(kRowThreads) k_row(DecView d, int step, int mo
     const int slot = __ldcg(P->slots + r);
     s_slot = slot;
     s_T = __ldcg(&P->T);
+    s_out_tok = P->out_tok;
+    s_out_frame = P->out_frame;
+    s_out_score = P->out_score;
+    s_out_count = P->out_count;
+    s_enc = P->enc;
+    s_lam = P->lambda;
+    s_beta = P->beta;
+    s_n = P->n;
     if (step == 0) {
       s_t = 0; s_sym = 0; s_cnt = 0;
     } else {
@@ -167,9 +183,9 @@ __global__ void __launch_bounds__(kRowThreads) k_row(DecView d, int step, int mo
           if (d.has_tr) d.s_tr_len[slot] = tn;
           const int cap = T * d.max_sym;
           const int o = r * cap + s_cnt;
-          P->out_tok[o] = y;
-          P->out_frame[o] = s_t;
-          P->out_score[o] = s_score;
+          s_out_tok[o] = y;
+          s_out_frame[o] = s_t;
+          s_out_score[o] = s_score;
           d.s_last[slot] = y;
         }
         s_cnt += 1;
@@ -185,7 +201,7 @@ __global__ void __launch_bounds__(kRowThreads) k_row(DecView d, int step, int mo
   }
 
   if (mode == 1) {
-    if (tid == 0) P->out_count[r] = s_cnt;
+    if (tid == 0) s_out_count[r] = s_cnt;
     return;
   }
   if (tid == 0 && commit) {
@@ -195,7 +211,7 @@ __global__ void __launch_bounds__(kRowThreads) k_row(DecView d, int step, int mo
   }
   const int t = commit ? s_t : min(s_t, T - 1);
   if (d.cap_rows && step < d.cap_steps && tid == 0 && commit) {
-    int* c = d.cap_rows + ((size_t)step * P->n + r) * 4;
+    int* c = d.cap_rows + ((size_t)step * s_n + r) * 4;
     if (t < T) {
       c[0] = t;
       c[1] = s_last;
@@ -211,8 +227,8 @@ __global__ void __launch_bounds__(kRowThreads) k_row(DecView d, int step, int mo
   // step (its loads overlap the records); 5. the fusion bias row
   const int nl = s_lm_len, nt = s_tr_len;
   row::bias_prepare(d, s_lm, nl, s_tr, nt, rc, lmv, dep);
-  row::build_joint_input(d, P->enc + ((size_t)r * T + t) * d.H, s_last, r);
-  row::bias_finish(d, nl, nt, rc, P->lambda, P->beta, d.bias + (size_t)r * d.N_pad, lmv, dep);
+  row::build_joint_input(d, s_enc + ((size_t)r * T + t) * d.H, s_last, r);
+  row::bias_finish(d, nl, nt, rc, s_lam, s_beta, d.bias + (size_t)r * d.N_pad, lmv, dep);
   if (mode == 2 && tid == 0) {
     // Algorithmic bytes of this row-step: selection partials, row state,
     // the searches of the emitted label (one probe per halving plus the arc
