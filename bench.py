@@ -50,6 +50,35 @@ def peaks():
     return dict(PEAKS_FALLBACK), "fallback"
 
 
+# DRAM traffic per launch (dram__bytes_read.sum + dram__bytes_write.sum) from
+# one ncu capture of the kernel inside this bench's graph, keyed by (config,
+# streams, kernel), with the hash of the kernel's sources at capture time: a
+# changed kernel reports null until it is captured again.  The captures and
+# their commands are summarised under profiles/.
+KERNEL_SOURCES = {
+    "joint": ["joint_tc.cu", "joint_tc.h", "decoder.h", "internal.h"],
+    "row": ["row_pass.cu", "row_beam.cu", "row_common.cuh", "decoder.h", "internal.h"],
+}
+TRAFFIC = {}
+
+
+def kernel_source_hash(kernel: str) -> str:
+    import hashlib
+
+    h = hashlib.sha256()
+    for f in KERNEL_SOURCES[kernel]:
+        with open(os.path.join(ROOT, "paper_2609_14991_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def recorded_traffic(w: synth.Workload, kernel: str):
+    rec = TRAFFIC.get((w.cfg, w.B, kernel))
+    if rec is None or rec[1] != kernel_source_hash(kernel):
+        return None
+    return rec[0]
+
+
 def workload_config(w: synth.Workload, lm_total: int, n_phr: int):
     return {"workload": f"cfg{w.cfg} {w.name}", "B_per_gpu": w.B, "T": w.T, "H": w.H, "V": w.V,
             "lm_order": w.lm_order, "lm_ngrams": lm_total, "boost_phrases": n_phr, "lambda": w.lam,
@@ -119,6 +148,39 @@ def _dist():
     rank = int(os.environ.get("RANK", "0"))
     local = int(os.environ.get("LOCAL_RANK", "0"))
     return ws, rank, local
+
+
+def rank_streams(rank: int, B: int):
+    """The global stream ids rank `rank` decodes: its own block of B (streams
+    are independent, so ranks share no data and exchange nothing)."""
+    return list(range(rank * B, (rank + 1) * B))
+
+
+def max_over_ranks(values, ws: int, device=None):
+    """Element-wise maximum of a list of floats over all ranks (identity at
+    ws == 1): the job's time is that of its slowest rank."""
+    if ws <= 1:
+        return [float(v) for v in values]
+    import torch
+    import torch.distributed as dist
+
+    t = torch.tensor([float(v) for v in values], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return [float(x) for x in t.cpu().tolist()]
+
+
+def latency_stats(step_ms):
+    a = np.asarray(step_ms, dtype=np.float64)
+    return {"p50_ms": float(np.percentile(a, 50)), "p99_ms": float(np.percentile(a, 99)),
+            "max_ms": float(a.max()), "steps": int(a.size)}
+
+
+def workload(cfg: int, streams=None) -> synth.Workload:
+    """The workload of a config, optionally with another stream count B."""
+    w = synth.WORKLOADS[cfg]
+    if streams and streams != w.B:
+        w = synth.scaled(w, B=int(streams), name=w.name.replace(f"B={w.B}", f"B={int(streams)}"))
+    return w
 
 
 def oracle_models(w, inp_lm, inp_ph, E, W):
@@ -201,7 +263,7 @@ def run_ours(args, w):
     lmA = synth.lm_for(w)
     ph = synth.phrases_for(w)
     E, W = synth.joint_weights(w)
-    streams = list(range(rank * w.B, (rank + 1) * w.B))  # this rank's streams
+    streams = rank_streams(rank, w.B)
     lm = tsd.NGram.from_arrays(lmA) if lmA is not None else None
     bo = tsd.Boost.from_phrases(w.V, ph, w.bonus) if ph is not None else None
     dec = tsd.Decoder(w.V, w.H, torch.from_numpy(W.view(np.int16)).to(dev), torch.from_numpy(E.view(np.int16)).to(dev),
@@ -240,14 +302,15 @@ def run_ours(args, w):
                 ends[k].record(stream)
             barrier()
             wall = time.perf_counter() - t0
-        return float(sum(s.elapsed_time(e) for s, e in zip(starts, ends))), wall, clk
+        per = [s.elapsed_time(e) for s, e in zip(starts, ends)]
+        return float(sum(per)), wall, clk, per
 
     # warm-up (captures the chunk graph)
     for c in range(args.warmup):
         step(c)
     barrier()
     # timed region: K steps through the captured graph, no instrumentation
-    t_ms, wall, clk = timed_loop(args.warmup)
+    t_ms, wall, clk, step_ms = timed_loop(args.warmup)
     # the same K steps again with a CUDA event recorded at every kernel
     # boundary inside the graph: per-kernel device time for the roofline
     dec.set_timing(True)
@@ -255,15 +318,12 @@ def run_ours(args, w):
         step(args.warmup + c)  # captures the two event-carrying graphs
     barrier()
     dec.timing(reset=True)
-    t_inst_ms, _, _ = timed_loop(args.warmup)
+    dec.timed_bytes(reset=True)
+    t_inst_ms, _, _, _ = timed_loop(args.warmup)
     kernel_ms, kernel_n = dec.timing(reset=True)
+    row_timed_bytes = dec.timed_bytes(reset=True)
     dec.set_timing(False)
-    if ws > 1:
-        import torch.distributed as dist
-
-        tt = torch.tensor([t_ms, t_inst_ms], dtype=torch.float64, device=dev)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        t_ms, t_inst_ms = float(tt[0].item()), float(tt[1].item())
+    t_ms, t_inst_ms = max_over_ranks([t_ms, t_inst_ms], ws, dev)
     frames = ws * w.B * w.T * args.steps
     value = frames / (t_ms / 1000.0)
 
@@ -318,28 +378,48 @@ def run_ours(args, w):
     if rank != 0:
         return
     pk, pk_kind = peaks()
-    S = w.T * w.max_sym
     M = w.B * w.beam
     flop_per_launch = 2.0 * M * w.H * (w.V + 1)
     share_joint = kernel_ms["joint"] / max(1e-9, sum(kernel_ms.values()))
+    # In-graph figures: CUDA events at every kernel boundary on the launching
+    # stream over the instrumented pass of the K timed steps.  A kernel timed
+    # inside a long step takes the sustained bf16 peak.
+    joint_ms = kernel_ms["joint"] / max(1, kernel_n["joint"])
+    row_ms = kernel_ms["row"] / max(1, kernel_n["row"])
+    shared_rows = w.V * ((4 if lmA is not None else 0) + (4 if ph is not None else 0))
+    row_launches_with_bias = kernel_n["row"] - args.steps  # the final row pass of a chunk builds no bias
+    row_bytes_graph = row_timed_bytes + shared_rows * max(0, row_launches_with_bias)
     joint_roof = {"kernel": "k_joint_tc: joint GEMM (tcgen05) + fused log-softmax/selection epilogue",
                   "bound": "tensor", "unit": "TFLOP/s",
-                  "achieved": flop_per_launch / (joint_cold / 1000.0) / 1e12,
-                  "achieved_warm_l2": flop_per_launch / (joint_warm / 1000.0) / 1e12,
-                  "peak": pk["bf16_tflops"], "peak_kind": f"{pk_kind} bf16 burst (kernel timed alone)",
+                  "achieved": flop_per_launch / (joint_ms / 1000.0) / 1e12,
+                  "peak": pk["bf16_tflops_sustained"],
+                  "peak_kind": f"{pk_kind} bf16 sustained (kernel timed inside the decode step)",
                   "algorithmic": f"2*M*H*(V+1) = {flop_per_launch:.4g} FLOP per launch (M={M} rows)",
-                  "avg_launch_ms": joint_cold, "avg_launch_ms_warm_l2": joint_warm,
-                  "bytes_per_launch": joint_bytes, "traffic": None,
-                  "share_of_device_time": share_joint}
+                  "avg_launch_ms": joint_ms, "launches": kernel_n["joint"],
+                  "traffic": recorded_traffic(w, "joint"),
+                  "bytes_per_launch": joint_bytes,
+                  "share_of_device_time": share_joint,
+                  "isolated": {"cold_l2_ms": joint_cold, "warm_l2_ms": joint_warm,
+                               "achieved_cold": flop_per_launch / (joint_cold / 1000.0) / 1e12,
+                               "achieved_warm": flop_per_launch / (joint_warm / 1000.0) / 1e12,
+                               "peak": pk["bf16_tflops"], "peak_kind": f"{pk_kind} bf16 burst"}}
     joint_roof["frac"] = joint_roof["achieved"] / joint_roof["peak"]
-    row_roof = {"kernel": "k_row: decision, LM/trie state advance, joint input, fusion bias",
+    row_roof = {"kernel": "k_row_beam" if w.beam > 1 else "k_row",
+                "what": "selection merge, LM/trie state advance, joint input, fusion bias",
                 "bound": "hbm", "unit": "GB/s",
-                "achieved": row_bytes / (row_cold / 1000.0) / 1e9,
-                "achieved_warm_l2": row_bytes / (row_warm / 1000.0) / 1e9,
+                "achieved": row_bytes_graph / (kernel_ms["row"] / 1000.0) / 1e9,
                 "peak": pk["hbm_gbs"], "peak_kind": f"{pk_kind} HBM copy",
-                "algorithmic": f"{row_bytes} B per launch ({M} rows; counted by the kernel, dense bias not counted)",
-                "avg_launch_ms": row_cold, "avg_launch_ms_warm_l2": row_warm, "traffic": None,
-                "share_of_device_time": 1.0 - share_joint}
+                "algorithmic": (f"{row_bytes_graph / max(1, kernel_n['row']):.0f} B per launch on average, "
+                                f"counted by the kernel per evaluated row (partials, row state, label searches, "
+                                f"joint input, every arc of the LM chain levels and trie chain nodes) plus the "
+                                f"shared unigram/root rows once per launch; the dense bias row is not counted"),
+                "avg_launch_ms": row_ms, "launches": kernel_n["row"],
+                "traffic": recorded_traffic(w, "row"),
+                "share_of_device_time": 1.0 - share_joint,
+                "isolated": {"what": "the chunk's last label step replayed with every row evaluated",
+                             "bytes_per_launch": row_bytes, "cold_l2_ms": row_cold, "warm_l2_ms": row_warm,
+                             "achieved_cold": row_bytes / (row_cold / 1000.0) / 1e9,
+                             "achieved_warm": row_bytes / (row_warm / 1000.0) / 1e9}}
     row_roof["frac"] = row_roof["achieved"] / row_roof["peak"]
     # the dominant kernel is the one with the larger device time in the graph
     roof, other = (joint_roof, row_roof) if share_joint >= 0.5 else (row_roof, joint_roof)
@@ -355,9 +435,7 @@ def run_ours(args, w):
             "gpu_launches": int(launches * args.steps),
             "roofline": roof,
             "roofline_other_kernel": other,
-            "in_graph_kernel_ms": {"row": kernel_ms["row"] / max(1, kernel_n["row"]),
-                                   "joint": kernel_ms["joint"] / max(1, kernel_n["joint"]),
-                                   "launches": kernel_n},
+            "latency_per_chunk": latency_stats(step_ms),
             "wall_s_timed_region": wall,
             "value_with_kernel_events": frames / (t_inst_ms / 1000.0),
             "kernel_timing": "per-kernel device time from CUDA events at every kernel boundary inside the "
@@ -382,13 +460,14 @@ def main():
     ap.add_argument("--cpu-streams", type=int, default=None)
     ap.add_argument("--cpu-chunks", type=int, default=None)
     ap.add_argument("--ref-streams", type=int, default=64)
+    ap.add_argument("--streams", type=int, default=None, help="streams B per GPU (default: the config's)")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
-    w = synth.WORKLOADS[args.config]
+    w = workload(args.config, args.streams)
     # bounded CPU samples (about 10-30 s of oracle work on 16 cores)
     cpu_default = {0: (4, 1), 1: (64, 12), 2: (256, 6), 3: (64, 2), 4: (32, 1)}[args.config]
-    args.cpu_streams = args.cpu_streams or cpu_default[0]
+    args.cpu_streams = args.cpu_streams or min(cpu_default[0], w.B)
     args.cpu_chunks = args.cpu_chunks or cpu_default[1]
     if args.impl == "reference":
         run_reference(args, w)

@@ -227,6 +227,13 @@ TSD_API tsd_status tsd_decoder_set_timing(tsd_decoder* dec, int32_t enable);
 TSD_API tsd_status tsd_decoder_timing(tsd_decoder* dec, double* ms, int64_t* launches, int32_t n_classes,
                               int32_t reset);
 
+/* Algorithmic bytes counted by the row passes of timed decode_chunk calls
+ * (set_timing(1)) since the last reset: per evaluated row, its partials, row
+ * state, label searches, joint input and every arc of its LM chain levels and
+ * trie chain nodes (the quantity the row pass's bandwidth roofline divides by
+ * its time).  Waits for the device.  reset != 0 clears the total after reading. */
+TSD_API tsd_status tsd_decoder_timed_bytes(tsd_decoder* dec, int64_t* row_bytes, int32_t reset);
+
 /* Selects the joint GEMM kernel of later decode_chunk calls: 0 (default)
  * the tcgen05 tensor-core kernel, 1 the CUDA-core kernel (a cross-check of
  * the same contraction and epilogue).  Drops captured graphs. */

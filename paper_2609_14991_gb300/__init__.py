@@ -62,6 +62,7 @@ SIGNATURES = {
     "tsd_decoder_set_timing": ([_vp, _i32], _i32),
     "tsd_decoder_timing": ([_vp, _vp, _vp, _i32, _i32], _i32),
     "tsd_decoder_launches_per_chunk": ([_vp, _i32, _i32, _P(_i64)], _i32),
+    "tsd_decoder_timed_bytes": ([_vp, _P(_i64), _i32], _i32),
     "tsd_decoder_debug_capture": ([_vp, _vp, _vp, _i32], _i32),
     "tsd_decoder_set_joint_kernel": ([_vp, _i32], _i32),
     "tsd_decoder_check": ([_vp], _i32),
@@ -328,6 +329,12 @@ class Decoder:
         ln = np.zeros(2, dtype=np.int64)
         _check(lib().tsd_decoder_timing(self.h, ms.ctypes.data, ln.ctypes.data, 2, 1 if reset else 0))
         return {"row": float(ms[0]), "joint": float(ms[1])}, {"row": int(ln[0]), "joint": int(ln[1])}
+
+    def timed_bytes(self, reset: bool = False) -> int:
+        """Algorithmic bytes counted by the row passes of timed chunks."""
+        x = _i64()
+        _check(lib().tsd_decoder_timed_bytes(self.h, ctypes.byref(x), 1 if reset else 0))
+        return x.value
 
     def launches_per_chunk(self, n: int, T: int) -> int:
         x = _i64()

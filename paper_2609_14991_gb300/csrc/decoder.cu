@@ -36,19 +36,25 @@ int steps_per_chunk(const tsd_decoder* d, int T) { return T * d->cfg.max_symbols
 void enqueue_chunk(tsd_decoder* d, int M, int T, cudaStream_t s, const std::vector<cudaEvent_t>* ev) {
   const int S = steps_per_chunk(d, T);
   int e = 0;
+  // timed chunks also count the row passes' algorithmic bytes (second counter)
+  DecView v = d->view;
+  if (ev) {
+    v.count = 1;
+    v.ctr = d->view.ctr + 1;
+  }
   auto mark = [&]() {
     if (ev) cudaEventRecordWithFlags((*ev)[(size_t)e++], s, cudaEventRecordExternal);
   };
-  launch_defaults(d->view, s);
+  launch_defaults(v, s);
   for (int step = 0; step <= S; ++step) {
     const bool pdl = d->pdl && !ev && step > 0;  // the first launch follows the parameter copy
     mark();
-    if (d->cfg.beam_k > 1) launch_row_beam(d->view, M / d->cfg.beam_k, step, step == S ? 1 : 0, d->row_smem, s, pdl);
-    else launch_row(d->view, M, step, step == S ? 1 : 0, d->row_smem, s, pdl);
+    if (d->cfg.beam_k > 1) launch_row_beam(v, M / d->cfg.beam_k, step, step == S ? 1 : 0, d->row_smem, s, pdl);
+    else launch_row(v, M, step, step == S ? 1 : 0, d->row_smem, s, pdl);
     if (step < S) {
       mark();
-      if (d->joint_kind == 0) launch_joint_tc(*d->jtc, d->view, M, step, s, d->pdl && !ev);
-      else launch_joint(d->view, M, step, s);
+      if (d->joint_kind == 0) launch_joint_tc(*d->jtc, v, M, step, s, d->pdl && !ev);
+      else launch_joint(v, M, step, s);
     }
   }
   mark();
@@ -134,7 +140,7 @@ extern "C" tsd_status tsd_decoder_create(const tsd_decoder_cfg* cfg, const void*
   tsd_status st;
   if ((st = A.alloc(&Wt, (size_t)d->N_pad * c.H)) || (st = A.alloc(&E, (size_t)d->N * c.H)) ||
       (st = A.alloc(&Abuf, (size_t)d->M_pad * c.H)) || (st = A.alloc(&bias, (size_t)d->M_pad * d->N_pad)) ||
-      (st = A.alloc(&part, (size_t)d->M_pad * (d->N_pad / 64))) || (st = A.alloc(&err, 1)) || (st = A.alloc(&ctr, 1)) || (st = A.alloc(&dflt, (size_t)c.V)) || (st = A.alloc(&rt, (size_t)d->M_pad)) ||
+      (st = A.alloc(&part, (size_t)d->M_pad * (d->N_pad / 64))) || (st = A.alloc(&err, 1)) || (st = A.alloc(&ctr, 2)) || (st = A.alloc(&dflt, (size_t)c.V)) || (st = A.alloc(&rt, (size_t)d->M_pad)) ||
       (st = A.alloc(&rs, (size_t)d->M_pad)) || (st = A.alloc(&rc, (size_t)d->M_pad)) ||
       (st = A.alloc(&sl, SK)) || (st = A.alloc(&sll, SK)) || (st = A.alloc(&slc, SK * kLmChain)) ||
       (st = A.alloc(&stl, SK)) || (st = A.alloc(&stc, SK * kTrChain)) || (st = A.alloc(&pdev, d->params_bytes))) {
@@ -172,7 +178,7 @@ extern "C" tsd_status tsd_decoder_create(const tsd_decoder_cfg* cfg, const void*
       (ce = cudaMemsetAsync(sll, 0, sizeof(int32_t) * SK, s)) != cudaSuccess ||
       (ce = cudaMemsetAsync(stl, 0, sizeof(int32_t) * SK, s)) != cudaSuccess ||
       (ce = cudaMemsetAsync(err, 0, sizeof(int32_t), s)) != cudaSuccess ||
-      (ce = cudaMemsetAsync(ctr, 0, sizeof(unsigned long long), s)) != cudaSuccess ||
+      (ce = cudaMemsetAsync(ctr, 0, 2 * sizeof(unsigned long long), s)) != cudaSuccess ||
       (ce = cudaMemcpyAsync(E, E_bf16, sizeof(uint16_t) * (size_t)d->N * c.H, cudaMemcpyDeviceToDevice, s)) != cudaSuccess)
     return cleanup(cuda_fail(ce, "tsd_decoder_create: initial copies"));
   launch_repack(static_cast<const uint16_t*>(W_out_bf16), Wt, c.H, d->N, d->N_pad, s);
@@ -234,6 +240,7 @@ extern "C" tsd_status tsd_decoder_create(const tsd_decoder_cfg* cfg, const void*
   v.cap_steps = 0;
   v.err = err;
   v.ctr = ctr;
+  v.count = 0;
   v.dflt = dflt;
   v.bpart = bpart;
   v.h_score = hscore;
@@ -527,6 +534,19 @@ extern "C" tsd_status tsd_decoder_timing(tsd_decoder* d, double* ms, int64_t* la
     d->ms[0] = d->ms[1] = 0;
     d->launches[0] = d->launches[1] = 0;
   }
+  return TSD_OK;
+}
+
+extern "C" tsd_status tsd_decoder_timed_bytes(tsd_decoder* d, int64_t* row_bytes, int32_t reset) {
+  clear_error();
+  if (!d || !row_bytes) return fail(TSD_EINVAL, "tsd_decoder_timed_bytes: NULL argument");
+  tsd_status st = set_device(d);
+  if (st) return st;
+  TSD_CUDA(cudaStreamSynchronize(d->last_stream));
+  unsigned long long b = 0;
+  TSD_CUDA(cudaMemcpy(&b, d->view.ctr + 1, sizeof(b), cudaMemcpyDeviceToHost));
+  *row_bytes = (int64_t)b;
+  if (reset) TSD_CUDA(cudaMemset(d->view.ctr + 1, 0, sizeof(b)));
   return TSD_OK;
 }
 

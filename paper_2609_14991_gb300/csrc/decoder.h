@@ -61,7 +61,8 @@ struct DecView {
   int32_t pool_cap;
   float2* dflt;  // [V] per-call bias defaults (lambda*log p(v), beta*bonus*[root child v])
   int32_t* err;  // device status word: nonzero after a bounded wait expired
-  unsigned long long* ctr;  // algorithmic bytes counted by replayed row passes
+  unsigned long long* ctr;  // algorithmic bytes counted by row passes (replayed or timed)
+  int32_t count;            // 1: every row pass adds its algorithmic bytes to *ctr
 };
 
 constexpr int kRowThreads = 256;

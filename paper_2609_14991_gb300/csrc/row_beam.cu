@@ -417,13 +417,23 @@ __global__ void __launch_bounds__(kRowThreads) k_row_beam(DecView d, int step, i
 
   // 6. joint input and fusion bias of every survivor for frame `step`
   const uint16_t* enc_row = P->enc + ((size_t)b * T + min(step, T - 1)) * d.H;
+  // Algorithmic bytes (counted when timing): the K hypotheses' partials and
+  // state, and per survivor its joint input and every arc of its LM chain
+  // levels and trie chain nodes with their records.
+  unsigned long long bytes = (unsigned long long)K * (d.n_ptiles * (1 + K) * 8 + 64);
   for (int j = 0; j < cnt; ++j) {
     const int r = b * K + j;
     row::bias_prepare(d, n_lm[j], n_lml[j], n_tr[j], n_trl[j], rc, lmv, dep);
     row::build_joint_input(d, enc_row, n_last[j], r);
     row::bias_finish(d, n_lml[j], n_trl[j], rc, P->lambda, P->beta, d.bias + (size_t)r * d.N_pad, lmv, dep);
+    if ((mode == 2 || d.count) && tid == 0) {
+      bytes += 6ull * d.H;
+      for (int l = 0; l < n_lml[j]; ++l) bytes += 12 + 8ull * rc.lc[l];
+      for (int k = 0; k < n_trl[j]; ++k) bytes += 12 + 4ull * rc.tc[k];
+    }
     __syncthreads();  // the scratch is reused by the next survivor
   }
+  if ((mode == 2 || d.count) && tid == 0) atomicAdd(d.ctr, bytes);
 }
 
 __global__ void k_open_beam(DecView d, int slot) {

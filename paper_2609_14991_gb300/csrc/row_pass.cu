@@ -229,7 +229,7 @@ __global__ void __launch_bounds__(kRowThreads, 8) k_row(DecView d, int step, int
   row::bias_prepare(d, s_lm, nl, s_tr, nt, rc, lmv, dep);
   row::build_joint_input(d, s_enc + ((size_t)r * T + t) * d.H, s_last, r);
   row::bias_finish(d, nl, nt, rc, s_lam, s_beta, d.bias + (size_t)r * d.N_pad, lmv, dep);
-  if (mode == 2 && tid == 0) {
+  if ((mode == 2 || d.count) && tid == 0) {
     // Algorithmic bytes of this row-step: selection partials, row state,
     // the searches of the emitted label (one probe per halving plus the arc
     // it found), the joint input (encoder frame and embedding row read, A
