@@ -130,7 +130,8 @@ extern "C" tsd_status tsd_decoder_create(const tsd_decoder_cfg* cfg, const void*
   int32_t *rt, *rs, *rc, *sl, *sll, *slc, *stl, *stc, *err;
   unsigned long long* ctr;
   float2* bpart = nullptr;
-  float2* dflt = nullptr;
+  float* dflt = nullptr;
+  uint32_t* droot = nullptr;
   double* hscore = nullptr;
   int32_t *hlive = nullptr, *hnode = nullptr, *hlen = nullptr, *ppar = nullptr, *ptok = nullptr, *pn = nullptr;
   unsigned long long* hhash = nullptr;
@@ -140,7 +141,7 @@ extern "C" tsd_status tsd_decoder_create(const tsd_decoder_cfg* cfg, const void*
   tsd_status st;
   if ((st = A.alloc(&Wt, (size_t)d->N_pad * c.H)) || (st = A.alloc(&E, (size_t)d->N * c.H)) ||
       (st = A.alloc(&Abuf, (size_t)d->M_pad * c.H)) || (st = A.alloc(&bias, (size_t)d->M_pad * d->N_pad)) ||
-      (st = A.alloc(&part, (size_t)d->M_pad * (d->N_pad / 64))) || (st = A.alloc(&err, 1)) || (st = A.alloc(&ctr, 2)) || (st = A.alloc(&dflt, (size_t)c.V)) || (st = A.alloc(&rt, (size_t)d->M_pad)) ||
+      (st = A.alloc(&part, (size_t)d->M_pad * (d->N_pad / 64))) || (st = A.alloc(&err, 1)) || (st = A.alloc(&ctr, 2)) || (st = A.alloc(&dflt, (size_t)d->V4)) || (st = A.alloc(&droot, (size_t)(d->V4 + 31) / 32)) || (st = A.alloc(&rt, (size_t)d->M_pad)) ||
       (st = A.alloc(&rs, (size_t)d->M_pad)) || (st = A.alloc(&rc, (size_t)d->M_pad)) ||
       (st = A.alloc(&sl, SK)) || (st = A.alloc(&sll, SK)) || (st = A.alloc(&slc, SK * kLmChain)) ||
       (st = A.alloc(&stl, SK)) || (st = A.alloc(&stc, SK * kTrChain)) || (st = A.alloc(&pdev, d->params_bytes))) {
@@ -242,6 +243,7 @@ extern "C" tsd_status tsd_decoder_create(const tsd_decoder_cfg* cfg, const void*
   v.ctr = ctr;
   v.count = 0;
   v.dflt = dflt;
+  v.droot = droot;
   v.bpart = bpart;
   v.h_score = hscore;
   v.h_live = hlive;

@@ -59,7 +59,8 @@ struct DecView {
   int32_t* pool_tok;    // [slots][pool_cap] label of the node
   int32_t* pool_n;      // [slots] nodes used
   int32_t pool_cap;
-  float2* dflt;  // [V] per-call bias defaults (lambda*log p(v), beta*bonus*[root child v])
+  float* dflt;        // [V4] per-call LM bias default lambda*log p(v) (0 past V)
+  uint32_t* droot;    // [ceil(V4/32)] bit v: the trie root has a child labelled v
   int32_t* err;  // device status word: nonzero after a bounded wait expired
   unsigned long long* ctr;  // algorithmic bytes counted by row passes (replayed or timed)
   int32_t count;            // 1: every row pass adds its algorithmic bytes to *ctr

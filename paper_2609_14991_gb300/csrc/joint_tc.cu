@@ -5,14 +5,15 @@
 // Wt (W_out label-major, bf16 [N_pad][H]) are both K-major, loaded by TMA
 // into 128-byte-swizzled shared-memory stages; one elected thread issues
 // tcgen05.mma (kind::f16, bf16 x bf16 -> fp32) into a 128 x BN accumulator in
-// tensor memory.  Four epilogue warps read the accumulator back with
-// tcgen05.ld (thread = row) and reduce it on chip to the row's selection
-// partial for this tile: softmax max and sum over the real labels, and the
-// best fused value logit + bias (lambda*LM + beta*boost; blank gets 0), ties
-// to the lowest label.  Logits never leave the SM.
+// tensor memory.  Eight epilogue warps read the accumulator back with
+// tcgen05.ld (thread = row; two warps per 32-lane quadrant take alternate
+// 32-column chunks) and reduce it on chip to the row's selection partial for
+// this tile: softmax max and sum over the real labels, and the best fused
+// value logit + bias (lambda*LM + beta*boost; blank gets 0), ties to the
+// lowest label.  Logits never leave the SM.
 //
-// Warp roles (192 threads): warp 0 TMA producer, warp 1 TMEM allocator and
-// MMA issuer, warps 2-5 epilogue.  Every wait on an mbarrier is bounded in
+// Warp roles (320 threads): warp 0 TMA producer, warp 1 TMEM allocator and
+// MMA issuer, warps 2-9 epilogue.  Every wait on an mbarrier is bounded in
 // time; on expiry the kernel records an error in the decoder's status word,
 // drains its own copies and returns.
 #include <cuda.h>
@@ -25,7 +26,8 @@ namespace tsd {
 namespace {
 
 constexpr int kBM = 128, kBK = 64;
-constexpr int kThreads = 192;
+constexpr int kThreads = 320;
+constexpr int kEpiThreads = 256;  // warps 2-9
 constexpr float kNegInf = -__builtin_huge_valf();
 constexpr unsigned long long kWaitNs = 1000000000ull;  // 1 s bound on any barrier wait
 constexpr float kLog2e = 1.4426950408889634f;
@@ -154,6 +156,8 @@ struct Smem {
   static constexpr int kBiasBytes = kEarly * kBoxBytes;
   static constexpr int kBytes = kStages * kStageBytes + kBiasBytes + 1024 /*align*/ + 256 /*barriers*/;
   static_assert((kBoxes - kEarly) * kBoxBytes <= kStages * kStageBytes, "late bias boxes fit the stages");
+  // the epilogue halves' exchange (per row 18 floats, 4 flags) after the late boxes
+  static_assert((kBoxes - kEarly) * kBoxBytes + kBM * 18 * 4 + 16 <= kStages * kStageBytes, "exchange fits");
 };
 
 // BEAM: instead of the single best fused label, each row keeps the top-K
@@ -198,6 +202,15 @@ __global__ void __launch_bounds__(kThreads, 1)
   fence_after();
   const uint32_t tmem = *tmem_slot;
   bool ok = true;
+  // W_out is constant, so the first stages' W_out tiles are requested before
+  // the dependency wait (each stage's barrier expects its A tile as well).
+  const int pre = min(KB, S::kStages);
+  if (warp == 0 && lane == 0) {
+    for (int kb = 0; kb < pre; ++kb) {
+      mbar_expect_tx(full + kb, S::kStageBytes);
+      tma_load_2d(smem + kb * S::kStageBytes + S::kABytes, &tmB, full + kb, kb * kBK, n0);
+    }
+  }
   // Programmatic dependent launch: the set-up above overlaps the row pass;
   // its outputs (joint input, bias) are read only after the wait.  The next
   // row pass may launch once every CTA is past this point.
@@ -213,8 +226,13 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int kb = 0; kb < KB; ++kb) {
         const int s = kb % S::kStages;
         const uint32_t ph = (uint32_t)(kb / S::kStages) & 1u;
-        if (!mbar_wait(empty + s, ph ^ 1u)) { ok = false; break; }
         unsigned char* sa = smem + s * S::kStageBytes;
+        if (kb < pre) {  // first use of the stage: W_out already requested
+          tma_load_2d(sa, &tmA, full + s, kb * kBK, m0);
+          ++issued;
+          continue;
+        }
+        if (!mbar_wait(empty + s, ph ^ 1u)) { ok = false; break; }
         mbar_expect_tx(full + s, S::kStageBytes);
         tma_load_2d(sa, &tmA, full + s, kb * kBK, m0);
         tma_load_2d(sa + S::kABytes, &tmB, full + s, kb * kBK, n0);
@@ -250,8 +268,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     __syncwarp();
   } else {
-    // epilogue: warps 2..5, thread = row of the tile
+    // epilogue: warps 2..9, thread = row of the tile; the two warps of a
+    // TMEM lane quadrant take alternate 32-column chunks
     const int q = warp & 3;  // TMEM lane quadrant this warp may access
+    const int half = (warp - 2) >> 2;
     const int row = q * 32 + lane;
     const int gr = m0 + row;
     const bool live = gr < M;
@@ -285,8 +305,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint32_t tbase = tmem + ((uint32_t)(q * 32) << 16);
       const int sw = row & 7;  // 128-byte swizzle: 16-byte chunk j of a row sits at j ^ (row % 8)
 #pragma unroll 1
-      for (int c = 0; c < BN / 32; ++c) {
-        if (c == S::kEarly) {
+      for (int c = half; c < BN / 32; c += 2) {
+        __syncwarp();  // the per-chunk selection branches; tcgen05.ld wants the warp whole
+        if (c >= S::kEarly && !late_done) {
           late_done = true;
           if (!__all_sync(0xffffffffu, mbar_wait(biasbar + 1, 0))) {
             if (lane == 0) atomicOr(d.err, 32);
@@ -370,20 +391,73 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (c0 + i < N) cl[c0 + i] = l[i];
         }
       }
-      if (live) {
-        if (!BEAM) {
-          d.part[(size_t)gr * d.n_ptiles + blockIdx.x] = make_float4(mx, se, bv, __int_as_float(bi));
-        } else {
-          float2* bp = d.bpart + ((size_t)gr * d.n_ptiles + blockIdx.x) * (1 + K);
-          bp[0] = make_float2(mx, se);
-#pragma unroll
-          for (int j = 0; j < 8; ++j)
-            if (j < K) bp[1 + j] = make_float2(tv[j], __int_as_float(ti[j]));
-        }
-      }
     }
     // never leave with bias boxes still landing in shared memory
     if (!late_done && warp == 2 && lane == 0) mbar_wait(biasbar + 1, 0);
+    // Merge the two halves' partials of each row: the second half leaves its
+    // partial in shared memory past the late bias boxes (the stages are
+    // drained: every MMA has completed), the first half combines and stores.
+    float* xbase = reinterpret_cast<float*>(smem + (S::kBoxes - S::kEarly) * S::kBoxBytes);
+    float* xch = xbase + row * 18;  // (max, sum, then best or top-8 (value, label))
+    int* xok = reinterpret_cast<int*>(xbase + kBM * 18);  // per quadrant: the second half finished
+    if (half == 1) {
+      if (ok) {
+        xch[0] = mx;
+        xch[1] = se;
+        if (!BEAM) {
+          xch[2] = bv;
+          xch[3] = __int_as_float(bi);
+        } else {
+#pragma unroll
+          for (int j = 0; j < 8; ++j) { xch[2 + 2 * j] = tv[j]; xch[3 + 2 * j] = __int_as_float(ti[j]); }
+        }
+      }
+      if (lane == 0) xok[q] = ok ? 1 : 0;
+    }
+    asm volatile("bar.sync 1, %0;" ::"n"(kEpiThreads) : "memory");
+    if (half == 0 && ok && xok[q] && live) {
+      const float m1 = xch[0], s1 = xch[1];
+      if (m1 != kNegInf) {
+        if (mx == kNegInf) { mx = m1; se = s1; }
+        else {
+          const float m2 = fmaxf(mx, m1);
+          se = se * ex2_approx((mx - m2) * kLog2e) + s1 * ex2_approx((m1 - m2) * kLog2e);
+          mx = m2;
+        }
+      }
+      if (!BEAM) {
+        const float v1 = xch[2];
+        const int i1 = __float_as_int(xch[3]);
+        if (v1 > bv || (v1 == bv && i1 < bi)) { bv = v1; bi = i1; }
+        d.part[(size_t)gr * d.n_ptiles + blockIdx.x] = make_float4(mx, se, bv, __int_as_float(bi));
+      } else {
+        // merge two lists sorted by (value desc, label asc): an entry's
+        // place is its index plus the other list's entries ordered before it
+        // (unfilled entries (-inf, INT_MAX) of both lists land on the same
+        // trailing places with the same contents)
+        float2* bp = d.bpart + ((size_t)gr * d.n_ptiles + blockIdx.x) * (1 + K);
+        bp[0] = make_float2(mx, se);
+        float ov[8];
+        int oi[8];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) { ov[j] = xch[2 + 2 * j]; oi[j] = __float_as_int(xch[3 + 2 * j]); }
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          if (i < K) {
+            int pa = i, pb = i;
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+              if (j < K) {
+                pa += (ov[j] > tv[i] || (ov[j] == tv[i] && oi[j] < ti[i])) ? 1 : 0;
+                pb += (tv[j] > ov[i] || (tv[j] == ov[i] && ti[j] < oi[i])) ? 1 : 0;
+              }
+            }
+            if (pa < K) bp[1 + pa] = make_float2(tv[i], __int_as_float(ti[i]));
+            if (pb < K) bp[1 + pb] = make_float2(ov[i], __int_as_float(oi[i]));
+          }
+        }
+      }
+    }
   }
   fence_before();
   __syncthreads();

@@ -105,7 +105,7 @@ __global__ void __launch_bounds__(kRowThreads) k_row_beam(DecView d, int step, i
     s_slot = __ldcg(P->slots + b);
     s_T = __ldcg(&P->T);
   }
-  __syncthreads();
+  row::block_sync();
   const int slot = s_slot, T = s_T;
   const int hb = slot * K;
   const int cap = d.pool_cap;
@@ -122,7 +122,7 @@ __global__ void __launch_bounds__(kRowThreads) k_row_beam(DecView d, int step, i
     o_lml[tid] = d.has_lm ? __ldcg(d.s_lm_len + h) : 0;
     o_trl[tid] = d.has_tr ? __ldcg(d.s_tr_len + h) : 0;
   }
-  __syncthreads();
+  row::block_sync();
   for (int i = tid; i < K * kLmChain; i += kRowThreads) {
     const int k = i / kLmChain, l = i % kLmChain;
     if (l < o_lml[k]) o_lm[k][l] = __ldcg(d.s_lm_chain + (size_t)(hb + k) * kLmChain + l);
@@ -131,7 +131,7 @@ __global__ void __launch_bounds__(kRowThreads) k_row_beam(DecView d, int step, i
     const int k = i / kTrChain, l = i % kTrChain;
     if (l < o_trl[k]) o_tr[k][l] = __ldcg(d.s_tr_chain + (size_t)(hb + k) * kTrChain + l);
   }
-  __syncthreads();
+  row::block_sync();
   asm volatile("griddepcontrol.wait;" ::: "memory");
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
@@ -149,6 +149,7 @@ __global__ void __launch_bounds__(kRowThreads) k_row_beam(DecView d, int step, i
           lse_merge(m, s, p.x, p.y);
         }
       }
+      row::reconverge();
 #pragma unroll
       for (int o = 16; o > 0; o >>= 1) {
         const float m2 = __shfl_xor_sync(0xffffffffu, m, o), s2 = __shfl_xor_sync(0xffffffffu, s, o);
@@ -170,6 +171,7 @@ __global__ void __launch_bounds__(kRowThreads) k_row_beam(DecView d, int step, i
         }
       }
       for (int round = 0; round < K; ++round) {
+        row::reconverge();
         // this lane's best remaining (value desc, label asc)
         float bv = kNegInf;
         int bt = INT_MAX, bq = -1;
@@ -198,7 +200,7 @@ __global__ void __launch_bounds__(kRowThreads) k_row_beam(DecView d, int step, i
         }
       }
     }
-    __syncthreads();
+    row::block_sync();
     // 2. global top K, then merge equal label sequences
     if (tid == 0) {
       bool used[kMaxK * kMaxK];
@@ -281,7 +283,7 @@ __global__ void __launch_bounds__(kRowThreads) k_row_beam(DecView d, int step, i
         }
       }
     }
-    __syncthreads();
+    row::block_sync();
     // 3. searches of each survivor's label in its parent's chains
     const int cnt = n_cnt;
     if (tid >= kRowThreads - kMaxK) {
@@ -314,7 +316,7 @@ __global__ void __launch_bounds__(kRowThreads) k_row_beam(DecView d, int step, i
         }
       }
     }
-    __syncthreads();
+    row::block_sync();
     // 4. survivors' chains (thread j for survivor j)
     if (tid < cnt) {
       const int j = tid, p = n_par[j], y = n_tok[j];
@@ -353,7 +355,7 @@ __global__ void __launch_bounds__(kRowThreads) k_row_beam(DecView d, int step, i
         n_trl[j] = tn;
       }
     }
-    __syncthreads();
+    row::block_sync();
   } else {
     // frame 0 of the chunk: the hypotheses carried over from the last chunk
     if (tid == 0) {
@@ -375,7 +377,7 @@ __global__ void __launch_bounds__(kRowThreads) k_row_beam(DecView d, int step, i
       for (int l = 0; l < o_lml[k]; ++l) n_lm[k][l] = o_lm[k][l];
       for (int l = 0; l < o_trl[k]; ++l) n_tr[k][l] = o_tr[k][l];
     }
-    __syncthreads();
+    row::block_sync();
   }
   const int cnt = n_cnt;
 
@@ -431,7 +433,7 @@ __global__ void __launch_bounds__(kRowThreads) k_row_beam(DecView d, int step, i
       for (int l = 0; l < n_lml[j]; ++l) bytes += 12 + 8ull * rc.lc[l];
       for (int k = 0; k < n_trl[j]; ++k) bytes += 12 + 4ull * rc.tc[k];
     }
-    __syncthreads();  // the scratch is reused by the next survivor
+    row::block_sync();  // the scratch is reused by the next survivor
   }
   if ((mode == 2 || d.count) && tid == 0) atomicAdd(d.ctr, bytes);
 }

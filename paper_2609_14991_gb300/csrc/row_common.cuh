@@ -8,8 +8,31 @@ namespace row {
 
 constexpr float kNegInf = -__builtin_huge_valf();
 
+// After divergent code (a single-thread section, a lane-strided loop) the
+// lanes of a warp can keep running apart past the point where they could
+// rejoin, and every warp-synchronous step after it (shuffle, ballot) then
+// costs about ten times as much.  These force the warp back together.
+__device__ __forceinline__ void reconverge() { __syncwarp(); }
+__device__ __forceinline__ void block_sync() {
+  __syncthreads();
+  __syncwarp();
+}
+
+// Requests the 128-byte line holding p into L1 (no result, no fault on a
+// valid address); later loads of it then wait for L1 rather than L2.
+__device__ __forceinline__ void prefetch_l1(const void* p) {
+  asm volatile("prefetch.global.L1 [%0];" ::"l"(p));
+}
+
+// Lines [0, bytes) from base, one line per thread of the block from `first`.
+__device__ __forceinline__ void prefetch_span(const void* base, size_t bytes, int first) {
+  const int i = (int)threadIdx.x - first;
+  if (i >= 0 && (size_t)i * 128 < bytes) prefetch_l1(static_cast<const char*>(base) + (size_t)i * 128);
+}
+
 // Position of y in the sorted arr[0, n), or -1: a 32-ary search by one warp.
 __device__ __forceinline__ int warp_find(const int32_t* __restrict__ arr, int n, int y, int lane) {
+  reconverge();
   int lo = 0, hi = n;
   while (hi - lo > 32) {
     int step = (hi - lo + 31) >> 5;
@@ -94,9 +117,11 @@ __device__ __forceinline__ void bias_prepare(const DecView& d, const int* lm_cha
     rc.td[tid - 32] = __ldg(d.tr.nd_depth + q) + 1;
   }
   const float unset = unset_value();
-  for (int v = tid; v < d.V; v += blockDim.x) {
-    lmv[v] = unset;
-    dep[v] = 0;
+  float4* l4 = reinterpret_cast<float4*>(lmv);
+  uint32_t* d4 = reinterpret_cast<uint32_t*>(dep);
+  for (int q = tid; q < d.V4 / 4; q += blockDim.x) {  // V4 is a multiple of 16
+    l4[q] = make_float4(unset, unset, unset, unset);
+    d4[q] = 0u;
   }
 }
 
@@ -105,13 +130,13 @@ __device__ __forceinline__ void bias_prepare(const DecView& d, const int* lm_cha
 // LM chain levels are applied deepest first, each label keeping the first
 // value it gets; trie chain nodes shallowest first, the deepest node's child
 // depth overwriting.  One barrier per level.  Labels no level touches take
-// the call's defaults dflt[v] = (lambda*log p(v), beta*bonus*[root has v]).
+// the call's defaults lambda*log p(v) and beta*bonus*[the root has a child v].
 __device__ __forceinline__ void bias_finish(const DecView& d, int nl, int nt, const ChainRecs& rc, float lam,
                                             float beta, float* brow, float* lmv, uint8_t* dep) {
   const int tid = threadIdx.x;
   const int V = d.V;
   const int step = blockDim.x;
-  __syncthreads();
+  block_sync();
   const float cum_top = nl ? rc.lo[nl - 1] : 0.f;
   const int phases = max(nl, nt);
   for (int p = 0; p < phases; ++p) {
@@ -144,36 +169,48 @@ __device__ __forceinline__ void bias_finish(const DecView& d, int nl, int nt, co
       const uint8_t dd = (uint8_t)rc.td[k];
       for (int j = tid; j < c; j += step) dep[__ldg(d.tr.ch_tok + b + j)] = dd;
     }
-    __syncthreads();
+    block_sync();
   }
   const int depth_cur = nt ? rc.td[0] - 1 : 0;
   const float bscale = beta * (d.has_tr ? d.tr.bonus : 0.f);
-  const float base = lam * cum_top - bscale * (float)depth_cur;
-  const float2* dflt = d.dflt;
-  int v = tid;
-  for (; v + 3 * step < V; v += 4 * step) {  // four labels' defaults in flight
-    float2 df[4];
+  const float lm_base = lam * cum_top;
+  const float tr_base = -bscale * (float)depth_cur;
+  // four consecutive labels per thread: one 16-byte load of the defaults and
+  // of the LM scratch, one 4-byte load of the trie scratch, one 16-byte store
+  const float4* df4 = reinterpret_cast<const float4*>(d.dflt);
+  const float4* l4 = reinterpret_cast<const float4*>(lmv);
+  const uint32_t* d4 = reinterpret_cast<const uint32_t*>(dep);
+  float4* b4 = reinterpret_cast<float4*>(brow);
+  const int nq = d.V4 / 4;
+  auto quad = [&](int q, float4 df, uint32_t rootw) {
+    const float4 l = l4[q];
+    const uint32_t dd = d4[q];
+    const uint32_t rb = rootw >> ((4 * q) & 31);
+    const float lv[4] = {l.x, l.y, l.z, l.w};
+    const float dv[4] = {df.x, df.y, df.z, df.w};
+    float o[4];
 #pragma unroll
-    for (int q = 0; q < 4; ++q) df[q] = __ldcg(dflt + v + q * step);
-#pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      const int u = v + q * step;
-      const float l = lmv[u];
-      const int dd = dep[u];
-      const float blm = isnan(l) ? df[q].x + lam * cum_top : lam * l;
-      const float btr = dd ? bscale * (float)(dd - depth_cur) : df[q].y - bscale * (float)depth_cur;
-      brow[u] = blm + btr;
+    for (int j = 0; j < 4; ++j) {
+      const int dj = (dd >> (8 * j)) & 0xff;
+      const float blm = isnan(lv[j]) ? dv[j] + lm_base : lam * lv[j];
+      const float btr = dj ? bscale * (float)(dj - depth_cur) : (((rb >> j) & 1u) ? bscale : 0.f) + tr_base;
+      o[j] = (4 * q + j < V) ? blm + btr : 0.f;
     }
+    b4[q] = make_float4(o[0], o[1], o[2], o[3]);
+  };
+  int q = tid;
+  for (; q + step < nq; q += 2 * step) {  // two quads' loads in flight
+    float4 df[2];
+    uint32_t rw[2];
+#pragma unroll
+    for (int k = 0; k < 2; ++k) {
+      df[k] = __ldg(df4 + q + k * step);
+      rw[k] = __ldg(d.droot + ((q + k * step) >> 3));
+    }
+#pragma unroll
+    for (int k = 0; k < 2; ++k) quad(q + k * step, df[k], rw[k]);
   }
-  for (; v < V; v += step) {
-    const float2 df = __ldcg(dflt + v);
-    const float l = lmv[v];
-    const int dd = dep[v];
-    const float blm = isnan(l) ? df.x + lam * cum_top : lam * l;
-    const float btr = dd ? bscale * (float)(dd - depth_cur) : df.y - bscale * (float)depth_cur;
-    brow[v] = blm + btr;
-  }
-  (void)base;
+  for (; q < nq; q += step) quad(q, __ldg(df4 + q), __ldg(d.droot + (q >> 3)));
   if (tid == 0) brow[V] = 0.f;
 }
 

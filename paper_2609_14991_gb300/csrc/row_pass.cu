@@ -28,7 +28,7 @@ using row::warp_find;
 // mode: 0 = label step, 1 = final step (apply the last decision only),
 // 2 = replay (redo the step's work without committing any state or output;
 // used only to time the kernel in isolation).
-__global__ void __launch_bounds__(kRowThreads, 8) k_row(DecView d, int step, int mode) {
+__global__ void __launch_bounds__(kRowThreads, 7) k_row(DecView d, int step, int mode) {
   const Params* __restrict__ P = d.params;
   const int r = blockIdx.x;
   const int V = d.V;
@@ -79,11 +79,20 @@ __global__ void __launch_bounds__(kRowThreads, 8) k_row(DecView d, int step, int
     s_tr_len = d.has_tr ? __ldcg(d.s_tr_len + slot) : 0;
     s_last = __ldcg(d.s_last + slot);
   }
-  __syncthreads();
+  row::block_sync();
   const int slot = s_slot, T = s_T;
   if (tid < s_lm_len) s_lm[tid] = __ldcg(d.s_lm_chain + slot * kLmChain + tid);
   if (tid >= 64 && tid - 64 < s_tr_len) s_tr[tid - 64] = __ldcg(d.s_tr_chain + slot * kTrChain + tid - 64);
-  __syncthreads();
+  // The encoder frames this step can use (t, or t+1 after a frame advance)
+  // go to L1 now, while the previous kernel still runs: no kernel of the
+  // chunk writes them.  (The call's bias defaults are not prefetched: every
+  // row would ask the same L2 lines for them at once.)
+  if (s_t < T) {
+    const size_t fb = (size_t)d.H * 2;
+    const uint16_t* f0 = s_enc + ((size_t)r * T + s_t) * d.H;
+    row::prefetch_span(f0, s_t + 1 < T ? 2 * fb : fb, 0);
+  }
+  row::block_sync();
   // In replay mode every row redoes a full step (decision, advance, joint
   // input, bias) even if it had finished the chunk, so the timing is that of
   // a mid-chunk step.
@@ -105,6 +114,7 @@ __global__ void __launch_bounds__(kRowThreads, 8) k_row(DecView d, int step, int
         lse_merge(m, s, p.x, p.y);
         best_merge(bv, bi, p.z, __float_as_int(p.w));
       }
+      row::reconverge();
       for (int o = 16; o > 0; o >>= 1) {
         float m2 = __shfl_xor_sync(0xffffffffu, m, o);
         float s2 = __shfl_xor_sync(0xffffffffu, s, o);
@@ -118,8 +128,9 @@ __global__ void __launch_bounds__(kRowThreads, 8) k_row(DecView d, int step, int
         s_score = bv - (m + logf(s));
       }
     }
-    __syncthreads();
+    row::block_sync();
     const int y = s_y;
+    row::prefetch_span(d.E + (size_t)(y != V ? y : s_last) * d.H, (size_t)d.H * 2, 32);  // this step's E row
     if (y != V) {
       // 2a. independent searches of y in every chain element, each warp
       //     also fetching what the new chain needs from the arc it found
@@ -134,7 +145,15 @@ __global__ void __launch_bounds__(kRowThreads, 8) k_row(DecView d, int step, int
           int st = s_lm[task];
           int b = __ldg(d.lm.st_begin + st), c = __ldg(d.lm.st_count + st);
           int i = warp_find(d.lm.arc_tok + b, c, y, lane);
-          if (lane == 0) s_lm_tgt[task] = (i >= 0) ? __ldg(d.lm.arc_tgt + b + i) : -2;
+          if (lane == 0) {
+            const int tg = (i >= 0) ? __ldg(d.lm.arc_tgt + b + i) : -2;
+            s_lm_tgt[task] = tg;
+            if (tg >= 0) {  // the new chain's state records
+              row::prefetch_l1(d.lm.st_begin + tg);
+              row::prefetch_l1(d.lm.st_count + tg);
+              row::prefetch_l1(d.lm.st_cum + tg);
+            }
+          }
         } else {
           int k = task - nl;
           int q = s_tr[k];
@@ -142,11 +161,17 @@ __global__ void __launch_bounds__(kRowThreads, 8) k_row(DecView d, int step, int
           int i = warp_find(d.tr.ch_tok + b, c, y, lane);
           if (lane == 0) {
             s_tr_node[k] = (i >= 0) ? __ldg(d.tr.ch_node + b + i) : -1;
+            if (i >= 0) {
+              const int nd = s_tr_node[k];
+              row::prefetch_l1(d.tr.nd_begin + nd);
+              row::prefetch_l1(d.tr.nd_count + nd);
+              row::prefetch_l1(d.tr.nd_depth + nd);
+            }
             s_tr_nxt[k] = (i >= 0) ? __ldg(d.tr.ch_next + b + i) : -1;
           }
         }
       }
-      __syncthreads();
+      row::block_sync();
       // 2b. assemble the new chains (shared memory only) and emit
       if (tid == 0) {
         int newlm[kLmChain];
@@ -197,7 +222,7 @@ __global__ void __launch_bounds__(kRowThreads, 8) k_row(DecView d, int step, int
       s_t += 1;
       s_sym = 0;
     }
-    __syncthreads();
+    row::block_sync();
   }
 
   if (mode == 1) {
@@ -264,7 +289,7 @@ __global__ void k_repack(const uint16_t* __restrict__ W, uint16_t* __restrict__ 
     int k = k0 + i, v = v0 + tx;
     tile[i][tx] = (k < H && v < N) ? W[(size_t)k * N + v] : (uint16_t)0;
   }
-  __syncthreads();
+  row::block_sync();
   for (int i = ty; i < 32; i += 8) {
     int v = v0 + i, k = k0 + tx;
     if (v < N_pad && k < H) Wt[(size_t)v * H + k] = tile[tx][i];
@@ -276,21 +301,28 @@ __global__ void k_repack(const uint16_t* __restrict__ W, uint16_t* __restrict__ 
 size_t row_smem_bytes(int V4) { return (size_t)V4 * (sizeof(float) + sizeof(uint8_t)); }
 
 namespace {
-// Per-call defaults of the fusion bias: (lambda * log p(v), beta * bonus *
-// [the trie root has a child v]) for every label; the row pass adds the
-// row's own terms.  One small launch at the start of every chunk.
+// Per-call defaults of the fusion bias, which the row pass combines with
+// the row's own terms: lambda * log p(v) for every label (0 past V), and a
+// bitmask of the labels the trie root has a child for.  One small launch at
+// the start of every chunk.
 __global__ void k_defaults(DecView d) {
   const Params* P = d.params;
-  const float lam = P->lambda, bscale = P->beta * (d.has_tr ? d.tr.bonus : 0.f);
-  for (int v = blockIdx.x * blockDim.x + threadIdx.x; v < d.V; v += gridDim.x * blockDim.x) {
-    const float lm = d.has_lm ? lam * __ldg(d.lm.uni_logp + v) : 0.f;
-    const float tr = (d.has_tr && __ldg(d.tr.root_child + v) != 0) ? bscale : 0.f;
-    d.dflt[v] = make_float2(lm, tr);
+  const float lam = P->lambda;
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i < d.V4) d.dflt[i] = (d.has_lm && i < d.V) ? lam * __ldg(d.lm.uni_logp + i) : 0.f;
+  if (i < (d.V4 + 31) / 32) {
+    uint32_t m = 0;
+    if (d.has_tr)
+      for (int b = 0; b < 32; ++b) {
+        const int v = i * 32 + b;
+        if (v < d.V && __ldg(d.tr.root_child + v) != 0) m |= 1u << b;
+      }
+    d.droot[i] = m;
   }
 }
 }  // namespace
 
-void launch_defaults(const DecView& d, cudaStream_t s) { k_defaults<<<(d.V + 255) / 256, 256, 0, s>>>(d); }
+void launch_defaults(const DecView& d, cudaStream_t s) { k_defaults<<<(d.V4 + 255) / 256, 256, 0, s>>>(d); }
 
 cudaError_t prepare_kernels(size_t row_smem) {
   // dynamic scratch plus the kernel's static shared memory may pass the
