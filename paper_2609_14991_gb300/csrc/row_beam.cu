@@ -1,4 +1,7 @@
-// Beam-search row pass: one CTA per stream, K hypotheses per stream.
+// Beam-search row pass: one cluster of K CTAs per stream, K hypotheses per
+// stream.  The cluster's first CTA does steps 1-3; then every CTA k of the
+// cluster builds step 4 for survivor k, reading that survivor's chains from
+// the first CTA's shared memory.
 //
 // At label step s (frame s of the chunk; one label or blank per frame) it
 //   1. turns the joint kernel's per-tile partials of frame s-1 into each live
@@ -15,6 +18,8 @@
 // Label sequences live in a per-stream pool of (parent, label) nodes; two
 // candidates are the same sequence when their lengths and rolling hashes
 // agree and their node chains compare equal label by label.
+#include <cooperative_groups.h>
+
 #include "row_common.cuh"
 
 namespace tsd {
@@ -71,8 +76,10 @@ __device__ __forceinline__ bool cand_before(double s1, int h1, int t1, double s2
 // 2 = replay (redo the step without committing anything; for timing).
 __global__ void __launch_bounds__(kRowThreads) k_row_beam(DecView d, int step, int mode) {
   const Params* __restrict__ P = d.params;
-  const int b = blockIdx.x;
+  cooperative_groups::cluster_group cluster = cooperative_groups::this_cluster();
   const int K = d.K, V = d.V;
+  const int b = blockIdx.x / K;                 // stream of this cluster
+  const int crank = (int)cluster.block_rank();  // survivor this CTA builds (step 4)
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const bool commit = (mode != 2);
   extern __shared__ __align__(16) unsigned char smem[];
@@ -99,6 +106,9 @@ __global__ void __launch_bounds__(kRowThreads) k_row_beam(DecView d, int step, i
   __shared__ int sr_uni[kMaxK], sr_rc[kMaxK], sr_rn[kMaxK];
   __shared__ row::ChainRecs rc;
 
+  __shared__ int m_cnt, m_lml, m_trl, m_last;  // survivor crank, copied from the first CTA
+  __shared__ int m_lm[kLmChain], m_tr[kTrChain];
+  if (crank == 0) {
   // previous state of this stream's hypotheses (written by the previous row
   // pass; L2-only loads, see the greedy pass)
   if (tid == 0) {
@@ -414,28 +424,55 @@ __global__ void __launch_bounds__(kRowThreads) k_row_beam(DecView d, int step, i
       P->out_count[b] = cnt ? n_len[best] : 0;
       P->out_score[(size_t)b * T * d.max_sym] = cnt ? (float)n_score[best] : 0.f;
     }
-    return;
   }
+  // Algorithmic bytes (counted when timing): the K hypotheses' partials and state
+  if (mode == 2 || d.count)
+    if (tid == 0) atomicAdd(d.ctr, (unsigned long long)K * (d.n_ptiles * (1 + K) * 8 + 64));
+  } else {
+    // the joint input and bias rows written below are read by the previous
+    // joint kernel: wait for it as the first CTA does
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  }
+  if (mode == 1) return;  // the same for every CTA: no cluster barrier below is left waiting
 
-  // 6. joint input and fusion bias of every survivor for frame `step`
-  const uint16_t* enc_row = P->enc + ((size_t)b * T + min(step, T - 1)) * d.H;
-  // Algorithmic bytes (counted when timing): the K hypotheses' partials and
-  // state, and per survivor its joint input and every arc of its LM chain
-  // levels and trie chain nodes with their records.
-  unsigned long long bytes = (unsigned long long)K * (d.n_ptiles * (1 + K) * 8 + 64);
-  for (int j = 0; j < cnt; ++j) {
-    const int r = b * K + j;
-    row::bias_prepare(d, n_lm[j], n_lml[j], n_tr[j], n_trl[j], rc, lmv, dep);
-    row::build_joint_input(d, enc_row, n_last[j], r);
-    row::bias_finish(d, n_lml[j], n_trl[j], rc, P->lambda, P->beta, d.bias + (size_t)r * d.N_pad, lmv, dep);
-    if ((mode == 2 || d.count) && tid == 0) {
-      bytes += 6ull * d.H;
-      for (int l = 0; l < n_lml[j]; ++l) bytes += 12 + 8ull * rc.lc[l];
-      for (int k = 0; k < n_trl[j]; ++k) bytes += 12 + 4ull * rc.tc[k];
+  // 6. survivor crank's joint input and fusion bias for frame `step`.  Its
+  //    chains come from the first CTA's shared memory (the cluster barrier
+  //    makes them visible); a second barrier keeps the first CTA resident
+  //    until every CTA has its copy.
+  cluster.sync();
+  {
+    const int* rcnt = cluster.map_shared_rank(&n_cnt, 0);
+    const int* rlml = cluster.map_shared_rank(&n_lml[0], 0);
+    const int* rtrl = cluster.map_shared_rank(&n_trl[0], 0);
+    const int* rlast = cluster.map_shared_rank(&n_last[0], 0);
+    const int* rlm = cluster.map_shared_rank(&n_lm[0][0], 0);
+    const int* rtr = cluster.map_shared_rank(&n_tr[0][0], 0);
+    if (tid == 0) {
+      m_cnt = *rcnt;
+      m_lml = rlml[crank];
+      m_trl = rtrl[crank];
+      m_last = rlast[crank];
     }
-    row::block_sync();  // the scratch is reused by the next survivor
+    if (tid < kLmChain) m_lm[tid] = rlm[crank * kLmChain + tid];
+    if (tid >= 32 && tid - 32 < kTrChain) m_tr[tid - 32] = rtr[crank * kTrChain + tid - 32];
   }
-  if ((mode == 2 || d.count) && tid == 0) atomicAdd(d.ctr, bytes);
+  cluster.sync();
+  if (crank >= m_cnt) return;
+  const int r = b * K + crank;
+  const int Tn = __ldcg(&P->T);
+  const uint16_t* enc_row = P->enc + ((size_t)b * Tn + min(step, Tn - 1)) * d.H;
+  row::bias_prepare(d, m_lm, m_lml, m_tr, m_trl, rc, lmv, dep);
+  row::build_joint_input(d, enc_row, m_last, r);
+  row::bias_finish(d, m_lml, m_trl, rc, P->lambda, P->beta, d.bias + (size_t)r * d.N_pad, lmv, dep);
+  if ((mode == 2 || d.count) && tid == 0) {
+    // per survivor: its joint input and every arc of its LM chain levels and
+    // trie chain nodes with their records
+    unsigned long long bytes = 6ull * d.H;
+    for (int l = 0; l < m_lml; ++l) bytes += 12 + 8ull * rc.lc[l];
+    for (int k = 0; k < m_trl; ++k) bytes += 12 + 4ull * rc.tc[k];
+    atomicAdd(d.ctr, bytes);
+  }
 }
 
 __global__ void k_open_beam(DecView d, int slot) {
@@ -458,15 +495,19 @@ __global__ void k_open_beam(DecView d, int slot) {
 
 void launch_row_beam(const DecView& d, int n, int step, int mode, size_t smem, cudaStream_t s, bool pdl) {
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(n);
+  cfg.gridDim = dim3(n * d.K);
   cfg.blockDim = dim3(kRowThreads);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = s;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeClusterDimension;  // one cluster of K CTAs per stream
+  attr[0].val.clusterDim.x = d.K;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = pdl ? 1 : 0;
+  cfg.numAttrs = pdl ? 2 : 1;
   cudaLaunchKernelEx(&cfg, k_row_beam, d, step, mode);
 }
 
