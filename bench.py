@@ -59,7 +59,14 @@ KERNEL_SOURCES = {
     "joint": ["joint_tc.cu", "joint_tc.h", "decoder.h", "internal.h"],
     "row": ["row_pass.cu", "row_beam.cu", "row_common.cuh", "decoder.h", "internal.h"],
 }
-TRAFFIC = {}
+TRAFFIC = {
+    (2, 256, "joint"): (4481067, "4a5ba6aa153cde3d"),
+    (2, 256, "row"): (2240580, "96117cbb17f1d671"),
+    (4, 1024, "joint"): (28863795, "4a5ba6aa153cde3d"),
+    (4, 1024, "row"): (13042278, "96117cbb17f1d671"),
+    (3, 128, "joint"): (6380356, "4a5ba6aa153cde3d"),
+    (3, 128, "row"): (1883358, "96117cbb17f1d671"),
+}
 
 
 def kernel_source_hash(kernel: str) -> str:
