@@ -141,33 +141,40 @@ __device__ __forceinline__ void bias_finish(const DecView& d, int nl, int nt, co
   const int phases = max(nl, nt);
   for (int p = 0; p < phases; ++p) {
     if (p < nl) {
+      // the level's arcs [b, b + c) in 16-byte groups of four from the
+      // aligned index below b (the arrays are padded past their last group)
       const int l = nl - 1 - p;
-      const int b = rc.lb[l], c = rc.lc[l];
+      const int b = rc.lb[l], e = b + rc.lc[l];
       const float off = cum_top - rc.lo[l];
-      int j = tid;
-      for (; j + 3 * step < c; j += 4 * step) {  // four arcs' loads in flight
-        int w[4];
-        float lp[4];
-#pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          w[q] = __ldg(d.lm.arc_tok + b + j + q * step);
-          lp[q] = __ldg(d.lm.arc_logp + b + j + q * step);
-        }
-#pragma unroll
-        for (int q = 0; q < 4; ++q)
-          if (isnan(lmv[w[q]])) lmv[w[q]] = off + lp[q];
-      }
-      for (; j < c; j += step) {
-        const int w = __ldg(d.lm.arc_tok + b + j);
-        const float lp = __ldg(d.lm.arc_logp + b + j);
-        if (isnan(lmv[w])) lmv[w] = off + lp;
+      const int a0 = b & ~3;
+      const int ng = (e - a0 + 3) >> 2;
+      const int4* t4 = reinterpret_cast<const int4*>(d.lm.arc_tok + a0);
+      const float4* p4 = reinterpret_cast<const float4*>(d.lm.arc_logp + a0);
+      for (int g = tid; g < ng; g += step) {
+        const int4 t = __ldg(t4 + g);
+        const float4 v = __ldg(p4 + g);
+        const int i0 = a0 + 4 * g;
+        if (i0 >= b && i0 < e && isnan(lmv[t.x])) lmv[t.x] = off + v.x;
+        if (i0 + 1 >= b && i0 + 1 < e && isnan(lmv[t.y])) lmv[t.y] = off + v.y;
+        if (i0 + 2 >= b && i0 + 2 < e && isnan(lmv[t.z])) lmv[t.z] = off + v.z;
+        if (i0 + 3 >= b && i0 + 3 < e && isnan(lmv[t.w])) lmv[t.w] = off + v.w;
       }
     }
     if (p < nt) {
       const int k = nt - 1 - p;
-      const int b = rc.tb[k], c = rc.tc[k];
+      const int b = rc.tb[k], e = b + rc.tc[k];
       const uint8_t dd = (uint8_t)rc.td[k];
-      for (int j = tid; j < c; j += step) dep[__ldg(d.tr.ch_tok + b + j)] = dd;
+      const int a0 = b & ~3;
+      const int ng = (e - a0 + 3) >> 2;
+      const int4* t4 = reinterpret_cast<const int4*>(d.tr.ch_tok + a0);
+      for (int g = tid; g < ng; g += step) {
+        const int4 t = __ldg(t4 + g);
+        const int i0 = a0 + 4 * g;
+        if (i0 >= b && i0 < e) dep[t.x] = dd;
+        if (i0 + 1 >= b && i0 + 1 < e) dep[t.y] = dd;
+        if (i0 + 2 >= b && i0 + 2 < e) dep[t.z] = dd;
+        if (i0 + 3 >= b && i0 + 3 < e) dep[t.w] = dd;
+      }
     }
     block_sync();
   }

@@ -261,6 +261,9 @@ extern "C" tsd_status tsd_ngram_build(int32_t V, int32_t order, const int64_t* c
   int32_t *d_b, *d_c, *d_at, *d_ag, *d_ut;
   float *d_cum, *d_al, *d_ul;
   tsd_status st;
+  // the row pass reads arcs in aligned groups of four: room for the last group
+  arc_tok.resize((size_t)total_arcs + 4, 0);
+  arc_logp.resize((size_t)total_arcs + 4, 0.f);
   if ((st = lm->arena.upload(&d_b, st_begin)) || (st = lm->arena.upload(&d_c, st_count)) ||
       (st = lm->arena.upload(&d_cum, st_cum)) || (st = lm->arena.upload(&d_at, arc_tok)) ||
       (st = lm->arena.upload(&d_al, arc_logp)) || (st = lm->arena.upload(&d_ag, arc_tgt)) ||
@@ -401,6 +404,7 @@ extern "C" tsd_status tsd_boost_build(int32_t V, int32_t n_phr, const int32_t* o
   v.bonus = token_bonus;
   int32_t *a0, *a1, *a2, *a3, *a4, *a5, *a6, *a7, *a8;
   tsd_status st;
+  ch_tok.resize(ch_tok.size() + 4, 0);  // aligned groups of four in the row pass
   if ((st = b->arena.upload(&a0, nd_begin)) || (st = b->arena.upload(&a1, nd_count)) ||
       (st = b->arena.upload(&a2, depth)) || (st = b->arena.upload(&a3, nd_fail)) ||
       (st = b->arena.upload(&a4, ch_tok)) || (st = b->arena.upload(&a5, ch_node)) ||
