@@ -2,7 +2,8 @@
 
 Python handle on ``oracle.cpp``: a plain, slow, double-precision CPU
 implementation of the fused Transducer decode step (Eq. 1 of the paper with
-one n-gram LM and one phrase list).  Only the test suite, the smoke check and
+one or more weighted n-gram LMs and one phrase list), and a plain reader of
+ARPA-format n-gram files (``read_arpa``).  Only the test suite, the smoke check and
 the benchmark's CPU-baseline leg may import this package; the product library
 never does, and this package never loads the product library.
 
@@ -66,6 +67,8 @@ def lib() -> ctypes.CDLL:
             "oracle_stream_set_history": ([vp, vp, i64, i64], None),
             "oracle_decode_chunk": ([vp, vp, vp, i32, i32, vp, vp, vp, i32, dbl, dbl, i32, vp, vp, vp, i32, dbl,
                                      vp, vp, vp, i32, vp], i32),
+            "oracle_decode_chunk_lms": ([vp, i32, vp, vp, vp, i32, i32, vp, vp, vp, i32, dbl, dbl, i32, vp, vp, vp,
+                                         i32, dbl, vp, vp, vp, i32, vp], i32),
             "oracle_beam_chunk": ([vp, vp, vp, i32, i32, vp, vp, vp, i32, dbl, dbl, i32], i32),
             "oracle_beam_hyp": ([vp, i32, vp, i64, vp, vp], i64),
             "oracle_beam_chunk_follow": ([vp, vp, vp, i32, i32, vp, vp, vp, i32, dbl, dbl, i32, vp, vp, vp, dbl,
@@ -246,6 +249,8 @@ def decode_chunk(stream: Stream, model: Model, lm: Optional[LM], boost: Optional
                  lam: float, beta: float, max_sym: int, follow=None, gap_tol: float = 1e-3):
     """Greedy decode of one chunk enc [T, H] for one stream.
 
+    lm: None, one LM (weight lam), or a list of (LM, w) pairs: LM i enters
+    Eq. 1 with weight alpha_i = lam * w.
     follow: None (free-running) or (tokens, frames, scores) of the decisions
     under test, which the oracle checks and then follows.
     Returns (tokens, frames, scores, report[8])."""
@@ -261,9 +266,19 @@ def decode_chunk(stream: Stream, model: Model, lm: Optional[LM], boost: Optional
         fargs = (_p(ft), _p(ff), _p(fs), len(ft))
     else:
         fargs = (None, None, None, 0)
-    n = lib().oracle_decode_chunk(stream.h, lm.h if lm else None, boost.h if boost else None, model.V, model.H,
-                                  _p(model.E), _p(model.W), _p(enc), T, float(lam), float(beta), int(max_sym),
-                                  *fargs, float(gap_tol), _p(ot), _p(of), _p(osc), cap, _p(rep))
+    if isinstance(lm, (list, tuple)):
+        hs = (ctypes.c_void_p * max(1, len(lm)))(*[m.h for m, _ in lm])
+        ws = np.array([w for _, w in lm] or [0.0], dtype=np.float64)
+        n = lib().oracle_decode_chunk_lms(stream.h, len(lm), hs, _p(ws), boost.h if boost else None, model.V,
+                                          model.H, _p(model.E), _p(model.W), _p(enc), T, float(lam), float(beta),
+                                          int(max_sym), *fargs, float(gap_tol), _p(ot), _p(of), _p(osc), cap,
+                                          _p(rep))
+        if n < 0:
+            raise ValueError("oracle_decode_chunk_lms rejected the LM list")
+    else:
+        n = lib().oracle_decode_chunk(stream.h, lm.h if lm else None, boost.h if boost else None, model.V,
+                                      model.H, _p(model.E), _p(model.W), _p(enc), T, float(lam), float(beta),
+                                      int(max_sym), *fargs, float(gap_tol), _p(ot), _p(of), _p(osc), cap, _p(rep))
     n = min(n, cap)
     return ot[:n].copy(), of[:n].copy(), osc[:n].copy(), rep
 
@@ -289,3 +304,66 @@ def beam_chunk_follow(stream: Stream, model: Model, lm: Optional[LM], boost: Opt
                                    _p(model.E), _p(model.W), _p(enc), enc.shape[0], float(lam), float(beta), int(K),
                                    _p(sh), _p(st), _p(si), float(gap_tol), _p(rep))
     return rep
+
+
+class ArpaArrays:
+    """Per-order n-gram arrays read from an ARPA file (natural log)."""
+
+    def __init__(self, V, tokens, logp, bow, skipped):
+        self.V, self.order = V, len(tokens)
+        self.tokens, self.logp, self.bow, self.skipped = tokens, logp, bow, skipped
+
+
+def read_arpa(text: str, V: int, vocab: Optional[Sequence[str]] = None) -> ArpaArrays:
+    """Reads an ARPA back-off n-gram file: the data header, then per order k a
+    section of lines 'log10 p <k words> [log10 backoff]'.  Words map to ids
+    through vocab (word i -> id i) or, without one, are decimal ids.  N-grams
+    holding a word outside the vocabulary (sentence markers, <unk>) are
+    skipped: the decoder scores no sentence boundaries.  log10 values are
+    turned into natural log."""
+    ln10 = float(np.log(10.0))
+    ids = {w: i for i, w in enumerate(vocab)} if vocab is not None else None
+
+    def word_id(w):
+        if ids is not None:
+            return ids.get(w)
+        try:
+            i = int(w)
+        except ValueError:
+            return None
+        return i if 0 <= i < V else None
+
+    lines = text.splitlines()
+    counts, pos = {}, 0
+    while pos < len(lines) and lines[pos].strip() != "\\data\\":
+        pos += 1
+    pos += 1
+    while pos < len(lines) and lines[pos].strip().startswith("ngram "):
+        k, n = lines[pos].strip()[len("ngram "):].split("=")
+        counts[int(k)] = int(n)
+        pos += 1
+    order = max(counts) if counts else 0
+    toks, lps, bws, skipped = [], [], [], 0
+    for k in range(1, order + 1):
+        while pos < len(lines) and lines[pos].strip() != "\\%d-grams:" % k:
+            pos += 1
+        pos += 1
+        t, lp, bw, seen = [], [], [], 0
+        while pos < len(lines) and lines[pos].strip() and not lines[pos].startswith("\\"):
+            f = lines[pos].split()
+            pos += 1
+            seen += 1
+            words = f[1:1 + k]
+            w_ids = [word_id(w) for w in words]
+            if any(i is None for i in w_ids):
+                skipped += 1
+                continue
+            t.append(w_ids)
+            lp.append(float(f[0]) * ln10)
+            bw.append(float(f[1 + k]) * ln10 if len(f) > 1 + k else 0.0)
+        if seen != counts.get(k, seen):
+            raise ValueError("ARPA order %d: header says %d n-grams, found %d" % (k, counts[k], seen))
+        toks.append(np.array(t, dtype=np.int32).reshape(-1, k))
+        lps.append(np.array(lp, dtype=np.float32))
+        bws.append(np.array(bw, dtype=np.float32))
+    return ArpaArrays(V, toks, lps, bws, skipped)

@@ -17,8 +17,9 @@
 //                       prediction + joint networks propose candidates)
 //   * log-softmax:      log p_AM(y|x) over all V+1 outputs (Eq. 1, term 1)
 //   * n-gram score:     textbook backoff over a dictionary of n-grams
-//                       (Eq. 1, term 2, one LM; "n-gram language models over
-//                       sub-word tokens", Sec. III-C).  Natural log.
+//                       (Eq. 1, term 2: a weighted sum over one or more LMs,
+//                       sum_i alpha_i log p_LM_i; "n-gram language models
+//                       over sub-word tokens", Sec. III-C).  Natural log.
 //   * boost bonus:      naive suffix matching against the phrase list
 //                       (Eq. 1, term 3; "phrase-boosting tree from a user word
 //                       list", Sec. III-C).  Reading: bonus per token times the
@@ -179,10 +180,34 @@ struct Model {
   const uint16_t* W;  // [H][V+1]
 };
 
-// fused[v] = log_softmax(logits)[v] + lambda*lm(v|y) + beta*boost(v|y[rho:]),
+// The LM term of Eq. 1: sum over the LMs of alpha_i * log p_LM_i(v | y),
+// summed in the LMs' order.
+struct LmTerm {
+  static constexpr int kMax = 8;
+  int n = 0;
+  const NGramDict* lm[kMax] = {};
+  double alpha[kMax] = {};
+  double score(const int32_t* y, int64_t len, int32_t v) const {
+    double t = alpha[0] * lm[0]->score(y, len, v);
+    for (int i = 1; i < n; ++i) t += alpha[i] * lm[i]->score(y, len, v);
+    return t;
+  }
+};
+
+LmTerm one_lm(const void* lmp, double lambda) {
+  LmTerm t;
+  if (lmp) {
+    t.n = 1;
+    t.lm[0] = static_cast<const NGramDict*>(lmp);
+    t.alpha[0] = lambda;
+  }
+  return t;
+}
+
+// fused[v] = log_softmax(logits)[v] + sum_i alpha_i*lm_i(v|y) + beta*boost(v|y[rho:]),
 // fused[V] = log_softmax(logits)[V]
-void fused_scores(const Model& m, const uint16_t* enc_t, const Hyp& h, const NGramDict* lm,
-                  const PhraseSet* boost, double lambda, double beta, std::vector<float>& x,
+void fused_scores(const Model& m, const uint16_t* enc_t, const Hyp& h, const LmTerm& lms,
+                  const PhraseSet* boost, double beta, std::vector<float>& x,
                   std::vector<double>& logits, std::vector<double>& fused) {
   const int32_t V = m.V, H = m.H, N = V + 1;
   const int32_t last = h.last(V);
@@ -208,7 +233,7 @@ void fused_scores(const Model& m, const uint16_t* enc_t, const Hyp& h, const NGr
   const int64_t ylen = (int64_t)h.y.size();
   for (int32_t v = 0; v < V; ++v) {
     double f = logits[(size_t)v] - lse;
-    if (lm) f += lambda * lm->score(y, ylen, v);
+    if (lms.n) f += lms.score(y, ylen, v);
     if (boost) f += beta * boost->score(y + h.rho, ylen - h.rho, v);
     fused[(size_t)v] = f;
   }
@@ -378,17 +403,12 @@ enum {
 // gap_tol of it, and that the followed label's fused score is within
 // score tolerance of its own (the largest difference is reported).
 // Returns the number of labels emitted (written to out_* up to out_cap).
-ORACLE_API int32_t oracle_decode_chunk(void* sp, const void* lmp, const void* boostp, int32_t V,
-                                       int32_t H, const uint16_t* E, const uint16_t* W,
-                                       const uint16_t* enc, int32_t T, double lambda, double beta,
-                                       int32_t max_sym, const int32_t* follow_tok,
-                                       const int32_t* follow_frame, const float* follow_score,
-                                       int32_t follow_count, double gap_tol, int32_t* out_tok,
-                                       int32_t* out_frame, double* out_score, int32_t out_cap,
-                                       double* report) {
-  Stream* s = static_cast<Stream*>(sp);
-  const NGramDict* lm = static_cast<const NGramDict*>(lmp);
-  const PhraseSet* boost = static_cast<const PhraseSet*>(boostp);
+namespace {
+int32_t decode_chunk_impl(Stream* s, const LmTerm& lm, const PhraseSet* boost, int32_t V, int32_t H,
+                          const uint16_t* E, const uint16_t* W, const uint16_t* enc, int32_t T, double beta,
+                          int32_t max_sym, const int32_t* follow_tok, const int32_t* follow_frame,
+                          const float* follow_score, int32_t follow_count, double gap_tol, int32_t* out_tok,
+                          int32_t* out_frame, double* out_score, int32_t out_cap, double* report) {
   Model m{V, H, E, W};
   std::vector<float> x;
   std::vector<double> logits, fused;
@@ -397,7 +417,7 @@ ORACLE_API int32_t oracle_decode_chunk(void* sp, const void* lmp, const void* bo
   Hyp& h = s->greedy;
   for (int32_t t = 0; t < T; ++t) {
     for (int32_t sym = 0; sym < max_sym;) {
-      fused_scores(m, enc + (size_t)t * H, h, lm, boost, lambda, beta, x, logits, fused);
+      fused_scores(m, enc + (size_t)t * H, h, lm, boost, beta, x, logits, fused);
       int32_t best = 0;
       for (int32_t v = 1; v <= V; ++v)
         if (fused[(size_t)v] > fused[(size_t)best]) best = v;
@@ -444,6 +464,43 @@ ORACLE_API int32_t oracle_decode_chunk(void* sp, const void* lmp, const void* bo
     for (int i = 0; i < REP_N; ++i) report[i] = rep[i];
   return emitted;
 }
+}  // namespace
+
+ORACLE_API int32_t oracle_decode_chunk(void* sp, const void* lmp, const void* boostp, int32_t V,
+                                       int32_t H, const uint16_t* E, const uint16_t* W,
+                                       const uint16_t* enc, int32_t T, double lambda, double beta,
+                                       int32_t max_sym, const int32_t* follow_tok,
+                                       const int32_t* follow_frame, const float* follow_score,
+                                       int32_t follow_count, double gap_tol, int32_t* out_tok,
+                                       int32_t* out_frame, double* out_score, int32_t out_cap,
+                                       double* report) {
+  return decode_chunk_impl(static_cast<Stream*>(sp), one_lm(lmp, lambda), static_cast<const PhraseSet*>(boostp),
+                           V, H, E, W, enc, T, beta, max_sym, follow_tok, follow_frame, follow_score, follow_count,
+                           gap_tol, out_tok, out_frame, out_score, out_cap, report);
+}
+
+// The same with several LMs (Eq. 1, term 2 summed over i): n_lm LMs with
+// weights alpha_i = lambda * weight[i].
+ORACLE_API int32_t oracle_decode_chunk_lms(void* sp, int32_t n_lm, const void* const* lms, const double* weight,
+                                           const void* boostp, int32_t V, int32_t H, const uint16_t* E,
+                                           const uint16_t* W, const uint16_t* enc, int32_t T, double lambda,
+                                           double beta, int32_t max_sym, const int32_t* follow_tok,
+                                           const int32_t* follow_frame, const float* follow_score,
+                                           int32_t follow_count, double gap_tol, int32_t* out_tok,
+                                           int32_t* out_frame, double* out_score, int32_t out_cap,
+                                           double* report) {
+  LmTerm t;
+  if (n_lm < 0 || n_lm > LmTerm::kMax) return -1;
+  t.n = n_lm;
+  for (int i = 0; i < n_lm; ++i) {
+    if (!lms[i]) return -1;
+    t.lm[i] = static_cast<const NGramDict*>(lms[i]);
+    t.alpha[i] = lambda * weight[i];
+  }
+  return decode_chunk_impl(static_cast<Stream*>(sp), t, static_cast<const PhraseSet*>(boostp), V, H, E, W, enc, T,
+                           beta, max_sym, follow_tok, follow_frame, follow_score, follow_count, gap_tol, out_tok,
+                           out_frame, out_score, out_cap, report);
+}
 
 // Beam search over one chunk (beam workload): every live hypothesis expands
 // to all V+1 outputs each frame (blank keeps its labels, token v appends v),
@@ -470,7 +527,7 @@ ORACLE_API int32_t oracle_beam_chunk(void* sp, const void* lmp, const void* boos
   for (int32_t t = 0; t < T; ++t) {
     std::vector<Cand> cands;
     for (int32_t i = 0; i < (int32_t)s->beam.size(); ++i) {
-      fused_scores(m, enc + (size_t)t * H, s->beam[(size_t)i], lm, boost, lambda, beta, x, logits, fused);
+      fused_scores(m, enc + (size_t)t * H, s->beam[(size_t)i], one_lm(lm, lambda), boost, beta, x, logits, fused);
       for (int32_t v = 0; v <= V; ++v) cands.push_back({s->beam[(size_t)i].score + fused[(size_t)v], i, v});
     }
     std::sort(cands.begin(), cands.end(), [](const Cand& a, const Cand& b) {
@@ -543,7 +600,7 @@ ORACLE_API int32_t oracle_beam_chunk_follow(void* sp, const void* lmp, const voi
     const size_t nh = s->beam.size();
     std::vector<std::vector<double>> f(nh);
     for (size_t i = 0; i < nh; ++i) {
-      fused_scores(m, enc + (size_t)t * H, s->beam[i], lm, boost, lambda, beta, x, logits, fused);
+      fused_scores(m, enc + (size_t)t * H, s->beam[i], one_lm(lm, lambda), boost, beta, x, logits, fused);
       f[i] = fused;
     }
     std::vector<std::pair<int32_t, int32_t>> kept;
@@ -611,7 +668,7 @@ ORACLE_API void oracle_joint_logits(int32_t V, int32_t H, const uint16_t* E, con
   if (last != V) h.y.push_back(last);
   std::vector<float> x;
   std::vector<double> logits, fused;
-  fused_scores(m, enc_t, h, nullptr, nullptr, 0.0, 0.0, x, logits, fused);
+  fused_scores(m, enc_t, h, LmTerm(), nullptr, 0.0, x, logits, fused);
   for (int32_t v = 0; v <= V; ++v) out[v] = logits[(size_t)v];
 }
 
@@ -624,8 +681,8 @@ ORACLE_API void oracle_fused_row(const void* sp, const void* lmp, const void* bo
   Model m{V, H, E, W};
   std::vector<float> x;
   std::vector<double> logits, fused;
-  fused_scores(m, enc_t, s->greedy, static_cast<const NGramDict*>(lmp),
-               static_cast<const PhraseSet*>(boostp), lambda, beta, x, logits, fused);
+  fused_scores(m, enc_t, s->greedy, one_lm(lmp, lambda), static_cast<const PhraseSet*>(boostp), beta, x, logits,
+               fused);
   for (int32_t v = 0; v <= V; ++v) out[v] = fused[(size_t)v];
 }
 

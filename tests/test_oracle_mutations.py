@@ -23,7 +23,7 @@ MUTATIONS = {
         "xk * (double)bf16_bits_to_float(m.W[((size_t)v * H + k) % ((size_t)H * N)]);"),
     "blank gets an LM score": ("fused[(size_t)V] = logits[(size_t)V] - lse;\n}",
                                "fused[(size_t)V] = logits[(size_t)V] - lse + "
-                               "(lm ? lambda * lm->score(y, ylen, 0) : 0.0);\n}"),
+                               "(lms.n ? lms.score(y, ylen, 0) : 0.0);\n}"),
     "ReLU missing": ("if (s < 0.0f) s = 0.0f;", ""),
     "no restart after a phrase": (
         "if (l > 0 && b->is_phrase(g + (len - l), l)) h.rho = (int64_t)h.y.size();", "(void)l;"),
@@ -31,6 +31,9 @@ MUTATIONS = {
     "beam without merging": ("if (o.y == h.y) {", "if (false) {"),
     "LM state takes the shortest suffix": ("for (int64_t l = n; l >= 1; --l) {\n      if (find(hist",
                                            "for (int64_t l = 1; l <= n; ++l) {\n      if (find(hist"),
+    "only the first LM of several": ("for (int i = 1; i < n; ++i) t += alpha[i] * lm[i]->score(y, len, v);",
+                                     "(void)0;"),
+    "LM weight ignored": ("double t = alpha[0] * lm[0]->score(y, len, v);", "double t = lm[0]->score(y, len, v);"),
     "failed match not cancelled": (
         "return bonus * (double)(match(gv.data(), len + 1) - match(g, len));",
         "return bonus * (double)std::max(0, match(gv.data(), len + 1) - match(g, len));"),
@@ -47,7 +50,7 @@ def test_pins_catch_planted_mistake(name, tmp_path):
     so = tmp_path / "mutant.so"
     subprocess.check_call(["g++", "-O1", "-std=c++17", "-ffp-contract=off", "-shared", "-fPIC", str(cpp), "-o",
                            str(so)])
-    r = subprocess.run([sys.executable, "-m", "pytest", os.path.join(ROOT, "tests", "test_oracle_pins.py"), "-q",
-                        "-x", "-p", "no:cacheprovider"], cwd=ROOT, capture_output=True, text=True,
+    r = subprocess.run([sys.executable, "-m", "pytest", os.path.join(ROOT, "tests", "test_oracle_pins.py"),
+                        os.path.join(ROOT, "tests", "test_oracle_multilm.py"), "-q", "-x", "-p", "no:cacheprovider"], cwd=ROOT, capture_output=True, text=True,
                        env=dict(os.environ, TSD_ORACLE_LIB=str(so)), timeout=600)
     assert r.returncode != 0, f"pins did not catch: {name}\n{r.stdout[-2000:]}"
