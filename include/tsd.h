@@ -106,6 +106,41 @@ TSD_API tsd_status tsd_ngram_state_tuple(const tsd_ngram* lm, int32_t state, int
                                  int32_t* len);
 
 /* ------------------------------------------------------------------------
+ * ARPA back-off n-gram files (the usual interchange format of n-gram
+ * toolkits; the paper's n-gram LMs over sub-word tokens, Sec. III-C, come
+ * as such files).  Host only: no device work.
+ *
+ * text[0, len): the file's contents: a "\data\" header with one
+ * "ngram k=count" line per order, then per order k a "\k-grams:" section of
+ * lines "log10 p  w1 .. wk  [log10 backoff]" separated by blanks or tabs.
+ * vocab: NULL (each word is its decimal label id in [0, V)) or V strings
+ * (word vocab[i] is label i; the strings are only read during the call).
+ * N-grams holding any other word (<s>, </s>, <unk>) are dropped and counted
+ * in *skipped: streams have no sentence start or end.  Values are converted
+ * to natural log.  Errors (TSD_EINVAL): no header, a section missing, a line
+ * with the wrong number of fields or a malformed number, a section whose
+ * line count differs from its header, order above 16, a repeated vocabulary
+ * word.  *out is owned by the caller (tsd_arpa_free). */
+typedef struct tsd_arpa tsd_arpa;
+TSD_API tsd_status tsd_arpa_parse(const char* text, int64_t len, int32_t V, const char* const* vocab,
+                                  tsd_arpa** out);
+/* The parsed order, the kept n-grams per order (counts[0 .. min(cap,
+ * order)) ) and the dropped lines. */
+TSD_API tsd_status tsd_arpa_info(const tsd_arpa* a, int32_t* order, int64_t* counts, int32_t cap,
+                                 int64_t* skipped);
+/* Order k's arrays in file order, valid until tsd_arpa_free: tokens
+ * [count][k] int32, logp and bow (natural log; bow 0 where the file has
+ * none) [count] float. */
+TSD_API tsd_status tsd_arpa_arrays(const tsd_arpa* a, int32_t k, const int32_t** tokens, const float** logp,
+                                   const float** bow);
+TSD_API void tsd_arpa_free(tsd_arpa* a);
+/* tsd_arpa_parse followed by tsd_ngram_build (same requirements: every
+ * unigram of [0, V) present, prefix- and suffix-closed after the dropped
+ * lines are removed). */
+TSD_API tsd_status tsd_ngram_build_arpa(const char* text, int64_t len, int32_t V, const char* const* vocab,
+                                        tsd_ngram** out);
+
+/* ------------------------------------------------------------------------
  * Phrase boosting tree (Eq. 1, third term; Sec. III-C "a phrase-boosting
  * tree from a user word list", Fig. 1).
  *

@@ -62,6 +62,11 @@ SIGNATURES = {
     "tsd_decoder_set_timing": ([_vp, _i32], _i32),
     "tsd_decoder_timing": ([_vp, _vp, _vp, _i32, _i32], _i32),
     "tsd_decoder_launches_per_chunk": ([_vp, _i32, _i32, _P(_i64)], _i32),
+    "tsd_arpa_parse": ([ctypes.c_char_p, _i64, _i32, _vp, _P(_vp)], _i32),
+    "tsd_arpa_info": ([_vp, _P(_i32), _vp, _i32, _P(_i64)], _i32),
+    "tsd_arpa_arrays": ([_vp, _i32, _P(_vp), _P(_vp), _P(_vp)], _i32),
+    "tsd_arpa_free": ([_vp], None),
+    "tsd_ngram_build_arpa": ([ctypes.c_char_p, _i64, _i32, _vp, _P(_vp)], _i32),
     "tsd_decoder_timed_bytes": ([_vp, _P(_i64), _i32], _i32),
     "tsd_decoder_debug_capture": ([_vp, _vp, _vp, _i32], _i32),
     "tsd_decoder_set_joint_kernel": ([_vp, _i32], _i32),
@@ -144,6 +149,18 @@ class NGram:
     @classmethod
     def from_arrays(cls, a) -> "NGram":
         return cls(a.V, a.tokens, a.logp, a.bow)
+
+    @classmethod
+    def from_arpa(cls, text, V: int, vocab: Optional[Sequence[str]] = None) -> "NGram":
+        """Tables from ARPA text (``tsd_ngram_build_arpa``)."""
+        data = text.encode() if isinstance(text, str) else bytes(text)
+        keep, vp = _vocab(vocab, V)
+        h = _vp()
+        _check(lib().tsd_ngram_build_arpa(data, len(data), V, vp, ctypes.byref(h)))
+        obj = cls.__new__(cls)
+        obj.h, obj.V = h, V
+        obj.order = 0
+        return obj
 
     def info(self) -> Tuple[int, int, int]:
         s, a, b = _i64(), _i64(), _i64()
@@ -345,3 +362,44 @@ class Decoder:
         self._keep = [logits, rows]
         _check(lib().tsd_decoder_debug_capture(self.h, _ptr(logits) if logits is not None else None,
                                                _ptr(rows) if rows is not None else None, int(max_steps)))
+
+
+def _vocab(vocab, V):
+    if vocab is None:
+        return None, None
+    if len(vocab) != V:
+        raise ValueError("vocabulary has %d words, V=%d" % (len(vocab), V))
+    keep = [w.encode() if isinstance(w, str) else bytes(w) for w in vocab]
+    arr = (ctypes.c_char_p * V)(*keep)
+    return (keep, arr), ctypes.cast(arr, ctypes.c_void_p)
+
+
+def parse_arpa(text, V: int, vocab: Optional[Sequence[str]] = None):
+    """(tokens per order, logp per order, bow per order, dropped lines) of
+    ARPA text, read by the library's host parser (``tsd_arpa_parse``)."""
+    data = text.encode() if isinstance(text, str) else bytes(text)
+    keep, vp = _vocab(vocab, V)
+    h = _vp()
+    _check(lib().tsd_arpa_parse(data, len(data), V, vp, ctypes.byref(h)))
+    try:
+        order = _i32()
+        skipped = _i64()
+        counts = np.zeros(16, dtype=np.int64)
+        _check(lib().tsd_arpa_info(h, ctypes.byref(order), counts.ctypes.data, 16, ctypes.byref(skipped)))
+        toks, lps, bws = [], [], []
+        for k in range(1, order.value + 1):
+            tp, lp, bp = _vp(), _vp(), _vp()
+            _check(lib().tsd_arpa_arrays(h, k, ctypes.byref(tp), ctypes.byref(lp), ctypes.byref(bp)))
+            n = int(counts[k - 1])
+            if n:
+                toks.append(np.ctypeslib.as_array(ctypes.cast(tp, ctypes.POINTER(ctypes.c_int32)), (n * k,))
+                            .reshape(n, k).copy())
+                lps.append(np.ctypeslib.as_array(ctypes.cast(lp, ctypes.POINTER(ctypes.c_float)), (n,)).copy())
+                bws.append(np.ctypeslib.as_array(ctypes.cast(bp, ctypes.POINTER(ctypes.c_float)), (n,)).copy())
+            else:
+                toks.append(np.zeros((0, k), dtype=np.int32))
+                lps.append(np.zeros(0, dtype=np.float32))
+                bws.append(np.zeros(0, dtype=np.float32))
+        return toks, lps, bws, int(skipped.value)
+    finally:
+        lib().tsd_arpa_free(h)
