@@ -188,6 +188,18 @@ typedef struct {
 TSD_API tsd_status tsd_decoder_create(const tsd_decoder_cfg* cfg, const void* W_out_bf16,
                               const void* E_bf16, const tsd_ngram* lm, const tsd_boost* boost,
                               void* cuda_stream, tsd_decoder** out);
+
+/* The same with several n-gram LMs fused at once (Eq. 1, the sum over LMs
+ * i of alpha_i log p_LM_i): LM i (host handle lms[i], same V, outliving the
+ * decoder) enters with alpha_i = lambda * lm_weights[i], lambda being
+ * decode_chunk's argument; lm_weights NULL means all 1.  0 <= n_lms <= 4;
+ * n_lms > 1 needs greedy decoding (beam_k 1), else TSD_EINVAL.  Each stream
+ * keeps one state per LM.  With n_lms 1 and weight 1 this is
+ * tsd_decoder_create. */
+TSD_API tsd_status tsd_decoder_create_multi(const tsd_decoder_cfg* cfg, const void* W_out_bf16,
+                                            const void* E_bf16, const tsd_ngram* const* lms,
+                                            const float* lm_weights, int32_t n_lms, const tsd_boost* boost,
+                                            void* cuda_stream, tsd_decoder** out);
 TSD_API void tsd_decoder_free(tsd_decoder* dec);
 
 /* Opens a stream slot and resets its state on the decoder's stream: no
@@ -230,6 +242,11 @@ TSD_API tsd_status tsd_decode_chunk(tsd_decoder* dec, int32_t n, const int32_t* 
  * Any output pointer may be NULL. */
 TSD_API tsd_status tsd_stream_state(tsd_decoder* dec, int32_t slot, int32_t* lm_state,
                             int32_t* trie_node, int32_t* last);
+
+/* The state of LM lm_index (0 <= lm_index < number of LMs) for a slot
+ * (beam: its first hypothesis), as tsd_stream_state reports the first LM's;
+ * synchronizes with the decoder's last stream. */
+TSD_API tsd_status tsd_stream_lm_state(tsd_decoder* dec, int32_t slot, int32_t lm_index, int32_t* lm_state);
 
 /* Beam: the best live hypothesis of a slot (synchronizes): up to cap labels
  * into buf (host), *len = its length, *score = its score (may be NULL).

@@ -51,6 +51,8 @@ SIGNATURES = {
     "tsd_boost_info": ([_vp, _P(_i32), _P(_i32), _P(_i64)], _i32),
     "tsd_boost_node_tuple": ([_vp, _i32, _vp, _i32, _P(_i32)], _i32),
     "tsd_decoder_create": ([_P(DecoderCfg), _vp, _vp, _vp, _vp, _vp, _P(_vp)], _i32),
+    "tsd_decoder_create_multi": ([_P(DecoderCfg), _vp, _vp, _vp, _vp, _i32, _vp, _vp, _P(_vp)], _i32),
+    "tsd_stream_lm_state": ([_vp, _i32, _i32, _P(_i32)], _i32),
     "tsd_decoder_free": ([_vp], None),
     "tsd_stream_open": ([_vp, _P(_i32)], _i32),
     "tsd_stream_close": ([_vp, _i32], _i32),
@@ -233,7 +235,10 @@ class Decoder:
     """A decoder on the current CUDA device (``tsd_decoder_create``)."""
 
     def __init__(self, V: int, H: int, W_out, E, lm: Optional[NGram] = None, boost: Optional[Boost] = None,
-                 max_symbols: int = 5, beam_k: int = 1, max_streams: int = 64, max_T: int = 64, stream=None):
+                 max_symbols: int = 5, beam_k: int = 1, max_streams: int = 64, max_T: int = 64, stream=None,
+                 lms: Optional[Sequence[Tuple[NGram, float]]] = None):
+        """lms: several LMs as (NGram, w) pairs instead of lm (LM i enters Eq. 1
+        with weight lambda * w; ``tsd_decoder_create_multi``)."""
         import torch
 
         assert W_out.is_cuda and E.is_cuda and W_out.element_size() == 2 and E.element_size() == 2
@@ -244,8 +249,17 @@ class Decoder:
         W_out = W_out.contiguous()
         E = E.contiguous()
         h = _vp()
-        _check(lib().tsd_decoder_create(ctypes.byref(self.cfg), _ptr(W_out), _ptr(E), lm.h if lm else None,
-                                        boost.h if boost else None, _stream(stream), ctypes.byref(h)))
+        if lms is not None:
+            assert lm is None, "give lm or lms, not both"
+            self.lm = [m for m, _ in lms]
+            hs = (_vp * max(1, len(lms)))(*[m.h for m, _ in lms])
+            ws = np.array([w for _, w in lms] or [0.0], dtype=np.float32)
+            _check(lib().tsd_decoder_create_multi(ctypes.byref(self.cfg), _ptr(W_out), _ptr(E), hs, ws.ctypes.data,
+                                                  len(lms), boost.h if boost else None, _stream(stream),
+                                                  ctypes.byref(h)))
+        else:
+            _check(lib().tsd_decoder_create(ctypes.byref(self.cfg), _ptr(W_out), _ptr(E), lm.h if lm else None,
+                                            boost.h if boost else None, _stream(stream), ctypes.byref(h)))
         self.h = h
         self._keep = []
 
@@ -296,6 +310,12 @@ class Decoder:
         a, b, c = _i32(), _i32(), _i32()
         _check(lib().tsd_stream_state(self.h, int(slot), ctypes.byref(a), ctypes.byref(b), ctypes.byref(c)))
         return a.value, b.value, c.value
+
+    def lm_state(self, slot: int, lm_index: int) -> int:
+        """State id of LM lm_index for a slot (``tsd_stream_lm_state``)."""
+        x = _i32()
+        _check(lib().tsd_stream_lm_state(self.h, int(slot), int(lm_index), ctypes.byref(x)))
+        return x.value
 
     def result(self, slot: int, cap: int = 1 << 16) -> Tuple[List[int], float]:
         buf = np.zeros(cap, dtype=np.int32)

@@ -83,15 +83,23 @@ void destroy_set(tsd_decoder::EventSet& es) {
 
 }  // namespace
 
-extern "C" tsd_status tsd_decoder_create(const tsd_decoder_cfg* cfg, const void* W_out_bf16,
-                                         const void* E_bf16, const tsd_ngram* lm,
-                                         const tsd_boost* boost, void* cuda_stream,
-                                         tsd_decoder** out) {
-  clear_error();
+namespace {
+tsd_status create_impl(const tsd_decoder_cfg* cfg, const void* W_out_bf16, const void* E_bf16,
+                       const tsd_ngram* const* lms, const float* lm_weights, int32_t n_lms, const tsd_boost* boost,
+                       void* cuda_stream, tsd_decoder** out) {
   if (!out) return fail(TSD_EINVAL, "tsd_decoder_create: out is NULL");
   *out = nullptr;
   if (!cfg || !W_out_bf16 || !E_bf16) return fail(TSD_EINVAL, "tsd_decoder_create: NULL argument");
   const tsd_decoder_cfg c = *cfg;
+  if (n_lms < 0 || n_lms > kMaxLm) return fail(TSD_EINVAL, "tsd_decoder_create: %d LMs, at most %d", n_lms, kMaxLm);
+  if (n_lms > 0 && !lms) return fail(TSD_EINVAL, "tsd_decoder_create: NULL LM list");
+  for (int i = 0; i < n_lms; ++i) {
+    if (!lms[i]) return fail(TSD_EINVAL, "tsd_decoder_create: LM %d is NULL", i);
+    if (lm_weights && !std::isfinite(lm_weights[i])) return fail(TSD_EINVAL, "tsd_decoder_create: LM weight %d not finite", i);
+    if (lms[i]->view.V != c.V) return fail(TSD_EINVAL, "tsd_decoder_create: LM %d has V=%d, decoder V=%d", i, lms[i]->view.V, c.V);
+  }
+  if (n_lms > 1 && c.beam_k > 1) return fail(TSD_EINVAL, "tsd_decoder_create: several LMs need greedy decoding (beam_k 1)");
+  const tsd_ngram* lm = n_lms > 0 ? lms[0] : nullptr;
   if (c.V < 1 || c.V > 16384) return fail(TSD_EINVAL, "tsd_decoder_create: V=%d out of range [1, 16384]", c.V);
   if (c.H < 64 || c.H > 8192 || c.H % 64) return fail(TSD_EINVAL, "tsd_decoder_create: H=%d must be a multiple of 64 in [64, 8192]", c.H);
   if (c.beam_k < 1 || c.beam_k > 8) return fail(TSD_EINVAL, "tsd_decoder_create: beam_k=%d outside [1, 8]", c.beam_k);
@@ -112,6 +120,7 @@ extern "C" tsd_status tsd_decoder_create(const tsd_decoder_cfg* cfg, const void*
   TSD_CUDA(cudaGetDevice(&d->device));
   cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
   d->lm = lm;
+  d->n_lm = n_lms;
   d->boost = boost;
   d->N = c.V + 1;
   d->N_pad = round_up(d->N, kNPad);
@@ -119,7 +128,7 @@ extern "C" tsd_status tsd_decoder_create(const tsd_decoder_cfg* cfg, const void*
   d->M_pad = round_up(d->M_max, kMPad);
   d->n_ptiles = d->N_pad / kPartialCols;
   d->V4 = round_up(c.V, 16);
-  d->row_smem = row_smem_bytes(d->V4);
+  d->row_smem = row_smem_bytes(d->V4, n_lms);
   if (d->row_smem > 200 * 1024) return fail(TSD_EINVAL, "tsd_decoder_create: V too large for the row pass");
 
   DevArena& A = d->arena;
@@ -136,6 +145,7 @@ extern "C" tsd_status tsd_decoder_create(const tsd_decoder_cfg* cfg, const void*
   int32_t *hlive = nullptr, *hnode = nullptr, *hlen = nullptr, *ppar = nullptr, *ptok = nullptr, *pn = nullptr;
   unsigned long long* hhash = nullptr;
   const size_t SK = (size_t)c.max_streams * c.beam_k;
+  const size_t NL = (size_t)std::max(1, n_lms);  // LM state blocks
   d->params_bytes = sizeof(Params) + sizeof(int32_t) * (size_t)c.max_streams;
   char* pdev = nullptr;
   tsd_status st;
@@ -143,7 +153,7 @@ extern "C" tsd_status tsd_decoder_create(const tsd_decoder_cfg* cfg, const void*
       (st = A.alloc(&Abuf, (size_t)d->M_pad * c.H)) || (st = A.alloc(&bias, (size_t)d->M_pad * d->N_pad)) ||
       (st = A.alloc(&part, (size_t)d->M_pad * (d->N_pad / 64))) || (st = A.alloc(&err, 1)) || (st = A.alloc(&ctr, 2)) || (st = A.alloc(&dflt, (size_t)d->V4)) || (st = A.alloc(&droot, (size_t)(d->V4 + 31) / 32)) || (st = A.alloc(&rt, (size_t)d->M_pad)) ||
       (st = A.alloc(&rs, (size_t)d->M_pad)) || (st = A.alloc(&rc, (size_t)d->M_pad)) ||
-      (st = A.alloc(&sl, SK)) || (st = A.alloc(&sll, SK)) || (st = A.alloc(&slc, SK * kLmChain)) ||
+      (st = A.alloc(&sl, SK)) || (st = A.alloc(&sll, SK * NL)) || (st = A.alloc(&slc, SK * NL * kLmChain)) ||
       (st = A.alloc(&stl, SK)) || (st = A.alloc(&stc, SK * kTrChain)) || (st = A.alloc(&pdev, d->params_bytes))) {
     A.release();
     return st;
@@ -176,7 +186,7 @@ extern "C" tsd_status tsd_decoder_create(const tsd_decoder_cfg* cfg, const void*
   cudaError_t ce;
   if ((ce = cudaMemsetAsync(Abuf, 0, sizeof(uint16_t) * (size_t)d->M_pad * c.H, s)) != cudaSuccess ||
       (ce = cudaMemsetAsync(bias, 0, sizeof(float) * (size_t)d->M_pad * d->N_pad, s)) != cudaSuccess ||
-      (ce = cudaMemsetAsync(sll, 0, sizeof(int32_t) * SK, s)) != cudaSuccess ||
+      (ce = cudaMemsetAsync(sll, 0, sizeof(int32_t) * SK * NL, s)) != cudaSuccess ||
       (ce = cudaMemsetAsync(stl, 0, sizeof(int32_t) * SK, s)) != cudaSuccess ||
       (ce = cudaMemsetAsync(err, 0, sizeof(int32_t), s)) != cudaSuccess ||
       (ce = cudaMemsetAsync(ctr, 0, 2 * sizeof(unsigned long long), s)) != cudaSuccess ||
@@ -235,6 +245,12 @@ extern "C" tsd_status tsd_decoder_create(const tsd_decoder_cfg* cfg, const void*
   v.has_lm = lm ? 1 : 0;
   v.has_tr = boost ? 1 : 0;
   if (lm) v.lm = lm->view;
+  v.n_lm = n_lms;
+  v.lm_stride = (int32_t)SK;
+  for (int i = 0; i < kMaxLm; ++i) {
+    v.lmx[i] = i < n_lms ? lms[i]->view : LmView();
+    v.lm_w[i] = i < n_lms ? (lm_weights ? lm_weights[i] : 1.f) : 0.f;
+  }
   if (boost) v.tr = boost->view;
   v.cap_logits = nullptr;
   v.cap_rows = nullptr;
@@ -258,6 +274,24 @@ extern "C" tsd_status tsd_decoder_create(const tsd_decoder_cfg* cfg, const void*
   d->last_stream = s;
   *out = d.release();
   return TSD_OK;
+}
+}  // namespace
+
+extern "C" tsd_status tsd_decoder_create(const tsd_decoder_cfg* cfg, const void* W_out_bf16,
+                                         const void* E_bf16, const tsd_ngram* lm,
+                                         const tsd_boost* boost, void* cuda_stream,
+                                         tsd_decoder** out) {
+  clear_error();
+  const tsd_ngram* one[1] = {lm};
+  return create_impl(cfg, W_out_bf16, E_bf16, one, nullptr, lm ? 1 : 0, boost, cuda_stream, out);
+}
+
+extern "C" tsd_status tsd_decoder_create_multi(const tsd_decoder_cfg* cfg, const void* W_out_bf16,
+                                               const void* E_bf16, const tsd_ngram* const* lms,
+                                               const float* lm_weights, int32_t n_lms, const tsd_boost* boost,
+                                               void* cuda_stream, tsd_decoder** out) {
+  clear_error();
+  return create_impl(cfg, W_out_bf16, E_bf16, lms, lm_weights, n_lms, boost, cuda_stream, out);
 }
 
 extern "C" void tsd_decoder_free(tsd_decoder* d) {
@@ -412,6 +446,25 @@ extern "C" tsd_status tsd_stream_state(tsd_decoder* d, int32_t slot, int32_t* lm
   if (lm_state) *lm_state = ll > 0 ? chain_lm[ll - 1] : 0;
   if (trie_node) *trie_node = tl > 0 ? chain_tr[0] : 0;
   if (last) *last = ls;
+  return TSD_OK;
+}
+
+extern "C" tsd_status tsd_stream_lm_state(tsd_decoder* d, int32_t slot, int32_t lm_index, int32_t* lm_state) {
+  clear_error();
+  if (!d || !lm_state) return fail(TSD_EINVAL, "tsd_stream_lm_state: NULL argument");
+  if (slot < 0 || slot >= d->cfg.max_streams || !d->slot_open[(size_t)slot])
+    return fail(TSD_ESTATE, "tsd_stream_lm_state: slot %d is not open", slot);
+  if (lm_index < 0 || lm_index >= d->n_lm)
+    return fail(TSD_EINVAL, "tsd_stream_lm_state: LM %d outside [0, %d)", lm_index, d->n_lm);
+  tsd_status st = set_device(d);
+  if (st) return st;
+  TSD_CUDA(cudaStreamSynchronize(d->last_stream));
+  const DecView& v = d->view;
+  const size_t h = (size_t)lm_index * (size_t)v.lm_stride + (size_t)slot * d->cfg.beam_k;
+  int32_t ll = 0, chain[kLmChain];
+  TSD_CUDA(cudaMemcpy(&ll, v.s_lm_len + h, 4, cudaMemcpyDeviceToHost));
+  TSD_CUDA(cudaMemcpy(chain, v.s_lm_chain + h * kLmChain, sizeof(chain), cudaMemcpyDeviceToHost));
+  *lm_state = ll > 0 ? chain[ll - 1] : 0;
   return TSD_OK;
 }
 

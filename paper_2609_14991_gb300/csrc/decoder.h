@@ -38,8 +38,8 @@ struct DecView {
   int32_t* r_cnt;      // [M_pad] labels emitted in this chunk
   // per-slot (x K hypotheses) persistent state
   int32_t* s_last;      // previous label (V = blank / start)
-  int32_t* s_lm_len;    // LM chain length (order of the LM state)
-  int32_t* s_lm_chain;  // [.][kLmChain]
+  int32_t* s_lm_len;    // [LMs][slots] LM chain length (order of the LM state)
+  int32_t* s_lm_chain;  // [LMs][slots][kLmChain]
   int32_t* s_tr_len;
   int32_t* s_tr_chain;  // [.][kTrChain]
   LmView lm;
@@ -59,6 +59,10 @@ struct DecView {
   int32_t* pool_tok;    // [slots][pool_cap] label of the node
   int32_t* pool_n;      // [slots] nodes used
   int32_t pool_cap;
+  int32_t n_lm;       // n-gram LMs fused (0: none; several: greedy only)
+  int32_t lm_stride;  // hypothesis slots per LM in s_lm_len / s_lm_chain
+  LmView lmx[kMaxLm]; // every LM; lmx[0] equals lm
+  float lm_w[kMaxLm]; // relative weights: LM i enters Eq. 1 with lambda * lm_w[i]
   float* dflt;        // [V4] per-call LM bias default lambda*log p(v) (0 past V)
   uint32_t* droot;    // [ceil(V4/32)] bit v: the trie root has a child labelled v
   int32_t* err;  // device status word: nonzero after a bounded wait expired
@@ -73,7 +77,7 @@ void launch_open(const DecView& d, int slot, cudaStream_t s);
 void launch_row(const DecView& d, int M, int step, int mode, size_t smem, cudaStream_t s, bool pdl);
 void launch_joint(const DecView& d, int M, int step, cudaStream_t s);
 void launch_defaults(const DecView& d, cudaStream_t s);
-size_t row_smem_bytes(int V4);
+size_t row_smem_bytes(int V4, int n_lm);
 cudaError_t prepare_kernels(size_t row_smem);
 void launch_row_beam(const DecView& d, int n, int step, int mode, size_t smem, cudaStream_t s, bool pdl);
 void launch_open_beam(const DecView& d, int slot, cudaStream_t s);
@@ -87,7 +91,8 @@ struct tsd_decoder {
   int device = 0;
   int N = 0, N_pad = 0, M_max = 0, M_pad = 0, n_ptiles = 0, V4 = 0;
   tsd::DevArena arena;
-  const tsd_ngram* lm = nullptr;
+  const tsd_ngram* lm = nullptr;  // the first LM
+  int n_lm = 0;
   const tsd_boost* boost = nullptr;
   tsd::DecView view{};
   tsd::Params* params_dev = nullptr;

@@ -20,6 +20,7 @@ constexpr int kTrChain = 32;    // trie suffix chain: nodes of depth >= 1, deepe
 constexpr int kPartialCols = 128;  // columns covered by one selection partial
 constexpr int kNPad = 256;         // the vocabulary axis is padded to this multiple
 constexpr int kMPad = 128;         // the row axis is padded to this multiple
+constexpr int kMaxLm = 4;          // n-gram LMs fused at once (Eq. 1, sum over i)
 
 // Records a message for tsd_last_error() and returns st.
 tsd_status fail(tsd_status st, const char* fmt, ...);

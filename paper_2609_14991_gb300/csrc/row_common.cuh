@@ -18,6 +18,14 @@ __device__ __forceinline__ void block_sync() {
   __syncwarp();
 }
 
+// Field f of LM i's tables (i < kMaxLm): a select over the kernel
+// parameter's per-LM views, so no copy of the parameter block is made.
+template <class T>
+__device__ __forceinline__ T lm_pick(int i, T a0, T a1, T a2, T a3) {
+  return i == 0 ? a0 : i == 1 ? a1 : i == 2 ? a2 : a3;
+}
+#define TSD_LMX(d, i, f) ::tsd::row::lm_pick((i), (d).lmx[0].f, (d).lmx[1].f, (d).lmx[2].f, (d).lmx[3].f)
+
 // Requests the 128-byte line holding p into L1 (no result, no fault on a
 // valid address); later loads of it then wait for L1 rather than L2.
 __device__ __forceinline__ void prefetch_l1(const void* p) {
@@ -125,6 +133,41 @@ __device__ __forceinline__ void bias_prepare(const DecView& d, const int* lm_cha
   }
 }
 
+// LM arcs [b, e) of one chain level into the scratch, in 16-byte groups of
+// four from the aligned index below b (the arc arrays are padded past their
+// last group); a label keeps the first value it gets.  Block-strided.
+__device__ __forceinline__ void scatter_lm_level(const int32_t* arc_tok, const float* arc_logp, int b, int e,
+                                                 float off, float* lmv) {
+  const int a0 = b & ~3;
+  const int ng = (e - a0 + 3) >> 2;
+  const int4* t4 = reinterpret_cast<const int4*>(arc_tok + a0);
+  const float4* p4 = reinterpret_cast<const float4*>(arc_logp + a0);
+  for (int g = threadIdx.x; g < ng; g += blockDim.x) {
+    const int4 t = __ldg(t4 + g);
+    const float4 v = __ldg(p4 + g);
+    const int i0 = a0 + 4 * g;
+    if (i0 >= b && i0 < e && isnan(lmv[t.x])) lmv[t.x] = off + v.x;
+    if (i0 + 1 >= b && i0 + 1 < e && isnan(lmv[t.y])) lmv[t.y] = off + v.y;
+    if (i0 + 2 >= b && i0 + 2 < e && isnan(lmv[t.z])) lmv[t.z] = off + v.z;
+    if (i0 + 3 >= b && i0 + 3 < e && isnan(lmv[t.w])) lmv[t.w] = off + v.w;
+  }
+}
+
+// Trie children [b, e) of one chain node: their labels get goto depth dd.
+__device__ __forceinline__ void scatter_trie_node(const int32_t* ch_tok, int b, int e, uint8_t dd, uint8_t* dep) {
+  const int a0 = b & ~3;
+  const int ng = (e - a0 + 3) >> 2;
+  const int4* t4 = reinterpret_cast<const int4*>(ch_tok + a0);
+  for (int g = threadIdx.x; g < ng; g += blockDim.x) {
+    const int4 t = __ldg(t4 + g);
+    const int i0 = a0 + 4 * g;
+    if (i0 >= b && i0 < e) dep[t.x] = dd;
+    if (i0 + 1 >= b && i0 + 1 < e) dep[t.y] = dd;
+    if (i0 + 2 >= b && i0 + 2 < e) dep[t.z] = dd;
+    if (i0 + 3 >= b && i0 + 3 < e) dep[t.w] = dd;
+  }
+}
+
 // Step 2: the dense fusion bias row lambda*log p_LM(v|state) +
 // beta*bonus*(goto depth - current depth) for every label v (blank: 0).
 // LM chain levels are applied deepest first, each label keeping the first
@@ -141,40 +184,12 @@ __device__ __forceinline__ void bias_finish(const DecView& d, int nl, int nt, co
   const int phases = max(nl, nt);
   for (int p = 0; p < phases; ++p) {
     if (p < nl) {
-      // the level's arcs [b, b + c) in 16-byte groups of four from the
-      // aligned index below b (the arrays are padded past their last group)
       const int l = nl - 1 - p;
-      const int b = rc.lb[l], e = b + rc.lc[l];
-      const float off = cum_top - rc.lo[l];
-      const int a0 = b & ~3;
-      const int ng = (e - a0 + 3) >> 2;
-      const int4* t4 = reinterpret_cast<const int4*>(d.lm.arc_tok + a0);
-      const float4* p4 = reinterpret_cast<const float4*>(d.lm.arc_logp + a0);
-      for (int g = tid; g < ng; g += step) {
-        const int4 t = __ldg(t4 + g);
-        const float4 v = __ldg(p4 + g);
-        const int i0 = a0 + 4 * g;
-        if (i0 >= b && i0 < e && isnan(lmv[t.x])) lmv[t.x] = off + v.x;
-        if (i0 + 1 >= b && i0 + 1 < e && isnan(lmv[t.y])) lmv[t.y] = off + v.y;
-        if (i0 + 2 >= b && i0 + 2 < e && isnan(lmv[t.z])) lmv[t.z] = off + v.z;
-        if (i0 + 3 >= b && i0 + 3 < e && isnan(lmv[t.w])) lmv[t.w] = off + v.w;
-      }
+      scatter_lm_level(d.lm.arc_tok, d.lm.arc_logp, rc.lb[l], rc.lb[l] + rc.lc[l], cum_top - rc.lo[l], lmv);
     }
     if (p < nt) {
       const int k = nt - 1 - p;
-      const int b = rc.tb[k], e = b + rc.tc[k];
-      const uint8_t dd = (uint8_t)rc.td[k];
-      const int a0 = b & ~3;
-      const int ng = (e - a0 + 3) >> 2;
-      const int4* t4 = reinterpret_cast<const int4*>(d.tr.ch_tok + a0);
-      for (int g = tid; g < ng; g += step) {
-        const int4 t = __ldg(t4 + g);
-        const int i0 = a0 + 4 * g;
-        if (i0 >= b && i0 < e) dep[t.x] = dd;
-        if (i0 + 1 >= b && i0 + 1 < e) dep[t.y] = dd;
-        if (i0 + 2 >= b && i0 + 2 < e) dep[t.z] = dd;
-        if (i0 + 3 >= b && i0 + 3 < e) dep[t.w] = dd;
-      }
+      scatter_trie_node(d.tr.ch_tok, rc.tb[k], rc.tb[k] + rc.tc[k], (uint8_t)rc.td[k], dep);
     }
     block_sync();
   }

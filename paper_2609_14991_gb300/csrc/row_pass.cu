@@ -25,6 +25,101 @@ using row::kNegInf;
 using row::lse_merge;
 using row::warp_find;
 
+// Algorithmic bytes of a row's LM chain levels: each level's state record
+// and arcs, and (when a label was emitted) its search: one probe per halving
+// plus the arc found.
+__device__ unsigned long long lm_level_bytes(const row::ChainRecs& rc, int nl, bool searched) {
+  unsigned long long b = 0;
+  for (int l = 0; l < nl; ++l) {
+    b += 12 + 8ull * rc.lc[l];
+    if (searched) b += 8 + 4ull * (32 - __clz(rc.lc[l] + 1)) + 4;
+  }
+  return b;
+}
+
+// The fusion bias row with several LMs (Eq. 1, the sum over LMs): per LM its
+// chain levels deepest first into the scratch (a label keeps the first value
+// it gets), then acc[v] += alpha_i * (that value, or the backoff to the
+// unigram: the chain's summed backoff weights + log p_i(v)); the trie as in
+// the single-LM pass; brow[v] = acc[v] + beta * boost(v).  All threads of
+// the block call it; it returns thread 0's count of LM bytes (if counting).
+__device__ unsigned long long bias_multi(const DecView& d, int L, const int (*lm_chain)[kLmChain], const int* nl,
+                                         const int* tr_chain, int nt, row::ChainRecs& rc, float lam, float beta,
+                                         float* brow, float* lmv, float* acc, uint8_t* dep, bool counting,
+                                         bool searched) {
+  const int tid = threadIdx.x, step = blockDim.x, V = d.V, nq = d.V4 / 4;
+  unsigned long long bytes = 0;
+  if (tid >= 32 && tid - 32 < nt) {
+    const int q = tr_chain[tid - 32];
+    rc.tb[tid - 32] = __ldg(d.tr.nd_begin + q);
+    rc.tc[tid - 32] = __ldg(d.tr.nd_count + q);
+    rc.td[tid - 32] = __ldg(d.tr.nd_depth + q) + 1;
+  }
+  uint32_t* d4 = reinterpret_cast<uint32_t*>(dep);
+  float4* l4 = reinterpret_cast<float4*>(lmv);
+  float4* a4 = reinterpret_cast<float4*>(acc);
+  for (int q = tid; q < nq; q += step) d4[q] = 0u;
+  const float unset = row::unset_value();
+  for (int m = 0; m < L; ++m) {
+    const int n = nl[m];
+    if (tid < n) {
+      const int st = lm_chain[m][tid];
+      rc.lb[tid] = __ldg(TSD_LMX(d, m, st_begin) + st);
+      rc.lc[tid] = __ldg(TSD_LMX(d, m, st_count) + st);
+      rc.lo[tid] = __ldg(TSD_LMX(d, m, st_cum) + st);
+    }
+    for (int q = tid; q < nq; q += step) l4[q] = make_float4(unset, unset, unset, unset);
+    row::block_sync();
+    const float cum_top = n ? rc.lo[n - 1] : 0.f;
+    const int32_t* arc_tok = TSD_LMX(d, m, arc_tok);
+    const float* arc_logp = TSD_LMX(d, m, arc_logp);
+    for (int p = 0; p < n; ++p) {
+      const int l = n - 1 - p;
+      row::scatter_lm_level(arc_tok, arc_logp, rc.lb[l], rc.lb[l] + rc.lc[l], cum_top - rc.lo[l], lmv);
+      row::block_sync();
+    }
+    if (counting && tid == 0) bytes += lm_level_bytes(rc, n, searched);
+    const float alpha = lam * row::lm_pick(m, d.lm_w[0], d.lm_w[1], d.lm_w[2], d.lm_w[3]);
+    const float4* u4 = reinterpret_cast<const float4*>(TSD_LMX(d, m, uni_logp));  // padded past V
+    for (int q = tid; q < nq; q += step) {
+      const float4 l = l4[q];
+      const float4 u = __ldg(u4 + q);
+      float4 a = (m == 0) ? make_float4(0.f, 0.f, 0.f, 0.f) : a4[q];
+      a.x += alpha * (isnan(l.x) ? u.x + cum_top : l.x);
+      a.y += alpha * (isnan(l.y) ? u.y + cum_top : l.y);
+      a.z += alpha * (isnan(l.z) ? u.z + cum_top : l.z);
+      a.w += alpha * (isnan(l.w) ? u.w + cum_top : l.w);
+      a4[q] = a;
+    }
+    row::block_sync();  // the scratch and the records are reused by the next LM
+  }
+  for (int p = 0; p < nt; ++p) {
+    const int k = nt - 1 - p;
+    row::scatter_trie_node(d.tr.ch_tok, rc.tb[k], rc.tb[k] + rc.tc[k], (uint8_t)rc.td[k], dep);
+    row::block_sync();
+  }
+  const int depth_cur = nt ? rc.td[0] - 1 : 0;
+  const float bscale = beta * (d.has_tr ? d.tr.bonus : 0.f);
+  const float tr_base = -bscale * (float)depth_cur;
+  float4* b4 = reinterpret_cast<float4*>(brow);
+  for (int q = tid; q < nq; q += step) {
+    const float4 a = a4[q];
+    const uint32_t dd = d4[q];
+    const uint32_t rb = __ldg(d.droot + (q >> 3)) >> ((4 * q) & 31);
+    const float av[4] = {a.x, a.y, a.z, a.w};
+    float o[4];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const int dj = (dd >> (8 * j)) & 0xff;
+      const float btr = dj ? bscale * (float)(dj - depth_cur) : (((rb >> j) & 1u) ? bscale : 0.f) + tr_base;
+      o[j] = (4 * q + j < V) ? av[j] + btr : 0.f;
+    }
+    b4[q] = make_float4(o[0], o[1], o[2], o[3]);
+  }
+  if (tid == 0) brow[V] = 0.f;
+  return bytes;
+}
+
 // mode: 0 = label step, 1 = final step (apply the last decision only),
 // 2 = replay (redo the step's work without committing any state or output;
 // used only to time the kernel in isolation).
@@ -35,11 +130,15 @@ __global__ void __launch_bounds__(kRowThreads, 7) k_row(DecView d, int step, int
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const bool commit = (mode != 2);
   extern __shared__ __align__(16) unsigned char smem[];
-  // per-label scratch: LM (level << 32 | value bits), trie depth of the goto
+  // per-label scratch: LM value from the chain (NaN unset), with several LMs
+  // also their weighted sum, then the trie depth of the goto
+  const int L = d.n_lm > 1 ? d.n_lm : 1;  // LM state blocks (1 without an LM)
   float* lmv = reinterpret_cast<float*>(smem);
-  uint8_t* dep = reinterpret_cast<uint8_t*>(lmv + d.V4);
+  float* acc = lmv + d.V4;
+  uint8_t* dep = reinterpret_cast<uint8_t*>(lmv + (L > 1 ? 2 : 1) * d.V4);
 
-  __shared__ int s_t, s_sym, s_cnt, s_y, s_lm_len, s_tr_len, s_last, s_slot, s_T;
+  __shared__ int s_t, s_sym, s_cnt, s_y, s_tr_len, s_last, s_slot, s_T;
+  __shared__ int s_lm_len[kMaxLm];
   // the call's parameters, read once before the dependency wait
   __shared__ int32_t* s_out_tok;
   __shared__ int32_t* s_out_frame;
@@ -49,10 +148,10 @@ __global__ void __launch_bounds__(kRowThreads, 7) k_row(DecView d, int step, int
   __shared__ float s_lam, s_beta;
   __shared__ int s_n;
   __shared__ float s_score;
-  __shared__ int s_lm[kLmChain], s_tr[kTrChain];
-  __shared__ int s_lm_tgt[kLmChain];            // target state of y's arc at each LM level (-2 none)
+  __shared__ int s_lm[kMaxLm][kLmChain], s_tr[kTrChain];
+  __shared__ int s_lm_tgt[kMaxLm][kLmChain];    // target state of y's arc at each LM level (-2 none)
   __shared__ int s_tr_node[kTrChain], s_tr_nxt[kTrChain];  // child by y of each trie chain node (-1 none)
-  __shared__ int s_uni_tgt, s_root_child, s_root_next;
+  __shared__ int s_uni_tgt[kMaxLm], s_root_child, s_root_next;
   __shared__ row::ChainRecs rc;
 
   // The row state below was written by the previous row pass; under
@@ -75,13 +174,16 @@ __global__ void __launch_bounds__(kRowThreads, 7) k_row(DecView d, int step, int
     } else {
       s_t = __ldcg(d.r_t + r); s_sym = __ldcg(d.r_sym + r); s_cnt = __ldcg(d.r_cnt + r);
     }
-    s_lm_len = d.has_lm ? __ldcg(d.s_lm_len + slot) : 0;
+    for (int i = 0; i < L; ++i) s_lm_len[i] = d.has_lm ? __ldcg(d.s_lm_len + i * d.lm_stride + slot) : 0;
     s_tr_len = d.has_tr ? __ldcg(d.s_tr_len + slot) : 0;
     s_last = __ldcg(d.s_last + slot);
   }
   row::block_sync();
   const int slot = s_slot, T = s_T;
-  if (tid < s_lm_len) s_lm[tid] = __ldcg(d.s_lm_chain + slot * kLmChain + tid);
+  if (tid < L * kLmChain) {
+    const int i = tid / kLmChain, l = tid % kLmChain;
+    if (l < s_lm_len[i]) s_lm[i][l] = __ldcg(d.s_lm_chain + ((size_t)i * d.lm_stride + slot) * kLmChain + l);
+  }
   if (tid >= 64 && tid - 64 < s_tr_len) s_tr[tid - 64] = __ldcg(d.s_tr_chain + slot * kTrChain + tid - 64);
   // The encoder frames this step can use (t, or t+1 after a frame advance)
   // go to L1 now, while the previous kernel still runs: no kernel of the
@@ -134,24 +236,33 @@ __global__ void __launch_bounds__(kRowThreads, 7) k_row(DecView d, int step, int
     if (y != V) {
       // 2a. independent searches of y in every chain element, each warp
       //     also fetching what the new chain needs from the arc it found
-      const int nl = s_lm_len, nt = s_tr_len;
+      int nl = 0;  // chain elements over all LMs
+      for (int i = 0; i < L; ++i) nl += s_lm_len[i];
+      const int nt = s_tr_len;
       if (tid == kRowThreads - 1) {
-        s_uni_tgt = (d.has_lm && d.lm.order >= 2) ? __ldg(d.lm.uni_tgt + y) : -1;
         s_root_child = d.has_tr ? __ldg(d.tr.root_child + y) : 0;
         s_root_next = d.has_tr ? __ldg(d.tr.root_next + y) : 0;
+      } else if (tid >= kRowThreads - 1 - L) {
+        const int i = tid - (kRowThreads - 1 - L);
+        s_uni_tgt[i] = (d.has_lm && TSD_LMX(d, i, order) >= 2) ? __ldg(TSD_LMX(d, i, uni_tgt) + y) : -1;
       }
       for (int task = warp; task < nl + nt; task += kRowThreads / 32) {
         if (task < nl) {
-          int st = s_lm[task];
-          int b = __ldg(d.lm.st_begin + st), c = __ldg(d.lm.st_count + st);
-          int i = warp_find(d.lm.arc_tok + b, c, y, lane);
+          int m = 0, l = task;  // LM m, level l
+          while (l >= s_lm_len[m]) l -= s_lm_len[m++];
+          const int32_t* st_begin = TSD_LMX(d, m, st_begin);
+          const int32_t* st_count = TSD_LMX(d, m, st_count);
+          const int32_t* arc_tgt = TSD_LMX(d, m, arc_tgt);
+          int st = s_lm[m][l];
+          int b = __ldg(st_begin + st), c = __ldg(st_count + st);
+          int i = warp_find(TSD_LMX(d, m, arc_tok) + b, c, y, lane);
           if (lane == 0) {
-            const int tg = (i >= 0) ? __ldg(d.lm.arc_tgt + b + i) : -2;
-            s_lm_tgt[task] = tg;
+            const int tg = (i >= 0) ? __ldg(arc_tgt + b + i) : -2;
+            s_lm_tgt[m][l] = tg;
             if (tg >= 0) {  // the new chain's state records
-              row::prefetch_l1(d.lm.st_begin + tg);
-              row::prefetch_l1(d.lm.st_count + tg);
-              row::prefetch_l1(d.lm.st_cum + tg);
+              row::prefetch_l1(st_begin + tg);
+              row::prefetch_l1(st_count + tg);
+              row::prefetch_l1(TSD_LMX(d, m, st_cum) + tg);
             }
           }
         } else {
@@ -174,37 +285,43 @@ __global__ void __launch_bounds__(kRowThreads, 7) k_row(DecView d, int step, int
       row::block_sync();
       // 2b. assemble the new chains (shared memory only) and emit
       if (tid == 0) {
-        int newlm[kLmChain];
-        int ln = 0;
-        if (s_uni_tgt >= 0) {
-          newlm[ln++] = s_uni_tgt;
-          for (int l = 0; l < nl && ln < kLmChain; ++l) {
-            int tgt = s_lm_tgt[l];
-            if (tgt < 0) break;  // no arc at this level (-2) or the top order (-1)
-            newlm[ln++] = tgt;
+        // each LM: y's unigram state, then the target of y's arc at every
+        // level of the old chain up to the first level without one (the old
+        // chain's arc targets are in s_lm_tgt, so the new chain is written
+        // over the old one in place)
+        for (int m = 0; m < L; ++m) {
+          const int nold = s_lm_len[m];
+          int ln = 0;
+          if (s_uni_tgt[m] >= 0) {
+            s_lm[m][ln++] = s_uni_tgt[m];
+            for (int l = 0; l < nold && ln < kLmChain; ++l) {
+              const int tgt = s_lm_tgt[m][l];
+              if (tgt < 0) break;  // no arc at this level (-2) or the top order (-1)
+              s_lm[m][ln++] = tgt;
+            }
+          }
+          s_lm_len[m] = ln;
+          if (commit) {
+            int32_t* ch = d.s_lm_chain + ((size_t)m * d.lm_stride + slot) * kLmChain;
+            for (int l = 0; l < ln; ++l) ch[l] = s_lm[m][l];
+            if (d.has_lm) d.s_lm_len[m * d.lm_stride + slot] = ln;
           }
         }
-        int newtr[kTrChain];
         int tn = 0;
         bool reset = false;
         for (int i = 0; i < nt; ++i) {
           if (s_tr_node[i] < 0) continue;
           if (tn == 0 && s_tr_nxt[i] == 0) reset = true;
-          if (tn < kTrChain) newtr[tn++] = s_tr_node[i];
+          if (tn < kTrChain) s_tr[tn++] = s_tr_node[i];
         }
         if (s_root_child != 0) {
           if (tn == 0 && s_root_next == 0) reset = true;
-          if (tn < kTrChain) newtr[tn++] = s_root_child;
+          if (tn < kTrChain) s_tr[tn++] = s_root_child;
         }
         if (reset) tn = 0;
-        for (int l = 0; l < ln; ++l) s_lm[l] = newlm[l];
-        for (int l = 0; l < tn; ++l) s_tr[l] = newtr[l];
-        s_lm_len = ln;
         s_tr_len = tn;
         if (commit) {
-          for (int l = 0; l < ln; ++l) d.s_lm_chain[slot * kLmChain + l] = newlm[l];
-          for (int l = 0; l < tn; ++l) d.s_tr_chain[slot * kTrChain + l] = newtr[l];
-          if (d.has_lm) d.s_lm_len[slot] = ln;
+          for (int l = 0; l < tn; ++l) d.s_tr_chain[slot * kTrChain + l] = s_tr[l];
           if (d.has_tr) d.s_tr_len[slot] = tn;
           const int cap = T * d.max_sym;
           const int o = r * cap + s_cnt;
@@ -240,7 +357,7 @@ __global__ void __launch_bounds__(kRowThreads, 7) k_row(DecView d, int step, int
     if (t < T) {
       c[0] = t;
       c[1] = s_last;
-      c[2] = s_lm_len ? s_lm[s_lm_len - 1] : 0;
+      c[2] = s_lm_len[0] ? s_lm[0][s_lm_len[0] - 1] : 0;
       c[3] = s_tr_len ? s_tr[0] : 0;
     } else {
       c[0] = -1; c[1] = -1; c[2] = -1; c[3] = -1;
@@ -250,11 +367,23 @@ __global__ void __launch_bounds__(kRowThreads, 7) k_row(DecView d, int step, int
 
   // 3. records of the new chains, scratch reset; 4. joint input of this
   // step (its loads overlap the records); 5. the fusion bias row
-  const int nl = s_lm_len, nt = s_tr_len;
-  row::bias_prepare(d, s_lm, nl, s_tr, nt, rc, lmv, dep);
-  row::build_joint_input(d, s_enc + ((size_t)r * T + t) * d.H, s_last, r);
-  row::bias_finish(d, nl, nt, rc, s_lam, s_beta, d.bias + (size_t)r * d.N_pad, lmv, dep);
-  if ((mode == 2 || d.count) && tid == 0) {
+  const int nt = s_tr_len;
+  const bool counting = (mode == 2 || d.count);
+  unsigned long long lm_bytes = 0;  // thread 0: LM levels' records, arcs and searches
+  int nl = s_lm_len[0];
+  if (L == 1) {
+    row::bias_prepare(d, s_lm[0], nl, s_tr, nt, rc, lmv, dep);
+    row::build_joint_input(d, s_enc + ((size_t)r * T + t) * d.H, s_last, r);
+    row::bias_finish(d, nl, nt, rc, s_lam, s_beta, d.bias + (size_t)r * d.N_pad, lmv, dep);
+    if (counting && tid == 0) lm_bytes = lm_level_bytes(rc, nl, s_y != V && evaluated);
+  } else {
+    row::build_joint_input(d, s_enc + ((size_t)r * T + t) * d.H, s_last, r);
+    lm_bytes = bias_multi(d, L, s_lm, s_lm_len, s_tr, nt, rc, s_lam, s_beta, d.bias + (size_t)r * d.N_pad, lmv,
+                          acc, dep, counting, s_y != V && evaluated);
+    nl = 0;
+    for (int i = 0; i < L; ++i) nl += s_lm_len[i];
+  }
+  if (counting && tid == 0) {
     // Algorithmic bytes of this row-step: selection partials, row state,
     // the searches of the emitted label (one probe per halving plus the arc
     // it found), the joint input (encoder frame and embedding row read, A
@@ -262,13 +391,10 @@ __global__ void __launch_bounds__(kRowThreads, 7) k_row(DecView d, int step, int
     // with its state record.  The dense bias row written for the GEMM
     // epilogue and the shared unigram/root rows are not counted here.
     unsigned long long bytes = (unsigned long long)d.n_ptiles * 16 + 2ull * (24 + 4 * (nl + nt));
-    bytes += 6ull * d.H;
-    for (int l = 0; l < nl; ++l) bytes += 12 + 8ull * rc.lc[l];
+    bytes += 6ull * d.H + lm_bytes;
     for (int k = 0; k < nt; ++k) bytes += 12 + 4ull * rc.tc[k];
-    if (s_y != V && evaluated) {
-      for (int l = 0; l < nl; ++l) bytes += 8 + 4ull * (32 - __clz(rc.lc[l] + 1)) + 4;
+    if (s_y != V && evaluated)
       for (int k = 0; k < nt; ++k) bytes += 8 + 4ull * (32 - __clz(rc.tc[k] + 1)) + 8;
-    }
     atomicAdd(d.ctr, bytes);
   }
 }
@@ -276,7 +402,7 @@ __global__ void __launch_bounds__(kRowThreads, 7) k_row(DecView d, int step, int
 __global__ void k_open(DecView d, int slot) {
   if (threadIdx.x == 0) {
     d.s_last[slot] = d.V;
-    d.s_lm_len[slot] = 0;
+    for (int i = 0; i < (d.n_lm > 1 ? d.n_lm : 1); ++i) d.s_lm_len[i * d.lm_stride + slot] = 0;
     d.s_tr_len[slot] = 0;
   }
 }
@@ -298,7 +424,9 @@ __global__ void k_repack(const uint16_t* __restrict__ W, uint16_t* __restrict__ 
 
 }  // namespace
 
-size_t row_smem_bytes(int V4) { return (size_t)V4 * (sizeof(float) + sizeof(uint8_t)); }
+size_t row_smem_bytes(int V4, int n_lm) {
+  return (size_t)V4 * ((n_lm > 1 ? 2 : 1) * sizeof(float) + sizeof(uint8_t));
+}
 
 namespace {
 // Per-call defaults of the fusion bias, which the row pass combines with

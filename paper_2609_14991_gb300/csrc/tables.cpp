@@ -153,7 +153,7 @@ extern "C" tsd_status tsd_ngram_build(int32_t V, int32_t order, const int64_t* c
   lm->st_tok.assign((size_t)S, -1);
   std::vector<int32_t> arc_tok((size_t)total_arcs), arc_tgt((size_t)total_arcs);
   std::vector<float> arc_logp((size_t)total_arcs);
-  std::vector<float> uni_logp((size_t)V);
+  std::vector<float> uni_logp((size_t)V + 16, 0.f);  // padded: read in 16-byte groups
   std::vector<int32_t> uni_tgt((size_t)V);
 
   // per sorted position: context and suffix index in the order below, and
