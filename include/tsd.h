@@ -243,6 +243,20 @@ TSD_API tsd_status tsd_decode_chunk(tsd_decoder* dec, int32_t n, const int32_t* 
 TSD_API tsd_status tsd_stream_state(tsd_decoder* dec, int32_t slot, int32_t* lm_state,
                             int32_t* trie_node, int32_t* last);
 
+/* A stream's whole decoding state as a byte blob (synchronizes the
+ * decoder's stream): previous label, every LM's and the trie's suffix
+ * chains, and for beam decoders the hypotheses with their label sequences.
+ * buf NULL: only *len (the bytes needed) is set; else cap must be >= *len
+ * (TSD_EINVAL otherwise).  The blob is plain host memory owned by the
+ * caller; importing it into an open slot of a decoder with the same V, beam
+ * width, LMs and phrase tree (same tables) continues the stream there, so a
+ * stream can move between decoders or devices, or be checkpointed.  Import
+ * checks the blob's header, length and every id against the decoder's
+ * tables before writing (TSD_EINVAL) and synchronizes. (No paper
+ * counterpart: the paper's decoder keeps its state in the serving process.) */
+TSD_API tsd_status tsd_stream_export(tsd_decoder* dec, int32_t slot, void* buf, int64_t cap, int64_t* len);
+TSD_API tsd_status tsd_stream_import(tsd_decoder* dec, int32_t slot, const void* buf, int64_t len);
+
 /* The state of LM lm_index (0 <= lm_index < number of LMs) for a slot
  * (beam: its first hypothesis), as tsd_stream_state reports the first LM's;
  * synchronizes with the decoder's last stream. */

@@ -53,6 +53,8 @@ SIGNATURES = {
     "tsd_decoder_create": ([_P(DecoderCfg), _vp, _vp, _vp, _vp, _vp, _P(_vp)], _i32),
     "tsd_decoder_create_multi": ([_P(DecoderCfg), _vp, _vp, _vp, _vp, _i32, _vp, _vp, _P(_vp)], _i32),
     "tsd_stream_lm_state": ([_vp, _i32, _i32, _P(_i32)], _i32),
+    "tsd_stream_export": ([_vp, _i32, _vp, _i64, _P(_i64)], _i32),
+    "tsd_stream_import": ([_vp, _i32, _vp, _i64], _i32),
     "tsd_decoder_free": ([_vp], None),
     "tsd_stream_open": ([_vp, _P(_i32)], _i32),
     "tsd_stream_close": ([_vp, _i32], _i32),
@@ -310,6 +312,19 @@ class Decoder:
         a, b, c = _i32(), _i32(), _i32()
         _check(lib().tsd_stream_state(self.h, int(slot), ctypes.byref(a), ctypes.byref(b), ctypes.byref(c)))
         return a.value, b.value, c.value
+
+    def export_state(self, slot: int) -> bytes:
+        """The slot's decoding state as bytes (``tsd_stream_export``)."""
+        n = _i64()
+        _check(lib().tsd_stream_export(self.h, int(slot), None, 0, ctypes.byref(n)))
+        buf = ctypes.create_string_buffer(max(1, n.value))
+        _check(lib().tsd_stream_export(self.h, int(slot), buf, n.value, ctypes.byref(n)))
+        return buf.raw[: n.value]
+
+    def import_state(self, slot: int, blob: bytes):
+        """Continues an exported stream in an open slot (``tsd_stream_import``)."""
+        buf = ctypes.create_string_buffer(bytes(blob), len(blob))
+        _check(lib().tsd_stream_import(self.h, int(slot), buf, len(blob)))
 
     def lm_state(self, slot: int, lm_index: int) -> int:
         """State id of LM lm_index for a slot (``tsd_stream_lm_state``)."""

@@ -12,6 +12,7 @@
 #include <memory>
 #include <new>
 #include <string>
+#include <type_traits>
 
 #include "decoder.h"
 #include "joint_tc.h"
@@ -465,6 +466,168 @@ extern "C" tsd_status tsd_stream_lm_state(tsd_decoder* d, int32_t slot, int32_t 
   TSD_CUDA(cudaMemcpy(&ll, v.s_lm_len + h, 4, cudaMemcpyDeviceToHost));
   TSD_CUDA(cudaMemcpy(chain, v.s_lm_chain + h * kLmChain, sizeof(chain), cudaMemcpyDeviceToHost));
   *lm_state = ll > 0 ? chain[ll - 1] : 0;
+  return TSD_OK;
+}
+
+namespace {
+// Stream state blob: a header, then per hypothesis (K = beam width) the
+// previous label, each LM's chain (length + kLmChain ids), the trie chain
+// (length + kTrChain ids), and for beam decoders the hypothesis record
+// (live, node, length, score, hash); then the beam's label-sequence nodes.
+struct BlobHeader {
+  uint32_t magic, version;
+  int32_t V, beam_k, n_lm, has_tr, pool_used, reserved;
+};
+constexpr uint32_t kBlobMagic = 0x53445354u;  // "TSDS"
+
+int64_t blob_bytes(const tsd_decoder* d, int32_t pool_used) {
+  const int K = d->cfg.beam_k, L = std::max(1, d->n_lm);
+  int64_t per = 4 + (int64_t)L * 4 * (1 + kLmChain) + 4 * (1 + kTrChain);
+  if (K > 1) per += 4 + 4 + 4 + 8 + 8;
+  return (int64_t)sizeof(BlobHeader) + per * K + (K > 1 ? 8ll * pool_used : 0);
+}
+
+template <class T>
+tsd_status copy_dev(T* dst, const T* src, size_t n, cudaMemcpyKind kind) {
+  TSD_CUDA(cudaMemcpy(dst, src, sizeof(T) * n, kind));
+  return TSD_OK;
+}
+}  // namespace
+
+extern "C" tsd_status tsd_stream_export(tsd_decoder* d, int32_t slot, void* buf, int64_t cap, int64_t* len) {
+  clear_error();
+  if (!d || !len) return fail(TSD_EINVAL, "tsd_stream_export: NULL argument");
+  if (slot < 0 || slot >= d->cfg.max_streams || !d->slot_open[(size_t)slot])
+    return fail(TSD_ESTATE, "tsd_stream_export: slot %d is not open", slot);
+  tsd_status st = set_device(d);
+  if (st) return st;
+  TSD_CUDA(cudaStreamSynchronize(d->last_stream));
+  const DecView& v = d->view;
+  const int K = d->cfg.beam_k, L = std::max(1, d->n_lm);
+  int32_t pool_used = 0;
+  if (K > 1) TSD_CUDA(cudaMemcpy(&pool_used, v.pool_n + slot, 4, cudaMemcpyDeviceToHost));
+  *len = blob_bytes(d, pool_used);
+  if (!buf) return TSD_OK;
+  if (cap < *len) return fail(TSD_EINVAL, "tsd_stream_export: %lld bytes needed, cap %lld", (long long)*len, (long long)cap);
+  char* p = static_cast<char*>(buf);
+  BlobHeader hd{kBlobMagic, 1u, d->cfg.V, K, d->n_lm, v.has_tr, pool_used, 0};
+  std::memcpy(p, &hd, sizeof(hd));
+  p += sizeof(hd);
+  auto put = [&](const auto* src, size_t n) -> tsd_status {
+    tsd_status s2 = copy_dev(reinterpret_cast<std::remove_const_t<std::remove_pointer_t<decltype(src)>>*>(p), src, n,
+                             cudaMemcpyDeviceToHost);
+    p += sizeof(*src) * n;
+    return s2;
+  };
+  for (int k = 0; k < K; ++k) {
+    const size_t h = (size_t)slot * K + k;
+    if ((st = put(v.s_last + h, 1))) return st;
+    for (int m = 0; m < L; ++m) {
+      const size_t hm = (size_t)m * v.lm_stride + h;
+      if ((st = put(v.s_lm_len + hm, 1)) || (st = put(v.s_lm_chain + hm * kLmChain, kLmChain))) return st;
+    }
+    if ((st = put(v.s_tr_len + h, 1)) || (st = put(v.s_tr_chain + h * kTrChain, kTrChain))) return st;
+    if (K > 1 && ((st = put(v.h_live + h, 1)) || (st = put(v.h_node + h, 1)) || (st = put(v.h_len + h, 1)) ||
+                  (st = put(v.h_score + h, 1)) || (st = put(v.h_hash + h, 1))))
+      return st;
+  }
+  if (K > 1 && pool_used > 0) {
+    if ((st = put(v.pool_parent + (size_t)slot * v.pool_cap, (size_t)pool_used)) ||
+        (st = put(v.pool_tok + (size_t)slot * v.pool_cap, (size_t)pool_used)))
+      return st;
+  }
+  return TSD_OK;
+}
+
+extern "C" tsd_status tsd_stream_import(tsd_decoder* d, int32_t slot, const void* buf, int64_t len) {
+  clear_error();
+  if (!d || !buf) return fail(TSD_EINVAL, "tsd_stream_import: NULL argument");
+  if (slot < 0 || slot >= d->cfg.max_streams || !d->slot_open[(size_t)slot])
+    return fail(TSD_ESTATE, "tsd_stream_import: slot %d is not open", slot);
+  if (len < (int64_t)sizeof(BlobHeader)) return fail(TSD_EINVAL, "tsd_stream_import: blob too short");
+  BlobHeader hd;
+  std::memcpy(&hd, buf, sizeof(hd));
+  const DecView& v = d->view;
+  const int K = d->cfg.beam_k, L = std::max(1, d->n_lm);
+  if (hd.magic != kBlobMagic || hd.version != 1u) return fail(TSD_EINVAL, "tsd_stream_import: not a stream state blob");
+  if (hd.V != d->cfg.V || hd.beam_k != K || hd.n_lm != d->n_lm || hd.has_tr != v.has_tr)
+    return fail(TSD_EINVAL, "tsd_stream_import: blob is for V=%d beam %d, %d LMs, boost %d; decoder has V=%d beam %d, %d LMs, boost %d",
+                hd.V, hd.beam_k, hd.n_lm, hd.has_tr, d->cfg.V, K, d->n_lm, v.has_tr);
+  if (hd.pool_used < 0 || hd.pool_used > v.pool_cap || len != blob_bytes(d, hd.pool_used))
+    return fail(TSD_EINVAL, "tsd_stream_import: blob length %lld does not match its header", (long long)len);
+  // check the contents before anything reaches the device
+  {
+    const char* q = static_cast<const char*>(buf) + sizeof(hd);
+    auto rd = [&](size_t bytes) { const char* r = q; q += bytes; return r; };
+    for (int k = 0; k < K; ++k) {
+      int32_t last;
+      std::memcpy(&last, rd(4), 4);
+      if (last < 0 || last > d->cfg.V) return fail(TSD_EINVAL, "tsd_stream_import: previous label %d out of range", last);
+      for (int m = 0; m < L; ++m) {
+        int32_t n;
+        std::memcpy(&n, rd(4), 4);
+        const char* ch = rd(4 * kLmChain);
+        if (n < 0 || n > kLmChain) return fail(TSD_EINVAL, "tsd_stream_import: LM chain length %d", n);
+        const int64_t S = m < d->n_lm ? v.lmx[m].n_states : 1;
+        for (int l = 0; l < n; ++l) {
+          int32_t sid;
+          std::memcpy(&sid, ch + 4 * l, 4);
+          if (sid < 0 || sid >= S) return fail(TSD_EINVAL, "tsd_stream_import: LM state %d out of range", sid);
+        }
+      }
+      int32_t tn;
+      std::memcpy(&tn, rd(4), 4);
+      const char* tch = rd(4 * kTrChain);
+      if (tn < 0 || tn > kTrChain) return fail(TSD_EINVAL, "tsd_stream_import: trie chain length %d", tn);
+      for (int l = 0; l < tn; ++l) {
+        int32_t nd;
+        std::memcpy(&nd, tch + 4 * l, 4);
+        if (nd < 0 || nd >= v.tr.n_nodes) return fail(TSD_EINVAL, "tsd_stream_import: trie node %d out of range", nd);
+      }
+      if (K > 1) {
+        int32_t node;
+        rd(4);
+        std::memcpy(&node, rd(4), 4);
+        rd(4 + 8 + 8);
+        if (node < -1 || node >= hd.pool_used) return fail(TSD_EINVAL, "tsd_stream_import: sequence node %d out of range", node);
+      }
+    }
+    for (int32_t i = 0; K > 1 && i < hd.pool_used; ++i) {
+      int32_t par, tok;
+      std::memcpy(&par, q + 4 * (size_t)i, 4);
+      std::memcpy(&tok, q + 4 * ((size_t)hd.pool_used + i), 4);
+      if (par < -1 || par >= i) return fail(TSD_EINVAL, "tsd_stream_import: sequence node %d has parent %d", i, par);
+      if (tok < 0 || tok >= d->cfg.V) return fail(TSD_EINVAL, "tsd_stream_import: sequence node %d has label %d", i, tok);
+    }
+  }
+  tsd_status st = set_device(d);
+  if (st) return st;
+  TSD_CUDA(cudaStreamSynchronize(d->last_stream));
+  const char* p = static_cast<const char*>(buf) + sizeof(hd);
+  auto get = [&](auto* dst, size_t n) -> tsd_status {
+    tsd_status s2 = copy_dev(dst, reinterpret_cast<const std::remove_pointer_t<decltype(dst)>*>(p), n,
+                             cudaMemcpyHostToDevice);
+    p += sizeof(*dst) * n;
+    return s2;
+  };
+  for (int k = 0; k < K; ++k) {
+    const size_t h = (size_t)slot * K + k;
+    if ((st = get(v.s_last + h, 1))) return st;
+    for (int m = 0; m < L; ++m) {
+      const size_t hm = (size_t)m * v.lm_stride + h;
+      if ((st = get(v.s_lm_len + hm, 1)) || (st = get(v.s_lm_chain + hm * kLmChain, kLmChain))) return st;
+    }
+    if ((st = get(v.s_tr_len + h, 1)) || (st = get(v.s_tr_chain + h * kTrChain, kTrChain))) return st;
+    if (K > 1 && ((st = get(v.h_live + h, 1)) || (st = get(v.h_node + h, 1)) || (st = get(v.h_len + h, 1)) ||
+                  (st = get(v.h_score + h, 1)) || (st = get(v.h_hash + h, 1))))
+      return st;
+  }
+  if (K > 1) {
+    if (hd.pool_used > 0 && ((st = get(v.pool_parent + (size_t)slot * v.pool_cap, (size_t)hd.pool_used)) ||
+                             (st = get(v.pool_tok + (size_t)slot * v.pool_cap, (size_t)hd.pool_used))))
+      return st;
+    TSD_CUDA(cudaMemcpy(v.pool_n + slot, &hd.pool_used, 4, cudaMemcpyHostToDevice));
+  }
   return TSD_OK;
 }
 
