@@ -69,6 +69,8 @@ def lib() -> ctypes.CDLL:
                                      vp, vp, vp, i32, vp], i32),
             "oracle_decode_chunk_lms": ([vp, i32, vp, vp, vp, i32, i32, vp, vp, vp, i32, dbl, dbl, i32, vp, vp, vp,
                                          i32, dbl, vp, vp, vp, i32, vp], i32),
+            "oracle_decode_chunk_pruned": ([vp, vp, vp, i32, i32, vp, vp, vp, i32, dbl, dbl, i32, i32, dbl, vp, vp,
+                                            vp, i32, dbl, vp, vp, vp, i32, vp], i32),
             "oracle_beam_chunk": ([vp, vp, vp, i32, i32, vp, vp, vp, i32, dbl, dbl, i32], i32),
             "oracle_beam_hyp": ([vp, i32, vp, i64, vp, vp], i64),
             "oracle_beam_chunk_follow": ([vp, vp, vp, i32, i32, vp, vp, vp, i32, dbl, dbl, i32, vp, vp, vp, dbl,
@@ -246,13 +248,16 @@ def fused_row(stream: Stream, model: Model, lm: Optional[LM], boost: Optional[Bo
 
 
 def decode_chunk(stream: Stream, model: Model, lm: Optional[LM], boost: Optional[Boost], enc: np.ndarray,
-                 lam: float, beta: float, max_sym: int, follow=None, gap_tol: float = 1e-3):
+                 lam: float, beta: float, max_sym: int, follow=None, gap_tol: float = 1e-3, prune_k: int = 0,
+                 am_tol: float = 2e-2):
     """Greedy decode of one chunk enc [T, H] for one stream.
 
     lm: None, one LM (weight lam), or a list of (LM, w) pairs: LM i enters
     Eq. 1 with weight alpha_i = lam * w.
     follow: None (free-running) or (tokens, frames, scores) of the decisions
     under test, which the oracle checks and then follows.
+    prune_k > 0: pruned fusion over the acoustic model's prune_k best outputs
+    (one LM); am_tol is the logit tolerance at the edge of that set.
     Returns (tokens, frames, scores, report[8])."""
     enc = np.ascontiguousarray(enc, dtype=np.uint16)
     T = enc.shape[0]
@@ -266,7 +271,13 @@ def decode_chunk(stream: Stream, model: Model, lm: Optional[LM], boost: Optional
         fargs = (_p(ft), _p(ff), _p(fs), len(ft))
     else:
         fargs = (None, None, None, 0)
-    if isinstance(lm, (list, tuple)):
+    if prune_k > 0:
+        assert not isinstance(lm, (list, tuple)), "pruned fusion takes one LM"
+        n = lib().oracle_decode_chunk_pruned(stream.h, lm.h if lm else None, boost.h if boost else None, model.V,
+                                             model.H, _p(model.E), _p(model.W), _p(enc), T, float(lam), float(beta),
+                                             int(max_sym), int(prune_k), float(am_tol), *fargs, float(gap_tol),
+                                             _p(ot), _p(of), _p(osc), cap, _p(rep))
+    elif isinstance(lm, (list, tuple)):
         hs = (ctypes.c_void_p * max(1, len(lm)))(*[m.h for m, _ in lm])
         ws = np.array([w for _, w in lm] or [0.0], dtype=np.float64)
         n = lib().oracle_decode_chunk_lms(stream.h, len(lm), hs, _p(ws), boost.h if boost else None, model.V,

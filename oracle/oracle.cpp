@@ -27,7 +27,11 @@
 //                       completed phrase is banked and matching restarts.
 //   * greedy decoding:  argmax of the fused score, lowest id on ties; blank
 //                       (id V) or max_sym emissions end the frame (Sec. III:
-//                       "greedy decoding emits text").
+//                       "greedy decoding emits text").  Pruned variant (the
+//                       reading of Sec. III-C's remark that fusion only
+//                       re-ranks the candidates the acoustic model proposes):
+//                       the argmax runs over the acoustic model's k best
+//                       outputs only (blank included, ties to the lower id).
 //   * beam search:      per frame, top-K of the K*(V+1) extensions, then
 //                       identical label sequences merged by log-sum-exp.
 //                       (Not in the paper; the beam workload defines it.)
@@ -404,11 +408,27 @@ enum {
 // score tolerance of its own (the largest difference is reported).
 // Returns the number of labels emitted (written to out_* up to out_cap).
 namespace {
+// The acoustic model's k best outputs by logit (ties to the lower id).
+std::vector<int32_t> am_top(const std::vector<double>& logits, int32_t k) {
+  std::vector<int32_t> idx(logits.size());
+  for (size_t v = 0; v < idx.size(); ++v) idx[v] = (int32_t)v;
+  std::stable_sort(idx.begin(), idx.end(),
+                   [&](int32_t a, int32_t b) { return logits[(size_t)a] > logits[(size_t)b]; });
+  idx.resize((size_t)std::min<int64_t>(k, (int64_t)idx.size()));
+  return idx;
+}
+
+// prune_k > 0: the decision is the best fused value among the acoustic
+// model's prune_k best outputs.  In follow mode a followed label at the
+// edge of that set (its logit within am_tol of the k-th) is accepted, and it
+// is compared with the best fused value among the outputs that are in the
+// set by more than am_tol.
 int32_t decode_chunk_impl(Stream* s, const LmTerm& lm, const PhraseSet* boost, int32_t V, int32_t H,
                           const uint16_t* E, const uint16_t* W, const uint16_t* enc, int32_t T, double beta,
                           int32_t max_sym, const int32_t* follow_tok, const int32_t* follow_frame,
                           const float* follow_score, int32_t follow_count, double gap_tol, int32_t* out_tok,
-                          int32_t* out_frame, double* out_score, int32_t out_cap, double* report) {
+                          int32_t* out_frame, double* out_score, int32_t out_cap, double* report,
+                          int32_t prune_k = 0, double am_tol = 0.0) {
   Model m{V, H, E, W};
   std::vector<float> x;
   std::vector<double> logits, fused;
@@ -418,12 +438,19 @@ int32_t decode_chunk_impl(Stream* s, const LmTerm& lm, const PhraseSet* boost, i
   for (int32_t t = 0; t < T; ++t) {
     for (int32_t sym = 0; sym < max_sym;) {
       fused_scores(m, enc + (size_t)t * H, h, lm, boost, beta, x, logits, fused);
-      int32_t best = 0;
-      for (int32_t v = 1; v <= V; ++v)
-        if (fused[(size_t)v] > fused[(size_t)best]) best = v;
+      std::vector<uint8_t> cand((size_t)V + 1, prune_k > 0 ? 0 : 1);
+      double kth = -std::numeric_limits<double>::infinity();
+      if (prune_k > 0) {
+        const std::vector<int32_t> top = am_top(logits, prune_k);
+        for (int32_t c : top) cand[(size_t)c] = 1;
+        kth = logits[(size_t)top.back()];
+      }
+      int32_t best = -1;
+      for (int32_t v = 0; v <= V; ++v)
+        if (cand[(size_t)v] && (best < 0 || fused[(size_t)v] > fused[(size_t)best])) best = v;
       double second = -std::numeric_limits<double>::infinity();
       for (int32_t v = 0; v <= V; ++v)
-        if (v != best) second = std::max(second, fused[(size_t)v]);
+        if (cand[(size_t)v] && v != best) second = std::max(second, fused[(size_t)v]);
       rep[REP_MIN_GAP] = std::min(rep[REP_MIN_GAP], fused[(size_t)best] - second);
       int32_t y = best;
       if (follow_tok) {
@@ -432,6 +459,14 @@ int32_t decode_chunk_impl(Stream* s, const LmTerm& lm, const PhraseSet* boost, i
         if (fy < 0 || fy > V) { rep[REP_INCONSISTENT] = 1; fy = V; }
         if (fy != best) {
           double gap = fused[(size_t)best] - fused[(size_t)fy];
+          if (prune_k > 0) {
+            // the best among the outputs surely in both candidate sets
+            int32_t sure = -1;
+            for (int32_t v = 0; v <= V; ++v)
+              if (logits[(size_t)v] > kth + am_tol && (sure < 0 || fused[(size_t)v] > fused[(size_t)sure])) sure = v;
+            gap = sure >= 0 ? fused[(size_t)sure] - fused[(size_t)fy] : 0.0;
+            if (logits[(size_t)fy] < kth - am_tol) gap = std::numeric_limits<double>::infinity();
+          }
           if (gap > gap_tol) {
             rep[REP_MISMATCH] += 1;
             if (rep[REP_FIRST_BAD] < 0) rep[REP_FIRST_BAD] = rep[REP_STEPS];
@@ -477,6 +512,22 @@ ORACLE_API int32_t oracle_decode_chunk(void* sp, const void* lmp, const void* bo
   return decode_chunk_impl(static_cast<Stream*>(sp), one_lm(lmp, lambda), static_cast<const PhraseSet*>(boostp),
                            V, H, E, W, enc, T, beta, max_sym, follow_tok, follow_frame, follow_score, follow_count,
                            gap_tol, out_tok, out_frame, out_score, out_cap, report);
+}
+
+// The pruned variant: fusion re-ranks only the acoustic model's prune_k
+// best outputs (see decode_chunk_impl); am_tol is the logit tolerance at the
+// edge of that set in follow mode.
+ORACLE_API int32_t oracle_decode_chunk_pruned(void* sp, const void* lmp, const void* boostp, int32_t V, int32_t H,
+                                              const uint16_t* E, const uint16_t* W, const uint16_t* enc, int32_t T,
+                                              double lambda, double beta, int32_t max_sym, int32_t prune_k,
+                                              double am_tol, const int32_t* follow_tok, const int32_t* follow_frame,
+                                              const float* follow_score, int32_t follow_count, double gap_tol,
+                                              int32_t* out_tok, int32_t* out_frame, double* out_score,
+                                              int32_t out_cap, double* report) {
+  if (prune_k < 1) return -1;
+  return decode_chunk_impl(static_cast<Stream*>(sp), one_lm(lmp, lambda), static_cast<const PhraseSet*>(boostp),
+                           V, H, E, W, enc, T, beta, max_sym, follow_tok, follow_frame, follow_score, follow_count,
+                           gap_tol, out_tok, out_frame, out_score, out_cap, report, prune_k, am_tol);
 }
 
 // The same with several LMs (Eq. 1, term 2 summed over i): n_lm LMs with

@@ -34,6 +34,9 @@ MUTATIONS = {
     "only the first LM of several": ("for (int i = 1; i < n; ++i) t += alpha[i] * lm[i]->score(y, len, v);",
                                      "(void)0;"),
     "LM weight ignored": ("double t = alpha[0] * lm[0]->score(y, len, v);", "double t = lm[0]->score(y, len, v);"),
+    "pruned set not ranked by the acoustic model": (
+        "[&](int32_t a, int32_t b) { return logits[(size_t)a] > logits[(size_t)b]; });",
+        "[&](int32_t a, int32_t b) { return fused_rank_bug(a, b); });"),
     "failed match not cancelled": (
         "return bonus * (double)(match(gv.data(), len + 1) - match(g, len));",
         "return bonus * (double)std::max(0, match(gv.data(), len + 1) - match(g, len));"),
@@ -46,11 +49,12 @@ def test_pins_catch_planted_mistake(name, tmp_path):
     a, b = MUTATIONS[name]
     assert a in src, "mutation anchor not found; update the mutation list"
     cpp = tmp_path / "mutant.cpp"
-    cpp.write_text(src.replace(a, b))
+    cpp.write_text(src.replace(a, b).replace("fused_rank_bug(a, b)", "a < b"))
     so = tmp_path / "mutant.so"
     subprocess.check_call(["g++", "-O1", "-std=c++17", "-ffp-contract=off", "-shared", "-fPIC", str(cpp), "-o",
                            str(so)])
     r = subprocess.run([sys.executable, "-m", "pytest", os.path.join(ROOT, "tests", "test_oracle_pins.py"),
-                        os.path.join(ROOT, "tests", "test_oracle_multilm.py"), "-q", "-x", "-p", "no:cacheprovider"], cwd=ROOT, capture_output=True, text=True,
+                        os.path.join(ROOT, "tests", "test_oracle_multilm.py"),
+                        os.path.join(ROOT, "tests", "test_oracle_pruned.py"), "-q", "-x", "-p", "no:cacheprovider"], cwd=ROOT, capture_output=True, text=True,
                        env=dict(os.environ, TSD_ORACLE_LIB=str(so)), timeout=600)
     assert r.returncode != 0, f"pins did not catch: {name}\n{r.stdout[-2000:]}"
