@@ -208,7 +208,7 @@ def oracle_models(w, inp_lm, inp_ph, E, W, extra=()):
     return olm, obo, oracle.Model(w.V, w.H, E, W)
 
 
-def oracle_baseline(w, models, streams, chunks, threads=None):
+def oracle_baseline(w, models, streams, chunks, threads=None, prune_k=0):
     """Times the oracle (as it stands) decoding `streams` x `chunks` of the
     workload on this host's cores; returns (frames/s, cores, sample, seconds)."""
     import concurrent.futures
@@ -222,7 +222,7 @@ def oracle_baseline(w, models, streams, chunks, threads=None):
     def one(i):
         st = oracle.Stream(w.V)
         for c in range(chunks):
-            oracle.decode_chunk(st, model, olm, obo, encs[c][i], w.lam, w.beta, w.max_sym)
+            oracle.decode_chunk(st, model, olm, obo, encs[c][i], w.lam, w.beta, w.max_sym, prune_k=prune_k)
 
     t0 = time.perf_counter()
     with concurrent.futures.ThreadPoolExecutor(max_workers=threads) as ex:
@@ -247,10 +247,11 @@ def run_reference(args, w):
     models = oracle_models(w, lmA, ph, E, W, extra)
     # warm-up steps, then K timed steps; each step decodes a bounded sample
     for _ in range(args.warmup):
-        oracle_baseline(w, models, list(range(2)), 1)
+        oracle_baseline(w, models, list(range(2)), 1, prune_k=args.prune_k)
     vals, dts = [], []
     for k in range(args.steps):
-        v, cores, sample, dt = oracle_baseline(w, models, list(range(k * n_str, (k + 1) * n_str)), 1)
+        v, cores, sample, dt = oracle_baseline(w, models, list(range(k * n_str, (k + 1) * n_str)), 1,
+                                               prune_k=args.prune_k)
         vals.append(v)
         dts.append(dt)
     value = float(np.mean(vals))
@@ -261,7 +262,10 @@ def run_reference(args, w):
             "config": dict(workload_config(w, lmA.total + sum(a.total for a, _ in extra), ph.n if ph else 0),
                            **({"lms": 1 + len(extra), "lm_weights": [1.0] + [wt for _, wt in extra],
                                "workload": f"cfg{w.cfg} {w.name} + {len(extra)} more LMs (half size, weight 0.5)"}
-                              if extra else {})),
+                              if extra else {}),
+                           **({"prune_k": args.prune_k,
+                               "workload": f"cfg{w.cfg} {w.name}, fusion pruned to the acoustic top {args.prune_k}"}
+                              if args.prune_k else {})),
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
                              "sample": f"per step: {sample}"},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
@@ -292,7 +296,7 @@ def run_ours(args, w):
     bo = tsd.Boost.from_phrases(w.V, ph, w.bonus) if ph is not None else None
     dec = tsd.Decoder(w.V, w.H, torch.from_numpy(W.view(np.int16)).to(dev), torch.from_numpy(E.view(np.int16)).to(dev),
                       lm=None if lms else lm, lms=lms, boost=bo, max_symbols=w.max_sym, beam_k=w.beam,
-                      max_streams=w.B, max_T=w.T)
+                      max_streams=w.B, max_T=w.T, prune_k=args.prune_k)
     slots = [dec.open() for _ in range(w.B)]
     slots_np = np.array(slots, dtype=np.int32)
     n_chunks = args.warmup + args.steps + 1
@@ -473,6 +477,9 @@ def run_ours(args, w):
                            **({"lms": 1 + len(extra), "lm_weights": [1.0] + [wt for _, wt in extra],
                                "workload": f"cfg{w.cfg} {w.name} + {len(extra)} more LMs (half size, weight 0.5)"}
                               if extra else {}),
+                           **({"prune_k": args.prune_k,
+                               "workload": f"cfg{w.cfg} {w.name}, fusion pruned to the acoustic top {args.prune_k}"}
+                              if args.prune_k else {}),
                            l2="flushed (256 MB write) before every timed step, outside the step's events",
                            parallelism=f"dp{ws} (independent streams per GPU)"),
             "e2e": {"value": e2e_val, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
@@ -488,7 +495,8 @@ def run_ours(args, w):
             "clocks": clk.summary()}
     if not args.no_cpu_baseline and ws == 1:
         models = oracle_models(w, lmA, ph, E, W, extra)
-        v, cores, sample, dt = oracle_baseline(w, models, list(range(args.cpu_streams)), args.cpu_chunks)
+        v, cores, sample, dt = oracle_baseline(w, models, list(range(args.cpu_streams)), args.cpu_chunks,
+                                               prune_k=args.prune_k)
         line["cpu_baseline"] = {"value": v, "unit": UNIT, "cores": cores, "kind": "oracle",
                                 "sample": sample, "seconds": dt}
     print(json.dumps(line), flush=True)
@@ -507,6 +515,8 @@ def main():
     ap.add_argument("--ref-streams", type=int, default=64)
     ap.add_argument("--streams", type=int, default=None, help="streams B per GPU (default: the config's)")
     ap.add_argument("--extra-lms", type=int, default=0, help="fuse this many further LMs (several-LM workload)")
+    ap.add_argument("--prune-k", type=int, default=0,
+                    help="pruned fusion over the acoustic model's k best outputs (0: every label)")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")

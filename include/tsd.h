@@ -176,6 +176,12 @@ typedef struct {
   int32_t beam_k;      /* 1 = greedy; 2..8 = beam search */
   int32_t max_streams; /* stream slots; max_streams * beam_k <= 4096 */
   int32_t max_T;       /* frames per chunk, 1 <= max_T <= 4096 */
+  int32_t prune_k;     /* 0: fusion over every label (Eq. 1 as written).  1..8: pruned
+                          fusion: the LM and boost terms re-rank only the acoustic
+                          model's prune_k best outputs (blank included, ties to the
+                          lower id), the reading of Sec. III-C's remark that fusion
+                          only re-ranks the candidates the model proposes.  Needs
+                          greedy decoding and at most one LM. */
 } tsd_decoder_cfg;
 
 /* Creates a decoder for one joint network and optional LM / phrase tree.

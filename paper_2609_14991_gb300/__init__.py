@@ -36,7 +36,7 @@ _P = ctypes.POINTER
 
 class DecoderCfg(ctypes.Structure):
     _fields_ = [("V", _i32), ("H", _i32), ("max_symbols", _i32), ("beam_k", _i32), ("max_streams", _i32),
-                ("max_T", _i32)]
+                ("max_T", _i32), ("prune_k", _i32)]
 
 
 SIGNATURES = {
@@ -238,14 +238,15 @@ class Decoder:
 
     def __init__(self, V: int, H: int, W_out, E, lm: Optional[NGram] = None, boost: Optional[Boost] = None,
                  max_symbols: int = 5, beam_k: int = 1, max_streams: int = 64, max_T: int = 64, stream=None,
-                 lms: Optional[Sequence[Tuple[NGram, float]]] = None):
+                 lms: Optional[Sequence[Tuple[NGram, float]]] = None, prune_k: int = 0):
         """lms: several LMs as (NGram, w) pairs instead of lm (LM i enters Eq. 1
-        with weight lambda * w; ``tsd_decoder_create_multi``)."""
+        with weight lambda * w; ``tsd_decoder_create_multi``).  prune_k > 0:
+        pruned fusion over the acoustic model's prune_k best outputs."""
         import torch
 
         assert W_out.is_cuda and E.is_cuda and W_out.element_size() == 2 and E.element_size() == 2
         assert tuple(W_out.shape) == (H, V + 1) and tuple(E.shape) == (V + 1, H)
-        self.cfg = DecoderCfg(V, H, max_symbols, beam_k, max_streams, max_T)
+        self.cfg = DecoderCfg(V, H, max_symbols, beam_k, max_streams, max_T, prune_k)
         self.V, self.H, self.max_symbols, self.beam_k = V, H, max_symbols, beam_k
         self.lm, self.boost = lm, boost  # kept alive: the decoder borrows them
         W_out = W_out.contiguous()

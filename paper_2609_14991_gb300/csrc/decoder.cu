@@ -51,6 +51,7 @@ void enqueue_chunk(tsd_decoder* d, int M, int T, cudaStream_t s, const std::vect
     const bool pdl = d->pdl && !ev && step > 0;  // the first launch follows the parameter copy
     mark();
     if (d->cfg.beam_k > 1) launch_row_beam(v, M / d->cfg.beam_k, step, step == S ? 1 : 0, d->row_smem, s, pdl);
+    else if (d->cfg.prune_k > 0) launch_row_pruned(v, M, step, step == S ? 1 : 0, s, pdl);
     else launch_row(v, M, step, step == S ? 1 : 0, d->row_smem, s, pdl);
     if (step < S) {
       mark();
@@ -100,6 +101,11 @@ tsd_status create_impl(const tsd_decoder_cfg* cfg, const void* W_out_bf16, const
     if (lms[i]->view.V != c.V) return fail(TSD_EINVAL, "tsd_decoder_create: LM %d has V=%d, decoder V=%d", i, lms[i]->view.V, c.V);
   }
   if (n_lms > 1 && c.beam_k > 1) return fail(TSD_EINVAL, "tsd_decoder_create: several LMs need greedy decoding (beam_k 1)");
+  if (c.prune_k < 0 || c.prune_k > 8) return fail(TSD_EINVAL, "tsd_decoder_create: prune_k=%d outside [0, 8]", c.prune_k);
+  if (c.prune_k > 0 && (c.beam_k > 1 || n_lms > 1))
+    return fail(TSD_EINVAL, "tsd_decoder_create: pruned fusion needs greedy decoding and at most one LM");
+  if (c.prune_k > 0 && ((c.V + 1 + kNPad - 1) / kNPad * kNPad / 64) * c.prune_k > 512)
+    return fail(TSD_EINVAL, "tsd_decoder_create: prune_k * (V+1)/64 must be <= 512");
   const tsd_ngram* lm = n_lms > 0 ? lms[0] : nullptr;
   if (c.V < 1 || c.V > 16384) return fail(TSD_EINVAL, "tsd_decoder_create: V=%d out of range [1, 16384]", c.V);
   if (c.H < 64 || c.H > 8192 || c.H % 64) return fail(TSD_EINVAL, "tsd_decoder_create: H=%d must be a multiple of 64 in [64, 8192]", c.H);
@@ -158,6 +164,13 @@ tsd_status create_impl(const tsd_decoder_cfg* cfg, const void* W_out_bf16, const
       (st = A.alloc(&stl, SK)) || (st = A.alloc(&stc, SK * kTrChain)) || (st = A.alloc(&pdev, d->params_bytes))) {
     A.release();
     return st;
+  }
+  const int topk = c.beam_k > 1 ? c.beam_k : c.prune_k;
+  if (c.beam_k == 1 && c.prune_k > 0) {
+    if ((st = A.alloc(&bpart, (size_t)d->M_pad * (d->N_pad / 64) * (1 + topk)))) {
+      A.release();
+      return st;
+    }
   }
   if (c.beam_k > 1) {
     const size_t pool = (size_t)c.max_streams * kPoolCap;
@@ -225,6 +238,8 @@ tsd_status create_impl(const tsd_decoder_cfg* cfg, const void* W_out_bf16, const
   v.H = c.H;
   v.max_sym = c.max_symbols;
   v.K = c.beam_k;
+  v.topk = topk;
+  v.prune = c.prune_k;
   d->n_ptiles = d->N_pad / d->jtc->bn;
   v.n_ptiles = d->n_ptiles;
   v.V4 = d->V4;
@@ -797,6 +812,8 @@ extern "C" tsd_status tsd_decoder_set_joint_kernel(tsd_decoder* d, int32_t kind)
   clear_error();
   if (!d) return fail(TSD_EINVAL, "tsd_decoder_set_joint_kernel: NULL decoder");
   if (kind != 0 && kind != 1) return fail(TSD_EINVAL, "tsd_decoder_set_joint_kernel: kind must be 0 or 1");
+  if (kind == 1 && d->cfg.prune_k > 0)
+    return fail(TSD_EINVAL, "tsd_decoder_set_joint_kernel: the CUDA-core kernel has no pruned-fusion epilogue");
   d->joint_kind = kind;
   d->n_ptiles = kind == 0 ? d->N_pad / d->jtc->bn : d->N_pad / kPartialCols;
   d->view.n_ptiles = d->n_ptiles;
@@ -842,6 +859,7 @@ extern "C" tsd_status tsd_decoder_replay(tsd_decoder* d, int32_t kernel, int32_t
   if (algo_bytes) TSD_CUDA(cudaMemsetAsync(d->view.ctr, 0, sizeof(unsigned long long), s));
   for (int i = 0; i < reps; ++i) {
     if (kernel == 0 && d->cfg.beam_k > 1) launch_row_beam(d->view, d->last_n, S - 1, 2, d->row_smem, s, false);
+    else if (kernel == 0 && d->cfg.prune_k > 0) launch_row_pruned(d->view, M, S - 1, 2, s, false);
     else if (kernel == 0) launch_row(d->view, M, S - 1, 2, d->row_smem, s, false);
     else if (d->joint_kind == 0) launch_joint_tc(*d->jtc, d->view, M, 1 << 30, s, false);
     else launch_joint(d->view, M, 1 << 30, s);

@@ -59,6 +59,8 @@ struct DecView {
   int32_t* pool_tok;    // [slots][pool_cap] label of the node
   int32_t* pool_n;      // [slots] nodes used
   int32_t pool_cap;
+  int32_t topk;       // entries per row and tile in bpart: beam width, or prune_k
+  int32_t prune;      // prune_k (0: fusion over every label)
   int32_t n_lm;       // n-gram LMs fused (0: none; several: greedy only)
   int32_t lm_stride;  // hypothesis slots per LM in s_lm_len / s_lm_chain
   LmView lmx[kMaxLm]; // every LM; lmx[0] equals lm
@@ -80,6 +82,7 @@ void launch_defaults(const DecView& d, cudaStream_t s);
 size_t row_smem_bytes(int V4, int n_lm);
 cudaError_t prepare_kernels(size_t row_smem);
 void launch_row_beam(const DecView& d, int n, int step, int mode, size_t smem, cudaStream_t s, bool pdl);
+void launch_row_pruned(const DecView& d, int M, int step, int mode, cudaStream_t s, bool pdl);
 void launch_open_beam(const DecView& d, int slot, cudaStream_t s);
 cudaError_t prepare_beam_kernels(size_t row_smem);
 constexpr int kPoolCap = 8192;  // label-sequence nodes per beam stream

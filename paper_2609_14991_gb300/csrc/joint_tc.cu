@@ -161,7 +161,9 @@ struct Smem {
 };
 
 // BEAM: instead of the single best fused label, each row keeps the top-K
-// (K = beam width <= 8) fused values of the tile, ties to the lower label.
+// (K = d.topk <= 8: the beam width, or the pruned-fusion candidate count)
+// values of the tile, ties to the lower label.  With pruned fusion (d.prune)
+// the values are the plain logits: no bias tile is loaded.
 template <int BN, bool BEAM>
 __global__ void __launch_bounds__(kThreads, 1)
     k_joint_tc(DecView d, int step, const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
@@ -178,6 +180,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int n0 = blockIdx.x * BN, m0 = blockIdx.y * kBM;
+  const bool use_bias = !(BEAM && d.prune);
   const int M = d.params->n * d.K;
   const int KB = d.H / kBK;
 
@@ -220,8 +223,11 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == 0) {
     if (lane == 0) {
       // the bias tile first: the epilogue needs it as soon as the MMAs end
-      mbar_expect_tx(biasbar, S::kEarly * S::kBoxBytes);
-      for (int c = 0; c < S::kEarly; ++c) tma_load_2d(bias_early + c * S::kBoxBytes, &tmBias, biasbar, n0 + 32 * c, m0);
+      if (use_bias) {
+        mbar_expect_tx(biasbar, S::kEarly * S::kBoxBytes);
+        for (int c = 0; c < S::kEarly; ++c)
+          tma_load_2d(bias_early + c * S::kBoxBytes, &tmBias, biasbar, n0 + 32 * c, m0);
+      }
       int issued = 0;
       for (int kb = 0; kb < KB; ++kb) {
         const int s = kb % S::kStages;
@@ -278,7 +284,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int N = d.N, V = d.V;
     float mx = kNegInf, se = 0.f, bv = kNegInf;
     int bi = INT_MAX;
-    const int K = d.K;
+    const int K = d.topk;
     float tv[8];
     int ti[8];
 #pragma unroll
@@ -289,13 +295,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     fence_after();
     // the second half of a 256-wide bias tile goes into the drained stages
     // (every MMA has completed, so nothing reads them any more)
-    const bool late = ok && S::kEarly < S::kBoxes;
+    const bool late = ok && use_bias && S::kEarly < S::kBoxes;
     if (late && warp == 2 && lane == 0) {
       mbar_expect_tx(biasbar + 1, (S::kBoxes - S::kEarly) * S::kBoxBytes);
       for (int c = S::kEarly; c < S::kBoxes; ++c)
         tma_load_2d(smem + (c - S::kEarly) * S::kBoxBytes, &tmBias, biasbar + 1, n0 + 32 * c, m0);
     }
-    const bool have_early = __all_sync(0xffffffffu, mbar_wait(biasbar, 0));
+    const bool have_early = use_bias ? __all_sync(0xffffffffu, mbar_wait(biasbar, 0)) : true;
     if (!have_early) {
       ok = false;
       if (lane == 0) atomicOr(d.err, 16);
@@ -307,7 +313,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll 1
       for (int c = half; c < BN / 32; c += 2) {
         __syncwarp();  // the per-chunk selection branches; tcgen05.ld wants the warp whole
-        if (c >= S::kEarly && !late_done) {
+        if (use_bias && c >= S::kEarly && !late_done) {
           late_done = true;
           if (!__all_sync(0xffffffffu, mbar_wait(biasbar + 1, 0))) {
             if (lane == 0) atomicOr(d.err, 32);
@@ -316,10 +322,15 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         const unsigned char* box = (c < S::kEarly) ? bias_early + c * S::kBoxBytes : smem + (c - S::kEarly) * S::kBoxBytes;
         float b[32];
+        if (use_bias) {
 #pragma unroll
-        for (int j = 0; j < 8; ++j) {
-          const float4 v = *reinterpret_cast<const float4*>(box + row * 128 + ((j ^ sw) << 4));
-          b[4 * j] = v.x; b[4 * j + 1] = v.y; b[4 * j + 2] = v.z; b[4 * j + 3] = v.w;
+          for (int j = 0; j < 8; ++j) {
+            const float4 v = *reinterpret_cast<const float4*>(box + row * 128 + ((j ^ sw) << 4));
+            b[4 * j] = v.x; b[4 * j + 1] = v.y; b[4 * j + 2] = v.z; b[4 * j + 3] = v.w;
+          }
+        } else {
+#pragma unroll
+          for (int j = 0; j < 32; ++j) b[j] = 0.f;
         }
         float l[32];
         tmem_ld32(tbase + (uint32_t)(c * 32), l);
@@ -543,7 +554,7 @@ void launch_joint_tc(const JointTc& jt, const DecView& d, int M, int step, cudaS
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = pdl ? 1 : 0;
-  const bool beam = d.K > 1;
+  const bool beam = d.topk > 1 || d.prune > 0;  // the top-K epilogue
   if (jt.bn == 256) {
     cfg.dynamicSmemBytes = Smem<256>::kBytes;
     if (beam) cudaLaunchKernelEx(&cfg, k_joint_tc<256, true>, d, step, jt.mapA, jt.mapB, jt.mapBias);
