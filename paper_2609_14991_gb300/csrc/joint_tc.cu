@@ -364,25 +364,41 @@ __global__ void __launch_bounds__(kThreads, 1)
             bi = c0 + j;
           }
         } else if (fm > tmin) {
+          // Take the chunk's values in decreasing order while they beat the
+          // K-th kept value: at most K rounds, usually none after the first
+          // chunks.  Each round finds the first (lowest-label) position of the
+          // chunk maximum, bubbles it into the sorted list (an equal value
+          // already kept stays ahead: it has the lower label), masks it out
+          // and takes the next maximum.
+          float cmx = fm;
+#pragma unroll 1
+          for (int it = 0; it < K && cmx > tmin; ++it) {
+            int jx = 31;
 #pragma unroll
-          for (int i = 0; i < 32; ++i) {
-            const float f = b[i];
-            if (f > tmin) {
-              // bubble the new value into the sorted list (labels arrive in
-              // increasing order, so a later equal value stays behind)
-              float cv = f;
-              int ci = c0 + i;
+            for (int i = 31; i >= 0; --i)
+              if (b[i] == cmx) jx = i;
+            float cv = cmx;
+            int ci = c0 + jx;
 #pragma unroll
-              for (int j = 0; j < 8; ++j) {
-                if (j < K && cv > tv[j]) {
-                  const float tf = tv[j]; tv[j] = cv; cv = tf;
-                  const int tk = ti[j]; ti[j] = ci; ci = tk;
-                }
+            for (int j = 0; j < 8; ++j) {
+              if (j < K && cv > tv[j]) {
+                const float tf = tv[j]; tv[j] = cv; cv = tf;
+                const int tk = ti[j]; ti[j] = ci; ci = tk;
               }
-#pragma unroll
-              for (int j = 0; j < 8; ++j)
-                if (j == K - 1) tmin = tv[j];
             }
+#pragma unroll
+            for (int j = 0; j < 8; ++j)
+              if (j == K - 1) tmin = tv[j];
+#pragma unroll
+            for (int i = 0; i < 32; ++i)
+              if (i == jx) b[i] = kNegInf;
+#pragma unroll
+            for (int i = 0; i < 16; ++i) u[i] = fmaxf(b[i], b[i + 16]);
+#pragma unroll
+            for (int w = 8; w > 0; w >>= 1)
+#pragma unroll
+              for (int i = 0; i < w; ++i) u[i] = fmaxf(u[i], u[i + w]);
+            cmx = u[0];
           }
         }
         if (cm != kNegInf) {
