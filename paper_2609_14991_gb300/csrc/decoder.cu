@@ -144,6 +144,7 @@ tsd_status create_impl(const tsd_decoder_cfg* cfg, const void* W_out_bf16, const
   float* bias;
   float4* part;
   int32_t *rt, *rs, *rc, *sl, *sll, *slc, *stl, *stc, *err;
+  int4 *slr = nullptr, *strc = nullptr;
   unsigned long long* ctr;
   float2* bpart = nullptr;
   float* dflt = nullptr;
@@ -161,7 +162,8 @@ tsd_status create_impl(const tsd_decoder_cfg* cfg, const void* W_out_bf16, const
       (st = A.alloc(&part, (size_t)d->M_pad * (d->N_pad / 64))) || (st = A.alloc(&err, 1)) || (st = A.alloc(&ctr, 2)) || (st = A.alloc(&dflt, (size_t)d->V4)) || (st = A.alloc(&droot, (size_t)(d->V4 + 31) / 32)) || (st = A.alloc(&rt, (size_t)d->M_pad)) ||
       (st = A.alloc(&rs, (size_t)d->M_pad)) || (st = A.alloc(&rc, (size_t)d->M_pad)) ||
       (st = A.alloc(&sl, SK)) || (st = A.alloc(&sll, SK * NL)) || (st = A.alloc(&slc, SK * NL * kLmChain)) ||
-      (st = A.alloc(&stl, SK)) || (st = A.alloc(&stc, SK * kTrChain)) || (st = A.alloc(&pdev, d->params_bytes))) {
+      (st = A.alloc(&stl, SK)) || (st = A.alloc(&stc, SK * kTrChain)) || (st = A.alloc(&pdev, d->params_bytes)) ||
+      (st = A.alloc(&slr, SK * kLmChain)) || (st = A.alloc(&strc, SK * kTrChain))) {
     A.release();
     return st;
   }
@@ -258,6 +260,8 @@ tsd_status create_impl(const tsd_decoder_cfg* cfg, const void* W_out_bf16, const
   v.s_lm_chain = slc;
   v.s_tr_len = stl;
   v.s_tr_chain = stc;
+  v.s_lm_rec = slr;
+  v.s_tr_rec = strc;
   v.has_lm = lm ? 1 : 0;
   v.has_tr = boost ? 1 : 0;
   if (lm) v.lm = lm->view;
@@ -642,6 +646,11 @@ extern "C" tsd_status tsd_stream_import(tsd_decoder* d, int32_t slot, const void
                              (st = get(v.pool_tok + (size_t)slot * v.pool_cap, (size_t)hd.pool_used))))
       return st;
     TSD_CUDA(cudaMemcpy(v.pool_n + slot, &hd.pool_used, 4, cudaMemcpyHostToDevice));
+  } else {
+    // the greedy pass keeps each chain element's table records: derive them
+    launch_fix_records(v, slot, d->last_stream);
+    TSD_CUDA(cudaGetLastError());
+    TSD_CUDA(cudaStreamSynchronize(d->last_stream));
   }
   return TSD_OK;
 }

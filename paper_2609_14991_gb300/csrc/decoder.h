@@ -42,6 +42,10 @@ struct DecView {
   int32_t* s_lm_chain;  // [LMs][slots][kLmChain]
   int32_t* s_tr_len;
   int32_t* s_tr_chain;  // [.][kTrChain]
+  // greedy: the table records of each chain element, kept with the chain so
+  // the next step's searches start without fetching them:
+  int4* s_lm_rec;       // [slots][kLmChain] first LM: (first arc, arcs, cumulative backoff bits, 0)
+  int4* s_tr_rec;       // [slots][kTrChain] trie: (first child, children, depth of the children, 0)
   LmView lm;
   TrieView tr;
   int32_t has_lm, has_tr;
@@ -76,6 +80,7 @@ constexpr int kRowThreads = 256;
 
 void launch_repack(const uint16_t* W, uint16_t* Wt, int H, int N, int N_pad, cudaStream_t s);
 void launch_open(const DecView& d, int slot, cudaStream_t s);
+void launch_fix_records(const DecView& d, int slot, cudaStream_t s);
 void launch_row(const DecView& d, int M, int step, int mode, size_t smem, cudaStream_t s, bool pdl);
 void launch_joint(const DecView& d, int M, int step, cudaStream_t s);
 void launch_defaults(const DecView& d, cudaStream_t s);

@@ -168,6 +168,17 @@ __device__ __forceinline__ void scatter_trie_node(const int32_t* ch_tok, int b, 
   }
 }
 
+// Step 1 when the chains' records are already in rc: the scratch reset only.
+__device__ __forceinline__ void bias_init(const DecView& d, float* lmv, uint8_t* dep) {
+  const float unset = unset_value();
+  float4* l4 = reinterpret_cast<float4*>(lmv);
+  uint32_t* d4 = reinterpret_cast<uint32_t*>(dep);
+  for (int q = threadIdx.x; q < d.V4 / 4; q += blockDim.x) {
+    l4[q] = make_float4(unset, unset, unset, unset);
+    d4[q] = 0u;
+  }
+}
+
 // Step 2: the dense fusion bias row lambda*log p_LM(v|state) +
 // beta*bonus*(goto depth - current depth) for every label v (blank: 0).
 // LM chain levels are applied deepest first, each label keeping the first

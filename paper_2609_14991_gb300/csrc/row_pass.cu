@@ -152,7 +152,8 @@ __global__ void __launch_bounds__(kRowThreads, 7) k_row(DecView d, int step, int
   __shared__ int s_lm_tgt[kMaxLm][kLmChain];    // target state of y's arc at each LM level (-2 none)
   __shared__ int s_tr_node[kTrChain], s_tr_nxt[kTrChain];  // child by y of each trie chain node (-1 none)
   __shared__ int s_uni_tgt[kMaxLm], s_root_child, s_root_next;
-  __shared__ row::ChainRecs rc;
+  __shared__ row::ChainRecs rc;   // records of the chains the bias row is built from
+  __shared__ row::ChainRecs rco;  // one LM: records of the current chains, kept with the state
 
   // The row state below was written by the previous row pass; under
   // programmatic launch this grid may start before its own wait, so these
@@ -182,9 +183,24 @@ __global__ void __launch_bounds__(kRowThreads, 7) k_row(DecView d, int step, int
   const int slot = s_slot, T = s_T;
   if (tid < L * kLmChain) {
     const int i = tid / kLmChain, l = tid % kLmChain;
-    if (l < s_lm_len[i]) s_lm[i][l] = __ldcg(d.s_lm_chain + ((size_t)i * d.lm_stride + slot) * kLmChain + l);
+    if (l < s_lm_len[i]) {
+      s_lm[i][l] = __ldcg(d.s_lm_chain + ((size_t)i * d.lm_stride + slot) * kLmChain + l);
+      if (L == 1) {
+        const int4 q = __ldcg(d.s_lm_rec + (size_t)slot * kLmChain + l);
+        rco.lb[l] = q.x;
+        rco.lc[l] = q.y;
+      }
+    }
   }
-  if (tid >= 64 && tid - 64 < s_tr_len) s_tr[tid - 64] = __ldcg(d.s_tr_chain + slot * kTrChain + tid - 64);
+  if (tid >= 64 && tid - 64 < s_tr_len) {
+    const int k = tid - 64;
+    s_tr[k] = __ldcg(d.s_tr_chain + slot * kTrChain + k);
+    if (L == 1) {
+      const int4 q = __ldcg(d.s_tr_rec + (size_t)slot * kTrChain + k);
+      rco.tb[k] = q.x;
+      rco.tc[k] = q.y;
+    }
+  }
   // The encoder frames this step can use (t, or t+1 after a frame advance)
   // go to L1 now, while the previous kernel still runs: no kernel of the
   // chunk writes them.  (The call's bias defaults are not prefetched: every
@@ -253,8 +269,15 @@ __global__ void __launch_bounds__(kRowThreads, 7) k_row(DecView d, int step, int
           const int32_t* st_begin = TSD_LMX(d, m, st_begin);
           const int32_t* st_count = TSD_LMX(d, m, st_count);
           const int32_t* arc_tgt = TSD_LMX(d, m, arc_tgt);
-          int st = s_lm[m][l];
-          int b = __ldg(st_begin + st), c = __ldg(st_count + st);
+          int b, c;
+          if (L == 1) {  // records kept with the chain
+            b = rco.lb[l];
+            c = rco.lc[l];
+          } else {
+            const int st = s_lm[m][l];
+            b = __ldg(st_begin + st);
+            c = __ldg(st_count + st);
+          }
           int i = warp_find(TSD_LMX(d, m, arc_tok) + b, c, y, lane);
           if (lane == 0) {
             const int tg = (i >= 0) ? __ldg(arc_tgt + b + i) : -2;
@@ -267,8 +290,15 @@ __global__ void __launch_bounds__(kRowThreads, 7) k_row(DecView d, int step, int
           }
         } else {
           int k = task - nl;
-          int q = s_tr[k];
-          int b = __ldg(d.tr.nd_begin + q), c = __ldg(d.tr.nd_count + q);
+          int b, c;
+          if (L == 1) {
+            b = rco.tb[k];
+            c = rco.tc[k];
+          } else {
+            const int q = s_tr[k];
+            b = __ldg(d.tr.nd_begin + q);
+            c = __ldg(d.tr.nd_count + q);
+          }
           int i = warp_find(d.tr.ch_tok + b, c, y, lane);
           if (lane == 0) {
             s_tr_node[k] = (i >= 0) ? __ldg(d.tr.ch_node + b + i) : -1;
@@ -343,6 +373,19 @@ __global__ void __launch_bounds__(kRowThreads, 7) k_row(DecView d, int step, int
   }
 
   if (mode == 1) {
+    // the chunk's last decision: the new chains' records for the next chunk
+    if (L == 1 && commit) {
+      if (tid < s_lm_len[0]) {
+        const int st = s_lm[0][tid];
+        d.s_lm_rec[(size_t)slot * kLmChain + tid] =
+            make_int4(__ldg(d.lm.st_begin + st), __ldg(d.lm.st_count + st), __float_as_int(__ldg(d.lm.st_cum + st)), 0);
+      }
+      if (tid >= 64 && tid - 64 < s_tr_len) {
+        const int q = s_tr[tid - 64];
+        d.s_tr_rec[(size_t)slot * kTrChain + tid - 64] =
+            make_int4(__ldg(d.tr.nd_begin + q), __ldg(d.tr.nd_count + q), __ldg(d.tr.nd_depth + q) + 1, 0);
+      }
+    }
     if (tid == 0) s_out_count[r] = s_cnt;
     return;
   }
@@ -373,6 +416,11 @@ __global__ void __launch_bounds__(kRowThreads, 7) k_row(DecView d, int step, int
   int nl = s_lm_len[0];
   if (L == 1) {
     row::bias_prepare(d, s_lm[0], nl, s_tr, nt, rc, lmv, dep);
+    if (commit) {  // the records stay with the chains for the next step's searches
+      if (tid < nl) d.s_lm_rec[(size_t)slot * kLmChain + tid] = make_int4(rc.lb[tid], rc.lc[tid], __float_as_int(rc.lo[tid]), 0);
+      if (tid >= 32 && tid - 32 < nt)
+        d.s_tr_rec[(size_t)slot * kTrChain + tid - 32] = make_int4(rc.tb[tid - 32], rc.tc[tid - 32], rc.td[tid - 32], 0);
+    }
     row::build_joint_input(d, s_enc + ((size_t)r * T + t) * d.H, s_last, r);
     row::bias_finish(d, nl, nt, rc, s_lam, s_beta, d.bias + (size_t)r * d.N_pad, lmv, dep);
     if (counting && tid == 0) lm_bytes = lm_level_bytes(rc, nl, s_y != V && evaluated);
@@ -396,6 +444,20 @@ __global__ void __launch_bounds__(kRowThreads, 7) k_row(DecView d, int step, int
     if (s_y != V && evaluated)
       for (int k = 0; k < nt; ++k) bytes += 8 + 4ull * (32 - __clz(rc.tc[k] + 1)) + 8;
     atomicAdd(d.ctr, bytes);
+  }
+}
+
+// After a chain is written from the host: its elements' table records.
+__global__ void k_fix_records(DecView d, int slot) {
+  const int l = threadIdx.x;
+  if (d.has_lm && l < kLmChain && l < d.s_lm_len[slot]) {
+    const int st = d.s_lm_chain[(size_t)slot * kLmChain + l];
+    d.s_lm_rec[(size_t)slot * kLmChain + l] =
+        make_int4(d.lm.st_begin[st], d.lm.st_count[st], __float_as_int(d.lm.st_cum[st]), 0);
+  }
+  if (d.has_tr && l < kTrChain && l < d.s_tr_len[slot]) {
+    const int q = d.s_tr_chain[(size_t)slot * kTrChain + l];
+    d.s_tr_rec[(size_t)slot * kTrChain + l] = make_int4(d.tr.nd_begin[q], d.tr.nd_count[q], d.tr.nd_depth[q] + 1, 0);
   }
 }
 
@@ -464,6 +526,8 @@ void launch_repack(const uint16_t* W, uint16_t* Wt, int H, int N, int N_pad, cud
 }
 
 void launch_open(const DecView& d, int slot, cudaStream_t s) { k_open<<<1, 32, 0, s>>>(d, slot); }
+
+void launch_fix_records(const DecView& d, int slot, cudaStream_t s) { k_fix_records<<<1, 32, 0, s>>>(d, slot); }
 
 void launch_row(const DecView& d, int M, int step, int mode, size_t smem, cudaStream_t s, bool pdl) {
   cudaLaunchConfig_t cfg = {};
