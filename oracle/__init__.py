@@ -71,6 +71,9 @@ def lib() -> ctypes.CDLL:
                                          i32, dbl, vp, vp, vp, i32, vp], i32),
             "oracle_decode_chunk_pruned": ([vp, vp, vp, i32, i32, vp, vp, vp, i32, dbl, dbl, i32, i32, dbl, vp, vp,
                                             vp, i32, dbl, vp, vp, vp, i32, vp], i32),
+            "oracle_decode_chunk_pred": ([vp, vp, vp, i32, i32, i32, i32, vp, vp, vp, vp, vp, vp, vp, vp, vp, i32,
+                                          dbl, dbl, i32, vp, vp, vp, i32, dbl, vp, vp, vp, i32, vp], i32),
+            "oracle_pred_state": ([vp, vp, vp], i32),
             "oracle_beam_chunk": ([vp, vp, vp, i32, i32, vp, vp, vp, i32, dbl, dbl, i32], i32),
             "oracle_beam_hyp": ([vp, i32, vp, i64, vp, vp], i64),
             "oracle_beam_chunk_follow": ([vp, vp, vp, i32, i32, vp, vp, vp, i32, dbl, dbl, i32, vp, vp, vp, dbl,
@@ -204,6 +207,14 @@ class Stream:
         y = _i32(y)
         lib().oracle_stream_set_history(self.h, _p(y), len(y), int(rho))
 
+    def pred_state(self, D: int):
+        """(h as bf16 bits [D], c [D]) of the prediction network, or None
+        before its first step."""
+        h = np.zeros(D, dtype=np.uint16)
+        c = np.zeros(D, dtype=np.float64)
+        ok = lib().oracle_pred_state(self.h, _p(h), _p(c))
+        return (h, c) if ok else None
+
     def beam_hyps(self, with_rho: bool = False):
         """[(labels, score)] or, with_rho, [(labels, score, restart index)]."""
         out = []
@@ -247,9 +258,25 @@ def fused_row(stream: Stream, model: Model, lm: Optional[LM], boost: Optional[Bo
     return out
 
 
+class PredNet:
+    """Prediction network and joint projections (synth.PredWeights layout)."""
+
+    def __init__(self, V: int, H: int, p):
+        self.V, self.H, self.D, self.Henc = V, H, p.D, p.Henc
+        self.Ep = np.ascontiguousarray(p.Ep, dtype=np.uint16)
+        self.Wg = np.ascontiguousarray(p.Wg, dtype=np.uint16)
+        self.bg = np.ascontiguousarray(p.bg, dtype=np.float32)
+        self.Wp = np.ascontiguousarray(p.Wp, dtype=np.uint16)
+        self.bp = np.ascontiguousarray(p.bp, dtype=np.float32)
+        self.We = np.ascontiguousarray(p.We, dtype=np.uint16)
+        self.be = np.ascontiguousarray(p.be, dtype=np.float32)
+        assert self.Ep.shape == (V + 1, self.D) and self.Wg.shape == (2 * self.D, 4 * self.D)
+        assert self.Wp.shape == (self.D, H) and self.We.shape == (self.Henc, H)
+
+
 def decode_chunk(stream: Stream, model: Model, lm: Optional[LM], boost: Optional[Boost], enc: np.ndarray,
                  lam: float, beta: float, max_sym: int, follow=None, gap_tol: float = 1e-3, prune_k: int = 0,
-                 am_tol: float = 2e-2):
+                 am_tol: float = 2e-2, pred: Optional[PredNet] = None):
     """Greedy decode of one chunk enc [T, H] for one stream.
 
     lm: None, one LM (weight lam), or a list of (LM, w) pairs: LM i enters
@@ -258,6 +285,8 @@ def decode_chunk(stream: Stream, model: Model, lm: Optional[LM], boost: Optional
     under test, which the oracle checks and then follows.
     prune_k > 0: pruned fusion over the acoustic model's prune_k best outputs
     (one LM); am_tol is the logit tolerance at the edge of that set.
+    pred: the stateful form (prediction network + joint projections); enc
+    rows are then pred.Henc wide and model.E is not used.
     Returns (tokens, frames, scores, report[8])."""
     enc = np.ascontiguousarray(enc, dtype=np.uint16)
     T = enc.shape[0]
@@ -271,7 +300,14 @@ def decode_chunk(stream: Stream, model: Model, lm: Optional[LM], boost: Optional
         fargs = (_p(ft), _p(ff), _p(fs), len(ft))
     else:
         fargs = (None, None, None, 0)
-    if prune_k > 0:
+    if pred is not None:
+        assert not isinstance(lm, (list, tuple)) and prune_k == 0
+        n = lib().oracle_decode_chunk_pred(stream.h, lm.h if lm else None, boost.h if boost else None, model.V,
+                                           model.H, pred.Henc, pred.D, _p(pred.Ep), _p(pred.Wg), _p(pred.bg),
+                                           _p(pred.Wp), _p(pred.bp), _p(pred.We), _p(pred.be), _p(model.W), _p(enc),
+                                           T, float(lam), float(beta), int(max_sym), *fargs, float(gap_tol),
+                                           _p(ot), _p(of), _p(osc), cap, _p(rep))
+    elif prune_k > 0:
         assert not isinstance(lm, (list, tuple)), "pruned fusion takes one LM"
         n = lib().oracle_decode_chunk_pruned(stream.h, lm.h if lm else None, boost.h if boost else None, model.V,
                                              model.H, _p(model.E), _p(model.W), _p(enc), T, float(lam), float(beta),

@@ -32,6 +32,12 @@
 //                       re-ranks the candidates the acoustic model proposes):
 //                       the argmax runs over the acoustic model's k best
 //                       outputs only (blank included, ties to the lower id).
+//   * prediction network (the Transducer's stateful form, Fig. 1's
+//                       prediction + joint networks): a one-layer LSTM over the
+//                       previous label (blank = start of sequence) and joint
+//                       projections, joint input = bf16(ReLU(W_enc enc_t + b_enc
+//                       + W_pred h + b_pred)); the LSTM advances on every
+//                       emitted label.
 //   * beam search:      per frame, top-K of the K*(V+1) extensions, then
 //                       identical label sequences merged by log-sum-exp.
 //                       (Not in the paper; the beam workload defines it.)
@@ -162,10 +168,30 @@ struct Hyp {
   int32_t last(int32_t V) const { return y.empty() ? V : y.back(); }
 };
 
+// Prediction network weights (bf16 bit patterns, fp32 biases).
+struct PredNet {
+  int32_t V, D, Henc, H;
+  const uint16_t* Ep;  // [V+1][D] label embedding; row V starts a sequence
+  const uint16_t* Wg;  // [2D][4D]: rows x (embedding) then h; column 4u+q is gate q (i, f, g, o) of unit u
+  const float* bg;     // [4D]
+  const uint16_t* Wp;  // [D][H]
+  const float* bp;     // [H]
+  const uint16_t* We;  // [Henc][H]
+  const float* be;     // [H]
+};
+
+// LSTM state: h as the bf16 the next products read, c in double.
+struct PredState {
+  std::vector<uint16_t> h;
+  std::vector<double> c;
+  bool ready = false;
+};
+
 struct Stream {
   int32_t V = 0;
   Hyp greedy;
   std::vector<Hyp> beam;  // empty until the first beam chunk
+  PredState pred;
 };
 
 // After v was appended to h.y: restart matching if the longest matched
@@ -183,6 +209,61 @@ struct Model {
   const uint16_t* E;  // [V+1][H]
   const uint16_t* W;  // [H][V+1]
 };
+
+double sigmoid(double x) { return 1.0 / (1.0 + std::exp(-x)); }
+
+// One LSTM step on label y: gates = bg + x W_g[0:D] + h W_g[D:2D] with
+// x = Ep[y]; c' = s(f) c + s(i) tanh(g); h' = s(o) tanh(c'); h' is kept as
+// the bf16 (through fp32) the next products read.
+void lstm_step(const PredNet& p, int32_t y, PredState& st) {
+  const int32_t D = p.D;
+  if (!st.ready) {
+    st.h.assign((size_t)D, 0);
+    st.c.assign((size_t)D, 0.0);
+    st.ready = true;
+  }
+  std::vector<double> g((size_t)4 * D);
+  for (int32_t j = 0; j < 4 * D; ++j) g[(size_t)j] = (double)p.bg[j];
+  for (int32_t k = 0; k < D; ++k) {
+    const double xk = (double)bf16_bits_to_float(p.Ep[(size_t)y * D + k]);
+    const double hk = (double)bf16_bits_to_float(st.h[(size_t)k]);
+    const uint16_t* wx = p.Wg + (size_t)k * 4 * D;
+    const uint16_t* wh = p.Wg + (size_t)(D + k) * 4 * D;
+    for (int32_t j = 0; j < 4 * D; ++j)
+      g[(size_t)j] += xk * (double)bf16_bits_to_float(wx[j]) + hk * (double)bf16_bits_to_float(wh[j]);
+  }
+  for (int32_t u = 0; u < D; ++u) {
+    const double i = sigmoid(g[(size_t)4 * u]), f = sigmoid(g[(size_t)4 * u + 1]);
+    const double gg = std::tanh(g[(size_t)4 * u + 2]), o = sigmoid(g[(size_t)4 * u + 3]);
+    const double c = f * st.c[(size_t)u] + i * gg;
+    st.c[(size_t)u] = c;
+    st.h[(size_t)u] = float_to_bf16_bits((float)(o * std::tanh(c)));
+  }
+}
+
+// Joint input of the stateful form: bf16(ReLU(W_enc enc_t + b_enc + W_pred h + b_pred)),
+// the sum taken to fp32 before the rounding to bf16 (as the kernels store it).
+void pred_joint_input(const PredNet& p, const uint16_t* enc_t, const PredState& st, std::vector<float>& x) {
+  const int32_t H = p.H;
+  std::vector<double> a((size_t)H);
+  for (int32_t j = 0; j < H; ++j) a[(size_t)j] = (double)p.be[j] + (double)p.bp[j];
+  for (int32_t k = 0; k < p.Henc; ++k) {
+    const double ek = (double)bf16_bits_to_float(enc_t[k]);
+    const uint16_t* w = p.We + (size_t)k * H;
+    for (int32_t j = 0; j < H; ++j) a[(size_t)j] += ek * (double)bf16_bits_to_float(w[j]);
+  }
+  for (int32_t k = 0; k < p.D; ++k) {
+    const double hk = (double)bf16_bits_to_float(st.h[(size_t)k]);
+    const uint16_t* w = p.Wp + (size_t)k * H;
+    for (int32_t j = 0; j < H; ++j) a[(size_t)j] += hk * (double)bf16_bits_to_float(w[j]);
+  }
+  x.resize((size_t)H);
+  for (int32_t j = 0; j < H; ++j) {
+    float v = (float)a[(size_t)j];
+    if (v < 0.0f) v = 0.0f;
+    x[(size_t)j] = bf16_bits_to_float(float_to_bf16_bits(v));
+  }
+}
 
 // The LM term of Eq. 1: sum over the LMs of alpha_i * log p_LM_i(v | y),
 // summed in the LMs' order.
@@ -212,11 +293,11 @@ LmTerm one_lm(const void* lmp, double lambda) {
 // fused[V] = log_softmax(logits)[V]
 void fused_scores(const Model& m, const uint16_t* enc_t, const Hyp& h, const LmTerm& lms,
                   const PhraseSet* boost, double beta, std::vector<float>& x,
-                  std::vector<double>& logits, std::vector<double>& fused) {
+                  std::vector<double>& logits, std::vector<double>& fused, bool x_given = false) {
   const int32_t V = m.V, H = m.H, N = V + 1;
   const int32_t last = h.last(V);
-  x.resize((size_t)H);
-  for (int32_t k = 0; k < H; ++k) {
+  if (!x_given) x.resize((size_t)H);
+  for (int32_t k = 0; k < H && !x_given; ++k) {
     float s = bf16_bits_to_float(enc_t[k]) + bf16_bits_to_float(m.E[(size_t)last * H + k]);
     if (s < 0.0f) s = 0.0f;
     x[(size_t)k] = bf16_bits_to_float(float_to_bf16_bits(s));
@@ -428,7 +509,7 @@ int32_t decode_chunk_impl(Stream* s, const LmTerm& lm, const PhraseSet* boost, i
                           int32_t max_sym, const int32_t* follow_tok, const int32_t* follow_frame,
                           const float* follow_score, int32_t follow_count, double gap_tol, int32_t* out_tok,
                           int32_t* out_frame, double* out_score, int32_t out_cap, double* report,
-                          int32_t prune_k = 0, double am_tol = 0.0) {
+                          int32_t prune_k = 0, double am_tol = 0.0, const PredNet* pn = nullptr) {
   Model m{V, H, E, W};
   std::vector<float> x;
   std::vector<double> logits, fused;
@@ -437,7 +518,11 @@ int32_t decode_chunk_impl(Stream* s, const LmTerm& lm, const PhraseSet* boost, i
   Hyp& h = s->greedy;
   for (int32_t t = 0; t < T; ++t) {
     for (int32_t sym = 0; sym < max_sym;) {
-      fused_scores(m, enc + (size_t)t * H, h, lm, boost, beta, x, logits, fused);
+      if (pn) {
+        if (!s->pred.ready) lstm_step(*pn, V, s->pred);  // start of sequence
+        pred_joint_input(*pn, enc + (size_t)t * pn->Henc, s->pred, x);
+      }
+      fused_scores(m, pn ? nullptr : enc + (size_t)t * H, h, lm, boost, beta, x, logits, fused, pn != nullptr);
       std::vector<uint8_t> cand((size_t)V + 1, prune_k > 0 ? 0 : 1);
       double kth = -std::numeric_limits<double>::infinity();
       if (prune_k > 0) {
@@ -491,6 +576,7 @@ int32_t decode_chunk_impl(Stream* s, const LmTerm& lm, const PhraseSet* boost, i
       ++emitted;
       h.y.push_back(y);
       advance_rho(boost, h);
+      if (pn) lstm_step(*pn, y, s->pred);  // the prediction network reads the emitted label
       ++sym;
     }
   }
@@ -528,6 +614,35 @@ ORACLE_API int32_t oracle_decode_chunk_pruned(void* sp, const void* lmp, const v
   return decode_chunk_impl(static_cast<Stream*>(sp), one_lm(lmp, lambda), static_cast<const PhraseSet*>(boostp),
                            V, H, E, W, enc, T, beta, max_sym, follow_tok, follow_frame, follow_score, follow_count,
                            gap_tol, out_tok, out_frame, out_score, out_cap, report, prune_k, am_tol);
+}
+
+// The stateful form: joint input from the prediction network and the
+// joint projections (enc rows have Henc entries); see PredNet.
+ORACLE_API int32_t oracle_decode_chunk_pred(void* sp, const void* lmp, const void* boostp, int32_t V, int32_t H,
+                                            int32_t Henc, int32_t D, const uint16_t* Ep, const uint16_t* Wg,
+                                            const float* bg, const uint16_t* Wp, const float* bp,
+                                            const uint16_t* We, const float* be, const uint16_t* W,
+                                            const uint16_t* enc, int32_t T, double lambda, double beta,
+                                            int32_t max_sym, const int32_t* follow_tok, const int32_t* follow_frame,
+                                            const float* follow_score, int32_t follow_count, double gap_tol,
+                                            int32_t* out_tok, int32_t* out_frame, double* out_score,
+                                            int32_t out_cap, double* report) {
+  PredNet pn{V, D, Henc, H, Ep, Wg, bg, Wp, bp, We, be};
+  return decode_chunk_impl(static_cast<Stream*>(sp), one_lm(lmp, lambda), static_cast<const PhraseSet*>(boostp),
+                           V, H, nullptr, W, enc, T, beta, max_sym, follow_tok, follow_frame, follow_score,
+                           follow_count, gap_tol, out_tok, out_frame, out_score, out_cap, report, 0, 0.0, &pn);
+}
+
+// A stream's prediction-network state: h (bf16 bits) and c, D entries each;
+// returns 0 before the first step.
+ORACLE_API int32_t oracle_pred_state(const void* sp, uint16_t* h, double* c) {
+  const Stream* s = static_cast<const Stream*>(sp);
+  if (!s->pred.ready) return 0;
+  for (size_t u = 0; u < s->pred.h.size(); ++u) {
+    h[u] = s->pred.h[u];
+    c[u] = s->pred.c[u];
+  }
+  return 1;
 }
 
 // The same with several LMs (Eq. 1, term 2 summed over i): n_lm LMs with

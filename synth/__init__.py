@@ -38,6 +38,12 @@ _LIB_PATH = os.path.join(_HERE, "libsynth.so")
 TENSOR_ENC = 1
 TENSOR_EMB = 2
 TENSOR_WOUT = 3
+TENSOR_PRED_EMB = 4
+TENSOR_PRED_GATES = 5
+TENSOR_PRED_GBIAS = 6
+TENSOR_PRED_PROJ = 7
+TENSOR_ENC_PROJ = 8
+TENSOR_PROJ_BIAS = 9
 
 
 def build(force: bool = False) -> str:
@@ -255,3 +261,47 @@ def phrases_for(w: Workload) -> Optional[Phrases]:
     if w.n_phr <= 0:
         return None
     return phrases(w.boost_seed, w.V, w.n_phr, w.phr_len[0], w.phr_len[1], w.share)
+
+
+@dataclasses.dataclass
+class PredWeights:
+    """Prediction network and joint projections of the stateful Transducer
+    form (bf16 bit patterns, fp32 biases): a one-layer LSTM of width D over
+    the previous label, then joint input = ReLU(enc We + be + h Wp + bp)."""
+
+    D: int
+    Henc: int
+    Ep: np.ndarray  # [V+1, D] label embedding (row V starts a sequence)
+    Wg: np.ndarray  # [2D, 4D] gates; column 4u+q is gate q (i, f, g, o) of unit u; rows x then h
+    bg: np.ndarray  # [4D] float32
+    Wp: np.ndarray  # [D, H]
+    bp: np.ndarray  # [H] float32
+    We: np.ndarray  # [Henc, H]
+    be: np.ndarray  # [H] float32
+
+
+def pred_weights(w: Workload, D: int = 640, Henc: int = None) -> PredWeights:
+    """Seeded prediction-network weights: Ep ~ N(0, 1); Wg ~ N(0, 1/sqrt(2D));
+    gate biases ~ N(0, 0.1) plus 1 on the forget gates; Wp ~ N(0, 3/sqrt(D));
+    We ~ N(0, 1/sqrt(Henc)); projection biases ~ N(0, 0.1).  The joint input
+    then has about the spread of the stateless form's enc + E[last]."""
+    Henc = Henc or w.H
+    N, H = w.N, w.H
+    bf = lambda t, n, std: normal_bf16(w.seed, t, 0, 0, n, std)
+    Ep = bf(TENSOR_PRED_EMB, N * D, 1.0).reshape(N, D)
+    Wg = bf(TENSOR_PRED_GATES, 2 * D * 4 * D, 1.0 / math.sqrt(2 * D)).reshape(2 * D, 4 * D)
+    bg = bf16_to_f32(bf(TENSOR_PRED_GBIAS, 4 * D, 0.1)).copy()
+    bg[1::4] += 1.0
+    Wp = bf(TENSOR_PRED_PROJ, D * H, 3.0 / math.sqrt(D)).reshape(D, H)
+    We = bf(TENSOR_ENC_PROJ, Henc * H, 1.0 / math.sqrt(Henc)).reshape(Henc, H)
+    pb = bf16_to_f32(normal_bf16(w.seed, TENSOR_PROJ_BIAS, 0, 0, 2 * H, 0.1))
+    return PredWeights(D, Henc, Ep, Wg, bg.astype(np.float32), Wp, pb[:H].copy(), We, pb[H:].copy())
+
+
+def enc_chunk_wide(w: Workload, streams, chunk: int, Henc: int, T: Optional[int] = None) -> np.ndarray:
+    """Encoder frames of width Henc (the stateful form projects them to H)."""
+    T = w.T if T is None else T
+    out = np.empty((len(streams), T, Henc), dtype=np.uint16)
+    for i, s in enumerate(streams):
+        out[i] = normal_bf16(w.seed, TENSOR_ENC, int(s), chunk * T * Henc, T * Henc, 1.0).reshape(T, Henc)
+    return out

@@ -37,6 +37,12 @@ MUTATIONS = {
     "pruned set not ranked by the acoustic model": (
         "[&](int32_t a, int32_t b) { return logits[(size_t)a] > logits[(size_t)b]; });",
         "[&](int32_t a, int32_t b) { return fused_rank_bug(a, b); });"),
+    "LSTM input and forget gates swapped": (
+        "const double i = sigmoid(g[(size_t)4 * u]), f = sigmoid(g[(size_t)4 * u + 1]);",
+        "const double f = sigmoid(g[(size_t)4 * u]), i = sigmoid(g[(size_t)4 * u + 1]);"),
+    "prediction network advances on blank": (
+        "      rep[REP_STEPS] += 1;\n      if (y == V) break;",
+        "      rep[REP_STEPS] += 1;\n      if (y == V && pn) lstm_step(*pn, V, s->pred);\n      if (y == V) break;"),
     "failed match not cancelled": (
         "return bonus * (double)(match(gv.data(), len + 1) - match(g, len));",
         "return bonus * (double)std::max(0, match(gv.data(), len + 1) - match(g, len));"),
@@ -55,6 +61,7 @@ def test_pins_catch_planted_mistake(name, tmp_path):
                            str(so)])
     r = subprocess.run([sys.executable, "-m", "pytest", os.path.join(ROOT, "tests", "test_oracle_pins.py"),
                         os.path.join(ROOT, "tests", "test_oracle_multilm.py"),
-                        os.path.join(ROOT, "tests", "test_oracle_pruned.py"), "-q", "-x", "-p", "no:cacheprovider"], cwd=ROOT, capture_output=True, text=True,
+                        os.path.join(ROOT, "tests", "test_oracle_pruned.py"),
+                        os.path.join(ROOT, "tests", "test_oracle_pred.py"), "-q", "-x", "-p", "no:cacheprovider"], cwd=ROOT, capture_output=True, text=True,
                        env=dict(os.environ, TSD_ORACLE_LIB=str(so)), timeout=600)
     assert r.returncode != 0, f"pins did not catch: {name}\n{r.stdout[-2000:]}"
