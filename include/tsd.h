@@ -195,6 +195,36 @@ TSD_API tsd_status tsd_decoder_create(const tsd_decoder_cfg* cfg, const void* W_
                               const void* E_bf16, const tsd_ngram* lm, const tsd_boost* boost,
                               void* cuda_stream, tsd_decoder** out);
 
+/* The stateful Transducer form: the joint input is
+ *   bf16(ReLU(W_enc enc_t + b_enc + W_pred h + b_pred))
+ * where h is the output of a one-layer LSTM prediction network over the
+ * previous label (Fig. 1: prediction and joint networks): on every emitted
+ * label y it reads x = emb[y] (emb[V] starts a sequence) and updates
+ *   gates = b_gates + (x, h) W_gates,   c' = s(f) c + s(i) tanh(g),
+ *   h' = s(o) tanh(c')   (h kept as bf16, c as fp32).
+ * Encoder frames passed to decode_chunk are then H_enc wide.  All weights
+ * are device arrays, copied (and repacked) at create. */
+typedef struct {
+  int32_t D;             /* LSTM width: multiple of 64, 64 <= D <= 2048 */
+  int32_t H_enc;         /* encoder frame width: multiple of 64, 64 <= H_enc <= 8192 */
+  const void* emb;       /* bf16 [V+1][D] */
+  const void* W_gates;   /* bf16 [2D][4D]: rows (x, then h); column 4u+q is gate q (i, f, g, o) of unit u */
+  const float* b_gates;  /* fp32 [4D] */
+  const void* W_pred;    /* bf16 [D][H] */
+  const float* b_pred;   /* fp32 [H] */
+  const void* W_enc;     /* bf16 [H_enc][H] */
+  const float* b_enc;    /* fp32 [H] */
+} tsd_pred_weights;
+
+/* A decoder of the stateful form (greedy; prune_k 0; one LM or none).  E is
+ * not used.  Stream export/import is not available for it. */
+TSD_API tsd_status tsd_decoder_create_pred(const tsd_decoder_cfg* cfg, const tsd_pred_weights* pred,
+                                           const void* W_out_bf16, const tsd_ngram* lm, const tsd_boost* boost,
+                                           void* cuda_stream, tsd_decoder** out);
+/* A stateful-form stream's prediction-network state: h (bf16 bits) and c,
+ * D entries each (synchronizes). */
+TSD_API tsd_status tsd_stream_pred_state(tsd_decoder* dec, int32_t slot, uint16_t* h, float* c);
+
 /* The same with several n-gram LMs fused at once (Eq. 1, the sum over LMs
  * i of alpha_i log p_LM_i): LM i (host handle lms[i], same V, outliving the
  * decoder) enters with alpha_i = lambda * lm_weights[i], lambda being

@@ -34,6 +34,11 @@ _vp, _i32, _i64, _f32 = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.
 _P = ctypes.POINTER
 
 
+class PredWeightsC(ctypes.Structure):
+    _fields_ = [("D", _i32), ("H_enc", _i32), ("emb", _vp), ("W_gates", _vp), ("b_gates", _vp), ("W_pred", _vp),
+                ("b_pred", _vp), ("W_enc", _vp), ("b_enc", _vp)]
+
+
 class DecoderCfg(ctypes.Structure):
     _fields_ = [("V", _i32), ("H", _i32), ("max_symbols", _i32), ("beam_k", _i32), ("max_streams", _i32),
                 ("max_T", _i32), ("prune_k", _i32)]
@@ -53,6 +58,8 @@ SIGNATURES = {
     "tsd_decoder_create": ([_P(DecoderCfg), _vp, _vp, _vp, _vp, _vp, _P(_vp)], _i32),
     "tsd_decoder_create_multi": ([_P(DecoderCfg), _vp, _vp, _vp, _vp, _i32, _vp, _vp, _P(_vp)], _i32),
     "tsd_stream_lm_state": ([_vp, _i32, _i32, _P(_i32)], _i32),
+    "tsd_decoder_create_pred": ([_P(DecoderCfg), _P(PredWeightsC), _vp, _vp, _vp, _vp, _P(_vp)], _i32),
+    "tsd_stream_pred_state": ([_vp, _i32, _vp, _vp], _i32),
     "tsd_stream_export": ([_vp, _i32, _vp, _i64, _P(_i64)], _i32),
     "tsd_stream_import": ([_vp, _i32, _vp, _i64], _i32),
     "tsd_decoder_free": ([_vp], None),
@@ -238,10 +245,13 @@ class Decoder:
 
     def __init__(self, V: int, H: int, W_out, E, lm: Optional[NGram] = None, boost: Optional[Boost] = None,
                  max_symbols: int = 5, beam_k: int = 1, max_streams: int = 64, max_T: int = 64, stream=None,
-                 lms: Optional[Sequence[Tuple[NGram, float]]] = None, prune_k: int = 0):
+                 lms: Optional[Sequence[Tuple[NGram, float]]] = None, prune_k: int = 0, pred=None):
         """lms: several LMs as (NGram, w) pairs instead of lm (LM i enters Eq. 1
         with weight lambda * w; ``tsd_decoder_create_multi``).  prune_k > 0:
-        pruned fusion over the acoustic model's prune_k best outputs."""
+        pruned fusion over the acoustic model's prune_k best outputs.  pred:
+        the stateful form's weights (fields D, Henc, Ep, Wg, bg, Wp, bp, We, be
+        as numpy arrays, bf16 bit patterns and fp32 biases;
+        ``tsd_decoder_create_pred``); E is then ignored."""
         import torch
 
         assert W_out.is_cuda and E.is_cuda and W_out.element_size() == 2 and E.element_size() == 2
@@ -252,7 +262,21 @@ class Decoder:
         W_out = W_out.contiguous()
         E = E.contiguous()
         h = _vp()
-        if lms is not None:
+        if pred is not None:
+            dev = W_out.device
+            up16 = lambda a: torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).to(dev)
+            up32 = lambda a: torch.from_numpy(np.ascontiguousarray(a, dtype=np.float32)).to(dev)
+            t = dict(emb=up16(pred.Ep), Wg=up16(pred.Wg), bg=up32(pred.bg), Wp=up16(pred.Wp), bp=up32(pred.bp),
+                     We=up16(pred.We), be=up32(pred.be))
+            self._pred_keep = t
+            self.pred_D = pred.D
+            self.pred_Henc = pred.Henc
+            pw = PredWeightsC(pred.D, pred.Henc, _ptr(t["emb"]), _ptr(t["Wg"]), _ptr(t["bg"]), _ptr(t["Wp"]),
+                              _ptr(t["bp"]), _ptr(t["We"]), _ptr(t["be"]))
+            _check(lib().tsd_decoder_create_pred(ctypes.byref(self.cfg), ctypes.byref(pw), _ptr(W_out),
+                                                 lm.h if lm else None, boost.h if boost else None, _stream(stream),
+                                                 ctypes.byref(h)))
+        elif lms is not None:
             assert lm is None, "give lm or lms, not both"
             self.lm = [m for m, _ in lms]
             hs = (_vp * max(1, len(lms)))(*[m.h for m, _ in lms])
@@ -293,7 +317,7 @@ class Decoder:
                      stream=None) -> ChunkOut:
         """enc: cuda bf16 (or int16/uint16 bit patterns) [n, T, H]."""
         n, T, H = enc.shape
-        assert n == len(slots) and H == self.H and enc.is_cuda and enc.is_contiguous()
+        assert n == len(slots) and H == getattr(self, "pred_Henc", self.H) and enc.is_cuda and enc.is_contiguous()
         if out is None:
             out = self.alloc_out(n, T)
         sl = _i32arr(slots)
@@ -326,6 +350,13 @@ class Decoder:
         """Continues an exported stream in an open slot (``tsd_stream_import``)."""
         buf = ctypes.create_string_buffer(bytes(blob), len(blob))
         _check(lib().tsd_stream_import(self.h, int(slot), buf, len(blob)))
+
+    def pred_state(self, slot: int):
+        """(h as bf16 bits [D], c [D]) of a stateful-form stream."""
+        h = np.zeros(self.pred_D, dtype=np.uint16)
+        c = np.zeros(self.pred_D, dtype=np.float32)
+        _check(lib().tsd_stream_pred_state(self.h, int(slot), h.ctypes.data, c.ctypes.data))
+        return h, c
 
     def lm_state(self, slot: int, lm_index: int) -> int:
         """State id of LM lm_index for a slot (``tsd_stream_lm_state``)."""

@@ -15,6 +15,7 @@
 #include <type_traits>
 
 #include "decoder.h"
+#include "gemm_tc.h"
 #include "joint_tc.h"
 
 using namespace tsd;
@@ -46,6 +47,13 @@ void enqueue_chunk(tsd_decoder* d, int M, int T, cudaStream_t s, const std::vect
   auto mark = [&]() {
     if (ev) cudaEventRecordWithFlags((*ev)[(size_t)e++], s, cudaEventRecordExternal);
   };
+  const tsd_decoder::Pred& pr = d->pred;
+  if (pr.D) {
+    // the chunk's encoder frames to a fixed buffer, then their projection
+    launch_copy_enc(v, (int64_t)M * T * pr.Henc, s, false);
+    GemmArgs ge{M * T, d->cfg.H, pr.Henc, d->cfg.H, pr.be, v.pred_penc};
+    launch_gemm_tc(kEncProj, v, ge, pr.encA, pr.encB, pr.H_pad, s, d->pdl && !ev);
+  }
   launch_defaults(v, s);
   for (int step = 0; step <= S; ++step) {
     const bool pdl = d->pdl && !ev && step > 0;  // the first launch follows the parameter copy
@@ -53,6 +61,16 @@ void enqueue_chunk(tsd_decoder* d, int M, int T, cudaStream_t s, const std::vect
     if (d->cfg.beam_k > 1) launch_row_beam(v, M / d->cfg.beam_k, step, step == S ? 1 : 0, d->row_smem, s, pdl);
     else if (d->cfg.prune_k > 0) launch_row_pruned(v, M, step, step == S ? 1 : 0, s, pdl);
     else launch_row(v, M, step, step == S ? 1 : 0, d->row_smem, s, pdl);
+    if (pr.D) {
+      // the prediction network reads the labels just emitted; after the last
+      // decision of the chunk only its state matters
+      GemmArgs gl{M, 4 * pr.D, 2 * pr.D, 0, pr.bg, nullptr};
+      launch_gemm_tc(kLstm, v, gl, pr.lstmA, pr.lstmB, pr.G_pad, s, d->pdl && !ev);
+      if (step < S) {
+        GemmArgs gp{M, d->cfg.H, pr.D, d->cfg.H, pr.bp, nullptr};
+        launch_gemm_tc(kJointIn, v, gp, pr.projA, pr.projB, pr.H_pad, s, d->pdl && !ev);
+      }
+    }
     if (step < S) {
       mark();
       if (d->joint_kind == 0) launch_joint_tc(*d->jtc, v, M, step, s, d->pdl && !ev);
@@ -88,10 +106,20 @@ void destroy_set(tsd_decoder::EventSet& es) {
 namespace {
 tsd_status create_impl(const tsd_decoder_cfg* cfg, const void* W_out_bf16, const void* E_bf16,
                        const tsd_ngram* const* lms, const float* lm_weights, int32_t n_lms, const tsd_boost* boost,
-                       void* cuda_stream, tsd_decoder** out) {
+                       void* cuda_stream, tsd_decoder** out, const tsd_pred_weights* pw = nullptr) {
   if (!out) return fail(TSD_EINVAL, "tsd_decoder_create: out is NULL");
   *out = nullptr;
-  if (!cfg || !W_out_bf16 || !E_bf16) return fail(TSD_EINVAL, "tsd_decoder_create: NULL argument");
+  if (!cfg || !W_out_bf16 || (!E_bf16 && !pw)) return fail(TSD_EINVAL, "tsd_decoder_create: NULL argument");
+  if (pw) {
+    if (pw->D < 64 || pw->D > 2048 || pw->D % 64)
+      return fail(TSD_EINVAL, "tsd_decoder_create_pred: D=%d must be a multiple of 64 in [64, 2048]", pw->D);
+    if (pw->H_enc < 64 || pw->H_enc > 8192 || pw->H_enc % 64)
+      return fail(TSD_EINVAL, "tsd_decoder_create_pred: H_enc=%d must be a multiple of 64 in [64, 8192]", pw->H_enc);
+    if (!pw->emb || !pw->W_gates || !pw->b_gates || !pw->W_pred || !pw->b_pred || !pw->W_enc || !pw->b_enc)
+      return fail(TSD_EINVAL, "tsd_decoder_create_pred: NULL weight");
+    if (cfg->beam_k != 1 || cfg->prune_k != 0)
+      return fail(TSD_EINVAL, "tsd_decoder_create_pred: greedy decoding without pruning only");
+  }
   const tsd_decoder_cfg c = *cfg;
   if (n_lms < 0 || n_lms > kMaxLm) return fail(TSD_EINVAL, "tsd_decoder_create: %d LMs, at most %d", n_lms, kMaxLm);
   if (n_lms > 0 && !lms) return fail(TSD_EINVAL, "tsd_decoder_create: NULL LM list");
@@ -188,6 +216,29 @@ tsd_status create_impl(const tsd_decoder_cfg* cfg, const void* W_out_bf16, const
       return fail(TSD_ENOMEM, "tsd_decoder_create: beam state not allocated");
     }
   }
+  // stateful form: weights (repacked K-major), state and step buffers
+  uint16_t *p_emb = nullptr, *p_h = nullptr, *p_x = nullptr, *p_hin = nullptr, *p_enc = nullptr;
+  float *p_c = nullptr, *p_penc = nullptr;
+  int32_t *p_fresh = nullptr, *p_flag = nullptr;
+  if (pw) {
+    tsd_decoder::Pred& pr = d->pred;
+    pr.D = pw->D;
+    pr.Henc = pw->H_enc;
+    pr.G_pad = round_up(4 * pw->D, 128);
+    pr.H_pad = round_up(c.H, 128);
+    pr.MT_pad = round_up(c.max_streams * c.max_T, 128);
+    const size_t D = (size_t)pw->D;
+    if ((st = A.alloc(&p_emb, (size_t)d->N * D)) || (st = A.alloc(&pr.Wg, (size_t)pr.G_pad * 2 * D)) ||
+        (st = A.alloc(&pr.bg, 4 * D)) || (st = A.alloc(&pr.Wp, (size_t)pr.H_pad * D)) ||
+        (st = A.alloc(&pr.bp, (size_t)c.H)) || (st = A.alloc(&pr.We, (size_t)pr.H_pad * pr.Henc)) ||
+        (st = A.alloc(&pr.be, (size_t)c.H)) || (st = A.alloc(&p_h, SK * D)) || (st = A.alloc(&p_c, SK * D)) ||
+        (st = A.alloc(&p_fresh, SK)) || (st = A.alloc(&p_x, (size_t)d->M_pad * 2 * D)) ||
+        (st = A.alloc(&p_hin, (size_t)d->M_pad * D)) || (st = A.alloc(&p_flag, (size_t)d->M_pad)) ||
+        (st = A.alloc(&p_enc, (size_t)pr.MT_pad * pr.Henc)) || (st = A.alloc(&p_penc, (size_t)pr.MT_pad * c.H))) {
+      A.release();
+      return st;
+    }
+  }
   auto cleanup = [&](tsd_status e) {
     delete d->jtc;
     d->jtc = nullptr;
@@ -206,10 +257,37 @@ tsd_status create_impl(const tsd_decoder_cfg* cfg, const void* W_out_bf16, const
       (ce = cudaMemsetAsync(stl, 0, sizeof(int32_t) * SK, s)) != cudaSuccess ||
       (ce = cudaMemsetAsync(err, 0, sizeof(int32_t), s)) != cudaSuccess ||
       (ce = cudaMemsetAsync(ctr, 0, 2 * sizeof(unsigned long long), s)) != cudaSuccess ||
-      (ce = cudaMemcpyAsync(E, E_bf16, sizeof(uint16_t) * (size_t)d->N * c.H, cudaMemcpyDeviceToDevice, s)) != cudaSuccess)
+      (ce = E_bf16 ? cudaMemcpyAsync(E, E_bf16, sizeof(uint16_t) * (size_t)d->N * c.H, cudaMemcpyDeviceToDevice, s)
+                   : cudaMemsetAsync(E, 0, sizeof(uint16_t) * (size_t)d->N * c.H, s)) != cudaSuccess)
     return cleanup(cuda_fail(ce, "tsd_decoder_create: initial copies"));
   launch_repack(static_cast<const uint16_t*>(W_out_bf16), Wt, c.H, d->N, d->N_pad, s);
   if ((ce = cudaGetLastError()) != cudaSuccess) return cleanup(cuda_fail(ce, "tsd_decoder_create: repack"));
+  if (pw) {
+    tsd_decoder::Pred& pr = d->pred;
+    const size_t D = (size_t)pr.D;
+    if ((ce = cudaMemcpyAsync(p_emb, pw->emb, 2 * (size_t)d->N * D, cudaMemcpyDeviceToDevice, s)) != cudaSuccess ||
+        (ce = cudaMemcpyAsync(pr.bg, pw->b_gates, 16 * D, cudaMemcpyDeviceToDevice, s)) != cudaSuccess ||
+        (ce = cudaMemcpyAsync(pr.bp, pw->b_pred, 4 * (size_t)c.H, cudaMemcpyDeviceToDevice, s)) != cudaSuccess ||
+        (ce = cudaMemcpyAsync(pr.be, pw->b_enc, 4 * (size_t)c.H, cudaMemcpyDeviceToDevice, s)) != cudaSuccess ||
+        (ce = cudaMemsetAsync(p_h, 0, 2 * SK * D, s)) != cudaSuccess ||
+        (ce = cudaMemsetAsync(p_c, 0, 4 * SK * D, s)) != cudaSuccess ||
+        (ce = cudaMemsetAsync(p_fresh, 0, 4 * SK, s)) != cudaSuccess ||
+        (ce = cudaMemsetAsync(p_flag, 0, 4 * (size_t)d->M_pad, s)) != cudaSuccess ||
+        (ce = cudaMemsetAsync(p_x, 0, 4 * (size_t)d->M_pad * D, s)) != cudaSuccess ||
+        (ce = cudaMemsetAsync(p_hin, 0, 2 * (size_t)d->M_pad * D, s)) != cudaSuccess ||
+        (ce = cudaMemsetAsync(p_enc, 0, 2 * (size_t)pr.MT_pad * pr.Henc, s)) != cudaSuccess)
+      return cleanup(cuda_fail(ce, "tsd_decoder_create_pred: weights"));
+    // K-major copies of the three weight matrices (rows past N are zero)
+    launch_repack(static_cast<const uint16_t*>(pw->W_gates), pr.Wg, 2 * pr.D, 4 * pr.D, pr.G_pad, s);
+    launch_repack(static_cast<const uint16_t*>(pw->W_pred), pr.Wp, pr.D, c.H, pr.H_pad, s);
+    launch_repack(static_cast<const uint16_t*>(pw->W_enc), pr.We, pr.Henc, c.H, pr.H_pad, s);
+    if ((ce = cudaGetLastError()) != cudaSuccess) return cleanup(cuda_fail(ce, "tsd_decoder_create_pred: repack"));
+    if (!gemm_tc_map_a(&pr.encA, p_enc, pr.MT_pad, pr.Henc) || !gemm_tc_map_b(&pr.encB, pr.We, pr.H_pad, pr.Henc) ||
+        !gemm_tc_map_a(&pr.lstmA, p_x, d->M_pad, 2 * pr.D) || !gemm_tc_map_b(&pr.lstmB, pr.Wg, pr.G_pad, 2 * pr.D) ||
+        !gemm_tc_map_a(&pr.projA, p_hin, d->M_pad, pr.D) || !gemm_tc_map_b(&pr.projB, pr.Wp, pr.H_pad, pr.D))
+      return cleanup(fail(TSD_ECUDA, "tsd_decoder_create_pred: TMA descriptors"));
+    if ((ce = gemm_tc_prepare()) != cudaSuccess) return cleanup(cuda_fail(ce, "tsd_decoder_create_pred: kernel attributes"));
+  }
   if ((ce = prepare_kernels(d->row_smem)) != cudaSuccess) return cleanup(cuda_fail(ce, "tsd_decoder_create: kernel attributes"));
   if ((ce = prepare_beam_kernels(d->row_smem)) != cudaSuccess) return cleanup(cuda_fail(ce, "tsd_decoder_create: kernel attributes"));
   if (hlive && (ce = cudaMemsetAsync(hlive, 0, sizeof(int32_t) * SK, s)) != cudaSuccess)
@@ -262,6 +340,16 @@ tsd_status create_impl(const tsd_decoder_cfg* cfg, const void* W_out_bf16, const
   v.s_tr_chain = stc;
   v.s_lm_rec = slr;
   v.s_tr_rec = strc;
+  v.pred_D = pw ? pw->D : 0;
+  v.pred_emb = p_emb;
+  v.pred_h = p_h;
+  v.pred_c = p_c;
+  v.pred_fresh = p_fresh;
+  v.pred_x = p_x;
+  v.pred_hin = p_hin;
+  v.pflag = p_flag;
+  v.pred_enc = p_enc;
+  v.pred_penc = p_penc;
   v.has_lm = lm ? 1 : 0;
   v.has_tr = boost ? 1 : 0;
   if (lm) v.lm = lm->view;
@@ -306,6 +394,30 @@ extern "C" tsd_status tsd_decoder_create(const tsd_decoder_cfg* cfg, const void*
   return create_impl(cfg, W_out_bf16, E_bf16, one, nullptr, lm ? 1 : 0, boost, cuda_stream, out);
 }
 
+extern "C" tsd_status tsd_decoder_create_pred(const tsd_decoder_cfg* cfg, const tsd_pred_weights* pred,
+                                              const void* W_out_bf16, const tsd_ngram* lm, const tsd_boost* boost,
+                                              void* cuda_stream, tsd_decoder** out) {
+  clear_error();
+  if (!pred) return fail(TSD_EINVAL, "tsd_decoder_create_pred: NULL weights");
+  const tsd_ngram* one[1] = {lm};
+  return create_impl(cfg, W_out_bf16, nullptr, one, nullptr, lm ? 1 : 0, boost, cuda_stream, out, pred);
+}
+
+extern "C" tsd_status tsd_stream_pred_state(tsd_decoder* d, int32_t slot, uint16_t* h, float* c) {
+  clear_error();
+  if (!d || !h || !c) return fail(TSD_EINVAL, "tsd_stream_pred_state: NULL argument");
+  if (!d->pred.D) return fail(TSD_EINVAL, "tsd_stream_pred_state: not a stateful-form decoder");
+  if (slot < 0 || slot >= d->cfg.max_streams || !d->slot_open[(size_t)slot])
+    return fail(TSD_ESTATE, "tsd_stream_pred_state: slot %d is not open", slot);
+  tsd_status st = set_device(d);
+  if (st) return st;
+  TSD_CUDA(cudaStreamSynchronize(d->last_stream));
+  const size_t D = (size_t)d->pred.D;
+  TSD_CUDA(cudaMemcpy(h, d->view.pred_h + (size_t)slot * D, 2 * D, cudaMemcpyDeviceToHost));
+  TSD_CUDA(cudaMemcpy(c, d->view.pred_c + (size_t)slot * D, 4 * D, cudaMemcpyDeviceToHost));
+  return TSD_OK;
+}
+
 extern "C" tsd_status tsd_decoder_create_multi(const tsd_decoder_cfg* cfg, const void* W_out_bf16,
                                                const void* E_bf16, const tsd_ngram* const* lms,
                                                const float* lm_weights, int32_t n_lms, const tsd_boost* boost,
@@ -345,6 +457,7 @@ extern "C" tsd_status tsd_stream_open(tsd_decoder* d, int32_t* slot_out) {
     return fail(TSD_ESTATE, "tsd_stream_open: beam state missing");
   if (d->cfg.beam_k > 1) launch_open_beam(d->view, slot, d->last_stream);
   else launch_open(d->view, slot, d->last_stream);
+  if (d->pred.D) launch_open_pred(d->view, slot, d->last_stream);
   TSD_CUDA(cudaGetLastError());
   *it = 1;
   *slot_out = slot;
@@ -516,6 +629,7 @@ tsd_status copy_dev(T* dst, const T* src, size_t n, cudaMemcpyKind kind) {
 extern "C" tsd_status tsd_stream_export(tsd_decoder* d, int32_t slot, void* buf, int64_t cap, int64_t* len) {
   clear_error();
   if (!d || !len) return fail(TSD_EINVAL, "tsd_stream_export: NULL argument");
+  if (d->pred.D) return fail(TSD_EINVAL, "tsd_stream_export: not available for the stateful form");
   if (slot < 0 || slot >= d->cfg.max_streams || !d->slot_open[(size_t)slot])
     return fail(TSD_ESTATE, "tsd_stream_export: slot %d is not open", slot);
   tsd_status st = set_device(d);
@@ -561,6 +675,7 @@ extern "C" tsd_status tsd_stream_export(tsd_decoder* d, int32_t slot, void* buf,
 extern "C" tsd_status tsd_stream_import(tsd_decoder* d, int32_t slot, const void* buf, int64_t len) {
   clear_error();
   if (!d || !buf) return fail(TSD_EINVAL, "tsd_stream_import: NULL argument");
+  if (d->pred.D) return fail(TSD_EINVAL, "tsd_stream_import: not available for the stateful form");
   if (slot < 0 || slot >= d->cfg.max_streams || !d->slot_open[(size_t)slot])
     return fail(TSD_ESTATE, "tsd_stream_import: slot %d is not open", slot);
   if (len < (int64_t)sizeof(BlobHeader)) return fail(TSD_EINVAL, "tsd_stream_import: blob too short");
@@ -797,7 +912,8 @@ extern "C" tsd_status tsd_decoder_launches_per_chunk(const tsd_decoder* d, int32
   clear_error();
   if (!d || !launches) return fail(TSD_EINVAL, "tsd_decoder_launches_per_chunk: NULL argument");
   (void)n;
-  *launches = 2 * (int64_t)steps_per_chunk(d, T) + 2;
+  const int64_t S = steps_per_chunk(d, T);
+  *launches = d->pred.D ? 4 * S + 4 : 2 * S + 2;  // stateful form: + copy, projection, LSTM and joint input
   return TSD_OK;
 }
 

@@ -1,6 +1,7 @@
 // Decoder internals shared by the host driver and the kernels.
 #pragma once
 
+#include <cuda.h>
 #include <cuda_bf16.h>
 
 #include <map>
@@ -46,6 +47,17 @@ struct DecView {
   // the next step's searches start without fetching them:
   int4* s_lm_rec;       // [slots][kLmChain] first LM: (first arc, arcs, cumulative backoff bits, 0)
   int4* s_tr_rec;       // [slots][kTrChain] trie: (first child, children, depth of the children, 0)
+  // stateful form (pred_D > 0): prediction network state and its buffers
+  int32_t pred_D;       // LSTM width (0: the stateless joint input enc + E[last])
+  uint16_t* pred_emb;   // [V+1][D] label embedding
+  uint16_t* pred_h;     // [slots][D] LSTM output (bf16, as the products read it)
+  float* pred_c;        // [slots][D] LSTM cell
+  int32_t* pred_fresh;  // [slots] 1 until the start-of-sequence step has run
+  uint16_t* pred_x;     // [M_pad][2D] LSTM input of the step: (embedding of the label, h)
+  uint16_t* pred_hin;   // [M_pad][D] h after the step, input of the projection
+  int32_t* pflag;       // [M_pad] 1 if the row's LSTM steps (a label was emitted, or the sequence starts)
+  uint16_t* pred_enc;   // [rows][Henc] the chunk's encoder frames (a fixed address for TMA)
+  float* pred_penc;     // [rows][H] W_enc enc + b_enc of the chunk
   LmView lm;
   TrieView tr;
   int32_t has_lm, has_tr;
@@ -81,6 +93,8 @@ constexpr int kRowThreads = 256;
 void launch_repack(const uint16_t* W, uint16_t* Wt, int H, int N, int N_pad, cudaStream_t s);
 void launch_open(const DecView& d, int slot, cudaStream_t s);
 void launch_fix_records(const DecView& d, int slot, cudaStream_t s);
+void launch_open_pred(const DecView& d, int slot, cudaStream_t s);
+void launch_copy_enc(const DecView& d, int64_t elems, cudaStream_t s, bool pdl);
 void launch_row(const DecView& d, int M, int step, int mode, size_t smem, cudaStream_t s, bool pdl);
 void launch_joint(const DecView& d, int M, int step, cudaStream_t s);
 void launch_defaults(const DecView& d, cudaStream_t s);
@@ -126,6 +140,13 @@ struct tsd_decoder {
   };
   std::map<std::tuple<int, int, int, int>, Entry> entries;  // (n, T, graphs, timing)
   tsd::JointTc* jtc = nullptr;  // tensor-core joint kernel state
+  // stateful form: repacked weights (K-major), biases and the GEMMs' TMA maps
+  struct Pred {
+    int D = 0, Henc = 0, G_pad = 0, H_pad = 0, MT_pad = 0;
+    uint16_t *Wg = nullptr, *Wp = nullptr, *We = nullptr;
+    float *bg = nullptr, *bp = nullptr, *be = nullptr;
+    CUtensorMap encA, encB, lstmA, lstmB, projA, projB;
+  } pred;
   int joint_kind = 0;           // 0 tensor cores, 1 CUDA cores
   int pdl = 1;                  // programmatic dependent launch between kernels
   int sms = 0;

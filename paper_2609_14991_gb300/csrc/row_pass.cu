@@ -14,6 +14,8 @@
 // LM state per order; every trie node that is a suffix of the current one),
 // so the next chain after label y is assembled from independent searches of
 // y in each chain element -- no dependent pointer chase.
+#include <algorithm>
+
 #include "row_common.cuh"
 
 namespace tsd {
@@ -372,6 +374,25 @@ __global__ void __launch_bounds__(kRowThreads, 7) k_row(DecView d, int step, int
     row::block_sync();
   }
 
+  if (d.pred_D) {
+    // Stateful form: the prediction network reads the label just emitted
+    // (or, at a stream's first step, the start of sequence) and the row's h
+    // from before this step; the LSTM kernel after this one runs the cell.
+    const bool fresh = step == 0 && __ldcg(d.pred_fresh + slot) != 0;
+    const bool stepped = fresh || (evaluated && s_y != V);
+    if (tid == 0) {
+      d.pflag[r] = stepped ? 1 : 0;
+      if (fresh && commit) d.pred_fresh[slot] = 0;
+    }
+    if (stepped) {
+      const int D = d.pred_D;
+      const int lab = fresh ? V : s_y;
+      const uint4* src_x = reinterpret_cast<const uint4*>(d.pred_emb + (size_t)lab * D);
+      const uint4* src_h = reinterpret_cast<const uint4*>(d.pred_h + (size_t)slot * D);
+      uint4* dst = reinterpret_cast<uint4*>(d.pred_x + (size_t)r * 2 * D);
+      for (int i = tid; i < D / 4; i += blockDim.x) dst[i] = (i < D / 8) ? __ldg(src_x + i) : __ldcg(src_h + i - D / 8);
+    }
+  }
   if (mode == 1) {
     // the chunk's last decision: the new chains' records for the next chunk
     if (L == 1 && commit) {
@@ -421,11 +442,11 @@ __global__ void __launch_bounds__(kRowThreads, 7) k_row(DecView d, int step, int
       if (tid >= 32 && tid - 32 < nt)
         d.s_tr_rec[(size_t)slot * kTrChain + tid - 32] = make_int4(rc.tb[tid - 32], rc.tc[tid - 32], rc.td[tid - 32], 0);
     }
-    row::build_joint_input(d, s_enc + ((size_t)r * T + t) * d.H, s_last, r);
+    if (!d.pred_D) row::build_joint_input(d, s_enc + ((size_t)r * T + t) * d.H, s_last, r);
     row::bias_finish(d, nl, nt, rc, s_lam, s_beta, d.bias + (size_t)r * d.N_pad, lmv, dep);
     if (counting && tid == 0) lm_bytes = lm_level_bytes(rc, nl, s_y != V && evaluated);
   } else {
-    row::build_joint_input(d, s_enc + ((size_t)r * T + t) * d.H, s_last, r);
+    if (!d.pred_D) row::build_joint_input(d, s_enc + ((size_t)r * T + t) * d.H, s_last, r);
     lm_bytes = bias_multi(d, L, s_lm, s_lm_len, s_tr, nt, rc, s_lam, s_beta, d.bias + (size_t)r * d.N_pad, lmv,
                           acc, dep, counting, s_y != V && evaluated);
     nl = 0;
@@ -528,6 +549,45 @@ void launch_repack(const uint16_t* W, uint16_t* Wt, int H, int N, int N_pad, cud
 void launch_open(const DecView& d, int slot, cudaStream_t s) { k_open<<<1, 32, 0, s>>>(d, slot); }
 
 void launch_fix_records(const DecView& d, int slot, cudaStream_t s) { k_fix_records<<<1, 32, 0, s>>>(d, slot); }
+
+namespace {
+// Stateful form, stream open: zero LSTM state, the start-of-sequence step pending.
+__global__ void k_open_pred(DecView d, int slot) {
+  const int D = d.pred_D;
+  for (int u = threadIdx.x; u < D; u += blockDim.x) {
+    d.pred_h[(size_t)slot * D + u] = 0;
+    d.pred_c[(size_t)slot * D + u] = 0.f;
+  }
+  if (threadIdx.x == 0) d.pred_fresh[slot] = 1;
+}
+
+// Stateful form: the chunk's encoder frames (from the call's parameter
+// block) to the fixed buffer the projection GEMM reads by TMA.
+__global__ void k_copy_enc(DecView d, int64_t n16) {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  const uint4* src = reinterpret_cast<const uint4*>(d.params->enc);
+  uint4* dst = reinterpret_cast<uint4*>(d.pred_enc);
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n16; i += (int64_t)gridDim.x * blockDim.x)
+    dst[i] = __ldg(src + i);
+}
+}  // namespace
+
+void launch_open_pred(const DecView& d, int slot, cudaStream_t s) { k_open_pred<<<1, 256, 0, s>>>(d, slot); }
+
+void launch_copy_enc(const DecView& d, int64_t elems, cudaStream_t s, bool pdl) {
+  const int64_t n16 = elems / 8;  // H_enc is a multiple of 64
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)std::min<int64_t>((n16 + 255) / 256, 152 * 8));
+  cfg.blockDim = dim3(256);
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl ? 1 : 0;
+  cudaLaunchKernelEx(&cfg, k_copy_enc, d, n16);
+}
 
 void launch_row(const DecView& d, int M, int step, int mode, size_t smem, cudaStream_t s, bool pdl) {
   cudaLaunchConfig_t cfg = {};
