@@ -198,14 +198,38 @@ def extra_lms(w: synth.Workload, k: int):
             for i in range(k)]
 
 
-def oracle_models(w, inp_lm, inp_ph, E, W, extra=()):
+def pred_weights(w: synth.Workload, D: int):
+    """The stateful form's prediction network (D LSTM units) and joint
+    projections; encoder frames stay H wide (H_enc = H)."""
+    return synth.pred_weights(w, D=D, Henc=w.H) if D else None
+
+
+def variant_config(args, w, extra):
+    """The config keys that name a variant of the workload."""
+    out, names = {}, []
+    if extra:
+        out.update(lms=1 + len(extra), lm_weights=[1.0] + [wt for _, wt in extra])
+        names.append(f"+ {len(extra)} more LMs (half size, weight 0.5)")
+    if args.prune_k:
+        out["prune_k"] = args.prune_k
+        names.append(f"fusion pruned to the acoustic top {args.prune_k}")
+    if args.pred:
+        out["prediction_network"] = {"kind": "1-layer LSTM over the previous label", "D": args.pred, "H_enc": w.H}
+        names.append(f"stateful form: LSTM prediction network D={args.pred} + joint projections")
+    if names:
+        out["workload"] = f"cfg{w.cfg} {w.name}, " + "; ".join(names)
+    return out
+
+
+def oracle_models(w, inp_lm, inp_ph, E, W, extra=(), pred=None):
     import oracle
 
     olm = oracle.LM.from_arrays(inp_lm) if inp_lm is not None else None
     if extra:
         olm = [(olm, 1.0)] + [(oracle.LM.from_arrays(a), wt) for a, wt in extra]
     obo = oracle.Boost.from_phrases(w.V, inp_ph, w.bonus) if inp_ph is not None else None
-    return olm, obo, oracle.Model(w.V, w.H, E, W)
+    pn = oracle.PredNet(w.V, w.H, pred) if pred is not None else None
+    return olm, obo, oracle.Model(w.V, w.H, E, W), pn
 
 
 def oracle_baseline(w, models, streams, chunks, threads=None, prune_k=0):
@@ -216,13 +240,14 @@ def oracle_baseline(w, models, streams, chunks, threads=None, prune_k=0):
     import oracle
 
     threads = threads or len(os.sched_getaffinity(0))
-    olm, obo, model = models
+    olm, obo, model, pn = models
     encs = {c: synth.enc_chunk(w, streams, c) for c in range(chunks)}
 
     def one(i):
         st = oracle.Stream(w.V)
         for c in range(chunks):
-            oracle.decode_chunk(st, model, olm, obo, encs[c][i], w.lam, w.beta, w.max_sym, prune_k=prune_k)
+            oracle.decode_chunk(st, model, olm, obo, encs[c][i], w.lam, w.beta, w.max_sym, prune_k=prune_k,
+                                pred=pn)
 
     t0 = time.perf_counter()
     with concurrent.futures.ThreadPoolExecutor(max_workers=threads) as ex:
@@ -244,7 +269,7 @@ def run_reference(args, w):
     E, W = synth.joint_weights(w)
     n_str = args.ref_streams
     extra = extra_lms(w, args.extra_lms) if args.extra_lms else []
-    models = oracle_models(w, lmA, ph, E, W, extra)
+    models = oracle_models(w, lmA, ph, E, W, extra, pred_weights(w, args.pred))
     # warm-up steps, then K timed steps; each step decodes a bounded sample
     for _ in range(args.warmup):
         oracle_baseline(w, models, list(range(2)), 1, prune_k=args.prune_k)
@@ -260,12 +285,7 @@ def run_reference(args, w):
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
             "data": "synthetic",
             "config": dict(workload_config(w, lmA.total + sum(a.total for a, _ in extra), ph.n if ph else 0),
-                           **({"lms": 1 + len(extra), "lm_weights": [1.0] + [wt for _, wt in extra],
-                               "workload": f"cfg{w.cfg} {w.name} + {len(extra)} more LMs (half size, weight 0.5)"}
-                              if extra else {}),
-                           **({"prune_k": args.prune_k,
-                               "workload": f"cfg{w.cfg} {w.name}, fusion pruned to the acoustic top {args.prune_k}"}
-                              if args.prune_k else {})),
+                           **variant_config(args, w, extra)),
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
                              "sample": f"per step: {sample}"},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
@@ -294,9 +314,10 @@ def run_ours(args, w):
     extra = extra_lms(w, args.extra_lms) if args.extra_lms else []
     lms = [(lm, 1.0)] + [(tsd.NGram.from_arrays(a), wt) for a, wt in extra] if extra else None
     bo = tsd.Boost.from_phrases(w.V, ph, w.bonus) if ph is not None else None
+    pw = pred_weights(w, args.pred)
     dec = tsd.Decoder(w.V, w.H, torch.from_numpy(W.view(np.int16)).to(dev), torch.from_numpy(E.view(np.int16)).to(dev),
                       lm=None if lms else lm, lms=lms, boost=bo, max_symbols=w.max_sym, beam_k=w.beam,
-                      max_streams=w.B, max_T=w.T, prune_k=args.prune_k)
+                      max_streams=w.B, max_T=w.T, prune_k=args.prune_k, pred=pw)
     slots = [dec.open() for _ in range(w.B)]
     slots_np = np.array(slots, dtype=np.int32)
     n_chunks = args.warmup + args.steps + 1
@@ -409,7 +430,10 @@ def run_ours(args, w):
     pk, pk_kind = peaks()
     M = w.B * w.beam
     flop_per_launch = 2.0 * M * w.H * (w.V + 1)
-    share_joint = kernel_ms["joint"] / max(1e-9, sum(kernel_ms.values()))
+    total_ms = max(1e-9, sum(kernel_ms.values()))
+    share_joint = kernel_ms["joint"] / total_ms
+    share_row = kernel_ms["row"] / total_ms
+    share_pred = kernel_ms["pred"] / total_ms
     # In-graph figures: CUDA events at every kernel boundary on the launching
     # stream over the instrumented pass of the K timed steps.  A kernel timed
     # inside a long step takes the sustained bf16 peak.
@@ -444,7 +468,7 @@ def run_ours(args, w):
                                 f"shared unigram/root rows once per launch; the dense bias row is not counted"),
                 "avg_launch_ms": row_ms, "launches": kernel_n["row"],
                 "traffic": recorded_traffic(w, "row"),
-                "share_of_device_time": 1.0 - share_joint,
+                "share_of_device_time": share_row,
                 "isolated": {"what": "the chunk's last label step replayed with every row evaluated",
                              "bytes_per_launch": row_bytes, "cold_l2_ms": row_cold, "warm_l2_ms": row_warm,
                              "achieved_cold": row_bytes / (row_cold / 1000.0) / 1e9,
@@ -458,7 +482,7 @@ def run_ours(args, w):
     step_ms = t_ms / args.steps
     for roof_k, share, n_per_step, work in (
             (joint_roof, share_joint, kernel_n["joint"] / args.steps, flop_per_launch / 1e12),
-            (row_roof, 1.0 - share_joint, kernel_n["row"] / args.steps,
+            (row_roof, share_row, kernel_n["row"] / args.steps,
              row_bytes_graph / max(1, kernel_n["row"]) / 1e9)):
         ms_in_graph = step_ms * share / max(1e-9, n_per_step)
         roof_k["in_production_graph"] = {
@@ -467,19 +491,38 @@ def run_ours(args, w):
             "achieved": work / (ms_in_graph / 1000.0),
         }
         roof_k["in_production_graph"]["frac"] = roof_k["in_production_graph"]["achieved"] / roof_k["peak"]
-    # the dominant kernel is the one with the larger device time in the graph
-    roof, other = (joint_roof, row_roof) if share_joint >= 0.5 else (row_roof, joint_roof)
+    pred_roof = None
+    if args.pred:
+        # the stateful form's GEMMs per chunk: the encoder projection, an LSTM
+        # gate GEMM per label step and after the last, a joint-input GEMM per step
+        S = w.T * w.max_sym
+        D = args.pred
+        pred_flop = 2.0 * M * w.T * w.H * w.H + (S + 1) * 2.0 * M * (2 * D) * (4 * D) + S * 2.0 * M * D * w.H
+        pred_chunk_ms = kernel_ms["pred"] / args.steps
+        pred_roof = {"kernel": "k_gemm_tc: encoder projection, LSTM cell and joint-input GEMMs (tcgen05)",
+                     "bound": "tensor", "unit": "TFLOP/s",
+                     "achieved": pred_flop / (pred_chunk_ms / 1000.0) / 1e12,
+                     "peak": pk["bf16_tflops_sustained"],
+                     "peak_kind": f"{pk_kind} bf16 sustained (kernels timed inside the decode step)",
+                     "algorithmic": f"{pred_flop:.4g} FLOP per chunk (M={M} rows, D={D}, S={S} label steps)",
+                     "ms_per_chunk": pred_chunk_ms, "launches": kernel_n["pred"],
+                     "traffic": None, "share_of_device_time": share_pred}
+        pred_roof["frac"] = pred_roof["achieved"] / pred_roof["peak"]
+        pred_roof["in_production_graph"] = {
+            "what": "uninstrumented step time x this class's share of device time",
+            "ms_per_chunk": step_ms * share_pred,
+            "achieved": pred_flop / (step_ms * share_pred / 1000.0) / 1e12}
+        pred_roof["in_production_graph"]["frac"] = pred_roof["in_production_graph"]["achieved"] / pred_roof["peak"]
+    # the dominant kernel is the one with the largest device time in the graph
+    ranked = sorted([(share_joint, joint_roof), (share_row, row_roof)] + ([(share_pred, pred_roof)] if pred_roof else []),
+                    key=lambda x: -x[0])
+    roof, other = ranked[0][1], ranked[1][1]
     launches = dec.launches_per_chunk(w.B, w.T)
     line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": t_ms / args.steps, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
             "config": dict(workload_config(w, lmA.total + sum(a.total for a, _ in extra), ph.n if ph else 0),
-                           **({"lms": 1 + len(extra), "lm_weights": [1.0] + [wt for _, wt in extra],
-                               "workload": f"cfg{w.cfg} {w.name} + {len(extra)} more LMs (half size, weight 0.5)"}
-                              if extra else {}),
-                           **({"prune_k": args.prune_k,
-                               "workload": f"cfg{w.cfg} {w.name}, fusion pruned to the acoustic top {args.prune_k}"}
-                              if args.prune_k else {}),
+                           **variant_config(args, w, extra),
                            l2="flushed (256 MB write) before every timed step, outside the step's events",
                            parallelism=f"dp{ws} (independent streams per GPU)"),
             "e2e": {"value": e2e_val, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
@@ -487,6 +530,7 @@ def run_ours(args, w):
             "gpu_launches": int(launches * args.steps),
             "roofline": roof,
             "roofline_other_kernel": other,
+            **({"roofline_third_kernel": ranked[2][1]} if len(ranked) > 2 else {}),
             "latency_per_chunk": latency_stats(step_ms),
             "wall_s_timed_region": wall,
             "value_with_kernel_events": frames / (t_inst_ms / 1000.0),
@@ -494,7 +538,7 @@ def run_ours(args, w):
                              "graph, over a second pass of the same K steps (value_with_kernel_events)",
             "clocks": clk.summary()}
     if not args.no_cpu_baseline and ws == 1:
-        models = oracle_models(w, lmA, ph, E, W, extra)
+        models = oracle_models(w, lmA, ph, E, W, extra, pw)
         v, cores, sample, dt = oracle_baseline(w, models, list(range(args.cpu_streams)), args.cpu_chunks,
                                                prune_k=args.prune_k)
         line["cpu_baseline"] = {"value": v, "unit": UNIT, "cores": cores, "kind": "oracle",
@@ -517,6 +561,8 @@ def main():
     ap.add_argument("--extra-lms", type=int, default=0, help="fuse this many further LMs (several-LM workload)")
     ap.add_argument("--prune-k", type=int, default=0,
                     help="pruned fusion over the acoustic model's k best outputs (0: every label)")
+    ap.add_argument("--pred", type=int, default=0,
+                    help="stateful form: an LSTM prediction network of this many units (0: stateless)")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")

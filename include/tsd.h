@@ -324,7 +324,10 @@ TSD_API tsd_status tsd_decoder_set_timing(tsd_decoder* dec, int32_t enable);
 
 /* Accumulated device time (ms) and launch counts since the last reset, per
  * kernel class: [0] row pass (state advance, LM + boost bias, joint input),
- * [1] joint GEMM with the fused log-softmax/selection epilogue.  Waits for
+ * [1] joint GEMM with the fused log-softmax/selection epilogue, [2] the
+ * stateful form's prediction network and projections (the chunk's encoder
+ * copy and projection, each step's LSTM and joint-input GEMMs; 0 for a
+ * stateless decoder).  n_classes (1..3) entries are written.  Waits for
  * outstanding timed work.  reset != 0 clears the totals after reading. */
 TSD_API tsd_status tsd_decoder_timing(tsd_decoder* dec, double* ms, int64_t* launches, int32_t n_classes,
                               int32_t reset);

@@ -408,11 +408,14 @@ class Decoder:
         _check(lib().tsd_decoder_set_timing(self.h, 1 if enable else 0))
 
     def timing(self, reset: bool = False):
-        """({'row': ms, 'joint': ms}, {'row': launches, 'joint': launches})"""
-        ms = np.zeros(2, dtype=np.float64)
-        ln = np.zeros(2, dtype=np.int64)
-        _check(lib().tsd_decoder_timing(self.h, ms.ctypes.data, ln.ctypes.data, 2, 1 if reset else 0))
-        return {"row": float(ms[0]), "joint": float(ms[1])}, {"row": int(ln[0]), "joint": int(ln[1])}
+        """({'row': ms, 'joint': ms, 'pred': ms}, {... launches}): device time
+        of timed chunks per kernel class; 'pred' is the stateful form's
+        prediction network and projections."""
+        ms = np.zeros(3, dtype=np.float64)
+        ln = np.zeros(3, dtype=np.int64)
+        _check(lib().tsd_decoder_timing(self.h, ms.ctypes.data, ln.ctypes.data, 3, 1 if reset else 0))
+        keys = ("row", "joint", "pred")
+        return {k: float(ms[i]) for i, k in enumerate(keys)}, {k: int(ln[i]) for i, k in enumerate(keys)}
 
     def timed_bytes(self, reset: bool = False) -> int:
         """Algorithmic bytes counted by the row passes of timed chunks."""

@@ -33,9 +33,15 @@ tsd_status set_device(const tsd_decoder* d) {
 
 int steps_per_chunk(const tsd_decoder* d, int T) { return T * d->cfg.max_symbols; }
 
+// Events enqueue_chunk records with timing on: a mark before every row pass
+// and joint launch (and, for the stateful form, before the chunk's encoder
+// projection and each step's prediction-network GEMMs), and one at the end.
+int n_marks(const tsd_decoder* d, int S) { return d->pred.D ? 3 * S + 4 : 2 * S + 2; }
+
 // Enqueues one chunk's launches; with events, records one at each kernel
 // boundary (external records, so they survive graph capture).
-void enqueue_chunk(tsd_decoder* d, int M, int T, cudaStream_t s, const std::vector<cudaEvent_t>* ev) {
+void enqueue_chunk(tsd_decoder* d, int M, int T, cudaStream_t s, const std::vector<cudaEvent_t>* ev,
+                   std::vector<int8_t>* cls_out) {
   const int S = steps_per_chunk(d, T);
   int e = 0;
   // timed chunks also count the row passes' algorithmic bytes (second counter)
@@ -44,26 +50,31 @@ void enqueue_chunk(tsd_decoder* d, int M, int T, cudaStream_t s, const std::vect
     v.count = 1;
     v.ctr = d->view.ctr + 1;
   }
-  auto mark = [&]() {
-    if (ev) cudaEventRecordWithFlags((*ev)[(size_t)e++], s, cudaEventRecordExternal);
+  auto mark = [&](int cls) {
+    if (!ev) return;
+    cudaEventRecordWithFlags((*ev)[(size_t)e], s, cudaEventRecordExternal);
+    if (cls_out) (*cls_out)[(size_t)e] = (int8_t)cls;
+    ++e;
   };
   const tsd_decoder::Pred& pr = d->pred;
+  launch_defaults(v, s);
   if (pr.D) {
     // the chunk's encoder frames to a fixed buffer, then their projection
+    mark(2);
     launch_copy_enc(v, (int64_t)M * T * pr.Henc, s, false);
     GemmArgs ge{M * T, d->cfg.H, pr.Henc, d->cfg.H, pr.be, v.pred_penc};
     launch_gemm_tc(kEncProj, v, ge, pr.encA, pr.encB, pr.H_pad, s, d->pdl && !ev);
   }
-  launch_defaults(v, s);
   for (int step = 0; step <= S; ++step) {
     const bool pdl = d->pdl && !ev && step > 0;  // the first launch follows the parameter copy
-    mark();
+    mark(0);
     if (d->cfg.beam_k > 1) launch_row_beam(v, M / d->cfg.beam_k, step, step == S ? 1 : 0, d->row_smem, s, pdl);
     else if (d->cfg.prune_k > 0) launch_row_pruned(v, M, step, step == S ? 1 : 0, s, pdl);
     else launch_row(v, M, step, step == S ? 1 : 0, d->row_smem, s, pdl);
     if (pr.D) {
       // the prediction network reads the labels just emitted; after the last
       // decision of the chunk only its state matters
+      mark(2);
       GemmArgs gl{M, 4 * pr.D, 2 * pr.D, 0, pr.bg, nullptr};
       launch_gemm_tc(kLstm, v, gl, pr.lstmA, pr.lstmB, pr.G_pad, s, d->pdl && !ev);
       if (step < S) {
@@ -72,12 +83,12 @@ void enqueue_chunk(tsd_decoder* d, int M, int T, cudaStream_t s, const std::vect
       }
     }
     if (step < S) {
-      mark();
+      mark(1);
       if (d->joint_kind == 0) launch_joint_tc(*d->jtc, v, M, step, s, d->pdl && !ev);
       else launch_joint(v, M, step, s);
     }
   }
-  mark();
+  mark(-1);
 }
 
 void harvest(tsd_decoder* d, tsd_decoder::EventSet& es) {
@@ -85,9 +96,10 @@ void harvest(tsd_decoder* d, tsd_decoder::EventSet& es) {
   cudaEventSynchronize(es.ev.back());
   for (size_t i = 0; i + 1 < es.ev.size(); ++i) {
     float ms = 0.f;
-    if (cudaEventElapsedTime(&ms, es.ev[i], es.ev[i + 1]) == cudaSuccess) {
-      d->ms[i & 1] += ms;
-      d->launches[i & 1] += 1;
+    const int c = es.cls[i];
+    if (c >= 0 && c < 3 && cudaEventElapsedTime(&ms, es.ev[i], es.ev[i + 1]) == cudaSuccess) {
+      d->ms[c] += ms;
+      d->launches[c] += 1;
     }
   }
   cudaGetLastError();
@@ -523,7 +535,7 @@ extern "C" tsd_status tsd_decode_chunk(tsd_decoder* d, int32_t n, const int32_t*
   const int S = steps_per_chunk(d, T);
   d->last_n = n;
   d->last_T = T;
-  const int n_events = 2 * S + 2;
+  const int n_events = n_marks(d, S);
   auto key = std::make_tuple(n, T, d->use_graphs, d->timing);
   tsd_decoder::Entry& ent = d->entries[key];
   tsd_decoder::EventSet& es = ent.set[ent.next];
@@ -532,6 +544,7 @@ extern "C" tsd_status tsd_decode_chunk(tsd_decoder* d, int32_t n, const int32_t*
     harvest(d, es);
     if (es.ev.empty()) {
       es.ev.resize((size_t)n_events);
+      es.cls.assign((size_t)n_events, -1);
       for (auto& e : es.ev) TSD_CUDA(cudaEventCreate(&e));
     }
   }
@@ -540,7 +553,7 @@ extern "C" tsd_status tsd_decode_chunk(tsd_decoder* d, int32_t n, const int32_t*
     if (!es.exec) {
       cudaGraph_t g = nullptr;
       TSD_CUDA(cudaStreamBeginCapture(d->cap_stream, cudaStreamCaptureModeThreadLocal));
-      enqueue_chunk(d, M, T, d->cap_stream, evp);
+      enqueue_chunk(d, M, T, d->cap_stream, evp, d->timing ? &es.cls : nullptr);
       cudaError_t ce = cudaStreamEndCapture(d->cap_stream, &g);
       if (ce != cudaSuccess) return cuda_fail(ce, "tsd_decode_chunk: graph capture");
       ce = cudaGraphInstantiate(&es.exec, g, 0);
@@ -552,7 +565,7 @@ extern "C" tsd_status tsd_decode_chunk(tsd_decoder* d, int32_t n, const int32_t*
     }
     TSD_CUDA(cudaGraphLaunch(es.exec, s));
   } else {
-    enqueue_chunk(d, M, T, s, evp);
+    enqueue_chunk(d, M, T, s, evp, d->timing ? &es.cls : nullptr);
     TSD_CUDA(cudaGetLastError());
   }
   if (d->timing) es.pending = true;
@@ -883,13 +896,15 @@ extern "C" tsd_status tsd_decoder_timing(tsd_decoder* d, double* ms, int64_t* la
     harvest(d, kv.second.set[0]);
     harvest(d, kv.second.set[1]);
   }
-  for (int i = 0; i < n_classes && i < 2; ++i) {
+  for (int i = 0; i < n_classes && i < 3; ++i) {
     if (ms) ms[i] = d->ms[i];
     if (launches) launches[i] = d->launches[i];
   }
   if (reset) {
-    d->ms[0] = d->ms[1] = 0;
-    d->launches[0] = d->launches[1] = 0;
+    for (int i = 0; i < 3; ++i) {
+      d->ms[i] = 0;
+      d->launches[i] = 0;
+    }
   }
   return TSD_OK;
 }

@@ -131,6 +131,7 @@ struct tsd_decoder {
 
   struct EventSet {
     std::vector<cudaEvent_t> ev;
+    std::vector<int8_t> cls;  // class of the interval that starts at ev[i]
     cudaGraphExec_t exec = nullptr;
     bool pending = false;
   };
@@ -151,6 +152,8 @@ struct tsd_decoder {
   int pdl = 1;                  // programmatic dependent launch between kernels
   int sms = 0;
   int last_n = 0, last_T = 0;   // shape of the last decode_chunk (for replay)
-  double ms[2] = {0, 0};
-  int64_t launches[2] = {0, 0};
+  // per-kernel-class device time of timed chunks: 0 row pass, 1 joint,
+  // 2 prediction network and projections (stateful form)
+  double ms[3] = {0, 0, 0};
+  int64_t launches[3] = {0, 0, 0};
 };

@@ -30,7 +30,8 @@ constexpr int kGThreads = 192;
 constexpr int kGABytes = kBM * kBK * 2;
 constexpr int kGBBytes = kGN * kBK * 2;
 constexpr int kGStageBytes = kGABytes + kGBBytes;
-constexpr int kGSmem = kGStages * kGStageBytes + 1024 /*align*/ + 256 /*barriers*/;
+constexpr int kGBar = 128;  // mbarriers and the TMEM address
+constexpr int kGSmem = kGStages * kGStageBytes + 1024 /*align*/ + kGBar + kGN * 4 /*bias*/;
 
 __device__ __forceinline__ float sigm(float x) { return 1.f / (1.f + expf(-x)); }
 
@@ -50,6 +51,7 @@ __global__ void __launch_bounds__(kGThreads, 1)
   uint64_t* empty = full + kGStages;
   uint64_t* accum = empty + kGStages;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(accum + 1);
+  float* s_bias = reinterpret_cast<float*>(smem + kGStages * kGStageBytes + kGBar);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int n0 = blockIdx.x * kGN, m0 = blockIdx.y * kBM;
@@ -68,6 +70,11 @@ __global__ void __launch_bounds__(kGThreads, 1)
                  "r"(kGN)
                  : "memory");
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  if (warp >= 2) {
+    // the tile's bias (a constant weight) to shared memory
+    const int j = threadIdx.x - 64;
+    s_bias[j] = n0 + j < g.N ? g.bias[n0 + j] : 0.f;
   }
   fence_before();
   __syncthreads();
@@ -134,67 +141,94 @@ __global__ void __launch_bounds__(kGThreads, 1)
     const int q = warp & 3;
     const int row = q * 32 + lane;
     const int gr = m0 + row;
+    // Per-row operands the epilogue combines with the accumulator are loaded
+    // into registers before the accumulator is ready: with the stores that
+    // follow (possibly aliasing, to the compiler) they would otherwise each
+    // cost a dependent round trip to memory.
+    const Params* P = d.params;
+    const bool live = gr < g.M;
+    int slot = 0, flag = 0, t = 0, T = 1;
+    float4 pre4[EPI == kLstm ? 8 : (EPI == kJointIn ? 32 : 1)];
+    uint4 h4[EPI == kLstm ? 4 : 1];
+    const int D = d.pred_D;
+    const int u0 = n0 / 4;  // kLstm: the tile's first LSTM unit
+    if (EPI == kLstm && live) {
+      slot = P->slots[gr];
+      flag = d.pflag[gr];
+      if (flag) {
+        const float4* cp = reinterpret_cast<const float4*>(d.pred_c + (size_t)slot * D + u0);
+#pragma unroll
+        for (int i = 0; i < 8; ++i) pre4[i] = cp[i];
+      } else {
+        const uint4* hp = reinterpret_cast<const uint4*>(d.pred_h + (size_t)slot * D + u0);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) h4[i] = hp[i];
+      }
+    }
+    if (EPI == kJointIn && live) {
+      t = d.r_t[gr];
+      T = P->T;
+      if (t < T) {
+        const float4* pe = reinterpret_cast<const float4*>(d.pred_penc + ((size_t)gr * T + t) * g.ld + n0);
+#pragma unroll
+        for (int i = 0; i < 32; ++i)
+          if (n0 + 4 * i < g.N) pre4[i] = pe[i];  // N is a multiple of 32: whole chunks
+      }
+    }
     ok = __all_sync(0xffffffffu, mbar_wait(accum, 0));
     if (!ok && lane == 0) atomicOr(d.err, 256);
     fence_after();
     if (ok) {
-      const Params* P = d.params;
       const uint32_t tbase = tmem + ((uint32_t)(q * 32) << 16);
-      // per-row context of the epilogue
-      const bool live = gr < g.M;
-      int slot = 0, flag = 0, t = 0, T = 1;
-      if (EPI == kLstm && live) {
-        slot = P->slots[gr];
-        flag = d.pflag[gr];
-      }
-      if (EPI == kJointIn && live) {
-        t = d.r_t[gr];
-        T = P->T;
-      }
-#pragma unroll 1
+#pragma unroll
       for (int c = 0; c < kGN / 32; ++c) {
         __syncwarp();
         float v[32];
         tmem_ld32(tbase + (uint32_t)(c * 32), v);
         const int c0 = n0 + c * 32;
         if (!live || c0 >= g.N) continue;
+        const float* bb = s_bias + c * 32;
         if (EPI == kEncProj) {
           float* out = g.out + (size_t)gr * g.ld + c0;
 #pragma unroll
           for (int i = 0; i < 32; i += 4)
             *reinterpret_cast<float4*>(out + i) =
-                make_float4(v[i] + g.bias[c0 + i], v[i + 1] + g.bias[c0 + i + 1], v[i + 2] + g.bias[c0 + i + 2],
-                            v[i + 3] + g.bias[c0 + i + 3]);
+                make_float4(v[i] + bb[i], v[i + 1] + bb[i + 1], v[i + 2] + bb[i + 2], v[i + 3] + bb[i + 3]);
         } else if (EPI == kLstm) {
-          const int D = d.pred_D;
+          // columns 4u+q of this chunk: gates (i, f, g, o) of units u0+8c .. u0+8c+7
+          const size_t base = (size_t)slot * D + u0 + 8 * c;
+          uint4 hv;
+          if (flag) {
+            float cn[8];
+            const float* cprev = reinterpret_cast<const float*>(&pre4[2 * c]);
+            uint16_t* hb = reinterpret_cast<uint16_t*>(&hv);
 #pragma unroll
-          for (int j = 0; j < 8; ++j) {
-            const int u = c0 / 4 + j;
-            uint16_t hb;
-            if (flag) {
-              const float gi = sigm(v[4 * j] + g.bias[c0 + 4 * j]);
-              const float gf = sigm(v[4 * j + 1] + g.bias[c0 + 4 * j + 1]);
-              const float gg = tanhf(v[4 * j + 2] + g.bias[c0 + 4 * j + 2]);
-              const float go = sigm(v[4 * j + 3] + g.bias[c0 + 4 * j + 3]);
-              const float cn = gf * d.pred_c[(size_t)slot * D + u] + gi * gg;
-              d.pred_c[(size_t)slot * D + u] = cn;
-              hb = bf16_bits(go * tanhf(cn));
-              d.pred_h[(size_t)slot * D + u] = hb;
-            } else {
-              hb = d.pred_h[(size_t)slot * D + u];
+            for (int j = 0; j < 8; ++j) {
+              const float gi = sigm(v[4 * j] + bb[4 * j]);
+              const float gf = sigm(v[4 * j + 1] + bb[4 * j + 1]);
+              const float gg = tanhf(v[4 * j + 2] + bb[4 * j + 2]);
+              const float go = sigm(v[4 * j + 3] + bb[4 * j + 3]);
+              cn[j] = gf * cprev[j] + gi * gg;
+              hb[j] = bf16_bits(go * tanhf(cn[j]));
             }
-            d.pred_hin[(size_t)gr * D + u] = hb;
+            float4* cw = reinterpret_cast<float4*>(d.pred_c + base);
+            cw[0] = make_float4(cn[0], cn[1], cn[2], cn[3]);
+            cw[1] = make_float4(cn[4], cn[5], cn[6], cn[7]);
+            *reinterpret_cast<uint4*>(d.pred_h + base) = hv;
+          } else {
+            hv = h4[c];
           }
+          *reinterpret_cast<uint4*>(d.pred_hin + (size_t)gr * D + u0 + 8 * c) = hv;
         } else {  // kJointIn
           if (t < T) {
-            const float* pe = d.pred_penc + ((size_t)gr * T + t) * g.ld + c0;
+            const float* pe = reinterpret_cast<const float*>(&pre4[8 * c]);
             uint16_t* a = d.A + (size_t)gr * d.H + c0;
 #pragma unroll
             for (int i = 0; i < 32; i += 8) {
               uint4 o;
               uint16_t* ob = reinterpret_cast<uint16_t*>(&o);
 #pragma unroll
-              for (int k = 0; k < 8; ++k) ob[k] = bf16_bits(fmaxf(pe[i + k] + (v[i + k] + g.bias[c0 + i + k]), 0.f));
+              for (int k = 0; k < 8; ++k) ob[k] = bf16_bits(fmaxf(pe[i + k] + (v[i + k] + bb[i + k]), 0.f));
               *reinterpret_cast<uint4*>(a + i) = o;
             }
           }
