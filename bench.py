@@ -56,7 +56,7 @@ def peaks():
 # changed kernel reports null until it is captured again.  The captures and
 # their commands are summarised under profiles/.
 KERNEL_SOURCES = {
-    "joint": ["joint_tc.cu", "joint_tc.h", "decoder.h", "internal.h"],
+    "joint": ["joint_tc.cu", "joint_tc.h", "tc_common.cuh", "decoder.h", "internal.h"],
     "row": ["row_pass.cu", "row_beam.cu", "row_common.cuh", "decoder.h", "internal.h"],
 }
 TRAFFIC = {

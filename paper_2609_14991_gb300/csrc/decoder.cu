@@ -63,7 +63,7 @@ void enqueue_chunk(tsd_decoder* d, int M, int T, cudaStream_t s, const std::vect
     mark(2);
     launch_copy_enc(v, (int64_t)M * T * pr.Henc, s, false);
     GemmArgs ge{M * T, d->cfg.H, pr.Henc, d->cfg.H, pr.be, v.pred_penc};
-    launch_gemm_tc(kEncProj, v, ge, pr.encA, pr.encB, pr.H_pad, s, d->pdl && !ev);
+    launch_gemm_tc(kEncProj, v, ge, pr.encA, pr.encB, s, d->pdl && !ev);
   }
   for (int step = 0; step <= S; ++step) {
     const bool pdl = d->pdl && !ev && step > 0;  // the first launch follows the parameter copy
@@ -76,10 +76,10 @@ void enqueue_chunk(tsd_decoder* d, int M, int T, cudaStream_t s, const std::vect
       // decision of the chunk only its state matters
       mark(2);
       GemmArgs gl{M, 4 * pr.D, 2 * pr.D, 0, pr.bg, nullptr};
-      launch_gemm_tc(kLstm, v, gl, pr.lstmA, pr.lstmB, pr.G_pad, s, d->pdl && !ev);
+      launch_gemm_tc(kLstm, v, gl, pr.lstmA, pr.lstmB, s, d->pdl && !ev);
       if (step < S) {
         GemmArgs gp{M, d->cfg.H, pr.D, d->cfg.H, pr.bp, nullptr};
-        launch_gemm_tc(kJointIn, v, gp, pr.projA, pr.projB, pr.H_pad, s, d->pdl && !ev);
+        launch_gemm_tc(kJointIn, v, gp, pr.projA, pr.projB, s, d->pdl && !ev);
       }
     }
     if (step < S) {
@@ -294,9 +294,9 @@ tsd_status create_impl(const tsd_decoder_cfg* cfg, const void* W_out_bf16, const
     launch_repack(static_cast<const uint16_t*>(pw->W_pred), pr.Wp, pr.D, c.H, pr.H_pad, s);
     launch_repack(static_cast<const uint16_t*>(pw->W_enc), pr.We, pr.Henc, c.H, pr.H_pad, s);
     if ((ce = cudaGetLastError()) != cudaSuccess) return cleanup(cuda_fail(ce, "tsd_decoder_create_pred: repack"));
-    if (!gemm_tc_map_a(&pr.encA, p_enc, pr.MT_pad, pr.Henc) || !gemm_tc_map_b(&pr.encB, pr.We, pr.H_pad, pr.Henc) ||
-        !gemm_tc_map_a(&pr.lstmA, p_x, d->M_pad, 2 * pr.D) || !gemm_tc_map_b(&pr.lstmB, pr.Wg, pr.G_pad, 2 * pr.D) ||
-        !gemm_tc_map_a(&pr.projA, p_hin, d->M_pad, pr.D) || !gemm_tc_map_b(&pr.projB, pr.Wp, pr.H_pad, pr.D))
+    if (!gemm_tc_map_a(&pr.encA, p_enc, pr.MT_pad, pr.Henc) || !gemm_tc_map_b(&pr.encB, kEncProj, pr.We, pr.H_pad, pr.Henc) ||
+        !gemm_tc_map_a(&pr.lstmA, p_x, d->M_pad, 2 * pr.D) || !gemm_tc_map_b(&pr.lstmB, kLstm, pr.Wg, pr.G_pad, 2 * pr.D) ||
+        !gemm_tc_map_a(&pr.projA, p_hin, d->M_pad, pr.D) || !gemm_tc_map_b(&pr.projB, kJointIn, pr.Wp, pr.H_pad, pr.D))
       return cleanup(fail(TSD_ECUDA, "tsd_decoder_create_pred: TMA descriptors"));
     if ((ce = gemm_tc_prepare()) != cudaSuccess) return cleanup(cuda_fail(ce, "tsd_decoder_create_pred: kernel attributes"));
   }

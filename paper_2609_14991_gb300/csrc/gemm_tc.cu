@@ -24,14 +24,21 @@ namespace {
 
 using namespace tc;
 
-constexpr int kGN = 128;  // output columns per tile
-constexpr int kGStages = 4;
+// Output-tile width per epilogue.  The per-step GEMMs have few rows (one
+// 128-row tile per 128 streams), so narrower tiles put more SMs on the
+// weights, and deeper pipelines keep more of each CTA's k-blocks in flight.
+template <int EPI>
+struct Shape {
+  static constexpr int BN = EPI == kEncProj ? 128 : (EPI == kLstm ? 64 : 32);
+  static constexpr int ABytes = kBM * kBK * 2;
+  static constexpr int BBytes = BN * kBK * 2;
+  static constexpr int StageBytes = ABytes + BBytes;
+  static constexpr int Stages = (200 * 1024) / StageBytes;  // 6 / 8 / 10
+  static constexpr int Smem = Stages * StageBytes + 1024 /*align*/ + 256 /*barriers*/ + BN * 4 /*bias*/;
+  static_assert((2 * Stages + 1) * 8 + 4 <= 256, "barrier area");
+};
 constexpr int kGThreads = 192;
-constexpr int kGABytes = kBM * kBK * 2;
-constexpr int kGBBytes = kGN * kBK * 2;
-constexpr int kGStageBytes = kGABytes + kGBBytes;
-constexpr int kGBar = 128;  // mbarriers and the TMEM address
-constexpr int kGSmem = kGStages * kGStageBytes + 1024 /*align*/ + kGBar + kGN * 4 /*bias*/;
+constexpr int kGBar = 256;  // mbarriers and the TMEM address
 
 __device__ __forceinline__ float sigm(float x) { return 1.f / (1.f + expf(-x)); }
 
@@ -45,6 +52,11 @@ __device__ __forceinline__ float bf16_val(uint16_t u) { return __uint_as_float((
 template <int EPI>
 __global__ void __launch_bounds__(kGThreads, 1)
     k_gemm_tc(DecView d, GemmArgs g, const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB) {
+  constexpr int kGN = Shape<EPI>::BN;
+  constexpr int kGStages = Shape<EPI>::Stages;
+  constexpr int kGABytes = Shape<EPI>::ABytes;
+  constexpr int kGStageBytes = Shape<EPI>::StageBytes;
+  static_assert(kGN % 32 == 0 && kGStageBytes % 1024 == 0, "tile shape");
   extern __shared__ __align__(1024) unsigned char smem_raw[];
   unsigned char* smem = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + kGStages * kGStageBytes);
@@ -74,7 +86,7 @@ __global__ void __launch_bounds__(kGThreads, 1)
   if (warp >= 2) {
     // the tile's bias (a constant weight) to shared memory
     const int j = threadIdx.x - 64;
-    s_bias[j] = n0 + j < g.N ? g.bias[n0 + j] : 0.f;
+    if (j < kGN) s_bias[j] = n0 + j < g.N ? g.bias[n0 + j] : 0.f;
   }
   fence_before();
   __syncthreads();
@@ -148,8 +160,8 @@ __global__ void __launch_bounds__(kGThreads, 1)
     const Params* P = d.params;
     const bool live = gr < g.M;
     int slot = 0, flag = 0, t = 0, T = 1;
-    float4 pre4[EPI == kLstm ? 8 : (EPI == kJointIn ? 32 : 1)];
-    uint4 h4[EPI == kLstm ? 4 : 1];
+    float4 pre4[EPI == kLstm ? kGN / 16 : (EPI == kJointIn ? kGN / 4 : 1)];
+    uint4 h4[EPI == kLstm ? kGN / 32 : 1];
     const int D = d.pred_D;
     const int u0 = n0 / 4;  // kLstm: the tile's first LSTM unit
     if (EPI == kLstm && live) {
@@ -158,11 +170,11 @@ __global__ void __launch_bounds__(kGThreads, 1)
       if (flag) {
         const float4* cp = reinterpret_cast<const float4*>(d.pred_c + (size_t)slot * D + u0);
 #pragma unroll
-        for (int i = 0; i < 8; ++i) pre4[i] = cp[i];
+        for (int i = 0; i < kGN / 16; ++i) pre4[i] = cp[i];
       } else {
         const uint4* hp = reinterpret_cast<const uint4*>(d.pred_h + (size_t)slot * D + u0);
 #pragma unroll
-        for (int i = 0; i < 4; ++i) h4[i] = hp[i];
+        for (int i = 0; i < kGN / 32; ++i) h4[i] = hp[i];
       }
     }
     if (EPI == kJointIn && live) {
@@ -171,7 +183,7 @@ __global__ void __launch_bounds__(kGThreads, 1)
       if (t < T) {
         const float4* pe = reinterpret_cast<const float4*>(d.pred_penc + ((size_t)gr * T + t) * g.ld + n0);
 #pragma unroll
-        for (int i = 0; i < 32; ++i)
+        for (int i = 0; i < kGN / 4; ++i)
           if (n0 + 4 * i < g.N) pre4[i] = pe[i];  // N is a multiple of 32: whole chunks
       }
     }
@@ -250,32 +262,45 @@ bool gemm_tc_map_a(CUtensorMap* m, const uint16_t* A, int rows, int K) {
   return make_map(m, A, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, K, rows, kBK, kBM);
 }
 
-bool gemm_tc_map_b(CUtensorMap* m, const uint16_t* B, int rows, int K) {
-  return make_map(m, B, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, K, rows, kBK, kGN);
+bool gemm_tc_map_b(CUtensorMap* m, int epi, const uint16_t* B, int rows, int K) {
+  const int bn = epi == kEncProj ? Shape<kEncProj>::BN : (epi == kLstm ? Shape<kLstm>::BN : Shape<kJointIn>::BN);
+  return make_map(m, B, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, K, rows, kBK, bn);
 }
 
 cudaError_t gemm_tc_prepare() {
-  cudaError_t e = cudaFuncSetAttribute(k_gemm_tc<kEncProj>, cudaFuncAttributeMaxDynamicSharedMemorySize, kGSmem);
-  if (e == cudaSuccess) e = cudaFuncSetAttribute(k_gemm_tc<kLstm>, cudaFuncAttributeMaxDynamicSharedMemorySize, kGSmem);
-  if (e == cudaSuccess) e = cudaFuncSetAttribute(k_gemm_tc<kJointIn>, cudaFuncAttributeMaxDynamicSharedMemorySize, kGSmem);
+  cudaError_t e = cudaFuncSetAttribute(k_gemm_tc<kEncProj>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       Shape<kEncProj>::Smem);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(k_gemm_tc<kLstm>, cudaFuncAttributeMaxDynamicSharedMemorySize, Shape<kLstm>::Smem);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(k_gemm_tc<kJointIn>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             Shape<kJointIn>::Smem);
   return e;
 }
 
-void launch_gemm_tc(int epi, const DecView& d, const GemmArgs& g, const CUtensorMap& a, const CUtensorMap& b,
-                    int n_pad, cudaStream_t s, bool pdl) {
+namespace {
+template <int EPI>
+void launch_one(const DecView& d, const GemmArgs& g, const CUtensorMap& a, const CUtensorMap& b, cudaStream_t s,
+                bool pdl) {
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(n_pad / kGN, (g.M + kBM - 1) / kBM);
+  cfg.gridDim = dim3((g.N + Shape<EPI>::BN - 1) / Shape<EPI>::BN, (g.M + kBM - 1) / kBM);
   cfg.blockDim = dim3(kGThreads);
-  cfg.dynamicSmemBytes = kGSmem;
+  cfg.dynamicSmemBytes = Shape<EPI>::Smem;
   cfg.stream = s;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = pdl ? 1 : 0;
-  if (epi == kEncProj) cudaLaunchKernelEx(&cfg, k_gemm_tc<kEncProj>, d, g, a, b);
-  else if (epi == kLstm) cudaLaunchKernelEx(&cfg, k_gemm_tc<kLstm>, d, g, a, b);
-  else cudaLaunchKernelEx(&cfg, k_gemm_tc<kJointIn>, d, g, a, b);
+  cudaLaunchKernelEx(&cfg, k_gemm_tc<EPI>, d, g, a, b);
+}
+}  // namespace
+
+void launch_gemm_tc(int epi, const DecView& d, const GemmArgs& g, const CUtensorMap& a, const CUtensorMap& b,
+                    cudaStream_t s, bool pdl) {
+  if (epi == kEncProj) launch_one<kEncProj>(d, g, a, b, s, pdl);
+  else if (epi == kLstm) launch_one<kLstm>(d, g, a, b, s, pdl);
+  else launch_one<kJointIn>(d, g, a, b, s, pdl);
 }
 
 }  // namespace tsd
