@@ -60,12 +60,12 @@ KERNEL_SOURCES = {
     "row": ["row_pass.cu", "row_beam.cu", "row_common.cuh", "decoder.h", "internal.h"],
 }
 TRAFFIC = {
-    (2, 256, "joint"): (4481067, "4a5ba6aa153cde3d"),
-    (2, 256, "row"): (2240580, "96117cbb17f1d671"),
-    (4, 1024, "joint"): (28863795, "4a5ba6aa153cde3d"),
-    (4, 1024, "row"): (13042278, "96117cbb17f1d671"),
-    (3, 128, "joint"): (6380356, "4a5ba6aa153cde3d"),
-    (3, 128, "row"): (1883358, "96117cbb17f1d671"),
+    (2, 256, "joint"): (4480503, "379506cffc5a29e4"),
+    (2, 256, "row"): (2375228, "604db958d36a6061"),
+    (4, 1024, "joint"): (28862839, "379506cffc5a29e4"),
+    (4, 1024, "row"): (14251947, "604db958d36a6061"),
+    (3, 128, "joint"): (6345199, "379506cffc5a29e4"),
+    (3, 128, "row"): (1882778, "604db958d36a6061"),
 }
 
 
