@@ -305,3 +305,144 @@ def enc_chunk_wide(w: Workload, streams, chunk: int, Henc: int, T: Optional[int]
     for i, s in enumerate(streams):
         out[i] = normal_bf16(w.seed, TENSOR_ENC, int(s), chunk * T * Henc, T * Henc, 1.0).reshape(T, Henc)
     return out
+
+
+# --------------------------------------------------------------------------
+# The cache-aware encoder (Sec. III-B): synthetic weights and features.
+
+TENSOR_FEAT = 10
+TENSOR_SUB_W = 11
+TENSOR_SUB_B = 12
+_TENSOR_LAYER0 = 1000  # layer l, tensor j -> 1000 + 64 l + j
+
+
+@dataclasses.dataclass(frozen=True)
+class EncoderCfg:
+    """Shape of a cache-aware Conformer encoder: d model width, `layers`
+    blocks of `heads` attention heads, feed-forward width ff, depthwise kernel
+    K; attention sees `left` cached frames plus the whole current chunk of
+    `chunk` frames; each encoder frame stacks `stack` feature frames of
+    `feat` log-mel bins (80 ms from 10 ms features)."""
+
+    name: str
+    d: int
+    layers: int
+    heads: int
+    ff: int
+    kernel: int = 9
+    left: int = 70
+    chunk: int = 13
+    feat: int = 80
+    stack: int = 8
+    seed: int = 777
+
+    @property
+    def dh(self) -> int:
+        return self.d // self.heads
+
+    @property
+    def n_off(self) -> int:
+        """Relative offsets query - key in a window: -(chunk-1) .. left+chunk-1."""
+        return self.left + 2 * self.chunk - 1
+
+
+# FastConformer-L-like (the 115M model) and FastConformer-XL-like (0.6B) shapes.
+ENCODERS: Dict[str, EncoderCfg] = {
+    "115m": EncoderCfg("115m", d=512, layers=17, heads=8, ff=2048),
+    "0.6b": EncoderCfg("0.6b", d=1024, layers=24, heads=8, ff=4096),
+}
+
+
+@dataclasses.dataclass
+class EncoderLayer:
+    """One Conformer block.  Matrices are bf16 bit patterns stored
+    [out][in] (y = W x); vectors are float32."""
+
+    ln_ff1: tuple  # (gamma [d], beta [d])
+    ff1_w1: np.ndarray  # [ff][d]
+    ff1_b1: np.ndarray
+    ff1_w2: np.ndarray  # [d][ff]
+    ff1_b2: np.ndarray
+    ln_att: tuple
+    qkv_w: np.ndarray  # [3d][d]: rows q, then k, then v; head h owns columns h*dh .. (h+1)*dh-1 of each
+    qkv_b: np.ndarray
+    pos_w: np.ndarray  # [d][d], no bias: P = pos_w r(delta)
+    pos_u: np.ndarray  # [d]: per head, the content bias added to the query
+    pos_v: np.ndarray  # [d]: per head, the position bias added to the query
+    out_w: np.ndarray  # [d][d]
+    out_b: np.ndarray
+    ln_conv: tuple
+    pw1_w: np.ndarray  # [2d][d]: rows 0..d-1 the GLU value, d..2d-1 its gate
+    pw1_b: np.ndarray
+    dw_w: np.ndarray  # [d][K] float32 (bf16 values): tap K-1 is the current frame
+    dw_b: np.ndarray
+    bn_scale: np.ndarray  # [d]: batch norm at inference, an affine map per channel
+    bn_shift: np.ndarray
+    pw2_w: np.ndarray  # [d][d]
+    pw2_b: np.ndarray
+    ln_ff2: tuple
+    ff2_w1: np.ndarray
+    ff2_b1: np.ndarray
+    ff2_w2: np.ndarray
+    ff2_b2: np.ndarray
+    ln_out: tuple
+
+
+@dataclasses.dataclass
+class EncoderWeights:
+    cfg: EncoderCfg
+    sub_w: np.ndarray  # [d][stack*feat]: the stacked feature frames -> d
+    sub_b: np.ndarray
+    layers: List[EncoderLayer]
+
+
+def encoder_weights(cfg: EncoderCfg, layers: Optional[int] = None) -> EncoderWeights:
+    """Seeded weights: matrices ~ N(0, 1/sqrt(fan_in)); biases ~ N(0, 0.02);
+    layer-norm gains 1 + N(0, 0.1) and shifts N(0, 0.05); position biases
+    u, v ~ N(0, 0.1); depthwise taps ~ N(0, 1/sqrt(K)); batch-norm scale
+    1 + N(0, 0.1), shift N(0, 0.05)."""
+    d, ff, K, s = cfg.d, cfg.ff, cfg.kernel, cfg.seed
+    n_layers = cfg.layers if layers is None else layers
+
+    def mat(t, rows, cols):
+        return normal_bf16(s, t, 0, 0, rows * cols, 1.0 / math.sqrt(cols)).reshape(rows, cols)
+
+    def vec(t, n, std, mean=0.0):
+        return (bf16_to_f32(normal_bf16(s, t, 0, 0, n, std)) + np.float32(mean)).astype(np.float32)
+
+    layers_out = []
+    for l in range(n_layers):
+        base = _TENSOR_LAYER0 + 64 * l
+        j = iter(range(64))
+        t = lambda: base + next(j)
+        ln = lambda: (vec(t(), d, 0.1, 1.0), vec(t(), d, 0.05))
+        L = EncoderLayer(
+            ln_ff1=ln(), ff1_w1=mat(t(), ff, d), ff1_b1=vec(t(), ff, 0.02), ff1_w2=mat(t(), d, ff),
+            ff1_b2=vec(t(), d, 0.02),
+            ln_att=ln(), qkv_w=mat(t(), 3 * d, d), qkv_b=vec(t(), 3 * d, 0.02), pos_w=mat(t(), d, d),
+            pos_u=vec(t(), d, 0.1), pos_v=vec(t(), d, 0.1), out_w=mat(t(), d, d), out_b=vec(t(), d, 0.02),
+            ln_conv=ln(), pw1_w=mat(t(), 2 * d, d), pw1_b=vec(t(), 2 * d, 0.02),
+            dw_w=bf16_to_f32(normal_bf16(s, t(), 0, 0, d * K, 1.0 / math.sqrt(K))).reshape(d, K).copy(),
+            dw_b=vec(t(), d, 0.02), bn_scale=vec(t(), d, 0.1, 1.0), bn_shift=vec(t(), d, 0.05),
+            pw2_w=mat(t(), d, d), pw2_b=vec(t(), d, 0.02),
+            ln_ff2=ln(), ff2_w1=mat(t(), ff, d), ff2_b1=vec(t(), ff, 0.02), ff2_w2=mat(t(), d, ff),
+            ff2_b2=vec(t(), d, 0.02),
+            ln_out=ln())
+        layers_out.append(L)
+    sub_w = normal_bf16(s, TENSOR_SUB_W, 0, 0, d * cfg.stack * cfg.feat,
+                        1.0 / math.sqrt(cfg.stack * cfg.feat)).reshape(d, cfg.stack * cfg.feat)
+    sub_b = bf16_to_f32(normal_bf16(s, TENSOR_SUB_B, 0, 0, d, 0.02)).copy()
+    return EncoderWeights(cfg, sub_w, sub_b, layers_out)
+
+
+def features(cfg: EncoderCfg, streams, first: int, C: Optional[int] = None) -> np.ndarray:
+    """Log-mel-like features of encoder frames first .. first+C-1 (C*stack
+    feature frames) of each stream: N(0, 1) as bf16, [n][C*stack][feat].
+    Frame f of a stream is the same whatever the chunking."""
+    C = cfg.chunk if C is None else C
+    per = cfg.stack * cfg.feat
+    out = np.empty((len(streams), C * cfg.stack, cfg.feat), dtype=np.uint16)
+    for i, st in enumerate(streams):
+        out[i] = normal_bf16(cfg.seed, TENSOR_FEAT, int(st), first * per, C * per, 1.0).reshape(C * cfg.stack,
+                                                                                             cfg.feat)
+    return out

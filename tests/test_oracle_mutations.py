@@ -65,3 +65,41 @@ def test_pins_catch_planted_mistake(name, tmp_path):
                         os.path.join(ROOT, "tests", "test_oracle_pred.py"), "-q", "-x", "-p", "no:cacheprovider"], cwd=ROOT, capture_output=True, text=True,
                        env=dict(os.environ, TSD_ORACLE_LIB=str(so)), timeout=600)
     assert r.returncode != 0, f"pins did not catch: {name}\n{r.stdout[-2000:]}"
+
+
+# Planted mistakes in copies of the encoder oracle (oracle/encoder.py).
+ENCODER_MUTATIONS = {
+    "content bias u dropped": ('qu = q[:, c] + P["pos_u"][c]', 'qu = q[:, c]'),
+    "relative offset sign flipped": ("delta = pos_q[:, None] - pos_k[None, :]",
+                                     "delta = pos_k[None, :] - pos_q[:, None]"),
+    "sin and cos swapped in the position code": ("r[:, 0::2] = np.sin(ang)\n    r[:, 1::2] = np.cos(ang)",
+                                                 "r[:, 0::2] = np.cos(ang)\n    r[:, 1::2] = np.sin(ang)"),
+    "attention cache ignored": ("K = np.concatenate([st.k[l], k])", "K = np.concatenate([st.k[l][:0], k])"),
+    "attention cache keeps the oldest frames": ("st.k[l] = K[-cfg.left:] if cfg.left > 0 else K[:0]",
+                                                "st.k[l] = K[:cfg.left]"),
+    "convolution cache not carried": ("st.conv[l] = seq[seq.shape[0] - (K - 1):]", "pass"),
+    "convolution taps reversed": ("dw[t] = (P[\"dw_w\"] * seq[t:t + K].T).sum(axis=1) + P[\"dw_b\"]",
+                                  "dw[t] = (P[\"dw_w\"][:, ::-1] * seq[t:t + K].T).sum(axis=1) + P[\"dw_b\"]"),
+    "GLU halves swapped": ("glu = rnd(y[:, :d] * sigmoid(y[:, d:]))", "glu = rnd(y[:, d:] * sigmoid(y[:, :d]))"),
+    "feed-forward half step dropped": ("x = x + 0.5 * _feed_forward(x, *P[\"ln_ff1\"]",
+                                       "x = x + 1.0 * _feed_forward(x, *P[\"ln_ff1\"]"),
+    "softmax over the head dimension": ("a = a / a.sum(axis=1, keepdims=True)",
+                                        "a = a / a.sum(axis=0, keepdims=True)"),
+    "batch norm shift dropped": ('z = rnd(swish(dw * P["bn_scale"] + P["bn_shift"]))',
+                                 'z = rnd(swish(dw * P["bn_scale"]))'),
+    "rounding to nearest truncates": ("return np.ldexp(np.rint(np.ldexp(m, 8)), e - 8)",
+                                      "return np.ldexp(np.trunc(np.ldexp(m, 8)), e - 8)"),
+}
+
+
+@pytest.mark.parametrize("name", sorted(ENCODER_MUTATIONS))
+def test_encoder_pins_catch_planted_mistake(name, tmp_path):
+    src = open(os.path.join(ROOT, "oracle", "encoder.py")).read()
+    a, b = ENCODER_MUTATIONS[name]
+    assert a in src, "mutation anchor not found; update the mutation list"
+    mod = tmp_path / "encoder_mutant.py"
+    mod.write_text(src.replace(a, b))
+    r = subprocess.run([sys.executable, "-m", "pytest", os.path.join(ROOT, "tests", "test_oracle_encoder.py"), "-q",
+                        "-x", "-p", "no:cacheprovider"], cwd=ROOT, capture_output=True, text=True,
+                       env=dict(os.environ, TSD_ORACLE_ENCODER=str(mod)), timeout=600)
+    assert r.returncode != 0, f"pins did not catch: {name}\n{r.stdout[-2000:]}"
