@@ -413,6 +413,104 @@ TSD_API tsd_status tsd_decoder_launches_per_chunk(const tsd_decoder* dec, int32_
 TSD_API tsd_status tsd_decoder_debug_capture(tsd_decoder* dec, float* logits, int32_t* rows,
                                      int32_t max_steps);
 
+/* ------------------------------------------------------------------------
+ * The cache-aware encoder chunk step (Sec. III-B: a FastConformer encoder
+ * made streamable by chunked, limited-context attention and causal
+ * convolutions, with a cache carried across chunks; Sec. IV-A: one encoder
+ * frame is 80 ms and the look-ahead is the chunk).  Its output frames are
+ * the enc input of tsd_decode_chunk (decoder H = d).
+ *
+ * Per stream and chunk of C encoder frames (C*stack feature frames):
+ *   x = W_sub stack(features) + b_sub, then per block:
+ *   x += 1/2 FF1(x);  x += MHSA(x);  x += Conv(x);  x += 1/2 FF2(x);
+ *   x = LN_out(x)
+ *   FF(x)   = W2 bf16(Swish(W1 bf16(LN(x)) + b1)) + b2
+ *   MHSA(x) = W_o bf16(attn) + b_o with (q, k, v) = bf16(W_qkv bf16(LN(x))
+ *             + b_qkv); per head a query frame sees the last `left` frames
+ *             before its chunk (cached k, v) and every frame of its chunk,
+ *             score = ((q + u).k + (q + v).p(delta)) / sqrt(dh), p(delta) =
+ *             W_pos r(delta), r(delta) sinusoidal (sin at 2k, cos at 2k+1 of
+ *             delta / 10000^(2k/d)), delta = query - key frame position
+ *   Conv(x) = W_pw2 bf16(Swish(bn_scale (dw * g) + bn_shift)) + b_pw2 with
+ *             g = bf16(a * sigmoid(b)), (a, b) = W_pw1 bf16(LN(x)) + b_pw1,
+ *             dw * g the causal depthwise convolution over the last K
+ *             frames of g (K-1 of them cached; zeros before the stream's
+ *             first frame) plus b_dw
+ * The chunk's output is bf16(x).  Matrix products take bf16 operands and
+ * accumulate in fp32 on the tensor cores; the rest is fp32. */
+typedef struct tsd_encoder tsd_encoder;
+
+typedef struct {
+  int32_t d;           /* model width: multiple of 128, 128 <= d <= 2048 */
+  int32_t layers;      /* blocks, 1..64 */
+  int32_t heads;       /* attention heads; d / heads is 64 or 128 */
+  int32_t ff;          /* feed-forward width: multiple of 128, <= 8192 */
+  int32_t kernel;      /* depthwise kernel K, 1..32 */
+  int32_t left;        /* cached frames a query sees before its chunk, 0..128 */
+  int32_t max_chunk;   /* largest C a call may pass, 1..32 */
+  int32_t feat;        /* feature bins per 10 ms frame */
+  int32_t stack;       /* feature frames per encoder frame; stack*feat a multiple of 64, <= 8192 */
+  int32_t max_streams; /* slots, 1..4096 */
+} tsd_encoder_cfg;
+
+/* One block's weights, all device arrays (copied at create).  Matrices are
+ * bf16 [out][in] row-major (y = W x); vectors fp32. */
+typedef struct {
+  const float *ln_ff1_g, *ln_ff1_b;
+  const void* ff1_w1;  const float* ff1_b1;   /* [ff][d], [ff] */
+  const void* ff1_w2;  const float* ff1_b2;   /* [d][ff], [d] */
+  const float *ln_att_g, *ln_att_b;
+  const void* qkv_w;   const float* qkv_b;    /* [3d][d] (rows q, k, v; head h owns columns h*dh..), [3d] */
+  const void* pos_w;                          /* [d][d] */
+  const float *pos_u, *pos_v;                 /* [d] each (head h: entries h*dh..) */
+  const void* out_w;   const float* out_b;    /* [d][d], [d] */
+  const float *ln_conv_g, *ln_conv_b;
+  const void* pw1_w;   const float* pw1_b;    /* [2d][d] (rows 0..d-1 the GLU value, d..2d-1 its gate), [2d] */
+  const float *dw_w, *dw_b;                   /* [d][K] (tap K-1 is the current frame), [d] */
+  const float *bn_scale, *bn_shift;           /* [d] each */
+  const void* pw2_w;   const float* pw2_b;    /* [d][d], [d] */
+  const float *ln_ff2_g, *ln_ff2_b;
+  const void* ff2_w1;  const float* ff2_b1;
+  const void* ff2_w2;  const float* ff2_b2;
+  const float *ln_out_g, *ln_out_b;
+} tsd_encoder_layer;
+
+/* Creates an encoder: sub_w bf16 [d][stack*feat] and sub_b fp32 [d] (device),
+ * layers[cfg.layers].  Allocates all device memory up front (weights,
+ * position tables, every slot's cache, work buffers for max_streams *
+ * max_chunk frames).  TSD_EINVAL on a shape outside the limits above. */
+TSD_API tsd_status tsd_encoder_create(const tsd_encoder_cfg* cfg, const void* sub_w, const float* sub_b,
+                                      const tsd_encoder_layer* layers, void* cuda_stream, tsd_encoder** out);
+TSD_API void tsd_encoder_free(tsd_encoder* enc);
+
+/* Opens a stream slot with an empty cache (its first chunk sees no
+ * history); TSD_ESTATE when every slot is open.  Asynchronous on the
+ * encoder's last stream. */
+TSD_API tsd_status tsd_encoder_open(tsd_encoder* enc, int32_t* slot_out);
+TSD_API tsd_status tsd_encoder_close(tsd_encoder* enc, int32_t slot);
+
+/* Encodes one chunk of C encoder frames for n open slots (host array
+ * slots[n], distinct).  feats: device bf16 [n][C*stack][feat] (stream i's
+ * feature frames, oldest first); out: device bf16 [n][C][d].  Each slot's
+ * cache advances by C frames.  Asynchronous on cuda_stream; the first call
+ * for an (n, C) captures a CUDA graph.  TSD_EINVAL on n, C outside
+ * [1, max_streams] x [1, max_chunk]; TSD_ESTATE on a slot that is not open. */
+TSD_API tsd_status tsd_encode_chunk(tsd_encoder* enc, int32_t n, const int32_t* slots, const void* feats_bf16,
+                                    int32_t C, void* out_bf16, void* cuda_stream);
+
+/* Waits for the encoder's stream; TSD_EDEVICE if a bounded wait inside a
+ * kernel expired (the code is cleared). */
+TSD_API tsd_status tsd_encoder_check(tsd_encoder* enc);
+
+/* 1: later encode_chunk calls record CUDA events around every kernel and
+ * accumulate device time per class: [0] tensor-core GEMMs, [1] attention,
+ * [2] the rest (layer norms, depthwise convolution, cache bookkeeping). */
+TSD_API tsd_status tsd_encoder_set_timing(tsd_encoder* enc, int32_t enable);
+TSD_API tsd_status tsd_encoder_timing(tsd_encoder* enc, double* ms, int64_t* launches, int32_t n_classes,
+                                      int32_t reset);
+/* Tensor-core FLOPs of one encode_chunk(n, C) (2 M N K summed over its GEMMs). */
+TSD_API tsd_status tsd_encoder_gemm_flops(const tsd_encoder* enc, int32_t n, int32_t C, double* flops);
+
 #ifdef __cplusplus
 }
 #endif

@@ -44,6 +44,22 @@ class DecoderCfg(ctypes.Structure):
                 ("max_T", _i32), ("prune_k", _i32)]
 
 
+class EncoderCfgC(ctypes.Structure):
+    _fields_ = [(n, _i32) for n in ("d", "layers", "heads", "ff", "kernel", "left", "max_chunk", "feat", "stack",
+                                    "max_streams")]
+
+
+# field order of tsd_encoder_layer
+_ENC_LAYER_FIELDS = ["ln_ff1_g", "ln_ff1_b", "ff1_w1", "ff1_b1", "ff1_w2", "ff1_b2", "ln_att_g", "ln_att_b", "qkv_w",
+                     "qkv_b", "pos_w", "pos_u", "pos_v", "out_w", "out_b", "ln_conv_g", "ln_conv_b", "pw1_w", "pw1_b",
+                     "dw_w", "dw_b", "bn_scale", "bn_shift", "pw2_w", "pw2_b", "ln_ff2_g", "ln_ff2_b", "ff2_w1",
+                     "ff2_b1", "ff2_w2", "ff2_b2", "ln_out_g", "ln_out_b"]
+
+
+class EncoderLayerC(ctypes.Structure):
+    _fields_ = [(n, _vp) for n in _ENC_LAYER_FIELDS]
+
+
 SIGNATURES = {
     "tsd_last_error": ([], ctypes.c_char_p),
     "tsd_version": ([], ctypes.c_char_p),
@@ -85,6 +101,15 @@ SIGNATURES = {
     "tsd_decoder_set_option": ([_vp, ctypes.c_char_p, _i64], _i32),
     "tsd_decoder_replay": ([_vp, _i32, _i32, _vp, _P(_i64)], _i32),
     "tsd_joint_select_noalloc": ([_i32, _i32, _i32, _vp, _vp, _vp, _vp, _vp, _vp], _i32),
+    "tsd_encoder_create": ([_P(EncoderCfgC), _vp, _vp, _vp, _vp, _P(_vp)], _i32),
+    "tsd_encoder_free": ([_vp], None),
+    "tsd_encoder_open": ([_vp, _P(_i32)], _i32),
+    "tsd_encoder_close": ([_vp, _i32], _i32),
+    "tsd_encode_chunk": ([_vp, _i32, _vp, _vp, _i32, _vp, _vp], _i32),
+    "tsd_encoder_check": ([_vp], _i32),
+    "tsd_encoder_set_timing": ([_vp, _i32], _i32),
+    "tsd_encoder_timing": ([_vp, _vp, _vp, _i32, _i32], _i32),
+    "tsd_encoder_gemm_flops": ([_vp, _i32, _i32, _P(ctypes.c_double)], _i32),
 }
 
 _lib = None
@@ -473,3 +498,98 @@ def parse_arpa(text, V: int, vocab: Optional[Sequence[str]] = None):
         return toks, lps, bws, int(skipped.value)
     finally:
         lib().tsd_arpa_free(h)
+
+
+class Encoder:
+    """The cache-aware encoder chunk step on the current CUDA device
+    (``tsd_encoder_create``).  weights: an object with fields cfg (d, layers,
+    heads, ff, kernel, left, chunk, feat, stack), sub_w, sub_b and layers (each
+    with the fields of ``tsd_encoder_layer``; a layer norm as a (gamma, beta)
+    pair named ln_ff1, ln_att, ln_conv, ln_ff2, ln_out), numpy arrays of bf16
+    bit patterns (matrices) and float32 (vectors)."""
+
+    def __init__(self, weights, max_streams: int = 64, max_chunk: Optional[int] = None, stream=None):
+        import torch
+
+        c = weights.cfg
+        self.d, self.stack, self.feat = c.d, c.stack, c.feat
+        self.max_chunk = max_chunk or c.chunk
+        self.cfg = EncoderCfgC(c.d, len(weights.layers), c.heads, c.ff, c.kernel, c.left, self.max_chunk, c.feat,
+                               c.stack, max_streams)
+        dev = torch.device("cuda", torch.cuda.current_device())
+
+        def up(a):
+            a = np.ascontiguousarray(a)
+            if a.dtype == np.uint16:
+                return torch.from_numpy(a.view(np.int16)).to(dev)
+            return torch.from_numpy(a.astype(np.float32)).to(dev)
+
+        keep = [up(weights.sub_w), up(weights.sub_b)]
+        layers = (EncoderLayerC * len(weights.layers))()
+        for i, L in enumerate(weights.layers):
+            vals = {}
+            for name in ("ln_ff1", "ln_att", "ln_conv", "ln_ff2", "ln_out"):
+                g, b = getattr(L, name)
+                vals[name + "_g"], vals[name + "_b"] = up(g), up(b)
+            for name in _ENC_LAYER_FIELDS:
+                if name not in vals:
+                    vals[name] = up(getattr(L, name))
+            keep.extend(vals.values())
+            for name in _ENC_LAYER_FIELDS:
+                setattr(layers[i], name, _ptr(vals[name]))
+        h = _vp()
+        _check(lib().tsd_encoder_create(ctypes.byref(self.cfg), _ptr(keep[0]), _ptr(keep[1]), ctypes.cast(layers, _vp),
+                                        _stream(stream), ctypes.byref(h)))
+        self.h = h  # the encoder copied every weight; the uploads can go
+
+    def __del__(self):
+        if getattr(self, "h", None):
+            lib().tsd_encoder_free(self.h)
+            self.h = None
+
+    def open(self) -> int:
+        s = _i32()
+        _check(lib().tsd_encoder_open(self.h, ctypes.byref(s)))
+        return s.value
+
+    def close(self, slot: int):
+        _check(lib().tsd_encoder_close(self.h, int(slot)))
+
+    def encode_chunk(self, slots: Sequence[int], feats, out=None, stream=None):
+        """feats: cuda bf16 (or int16 bit patterns) [n, C*stack, feat] ->
+        out: cuda int16 (bf16 bit patterns) [n, C, d]."""
+        import torch
+
+        n = len(slots)
+        assert feats.is_cuda and feats.element_size() == 2 and feats.shape[0] == n
+        assert feats.shape[2] == self.feat and feats.shape[1] % self.stack == 0
+        C = feats.shape[1] // self.stack
+        feats = feats.contiguous()
+        if out is None:
+            out = torch.empty((n, C, self.d), dtype=torch.int16, device=feats.device)
+        sl = _i32arr(slots)
+        _check(lib().tsd_encode_chunk(self.h, n, sl.ctypes.data, _ptr(feats), C, _ptr(out), _stream(stream)))
+        return out
+
+    def encode_chunk_raw(self, slots_np: np.ndarray, feats_ptr: int, C: int, out_ptr: int, stream_handle: int):
+        _check(lib().tsd_encode_chunk(self.h, len(slots_np), slots_np.ctypes.data, feats_ptr, C, out_ptr,
+                                      stream_handle))
+
+    def check(self):
+        _check(lib().tsd_encoder_check(self.h))
+
+    def set_timing(self, on: bool):
+        _check(lib().tsd_encoder_set_timing(self.h, 1 if on else 0))
+
+    def timing(self, reset: bool = False):
+        """({'gemm': ms, 'attention': ms, 'other': ms}, {... launches})"""
+        ms = np.zeros(3, dtype=np.float64)
+        ln = np.zeros(3, dtype=np.int64)
+        _check(lib().tsd_encoder_timing(self.h, ms.ctypes.data, ln.ctypes.data, 3, 1 if reset else 0))
+        keys = ("gemm", "attention", "other")
+        return {k: float(ms[i]) for i, k in enumerate(keys)}, {k: int(ln[i]) for i, k in enumerate(keys)}
+
+    def gemm_flops(self, n: int, C: int) -> float:
+        x = ctypes.c_double()
+        _check(lib().tsd_encoder_gemm_flops(self.h, n, C, ctypes.byref(x)))
+        return x.value

@@ -1,0 +1,664 @@
+// The cache-aware encoder chunk step (Sec. III-B: chunked, limited-context
+// attention, causal convolutions and a cache carried across chunks; Sec.
+// IV-A: 80 ms encoder frames, look-ahead = the chunk): host driver and the
+// kernels that are not GEMMs.  See tsd.h for the computation.
+//
+// Per chunk of n streams x C frames (M = n C rows, row b C + t = frame t of
+// the call's stream b), one CUDA graph runs: the subsampling GEMM into the
+// fp32 residual stream x, then per block 15 launches (layer norms, the
+// tensor-core GEMMs of encoder_gemm.cu with their fused epilogues, the
+// attention kernel, the depthwise convolution), then a kernel that advances
+// every stream's frame count.  Caches live per slot in device memory:
+// k and v of the last `left` frames per block and head in a ring indexed by
+// frame position mod left, and the last K-1 GLU outputs per block.
+#include <cuda.h>
+#include <cuda_bf16.h>
+
+#include <algorithm>
+#include <cmath>
+#include <cstring>
+#include <memory>
+
+#include "encoder.h"
+
+namespace tsd {
+
+namespace {
+
+constexpr float kLnEps = 1e-5f;
+
+__device__ __forceinline__ uint16_t f2bf(float v) {
+  const __nv_bfloat16 b = __float2bfloat16_rn(v);
+  return *reinterpret_cast<const uint16_t*>(&b);
+}
+__device__ __forceinline__ float bf2f(uint16_t u) { return __uint_as_float((uint32_t)u << 16); }
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+__device__ __forceinline__ float warp_max(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+  return v;
+}
+
+// Layer norm of rows of the fp32 stream x [M][d] (one warp per row):
+// FINAL = false: y = bf16(LN(x)) (a module's input);
+// FINAL = true:  x = LN(x) in place, and y = bf16(LN(x)) when y != nullptr.
+template <bool FINAL>
+__global__ void __launch_bounds__(256) k_ln(float* x, uint16_t* y, int M, int d, const float* g, const float* b) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int r = blockIdx.x * 8 + warp;
+  if (r >= M) return;
+  float* xr = x + (size_t)r * d;
+  float s = 0.f;
+  for (int c = lane * 4; c < d; c += 128) {
+    const float4 v = *reinterpret_cast<const float4*>(xr + c);
+    s += (v.x + v.y) + (v.z + v.w);
+  }
+  const float mean = warp_sum(s) / (float)d;
+  float q = 0.f;
+  for (int c = lane * 4; c < d; c += 128) {
+    const float4 v = *reinterpret_cast<const float4*>(xr + c);
+    const float a = v.x - mean, bb = v.y - mean, cc = v.z - mean, dd = v.w - mean;
+    q += (a * a + bb * bb) + (cc * cc + dd * dd);
+  }
+  const float rstd = 1.f / sqrtf(warp_sum(q) / (float)d + kLnEps);
+  for (int c = lane * 4; c < d; c += 128) {
+    const float4 v = *reinterpret_cast<const float4*>(xr + c);
+    const float4 gg = *reinterpret_cast<const float4*>(g + c);
+    const float4 be = *reinterpret_cast<const float4*>(b + c);
+    const float o0 = (v.x - mean) * rstd * gg.x + be.x, o1 = (v.y - mean) * rstd * gg.y + be.y;
+    const float o2 = (v.z - mean) * rstd * gg.z + be.z, o3 = (v.w - mean) * rstd * gg.w + be.w;
+    if (FINAL) *reinterpret_cast<float4*>(xr + c) = make_float4(o0, o1, o2, o3);
+    if (y) {
+      uint2 w;
+      w.x = (uint32_t)f2bf(o0) | ((uint32_t)f2bf(o1) << 16);
+      w.y = (uint32_t)f2bf(o2) | ((uint32_t)f2bf(o3) << 16);
+      *reinterpret_cast<uint2*>(y + (size_t)r * d + c) = w;
+    }
+  }
+}
+
+struct AttnArgs {
+  const uint16_t* qkv;    // [M][3d] bf16: q, k, v of the chunk's frames
+  uint16_t* out;          // [M][d] bf16
+  const float* pos_tab;   // [n_off][d] this block's W_pos r(delta), row delta + cmax - 1
+  const float* pu;        // [d] content bias u
+  const float* pv;        // [d] position bias v
+  uint16_t* kc;           // k cache: [slot][layer][head][left][dh]
+  uint16_t* vc;
+  const int32_t* seen;    // frames seen per slot (before this chunk)
+  const int32_t* slots;   // [n]
+  int d, heads, left, layers, layer, C, cmax;
+  float scale;            // 1 / sqrt(dh)
+};
+
+// Shared memory of k_attn for a chunk of C frames (worst case nv = left).
+__host__ __device__ constexpr size_t attn_smem(int dh, int left, int C) {
+  return (size_t)(left + C) * (dh + 2) * 2 /*K*/ + (size_t)(left + C) * dh * 2 /*V*/ +
+         (size_t)2 * C * dh * 4 /*Qu, Qv*/ + (size_t)32 * (dh + 1) * 4 /*P tile*/ +
+         (size_t)C * (left + 2 * C - 1) * 4 /*Sp*/ + (size_t)C * (left + C) * 4 /*S*/;
+}
+
+// One (stream, head) per CTA: chunked, limited-context attention with the
+// relative-position term over the window [cached frames, chunk frames], then
+// the chunk's k and v go into the ring cache.
+template <int DH>
+__global__ void __launch_bounds__(256) k_attn(AttnArgs a) {
+  extern __shared__ __align__(16) unsigned char sm[];
+  const int b = blockIdx.x, h = blockIdx.y, tid = threadIdx.x;
+  const int C = a.C, d = a.d;
+  const int slot = a.slots[b];
+  const int sn = a.seen[slot];
+  const int nv = min(sn, a.left);
+  const int W = nv + C;
+  const int nrel = nv + 2 * C - 1;  // offsets -(C-1) .. nv+C-1
+  const int Wm = a.left + C, nrm = a.left + 2 * C - 1;
+  constexpr int KS = DH + 2;  // padded k row (bf16)
+  uint16_t* Kb = reinterpret_cast<uint16_t*>(sm);
+  uint16_t* Vb = Kb + (size_t)Wm * KS;
+  float* Qu = reinterpret_cast<float*>(Vb + (size_t)Wm * DH);
+  float* Qv = Qu + C * DH;
+  float* Pt = Qv + C * DH;
+  float* Sp = Pt + 32 * (DH + 1);
+  float* S = Sp + C * nrm;
+
+  const size_t cb = (((size_t)slot * a.layers + a.layer) * a.heads + h) * (size_t)a.left * DH;
+  constexpr int P2 = DH / 2;  // bf16 pairs per row
+  for (int idx = tid; idx < nv * P2; idx += blockDim.x) {
+    const int jj = idx / P2, e2 = idx - jj * P2;
+    const int ring = (sn - nv + jj) % a.left;
+    const uint32_t kw = reinterpret_cast<const uint32_t*>(a.kc + cb + (size_t)ring * DH)[e2];
+    const uint32_t vw = reinterpret_cast<const uint32_t*>(a.vc + cb + (size_t)ring * DH)[e2];
+    reinterpret_cast<uint32_t*>(Kb + (size_t)jj * KS)[e2] = kw;
+    reinterpret_cast<uint32_t*>(Vb + (size_t)jj * DH)[e2] = vw;
+  }
+  for (int idx = tid; idx < C * P2; idx += blockDim.x) {
+    const int i = idx / P2, e2 = idx - i * P2;
+    const uint16_t* row = a.qkv + (size_t)(b * C + i) * 3 * d + h * DH;
+    const uint32_t qw = reinterpret_cast<const uint32_t*>(row)[e2];
+    reinterpret_cast<uint32_t*>(Kb + (size_t)(nv + i) * KS)[e2] = reinterpret_cast<const uint32_t*>(row + d)[e2];
+    reinterpret_cast<uint32_t*>(Vb + (size_t)(nv + i) * DH)[e2] = reinterpret_cast<const uint32_t*>(row + 2 * d)[e2];
+    const float q0 = __uint_as_float(qw << 16), q1 = __uint_as_float(qw & 0xffff0000u);
+    const int c = h * DH + 2 * e2;
+    Qu[i * DH + 2 * e2] = q0 + a.pu[c];
+    Qu[i * DH + 2 * e2 + 1] = q1 + a.pu[c + 1];
+    Qv[i * DH + 2 * e2] = q0 + a.pv[c];
+    Qv[i * DH + 2 * e2 + 1] = q1 + a.pv[c + 1];
+  }
+  __syncthreads();
+  // the cache was read above: the chunk's k and v replace the oldest frames
+  if (a.left > 0) {
+    for (int idx = tid; idx < C * P2; idx += blockDim.x) {
+      const int i = idx / P2, e2 = idx - i * P2;
+      if (i < C - a.left) continue;
+      const int ring = (sn + i) % a.left;
+      const uint16_t* row = a.qkv + (size_t)(b * C + i) * 3 * d + h * DH;
+      reinterpret_cast<uint32_t*>(a.kc + cb + (size_t)ring * DH)[e2] = reinterpret_cast<const uint32_t*>(row + d)[e2];
+      reinterpret_cast<uint32_t*>(a.vc + cb + (size_t)ring * DH)[e2] =
+          reinterpret_cast<const uint32_t*>(row + 2 * d)[e2];
+    }
+  }
+  // position scores Sp[i][t] = (q_i + v) . p(t - (C-1)), 32 table rows at a time
+  for (int t0 = 0; t0 < nrel; t0 += 32) {
+    for (int idx = tid; idx < 32 * DH; idx += blockDim.x) {
+      const int tt = idx / DH, e = idx - tt * DH;
+      const int t = t0 + tt;
+      Pt[tt * (DH + 1) + e] = t < nrel ? a.pos_tab[(size_t)(t + a.cmax - C) * d + h * DH + e] : 0.f;
+    }
+    __syncthreads();
+    for (int idx = tid; idx < C * 32; idx += blockDim.x) {
+      const int i = idx >> 5, tt = idx & 31;
+      if (t0 + tt >= nrel) continue;
+      const float* qv = Qv + i * DH;
+      const float* p = Pt + tt * (DH + 1);
+      float acc = 0.f;
+#pragma unroll 16
+      for (int e = 0; e < DH; ++e) acc = fmaf(qv[e], p[e], acc);
+      Sp[i * nrm + t0 + tt] = acc;
+    }
+    __syncthreads();
+  }
+  // scores: content + position, scaled
+  for (int idx = tid; idx < C * W; idx += blockDim.x) {
+    const int i = idx / W, jj = idx - i * W;
+    const float* qu = Qu + i * DH;
+    const uint32_t* kr = reinterpret_cast<const uint32_t*>(Kb + (size_t)jj * KS);
+    float acc = 0.f;
+#pragma unroll 16
+    for (int e2 = 0; e2 < P2; ++e2) {
+      const uint32_t w = kr[e2];
+      acc = fmaf(qu[2 * e2], __uint_as_float(w << 16), acc);
+      acc = fmaf(qu[2 * e2 + 1], __uint_as_float(w & 0xffff0000u), acc);
+    }
+    S[i * Wm + jj] = (acc + Sp[i * nrm + (i - jj + nv + C - 1)]) * a.scale;
+  }
+  __syncthreads();
+  // softmax per query row (one warp per row)
+  {
+    const int warp = tid >> 5, lane = tid & 31;
+    for (int i = warp; i < C; i += blockDim.x >> 5) {
+      float* s = S + i * Wm;
+      float m = -INFINITY;
+      for (int j = lane; j < W; j += 32) m = fmaxf(m, s[j]);
+      m = warp_max(m);
+      float z = 0.f;
+      for (int j = lane; j < W; j += 32) {
+        const float e = expf(s[j] - m);
+        s[j] = e;
+        z += e;
+      }
+      z = warp_sum(z);
+      const float inv = 1.f / z;
+      for (int j = lane; j < W; j += 32) s[j] *= inv;
+    }
+  }
+  __syncthreads();
+  for (int idx = tid; idx < C * DH; idx += blockDim.x) {
+    const int i = idx / DH, e = idx - i * DH;
+    const float* s = S + i * Wm;
+    float acc = 0.f;
+    for (int jj = 0; jj < W; ++jj) acc = fmaf(s[jj], bf2f(Vb[(size_t)jj * DH + e]), acc);
+    a.out[(size_t)(b * C + i) * d + h * DH + e] = f2bf(acc);
+  }
+}
+
+struct ConvArgs {
+  const uint16_t* glu;  // [M][d]
+  uint16_t* z;          // [M][d]
+  uint16_t* cache;      // [slot][layer][K-1][d]
+  const float *w, *bias, *sc, *sh;
+  const int32_t* slots;
+  int d, K, C, layers, layer;
+};
+
+// Causal depthwise convolution over [cached K-1 frames, chunk frames], the
+// batch-norm affine map and Swish; thread = channel.  The last K-1 frames of
+// the window become the cache.
+__global__ void __launch_bounds__(128) k_dwconv(ConvArgs a) {
+  extern __shared__ float seq[];  // [K-1+C][128]
+  const int b = blockIdx.x, c = blockIdx.y * 128 + threadIdx.x, tid = threadIdx.x;
+  const int K1 = a.K - 1, C = a.C, d = a.d;
+  const int slot = a.slots[b];
+  uint16_t* cc = a.cache + ((size_t)slot * a.layers + a.layer) * (size_t)K1 * d;
+  for (int t = 0; t < K1; ++t) seq[t * 128 + tid] = bf2f(cc[(size_t)t * d + c]);
+  for (int t = 0; t < C; ++t) seq[(K1 + t) * 128 + tid] = bf2f(a.glu[(size_t)(b * C + t) * d + c]);
+  const float* w = a.w + (size_t)c * a.K;
+  const float bias = a.bias[c], sc = a.sc[c], sh = a.sh[c];
+  for (int t = 0; t < C; ++t) {
+    float acc = 0.f;
+    for (int k = 0; k < a.K; ++k) acc = fmaf(w[k], seq[(t + k) * 128 + tid], acc);
+    const float y = (acc + bias) * sc + sh;
+    a.z[(size_t)(b * C + t) * d + c] = f2bf(y / (1.f + expf(-y)));
+  }
+  for (int t = 0; t < K1; ++t) cc[(size_t)t * d + c] = f2bf(seq[(C + t) * 128 + tid]);
+}
+
+// P[row][c] = sum_k W_pos[c][k] r_k(delta), delta = row - (cmax - 1), r the
+// sinusoidal code (sin at 2j, cos at 2j+1 of delta / 10000^(2j/d)); computed
+// in double once at create.
+__global__ void k_pos_table(const uint16_t* pos_w, float* tab, int d, int cmax) {
+  extern __shared__ double r[];
+  const double delta = (double)((int)blockIdx.x - (cmax - 1));
+  for (int k = threadIdx.x; k < d; k += blockDim.x) {
+    const double w = pow(10000.0, -2.0 * (double)(k / 2) / (double)d);
+    r[k] = (k & 1) ? cos(delta * w) : sin(delta * w);
+  }
+  __syncthreads();
+  for (int c = threadIdx.x; c < d; c += blockDim.x) {
+    const uint16_t* wr = pos_w + (size_t)c * d;
+    double acc = 0.0;
+    for (int k = 0; k < d; ++k) acc += (double)bf2f(wr[k]) * r[k];
+    tab[(size_t)blockIdx.x * d + c] = (float)acc;
+  }
+}
+
+// W_pw1 [2d][d] -> rows interleaved in groups of 32: output group p's value
+// rows, then its gate rows (the GLU epilogue finds both in one tile).
+__global__ void k_glu_repack(const uint16_t* src, const float* bsrc, uint16_t* dst, float* bdst, int d) {
+  const int r = blockIdx.x;  // destination row
+  const int p = r / 64, w = r % 64;
+  const int s = w < 32 ? 32 * p + w : d + 32 * p + (w - 32);
+  for (int k = threadIdx.x; k < d; k += blockDim.x) dst[(size_t)r * d + k] = src[(size_t)s * d + k];
+  if (threadIdx.x == 0) bdst[r] = bsrc[s];
+}
+
+__global__ void k_advance(int32_t* seen, const int32_t* slots, int n, int C) {
+  for (int b = threadIdx.x; b < n; b += blockDim.x) seen[slots[b]] += C;
+}
+
+tsd_status set_device(tsd_encoder* e) {
+  int cur = -1;
+  TSD_CUDA(cudaGetDevice(&cur));
+  if (cur != e->device) TSD_CUDA(cudaSetDevice(e->device));
+  return TSD_OK;
+}
+
+int n_marks(const tsd_encoder* e) { return 1 + 15 * e->cfg.layers + 1 + 1; }
+
+void launch_attn(const tsd_encoder* e, const AttnArgs& a, int n, cudaStream_t s) {
+  const size_t sm = attn_smem(e->cfg.d / e->cfg.heads, e->cfg.left, a.C);
+  dim3 grid(n, e->cfg.heads);
+  if (e->cfg.d / e->cfg.heads == 64) k_attn<64><<<grid, 256, sm, s>>>(a);
+  else k_attn<128><<<grid, 256, sm, s>>>(a);
+}
+
+void enqueue(tsd_encoder* e, int n, int C, cudaStream_t s, const std::vector<cudaEvent_t>* ev,
+             std::vector<int8_t>* cls) {
+  const tsd_encoder_cfg& c = e->cfg;
+  const int M = n * C, d = c.d;
+  int mk = 0;
+  auto mark = [&](int k) {
+    if (!ev) return;
+    cudaEventRecordWithFlags((*ev)[(size_t)mk], s, cudaEventRecordExternal);
+    if (cls) (*cls)[(size_t)mk] = (int8_t)k;
+    ++mk;
+  };
+  const dim3 ln_grid((M + 7) / 8);
+  auto gemm = [&](int epi, const CUtensorMap& A, const CUtensorMap& B, int N, int K, const float* bias, void* out,
+                  int ld, float alpha) {
+    mark(0);
+    EGemm g{M, N, K, bias, out, ld, alpha, e->err};
+    launch_egemm(epi, g, A, B, s);
+  };
+  gemm(kEInit, e->m_feat, e->m_sub, d, c.stack * c.feat, e->sub_b, e->x, d, 1.f);
+  for (int l = 0; l < c.layers; ++l) {
+    EncLayerDev& L = e->L[(size_t)l];
+    mark(2);
+    k_ln<false><<<ln_grid, 256, 0, s>>>(e->x, e->nrm, M, d, L.ln_ff1_g, L.ln_ff1_b);
+    gemm(kESwish, e->m_nrm, L.m_ff1_w1, c.ff, d, L.ff1_b1, e->hid, c.ff, 1.f);
+    gemm(kEResid, e->m_hid, L.m_ff1_w2, d, c.ff, L.ff1_b2, e->x, d, 0.5f);
+    mark(2);
+    k_ln<false><<<ln_grid, 256, 0, s>>>(e->x, e->nrm, M, d, L.ln_att_g, L.ln_att_b);
+    gemm(kEPlain, e->m_nrm, L.m_qkv, 3 * d, d, L.qkv_b, e->qkv, 3 * d, 1.f);
+    mark(1);
+    AttnArgs aa{e->qkv, e->att, L.pos_tab, L.pos_u, L.pos_v, e->kc, e->vc, e->seen, e->slots_dev,
+                d, c.heads, c.left, c.layers, l, C, c.max_chunk, 1.f / sqrtf((float)(d / c.heads))};
+    launch_attn(e, aa, n, s);
+    gemm(kEResid, e->m_att, L.m_out, d, d, L.out_b, e->x, d, 1.f);
+    mark(2);
+    k_ln<false><<<ln_grid, 256, 0, s>>>(e->x, e->nrm, M, d, L.ln_conv_g, L.ln_conv_b);
+    gemm(kEGlu, e->m_nrm, L.m_pw1, 2 * d, d, L.pw1_b, e->glu, d, 1.f);
+    mark(2);
+    ConvArgs ca{e->glu, e->convz, e->cc, L.dw_w, L.dw_b, L.bn_scale, L.bn_shift, e->slots_dev, d, c.kernel, C,
+                c.layers, l};
+    k_dwconv<<<dim3(n, d / 128), 128, (size_t)(c.kernel - 1 + C) * 128 * sizeof(float), s>>>(ca);
+    gemm(kEResid, e->m_convz, L.m_pw2, d, d, L.pw2_b, e->x, d, 1.f);
+    mark(2);
+    k_ln<false><<<ln_grid, 256, 0, s>>>(e->x, e->nrm, M, d, L.ln_ff2_g, L.ln_ff2_b);
+    gemm(kESwish, e->m_nrm, L.m_ff2_w1, c.ff, d, L.ff2_b1, e->hid, c.ff, 1.f);
+    gemm(kEResid, e->m_hid, L.m_ff2_w2, d, c.ff, L.ff2_b2, e->x, d, 0.5f);
+    mark(2);
+    k_ln<true><<<ln_grid, 256, 0, s>>>(e->x, l + 1 == c.layers ? e->outb : nullptr, M, d, L.ln_out_g, L.ln_out_b);
+  }
+  mark(2);
+  k_advance<<<1, 256, 0, s>>>(e->seen, e->slots_dev, n, C);
+  mark(-1);
+}
+
+void harvest(tsd_encoder* e, tsd_encoder::Graph& g) {
+  if (!g.pending) return;
+  cudaEventSynchronize(g.ev.back());
+  for (size_t i = 0; i + 1 < g.ev.size(); ++i) {
+    float ms = 0.f;
+    const int k = g.cls[i];
+    if (k >= 0 && k < 3 && cudaEventElapsedTime(&ms, g.ev[i], g.ev[i + 1]) == cudaSuccess) {
+      e->ms[k] += ms;
+      e->launches[k] += 1;
+    }
+  }
+  cudaGetLastError();
+  g.pending = false;
+}
+
+tsd_status copy_dev(tsd::DevArena& A, uint16_t** dst, const void* src, size_t n, cudaStream_t s) {
+  tsd_status st = A.alloc(dst, n);
+  if (st) return st;
+  TSD_CUDA(cudaMemcpyAsync(*dst, src, n * 2, cudaMemcpyDeviceToDevice, s));
+  return TSD_OK;
+}
+
+tsd_status copy_dev(tsd::DevArena& A, float** dst, const float* src, size_t n, cudaStream_t s) {
+  tsd_status st = A.alloc(dst, n);
+  if (st) return st;
+  TSD_CUDA(cudaMemcpyAsync(*dst, src, n * 4, cudaMemcpyDeviceToDevice, s));
+  return TSD_OK;
+}
+
+size_t round_up(size_t x, size_t m) { return (x + m - 1) / m * m; }
+
+}  // namespace
+
+}  // namespace tsd
+
+using namespace tsd;
+
+extern "C" tsd_status tsd_encoder_create(const tsd_encoder_cfg* cfg, const void* sub_w, const float* sub_b,
+                                         const tsd_encoder_layer* layers, void* cuda_stream, tsd_encoder** out) {
+  clear_error();
+  if (!cfg || !sub_w || !sub_b || !layers || !out) return fail(TSD_EINVAL, "tsd_encoder_create: NULL argument");
+  const tsd_encoder_cfg c = *cfg;
+  if (c.d < 128 || c.d > 2048 || c.d % 128) return fail(TSD_EINVAL, "tsd_encoder_create: d=%d", c.d);
+  if (c.heads < 1 || c.d % c.heads || (c.d / c.heads != 64 && c.d / c.heads != 128))
+    return fail(TSD_EINVAL, "tsd_encoder_create: d/heads must be 64 or 128 (d=%d heads=%d)", c.d, c.heads);
+  if (c.ff < 128 || c.ff > 8192 || c.ff % 128) return fail(TSD_EINVAL, "tsd_encoder_create: ff=%d", c.ff);
+  if (c.layers < 1 || c.layers > 64) return fail(TSD_EINVAL, "tsd_encoder_create: layers=%d", c.layers);
+  if (c.kernel < 1 || c.kernel > 32) return fail(TSD_EINVAL, "tsd_encoder_create: kernel=%d", c.kernel);
+  if (c.left < 0 || c.left > 128) return fail(TSD_EINVAL, "tsd_encoder_create: left=%d", c.left);
+  if (c.max_chunk < 1 || c.max_chunk > 32) return fail(TSD_EINVAL, "tsd_encoder_create: max_chunk=%d", c.max_chunk);
+  if (c.feat < 1 || c.stack < 1 || (c.stack * c.feat) % 64 || c.stack * c.feat > 8192)
+    return fail(TSD_EINVAL, "tsd_encoder_create: stack*feat=%d must be a multiple of 64, <= 8192", c.stack * c.feat);
+  if (c.max_streams < 1 || c.max_streams > 4096)
+    return fail(TSD_EINVAL, "tsd_encoder_create: max_streams=%d", c.max_streams);
+  for (int l = 0; l < c.layers; ++l) {
+    const tsd_encoder_layer& L = layers[l];
+    const void* ptrs[] = {L.ln_ff1_g, L.ln_ff1_b, L.ff1_w1, L.ff1_b1, L.ff1_w2, L.ff1_b2, L.ln_att_g, L.ln_att_b,
+                          L.qkv_w, L.qkv_b, L.pos_w, L.pos_u, L.pos_v, L.out_w, L.out_b, L.ln_conv_g, L.ln_conv_b,
+                          L.pw1_w, L.pw1_b, L.dw_w, L.dw_b, L.bn_scale, L.bn_shift, L.pw2_w, L.pw2_b, L.ln_ff2_g,
+                          L.ln_ff2_b, L.ff2_w1, L.ff2_b1, L.ff2_w2, L.ff2_b2, L.ln_out_g, L.ln_out_b};
+    for (const void* p : ptrs)
+      if (!p) return fail(TSD_EINVAL, "tsd_encoder_create: layer %d has a NULL weight", l);
+  }
+  std::unique_ptr<tsd_encoder> e(new tsd_encoder());
+  e->cfg = c;
+  TSD_CUDA(cudaGetDevice(&e->device));
+  cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
+  e->last_stream = s;
+  TSD_CUDA(egemm_prepare());
+  const int d = c.d, ff = c.ff, K1 = c.kernel - 1, dh = d / c.heads;
+  const size_t asm_ = attn_smem(dh, c.left, c.max_chunk);
+  if (asm_ > 227 * 1024) return fail(TSD_EINVAL, "tsd_encoder_create: attention window too large");
+  if (dh == 64) TSD_CUDA(cudaFuncSetAttribute(k_attn<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)asm_));
+  else TSD_CUDA(cudaFuncSetAttribute(k_attn<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)asm_));
+  e->n_off = c.left + 2 * c.max_chunk - 1;
+  e->M_pad = (int)round_up((size_t)c.max_streams * c.max_chunk, 128);
+  DevArena& A = e->arena;
+  tsd_status st;
+  if ((st = copy_dev(A, &e->sub_w, sub_w, (size_t)d * c.stack * c.feat, s)) || (st = copy_dev(A, &e->sub_b, sub_b, d, s)))
+    return st;
+  e->L.resize((size_t)c.layers);
+  for (int l = 0; l < c.layers; ++l) {
+    const tsd_encoder_layer& W = layers[l];
+    EncLayerDev& L = e->L[(size_t)l];
+    float *g[10];
+    const float* gs[10] = {W.ln_ff1_g, W.ln_ff1_b, W.ln_att_g, W.ln_att_b, W.ln_conv_g,
+                           W.ln_conv_b, W.ln_ff2_g, W.ln_ff2_b, W.ln_out_g, W.ln_out_b};
+    for (int i = 0; i < 10; ++i)
+      if ((st = copy_dev(A, &g[i], gs[i], d, s))) return st;
+    L.ln_ff1_g = g[0], L.ln_ff1_b = g[1], L.ln_att_g = g[2], L.ln_att_b = g[3], L.ln_conv_g = g[4];
+    L.ln_conv_b = g[5], L.ln_ff2_g = g[6], L.ln_ff2_b = g[7], L.ln_out_g = g[8], L.ln_out_b = g[9];
+    if ((st = copy_dev(A, &L.ff1_w1, W.ff1_w1, (size_t)ff * d, s)) || (st = copy_dev(A, &L.ff1_b1, W.ff1_b1, ff, s)) ||
+        (st = copy_dev(A, &L.ff1_w2, W.ff1_w2, (size_t)d * ff, s)) || (st = copy_dev(A, &L.ff1_b2, W.ff1_b2, d, s)) ||
+        (st = copy_dev(A, &L.qkv_w, W.qkv_w, (size_t)3 * d * d, s)) || (st = copy_dev(A, &L.qkv_b, W.qkv_b, 3 * d, s)) ||
+        (st = copy_dev(A, &L.pos_w, W.pos_w, (size_t)d * d, s)) || (st = copy_dev(A, &L.pos_u, W.pos_u, d, s)) ||
+        (st = copy_dev(A, &L.pos_v, W.pos_v, d, s)) || (st = copy_dev(A, &L.out_w, W.out_w, (size_t)d * d, s)) ||
+        (st = copy_dev(A, &L.out_b, W.out_b, d, s)) || (st = A.alloc(&L.pw1_w, (size_t)2 * d * d)) ||
+        (st = A.alloc(&L.pw1_b, (size_t)2 * d)) || (st = copy_dev(A, &L.dw_w, W.dw_w, (size_t)d * c.kernel, s)) ||
+        (st = copy_dev(A, &L.dw_b, W.dw_b, d, s)) || (st = copy_dev(A, &L.bn_scale, W.bn_scale, d, s)) ||
+        (st = copy_dev(A, &L.bn_shift, W.bn_shift, d, s)) || (st = copy_dev(A, &L.pw2_w, W.pw2_w, (size_t)d * d, s)) ||
+        (st = copy_dev(A, &L.pw2_b, W.pw2_b, d, s)) || (st = copy_dev(A, &L.ff2_w1, W.ff2_w1, (size_t)ff * d, s)) ||
+        (st = copy_dev(A, &L.ff2_b1, W.ff2_b1, ff, s)) || (st = copy_dev(A, &L.ff2_w2, W.ff2_w2, (size_t)d * ff, s)) ||
+        (st = copy_dev(A, &L.ff2_b2, W.ff2_b2, d, s)) || (st = A.alloc(&L.pos_tab, (size_t)e->n_off * d)))
+      return st;
+    k_glu_repack<<<2 * d, 128, 0, s>>>(static_cast<const uint16_t*>(W.pw1_w), W.pw1_b, L.pw1_w, L.pw1_b, d);
+    k_pos_table<<<e->n_off, 256, (size_t)d * sizeof(double), s>>>(L.pos_w, L.pos_tab, d, c.max_chunk);
+    TSD_CUDA(cudaGetLastError());
+    if (!egemm_map_b(&L.m_ff1_w1, L.ff1_w1, ff, d) || !egemm_map_b(&L.m_ff1_w2, L.ff1_w2, d, ff) ||
+        !egemm_map_b(&L.m_qkv, L.qkv_w, 3 * d, d) || !egemm_map_b(&L.m_out, L.out_w, d, d) ||
+        !egemm_map_b(&L.m_pw1, L.pw1_w, 2 * d, d) || !egemm_map_b(&L.m_pw2, L.pw2_w, d, d) ||
+        !egemm_map_b(&L.m_ff2_w1, L.ff2_w1, ff, d) || !egemm_map_b(&L.m_ff2_w2, L.ff2_w2, d, ff))
+      return fail(TSD_ECUDA, "tsd_encoder_create: tensor map encoding failed");
+  }
+  const size_t Mp = (size_t)e->M_pad, SF = (size_t)c.stack * c.feat;
+  if ((st = A.alloc(&e->feat, Mp * SF)) || (st = A.alloc(&e->x, Mp * d)) || (st = A.alloc(&e->nrm, Mp * d)) ||
+      (st = A.alloc(&e->hid, Mp * ff)) || (st = A.alloc(&e->qkv, Mp * 3 * d)) || (st = A.alloc(&e->att, Mp * d)) ||
+      (st = A.alloc(&e->glu, Mp * d)) || (st = A.alloc(&e->convz, Mp * d)) || (st = A.alloc(&e->outb, Mp * d)))
+    return st;
+  const size_t kv = (size_t)c.max_streams * c.layers * c.left * d;
+  const size_t cv = (size_t)c.max_streams * c.layers * std::max(K1, 1) * d;
+  if ((st = A.alloc(&e->kc, std::max<size_t>(kv, 1))) || (st = A.alloc(&e->vc, std::max<size_t>(kv, 1))) ||
+      (st = A.alloc(&e->cc, cv)) || (st = A.alloc(&e->seen, (size_t)c.max_streams)) ||
+      (st = A.alloc(&e->slots_dev, (size_t)c.max_streams)) || (st = A.alloc(&e->err, 1)))
+    return st;
+  TSD_CUDA(cudaMemsetAsync(e->kc, 0, std::max<size_t>(kv, 1) * 2, s));
+  TSD_CUDA(cudaMemsetAsync(e->vc, 0, std::max<size_t>(kv, 1) * 2, s));
+  TSD_CUDA(cudaMemsetAsync(e->cc, 0, cv * 2, s));
+  TSD_CUDA(cudaMemsetAsync(e->seen, 0, (size_t)c.max_streams * 4, s));
+  TSD_CUDA(cudaMemsetAsync(e->err, 0, 4, s));
+  TSD_CUDA(cudaMemsetAsync(e->feat, 0, Mp * SF * 2, s));
+  TSD_CUDA(cudaMemsetAsync(e->nrm, 0, Mp * d * 2, s));
+  TSD_CUDA(cudaMemsetAsync(e->hid, 0, Mp * ff * 2, s));
+  TSD_CUDA(cudaMemsetAsync(e->att, 0, Mp * d * 2, s));
+  TSD_CUDA(cudaMemsetAsync(e->convz, 0, Mp * d * 2, s));
+  if (!egemm_map_a(&e->m_feat, e->feat, e->M_pad, (int)SF) || !egemm_map_a(&e->m_nrm, e->nrm, e->M_pad, d) ||
+      !egemm_map_a(&e->m_hid, e->hid, e->M_pad, ff) || !egemm_map_a(&e->m_att, e->att, e->M_pad, d) ||
+      !egemm_map_a(&e->m_convz, e->convz, e->M_pad, d) || !egemm_map_b(&e->m_sub, e->sub_w, d, (int)SF))
+    return fail(TSD_ECUDA, "tsd_encoder_create: tensor map encoding failed");
+  TSD_CUDA(cudaMallocHost(&e->slots_host, sizeof(int32_t) * (size_t)c.max_streams));
+  TSD_CUDA(cudaEventCreateWithFlags(&e->slots_ev, cudaEventDisableTiming));
+  TSD_CUDA(cudaStreamCreateWithFlags(&e->cap_stream, cudaStreamNonBlocking));
+  TSD_CUDA(cudaStreamSynchronize(s));
+  TSD_CUDA(cudaGetLastError());
+  e->slot_open.assign((size_t)c.max_streams, 0);
+  *out = e.release();
+  return TSD_OK;
+}
+
+extern "C" void tsd_encoder_free(tsd_encoder* e) {
+  if (!e) return;
+  set_device(e);
+  cudaDeviceSynchronize();
+  for (auto& kv : e->graphs) {
+    if (kv.second.exec) cudaGraphExecDestroy(kv.second.exec);
+    for (cudaEvent_t ev : kv.second.ev) cudaEventDestroy(ev);
+  }
+  if (e->slots_host) cudaFreeHost(e->slots_host);
+  if (e->slots_ev) cudaEventDestroy(e->slots_ev);
+  if (e->cap_stream) cudaStreamDestroy(e->cap_stream);
+  e->arena.release();
+  cudaGetLastError();
+  delete e;
+}
+
+extern "C" tsd_status tsd_encoder_open(tsd_encoder* e, int32_t* slot_out) {
+  clear_error();
+  if (!e || !slot_out) return fail(TSD_EINVAL, "tsd_encoder_open: NULL argument");
+  auto it = std::find(e->slot_open.begin(), e->slot_open.end(), 0);
+  if (it == e->slot_open.end()) return fail(TSD_ESTATE, "tsd_encoder_open: all %d slots are open", e->cfg.max_streams);
+  tsd_status st = set_device(e);
+  if (st) return st;
+  const int slot = (int)(it - e->slot_open.begin());
+  const tsd_encoder_cfg& c = e->cfg;
+  const size_t kv = (size_t)c.layers * c.left * c.d, cv = (size_t)c.layers * (c.kernel - 1) * c.d;
+  cudaStream_t s = e->last_stream;
+  if (kv) {
+    TSD_CUDA(cudaMemsetAsync(e->kc + (size_t)slot * kv, 0, kv * 2, s));
+    TSD_CUDA(cudaMemsetAsync(e->vc + (size_t)slot * kv, 0, kv * 2, s));
+  }
+  if (cv) TSD_CUDA(cudaMemsetAsync(e->cc + (size_t)slot * cv, 0, cv * 2, s));
+  TSD_CUDA(cudaMemsetAsync(e->seen + slot, 0, 4, s));
+  *it = 1;
+  *slot_out = slot;
+  return TSD_OK;
+}
+
+extern "C" tsd_status tsd_encoder_close(tsd_encoder* e, int32_t slot) {
+  clear_error();
+  if (!e) return fail(TSD_EINVAL, "tsd_encoder_close: NULL encoder");
+  if (slot < 0 || slot >= e->cfg.max_streams || !e->slot_open[(size_t)slot])
+    return fail(TSD_ESTATE, "tsd_encoder_close: slot %d is not open", slot);
+  e->slot_open[(size_t)slot] = 0;
+  return TSD_OK;
+}
+
+extern "C" tsd_status tsd_encode_chunk(tsd_encoder* e, int32_t n, const int32_t* slots, const void* feats_bf16,
+                                       int32_t C, void* out_bf16, void* cuda_stream) {
+  clear_error();
+  if (!e || !slots || !feats_bf16 || !out_bf16) return fail(TSD_EINVAL, "tsd_encode_chunk: NULL argument");
+  const tsd_encoder_cfg& c = e->cfg;
+  if (n < 1 || n > c.max_streams) return fail(TSD_EINVAL, "tsd_encode_chunk: n=%d out of [1, %d]", n, c.max_streams);
+  if (C < 1 || C > c.max_chunk) return fail(TSD_EINVAL, "tsd_encode_chunk: C=%d out of [1, %d]", C, c.max_chunk);
+  {
+    std::vector<uint8_t> seen((size_t)c.max_streams, 0);
+    for (int i = 0; i < n; ++i) {
+      const int s = slots[i];
+      if (s < 0 || s >= c.max_streams || !e->slot_open[(size_t)s])
+        return fail(TSD_ESTATE, "tsd_encode_chunk: slot %d is not open", s);
+      if (seen[(size_t)s]) return fail(TSD_EINVAL, "tsd_encode_chunk: slot %d listed twice", s);
+      seen[(size_t)s] = 1;
+    }
+  }
+  tsd_status st = set_device(e);
+  if (st) return st;
+  cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
+  e->last_stream = s;
+  TSD_CUDA(cudaEventSynchronize(e->slots_ev));
+  std::memcpy(e->slots_host, slots, sizeof(int32_t) * (size_t)n);
+  TSD_CUDA(cudaMemcpyAsync(e->slots_dev, e->slots_host, sizeof(int32_t) * (size_t)n, cudaMemcpyHostToDevice, s));
+  TSD_CUDA(cudaEventRecord(e->slots_ev, s));
+  const size_t M = (size_t)n * C;
+  TSD_CUDA(cudaMemcpyAsync(e->feat, feats_bf16, M * c.stack * c.feat * 2, cudaMemcpyDeviceToDevice, s));
+  auto key = std::make_pair(std::make_pair(n, C), e->timing);
+  tsd_encoder::Graph& g = e->graphs[key];
+  if (e->timing) {
+    harvest(e, g);
+    if (g.ev.empty()) {
+      g.ev.resize((size_t)n_marks(e));
+      g.cls.assign(g.ev.size(), -1);
+      for (auto& ev : g.ev) TSD_CUDA(cudaEventCreate(&ev));
+    }
+  }
+  if (!g.exec) {
+    cudaGraph_t gr = nullptr;
+    TSD_CUDA(cudaStreamBeginCapture(e->cap_stream, cudaStreamCaptureModeThreadLocal));
+    enqueue(e, n, C, e->cap_stream, e->timing ? &g.ev : nullptr, e->timing ? &g.cls : nullptr);
+    cudaError_t ce = cudaStreamEndCapture(e->cap_stream, &gr);
+    if (ce != cudaSuccess) return cuda_fail(ce, "tsd_encode_chunk: graph capture");
+    ce = cudaGraphInstantiate(&g.exec, gr, 0);
+    cudaGraphDestroy(gr);
+    if (ce != cudaSuccess) {
+      g.exec = nullptr;
+      return cuda_fail(ce, "tsd_encode_chunk: graph instantiate");
+    }
+  }
+  TSD_CUDA(cudaGraphLaunch(g.exec, s));
+  if (e->timing) g.pending = true;
+  TSD_CUDA(cudaMemcpyAsync(out_bf16, e->outb, M * c.d * 2, cudaMemcpyDeviceToDevice, s));
+  return TSD_OK;
+}
+
+extern "C" tsd_status tsd_encoder_check(tsd_encoder* e) {
+  clear_error();
+  if (!e) return fail(TSD_EINVAL, "tsd_encoder_check: NULL encoder");
+  tsd_status st = set_device(e);
+  if (st) return st;
+  TSD_CUDA(cudaStreamSynchronize(e->last_stream));
+  unsigned int v = 0;
+  TSD_CUDA(cudaMemcpy(&v, e->err, 4, cudaMemcpyDeviceToHost));
+  if (v) {
+    TSD_CUDA(cudaMemset(e->err, 0, 4));
+    return fail(TSD_EDEVICE, "tsd_encoder_check: a bounded wait expired in the encoder GEMM (code %u)", v);
+  }
+  return TSD_OK;
+}
+
+extern "C" tsd_status tsd_encoder_set_timing(tsd_encoder* e, int32_t enable) {
+  clear_error();
+  if (!e) return fail(TSD_EINVAL, "tsd_encoder_set_timing: NULL encoder");
+  e->timing = enable ? 1 : 0;
+  return TSD_OK;
+}
+
+extern "C" tsd_status tsd_encoder_timing(tsd_encoder* e, double* ms, int64_t* launches, int32_t n_classes,
+                                         int32_t reset) {
+  clear_error();
+  if (!e) return fail(TSD_EINVAL, "tsd_encoder_timing: NULL encoder");
+  tsd_status st = set_device(e);
+  if (st) return st;
+  for (auto& kv : e->graphs) harvest(e, kv.second);
+  for (int i = 0; i < n_classes && i < 3; ++i) {
+    if (ms) ms[i] = e->ms[i];
+    if (launches) launches[i] = e->launches[i];
+  }
+  if (reset)
+    for (int i = 0; i < 3; ++i) {
+      e->ms[i] = 0;
+      e->launches[i] = 0;
+    }
+  return TSD_OK;
+}
+
+extern "C" tsd_status tsd_encoder_gemm_flops(const tsd_encoder* e, int32_t n, int32_t C, double* flops) {
+  clear_error();
+  if (!e || !flops) return fail(TSD_EINVAL, "tsd_encoder_gemm_flops: NULL argument");
+  const tsd_encoder_cfg& c = e->cfg;
+  const double M = (double)n * C, d = c.d, ff = c.ff;
+  // subsampling; per block q/k/v (3d^2), output (d^2), GLU pointwise (2d^2), pointwise (d^2), two
+  // feed-forward halves (2 x 2 ff d)
+  *flops = 2.0 * M * d * c.stack * c.feat + c.layers * 2.0 * M * (7.0 * d * d + 4.0 * ff * d);
+  return TSD_OK;
+}
