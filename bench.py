@@ -216,6 +216,12 @@ def variant_config(args, w, extra):
     if args.pred:
         out["prediction_network"] = {"kind": "1-layer LSTM over the previous label", "D": args.pred, "H_enc": w.H}
         names.append(f"stateful form: LSTM prediction network D={args.pred} + joint projections")
+    if args.encoder:
+        e = synth.ENCODERS[args.encoder]
+        out["encoder"] = {"shape": e.name, "d": e.d, "blocks": e.layers, "heads": e.heads, "ff": e.ff,
+                          "kernel": e.kernel, "left_context_frames": e.left, "chunk_frames": w.T,
+                          "features": f"{e.stack} x {e.feat} log-mel-like bins per 80 ms frame"}
+        names.append(f"with the cache-aware encoder chunk step ({e.name}-shaped)")
     if names:
         out["workload"] = f"cfg{w.cfg} {w.name}, " + "; ".join(names)
     return out
@@ -232,21 +238,30 @@ def oracle_models(w, inp_lm, inp_ph, E, W, extra=(), pred=None):
     return olm, obo, oracle.Model(w.V, w.H, E, W), pn
 
 
-def oracle_baseline(w, models, streams, chunks, threads=None, prune_k=0):
+def oracle_baseline(w, models, streams, chunks, threads=None, prune_k=0, encoder=None):
     """Times the oracle (as it stands) decoding `streams` x `chunks` of the
-    workload on this host's cores; returns (frames/s, cores, sample, seconds)."""
+    workload on this host's cores; returns (frames/s, cores, sample, seconds).
+    encoder: (oracle Encoder, its cfg) to run the encoder chunk step first."""
     import concurrent.futures
 
     import oracle
 
     threads = threads or len(os.sched_getaffinity(0))
     olm, obo, model, pn = models
-    encs = {c: synth.enc_chunk(w, streams, c) for c in range(chunks)}
+    if encoder is None:
+        encs = {c: synth.enc_chunk(w, streams, c) for c in range(chunks)}
+    else:
+        from oracle import encoder as oe
+
+        ecfg = encoder[1]
+        feats = {c: synth.features(ecfg, streams, c * w.T, w.T) for c in range(chunks)}
 
     def one(i):
         st = oracle.Stream(w.V)
+        est = oe.EncoderStream(ecfg) if encoder is not None else None
         for c in range(chunks):
-            oracle.decode_chunk(st, model, olm, obo, encs[c][i], w.lam, w.beta, w.max_sym, prune_k=prune_k,
+            frames = encs[c][i] if encoder is None else oe.encode_chunk(encoder[0], est, feats[c][i])
+            oracle.decode_chunk(st, model, olm, obo, frames, w.lam, w.beta, w.max_sym, prune_k=prune_k,
                                 pred=pn)
 
     t0 = time.perf_counter()
@@ -257,6 +272,16 @@ def oracle_baseline(w, models, streams, chunks, threads=None, prune_k=0):
     used = min(threads, len(streams))
     sample = f"{len(streams)} streams x {chunks} chunks x {w.T} frames of the same workload ({frames} frames)"
     return frames / dt, used, sample, dt
+
+
+def oracle_encoder(args):
+    """(oracle encoder, its cfg) for --encoder, else None."""
+    if not args.encoder:
+        return None
+    from oracle import encoder as oe
+
+    cfg = synth.ENCODERS[args.encoder]
+    return oe.Encoder(synth.encoder_weights(cfg)), cfg
 
 
 def run_reference(args, w):
@@ -270,13 +295,16 @@ def run_reference(args, w):
     n_str = args.ref_streams
     extra = extra_lms(w, args.extra_lms) if args.extra_lms else []
     models = oracle_models(w, lmA, ph, E, W, extra, pred_weights(w, args.pred))
+    enc_o = oracle_encoder(args)
+    if enc_o is not None:
+        n_str = min(n_str, 16)  # the encoder step dominates the oracle's time
     # warm-up steps, then K timed steps; each step decodes a bounded sample
     for _ in range(args.warmup):
-        oracle_baseline(w, models, list(range(2)), 1, prune_k=args.prune_k)
+        oracle_baseline(w, models, list(range(2)), 1, prune_k=args.prune_k, encoder=enc_o)
     vals, dts = [], []
     for k in range(args.steps):
         v, cores, sample, dt = oracle_baseline(w, models, list(range(k * n_str, (k + 1) * n_str)), 1,
-                                               prune_k=args.prune_k)
+                                               prune_k=args.prune_k, encoder=enc_o)
         vals.append(v)
         dts.append(dt)
     value = float(np.mean(vals))
@@ -321,15 +349,35 @@ def run_ours(args, w):
     slots = [dec.open() for _ in range(w.B)]
     slots_np = np.array(slots, dtype=np.int32)
     n_chunks = args.warmup + args.steps + 1
-    encs = [torch.from_numpy(synth.enc_chunk(w, streams, c % w.chunks).view(np.int16)).to(dev)
-            for c in range(n_chunks)]
+    encoder = None
+    if args.encoder:
+        # the cache-aware encoder chunk step runs first in every step; its
+        # frames are the decoder's input
+        ecfg = synth.ENCODERS[args.encoder]
+        need = pw.Henc if pw is not None else w.H
+        if ecfg.d != need or w.T > 32:
+            raise SystemExit(f"--encoder {args.encoder}: d={ecfg.d} must equal the decoder's input width {need} "
+                             f"and chunks must be <= 32 frames")
+        encoder = tsd.Encoder(synth.encoder_weights(ecfg), max_streams=w.B, max_chunk=w.T)
+        eslots = np.array([encoder.open() for _ in range(w.B)], dtype=np.int32)
+        encs = [torch.from_numpy(synth.features(ecfg, streams, (c % w.chunks) * w.T, w.T).view(np.int16)).to(dev)
+                for c in range(n_chunks)]
+        enc_frames = torch.empty((w.B, w.T, ecfg.d), dtype=torch.int16, device=dev)
+    else:
+        encs = [torch.from_numpy(synth.enc_chunk(w, streams, c % w.chunks).view(np.int16)).to(dev)
+                for c in range(n_chunks)]
     out = dec.alloc_out(w.B, w.T)
     outp = (out.tokens.data_ptr(), out.frames.data_ptr(), out.scores.data_ptr(), out.counts.data_ptr())
     sh = stream.cuda_stream
     flush = torch.empty(256 * 1024 * 1024, dtype=torch.uint8, device=dev)  # > 129 MB L2
 
-    def step(c):
-        dec.decode_chunk_raw(slots_np, encs[c].data_ptr(), w.T, w.lam, w.beta, outp, sh)
+    def step(c, src=None):
+        src = encs[c] if src is None else src
+        if encoder is not None:
+            encoder.encode_chunk_raw(eslots, src.data_ptr(), w.T, enc_frames.data_ptr(), sh)
+            dec.decode_chunk_raw(slots_np, enc_frames.data_ptr(), w.T, w.lam, w.beta, outp, sh)
+        else:
+            dec.decode_chunk_raw(slots_np, src.data_ptr(), w.T, w.lam, w.beta, outp, sh)
 
     def barrier():
         torch.cuda.synchronize()
@@ -364,15 +412,22 @@ def run_ours(args, w):
     # the same K steps again with a CUDA event recorded at every kernel
     # boundary inside the graph: per-kernel device time for the roofline
     dec.set_timing(True)
+    if encoder is not None:
+        encoder.set_timing(True)
     for c in range(2):
         step(args.warmup + c)  # captures the two event-carrying graphs
     barrier()
     dec.timing(reset=True)
     dec.timed_bytes(reset=True)
+    if encoder is not None:
+        encoder.timing(reset=True)
     t_inst_ms, _, _, _ = timed_loop(args.warmup)
     kernel_ms, kernel_n = dec.timing(reset=True)
     row_timed_bytes = dec.timed_bytes(reset=True)
     dec.set_timing(False)
+    enc_ms, enc_n = encoder.timing(reset=True) if encoder is not None else ({}, {})
+    if encoder is not None:
+        encoder.set_timing(False)
     t_ms, t_inst_ms = max_over_ranks([t_ms, t_inst_ms], ws, dev)
     frames = ws * w.B * w.T * args.steps
     value = frames / (t_ms / 1000.0)
@@ -390,7 +445,7 @@ def run_ours(args, w):
     e0.record(stream)
     for k in range(e2e_steps):
         dev_enc.copy_(host_enc[k % len(host_enc)], non_blocking=True)
-        dec.decode_chunk_raw(slots_np, dev_enc.data_ptr(), w.T, w.lam, w.beta, outp, sh)
+        step(0, dev_enc)
         for h, d in zip(host_out, (out.tokens, out.frames, out.scores, out.counts)):
             h.copy_(d, non_blocking=True)
     e1.record(stream)
@@ -430,7 +485,7 @@ def run_ours(args, w):
     pk, pk_kind = peaks()
     M = w.B * w.beam
     flop_per_launch = 2.0 * M * w.H * (w.V + 1)
-    total_ms = max(1e-9, sum(kernel_ms.values()))
+    total_ms = max(1e-9, sum(kernel_ms.values()) + sum(enc_ms.values()))
     share_joint = kernel_ms["joint"] / total_ms
     share_row = kernel_ms["row"] / total_ms
     share_pred = kernel_ms["pred"] / total_ms
@@ -513,11 +568,39 @@ def run_ours(args, w):
             "ms_per_chunk": step_ms * share_pred,
             "achieved": pred_flop / (step_ms * share_pred / 1000.0) / 1e12}
         pred_roof["in_production_graph"]["frac"] = pred_roof["in_production_graph"]["achieved"] / pred_roof["peak"]
+    enc_roof = None
+    if encoder is not None:
+        # the encoder's tensor-core GEMMs (subsampling, q/k/v, attention
+        # output, the convolution module's pointwise maps, feed-forward)
+        enc_flop = encoder.gemm_flops(w.B, w.T)
+        share_enc = enc_ms["gemm"] / total_ms
+        gemm_chunk_ms = enc_ms["gemm"] / args.steps
+        enc_roof = {"kernel": "k_egemm: encoder GEMMs with fused bias/Swish/GLU/residual epilogues (tcgen05)",
+                    "bound": "tensor", "unit": "TFLOP/s",
+                    "achieved": enc_flop / (gemm_chunk_ms / 1000.0) / 1e12,
+                    "peak": pk["bf16_tflops_sustained"],
+                    "peak_kind": f"{pk_kind} bf16 sustained (kernels timed inside the step)",
+                    "algorithmic": f"{enc_flop:.4g} FLOP per chunk (M={w.B * w.T} frame rows, 2 M N K per GEMM)",
+                    "ms_per_chunk": gemm_chunk_ms, "launches": enc_n["gemm"], "traffic": None,
+                    "share_of_device_time": share_enc,
+                    "encoder_other_kernels": {
+                        "attention_ms_per_chunk": enc_ms["attention"] / args.steps,
+                        "attention_share": enc_ms["attention"] / total_ms,
+                        "layer_norm_conv_cache_ms_per_chunk": enc_ms["other"] / args.steps,
+                        "layer_norm_conv_cache_share": enc_ms["other"] / total_ms}}
+        enc_roof["frac"] = enc_roof["achieved"] / enc_roof["peak"]
+        enc_roof["in_production_graph"] = {
+            "what": "uninstrumented step time x this class's share of device time",
+            "ms_per_chunk": step_ms * share_enc,
+            "achieved": enc_flop / (step_ms * share_enc / 1000.0) / 1e12}
+        enc_roof["in_production_graph"]["frac"] = enc_roof["in_production_graph"]["achieved"] / enc_roof["peak"]
     # the dominant kernel is the one with the largest device time in the graph
-    ranked = sorted([(share_joint, joint_roof), (share_row, row_roof)] + ([(share_pred, pred_roof)] if pred_roof else []),
-                    key=lambda x: -x[0])
+    ranked = sorted([(share_joint, joint_roof), (share_row, row_roof)] + ([(share_pred, pred_roof)] if pred_roof else [])
+                    + ([(share_enc, enc_roof)] if enc_roof else []), key=lambda x: -x[0])
     roof, other = ranked[0][1], ranked[1][1]
     launches = dec.launches_per_chunk(w.B, w.T)
+    if encoder is not None:
+        launches += 2 + 15 * synth.ENCODERS[args.encoder].layers  # subsampling, 15 per block, frame counts
     line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": t_ms / args.steps, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
@@ -532,6 +615,10 @@ def run_ours(args, w):
             "roofline_other_kernel": other,
             **({"roofline_third_kernel": ranked[2][1]} if len(ranked) > 2 else {}),
             "latency_per_chunk": latency_stats(step_ms),
+            **({"first_token_latency_s": {
+                "value": w.T * 0.080 + float(np.median(step_ms)) / 1000.0,
+                "what": "a chunk's audio (T x 80 ms) arrives before it is encoded, then the chunk's encoder and "
+                        "decoder compute (median timed step at this batch)"}} if encoder is not None else {}),
             "wall_s_timed_region": wall,
             "value_with_kernel_events": frames / (t_inst_ms / 1000.0),
             "kernel_timing": "per-kernel device time from CUDA events at every kernel boundary inside the "
@@ -539,8 +626,10 @@ def run_ours(args, w):
             "clocks": clk.summary()}
     if not args.no_cpu_baseline and ws == 1:
         models = oracle_models(w, lmA, ph, E, W, extra, pw)
-        v, cores, sample, dt = oracle_baseline(w, models, list(range(args.cpu_streams)), args.cpu_chunks,
-                                               prune_k=args.prune_k)
+        enc_o = oracle_encoder(args)
+        n_cpu = min(args.cpu_streams, 16) if enc_o is not None else args.cpu_streams
+        v, cores, sample, dt = oracle_baseline(w, models, list(range(n_cpu)), 1 if enc_o else args.cpu_chunks,
+                                               prune_k=args.prune_k, encoder=enc_o)
         line["cpu_baseline"] = {"value": v, "unit": UNIT, "cores": cores, "kind": "oracle",
                                 "sample": sample, "seconds": dt}
     print(json.dumps(line), flush=True)
@@ -563,6 +652,8 @@ def main():
                     help="pruned fusion over the acoustic model's k best outputs (0: every label)")
     ap.add_argument("--pred", type=int, default=0,
                     help="stateful form: an LSTM prediction network of this many units (0: stateless)")
+    ap.add_argument("--encoder", default=None, choices=sorted(synth.ENCODERS),
+                    help="run the cache-aware encoder chunk step before the decode in every step")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
