@@ -99,17 +99,32 @@ struct AttnArgs {
 
 // Shared memory of k_attn for a chunk of C frames (worst case nv = left).
 __host__ __device__ constexpr size_t attn_smem(int dh, int left, int C) {
-  return (size_t)(left + C) * (dh + 2) * 2 /*K*/ + (size_t)(left + C) * dh * 2 /*V*/ +
-         (size_t)2 * C * dh * 4 /*Qu, Qv*/ + (size_t)32 * (dh + 1) * 4 /*P tile*/ +
-         (size_t)C * (left + 2 * C - 1) * 4 /*Sp*/ + (size_t)C * (left + C) * 4 /*S*/;
+  return (size_t)(left + C) * (dh + 8) * 2 /*K*/ + (size_t)(left + C) * dh * 2 /*V*/ +
+         (size_t)2 * ((C + 15) / 16 * 16) * dh * 4 /*Qu, Qv*/ + (size_t)2 * (left + 2 * C - 1) * 16 * 4 /*SpT*/ +
+         (size_t)2 * (left + C) * 16 * 4 /*ST*/ + (size_t)2 * 16 * dh * 4 /*O partials*/;
+}
+
+__device__ __forceinline__ void bf16x8(const uint4 w, float* f) {
+  f[0] = __uint_as_float(w.x << 16), f[1] = __uint_as_float(w.x & 0xffff0000u);
+  f[2] = __uint_as_float(w.y << 16), f[3] = __uint_as_float(w.y & 0xffff0000u);
+  f[4] = __uint_as_float(w.z << 16), f[5] = __uint_as_float(w.z & 0xffff0000u);
+  f[6] = __uint_as_float(w.w << 16), f[7] = __uint_as_float(w.w & 0xffff0000u);
 }
 
 // One (stream, head) per CTA: chunked, limited-context attention with the
 // relative-position term over the window [cached frames, chunk frames], then
-// the chunk's k and v go into the ring cache.
+// the chunk's k and v go into the ring cache.  The three products (query
+// rows against the position table, against the keys, and probabilities
+// against the values) run as register tiles: a thread keeps 16 query rows'
+// sums for one key (or table row, or 4 x 4 outputs) and reads its operands
+// as 16-byte vectors from padded, bank-conflict-free shared rows; the inner
+// dimension is split over two threads whose halves are added afterwards.
 template <int DH>
 __global__ void __launch_bounds__(256) k_attn(AttnArgs a) {
   extern __shared__ __align__(16) unsigned char sm[];
+  constexpr int KS = DH + 8;  // padded k row (bf16): 16-byte aligned, conflict-free 16-byte reads
+  constexpr int HALF = DH / 2;
+  constexpr int NQ = DH / 4;  // column quads
   const int b = blockIdx.x, h = blockIdx.y, tid = threadIdx.x;
   const int C = a.C, d = a.d;
   const int slot = a.slots[b];
@@ -117,113 +132,172 @@ __global__ void __launch_bounds__(256) k_attn(AttnArgs a) {
   const int nv = min(sn, a.left);
   const int W = nv + C;
   const int nrel = nv + 2 * C - 1;  // offsets -(C-1) .. nv+C-1
-  const int Wm = a.left + C, nrm = a.left + 2 * C - 1;
-  constexpr int KS = DH + 2;  // padded k row (bf16)
+  const int Wm = a.left + C, nrm = a.left + 2 * C - 1, CR = (C + 15) / 16 * 16;
   uint16_t* Kb = reinterpret_cast<uint16_t*>(sm);
   uint16_t* Vb = Kb + (size_t)Wm * KS;
   float* Qu = reinterpret_cast<float*>(Vb + (size_t)Wm * DH);
-  float* Qv = Qu + C * DH;
-  float* Pt = Qv + C * DH;
-  float* Sp = Pt + 32 * (DH + 1);
-  float* S = Sp + C * nrm;
+  float* Qv = Qu + CR * DH;
+  float* SpT = Qv + CR * DH;       // [2][nrm][16]: halves of (q + v) . p(t), transposed
+  float* ST = SpT + 2 * nrm * 16;  // [2][Wm][16]: halves of (q + u) . k, transposed; [0] then holds the scores
+  float* Op = ST + 2 * Wm * 16;    // [2][16][DH]: output halves
 
   const size_t cb = (((size_t)slot * a.layers + a.layer) * a.heads + h) * (size_t)a.left * DH;
-  constexpr int P2 = DH / 2;  // bf16 pairs per row
-  for (int idx = tid; idx < nv * P2; idx += blockDim.x) {
-    const int jj = idx / P2, e2 = idx - jj * P2;
+  constexpr int E8 = DH / 8;  // 16-byte groups per row
+  for (int idx = tid; idx < nv * E8; idx += blockDim.x) {
+    const int jj = idx / E8, e8 = idx - jj * E8;
     const int ring = (sn - nv + jj) % a.left;
-    const uint32_t kw = reinterpret_cast<const uint32_t*>(a.kc + cb + (size_t)ring * DH)[e2];
-    const uint32_t vw = reinterpret_cast<const uint32_t*>(a.vc + cb + (size_t)ring * DH)[e2];
-    reinterpret_cast<uint32_t*>(Kb + (size_t)jj * KS)[e2] = kw;
-    reinterpret_cast<uint32_t*>(Vb + (size_t)jj * DH)[e2] = vw;
+    *reinterpret_cast<uint4*>(Kb + (size_t)jj * KS + 8 * e8) =
+        reinterpret_cast<const uint4*>(a.kc + cb + (size_t)ring * DH)[e8];
+    *reinterpret_cast<uint4*>(Vb + (size_t)jj * DH + 8 * e8) =
+        reinterpret_cast<const uint4*>(a.vc + cb + (size_t)ring * DH)[e8];
   }
-  for (int idx = tid; idx < C * P2; idx += blockDim.x) {
-    const int i = idx / P2, e2 = idx - i * P2;
-    const uint16_t* row = a.qkv + (size_t)(b * C + i) * 3 * d + h * DH;
-    const uint32_t qw = reinterpret_cast<const uint32_t*>(row)[e2];
-    reinterpret_cast<uint32_t*>(Kb + (size_t)(nv + i) * KS)[e2] = reinterpret_cast<const uint32_t*>(row + d)[e2];
-    reinterpret_cast<uint32_t*>(Vb + (size_t)(nv + i) * DH)[e2] = reinterpret_cast<const uint32_t*>(row + 2 * d)[e2];
-    const float q0 = __uint_as_float(qw << 16), q1 = __uint_as_float(qw & 0xffff0000u);
-    const int c = h * DH + 2 * e2;
-    Qu[i * DH + 2 * e2] = q0 + a.pu[c];
-    Qu[i * DH + 2 * e2 + 1] = q1 + a.pu[c + 1];
-    Qv[i * DH + 2 * e2] = q0 + a.pv[c];
-    Qv[i * DH + 2 * e2 + 1] = q1 + a.pv[c + 1];
+  for (int idx = tid; idx < CR * E8; idx += blockDim.x) {
+    const int i = idx / E8, e8 = idx - i * E8;
+    float q[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+    float* qu = Qu + i * DH + 8 * e8;
+    float* qv = Qv + i * DH + 8 * e8;
+    if (i < C) {
+      const uint16_t* row = a.qkv + (size_t)(b * C + i) * 3 * d + h * DH;
+      *reinterpret_cast<uint4*>(Kb + (size_t)(nv + i) * KS + 8 * e8) = reinterpret_cast<const uint4*>(row + d)[e8];
+      *reinterpret_cast<uint4*>(Vb + (size_t)(nv + i) * DH + 8 * e8) = reinterpret_cast<const uint4*>(row + 2 * d)[e8];
+      bf16x8(reinterpret_cast<const uint4*>(row)[e8], q);
+      const float* u = a.pu + h * DH + 8 * e8;
+      const float* v = a.pv + h * DH + 8 * e8;
+#pragma unroll
+      for (int k = 0; k < 8; ++k) {
+        qu[k] = q[k] + u[k];
+        qv[k] = q[k] + v[k];
+      }
+    } else {
+#pragma unroll
+      for (int k = 0; k < 8; ++k) qu[k] = qv[k] = 0.f;  // padding rows
+    }
   }
   __syncthreads();
   // the cache was read above: the chunk's k and v replace the oldest frames
   if (a.left > 0) {
-    for (int idx = tid; idx < C * P2; idx += blockDim.x) {
-      const int i = idx / P2, e2 = idx - i * P2;
+    for (int idx = tid; idx < C * E8; idx += blockDim.x) {
+      const int i = idx / E8, e8 = idx - i * E8;
       if (i < C - a.left) continue;
       const int ring = (sn + i) % a.left;
       const uint16_t* row = a.qkv + (size_t)(b * C + i) * 3 * d + h * DH;
-      reinterpret_cast<uint32_t*>(a.kc + cb + (size_t)ring * DH)[e2] = reinterpret_cast<const uint32_t*>(row + d)[e2];
-      reinterpret_cast<uint32_t*>(a.vc + cb + (size_t)ring * DH)[e2] =
-          reinterpret_cast<const uint32_t*>(row + 2 * d)[e2];
+      reinterpret_cast<uint4*>(a.kc + cb + (size_t)ring * DH)[e8] = reinterpret_cast<const uint4*>(row + d)[e8];
+      reinterpret_cast<uint4*>(a.vc + cb + (size_t)ring * DH)[e8] = reinterpret_cast<const uint4*>(row + 2 * d)[e8];
     }
   }
-  // position scores Sp[i][t] = (q_i + v) . p(t - (C-1)), 32 table rows at a time
-  for (int t0 = 0; t0 < nrel; t0 += 32) {
-    for (int idx = tid; idx < 32 * DH; idx += blockDim.x) {
-      const int tt = idx / DH, e = idx - tt * DH;
-      const int t = t0 + tt;
-      Pt[tt * (DH + 1) + e] = t < nrel ? a.pos_tab[(size_t)(t + a.cmax - C) * d + h * DH + e] : 0.f;
+  for (int rb = 0; rb < CR; rb += 16) {
+    // position term: SpT[s][t][r] = sum over half s of (q + v)[rb + r] . p(t - (C-1))
+    for (int item = tid; item < 2 * nrel; item += blockDim.x) {
+      const int s = item / nrel, t = item - s * nrel;
+      const float4* p = reinterpret_cast<const float4*>(a.pos_tab + (size_t)(t + a.cmax - C) * d + h * DH + s * HALF);
+      const float* q = Qv + rb * DH + s * HALF;
+      float acc[16];
+#pragma unroll
+      for (int r = 0; r < 16; ++r) acc[r] = 0.f;
+#pragma unroll 2
+      for (int q4 = 0; q4 < HALF / 4; ++q4) {
+        const float4 pv = p[q4];
+#pragma unroll
+        for (int r = 0; r < 16; ++r) {
+          const float4 qq = *reinterpret_cast<const float4*>(q + r * DH + 4 * q4);
+          acc[r] = fmaf(qq.x, pv.x, fmaf(qq.y, pv.y, fmaf(qq.z, pv.z, fmaf(qq.w, pv.w, acc[r]))));
+        }
+      }
+      float4* o = reinterpret_cast<float4*>(SpT + ((size_t)s * nrm + t) * 16);
+#pragma unroll
+      for (int r = 0; r < 16; r += 4) o[r / 4] = make_float4(acc[r], acc[r + 1], acc[r + 2], acc[r + 3]);
+    }
+    // content term: ST[s][jj][r] = sum over half s of (q + u)[rb + r] . k_jj
+    for (int item = tid; item < 2 * W; item += blockDim.x) {
+      const int s = item / W, jj = item - s * W;
+      const uint16_t* kr = Kb + (size_t)jj * KS + s * HALF;
+      const float* q = Qu + rb * DH + s * HALF;
+      float acc[16];
+#pragma unroll
+      for (int r = 0; r < 16; ++r) acc[r] = 0.f;
+#pragma unroll 1
+      for (int o8 = 0; o8 < HALF / 8; ++o8) {
+        float kf[8];
+        bf16x8(*reinterpret_cast<const uint4*>(kr + 8 * o8), kf);
+#pragma unroll
+        for (int r = 0; r < 16; ++r) {
+          const float4 q0 = *reinterpret_cast<const float4*>(q + r * DH + 8 * o8);
+          const float4 q1 = *reinterpret_cast<const float4*>(q + r * DH + 8 * o8 + 4);
+          acc[r] = fmaf(q0.x, kf[0], fmaf(q0.y, kf[1], fmaf(q0.z, kf[2], fmaf(q0.w, kf[3], acc[r]))));
+          acc[r] = fmaf(q1.x, kf[4], fmaf(q1.y, kf[5], fmaf(q1.z, kf[6], fmaf(q1.w, kf[7], acc[r]))));
+        }
+      }
+      float4* o = reinterpret_cast<float4*>(ST + ((size_t)s * Wm + jj) * 16);
+#pragma unroll
+      for (int r = 0; r < 16; r += 4) o[r / 4] = make_float4(acc[r], acc[r + 1], acc[r + 2], acc[r + 3]);
     }
     __syncthreads();
-    for (int idx = tid; idx < C * 32; idx += blockDim.x) {
-      const int i = idx >> 5, tt = idx & 31;
-      if (t0 + tt >= nrel) continue;
-      const float* qv = Qv + i * DH;
-      const float* p = Pt + tt * (DH + 1);
-      float acc = 0.f;
-#pragma unroll 16
-      for (int e = 0; e < DH; ++e) acc = fmaf(qv[e], p[e], acc);
-      Sp[i * nrm + t0 + tt] = acc;
+    // scores of rows rb..rb+15 into ST[0]
+    for (int item = tid; item < W * 16; item += blockDim.x) {
+      const int jj = item >> 4, r = item & 15, i = rb + r;
+      float v = 0.f;
+      if (i < C) {
+        const int t = i - jj + nv + C - 1;
+        v = (ST[jj * 16 + r] + ST[(Wm + jj) * 16 + r] + SpT[t * 16 + r] + SpT[(nrm + t) * 16 + r]) * a.scale;
+      }
+      ST[jj * 16 + r] = v;
     }
     __syncthreads();
-  }
-  // scores: content + position, scaled
-  for (int idx = tid; idx < C * W; idx += blockDim.x) {
-    const int i = idx / W, jj = idx - i * W;
-    const float* qu = Qu + i * DH;
-    const uint32_t* kr = reinterpret_cast<const uint32_t*>(Kb + (size_t)jj * KS);
-    float acc = 0.f;
-#pragma unroll 16
-    for (int e2 = 0; e2 < P2; ++e2) {
-      const uint32_t w = kr[e2];
-      acc = fmaf(qu[2 * e2], __uint_as_float(w << 16), acc);
-      acc = fmaf(qu[2 * e2 + 1], __uint_as_float(w & 0xffff0000u), acc);
-    }
-    S[i * Wm + jj] = (acc + Sp[i * nrm + (i - jj + nv + C - 1)]) * a.scale;
-  }
-  __syncthreads();
-  // softmax per query row (one warp per row)
-  {
-    const int warp = tid >> 5, lane = tid & 31;
-    for (int i = warp; i < C; i += blockDim.x >> 5) {
-      float* s = S + i * Wm;
+    if (tid < 16 && rb + tid < C) {  // softmax, one thread per query row
       float m = -INFINITY;
-      for (int j = lane; j < W; j += 32) m = fmaxf(m, s[j]);
-      m = warp_max(m);
+      for (int jj = 0; jj < W; ++jj) m = fmaxf(m, ST[jj * 16 + tid]);
       float z = 0.f;
-      for (int j = lane; j < W; j += 32) {
-        const float e = expf(s[j] - m);
-        s[j] = e;
+      for (int jj = 0; jj < W; ++jj) {
+        const float e = expf(ST[jj * 16 + tid] - m);
+        ST[jj * 16 + tid] = e;
         z += e;
       }
-      z = warp_sum(z);
       const float inv = 1.f / z;
-      for (int j = lane; j < W; j += 32) s[j] *= inv;
+      for (int jj = 0; jj < W; ++jj) ST[jj * 16 + tid] *= inv;
     }
-  }
-  __syncthreads();
-  for (int idx = tid; idx < C * DH; idx += blockDim.x) {
-    const int i = idx / DH, e = idx - i * DH;
-    const float* s = S + i * Wm;
-    float acc = 0.f;
-    for (int jj = 0; jj < W; ++jj) acc = fmaf(s[jj], bf2f(Vb[(size_t)jj * DH + e]), acc);
-    a.out[(size_t)(b * C + i) * d + h * DH + e] = f2bf(acc);
+    __syncthreads();
+    // output halves: Op[s][4g + r][4q + c] over the keys of half s
+    {
+      const int s = tid >> 7, rem = tid & 127, g = rem / NQ, q = rem - g * NQ;
+      if (g < 4) {
+        const int j0 = s == 0 ? 0 : W / 2, j1 = s == 0 ? W / 2 : W;
+        float acc[4][4];
+#pragma unroll
+        for (int r = 0; r < 4; ++r)
+#pragma unroll
+          for (int c = 0; c < 4; ++c) acc[r][c] = 0.f;
+        for (int jj = j0; jj < j1; ++jj) {
+          const uint2 vw = *reinterpret_cast<const uint2*>(Vb + (size_t)jj * DH + 4 * q);
+          const float v0 = __uint_as_float(vw.x << 16), v1 = __uint_as_float(vw.x & 0xffff0000u);
+          const float v2 = __uint_as_float(vw.y << 16), v3 = __uint_as_float(vw.y & 0xffff0000u);
+          const float4 p = *reinterpret_cast<const float4*>(ST + jj * 16 + 4 * g);
+          const float pr[4] = {p.x, p.y, p.z, p.w};
+#pragma unroll
+          for (int r = 0; r < 4; ++r) {
+            acc[r][0] = fmaf(pr[r], v0, acc[r][0]);
+            acc[r][1] = fmaf(pr[r], v1, acc[r][1]);
+            acc[r][2] = fmaf(pr[r], v2, acc[r][2]);
+            acc[r][3] = fmaf(pr[r], v3, acc[r][3]);
+          }
+        }
+#pragma unroll
+        for (int r = 0; r < 4; ++r)
+          *reinterpret_cast<float4*>(Op + ((size_t)s * 16 + 4 * g + r) * DH + 4 * q) =
+              make_float4(acc[r][0], acc[r][1], acc[r][2], acc[r][3]);
+      }
+    }
+    __syncthreads();
+    for (int item = tid; item < 16 * NQ; item += blockDim.x) {
+      const int r = item / NQ, q = item - r * NQ, i = rb + r;
+      if (i >= C) continue;
+      const float4 x = *reinterpret_cast<const float4*>(Op + (size_t)r * DH + 4 * q);
+      const float4 y = *reinterpret_cast<const float4*>(Op + (size_t)(16 + r) * DH + 4 * q);
+      uint2 w;
+      w.x = (uint32_t)f2bf(x.x + y.x) | ((uint32_t)f2bf(x.y + y.y) << 16);
+      w.y = (uint32_t)f2bf(x.z + y.z) | ((uint32_t)f2bf(x.w + y.w) << 16);
+      *reinterpret_cast<uint2*>(a.out + (size_t)(b * C + i) * d + h * DH + 4 * q) = w;
+    }
+    __syncthreads();
   }
 }
 

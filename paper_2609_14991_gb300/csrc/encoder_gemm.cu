@@ -1,6 +1,6 @@
 // Tensor-core GEMM of the cache-aware encoder: out = A . B^T with A [M][K]
 // and B [N][K] bf16 K-major (B = a weight stored [out][in]), fp32 accumulate
-// in TMEM, 128 x 128 output tiles, TMA loads into a 6-stage ring of
+// in TMEM, 128 x 128 output tiles, TMA loads into a 3-stage ring of
 // 128-byte-swizzled stages.  Warp 0 is the TMA producer, warp 1 allocates
 // TMEM and issues the MMAs, warps 2-5 run the epilogue (thread = output row;
 // warp w reads TMEM lanes 32 (w mod 4) ..).  The epilogue applies the bias
@@ -21,7 +21,7 @@ namespace {
 using namespace tc;
 
 constexpr int kBN = kEgBN;
-constexpr int kStages = 6;
+constexpr int kStages = 3;
 constexpr int kThreads = 192;
 constexpr int kABytes = kBM * kBK * 2;
 constexpr int kBBytes = kBN * kBK * 2;
@@ -38,7 +38,7 @@ __device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
 }
 
 template <int EPI>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(kThreads, 2)
     k_egemm(EGemm g, const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB) {
   extern __shared__ __align__(1024) unsigned char smem_raw[];
   unsigned char* smem = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
