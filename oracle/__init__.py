@@ -74,10 +74,10 @@ def lib() -> ctypes.CDLL:
             "oracle_decode_chunk_pred": ([vp, vp, vp, i32, i32, i32, i32, vp, vp, vp, vp, vp, vp, vp, vp, vp, i32,
                                           dbl, dbl, i32, vp, vp, vp, i32, dbl, vp, vp, vp, i32, vp], i32),
             "oracle_pred_state": ([vp, vp, vp], i32),
-            "oracle_beam_chunk": ([vp, vp, vp, i32, i32, vp, vp, vp, i32, dbl, dbl, i32], i32),
+            "oracle_beam_chunk": ([vp, vp, vp, i32, i32, vp, vp, vp, i32, dbl, dbl, i32, i32], i32),
             "oracle_beam_hyp": ([vp, i32, vp, i64, vp, vp], i64),
             "oracle_beam_chunk_follow": ([vp, vp, vp, i32, i32, vp, vp, vp, i32, dbl, dbl, i32, vp, vp, vp, dbl,
-                                          vp], i32),
+                                          vp, i32, i32], i32),
             "oracle_joint_logits": ([i32, i32, vp, vp, vp, i32, vp], None),
             "oracle_fused_row": ([vp, vp, vp, i32, i32, vp, vp, vp, dbl, dbl, vp], None),
             "oracle_boost_trajectory": ([vp, vp, i64, vp, vp], None),
@@ -331,25 +331,28 @@ def decode_chunk(stream: Stream, model: Model, lm: Optional[LM], boost: Optional
 
 
 def beam_chunk(stream: Stream, model: Model, lm: Optional[LM], boost: Optional[Boost], enc: np.ndarray,
-               lam: float, beta: float, K: int) -> int:
+               lam: float, beta: float, K: int, S: int = 1) -> int:
+    """Beam search over one chunk, at most S labels per frame."""
     enc = np.ascontiguousarray(enc, dtype=np.uint16)
     return lib().oracle_beam_chunk(stream.h, lm.h if lm else None, boost.h if boost else None, model.V, model.H,
                                    _p(model.E), _p(model.W), _p(enc), enc.shape[0], float(lam), float(beta),
-                                   int(K))
+                                   int(K), int(S))
 
 
 def beam_chunk_follow(stream: Stream, model: Model, lm: Optional[LM], boost: Optional[Boost], enc: np.ndarray,
                       lam: float, beta: float, K: int, sel_hyp: np.ndarray, sel_tok: np.ndarray,
-                      sel_inc: np.ndarray, gap_tol: float = 1e-3) -> np.ndarray:
-    """Beam search over one chunk following kept candidates [T, K] under test;
-    returns the report (see oracle_beam_chunk_follow)."""
+                      sel_inc: np.ndarray, gap_tol: float = 1e-3, S: int = 1) -> np.ndarray:
+    """Beam search over one chunk following kept candidates [steps, K] under
+    test (one row per expansion); returns the report (see
+    oracle_beam_chunk_follow)."""
     enc = np.ascontiguousarray(enc, dtype=np.uint16)
+    n_steps = np.asarray(sel_hyp).shape[0]
     sh, st = _i32(sel_hyp).reshape(-1), _i32(sel_tok).reshape(-1)
     si = np.ascontiguousarray(sel_inc, dtype=np.float32).reshape(-1)
     rep = np.zeros(8, dtype=np.float64)
     lib().oracle_beam_chunk_follow(stream.h, lm.h if lm else None, boost.h if boost else None, model.V, model.H,
                                    _p(model.E), _p(model.W), _p(enc), enc.shape[0], float(lam), float(beta), int(K),
-                                   _p(sh), _p(st), _p(si), float(gap_tol), _p(rep))
+                                   _p(sh), _p(st), _p(si), float(gap_tol), _p(rep), int(S), int(n_steps))
     return rep
 
 

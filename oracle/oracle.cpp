@@ -38,7 +38,8 @@
 //                       projections, joint input = bf16(ReLU(W_enc enc_t + b_enc
 //                       + W_pred h + b_pred)); the LSTM advances on every
 //                       emitted label.
-//   * beam search:      per frame, top-K of the K*(V+1) extensions, then
+//   * beam search:      per frame up to S expansions, each the top-K of the
+//                       extensions of the hypotheses still in the frame;
 //                       identical label sequences merged by log-sum-exp.
 //                       (Not in the paper; the beam workload defines it.)
 #include <algorithm>
@@ -668,17 +669,68 @@ ORACLE_API int32_t oracle_decode_chunk_lms(void* sp, int32_t n_lm, const void* c
                            out_frame, out_score, out_cap, report);
 }
 
-// Beam search over one chunk (beam workload): every live hypothesis expands
-// to all V+1 outputs each frame (blank keeps its labels, token v appends v),
-// with at most one label per frame; the global top-K of the K*(V+1)
-// candidates is taken by (score desc, hypothesis index asc, token asc), then
-// candidates with identical label sequences are merged by log-sum-exp in
-// order of first appearance (so fewer than K may survive).
+// Beam search, one frame-synchronous expansion (beam workload; several
+// labels per frame).  A frame starts with the beam as its set A of
+// hypotheses still in the frame and an empty set F of hypotheses that have
+// left it.  One expansion takes, over every hypothesis of A and every
+// output, the top K candidates by (score desc, hypothesis index in A asc,
+// label asc); in that order a candidate goes to F if it is the blank (labels
+// kept) or a label at the frame's S-th expansion (the frame then advances
+// without another evaluation, as in greedy decoding), else to the next A;
+// in either set equal label sequences merge by log-sum-exp in order of first
+// appearance.  F then keeps its K best (score desc, earlier first), in
+// insertion order.  The frame ends when A is empty or after S expansions,
+// and F is the next frame's beam.  With S = 1 every kept candidate lands in
+// F: the top K of the K (V+1) extensions, merged -- one label per frame.
+namespace {
+struct Kept {
+  int32_t hyp, tok;
+  double score;
+};
+
+void merge_into(std::vector<Hyp>& set, Hyp&& h) {
+  for (Hyp& o : set) {
+    if (o.y == h.y) {
+      o.score = logaddexp(o.score, h.score);
+      return;
+    }
+  }
+  set.push_back(std::move(h));
+}
+
+void beam_expand(const PhraseSet* boost, int32_t V, int32_t S, int32_t K, int32_t e, std::vector<Hyp>& A,
+                 std::vector<Hyp>& F, const std::vector<Kept>& kept) {
+  std::vector<Hyp> A2;
+  for (const Kept& c : kept) {
+    Hyp h = A[(size_t)c.hyp];
+    if (c.tok != V) {
+      h.y.push_back(c.tok);
+      advance_rho(boost, h);
+    }
+    h.score = c.score;
+    merge_into((c.tok == V || e == S - 1) ? F : A2, std::move(h));
+  }
+  if ((int32_t)F.size() > K) {
+    std::vector<size_t> order(F.size());
+    for (size_t i = 0; i < order.size(); ++i) order[i] = i;
+    std::stable_sort(order.begin(), order.end(), [&](size_t x, size_t y) { return F[x].score > F[y].score; });
+    std::vector<char> keep(F.size(), 0);
+    for (int32_t r = 0; r < K; ++r) keep[order[(size_t)r]] = 1;
+    std::vector<Hyp> F2;
+    for (size_t i = 0; i < F.size(); ++i)
+      if (keep[i]) F2.push_back(std::move(F[i]));
+    F = std::move(F2);
+  }
+  A = std::move(A2);
+}
+}  // namespace
+
+// Beam search over one chunk with at most S labels per frame (see above).
 // Returns the number of live hypotheses after the chunk.
 ORACLE_API int32_t oracle_beam_chunk(void* sp, const void* lmp, const void* boostp, int32_t V,
                                      int32_t H, const uint16_t* E, const uint16_t* W,
                                      const uint16_t* enc, int32_t T, double lambda, double beta,
-                                     int32_t K) {
+                                     int32_t K, int32_t S) {
   Stream* s = static_cast<Stream*>(sp);
   const NGramDict* lm = static_cast<const NGramDict*>(lmp);
   const PhraseSet* boost = static_cast<const PhraseSet*>(boostp);
@@ -686,41 +738,23 @@ ORACLE_API int32_t oracle_beam_chunk(void* sp, const void* lmp, const void* boos
   if (s->beam.empty()) s->beam.push_back(Hyp());
   std::vector<float> x;
   std::vector<double> logits, fused;
-  struct Cand {
-    double score;
-    int32_t hyp, tok;
-  };
   for (int32_t t = 0; t < T; ++t) {
-    std::vector<Cand> cands;
-    for (int32_t i = 0; i < (int32_t)s->beam.size(); ++i) {
-      fused_scores(m, enc + (size_t)t * H, s->beam[(size_t)i], one_lm(lm, lambda), boost, beta, x, logits, fused);
-      for (int32_t v = 0; v <= V; ++v) cands.push_back({s->beam[(size_t)i].score + fused[(size_t)v], i, v});
-    }
-    std::sort(cands.begin(), cands.end(), [](const Cand& a, const Cand& b) {
-      if (a.score != b.score) return a.score > b.score;
-      if (a.hyp != b.hyp) return a.hyp < b.hyp;
-      return a.tok < b.tok;
-    });
-    if ((int32_t)cands.size() > K) cands.resize((size_t)K);
-    std::vector<Hyp> next;
-    for (const Cand& c : cands) {
-      Hyp h = s->beam[(size_t)c.hyp];
-      if (c.tok != V) {
-        h.y.push_back(c.tok);
-        advance_rho(boost, h);
+    std::vector<Hyp> A = std::move(s->beam), F;
+    for (int32_t e = 0; e < S && !A.empty(); ++e) {
+      std::vector<Kept> cands;
+      for (int32_t i = 0; i < (int32_t)A.size(); ++i) {
+        fused_scores(m, enc + (size_t)t * H, A[(size_t)i], one_lm(lm, lambda), boost, beta, x, logits, fused);
+        for (int32_t v = 0; v <= V; ++v) cands.push_back({i, v, A[(size_t)i].score + fused[(size_t)v]});
       }
-      h.score = c.score;
-      bool merged = false;
-      for (Hyp& o : next) {
-        if (o.y == h.y) {
-          o.score = logaddexp(o.score, h.score);
-          merged = true;
-          break;
-        }
-      }
-      if (!merged) next.push_back(std::move(h));
+      std::sort(cands.begin(), cands.end(), [](const Kept& a, const Kept& b) {
+        if (a.score != b.score) return a.score > b.score;
+        if (a.hyp != b.hyp) return a.hyp < b.hyp;
+        return a.tok < b.tok;
+      });
+      if ((int32_t)cands.size() > K) cands.resize((size_t)K);
+      beam_expand(boost, V, S, K, e, A, F, cands);
     }
-    s->beam = std::move(next);
+    s->beam = std::move(F);
   }
   return (int32_t)s->beam.size();
 }
@@ -738,22 +772,24 @@ ORACLE_API int64_t oracle_beam_hyp(const void* sp, int32_t i, int32_t* buf, int6
   return (int64_t)h.y.size();
 }
 
-// Beam search over one chunk following the selections under test.  For
-// frame t, sel_hyp/sel_tok/sel_inc[t*K + i] (i < K) are the candidates that
-// were kept, in their order (hypothesis -1 = none): the hypothesis index,
-// the label (V = blank) and the score increment that was used.  The oracle
-// scores every candidate itself and checks that
+// Beam search over one chunk following the selections under test.  Step s
+// (an expansion; a stream's frames may take different numbers of them) kept
+// sel_hyp/sel_tok/sel_inc[s*K + i] (i < K), in their order (hypothesis -1
+// = none; hypothesis = index in the frame's set A): the hypothesis, the
+// label (V = blank) and the score increment that was used.  After the last
+// frame every remaining step must be empty.  The oracle scores every
+// candidate itself and checks that
 //   * each kept candidate's increment is its own fused value (largest
 //     difference reported),
 //   * no candidate left out beats a kept one by more than gap_tol, and the
 //     kept ones are in non-increasing order up to gap_tol,
-// then applies the selection in that order, merging equal label sequences
-// by log-sum-exp of its own scores.
+// then applies the expansion with its own scores (merges by log-sum-exp).
 ORACLE_API int32_t oracle_beam_chunk_follow(void* sp, const void* lmp, const void* boostp, int32_t V,
                                             int32_t H, const uint16_t* E, const uint16_t* W,
                                             const uint16_t* enc, int32_t T, double lambda, double beta,
                                             int32_t K, const int32_t* sel_hyp, const int32_t* sel_tok,
-                                            const float* sel_inc, double gap_tol, double* report) {
+                                            const float* sel_inc, double gap_tol, double* report, int32_t S,
+                                            int32_t n_steps) {
   Stream* s = static_cast<Stream*>(sp);
   const NGramDict* lm = static_cast<const NGramDict*>(lmp);
   const PhraseSet* boost = static_cast<const PhraseSet*>(boostp);
@@ -762,64 +798,54 @@ ORACLE_API int32_t oracle_beam_chunk_follow(void* sp, const void* lmp, const voi
   double rep[REP_N] = {0, 0, 0, 0, std::numeric_limits<double>::infinity(), -1, 0, 0};
   std::vector<float> x;
   std::vector<double> logits, fused;
+  int32_t step = 0;
   for (int32_t t = 0; t < T; ++t) {
-    const size_t nh = s->beam.size();
-    std::vector<std::vector<double>> f(nh);
-    for (size_t i = 0; i < nh; ++i) {
-      fused_scores(m, enc + (size_t)t * H, s->beam[i], one_lm(lm, lambda), boost, beta, x, logits, fused);
-      f[i] = fused;
-    }
-    std::vector<std::pair<int32_t, int32_t>> kept;
-    std::vector<char> is_kept(nh * (size_t)(V + 1), 0);
-    double min_kept = std::numeric_limits<double>::infinity(), prev = std::numeric_limits<double>::infinity();
-    for (int32_t i = 0; i < K; ++i) {
-      const int32_t h = sel_hyp[(size_t)t * K + i], v = sel_tok[(size_t)t * K + i];
-      if (h < 0) continue;
-      if (h >= (int32_t)nh || v < 0 || v > V) { rep[REP_INCONSISTENT] = 1; continue; }
-      const double sc = s->beam[(size_t)h].score + f[(size_t)h][(size_t)v];
-      rep[REP_MAX_SCORE_DIFF] = std::max(rep[REP_MAX_SCORE_DIFF],
-                                         std::fabs((double)sel_inc[(size_t)t * K + i] - f[(size_t)h][(size_t)v]));
-      if (sc > prev + gap_tol) rep[REP_MISMATCH] += 1;  // out of order
-      prev = sc;
-      min_kept = std::min(min_kept, sc);
-      is_kept[(size_t)h * (V + 1) + (size_t)v] = 1;
-      kept.push_back({h, v});
-    }
-    const size_t want = std::min((size_t)K, nh * (size_t)(V + 1));
-    if (kept.size() != want) rep[REP_INCONSISTENT] = 1;
-    double best_out = -std::numeric_limits<double>::infinity();
-    for (size_t h = 0; h < nh; ++h)
-      for (int32_t v = 0; v <= V; ++v)
-        if (!is_kept[h * (V + 1) + (size_t)v]) best_out = std::max(best_out, s->beam[h].score + f[h][(size_t)v]);
-    if (best_out > min_kept + gap_tol) {
-      rep[REP_MISMATCH] += 1;
-      if (rep[REP_FIRST_BAD] < 0) rep[REP_FIRST_BAD] = t;
-    } else if (best_out > min_kept) {
-      rep[REP_NEAR_TIE] += 1;
-    }
-    rep[REP_MIN_GAP] = std::min(rep[REP_MIN_GAP], min_kept - best_out);
-    std::vector<Hyp> next;
-    for (const auto& kv : kept) {
-      Hyp h = s->beam[(size_t)kv.first];
-      const double sc = h.score + f[(size_t)kv.first][(size_t)kv.second];
-      if (kv.second != V) {
-        h.y.push_back(kv.second);
-        advance_rho(boost, h);
+    std::vector<Hyp> A = std::move(s->beam), F;
+    for (int32_t e = 0; e < S && !A.empty(); ++e, ++step) {
+      if (step >= n_steps) { rep[REP_INCONSISTENT] = 1; break; }
+      const size_t nh = A.size();
+      std::vector<std::vector<double>> f(nh);
+      for (size_t i = 0; i < nh; ++i) {
+        fused_scores(m, enc + (size_t)t * H, A[i], one_lm(lm, lambda), boost, beta, x, logits, fused);
+        f[i] = fused;
       }
-      h.score = sc;
-      bool merged = false;
-      for (Hyp& o : next) {
-        if (o.y == h.y) {
-          o.score = logaddexp(o.score, h.score);
-          merged = true;
-          break;
-        }
+      std::vector<Kept> kept;
+      std::vector<char> is_kept(nh * (size_t)(V + 1), 0);
+      double min_kept = std::numeric_limits<double>::infinity(), prev = std::numeric_limits<double>::infinity();
+      for (int32_t i = 0; i < K; ++i) {
+        const int32_t h = sel_hyp[(size_t)step * K + i], v = sel_tok[(size_t)step * K + i];
+        if (h < 0) continue;
+        if (h >= (int32_t)nh || v < 0 || v > V) { rep[REP_INCONSISTENT] = 1; continue; }
+        const double sc = A[(size_t)h].score + f[(size_t)h][(size_t)v];
+        rep[REP_MAX_SCORE_DIFF] = std::max(rep[REP_MAX_SCORE_DIFF],
+                                           std::fabs((double)sel_inc[(size_t)step * K + i] - f[(size_t)h][(size_t)v]));
+        if (sc > prev + gap_tol) rep[REP_MISMATCH] += 1;  // out of order
+        prev = sc;
+        min_kept = std::min(min_kept, sc);
+        is_kept[(size_t)h * (V + 1) + (size_t)v] = 1;
+        kept.push_back({h, v, sc});
       }
-      if (!merged) next.push_back(std::move(h));
+      const size_t want = std::min((size_t)K, nh * (size_t)(V + 1));
+      if (kept.size() != want) rep[REP_INCONSISTENT] = 1;
+      double best_out = -std::numeric_limits<double>::infinity();
+      for (size_t h = 0; h < nh; ++h)
+        for (int32_t v = 0; v <= V; ++v)
+          if (!is_kept[h * (V + 1) + (size_t)v]) best_out = std::max(best_out, A[h].score + f[h][(size_t)v]);
+      if (best_out > min_kept + gap_tol) {
+        rep[REP_MISMATCH] += 1;
+        if (rep[REP_FIRST_BAD] < 0) rep[REP_FIRST_BAD] = step;
+      } else if (best_out > min_kept) {
+        rep[REP_NEAR_TIE] += 1;
+      }
+      rep[REP_MIN_GAP] = std::min(rep[REP_MIN_GAP], min_kept - best_out);
+      beam_expand(boost, V, S, K, e, A, F, kept);
+      rep[REP_STEPS] += 1;
     }
-    s->beam = std::move(next);
-    rep[REP_STEPS] += 1;
+    s->beam = std::move(F);
   }
+  for (; step < n_steps; ++step)
+    for (int32_t i = 0; i < K; ++i)
+      if (sel_hyp[(size_t)step * K + i] >= 0) rep[REP_INCONSISTENT] = 1;
   if (report)
     for (int i = 0; i < REP_N; ++i) report[i] = rep[i];
   return (int32_t)s->beam.size();

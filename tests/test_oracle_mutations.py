@@ -43,6 +43,10 @@ MUTATIONS = {
     "prediction network advances on blank": (
         "      rep[REP_STEPS] += 1;\n      if (y == V) break;",
         "      rep[REP_STEPS] += 1;\n      if (y == V && pn) lstm_step(*pn, V, s->pred);\n      if (y == V) break;"),
+    "S-th label of a frame stays in the frame": ("merge_into((c.tok == V || e == S - 1) ? F : A2, std::move(h));",
+                                                  "merge_into((c.tok == V) ? F : A2, std::move(h));"),
+    "frame-exit set re-sorted by score": ("    for (size_t i = 0; i < F.size(); ++i)\n      if (keep[i]) F2.push_back(std::move(F[i]));",
+                                          "    for (size_t r = 0; r < (size_t)K; ++r) F2.push_back(std::move(F[order[r]]));"),
     "failed match not cancelled": (
         "return bonus * (double)(match(gv.data(), len + 1) - match(g, len));",
         "return bonus * (double)std::max(0, match(gv.data(), len + 1) - match(g, len));"),
@@ -62,7 +66,9 @@ def test_pins_catch_planted_mistake(name, tmp_path):
     r = subprocess.run([sys.executable, "-m", "pytest", os.path.join(ROOT, "tests", "test_oracle_pins.py"),
                         os.path.join(ROOT, "tests", "test_oracle_multilm.py"),
                         os.path.join(ROOT, "tests", "test_oracle_pruned.py"),
-                        os.path.join(ROOT, "tests", "test_oracle_pred.py"), "-q", "-x", "-p", "no:cacheprovider"], cwd=ROOT, capture_output=True, text=True,
+                        os.path.join(ROOT, "tests", "test_oracle_pred.py"),
+                        os.path.join(ROOT, "tests", "test_oracle_beam_multi.py"), "-q", "-x", "-p", "no:cacheprovider"],
+                       cwd=ROOT, capture_output=True, text=True,
                        env=dict(os.environ, TSD_ORACLE_LIB=str(so)), timeout=600)
     assert r.returncode != 0, f"pins did not catch: {name}\n{r.stdout[-2000:]}"
 
