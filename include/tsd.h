@@ -172,7 +172,7 @@ TSD_API tsd_status tsd_boost_node_tuple(const tsd_boost* b, int32_t node, int32_
 typedef struct {
   int32_t V;           /* non-blank labels; blank = V; 1 <= V <= 16384 */
   int32_t H;           /* joint hidden size; multiple of 64, 64 <= H <= 8192 */
-  int32_t max_symbols; /* labels per frame (greedy; Sec. III); beam requires 1 */
+  int32_t max_symbols; /* labels per frame, 1..64 (greedy: Sec. III; beam: expansions per frame) */
   int32_t beam_k;      /* 1 = greedy; 2..8 = beam search */
   int32_t max_streams; /* stream slots; max_streams * beam_k <= 4096 */
   int32_t max_T;       /* frames per chunk, 1 <= max_T <= 4096 */
@@ -257,12 +257,19 @@ TSD_API tsd_status tsd_stream_close(tsd_decoder* dec, int32_t slot);
  *     out_frames  device int32 [n][T*max_symbols]: frame (0..T-1) of each;
  *     out_scores  device float [n][T*max_symbols]: its fused score (Eq. 1);
  *     out_counts  device int32 [n]: labels emitted this chunk.
- *   Beam (beam_k > 1): every live hypothesis is extended by blank or one
- *   label per frame; the top beam_k of all extensions survive and those with
- *   equal label sequences are merged by log-sum-exp.  out_counts[i] = length
- *   of the best hypothesis, out_scores[i*T*max_symbols] = its score,
- *   out_tokens/out_frames are not written; read the labels with
- *   tsd_stream_result.
+ *   Beam (beam_k > 1), frame-synchronous with up to S = max_symbols labels
+ *   per frame: each label step expands the hypotheses still in their frame
+ *   by blank or a label; the top beam_k extensions are kept and, in order, a
+ *   blank (or a label at the frame's S-th expansion) leaves the frame, the
+ *   rest stay in it; within each set equal label sequences merge by
+ *   log-sum-exp; the set that left keeps its beam_k best (in order of
+ *   arrival) and becomes the next frame's beam when no hypothesis stays or
+ *   after S expansions.  S = 1: one label or blank per frame.
+ *   out_counts[i] = length of the best hypothesis, out_scores[i*T*max_symbols]
+ *   = its score, out_tokens/out_frames are not written; read the labels with
+ *   tsd_stream_result.  Each stream holds up to 8192 label-sequence nodes
+ *   (at most beam_k per label step are added); a stream that outgrows them
+ *   stops recording labels and tsd_decoder_check reports TSD_EDEVICE.
  * Asynchronous on cuda_stream (must be the decoder's stream order, see
  * above); the device arrays are borrowed until the stream passes this call.
  * T <= max_T and n <= max_streams, else TSD_EINVAL. */

@@ -150,8 +150,6 @@ tsd_status create_impl(const tsd_decoder_cfg* cfg, const void* W_out_bf16, const
   if (c.V < 1 || c.V > 16384) return fail(TSD_EINVAL, "tsd_decoder_create: V=%d out of range [1, 16384]", c.V);
   if (c.H < 64 || c.H > 8192 || c.H % 64) return fail(TSD_EINVAL, "tsd_decoder_create: H=%d must be a multiple of 64 in [64, 8192]", c.H);
   if (c.beam_k < 1 || c.beam_k > 8) return fail(TSD_EINVAL, "tsd_decoder_create: beam_k=%d outside [1, 8]", c.beam_k);
-  if (c.beam_k > 1 && c.max_symbols != 1)
-    return fail(TSD_EINVAL, "tsd_decoder_create: beam search emits at most one label per frame (max_symbols must be 1)");
   if (c.beam_k > 1 && ((c.V + 1 + kNPad - 1) / kNPad * kNPad / 64) * c.beam_k > 512)
     return fail(TSD_EINVAL, "tsd_decoder_create: beam_k * (V+1)/64 must be <= 512");
   if (c.max_symbols < 1 || c.max_symbols > 64) return fail(TSD_EINVAL, "tsd_decoder_create: max_symbols=%d out of range", c.max_symbols);
@@ -219,10 +217,18 @@ tsd_status create_impl(const tsd_decoder_cfg* cfg, const void* W_out_bf16, const
     if ((st = A.alloc(&bpart, (size_t)d->M_pad * (d->N_pad / 64) * (1 + c.beam_k))) || (st = A.alloc(&hscore, SK)) ||
         (st = A.alloc(&hlive, SK)) || (st = A.alloc(&hnode, SK)) || (st = A.alloc(&hlen, SK)) ||
         (st = A.alloc(&hhash, SK)) || (st = A.alloc(&ppar, pool)) || (st = A.alloc(&ptok, pool)) ||
-        (st = A.alloc(&pn, (size_t)c.max_streams))) {
+        (st = A.alloc(&pn, (size_t)c.max_streams)) || (st = A.alloc(&v.f_score, SK)) ||
+        (st = A.alloc(&v.f_live, SK)) || (st = A.alloc(&v.f_node, SK)) || (st = A.alloc(&v.f_len, SK)) ||
+        (st = A.alloc(&v.f_last, SK)) || (st = A.alloc(&v.f_lml, SK)) || (st = A.alloc(&v.f_trl, SK)) ||
+        (st = A.alloc(&v.f_lmc, SK * kLmChain)) || (st = A.alloc(&v.f_trc, SK * kTrChain)) ||
+        (st = A.alloc(&v.f_hash, SK)) || (st = A.alloc(&v.b_frame, (size_t)c.max_streams)) ||
+        (st = A.alloc(&v.b_exp, (size_t)c.max_streams))) {
       A.release();
       return st;
     }
+    TSD_CUDA(cudaMemsetAsync(v.f_live, 0, SK * sizeof(int32_t), s));
+    TSD_CUDA(cudaMemsetAsync(v.b_frame, 0, (size_t)c.max_streams * sizeof(int32_t), s));
+    TSD_CUDA(cudaMemsetAsync(v.b_exp, 0, (size_t)c.max_streams * sizeof(int32_t), s));
     if (!bpart || !hscore || !hlive || !hnode || !hlen || !hhash || !ppar || !ptok || !pn) {
       A.release();
       return fail(TSD_ENOMEM, "tsd_decoder_create: beam state not allocated");

@@ -75,6 +75,16 @@ struct DecView {
   int32_t* pool_tok;    // [slots][pool_cap] label of the node
   int32_t* pool_n;      // [slots] nodes used
   int32_t pool_cap;
+  // beam search with several labels per frame: the frame-exit set (same
+  // layout as the hypotheses, [slots][K]) and each stream's frame and
+  // expansion within it
+  double* f_score;
+  int32_t *f_live, *f_node, *f_len, *f_last, *f_lml, *f_trl;
+  int32_t* f_lmc;       // [slots][K][kLmChain]
+  int32_t* f_trc;       // [slots][K][kTrChain]
+  unsigned long long* f_hash;
+  int32_t* b_frame;     // [slots] frame of the chunk the beam is in (T: done)
+  int32_t* b_exp;       // [slots] expansions taken in that frame
   int32_t topk;       // entries per row and tile in bpart: beam width, or prune_k
   int32_t prune;      // prune_k (0: fusion over every label)
   int32_t n_lm;       // n-gram LMs fused (0: none; several: greedy only)

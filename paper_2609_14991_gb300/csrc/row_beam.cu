@@ -1,20 +1,28 @@
 // Beam-search row pass: one cluster of K CTAs per stream, K hypotheses per
-// stream.  The cluster's first CTA does steps 1-3; then every CTA k of the
-// cluster builds step 4 for survivor k, reading that survivor's chains from
-// the first CTA's shared memory.
+// stream.  The cluster's first CTA does steps 1-5; then every CTA k of the
+// cluster builds step 6 for beam member k, reading its chains from the
+// first CTA's shared memory.
 //
-// At label step s (frame s of the chunk; one label or blank per frame) it
-//   1. turns the joint kernel's per-tile partials of frame s-1 into each live
-//      hypothesis's log-sum-exp and its K best extensions (blank keeps the
-//      labels, label v appends v), scored hypothesis score + fused value -
-//      log-sum-exp (Eq. 1 summed along the hypothesis);
-//   2. keeps the global top K of those candidates by (score desc,
-//      hypothesis asc, label asc) and merges candidates with equal label
-//      sequences by log-sum-exp of their scores, in order of first appearance
-//      (so fewer than K may survive);
-//   3. advances each survivor's LM and phrase-trie suffix chains from its
-//      parent's (independent per-level searches, as in the greedy pass);
-//   4. writes the joint input and the fusion bias row of every survivor.
+// The search is frame-synchronous with at most S = max_symbols labels per
+// frame: each label step is one expansion of the hypotheses still in their
+// frame (set A).  At a step the first CTA
+//   1. turns the joint kernel's per-tile partials into each hypothesis of A's
+//      log-sum-exp and its K best extensions (blank keeps the labels, label v
+//      appends v), scored hypothesis score + fused value - log-sum-exp (Eq. 1
+//      summed along the hypothesis);
+//   2. keeps the top K of those candidates by (score desc, hypothesis asc,
+//      label asc) and sends each, in that order, to the frame-exit set F
+//      (the blank, or a label at the frame's S-th expansion) or to the next A,
+//      merging equal label sequences within a set by log-sum-exp of their
+//      scores (F also holds the earlier expansions' exits);
+//   3. searches each new label in its parent's LM and phrase-trie suffix
+//      chains (independent per-level searches, as in the greedy pass);
+//   4. builds the new hypotheses' chains;
+//   5. keeps F's K best in insertion order; when A is empty or the S-th
+//      expansion is done the frame ends and F is the beam of the next frame;
+//      commits the beam, F and the stream's frame and expansion counters.
+// With S = 1 every kept candidate leaves the frame: one label or blank per
+// frame, the top K of the K (V+1) extensions merged.
 // Label sequences live in a per-stream pool of (parent, label) nodes; two
 // candidates are the same sequence when their lengths and rolling hashes
 // agree and their node chains compare equal label by label.
@@ -106,7 +114,24 @@ __global__ void __launch_bounds__(kRowThreads) k_row_beam(DecView d, int step, i
   __shared__ int sr_uni[kMaxK], sr_rc[kMaxK], sr_rn[kMaxK];
   __shared__ row::ChainRecs rc;
 
-  __shared__ int m_cnt, m_lml, m_trl, m_last;  // survivor crank, copied from the first CTA
+  // frame-exit set F as loaded (entries of earlier expansions of this frame)
+  __shared__ int e_cnt, e_node[kMaxK], e_len[kMaxK], e_last[kMaxK], e_lml[kMaxK], e_trl[kMaxK];
+  __shared__ double e_score[kMaxK];
+  __shared__ unsigned long long e_hash[kMaxK];
+  __shared__ int e_lm[kMaxK][kLmChain], e_tr[kMaxK][kTrChain];
+  __shared__ int n_dst[kMaxK];  // new record goes to F (1) or stays in the frame (0)
+  // the beam after this step (its members' joint inputs and bias rows are built)
+  __shared__ int a_cnt, a_build, a_frame;
+  __shared__ int a_node[kMaxK], a_len[kMaxK], a_last[kMaxK], a_lml[kMaxK], a_trl[kMaxK];
+  __shared__ double a_score[kMaxK];
+  __shared__ unsigned long long a_hash[kMaxK];
+  __shared__ int a_lm[kMaxK][kLmChain], a_tr[kMaxK][kTrChain];
+  __shared__ int f_cnt, f_src[kMaxK];  // F after this step: entry (>= 0 new record j, <= -2 loaded entry -2-j)
+  __shared__ int q_src[2 * kMaxK];     // F before pruning, in insertion order
+  __shared__ double q_score[2 * kMaxK];
+  __shared__ int s_bt, s_be, s_done;
+
+  __shared__ int m_cnt, m_lml, m_trl, m_last, m_frame;  // member crank, copied from the first CTA
   __shared__ int m_lm[kLmChain], m_tr[kTrChain];
   if (crank == 0) {
   // previous state of this stream's hypotheses (written by the previous row
@@ -132,6 +157,14 @@ __global__ void __launch_bounds__(kRowThreads) k_row_beam(DecView d, int step, i
     o_lml[tid] = d.has_lm ? __ldcg(d.s_lm_len + h) : 0;
     o_trl[tid] = d.has_tr ? __ldcg(d.s_tr_len + h) : 0;
   }
+  if (tid == K) {
+    // frame and expansion of this stream (reset at the chunk's first step;
+    // a replay redoes one expansion of the final beam)
+    s_bt = (step == 0 || mode == 2) ? 0 : __ldcg(d.b_frame + slot);
+    s_be = (step == 0 || mode == 2) ? 0 : __ldcg(d.b_exp + slot);
+    s_done = (step > 0 && mode != 2 && s_bt >= T) ? 1 : 0;
+    e_cnt = 0;
+  }
   row::block_sync();
   for (int i = tid; i < K * kLmChain; i += kRowThreads) {
     const int k = i / kLmChain, l = i % kLmChain;
@@ -141,11 +174,38 @@ __global__ void __launch_bounds__(kRowThreads) k_row_beam(DecView d, int step, i
     const int k = i / kTrChain, l = i % kTrChain;
     if (l < o_trl[k]) o_tr[k][l] = __ldcg(d.s_tr_chain + (size_t)(hb + k) * kTrChain + l);
   }
+  const int S = d.max_sym;
+  if (S > 1 && step > 0 && !s_done && s_be > 0) {
+    // F holds the exits of this frame's earlier expansions
+    if (tid < K) {
+      const int h = hb + tid;
+      const int live = __ldcg(d.f_live + h);
+      if (live) {
+        e_node[tid] = __ldcg(d.f_node + h);
+        e_len[tid] = __ldcg(d.f_len + h);
+        e_last[tid] = __ldcg(d.f_last + h);
+        e_score[tid] = __ldcg(d.f_score + h);
+        e_hash[tid] = __ldcg(d.f_hash + h);
+        e_lml[tid] = __ldcg(d.f_lml + h);
+        e_trl[tid] = __ldcg(d.f_trl + h);
+      }
+      if (live) atomicAdd(&e_cnt, 1);  // F is stored compact: live entries first
+    }
+    row::block_sync();
+    for (int i = tid; i < K * kLmChain; i += kRowThreads) {
+      const int k = i / kLmChain, l = i % kLmChain;
+      if (k < e_cnt && l < e_lml[k]) e_lm[k][l] = __ldcg(d.f_lmc + (size_t)(hb + k) * kLmChain + l);
+    }
+    for (int i = tid; i < K * kTrChain; i += kRowThreads) {
+      const int k = i / kTrChain, l = i % kTrChain;
+      if (k < e_cnt && l < e_trl[k]) e_tr[k][l] = __ldcg(d.f_trc + (size_t)(hb + k) * kTrChain + l);
+    }
+  }
   row::block_sync();
   asm volatile("griddepcontrol.wait;" ::: "memory");
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
-  if (step > 0) {
+  if (step > 0 && !s_done) {
     // 1. per live hypothesis (warp k): log-sum-exp and its K best extensions
     if (warp < K) {
       const int k = warp;
@@ -227,22 +287,38 @@ __global__ void __launch_bounds__(kRowThreads) k_row_beam(DecView d, int step, i
         s_sel[nsel++] = best;
       }
       s_nsel = nsel;
+      const bool last_exp = s_be >= S - 1;
       int cnt = 0;
       int pool_used = __ldcg(d.pool_n + slot);
       for (int i = 0; i < nsel; ++i) {
         const int c = s_sel[i], p = c / K, y = c_tok[c];
+        const int dst = (y == V || last_exp) ? 1 : 0;
         const int len = o_len[p] + (y != V ? 1 : 0);
         const unsigned long long hsh = (y != V) ? hash_push(o_hash[p], y) : o_hash[p];
         int into = -1;
-        for (int j = 0; j < cnt; ++j) {
-          if (n_len[j] != len || n_hash[j] != hsh) continue;
-          const int pj = n_par[j];
-          if (seq_equal(pool_par, pool_tok, o_node[p], y != V ? y : -1, o_node[pj], n_tok[j] != V ? n_tok[j] : -1, cap)) {
-            into = j;
-            break;
+        if (dst == 1) {
+          for (int j = 0; j < e_cnt; ++j) {
+            if (e_len[j] != len || e_hash[j] != hsh) continue;
+            if (seq_equal(pool_par, pool_tok, o_node[p], y != V ? y : -1, e_node[j], -1, cap)) {
+              into = -2 - j;
+              break;
+            }
           }
         }
-        if (into >= 0) {
+        if (into == -1) {
+          for (int j = 0; j < cnt; ++j) {
+            if (n_dst[j] != dst || n_len[j] != len || n_hash[j] != hsh) continue;
+            const int pj = n_par[j];
+            if (seq_equal(pool_par, pool_tok, o_node[p], y != V ? y : -1, o_node[pj], n_tok[j] != V ? n_tok[j] : -1,
+                          cap)) {
+              into = j;
+              break;
+            }
+          }
+        }
+        if (into <= -2) {
+          e_score[-2 - into] = log_add(e_score[-2 - into], c_score[c]);
+        } else if (into >= 0) {
           n_score[into] = log_add(n_score[into], c_score[c]);
         } else {
           into = cnt++;
@@ -251,6 +327,7 @@ __global__ void __launch_bounds__(kRowThreads) k_row_beam(DecView d, int step, i
           n_score[into] = c_score[c];
           n_len[into] = len;
           n_hash[into] = hsh;
+          n_dst[into] = dst;
         }
         s_into[i] = into;
       }
@@ -366,63 +443,173 @@ __global__ void __launch_bounds__(kRowThreads) k_row_beam(DecView d, int step, i
       }
     }
     row::block_sync();
+    // 5. F keeps its K best (score desc, earlier first) in insertion order:
+    //    loaded entries, then this step's exits.  The frame ends when nothing
+    //    stays in it or after its S-th expansion; F is then the beam.
+    if (tid == 0) {
+      const bool last_exp = s_be >= S - 1;
+      int nf = 0;
+      for (int j = 0; j < e_cnt; ++j) { q_src[nf] = -2 - j; q_score[nf++] = e_score[j]; }
+      for (int j = 0; j < cnt; ++j)
+        if (n_dst[j] == 1) { q_src[nf] = j; q_score[nf++] = n_score[j]; }
+      int fc = 0;
+      if (nf <= K) {
+        for (int x = 0; x < nf; ++x) f_src[fc++] = q_src[x];
+      } else {
+        for (int x = 0; x < nf; ++x) {
+          int rank = 0;
+          for (int y = 0; y < nf; ++y)
+            if (q_score[y] > q_score[x] || (q_score[y] == q_score[x] && y < x)) ++rank;
+          if (rank < K) f_src[fc++] = q_src[x];
+        }
+      }
+      f_cnt = fc;
+      int na = 0;
+      for (int j = 0; j < cnt; ++j) na += n_dst[j] == 0 ? 1 : 0;
+      const bool frame_end = na == 0 || last_exp;
+      if (frame_end) {
+        for (int k = 0; k < fc; ++k) s_into[k] = f_src[k];  // the beam's sources
+        a_cnt = fc;
+        f_cnt = 0;
+        s_bt = s_bt + 1;
+        s_be = 0;
+      } else {
+        int k = 0;
+        for (int j = 0; j < cnt; ++j)
+          if (n_dst[j] == 0) s_into[k++] = j;
+        a_cnt = k;
+        s_be = s_be + 1;
+      }
+      a_frame = s_bt;
+      a_build = s_bt < T ? a_cnt : 0;  // a finished stream evaluates nothing more
+    }
+    row::block_sync();
+    // the beam's records from this step's new records (>= 0) or loaded F
+    // entries; chains copied by the whole block
+    if (tid < a_cnt) {
+      const int k = tid, sidx = s_into[k];
+      if (sidx >= 0) {
+        a_node[k] = n_node[sidx]; a_len[k] = n_len[sidx]; a_last[k] = n_last[sidx]; a_score[k] = n_score[sidx];
+        a_hash[k] = n_hash[sidx]; a_lml[k] = n_lml[sidx]; a_trl[k] = n_trl[sidx];
+      } else {
+        const int j = -2 - sidx;
+        a_node[k] = e_node[j]; a_len[k] = e_len[j]; a_last[k] = e_last[j]; a_score[k] = e_score[j];
+        a_hash[k] = e_hash[j]; a_lml[k] = e_lml[j]; a_trl[k] = e_trl[j];
+      }
+    }
+    for (int i = tid; i < a_cnt * (kLmChain + kTrChain); i += kRowThreads) {
+      const int k = i / (kLmChain + kTrChain), l = i % (kLmChain + kTrChain), sidx = s_into[k];
+      const int j = sidx >= 0 ? sidx : -2 - sidx;
+      if (l < kLmChain) a_lm[k][l] = sidx >= 0 ? n_lm[j][l] : e_lm[j][l];
+      else a_tr[k][l - kLmChain] = sidx >= 0 ? n_tr[j][l - kLmChain] : e_tr[j][l - kLmChain];
+    }
+    row::block_sync();
   } else {
-    // frame 0 of the chunk: the hypotheses carried over from the last chunk
+    // the chunk's first step, or a stream that finished its frames: the beam
+    // as stored (at the first step, the hypotheses carried over)
     if (tid == 0) {
       int cnt = 0;
       for (int k = 0; k < K; ++k) cnt += o_live[k] ? 1 : 0;
-      n_cnt = cnt;
+      a_cnt = cnt;
+      f_cnt = 0;
+      a_frame = s_bt;
+      a_build = s_done ? 0 : cnt;
     }
     if (tid < K) {
       const int k = tid;
-      n_par[k] = k;
-      n_tok[k] = V;
-      n_score[k] = o_score[k];
-      n_node[k] = o_node[k];
-      n_len[k] = o_len[k];
-      n_hash[k] = o_hash[k];
-      n_last[k] = o_last[k];
-      n_lml[k] = o_lml[k];
-      n_trl[k] = o_trl[k];
-      for (int l = 0; l < o_lml[k]; ++l) n_lm[k][l] = o_lm[k][l];
-      for (int l = 0; l < o_trl[k]; ++l) n_tr[k][l] = o_tr[k][l];
+      a_node[k] = o_node[k];
+      a_len[k] = o_len[k];
+      a_last[k] = o_last[k];
+      a_score[k] = o_score[k];
+      a_hash[k] = o_hash[k];
+      a_lml[k] = o_lml[k];
+      a_trl[k] = o_trl[k];
+    }
+    for (int i = tid; i < K * (kLmChain + kTrChain); i += kRowThreads) {
+      const int k = i / (kLmChain + kTrChain), l = i % (kLmChain + kTrChain);
+      if (l < kLmChain) a_lm[k][l] = o_lm[k][l];
+      else a_tr[k][l - kLmChain] = o_tr[k][l - kLmChain];
+    }
+    if (d.cap_rows && step > 0 && step - 1 < d.cap_steps && commit && tid < K) {
+      int* cr = d.cap_rows + ((size_t)(step - 1) * P->n * K + (size_t)b * K + tid) * 4;
+      cr[0] = -1; cr[1] = -1; cr[2] = 0; cr[3] = -1;
     }
     row::block_sync();
   }
-  const int cnt = n_cnt;
+  const int cnt = a_cnt;
 
-  // 5. commit the survivors (compact, first cnt slots) and retire the rest
-  if (commit && step > 0) {
-    if (tid < K) {
+  // commit: the beam (compact, first cnt slots), F, and the counters
+  if (commit && !(step > 0 && s_done)) {
+    if (step > 0 && tid < K) {
       const int h = hb + tid;
       const bool live = tid < cnt;
       d.h_live[h] = live ? 1 : 0;
       if (live) {
-        d.h_score[h] = n_score[tid];
-        d.h_node[h] = n_node[tid];
-        d.h_len[h] = n_len[tid];
-        d.h_hash[h] = n_hash[tid];
-        d.s_last[h] = n_last[tid];
-        if (d.has_lm) d.s_lm_len[h] = n_lml[tid];
-        if (d.has_tr) d.s_tr_len[h] = n_trl[tid];
+        d.h_score[h] = a_score[tid];
+        d.h_node[h] = a_node[tid];
+        d.h_len[h] = a_len[tid];
+        d.h_hash[h] = a_hash[tid];
+        d.s_last[h] = a_last[tid];
+        if (d.has_lm) d.s_lm_len[h] = a_lml[tid];
+        if (d.has_tr) d.s_tr_len[h] = a_trl[tid];
       }
     }
-    for (int i = tid; i < cnt * kLmChain; i += kRowThreads) {
-      const int k = i / kLmChain, l = i % kLmChain;
-      if (l < n_lml[k]) d.s_lm_chain[(size_t)(hb + k) * kLmChain + l] = n_lm[k][l];
+    if (step > 0) {
+      for (int i = tid; i < cnt * kLmChain; i += kRowThreads) {
+        const int k = i / kLmChain, l = i % kLmChain;
+        if (l < a_lml[k]) d.s_lm_chain[(size_t)(hb + k) * kLmChain + l] = a_lm[k][l];
+      }
+      for (int i = tid; i < cnt * kTrChain; i += kRowThreads) {
+        const int k = i / kTrChain, l = i % kTrChain;
+        if (l < a_trl[k]) d.s_tr_chain[(size_t)(hb + k) * kTrChain + l] = a_tr[k][l];
+      }
     }
-    for (int i = tid; i < cnt * kTrChain; i += kRowThreads) {
-      const int k = i / kTrChain, l = i % kTrChain;
-      if (l < n_trl[k]) d.s_tr_chain[(size_t)(hb + k) * kTrChain + l] = n_tr[k][l];
+    if (S > 1) {
+      // F (compact) for the frame's next expansion
+      if (tid < K) {
+        const int h = hb + tid, k = tid;
+        const bool live = k < f_cnt;
+        d.f_live[h] = live ? 1 : 0;
+        if (live) {
+          const int sidx = f_src[k];
+          const bool nw = sidx >= 0;
+          const int j = nw ? sidx : -2 - sidx;
+          d.f_score[h] = nw ? n_score[j] : e_score[j];
+          d.f_node[h] = nw ? n_node[j] : e_node[j];
+          d.f_len[h] = nw ? n_len[j] : e_len[j];
+          d.f_hash[h] = nw ? n_hash[j] : e_hash[j];
+          d.f_last[h] = nw ? n_last[j] : e_last[j];
+          d.f_lml[h] = nw ? n_lml[j] : e_lml[j];
+          d.f_trl[h] = nw ? n_trl[j] : e_trl[j];
+        }
+      }
+      for (int i = tid; i < f_cnt * (kLmChain + kTrChain); i += kRowThreads) {
+        const int k = i / (kLmChain + kTrChain), l = i % (kLmChain + kTrChain);
+        const int sidx = f_src[k];
+        const bool nw = sidx >= 0;
+        const int j = nw ? sidx : -2 - sidx;
+        if (l < kLmChain) {
+          if (l < (nw ? n_lml[j] : e_lml[j]))
+            d.f_lmc[(size_t)(hb + k) * kLmChain + l] = nw ? n_lm[j][l] : e_lm[j][l];
+        } else {
+          const int q = l - kLmChain;
+          if (q < (nw ? n_trl[j] : e_trl[j]))
+            d.f_trc[(size_t)(hb + k) * kTrChain + q] = nw ? n_tr[j][q] : e_tr[j][q];
+        }
+      }
+    }
+    if (tid == 0) {
+      d.b_frame[slot] = s_bt;
+      d.b_exp[slot] = s_be;
     }
   }
   if (mode == 1) {
     if (tid == 0) {
       int best = 0;
       for (int j = 1; j < cnt; ++j)
-        if (n_score[j] > n_score[best]) best = j;
-      P->out_count[b] = cnt ? n_len[best] : 0;
-      P->out_score[(size_t)b * T * d.max_sym] = cnt ? (float)n_score[best] : 0.f;
+        if (a_score[j] > a_score[best]) best = j;
+      P->out_count[b] = cnt ? a_len[best] : 0;
+      P->out_score[(size_t)b * T * d.max_sym] = cnt ? (float)a_score[best] : 0.f;
     }
   }
   // Algorithmic bytes (counted when timing): the K hypotheses' partials and state
@@ -442,14 +629,16 @@ __global__ void __launch_bounds__(kRowThreads) k_row_beam(DecView d, int step, i
   //    until every CTA has its copy.
   cluster.sync();
   {
-    const int* rcnt = cluster.map_shared_rank(&n_cnt, 0);
-    const int* rlml = cluster.map_shared_rank(&n_lml[0], 0);
-    const int* rtrl = cluster.map_shared_rank(&n_trl[0], 0);
-    const int* rlast = cluster.map_shared_rank(&n_last[0], 0);
-    const int* rlm = cluster.map_shared_rank(&n_lm[0][0], 0);
-    const int* rtr = cluster.map_shared_rank(&n_tr[0][0], 0);
+    const int* rcnt = cluster.map_shared_rank(&a_build, 0);
+    const int* rframe = cluster.map_shared_rank(&a_frame, 0);
+    const int* rlml = cluster.map_shared_rank(&a_lml[0], 0);
+    const int* rtrl = cluster.map_shared_rank(&a_trl[0], 0);
+    const int* rlast = cluster.map_shared_rank(&a_last[0], 0);
+    const int* rlm = cluster.map_shared_rank(&a_lm[0][0], 0);
+    const int* rtr = cluster.map_shared_rank(&a_tr[0][0], 0);
     if (tid == 0) {
       m_cnt = *rcnt;
+      m_frame = *rframe;
       m_lml = rlml[crank];
       m_trl = rtrl[crank];
       m_last = rlast[crank];
@@ -461,7 +650,7 @@ __global__ void __launch_bounds__(kRowThreads) k_row_beam(DecView d, int step, i
   if (crank >= m_cnt) return;
   const int r = b * K + crank;
   const int Tn = __ldcg(&P->T);
-  const uint16_t* enc_row = P->enc + ((size_t)b * Tn + min(step, Tn - 1)) * d.H;
+  const uint16_t* enc_row = P->enc + ((size_t)b * Tn + min(m_frame, Tn - 1)) * d.H;
   row::bias_prepare(d, m_lm, m_lml, m_tr, m_trl, rc, lmv, dep);
   row::build_joint_input(d, enc_row, m_last, r);
   row::bias_finish(d, m_lml, m_trl, rc, P->lambda, P->beta, d.bias + (size_t)r * d.N_pad, lmv, dep);

@@ -29,6 +29,14 @@ SCORE_TOL = 1e-4  # fused scores, fp32 on the GPU vs double in the oracle
 LOGIT_TOL = 2e-2  # joint logits vs the oracle's double product of the same bf16 inputs
 
 
+def bf16_bits(x) -> np.ndarray:
+    """float32 -> bf16 bit patterns, round to nearest even."""
+    u = np.asarray(x, dtype=np.float32).view(np.uint32).astype(np.uint64)
+    keep, rest = u >> 16, u & 0xFFFF
+    keep = keep + ((rest > 0x8000) | ((rest == 0x8000) & (keep & 1 == 1)))
+    return keep.astype(np.uint16)
+
+
 class Inputs:
     def __init__(self, w: synth.Workload, lmA=None, ph=None, with_lm=True, with_boost=True):
         self.w = w
@@ -177,9 +185,10 @@ def replay_beam_stream(inp: Inputs, run: GpuRun, i: int, olm, obo, model) -> Dic
     out = {"steps": 0, "mismatch": 0, "near_tie": 0, "max_score_diff": 0.0, "inconsistent": 0, "state_errors": []}
     frames = 0
     for c in range(len(run.chunks)):
-        sel = run.beam_sel[c][:, i * K:(i + 1) * K, :]  # [T, K, 4]
+        sel = run.beam_sel[c][:, i * K:(i + 1) * K, :]  # [steps, K, 4]: one row per expansion
         rep = oracle.beam_chunk_follow(st, model, olm, obo, run.enc[c][i], inp.lam, inp.beta, K,
-                                       sel[:, :, 0], sel[:, :, 1], sel[:, :, 2].view(np.float32), GAP_TOL)
+                                       sel[:, :, 0], sel[:, :, 1], sel[:, :, 2].view(np.float32), GAP_TOL,
+                                       S=w.max_sym)
         frames += run.T
         out["steps"] += int(rep[oracle.REP_STEPS])
         out["mismatch"] += int(rep[oracle.REP_MISMATCH])

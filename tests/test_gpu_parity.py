@@ -140,6 +140,37 @@ def test_beam_small_exhaustive_against_free_oracle():
     pu.assert_reports(pu.replay_beam(inp, run, range(w.B)))
 
 
+@pytest.mark.parametrize("S", [2, 5])
+def test_beam_several_labels_per_frame(S):
+    """Beam search with up to S labels per frame (frame-synchronous): every
+    expansion's kept candidates checked and followed by the oracle, the
+    surviving label sequences and scores compared after every chunk."""
+    for K in (2, 4):
+        w = synth.scaled(synth.WORKLOADS[0], V=15, H=64, B=4, T=7, beam=K, max_sym=S, lm_total=60)
+        inp = pu.Inputs(w, lmA=synth.ngram_lm(7, 15, 3, 60, 1.1), ph=synth.phrases(7, 15, 3, 1, 3, 0.0))
+        run = pu.GpuRun(inp, range(w.B), 3, capture_steps=w.T * S)
+        pu.assert_reports(pu.replay_beam(inp, run, range(w.B)))
+    # a stronger blank: frames end after fewer than S expansions
+    w = synth.scaled(synth.WORKLOADS[0], V=15, H=64, B=3, T=8, beam=3, max_sym=S, lm_total=60)
+    inp = pu.Inputs(w, lmA=synth.ngram_lm(7, 15, 3, 60, 1.1), ph=synth.phrases(7, 15, 3, 1, 3, 0.0))
+    inp.W = inp.W.copy()
+    inp.W[:, w.V] = pu.bf16_bits(np.full(w.H, 2.5 / np.sqrt(w.H), dtype=np.float32))
+    run = pu.GpuRun(inp, range(w.B), 2, capture_steps=w.T * S)
+    reps = pu.replay_beam(inp, run, range(w.B))
+    pu.assert_reports(reps)
+    assert sum(r["steps"] for r in reps) < w.B * 2 * w.T * S  # some frames ended early
+
+
+def test_beam_several_labels_cfg3_shape():
+    """The beam workload's shapes (V+1 = 1025, H = 1024, 6-gram 20M LM, 5,000
+    phrases, K = 4) with up to 3 labels per frame, two chunks, three streams
+    checked."""
+    w = synth.scaled(synth.WORKLOADS[3], B=32, max_sym=3)
+    inp = pu.Inputs(w)
+    run = pu.GpuRun(inp, range(w.B), 2, capture_steps=w.T * 3)
+    pu.assert_reports(pu.replay_beam(inp, run, [0, 15, 31]))
+
+
 def _tokens(run, i):
     return np.concatenate([run.emitted(i, c)[0] for c in range(len(run.chunks))])
 
