@@ -346,6 +346,9 @@ def run_ours(args, w):
     dec = tsd.Decoder(w.V, w.H, torch.from_numpy(W.view(np.int16)).to(dev), torch.from_numpy(E.view(np.int16)).to(dev),
                       lm=None if lms else lm, lms=lms, boost=bo, max_symbols=w.max_sym, beam_k=w.beam,
                       max_streams=w.B, max_T=w.T, prune_k=args.prune_k, pred=pw)
+    for kv in args.set or []:
+        k, v = kv.split("=")
+        dec.set_option(k, int(v))
     slots = [dec.open() for _ in range(w.B)]
     slots_np = np.array(slots, dtype=np.int32)
     n_chunks = args.warmup + args.steps + 1
@@ -606,6 +609,7 @@ def run_ours(args, w):
             "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
             "config": dict(workload_config(w, lmA.total + sum(a.total for a, _ in extra), ph.n if ph else 0),
                            **variant_config(args, w, extra),
+                           **({"options": args.set} if args.set else {}),
                            l2="flushed (256 MB write) before every timed step, outside the step's events",
                            parallelism=f"dp{ws} (independent streams per GPU)"),
             "e2e": {"value": e2e_val, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
@@ -652,6 +656,8 @@ def main():
                     help="pruned fusion over the acoustic model's k best outputs (0: every label)")
     ap.add_argument("--pred", type=int, default=0,
                     help="stateful form: an LSTM prediction network of this many units (0: stateless)")
+    ap.add_argument("--set", action="append", metavar="NAME=VALUE",
+                    help="a decoder tuning option (tsd_decoder_set_option), e.g. pdl=0 or joint_bn=128")
     ap.add_argument("--encoder", default=None, choices=sorted(synth.ENCODERS),
                     help="run the cache-aware encoder chunk step before the decode in every step")
     args = ap.parse_args()
