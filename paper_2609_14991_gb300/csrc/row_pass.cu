@@ -125,7 +125,12 @@ __device__ unsigned long long bias_multi(const DecView& d, int L, const int (*lm
 // mode: 0 = label step, 1 = final step (apply the last decision only),
 // 2 = replay (redo the step's work without committing any state or output;
 // used only to time the kernel in isolation).
+// VAR bit 0: the stateful form (LSTM input rows instead of the joint input);
+// bit 1: several LMs.  Each combination is its own instantiation, so the
+// common one (neither) carries none of the other paths' code or registers.
+template <int VAR>
 __global__ void __launch_bounds__(kRowThreads, 7) k_row(DecView d, int step, int mode) {
+  constexpr bool PRED = (VAR & 1) != 0, MULTI = (VAR & 2) != 0;
   const Params* __restrict__ P = d.params;
   const int r = blockIdx.x;
   const int V = d.V;
@@ -134,7 +139,7 @@ __global__ void __launch_bounds__(kRowThreads, 7) k_row(DecView d, int step, int
   extern __shared__ __align__(16) unsigned char smem[];
   // per-label scratch: LM value from the chain (NaN unset), with several LMs
   // also their weighted sum, then the trie depth of the goto
-  const int L = d.n_lm > 1 ? d.n_lm : 1;  // LM state blocks (1 without an LM)
+  const int L = (MULTI && d.n_lm > 1) ? d.n_lm : 1;  // LM state blocks (1 without an LM)
   float* lmv = reinterpret_cast<float*>(smem);
   float* acc = lmv + d.V4;
   uint8_t* dep = reinterpret_cast<uint8_t*>(lmv + (L > 1 ? 2 : 1) * d.V4);
@@ -374,7 +379,7 @@ __global__ void __launch_bounds__(kRowThreads, 7) k_row(DecView d, int step, int
     row::block_sync();
   }
 
-  if (d.pred_D) {
+  if (PRED) {
     // Stateful form: the prediction network reads the label just emitted
     // (or, at a stream's first step, the start of sequence) and the row's h
     // from before this step; the LSTM kernel after this one runs the cell.
@@ -442,11 +447,11 @@ __global__ void __launch_bounds__(kRowThreads, 7) k_row(DecView d, int step, int
       if (tid >= 32 && tid - 32 < nt)
         d.s_tr_rec[(size_t)slot * kTrChain + tid - 32] = make_int4(rc.tb[tid - 32], rc.tc[tid - 32], rc.td[tid - 32], 0);
     }
-    if (!d.pred_D) row::build_joint_input(d, s_enc + ((size_t)r * T + t) * d.H, s_last, r);
+    if (!PRED) row::build_joint_input(d, s_enc + ((size_t)r * T + t) * d.H, s_last, r);
     row::bias_finish(d, nl, nt, rc, s_lam, s_beta, d.bias + (size_t)r * d.N_pad, lmv, dep);
     if (counting && tid == 0) lm_bytes = lm_level_bytes(rc, nl, s_y != V && evaluated);
-  } else {
-    if (!d.pred_D) row::build_joint_input(d, s_enc + ((size_t)r * T + t) * d.H, s_last, r);
+  } else if (MULTI) {
+    if (!PRED) row::build_joint_input(d, s_enc + ((size_t)r * T + t) * d.H, s_last, r);
     lm_bytes = bias_multi(d, L, s_lm, s_lm_len, s_tr, nt, rc, s_lam, s_beta, d.bias + (size_t)r * d.N_pad, lmv,
                           acc, dep, counting, s_y != V && evaluated);
     nl = 0;
@@ -538,7 +543,11 @@ void launch_defaults(const DecView& d, cudaStream_t s) { k_defaults<<<(d.V4 + 25
 cudaError_t prepare_kernels(size_t row_smem) {
   // dynamic scratch plus the kernel's static shared memory may pass the
   // 48 KB default even when the scratch alone does not
-  return cudaFuncSetAttribute(k_row, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)row_smem);
+  cudaError_t e = cudaFuncSetAttribute(k_row<0>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)row_smem);
+  if (e == cudaSuccess) e = cudaFuncSetAttribute(k_row<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)row_smem);
+  if (e == cudaSuccess) e = cudaFuncSetAttribute(k_row<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)row_smem);
+  if (e == cudaSuccess) e = cudaFuncSetAttribute(k_row<3>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)row_smem);
+  return e;
 }
 
 void launch_repack(const uint16_t* W, uint16_t* Wt, int H, int N, int N_pad, cudaStream_t s) {
@@ -600,7 +609,11 @@ void launch_row(const DecView& d, int M, int step, int mode, size_t smem, cudaSt
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = pdl ? 1 : 0;
-  cudaLaunchKernelEx(&cfg, k_row, d, step, mode);
+  const int var = (d.pred_D ? 1 : 0) | (d.n_lm > 1 ? 2 : 0);
+  if (var == 0) cudaLaunchKernelEx(&cfg, k_row<0>, d, step, mode);
+  else if (var == 1) cudaLaunchKernelEx(&cfg, k_row<1>, d, step, mode);
+  else if (var == 2) cudaLaunchKernelEx(&cfg, k_row<2>, d, step, mode);
+  else cudaLaunchKernelEx(&cfg, k_row<3>, d, step, mode);
 }
 
 }  // namespace tsd
