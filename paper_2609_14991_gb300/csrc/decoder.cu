@@ -317,6 +317,7 @@ tsd_status create_impl(const tsd_decoder_cfg* cfg, const void* W_out_bf16, const
     d->jtc = new (std::nothrow) JointTc();
     if (!d->jtc) return cleanup(fail(TSD_ENOMEM, "tsd_decoder_create: host allocation failed"));
     d->sms = sms;
+    d->view.sms = sms;
     const int bn = joint_tc_pick_bn(d->M_max, d->N_pad, sms);
     if ((ce = joint_tc_prepare(d->jtc, Abuf, d->M_pad, Wt, d->N_pad, c.H, bn, bias)) != cudaSuccess)
       return cleanup(cuda_fail(ce, "tsd_decoder_create: tensor-core GEMM setup (TMA descriptors)"));

@@ -88,6 +88,7 @@ struct DecView {
   int32_t topk;       // entries per row and tile in bpart: beam width, or prune_k
   int32_t prune;      // prune_k (0: fusion over every label)
   int32_t n_lm;       // n-gram LMs fused (0: none; several: greedy only)
+  int32_t sms;        // SMs of the device (launch shapes)
   int32_t lm_stride;  // hypothesis slots per LM in s_lm_len / s_lm_chain
   LmView lmx[kMaxLm]; // every LM; lmx[0] equals lm
   float lm_w[kMaxLm]; // relative weights: LM i enters Eq. 1 with lambda * lm_w[i]

@@ -126,10 +126,12 @@ __device__ unsigned long long bias_multi(const DecView& d, int L, const int (*lm
 // 2 = replay (redo the step's work without committing any state or output;
 // used only to time the kernel in isolation).
 // VAR bit 0: the stateful form (LSTM input rows instead of the joint input);
-// bit 1: several LMs.  Each combination is its own instantiation, so the
-// common one (neither) carries none of the other paths' code or registers.
+// bit 1: several LMs; bit 2: few rows (at most two CTAs per SM are needed,
+// so the kernel may use registers freely instead of fitting seven per SM).
+// Each combination is its own instantiation, so the common ones carry none
+// of the other paths' code or registers.
 template <int VAR>
-__global__ void __launch_bounds__(kRowThreads, 7) k_row(DecView d, int step, int mode) {
+__global__ void __launch_bounds__(kRowThreads, (VAR & 4) ? 2 : 7) k_row(DecView d, int step, int mode) {
   constexpr bool PRED = (VAR & 1) != 0, MULTI = (VAR & 2) != 0;
   const Params* __restrict__ P = d.params;
   const int r = blockIdx.x;
@@ -547,6 +549,7 @@ cudaError_t prepare_kernels(size_t row_smem) {
   if (e == cudaSuccess) e = cudaFuncSetAttribute(k_row<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)row_smem);
   if (e == cudaSuccess) e = cudaFuncSetAttribute(k_row<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)row_smem);
   if (e == cudaSuccess) e = cudaFuncSetAttribute(k_row<3>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)row_smem);
+  if (e == cudaSuccess) e = cudaFuncSetAttribute(k_row<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)row_smem);
   return e;
 }
 
@@ -610,7 +613,8 @@ void launch_row(const DecView& d, int M, int step, int mode, size_t smem, cudaSt
   cfg.attrs = attr;
   cfg.numAttrs = pdl ? 1 : 0;
   const int var = (d.pred_D ? 1 : 0) | (d.n_lm > 1 ? 2 : 0);
-  if (var == 0) cudaLaunchKernelEx(&cfg, k_row<0>, d, step, mode);
+  if (var == 0 && M <= 2 * d.sms) cudaLaunchKernelEx(&cfg, k_row<4>, d, step, mode);
+  else if (var == 0) cudaLaunchKernelEx(&cfg, k_row<0>, d, step, mode);
   else if (var == 1) cudaLaunchKernelEx(&cfg, k_row<1>, d, step, mode);
   else if (var == 2) cudaLaunchKernelEx(&cfg, k_row<2>, d, step, mode);
   else cudaLaunchKernelEx(&cfg, k_row<3>, d, step, mode);
