@@ -82,6 +82,9 @@ __device__ __forceinline__ bool cand_before(double s1, int h1, int t1, double s2
 
 // mode: 0 = label step, 1 = final step (apply the last frame's selection),
 // 2 = replay (redo the step without committing anything; for timing).
+// MS: several labels per frame (max_symbols > 1); without it the frame-exit
+// set and the expansion counter fold away at compile time.
+template <bool MS>
 __global__ void __launch_bounds__(kRowThreads) k_row_beam(DecView d, int step, int mode) {
   const Params* __restrict__ P = d.params;
   cooperative_groups::cluster_group cluster = cooperative_groups::this_cluster();
@@ -174,7 +177,7 @@ __global__ void __launch_bounds__(kRowThreads) k_row_beam(DecView d, int step, i
     const int k = i / kTrChain, l = i % kTrChain;
     if (l < o_trl[k]) o_tr[k][l] = __ldcg(d.s_tr_chain + (size_t)(hb + k) * kTrChain + l);
   }
-  const int S = d.max_sym;
+  const int S = MS ? d.max_sym : 1;
   if (S > 1 && step > 0 && !s_done && s_be > 0) {
     // F holds the exits of this frame's earlier expansions
     if (tid < K) {
@@ -697,7 +700,8 @@ void launch_row_beam(const DecView& d, int n, int step, int mode, size_t smem, c
   attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = pdl ? 2 : 1;
-  cudaLaunchKernelEx(&cfg, k_row_beam, d, step, mode);
+  if (d.max_sym > 1) cudaLaunchKernelEx(&cfg, k_row_beam<true>, d, step, mode);
+  else cudaLaunchKernelEx(&cfg, k_row_beam<false>, d, step, mode);
 }
 
 void launch_open_beam(const DecView& d, int slot, cudaStream_t s) { k_open_beam<<<1, 32, 0, s>>>(d, slot); }
@@ -705,7 +709,10 @@ void launch_open_beam(const DecView& d, int slot, cudaStream_t s) { k_open_beam<
 cudaError_t prepare_beam_kernels(size_t row_smem) {
   // dynamic scratch plus the kernel's static shared memory may pass the
   // 48 KB default even when the scratch alone does not
-  return cudaFuncSetAttribute(k_row_beam, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)row_smem);
+  cudaError_t e = cudaFuncSetAttribute(k_row_beam<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)row_smem);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(k_row_beam<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)row_smem);
+  return e;
 }
 
 }  // namespace tsd
