@@ -186,48 +186,48 @@ __global__ void __launch_bounds__(256) k_attn(AttnArgs a) {
     }
   }
   for (int rb = 0; rb < CR; rb += 16) {
-    // position term: SpT[s][t][r] = sum over half s of (q + v)[rb + r] . p(t - (C-1))
-    for (int item = tid; item < 2 * nrel; item += blockDim.x) {
-      const int s = item / nrel, t = item - s * nrel;
-      const float4* p = reinterpret_cast<const float4*>(a.pos_tab + (size_t)(t + a.cmax - C) * d + h * DH + s * HALF);
-      const float* q = Qv + rb * DH + s * HALF;
+    // position term SpT[s][t][r] = sum over half s of (q + v)[rb + r] . p(t - (C-1)),
+    // and content term ST[s][jj][r] = sum over half s of (q + u)[rb + r] . k_jj,
+    // as one list of items
+    for (int item = tid; item < 2 * nrel + 2 * W; item += blockDim.x) {
       float acc[16];
 #pragma unroll
       for (int r = 0; r < 16; ++r) acc[r] = 0.f;
+      float* dst;
+      if (item < 2 * nrel) {
+        const int s = item / nrel, t = item - s * nrel;
+        const float4* p = reinterpret_cast<const float4*>(a.pos_tab + (size_t)(t + a.cmax - C) * d + h * DH + s * HALF);
+        const float* q = Qv + rb * DH + s * HALF;
 #pragma unroll 2
-      for (int q4 = 0; q4 < HALF / 4; ++q4) {
-        const float4 pv = p[q4];
+        for (int q4 = 0; q4 < HALF / 4; ++q4) {
+          const float4 pv = p[q4];
 #pragma unroll
-        for (int r = 0; r < 16; ++r) {
-          const float4 qq = *reinterpret_cast<const float4*>(q + r * DH + 4 * q4);
-          acc[r] = fmaf(qq.x, pv.x, fmaf(qq.y, pv.y, fmaf(qq.z, pv.z, fmaf(qq.w, pv.w, acc[r]))));
+          for (int r = 0; r < 16; ++r) {
+            const float4 qq = *reinterpret_cast<const float4*>(q + r * DH + 4 * q4);
+            acc[r] = fmaf(qq.x, pv.x, fmaf(qq.y, pv.y, fmaf(qq.z, pv.z, fmaf(qq.w, pv.w, acc[r]))));
+          }
         }
-      }
-      float4* o = reinterpret_cast<float4*>(SpT + ((size_t)s * nrm + t) * 16);
-#pragma unroll
-      for (int r = 0; r < 16; r += 4) o[r / 4] = make_float4(acc[r], acc[r + 1], acc[r + 2], acc[r + 3]);
-    }
-    // content term: ST[s][jj][r] = sum over half s of (q + u)[rb + r] . k_jj
-    for (int item = tid; item < 2 * W; item += blockDim.x) {
-      const int s = item / W, jj = item - s * W;
-      const uint16_t* kr = Kb + (size_t)jj * KS + s * HALF;
-      const float* q = Qu + rb * DH + s * HALF;
-      float acc[16];
-#pragma unroll
-      for (int r = 0; r < 16; ++r) acc[r] = 0.f;
+        dst = SpT + ((size_t)s * nrm + t) * 16;
+      } else {
+        const int i2 = item - 2 * nrel;
+        const int s = i2 / W, jj = i2 - s * W;
+        const uint16_t* kr = Kb + (size_t)jj * KS + s * HALF;
+        const float* q = Qu + rb * DH + s * HALF;
 #pragma unroll 1
-      for (int o8 = 0; o8 < HALF / 8; ++o8) {
-        float kf[8];
-        bf16x8(*reinterpret_cast<const uint4*>(kr + 8 * o8), kf);
+        for (int o8 = 0; o8 < HALF / 8; ++o8) {
+          float kf[8];
+          bf16x8(*reinterpret_cast<const uint4*>(kr + 8 * o8), kf);
 #pragma unroll
-        for (int r = 0; r < 16; ++r) {
-          const float4 q0 = *reinterpret_cast<const float4*>(q + r * DH + 8 * o8);
-          const float4 q1 = *reinterpret_cast<const float4*>(q + r * DH + 8 * o8 + 4);
-          acc[r] = fmaf(q0.x, kf[0], fmaf(q0.y, kf[1], fmaf(q0.z, kf[2], fmaf(q0.w, kf[3], acc[r]))));
-          acc[r] = fmaf(q1.x, kf[4], fmaf(q1.y, kf[5], fmaf(q1.z, kf[6], fmaf(q1.w, kf[7], acc[r]))));
+          for (int r = 0; r < 16; ++r) {
+            const float4 q0 = *reinterpret_cast<const float4*>(q + r * DH + 8 * o8);
+            const float4 q1 = *reinterpret_cast<const float4*>(q + r * DH + 8 * o8 + 4);
+            acc[r] = fmaf(q0.x, kf[0], fmaf(q0.y, kf[1], fmaf(q0.z, kf[2], fmaf(q0.w, kf[3], acc[r]))));
+            acc[r] = fmaf(q1.x, kf[4], fmaf(q1.y, kf[5], fmaf(q1.z, kf[6], fmaf(q1.w, kf[7], acc[r]))));
+          }
         }
+        dst = ST + ((size_t)s * Wm + jj) * 16;
       }
-      float4* o = reinterpret_cast<float4*>(ST + ((size_t)s * Wm + jj) * 16);
+      float4* o = reinterpret_cast<float4*>(dst);
 #pragma unroll
       for (int r = 0; r < 16; r += 4) o[r / 4] = make_float4(acc[r], acc[r + 1], acc[r + 2], acc[r + 3]);
     }
@@ -243,17 +243,32 @@ __global__ void __launch_bounds__(256) k_attn(AttnArgs a) {
       ST[jj * 16 + r] = v;
     }
     __syncthreads();
-    if (tid < 16 && rb + tid < C) {  // softmax, one thread per query row
+    {
+      // softmax over the keys of each row: thread (row r = tid mod 16, j0 =
+      // tid / 16) takes keys j0, j0 + 16, ..; the 16 partial maxima and sums
+      // of a row meet in shared memory (the output buffer, free until below)
+      const int r = tid & 15, j0 = tid >> 4;
+      float* red = Op;  // [16][16] maxima, then [16][16] sums
       float m = -INFINITY;
-      for (int jj = 0; jj < W; ++jj) m = fmaxf(m, ST[jj * 16 + tid]);
+      for (int jj = j0; jj < W; jj += 16) m = fmaxf(m, ST[jj * 16 + r]);
+      red[j0 * 16 + r] = m;
+      __syncthreads();
+      float mm = -INFINITY;
+#pragma unroll
+      for (int k = 0; k < 16; ++k) mm = fmaxf(mm, red[k * 16 + r]);
       float z = 0.f;
-      for (int jj = 0; jj < W; ++jj) {
-        const float e = expf(ST[jj * 16 + tid] - m);
-        ST[jj * 16 + tid] = e;
+      for (int jj = j0; jj < W; jj += 16) {
+        const float e = expf(ST[jj * 16 + r] - mm);
+        ST[jj * 16 + r] = e;
         z += e;
       }
-      const float inv = 1.f / z;
-      for (int jj = 0; jj < W; ++jj) ST[jj * 16 + tid] *= inv;
+      red[256 + j0 * 16 + r] = z;
+      __syncthreads();
+      float zz = 0.f;
+#pragma unroll
+      for (int k = 0; k < 16; ++k) zz += red[256 + k * 16 + r];
+      const float inv = 1.f / zz;
+      for (int jj = j0; jj < W; jj += 16) ST[jj * 16 + r] *= inv;
     }
     __syncthreads();
     // output halves: Op[s][4g + r][4q + c] over the keys of half s
