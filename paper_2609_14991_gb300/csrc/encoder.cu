@@ -512,7 +512,14 @@ extern "C" tsd_status tsd_encoder_create(const tsd_encoder_cfg* cfg, const void*
     for (const void* p : ptrs)
       if (!p) return fail(TSD_EINVAL, "tsd_encoder_create: layer %d has a NULL weight", l);
   }
-  std::unique_ptr<tsd_encoder> e(new tsd_encoder());
+  struct Guard {  // on a failed create, let queued copies finish before the memory is released
+    std::unique_ptr<tsd_encoder> p;
+    cudaStream_t s;
+    ~Guard() {
+      if (p) cudaStreamSynchronize(s);
+    }
+  } guard{std::unique_ptr<tsd_encoder>(new tsd_encoder()), static_cast<cudaStream_t>(cuda_stream)};
+  tsd_encoder* const e = guard.p.get();
   e->cfg = c;
   TSD_CUDA(cudaGetDevice(&e->device));
   cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
@@ -593,7 +600,7 @@ extern "C" tsd_status tsd_encoder_create(const tsd_encoder_cfg* cfg, const void*
   TSD_CUDA(cudaStreamSynchronize(s));
   TSD_CUDA(cudaGetLastError());
   e->slot_open.assign((size_t)c.max_streams, 0);
-  *out = e.release();
+  *out = guard.p.release();
   return TSD_OK;
 }
 
@@ -601,16 +608,7 @@ extern "C" void tsd_encoder_free(tsd_encoder* e) {
   if (!e) return;
   set_device(e);
   cudaDeviceSynchronize();
-  for (auto& kv : e->graphs) {
-    if (kv.second.exec) cudaGraphExecDestroy(kv.second.exec);
-    for (cudaEvent_t ev : kv.second.ev) cudaEventDestroy(ev);
-  }
-  if (e->slots_host) cudaFreeHost(e->slots_host);
-  if (e->slots_ev) cudaEventDestroy(e->slots_ev);
-  if (e->cap_stream) cudaStreamDestroy(e->cap_stream);
-  e->arena.release();
-  cudaGetLastError();
-  delete e;
+  delete e;  // the destructor releases graphs, events, the stream and device memory
 }
 
 extern "C" tsd_status tsd_encoder_open(tsd_encoder* e, int32_t* slot_out) {

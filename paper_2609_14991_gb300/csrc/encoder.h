@@ -86,4 +86,17 @@ struct tsd_encoder {
   int timing = 0;
   double ms[3] = {0, 0, 0};
   int64_t launches[3] = {0, 0, 0};
+
+  // releases everything the encoder holds (also after a failed create)
+  ~tsd_encoder() {
+    for (auto& kv : graphs) {
+      if (kv.second.exec) cudaGraphExecDestroy(kv.second.exec);
+      for (cudaEvent_t ev : kv.second.ev) cudaEventDestroy(ev);
+    }
+    if (slots_host) cudaFreeHost(slots_host);
+    if (slots_ev) cudaEventDestroy(slots_ev);
+    if (cap_stream) cudaStreamDestroy(cap_stream);
+    arena.release();
+    cudaGetLastError();
+  }
 };
