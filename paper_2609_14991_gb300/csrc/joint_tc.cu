@@ -36,7 +36,7 @@ constexpr float kNegInf = -__builtin_huge_valf();
 // has its own buffer and the second half lands in the drained stages.
 template <int BN>
 struct Smem {
-  static constexpr int kStages = (BN == 256) ? 3 : (BN == 128 ? 4 : 6);
+  static constexpr int kStages = (BN == 256) ? 3 : (BN == 128 ? 4 : 8);
   static constexpr int kABytes = kBM * kBK * 2;
   static constexpr int kBBytes = BN * kBK * 2;
   static constexpr int kStageBytes = kABytes + kBBytes;
