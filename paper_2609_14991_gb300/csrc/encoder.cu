@@ -45,42 +45,50 @@ __device__ __forceinline__ float warp_max(float v) {
   return v;
 }
 
-// Layer norm of rows of the fp32 stream x [M][d] (one warp per row):
+// Layer norm of rows of the fp32 stream x [M][d] (one warp per row; the row
+// stays in registers: lane j holds float4 groups j, j + 32, ..):
 // FINAL = false: y = bf16(LN(x)) (a module's input);
 // FINAL = true:  x = LN(x) in place, and y = bf16(LN(x)) when y != nullptr.
-template <bool FINAL>
+template <bool FINAL, int kMaxQ>  // d <= 128 kMaxQ
 __global__ void __launch_bounds__(256) k_ln(float* x, uint16_t* y, int M, int d, const float* g, const float* b) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int r = blockIdx.x * 8 + warp;
   if (r >= M) return;
   float* xr = x + (size_t)r * d;
+  const int nq = d / 128;  // float4 groups per lane
+  float4 v[kMaxQ];
   float s = 0.f;
-  for (int c = lane * 4; c < d; c += 128) {
-    const float4 v = *reinterpret_cast<const float4*>(xr + c);
-    s += (v.x + v.y) + (v.z + v.w);
-  }
+#pragma unroll
+  for (int i = 0; i < kMaxQ; ++i)
+    if (i < nq) {
+      v[i] = *reinterpret_cast<const float4*>(xr + 128 * i + 4 * lane);
+      s += (v[i].x + v[i].y) + (v[i].z + v[i].w);
+    }
   const float mean = warp_sum(s) / (float)d;
   float q = 0.f;
-  for (int c = lane * 4; c < d; c += 128) {
-    const float4 v = *reinterpret_cast<const float4*>(xr + c);
-    const float a = v.x - mean, bb = v.y - mean, cc = v.z - mean, dd = v.w - mean;
-    q += (a * a + bb * bb) + (cc * cc + dd * dd);
-  }
-  const float rstd = 1.f / sqrtf(warp_sum(q) / (float)d + kLnEps);
-  for (int c = lane * 4; c < d; c += 128) {
-    const float4 v = *reinterpret_cast<const float4*>(xr + c);
-    const float4 gg = *reinterpret_cast<const float4*>(g + c);
-    const float4 be = *reinterpret_cast<const float4*>(b + c);
-    const float o0 = (v.x - mean) * rstd * gg.x + be.x, o1 = (v.y - mean) * rstd * gg.y + be.y;
-    const float o2 = (v.z - mean) * rstd * gg.z + be.z, o3 = (v.w - mean) * rstd * gg.w + be.w;
-    if (FINAL) *reinterpret_cast<float4*>(xr + c) = make_float4(o0, o1, o2, o3);
-    if (y) {
-      uint2 w;
-      w.x = (uint32_t)f2bf(o0) | ((uint32_t)f2bf(o1) << 16);
-      w.y = (uint32_t)f2bf(o2) | ((uint32_t)f2bf(o3) << 16);
-      *reinterpret_cast<uint2*>(y + (size_t)r * d + c) = w;
+#pragma unroll
+  for (int i = 0; i < kMaxQ; ++i)
+    if (i < nq) {
+      const float a0 = v[i].x - mean, a1 = v[i].y - mean, a2 = v[i].z - mean, a3 = v[i].w - mean;
+      q += (a0 * a0 + a1 * a1) + (a2 * a2 + a3 * a3);
     }
-  }
+  const float rstd = 1.f / sqrtf(warp_sum(q) / (float)d + kLnEps);
+#pragma unroll
+  for (int i = 0; i < kMaxQ; ++i)
+    if (i < nq) {
+      const int c = 128 * i + 4 * lane;
+      const float4 gg = *reinterpret_cast<const float4*>(g + c);
+      const float4 be = *reinterpret_cast<const float4*>(b + c);
+      const float o0 = (v[i].x - mean) * rstd * gg.x + be.x, o1 = (v[i].y - mean) * rstd * gg.y + be.y;
+      const float o2 = (v[i].z - mean) * rstd * gg.z + be.z, o3 = (v[i].w - mean) * rstd * gg.w + be.w;
+      if (FINAL) *reinterpret_cast<float4*>(xr + c) = make_float4(o0, o1, o2, o3);
+      if (y) {
+        uint2 w;
+        w.x = (uint32_t)f2bf(o0) | ((uint32_t)f2bf(o1) << 16);
+        w.y = (uint32_t)f2bf(o2) | ((uint32_t)f2bf(o3) << 16);
+        *reinterpret_cast<uint2*>(y + (size_t)r * d + c) = w;
+      }
+    }
 }
 
 struct AttnArgs {
@@ -327,22 +335,35 @@ struct ConvArgs {
 
 // Causal depthwise convolution over [cached K-1 frames, chunk frames], the
 // batch-norm affine map and Swish; thread = channel.  The last K-1 frames of
-// the window become the cache.
+// the window become the cache.  KT > 0: the kernel width as a constant, so
+// the taps stay in registers.
+template <int KT>
 __global__ void __launch_bounds__(128) k_dwconv(ConvArgs a) {
   extern __shared__ float seq[];  // [K-1+C][128]
   const int b = blockIdx.x, c = blockIdx.y * 128 + threadIdx.x, tid = threadIdx.x;
-  const int K1 = a.K - 1, C = a.C, d = a.d;
+  const int K = KT > 0 ? KT : a.K;
+  const int K1 = K - 1, C = a.C, d = a.d;
   const int slot = a.slots[b];
   uint16_t* cc = a.cache + ((size_t)slot * a.layers + a.layer) * (size_t)K1 * d;
   for (int t = 0; t < K1; ++t) seq[t * 128 + tid] = bf2f(cc[(size_t)t * d + c]);
   for (int t = 0; t < C; ++t) seq[(K1 + t) * 128 + tid] = bf2f(a.glu[(size_t)(b * C + t) * d + c]);
-  const float* w = a.w + (size_t)c * a.K;
+  const float* w = a.w + (size_t)c * K;
   const float bias = a.bias[c], sc = a.sc[c], sh = a.sh[c];
+  float wk[KT > 0 ? KT : 1];
+  if (KT > 0) {
+#pragma unroll
+    for (int k = 0; k < KT; ++k) wk[k] = w[k];
+  }
   for (int t = 0; t < C; ++t) {
     float acc = 0.f;
-    for (int k = 0; k < a.K; ++k) acc = fmaf(w[k], seq[(t + k) * 128 + tid], acc);
-    const float y = (acc + bias) * sc + sh;
-    a.z[(size_t)(b * C + t) * d + c] = f2bf(y / (1.f + expf(-y)));
+    if (KT > 0) {
+#pragma unroll
+      for (int k = 0; k < KT; ++k) acc = fmaf(wk[k], seq[(t + k) * 128 + tid], acc);
+    } else {
+      for (int k = 0; k < K; ++k) acc = fmaf(w[k], seq[(t + k) * 128 + tid], acc);
+    }
+    const float yv = (acc + bias) * sc + sh;
+    a.z[(size_t)(b * C + t) * d + c] = f2bf(yv / (1.f + expf(-yv)));
   }
   for (int t = 0; t < K1; ++t) cc[(size_t)t * d + c] = f2bf(seq[(C + t) * 128 + tid]);
 }
@@ -396,6 +417,13 @@ void launch_attn(const tsd_encoder* e, const AttnArgs& a, int n, cudaStream_t s)
   else k_attn<128><<<grid, 256, sm, s>>>(a);
 }
 
+template <bool FINAL>
+void ln_launch(dim3 grid, cudaStream_t s, float* x, uint16_t* y, int M, int d, const float* g, const float* b) {
+  if (d <= 512) k_ln<FINAL, 4><<<grid, 256, 0, s>>>(x, y, M, d, g, b);
+  else if (d <= 1024) k_ln<FINAL, 8><<<grid, 256, 0, s>>>(x, y, M, d, g, b);
+  else k_ln<FINAL, 16><<<grid, 256, 0, s>>>(x, y, M, d, g, b);
+}
+
 void enqueue(tsd_encoder* e, int n, int C, cudaStream_t s, const std::vector<cudaEvent_t>* ev,
              std::vector<int8_t>* cls) {
   const tsd_encoder_cfg& c = e->cfg;
@@ -418,11 +446,11 @@ void enqueue(tsd_encoder* e, int n, int C, cudaStream_t s, const std::vector<cud
   for (int l = 0; l < c.layers; ++l) {
     EncLayerDev& L = e->L[(size_t)l];
     mark(2);
-    k_ln<false><<<ln_grid, 256, 0, s>>>(e->x, e->nrm, M, d, L.ln_ff1_g, L.ln_ff1_b);
+    ln_launch<false>(ln_grid, s, e->x, e->nrm, M, d, L.ln_ff1_g, L.ln_ff1_b);
     gemm(kESwish, e->m_nrm, L.m_ff1_w1, c.ff, d, L.ff1_b1, e->hid, c.ff, 1.f);
     gemm(kEResid, e->m_hid, L.m_ff1_w2, d, c.ff, L.ff1_b2, e->x, d, 0.5f);
     mark(2);
-    k_ln<false><<<ln_grid, 256, 0, s>>>(e->x, e->nrm, M, d, L.ln_att_g, L.ln_att_b);
+    ln_launch<false>(ln_grid, s, e->x, e->nrm, M, d, L.ln_att_g, L.ln_att_b);
     gemm(kEPlain, e->m_nrm, L.m_qkv, 3 * d, d, L.qkv_b, e->qkv, 3 * d, 1.f);
     mark(1);
     AttnArgs aa{e->qkv, e->att, L.pos_tab, L.pos_u, L.pos_v, e->kc, e->vc, e->seen, e->slots_dev,
@@ -430,19 +458,21 @@ void enqueue(tsd_encoder* e, int n, int C, cudaStream_t s, const std::vector<cud
     launch_attn(e, aa, n, s);
     gemm(kEResid, e->m_att, L.m_out, d, d, L.out_b, e->x, d, 1.f);
     mark(2);
-    k_ln<false><<<ln_grid, 256, 0, s>>>(e->x, e->nrm, M, d, L.ln_conv_g, L.ln_conv_b);
+    ln_launch<false>(ln_grid, s, e->x, e->nrm, M, d, L.ln_conv_g, L.ln_conv_b);
     gemm(kEGlu, e->m_nrm, L.m_pw1, 2 * d, d, L.pw1_b, e->glu, d, 1.f);
     mark(2);
     ConvArgs ca{e->glu, e->convz, e->cc, L.dw_w, L.dw_b, L.bn_scale, L.bn_shift, e->slots_dev, d, c.kernel, C,
                 c.layers, l};
-    k_dwconv<<<dim3(n, d / 128), 128, (size_t)(c.kernel - 1 + C) * 128 * sizeof(float), s>>>(ca);
+    const size_t conv_smem = (size_t)(c.kernel - 1 + C) * 128 * sizeof(float);
+    if (c.kernel == 9) k_dwconv<9><<<dim3(n, d / 128), 128, conv_smem, s>>>(ca);
+    else k_dwconv<0><<<dim3(n, d / 128), 128, conv_smem, s>>>(ca);
     gemm(kEResid, e->m_convz, L.m_pw2, d, d, L.pw2_b, e->x, d, 1.f);
     mark(2);
-    k_ln<false><<<ln_grid, 256, 0, s>>>(e->x, e->nrm, M, d, L.ln_ff2_g, L.ln_ff2_b);
+    ln_launch<false>(ln_grid, s, e->x, e->nrm, M, d, L.ln_ff2_g, L.ln_ff2_b);
     gemm(kESwish, e->m_nrm, L.m_ff2_w1, c.ff, d, L.ff2_b1, e->hid, c.ff, 1.f);
     gemm(kEResid, e->m_hid, L.m_ff2_w2, d, c.ff, L.ff2_b2, e->x, d, 0.5f);
     mark(2);
-    k_ln<true><<<ln_grid, 256, 0, s>>>(e->x, l + 1 == c.layers ? e->outb : nullptr, M, d, L.ln_out_g, L.ln_out_b);
+    ln_launch<true>(ln_grid, s, e->x, l + 1 == c.layers ? e->outb : nullptr, M, d, L.ln_out_g, L.ln_out_b);
   }
   mark(2);
   k_advance<<<1, 256, 0, s>>>(e->seen, e->slots_dev, n, C);
