@@ -88,6 +88,33 @@ def test_ragged_chunks_and_zero_left_context():
             first += C
 
 
+def test_chunk_longer_than_the_left_context():
+    """C > left: only the chunk's last `left` frames go into the cache ring."""
+    cfg = synth.EncoderCfg("short-left", d=128, layers=2, heads=2, ff=256, kernel=4, left=3, chunk=5, feat=16,
+                           stack=4)
+    w = synth.encoder_weights(cfg)
+    enc = _gpu(w, max_streams=2)
+    slots = [enc.open() for _ in range(2)]
+    got = np.stack([enc.encode_chunk(slots, _feats(cfg, [4, 9], c * 5, 5)).cpu().numpy() for c in range(4)], axis=1)
+    for i, s in enumerate((4, 9)):
+        _close(got[i].view(np.uint16), _oracle_stream(w, s, 4, 5), 0.008, 0.032)
+
+
+def test_interface_limits():
+    """The largest left context (128 frames), chunks of 32 frames and 128-wide
+    heads: the attention window and its shared memory at their maximum."""
+    cfg = synth.EncoderCfg("limits", d=256, layers=1, heads=2, ff=256, kernel=32, left=128, chunk=32, feat=16,
+                           stack=4)
+    w = synth.encoder_weights(cfg)
+    enc = _gpu(w, max_streams=2)
+    slots = [enc.open() for _ in range(2)]
+    got = np.stack([enc.encode_chunk(slots, _feats(cfg, [1, 2], c * 32, 32)).cpu().numpy() for c in range(6)],
+                   axis=1)
+    enc.check()
+    for i, s in enumerate((1, 2)):
+        _close(got[i].view(np.uint16), _oracle_stream(w, s, 6, 32), 0.008, 0.032)
+
+
 def test_0p6b_shape_sampled_streams():
     """The 0.6B-shaped encoder (d 1024, 24 blocks, 8 heads, ff 4096, left 70,
     13-frame chunks) at the bench's launch configuration (256 streams per
