@@ -27,7 +27,8 @@ a final layer norm), with these readings:
 Rounding contract (the CUDA path computes in fp32 and rounds at the same
 points): the operands of every matrix product are bf16 (each module's
 layer-normed input, the feed-forward hidden layer after Swish, q/k/v and
-the cached k/v, the attention output, the GLU output and the cached GLU
+the cached k/v, q + u and q + v, the position rows p(delta), the softmax
+probabilities, the attention output, the GLU output and the cached GLU
 output, the convolution module's Swish output) and the chunk's output is
 bf16; everything else is float64 here.  With bf16_points=False nothing is
 rounded (used by the pins, which compare exact arithmetic).
@@ -135,17 +136,17 @@ def _attention(cfg, P, st, l, x, rnd):
     pos_q = st.seen + np.arange(C)
     pos_k = st.seen - nv + np.arange(nv + C)
     delta = pos_q[:, None] - pos_k[None, :]
-    p = sinusoid(delta.reshape(-1), d) @ P["pos_w"].T  # [C*(nv+C)][d]
+    p = rnd(sinusoid(delta.reshape(-1), d) @ P["pos_w"].T)  # [C*(nv+C)][d]
     p = p.reshape(C, nv + C, d)
     out = np.zeros((C, d))
     for h in range(H):
         c = slice(h * dh, (h + 1) * dh)
-        qu = q[:, c] + P["pos_u"][c]
-        qv = q[:, c] + P["pos_v"][c]
+        qu = rnd(q[:, c] + P["pos_u"][c])
+        qv = rnd(q[:, c] + P["pos_v"][c])
         s = (qu @ K[:, c].T + np.einsum("ie,ije->ij", qv, p[:, :, c])) / math.sqrt(dh)
         s = s - s.max(axis=1, keepdims=True)
         a = np.exp(s)
-        a = a / a.sum(axis=1, keepdims=True)
+        a = rnd(a / a.sum(axis=1, keepdims=True))
         out[:, c] = a @ V[:, c]
     o = rnd(out)
     st.k[l] = K[-cfg.left:] if cfg.left > 0 else K[:0]

@@ -39,12 +39,6 @@ __device__ __forceinline__ float warp_sum(float v) {
   return v;
 }
 
-__device__ __forceinline__ float warp_max(float v) {
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
-  return v;
-}
-
 // Layer norm of rows of the fp32 stream x [M][d] (one warp per row; the row
 // stays in registers: lane j holds float4 groups j, j + 32, ..):
 // FINAL = false: y = bf16(LN(x)) (a module's input);
@@ -92,94 +86,127 @@ __global__ void __launch_bounds__(256) k_ln(float* x, uint16_t* y, int M, int d,
 }
 
 struct AttnArgs {
-  const uint16_t* qkv;    // [M][3d] bf16: q, k, v of the chunk's frames
-  uint16_t* out;          // [M][d] bf16
-  const float* pos_tab;   // [n_off][d] this block's W_pos r(delta), row delta + cmax - 1
-  const float* pu;        // [d] content bias u
-  const float* pv;        // [d] position bias v
-  uint16_t* kc;           // k cache: [slot][layer][head][left][dh]
+  const uint16_t* qkv;      // [M][3d] bf16: q, k, v of the chunk's frames
+  uint16_t* out;            // [M][d] bf16
+  const uint16_t* pos_tab;  // [n_off][d] bf16: this block's W_pos r(delta), row delta + cmax - 1
+  const float* pu;          // [d] content bias u
+  const float* pv;          // [d] position bias v
+  uint16_t* kc;             // k cache: [slot][layer][head][left][dh]
   uint16_t* vc;
-  const int32_t* seen;    // frames seen per slot (before this chunk)
-  const int32_t* slots;   // [n]
+  const int32_t* seen;      // frames seen per slot (before this chunk)
+  const int32_t* slots;     // [n]
   int d, heads, left, layers, layer, C, cmax;
-  float scale;            // 1 / sqrt(dh)
+  float scale;              // 1 / sqrt(dh)
 };
 
-// Shared memory of k_attn for a chunk of C frames (worst case nv = left).
+__host__ __device__ constexpr int round16(int x) { return (x + 15) / 16 * 16; }
+
+// Shared memory of k_attn for a chunk of C frames (worst case nv = left):
+// q + u and q + v, k, v and the table rows as bf16 rows padded by 8 elements
+// (16-byte aligned, conflict-free ldmatrix), then one 16-row block's scores,
+// position scores (fp32) and probabilities (bf16).
 __host__ __device__ constexpr size_t attn_smem(int dh, int left, int C) {
-  return (size_t)(left + C) * (dh + 8) * 2 /*K*/ + (size_t)(left + C) * dh * 2 /*V*/ +
-         (size_t)2 * ((C + 15) / 16 * 16) * dh * 4 /*Qu, Qv*/ + (size_t)2 * (left + 2 * C - 1) * 16 * 4 /*SpT*/ +
-         (size_t)2 * (left + C) * 16 * 4 /*ST*/ + (size_t)2 * 16 * dh * 4 /*O partials*/;
+  return (size_t)2 * round16(C) * (dh + 8) * 2 + (size_t)2 * round16(left + C) * (dh + 8) * 2 +
+         (size_t)round16(left + 2 * C - 1) * (dh + 8) * 2 + (size_t)16 * (round16(left + C) + 4) * 4 +
+         (size_t)16 * (round16(left + 2 * C - 1) + 4) * 4 + (size_t)16 * (round16(left + C) + 8) * 2;
 }
 
-__device__ __forceinline__ void bf16x8(const uint4 w, float* f) {
-  f[0] = __uint_as_float(w.x << 16), f[1] = __uint_as_float(w.x & 0xffff0000u);
-  f[2] = __uint_as_float(w.y << 16), f[3] = __uint_as_float(w.y & 0xffff0000u);
-  f[4] = __uint_as_float(w.z << 16), f[5] = __uint_as_float(w.z & 0xffff0000u);
-  f[6] = __uint_as_float(w.w << 16), f[7] = __uint_as_float(w.w & 0xffff0000u);
+__device__ __forceinline__ void ldsm_x4(const void* p, uint32_t* r) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+               : "r"((uint32_t)__cvta_generic_to_shared(p)));
+}
+__device__ __forceinline__ void ldsm_x2(const void* p, uint32_t* r) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x2.shared.b16 {%0, %1}, [%2];"
+               : "=r"(r[0]), "=r"(r[1])
+               : "r"((uint32_t)__cvta_generic_to_shared(p)));
+}
+__device__ __forceinline__ void ldsm_x2_trans(const void* p, uint32_t* r) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x2.trans.shared.b16 {%0, %1}, [%2];"
+               : "=r"(r[0]), "=r"(r[1])
+               : "r"((uint32_t)__cvta_generic_to_shared(p)));
+}
+// D (16x8 fp32) += A (16x16 bf16, row-major) . B (16x8 bf16, column-major)
+__device__ __forceinline__ void mma16816(float* c, const uint32_t* a, const uint32_t* b) {
+  asm volatile("mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
+               "{%0, %1, %2, %3};"
+               : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+               : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b[0]), "r"(b[1]));
 }
 
-// One (stream, head) per CTA: chunked, limited-context attention with the
-// relative-position term over the window [cached frames, chunk frames], then
-// the chunk's k and v go into the ring cache.  The three products (query
-// rows against the position table, against the keys, and probabilities
-// against the values) run as register tiles: a thread keeps 16 query rows'
-// sums for one key (or table row, or 4 x 4 outputs) and reads its operands
-// as 16-byte vectors from padded, bank-conflict-free shared rows; the inner
-// dimension is split over two threads whose halves are added afterwards.
+// One (stream, head) per CTA, 4 warps: chunked, limited-context attention
+// with the relative-position term over the window [cached frames, chunk
+// frames].  The three products -- (q + u) against the keys, (q + v)
+// against the position-table rows, the probabilities against the values --
+// run on the tensor cores as 16 x 8 x 16 bf16 MMAs with fp32 accumulation
+// (a chunk has 13 query rows: one 16-row tile).  Then the chunk's k and v go
+// into the ring cache.
 template <int DH>
-__global__ void __launch_bounds__(256) k_attn(AttnArgs a) {
+__global__ void __launch_bounds__(128) k_attn(AttnArgs a) {
   extern __shared__ __align__(16) unsigned char sm[];
-  constexpr int KS = DH + 8;  // padded k row (bf16): 16-byte aligned, conflict-free 16-byte reads
-  constexpr int HALF = DH / 2;
-  constexpr int NQ = DH / 4;  // column quads
-  const int b = blockIdx.x, h = blockIdx.y, tid = threadIdx.x;
+  constexpr int RS = DH + 8;  // bf16 row stride
+  constexpr int E8 = DH / 8;  // 16-byte groups per row
+  const int b = blockIdx.x, h = blockIdx.y, tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int C = a.C, d = a.d;
   const int slot = a.slots[b];
   const int sn = a.seen[slot];
   const int nv = min(sn, a.left);
   const int W = nv + C;
   const int nrel = nv + 2 * C - 1;  // offsets -(C-1) .. nv+C-1
-  const int Wm = a.left + C, nrm = a.left + 2 * C - 1, CR = (C + 15) / 16 * 16;
-  uint16_t* Kb = reinterpret_cast<uint16_t*>(sm);
-  uint16_t* Vb = Kb + (size_t)Wm * KS;
-  float* Qu = reinterpret_cast<float*>(Vb + (size_t)Wm * DH);
-  float* Qv = Qu + CR * DH;
-  float* SpT = Qv + CR * DH;       // [2][nrm][16]: halves of (q + v) . p(t), transposed
-  float* ST = SpT + 2 * nrm * 16;  // [2][Wm][16]: halves of (q + u) . k, transposed; [0] then holds the scores
-  float* Op = ST + 2 * Wm * 16;    // [2][16][DH]: output halves
+  const int CR = round16(C), Wp = round16(a.left + C), Np = round16(a.left + 2 * C - 1);
+  const int Wa = round16(W), Na = round16(nrel);  // this stream's padded extents
+  const int SS = Wp + 4, SPS = Np + 4, PRS = Wp + 8;
+  uint16_t* Qu = reinterpret_cast<uint16_t*>(sm);
+  uint16_t* Qv = Qu + CR * RS;
+  uint16_t* Kb = Qv + CR * RS;
+  uint16_t* Vb = Kb + Wp * RS;
+  uint16_t* Pb = Vb + Wp * RS;
+  float* S = reinterpret_cast<float*>(Pb + Np * RS);  // [16][SS]
+  float* Sp = S + 16 * SS;                             // [16][SPS]
+  uint16_t* Pr = reinterpret_cast<uint16_t*>(Sp + 16 * SPS);  // [16][PRS]
 
   const size_t cb = (((size_t)slot * a.layers + a.layer) * a.heads + h) * (size_t)a.left * DH;
-  constexpr int E8 = DH / 8;  // 16-byte groups per row
-  for (int idx = tid; idx < nv * E8; idx += blockDim.x) {
+  const uint4 zero = make_uint4(0u, 0u, 0u, 0u);
+  for (int idx = tid; idx < Wa * E8; idx += blockDim.x) {
     const int jj = idx / E8, e8 = idx - jj * E8;
-    const int ring = (sn - nv + jj) % a.left;
-    *reinterpret_cast<uint4*>(Kb + (size_t)jj * KS + 8 * e8) =
-        reinterpret_cast<const uint4*>(a.kc + cb + (size_t)ring * DH)[e8];
-    *reinterpret_cast<uint4*>(Vb + (size_t)jj * DH + 8 * e8) =
-        reinterpret_cast<const uint4*>(a.vc + cb + (size_t)ring * DH)[e8];
+    uint4 kw = zero, vw = zero;
+    if (jj < nv) {
+      const int ring = (sn - nv + jj) % a.left;
+      kw = reinterpret_cast<const uint4*>(a.kc + cb + (size_t)ring * DH)[e8];
+      vw = reinterpret_cast<const uint4*>(a.vc + cb + (size_t)ring * DH)[e8];
+    } else if (jj < W) {
+      const uint16_t* row = a.qkv + (size_t)(b * C + jj - nv) * 3 * d + h * DH;
+      kw = reinterpret_cast<const uint4*>(row + d)[e8];
+      vw = reinterpret_cast<const uint4*>(row + 2 * d)[e8];
+    }
+    *reinterpret_cast<uint4*>(Kb + jj * RS + 8 * e8) = kw;
+    *reinterpret_cast<uint4*>(Vb + jj * RS + 8 * e8) = vw;
   }
   for (int idx = tid; idx < CR * E8; idx += blockDim.x) {
     const int i = idx / E8, e8 = idx - i * E8;
-    float q[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-    float* qu = Qu + i * DH + 8 * e8;
-    float* qv = Qv + i * DH + 8 * e8;
+    uint4 qu = zero, qv = zero;
     if (i < C) {
-      const uint16_t* row = a.qkv + (size_t)(b * C + i) * 3 * d + h * DH;
-      *reinterpret_cast<uint4*>(Kb + (size_t)(nv + i) * KS + 8 * e8) = reinterpret_cast<const uint4*>(row + d)[e8];
-      *reinterpret_cast<uint4*>(Vb + (size_t)(nv + i) * DH + 8 * e8) = reinterpret_cast<const uint4*>(row + 2 * d)[e8];
-      bf16x8(reinterpret_cast<const uint4*>(row)[e8], q);
+      const uint4 qw = reinterpret_cast<const uint4*>(a.qkv + (size_t)(b * C + i) * 3 * d + h * DH)[e8];
+      const uint32_t* qp = reinterpret_cast<const uint32_t*>(&qw);
       const float* u = a.pu + h * DH + 8 * e8;
       const float* v = a.pv + h * DH + 8 * e8;
+      uint32_t* up = reinterpret_cast<uint32_t*>(&qu);
+      uint32_t* vp = reinterpret_cast<uint32_t*>(&qv);
 #pragma unroll
-      for (int k = 0; k < 8; ++k) {
-        qu[k] = q[k] + u[k];
-        qv[k] = q[k] + v[k];
+      for (int k = 0; k < 4; ++k) {
+        const float q0 = __uint_as_float(qp[k] << 16), q1 = __uint_as_float(qp[k] & 0xffff0000u);
+        up[k] = (uint32_t)f2bf(q0 + u[2 * k]) | ((uint32_t)f2bf(q1 + u[2 * k + 1]) << 16);
+        vp[k] = (uint32_t)f2bf(q0 + v[2 * k]) | ((uint32_t)f2bf(q1 + v[2 * k + 1]) << 16);
       }
-    } else {
-#pragma unroll
-      for (int k = 0; k < 8; ++k) qu[k] = qv[k] = 0.f;  // padding rows
     }
+    *reinterpret_cast<uint4*>(Qu + i * RS + 8 * e8) = qu;
+    *reinterpret_cast<uint4*>(Qv + i * RS + 8 * e8) = qv;
+  }
+  for (int idx = tid; idx < Na * E8; idx += blockDim.x) {
+    const int t = idx / E8, e8 = idx - t * E8;
+    const uint4 pw = t < nrel ? reinterpret_cast<const uint4*>(a.pos_tab + (size_t)(t + a.cmax - C) * d + h * DH)[e8]
+                              : zero;
+    *reinterpret_cast<uint4*>(Pb + t * RS + 8 * e8) = pw;
   }
   __syncthreads();
   // the cache was read above: the chunk's k and v replace the oldest frames
@@ -193,132 +220,71 @@ __global__ void __launch_bounds__(256) k_attn(AttnArgs a) {
       reinterpret_cast<uint4*>(a.vc + cb + (size_t)ring * DH)[e8] = reinterpret_cast<const uint4*>(row + 2 * d)[e8];
     }
   }
+  const int fr = lane >> 2, fc = (lane & 3) * 2;  // this lane's place in a 16 x 8 result
   for (int rb = 0; rb < CR; rb += 16) {
-    // position term SpT[s][t][r] = sum over half s of (q + v)[rb + r] . p(t - (C-1)),
-    // and content term ST[s][jj][r] = sum over half s of (q + u)[rb + r] . k_jj,
-    // as one list of items
-    for (int item = tid; item < 2 * nrel + 2 * W; item += blockDim.x) {
-      float acc[16];
+    // content scores S = (q + u) k^T and position scores Sp = (q + v) p^T,
+    // one 16 x 8 tile per warp at a time
+    const int nts = Wa / 8, ntp = Na / 8;
+    for (int nt = warp; nt < nts + ntp; nt += 4) {
+      const bool pos = nt >= nts;
+      const int n0 = (pos ? nt - nts : nt) * 8;
+      const uint16_t* A = (pos ? Qv : Qu) + (rb + (lane & 15)) * RS + (lane >> 4) * 8;
+      const uint16_t* B = (pos ? Pb : Kb) + (n0 + (lane & 7)) * RS + ((lane >> 3) & 1) * 8;
+      float c[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-      for (int r = 0; r < 16; ++r) acc[r] = 0.f;
-      float* dst;
-      if (item < 2 * nrel) {
-        const int s = item / nrel, t = item - s * nrel;
-        const float4* p = reinterpret_cast<const float4*>(a.pos_tab + (size_t)(t + a.cmax - C) * d + h * DH + s * HALF);
-        const float* q = Qv + rb * DH + s * HALF;
-#pragma unroll 2
-        for (int q4 = 0; q4 < HALF / 4; ++q4) {
-          const float4 pv = p[q4];
-#pragma unroll
-          for (int r = 0; r < 16; ++r) {
-            const float4 qq = *reinterpret_cast<const float4*>(q + r * DH + 4 * q4);
-            acc[r] = fmaf(qq.x, pv.x, fmaf(qq.y, pv.y, fmaf(qq.z, pv.z, fmaf(qq.w, pv.w, acc[r]))));
-          }
-        }
-        dst = SpT + ((size_t)s * nrm + t) * 16;
-      } else {
-        const int i2 = item - 2 * nrel;
-        const int s = i2 / W, jj = i2 - s * W;
-        const uint16_t* kr = Kb + (size_t)jj * KS + s * HALF;
-        const float* q = Qu + rb * DH + s * HALF;
-#pragma unroll 1
-        for (int o8 = 0; o8 < HALF / 8; ++o8) {
-          float kf[8];
-          bf16x8(*reinterpret_cast<const uint4*>(kr + 8 * o8), kf);
-#pragma unroll
-          for (int r = 0; r < 16; ++r) {
-            const float4 q0 = *reinterpret_cast<const float4*>(q + r * DH + 8 * o8);
-            const float4 q1 = *reinterpret_cast<const float4*>(q + r * DH + 8 * o8 + 4);
-            acc[r] = fmaf(q0.x, kf[0], fmaf(q0.y, kf[1], fmaf(q0.z, kf[2], fmaf(q0.w, kf[3], acc[r]))));
-            acc[r] = fmaf(q1.x, kf[4], fmaf(q1.y, kf[5], fmaf(q1.z, kf[6], fmaf(q1.w, kf[7], acc[r]))));
-          }
-        }
-        dst = ST + ((size_t)s * Wm + jj) * 16;
+      for (int kk = 0; kk < DH / 16; ++kk) {
+        uint32_t af[4], bf[2];
+        ldsm_x4(A + kk * 16, af);
+        ldsm_x2(B + kk * 16, bf);
+        mma16816(c, af, bf);
       }
-      float4* o = reinterpret_cast<float4*>(dst);
-#pragma unroll
-      for (int r = 0; r < 16; r += 4) o[r / 4] = make_float4(acc[r], acc[r + 1], acc[r + 2], acc[r + 3]);
-    }
-    __syncthreads();
-    // scores of rows rb..rb+15 into ST[0]
-    for (int item = tid; item < W * 16; item += blockDim.x) {
-      const int jj = item >> 4, r = item & 15, i = rb + r;
-      float v = 0.f;
-      if (i < C) {
-        const int t = i - jj + nv + C - 1;
-        v = (ST[jj * 16 + r] + ST[(Wm + jj) * 16 + r] + SpT[t * 16 + r] + SpT[(nrm + t) * 16 + r]) * a.scale;
-      }
-      ST[jj * 16 + r] = v;
+      float* o = pos ? Sp : S;
+      const int os = pos ? SPS : SS;
+      *reinterpret_cast<float2*>(o + fr * os + n0 + fc) = make_float2(c[0], c[1]);
+      *reinterpret_cast<float2*>(o + (fr + 8) * os + n0 + fc) = make_float2(c[2], c[3]);
     }
     __syncthreads();
     {
-      // softmax over the keys of each row: thread (row r = tid mod 16, j0 =
-      // tid / 16) takes keys j0, j0 + 16, ..; the 16 partial maxima and sums
-      // of a row meet in shared memory (the output buffer, free until below)
-      const int r = tid & 15, j0 = tid >> 4;
-      float* red = Op;  // [16][16] maxima, then [16][16] sums
+      // scores, softmax and bf16 probabilities: 8 threads per query row
+      const int r = tid >> 3, l8 = tid & 7, i = rb + r;
       float m = -INFINITY;
-      for (int jj = j0; jj < W; jj += 16) m = fmaxf(m, ST[jj * 16 + r]);
-      red[j0 * 16 + r] = m;
-      __syncthreads();
-      float mm = -INFINITY;
-#pragma unroll
-      for (int k = 0; k < 16; ++k) mm = fmaxf(mm, red[k * 16 + r]);
-      float z = 0.f;
-      for (int jj = j0; jj < W; jj += 16) {
-        const float e = expf(ST[jj * 16 + r] - mm);
-        ST[jj * 16 + r] = e;
-        z += e;
-      }
-      red[256 + j0 * 16 + r] = z;
-      __syncthreads();
-      float zz = 0.f;
-#pragma unroll
-      for (int k = 0; k < 16; ++k) zz += red[256 + k * 16 + r];
-      const float inv = 1.f / zz;
-      for (int jj = j0; jj < W; jj += 16) ST[jj * 16 + r] *= inv;
-    }
-    __syncthreads();
-    // output halves: Op[s][4g + r][4q + c] over the keys of half s
-    {
-      const int s = tid >> 7, rem = tid & 127, g = rem / NQ, q = rem - g * NQ;
-      if (g < 4) {
-        const int j0 = s == 0 ? 0 : W / 2, j1 = s == 0 ? W / 2 : W;
-        float acc[4][4];
-#pragma unroll
-        for (int r = 0; r < 4; ++r)
-#pragma unroll
-          for (int c = 0; c < 4; ++c) acc[r][c] = 0.f;
-        for (int jj = j0; jj < j1; ++jj) {
-          const uint2 vw = *reinterpret_cast<const uint2*>(Vb + (size_t)jj * DH + 4 * q);
-          const float v0 = __uint_as_float(vw.x << 16), v1 = __uint_as_float(vw.x & 0xffff0000u);
-          const float v2 = __uint_as_float(vw.y << 16), v3 = __uint_as_float(vw.y & 0xffff0000u);
-          const float4 p = *reinterpret_cast<const float4*>(ST + jj * 16 + 4 * g);
-          const float pr[4] = {p.x, p.y, p.z, p.w};
-#pragma unroll
-          for (int r = 0; r < 4; ++r) {
-            acc[r][0] = fmaf(pr[r], v0, acc[r][0]);
-            acc[r][1] = fmaf(pr[r], v1, acc[r][1]);
-            acc[r][2] = fmaf(pr[r], v2, acc[r][2]);
-            acc[r][3] = fmaf(pr[r], v3, acc[r][3]);
-          }
+      if (i < C)
+        for (int jj = l8; jj < W; jj += 8) {
+          const float v = (S[r * SS + jj] + Sp[r * SPS + (i - jj + nv + C - 1)]) * a.scale;
+          S[r * SS + jj] = v;
+          m = fmaxf(m, v);
         }
 #pragma unroll
-        for (int r = 0; r < 4; ++r)
-          *reinterpret_cast<float4*>(Op + ((size_t)s * 16 + 4 * g + r) * DH + 4 * q) =
-              make_float4(acc[r][0], acc[r][1], acc[r][2], acc[r][3]);
-      }
+      for (int o = 4; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
+      float z = 0.f;
+      if (i < C)
+        for (int jj = l8; jj < W; jj += 8) {
+          const float e = expf(S[r * SS + jj] - m);
+          S[r * SS + jj] = e;
+          z += e;
+        }
+#pragma unroll
+      for (int o = 4; o > 0; o >>= 1) z += __shfl_xor_sync(0xffffffffu, z, o);
+      const float inv = i < C ? 1.f / z : 0.f;
+      for (int jj = l8; jj < Wa; jj += 8) Pr[r * PRS + jj] = (i < C && jj < W) ? f2bf(S[r * SS + jj] * inv) : 0;
     }
     __syncthreads();
-    for (int item = tid; item < 16 * NQ; item += blockDim.x) {
-      const int r = item / NQ, q = item - r * NQ, i = rb + r;
-      if (i >= C) continue;
-      const float4 x = *reinterpret_cast<const float4*>(Op + (size_t)r * DH + 4 * q);
-      const float4 y = *reinterpret_cast<const float4*>(Op + (size_t)(16 + r) * DH + 4 * q);
-      uint2 w;
-      w.x = (uint32_t)f2bf(x.x + y.x) | ((uint32_t)f2bf(x.y + y.y) << 16);
-      w.y = (uint32_t)f2bf(x.z + y.z) | ((uint32_t)f2bf(x.w + y.w) << 16);
-      *reinterpret_cast<uint2*>(a.out + (size_t)(b * C + i) * d + h * DH + 4 * q) = w;
+    // out = probabilities . v, one 16 x 8 tile of head columns per warp at a time
+    for (int nt = warp; nt < DH / 8; nt += 4) {
+      float c[4] = {0.f, 0.f, 0.f, 0.f};
+      for (int kk = 0; kk < Wa / 16; ++kk) {
+        uint32_t af[4], bf[2];
+        ldsm_x4(Pr + (lane & 15) * PRS + kk * 16 + (lane >> 4) * 8, af);
+        ldsm_x2_trans(Vb + (kk * 16 + (lane & 15)) * RS + nt * 8, bf);
+        mma16816(c, af, bf);
+      }
+      const int i0 = rb + fr, i1 = rb + fr + 8, col = h * DH + nt * 8 + fc;
+      if (i0 < C)
+        *reinterpret_cast<uint32_t*>(a.out + (size_t)(b * C + i0) * d + col) =
+            (uint32_t)f2bf(c[0]) | ((uint32_t)f2bf(c[1]) << 16);
+      if (i1 < C)
+        *reinterpret_cast<uint32_t*>(a.out + (size_t)(b * C + i1) * d + col) =
+            (uint32_t)f2bf(c[2]) | ((uint32_t)f2bf(c[3]) << 16);
     }
     __syncthreads();
   }
@@ -368,10 +334,11 @@ __global__ void __launch_bounds__(128) k_dwconv(ConvArgs a) {
   for (int t = 0; t < K1; ++t) cc[(size_t)t * d + c] = f2bf(seq[(C + t) * 128 + tid]);
 }
 
-// P[row][c] = sum_k W_pos[c][k] r_k(delta), delta = row - (cmax - 1), r the
-// sinusoidal code (sin at 2j, cos at 2j+1 of delta / 10000^(2j/d)); computed
-// in double once at create.
-__global__ void k_pos_table(const uint16_t* pos_w, float* tab, int d, int cmax) {
+// P[row][c] = bf16(sum_k W_pos[c][k] r_k(delta)), delta = row - (cmax - 1), r
+// the sinusoidal code (sin at 2j, cos at 2j+1 of delta / 10000^(2j/d));
+// computed in double once at create and rounded once to bf16 (it is an MMA
+// operand).
+__global__ void k_pos_table(const uint16_t* pos_w, uint16_t* tab, int d, int cmax) {
   extern __shared__ double r[];
   const double delta = (double)((int)blockIdx.x - (cmax - 1));
   for (int k = threadIdx.x; k < d; k += blockDim.x) {
@@ -383,7 +350,8 @@ __global__ void k_pos_table(const uint16_t* pos_w, float* tab, int d, int cmax) 
     const uint16_t* wr = pos_w + (size_t)c * d;
     double acc = 0.0;
     for (int k = 0; k < d; ++k) acc += (double)bf2f(wr[k]) * r[k];
-    tab[(size_t)blockIdx.x * d + c] = (float)acc;
+    const __nv_bfloat16 v = __double2bfloat16(acc);
+    tab[(size_t)blockIdx.x * d + c] = *reinterpret_cast<const uint16_t*>(&v);
   }
 }
 
@@ -413,8 +381,8 @@ int n_marks(const tsd_encoder* e) { return 1 + 15 * e->cfg.layers + 1 + 1; }
 void launch_attn(const tsd_encoder* e, const AttnArgs& a, int n, cudaStream_t s) {
   const size_t sm = attn_smem(e->cfg.d / e->cfg.heads, e->cfg.left, a.C);
   dim3 grid(n, e->cfg.heads);
-  if (e->cfg.d / e->cfg.heads == 64) k_attn<64><<<grid, 256, sm, s>>>(a);
-  else k_attn<128><<<grid, 256, sm, s>>>(a);
+  if (e->cfg.d / e->cfg.heads == 64) k_attn<64><<<grid, 128, sm, s>>>(a);
+  else k_attn<128><<<grid, 128, sm, s>>>(a);
 }
 
 template <bool FINAL>

@@ -45,7 +45,7 @@ struct EncLayerDev {
   uint16_t *ff1_w1, *ff1_w2, *qkv_w, *pos_w, *out_w, *pw1_w /*GLU-interleaved*/, *pw2_w, *ff2_w1, *ff2_w2;
   float *ff1_b1, *ff1_b2, *qkv_b, *pos_u, *pos_v, *out_b, *pw1_b /*interleaved*/, *dw_w, *dw_b, *bn_scale,
       *bn_shift, *pw2_b, *ff2_b1, *ff2_b2;
-  float* pos_tab;  // [n_off][d]: W_pos r(delta) for delta = -(max_chunk-1) .. left+max_chunk-1
+  uint16_t* pos_tab;  // [n_off][d] bf16: W_pos r(delta) for delta = -(max_chunk-1) .. left+max_chunk-1
   CUtensorMap m_ff1_w1, m_ff1_w2, m_qkv, m_out, m_pw1, m_pw2, m_ff2_w1, m_ff2_w2;
 };
 

@@ -4,9 +4,9 @@ Tolerance.  Both sides round to bf16 at the same points but reach them
 through different sums (tensor-core fp32 vs float64), so a rounding point can
 land on either side of a bf16 boundary, and the flip travels on.  Measured
 on the oracle itself: perturbing its weights by 3e-7 (relative, the size of
-fp32 rounding) moves the bf16 outputs of a 2-block encoder by 0.002 on
+fp32 rounding) moves the bf16 outputs of a 2-block encoder by 0.0024 on
 average and at most one output ulp (0.016), and of the 24-block 0.6B-shaped
-encoder by 0.005 on average and at most 0.031.  The GPU is held to four times
+encoder by 0.0054 on average and at most 0.033.  The GPU is held to four times
 the average and twice the maximum; outputs have unit scale.  Where results
 must be exact, they are: a stream's output does not depend on the other
 streams of the call or on its slot."""
@@ -67,7 +67,7 @@ def test_small_encoder_matches_oracle(dh):
     enc.check()
     got = np.stack(got, axis=1)  # [stream][chunk][C][d]
     for i, s in enumerate(streams):
-        _close(got[i].view(np.uint16), _oracle_stream(w, s, 7, cfg.chunk), 0.008, 0.032)
+        _close(got[i].view(np.uint16), _oracle_stream(w, s, 7, cfg.chunk), 0.0095, 0.032)
 
 
 def test_ragged_chunks_and_zero_left_context():
@@ -84,7 +84,7 @@ def test_ragged_chunks_and_zero_left_context():
         for C in (4, 1, 6, 3, 6, 2):
             g = enc.encode_chunk([slot], _feats(cfg, [5], first, C)).cpu().numpy()[0]
             want = oe.bits_to_f64(oe.encode_chunk(E, st, synth.features(cfg, [5], first, C)[0]))
-            _close(g.view(np.uint16), want, 0.008, 0.032)
+            _close(g.view(np.uint16), want, 0.0095, 0.032)
             first += C
 
 
@@ -97,7 +97,7 @@ def test_chunk_longer_than_the_left_context():
     slots = [enc.open() for _ in range(2)]
     got = np.stack([enc.encode_chunk(slots, _feats(cfg, [4, 9], c * 5, 5)).cpu().numpy() for c in range(4)], axis=1)
     for i, s in enumerate((4, 9)):
-        _close(got[i].view(np.uint16), _oracle_stream(w, s, 4, 5), 0.008, 0.032)
+        _close(got[i].view(np.uint16), _oracle_stream(w, s, 4, 5), 0.0095, 0.032)
 
 
 def test_interface_limits():
@@ -112,7 +112,7 @@ def test_interface_limits():
                    axis=1)
     enc.check()
     for i, s in enumerate((1, 2)):
-        _close(got[i].view(np.uint16), _oracle_stream(w, s, 6, 32), 0.008, 0.032)
+        _close(got[i].view(np.uint16), _oracle_stream(w, s, 6, 32), 0.0095, 0.032)
 
 
 def test_0p6b_shape_sampled_streams():
@@ -130,7 +130,7 @@ def test_0p6b_shape_sampled_streams():
     enc.check()
     got = np.stack(got, axis=1)
     for s in (0, 131, 255):
-        _close(got[s].view(np.uint16), _oracle_stream(w, s, 2, cfg.chunk), 0.02, 0.0625)
+        _close(got[s].view(np.uint16), _oracle_stream(w, s, 2, cfg.chunk), 0.022, 0.07)
 
 
 def test_streams_do_not_interact():

@@ -75,7 +75,7 @@ def test_pins_catch_planted_mistake(name, tmp_path):
 
 # Planted mistakes in copies of the encoder oracle (oracle/encoder.py).
 ENCODER_MUTATIONS = {
-    "content bias u dropped": ('qu = q[:, c] + P["pos_u"][c]', 'qu = q[:, c]'),
+    "content bias u dropped": ('qu = rnd(q[:, c] + P["pos_u"][c])', 'qu = rnd(q[:, c])'),
     "relative offset sign flipped": ("delta = pos_q[:, None] - pos_k[None, :]",
                                      "delta = pos_k[None, :] - pos_q[:, None]"),
     "sin and cos swapped in the position code": ("r[:, 0::2] = np.sin(ang)\n    r[:, 1::2] = np.cos(ang)",
@@ -89,8 +89,8 @@ ENCODER_MUTATIONS = {
     "GLU halves swapped": ("glu = rnd(y[:, :d] * sigmoid(y[:, d:]))", "glu = rnd(y[:, d:] * sigmoid(y[:, :d]))"),
     "feed-forward half step dropped": ("x = x + 0.5 * _feed_forward(x, *P[\"ln_ff1\"]",
                                        "x = x + 1.0 * _feed_forward(x, *P[\"ln_ff1\"]"),
-    "softmax over the head dimension": ("a = a / a.sum(axis=1, keepdims=True)",
-                                        "a = a / a.sum(axis=0, keepdims=True)"),
+    "softmax over the head dimension": ("a = rnd(a / a.sum(axis=1, keepdims=True))",
+                                        "a = rnd(a / a.sum(axis=0, keepdims=True))"),
     "batch norm shift dropped": ('z = rnd(swish(dw * P["bn_scale"] + P["bn_shift"]))',
                                  'z = rnd(swish(dw * P["bn_scale"]))'),
     "rounding to nearest truncates": ("return np.ldexp(np.rint(np.ldexp(m, 8)), e - 8)",
