@@ -134,15 +134,17 @@ __device__ __forceinline__ void mma16816(float* c, const uint32_t* a, const uint
                : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b[0]), "r"(b[1]));
 }
 
-// One (stream, head) per CTA, 4 warps: chunked, limited-context attention
+// One (stream, head) per CTA, 8 warps: chunked, limited-context attention
 // with the relative-position term over the window [cached frames, chunk
 // frames].  The three products -- (q + u) against the keys, (q + v)
 // against the position-table rows, the probabilities against the values --
 // run on the tensor cores as 16 x 8 x 16 bf16 MMAs with fp32 accumulation
 // (a chunk has 13 query rows: one 16-row tile).  Then the chunk's k and v go
 // into the ring cache.
+constexpr int kAttnThreads = 256;
+
 template <int DH>
-__global__ void __launch_bounds__(128) k_attn(AttnArgs a) {
+__global__ void __launch_bounds__(kAttnThreads) k_attn(AttnArgs a) {
   extern __shared__ __align__(16) unsigned char sm[];
   constexpr int RS = DH + 8;  // bf16 row stride
   constexpr int E8 = DH / 8;  // 16-byte groups per row
@@ -225,7 +227,7 @@ __global__ void __launch_bounds__(128) k_attn(AttnArgs a) {
     // content scores S = (q + u) k^T and position scores Sp = (q + v) p^T,
     // one 16 x 8 tile per warp at a time
     const int nts = Wa / 8, ntp = Na / 8;
-    for (int nt = warp; nt < nts + ntp; nt += 4) {
+    for (int nt = warp; nt < nts + ntp; nt += kAttnThreads / 32) {
       const bool pos = nt >= nts;
       const int n0 = (pos ? nt - nts : nt) * 8;
       const uint16_t* A = (pos ? Qv : Qu) + (rb + (lane & 15)) * RS + (lane >> 4) * 8;
@@ -245,32 +247,33 @@ __global__ void __launch_bounds__(128) k_attn(AttnArgs a) {
     }
     __syncthreads();
     {
-      // scores, softmax and bf16 probabilities: 8 threads per query row
-      const int r = tid >> 3, l8 = tid & 7, i = rb + r;
+      // scores, softmax and bf16 probabilities: 16 threads per query row
+      constexpr int G = kAttnThreads / 16;
+      const int r = tid / G, l8 = tid % G, i = rb + r;
       float m = -INFINITY;
       if (i < C)
-        for (int jj = l8; jj < W; jj += 8) {
+        for (int jj = l8; jj < W; jj += G) {
           const float v = (S[r * SS + jj] + Sp[r * SPS + (i - jj + nv + C - 1)]) * a.scale;
           S[r * SS + jj] = v;
           m = fmaxf(m, v);
         }
 #pragma unroll
-      for (int o = 4; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
+      for (int o = G / 2; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
       float z = 0.f;
       if (i < C)
-        for (int jj = l8; jj < W; jj += 8) {
+        for (int jj = l8; jj < W; jj += G) {
           const float e = expf(S[r * SS + jj] - m);
           S[r * SS + jj] = e;
           z += e;
         }
 #pragma unroll
-      for (int o = 4; o > 0; o >>= 1) z += __shfl_xor_sync(0xffffffffu, z, o);
+      for (int o = G / 2; o > 0; o >>= 1) z += __shfl_xor_sync(0xffffffffu, z, o);
       const float inv = i < C ? 1.f / z : 0.f;
-      for (int jj = l8; jj < Wa; jj += 8) Pr[r * PRS + jj] = (i < C && jj < W) ? f2bf(S[r * SS + jj] * inv) : 0;
+      for (int jj = l8; jj < Wa; jj += G) Pr[r * PRS + jj] = (i < C && jj < W) ? f2bf(S[r * SS + jj] * inv) : 0;
     }
     __syncthreads();
     // out = probabilities . v, one 16 x 8 tile of head columns per warp at a time
-    for (int nt = warp; nt < DH / 8; nt += 4) {
+    for (int nt = warp; nt < DH / 8; nt += kAttnThreads / 32) {
       float c[4] = {0.f, 0.f, 0.f, 0.f};
       for (int kk = 0; kk < Wa / 16; ++kk) {
         uint32_t af[4], bf[2];
@@ -381,8 +384,8 @@ int n_marks(const tsd_encoder* e) { return 1 + 15 * e->cfg.layers + 1 + 1; }
 void launch_attn(const tsd_encoder* e, const AttnArgs& a, int n, cudaStream_t s) {
   const size_t sm = attn_smem(e->cfg.d / e->cfg.heads, e->cfg.left, a.C);
   dim3 grid(n, e->cfg.heads);
-  if (e->cfg.d / e->cfg.heads == 64) k_attn<64><<<grid, 128, sm, s>>>(a);
-  else k_attn<128><<<grid, 128, sm, s>>>(a);
+  if (e->cfg.d / e->cfg.heads == 64) k_attn<64><<<grid, kAttnThreads, sm, s>>>(a);
+  else k_attn<128><<<grid, kAttnThreads, sm, s>>>(a);
 }
 
 template <bool FINAL>
