@@ -134,14 +134,14 @@ __device__ __forceinline__ void mma16816(float* c, const uint32_t* a, const uint
                : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b[0]), "r"(b[1]));
 }
 
-// One (stream, head) per CTA, 8 warps: chunked, limited-context attention
+// One (stream, head) per CTA, 16 warps: chunked, limited-context attention
 // with the relative-position term over the window [cached frames, chunk
 // frames].  The three products -- (q + u) against the keys, (q + v)
 // against the position-table rows, the probabilities against the values --
 // run on the tensor cores as 16 x 8 x 16 bf16 MMAs with fp32 accumulation
 // (a chunk has 13 query rows: one 16-row tile).  Then the chunk's k and v go
 // into the ring cache.
-constexpr int kAttnThreads = 256;
+constexpr int kAttnThreads = 512;
 
 template <int DH>
 __global__ void __launch_bounds__(kAttnThreads) k_attn(AttnArgs a) {
