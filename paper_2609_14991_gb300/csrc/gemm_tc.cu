@@ -47,8 +47,6 @@ __device__ __forceinline__ uint16_t bf16_bits(float v) {
   return *reinterpret_cast<const uint16_t*>(&b);
 }
 
-__device__ __forceinline__ float bf16_val(uint16_t u) { return __uint_as_float((uint32_t)u << 16); }
-
 template <int EPI>
 __global__ void __launch_bounds__(kGThreads, 1)
     k_gemm_tc(DecView d, GemmArgs g, const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB) {

@@ -171,7 +171,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int row = q * 32 + lane;
     const int gr = m0 + row;
     const bool live = gr < M;
-    const int N = d.N, V = d.V;
+    const int N = d.N;
     float mx = kNegInf, se = 0.f, bv = kNegInf;
     int bi = INT_MAX;
     const int K = d.topk;

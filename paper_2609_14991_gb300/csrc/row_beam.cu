@@ -110,7 +110,7 @@ __global__ void __launch_bounds__(kRowThreads) k_row_beam(DecView d, int step, i
   __shared__ double c_score[kMaxK * kMaxK];
   __shared__ float c_inc[kMaxK * kMaxK];
   __shared__ int c_tok[kMaxK * kMaxK];
-  __shared__ int s_sel[kMaxK], s_into[kMaxK], s_nsel;
+  __shared__ int s_sel[kMaxK], s_into[kMaxK];
   __shared__ int s_task0[kMaxK + 1];
   __shared__ int sr_lm[kMaxK][kLmChain];
   __shared__ int sr_trn[kMaxK][kTrChain], sr_trx[kMaxK][kTrChain];
@@ -289,7 +289,6 @@ __global__ void __launch_bounds__(kRowThreads) k_row_beam(DecView d, int step, i
         used[best] = true;
         s_sel[nsel++] = best;
       }
-      s_nsel = nsel;
       const bool last_exp = s_be >= S - 1;
       int cnt = 0;
       int pool_used = __ldcg(d.pool_n + slot);

@@ -35,7 +35,6 @@ __global__ void __launch_bounds__(kRowThreads) k_row_pruned(DecView d, int step,
   const bool commit = (mode != 2);
 
   __shared__ int s_t, s_sym, s_cnt, s_y, s_lm_len, s_tr_len, s_last, s_slot, s_T, s_nc;
-  __shared__ float s_score;
   __shared__ int s_lm[kLmChain], s_tr[kTrChain];
   __shared__ row::ChainRecs rc;
   __shared__ float c_logit[kMaxCand], c_fused[kMaxCand];

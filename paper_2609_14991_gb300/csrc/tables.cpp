@@ -402,7 +402,8 @@ extern "C" tsd_status tsd_boost_build(int32_t V, int32_t n_phr, const int32_t* o
   v.n_nodes = Q;
   v.max_depth = max_depth;
   v.bonus = token_bonus;
-  int32_t *a0, *a1, *a2, *a3, *a4, *a5, *a6, *a7, *a8;
+  int32_t *a0 = nullptr, *a1 = nullptr, *a2 = nullptr, *a3 = nullptr, *a4 = nullptr, *a5 = nullptr, *a6 = nullptr,
+          *a7 = nullptr, *a8 = nullptr;
   tsd_status st;
   ch_tok.resize(ch_tok.size() + 4, 0);  // aligned groups of four in the row pass
   if ((st = b->arena.upload(&a0, nd_begin)) || (st = b->arena.upload(&a1, nd_count)) ||
