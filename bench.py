@@ -60,12 +60,12 @@ KERNEL_SOURCES = {
     "row": ["row_pass.cu", "row_beam.cu", "row_common.cuh", "decoder.h", "internal.h"],
 }
 TRAFFIC = {
-    (2, 256, "joint"): (4480751, "62a394abb77c04c9"),
-    (2, 256, "row"): (2177050, "1fdffc2eebe3506b"),
-    (4, 1024, "joint"): (28862822, "62a394abb77c04c9"),
-    (4, 1024, "row"): (12059827, "1fdffc2eebe3506b"),
-    (3, 128, "joint"): (6344858, "62a394abb77c04c9"),
-    (3, 128, "row"): (1902558, "1fdffc2eebe3506b"),
+    (2, 256, "joint"): (4480879, "c364bfcf57dcdddc"),
+    (2, 256, "row"): (2176478, "4cb5e8bf2d6d8afb"),
+    (4, 1024, "joint"): (28863138, "c364bfcf57dcdddc"),
+    (4, 1024, "row"): (12059614, "4cb5e8bf2d6d8afb"),
+    (3, 128, "joint"): (6346155, "c364bfcf57dcdddc"),
+    (3, 128, "row"): (1901841, "4cb5e8bf2d6d8afb"),
 }
 
 
