@@ -126,6 +126,12 @@ __device__ __forceinline__ void ldsm_x2_trans(const void* p, uint32_t* r) {
                : "=r"(r[0]), "=r"(r[1])
                : "r"((uint32_t)__cvta_generic_to_shared(p)));
 }
+// 16-byte global -> shared copy that completes asynchronously (waited for
+// with cp.async.wait_group); both addresses 16-byte aligned.
+__device__ __forceinline__ void cp_async16(void* dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"((uint32_t)__cvta_generic_to_shared(dst)), "l"(src)
+               : "memory");
+}
 // D (16x8 fp32) += A (16x16 bf16, row-major) . B (16x8 bf16, column-major)
 __device__ __forceinline__ void mma16816(float* c, const uint32_t* a, const uint32_t* b) {
   asm volatile("mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
@@ -169,21 +175,33 @@ __global__ void __launch_bounds__(kAttnThreads) k_attn(AttnArgs a) {
 
   const size_t cb = (((size_t)slot * a.layers + a.layer) * a.heads + h) * (size_t)a.left * DH;
   const uint4 zero = make_uint4(0u, 0u, 0u, 0u);
+  // keys, values and table rows go global -> shared with asynchronous 16-byte
+  // copies (all of a thread's copies in flight at once); padding rows are
+  // zeroed with plain stores
   for (int idx = tid; idx < Wa * E8; idx += blockDim.x) {
     const int jj = idx / E8, e8 = idx - jj * E8;
-    uint4 kw = zero, vw = zero;
+    uint16_t* kd = Kb + jj * RS + 8 * e8;
+    uint16_t* vd = Vb + jj * RS + 8 * e8;
     if (jj < nv) {
       const int ring = (sn - nv + jj) % a.left;
-      kw = reinterpret_cast<const uint4*>(a.kc + cb + (size_t)ring * DH)[e8];
-      vw = reinterpret_cast<const uint4*>(a.vc + cb + (size_t)ring * DH)[e8];
+      cp_async16(kd, a.kc + cb + (size_t)ring * DH + 8 * e8);
+      cp_async16(vd, a.vc + cb + (size_t)ring * DH + 8 * e8);
     } else if (jj < W) {
-      const uint16_t* row = a.qkv + (size_t)(b * C + jj - nv) * 3 * d + h * DH;
-      kw = reinterpret_cast<const uint4*>(row + d)[e8];
-      vw = reinterpret_cast<const uint4*>(row + 2 * d)[e8];
+      const uint16_t* row = a.qkv + (size_t)(b * C + jj - nv) * 3 * d + h * DH + 8 * e8;
+      cp_async16(kd, row + d);
+      cp_async16(vd, row + 2 * d);
+    } else {
+      *reinterpret_cast<uint4*>(kd) = zero;
+      *reinterpret_cast<uint4*>(vd) = zero;
     }
-    *reinterpret_cast<uint4*>(Kb + jj * RS + 8 * e8) = kw;
-    *reinterpret_cast<uint4*>(Vb + jj * RS + 8 * e8) = vw;
   }
+  for (int idx = tid; idx < Na * E8; idx += blockDim.x) {
+    const int t = idx / E8, e8 = idx - t * E8;
+    uint16_t* pd = Pb + t * RS + 8 * e8;
+    if (t < nrel) cp_async16(pd, a.pos_tab + (size_t)(t + a.cmax - C) * d + h * DH + 8 * e8);
+    else *reinterpret_cast<uint4*>(pd) = zero;
+  }
+  asm volatile("cp.async.commit_group;" ::: "memory");
   for (int idx = tid; idx < CR * E8; idx += blockDim.x) {
     const int i = idx / E8, e8 = idx - i * E8;
     uint4 qu = zero, qv = zero;
@@ -204,22 +222,19 @@ __global__ void __launch_bounds__(kAttnThreads) k_attn(AttnArgs a) {
     *reinterpret_cast<uint4*>(Qu + i * RS + 8 * e8) = qu;
     *reinterpret_cast<uint4*>(Qv + i * RS + 8 * e8) = qv;
   }
-  for (int idx = tid; idx < Na * E8; idx += blockDim.x) {
-    const int t = idx / E8, e8 = idx - t * E8;
-    const uint4 pw = t < nrel ? reinterpret_cast<const uint4*>(a.pos_tab + (size_t)(t + a.cmax - C) * d + h * DH)[e8]
-                              : zero;
-    *reinterpret_cast<uint4*>(Pb + t * RS + 8 * e8) = pw;
-  }
+  asm volatile("cp.async.wait_group 0;" ::: "memory");
   __syncthreads();
-  // the cache was read above: the chunk's k and v replace the oldest frames
+  // the cache was read above: the chunk's k and v (window rows nv .. W-1 in
+  // shared memory) replace the oldest frames
   if (a.left > 0) {
     for (int idx = tid; idx < C * E8; idx += blockDim.x) {
       const int i = idx / E8, e8 = idx - i * E8;
       if (i < C - a.left) continue;
       const int ring = (sn + i) % a.left;
-      const uint16_t* row = a.qkv + (size_t)(b * C + i) * 3 * d + h * DH;
-      reinterpret_cast<uint4*>(a.kc + cb + (size_t)ring * DH)[e8] = reinterpret_cast<const uint4*>(row + d)[e8];
-      reinterpret_cast<uint4*>(a.vc + cb + (size_t)ring * DH)[e8] = reinterpret_cast<const uint4*>(row + 2 * d)[e8];
+      reinterpret_cast<uint4*>(a.kc + cb + (size_t)ring * DH)[e8] =
+          *reinterpret_cast<const uint4*>(Kb + (nv + i) * RS + 8 * e8);
+      reinterpret_cast<uint4*>(a.vc + cb + (size_t)ring * DH)[e8] =
+          *reinterpret_cast<const uint4*>(Vb + (nv + i) * RS + 8 * e8);
     }
   }
   const int fr = lane >> 2, fc = (lane & 3) * 2;  // this lane's place in a 16 x 8 result
@@ -314,7 +329,9 @@ __global__ void __launch_bounds__(128) k_dwconv(ConvArgs a) {
   const int K1 = K - 1, C = a.C, d = a.d;
   const int slot = a.slots[b];
   uint16_t* cc = a.cache + ((size_t)slot * a.layers + a.layer) * (size_t)K1 * d;
+#pragma unroll 4
   for (int t = 0; t < K1; ++t) seq[t * 128 + tid] = bf2f(cc[(size_t)t * d + c]);
+#pragma unroll 4
   for (int t = 0; t < C; ++t) seq[(K1 + t) * 128 + tid] = bf2f(a.glu[(size_t)(b * C + t) * d + c]);
   const float* w = a.w + (size_t)c * K;
   const float bias = a.bias[c], sc = a.sc[c], sh = a.sh[c];
