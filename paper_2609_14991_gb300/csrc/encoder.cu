@@ -412,11 +412,13 @@ void ln_launch(dim3 grid, cudaStream_t s, float* x, uint16_t* y, int M, int d, c
   else k_ln<FINAL, 16><<<grid, 256, 0, s>>>(x, y, M, d, g, b);
 }
 
-void enqueue(tsd_encoder* e, int n, int C, cudaStream_t s, const std::vector<cudaEvent_t>* ev,
-             std::vector<int8_t>* cls) {
+// The block sequence for streams [off, off + n) of the call (their rows
+// off*C .. (off+n)*C - 1 of every work buffer), on stream s.  With events,
+// each kernel's start is marked and classed (0 GEMM, 1 attention, 2 other).
+void enqueue_rows(tsd_encoder* e, int off, int n, int C, cudaStream_t s, const std::vector<cudaEvent_t>* ev,
+                  std::vector<int8_t>* cls, int& mk) {
   const tsd_encoder_cfg& c = e->cfg;
-  const int M = n * C, d = c.d;
-  int mk = 0;
+  const int M = n * C, d = c.d, r0 = off * C;
   auto mark = [&](int k) {
     if (!ev) return;
     cudaEventRecordWithFlags((*ev)[(size_t)mk], s, cudaEventRecordExternal);
@@ -427,44 +429,86 @@ void enqueue(tsd_encoder* e, int n, int C, cudaStream_t s, const std::vector<cud
   auto gemm = [&](int epi, const CUtensorMap& A, const CUtensorMap& B, int N, int K, const float* bias, void* out,
                   int ld, float alpha) {
     mark(0);
-    EGemm g{M, N, K, bias, out, ld, alpha, e->err};
+    EGemm g{M, N, K, bias, out, ld, alpha, e->err, r0};
     launch_egemm(epi, g, A, B, s);
   };
+  float* x = e->x + (size_t)r0 * d;
+  uint16_t* nrm = e->nrm + (size_t)r0 * d;
+  const int32_t* slots = e->slots_dev + off;
   gemm(kEInit, e->m_feat, e->m_sub, d, c.stack * c.feat, e->sub_b, e->x, d, 1.f);
   for (int l = 0; l < c.layers; ++l) {
     EncLayerDev& L = e->L[(size_t)l];
     mark(2);
-    ln_launch<false>(ln_grid, s, e->x, e->nrm, M, d, L.ln_ff1_g, L.ln_ff1_b);
+    ln_launch<false>(ln_grid, s, x, nrm, M, d, L.ln_ff1_g, L.ln_ff1_b);
     gemm(kESwish, e->m_nrm, L.m_ff1_w1, c.ff, d, L.ff1_b1, e->hid, c.ff, 1.f);
     gemm(kEResid, e->m_hid, L.m_ff1_w2, d, c.ff, L.ff1_b2, e->x, d, 0.5f);
     mark(2);
-    ln_launch<false>(ln_grid, s, e->x, e->nrm, M, d, L.ln_att_g, L.ln_att_b);
+    ln_launch<false>(ln_grid, s, x, nrm, M, d, L.ln_att_g, L.ln_att_b);
     gemm(kEPlain, e->m_nrm, L.m_qkv, 3 * d, d, L.qkv_b, e->qkv, 3 * d, 1.f);
     mark(1);
-    AttnArgs aa{e->qkv, e->att, L.pos_tab, L.pos_u, L.pos_v, e->kc, e->vc, e->seen, e->slots_dev,
-                d, c.heads, c.left, c.layers, l, C, c.max_chunk, 1.f / sqrtf((float)(d / c.heads))};
+    AttnArgs aa{e->qkv + (size_t)r0 * 3 * d, e->att + (size_t)r0 * d, L.pos_tab, L.pos_u, L.pos_v, e->kc, e->vc,
+                e->seen, slots, d, c.heads, c.left, c.layers, l, C, c.max_chunk, 1.f / sqrtf((float)(d / c.heads))};
     launch_attn(e, aa, n, s);
     gemm(kEResid, e->m_att, L.m_out, d, d, L.out_b, e->x, d, 1.f);
     mark(2);
-    ln_launch<false>(ln_grid, s, e->x, e->nrm, M, d, L.ln_conv_g, L.ln_conv_b);
+    ln_launch<false>(ln_grid, s, x, nrm, M, d, L.ln_conv_g, L.ln_conv_b);
     gemm(kEGlu, e->m_nrm, L.m_pw1, 2 * d, d, L.pw1_b, e->glu, d, 1.f);
     mark(2);
-    ConvArgs ca{e->glu, e->convz, e->cc, L.dw_w, L.dw_b, L.bn_scale, L.bn_shift, e->slots_dev, d, c.kernel, C,
-                c.layers, l};
+    ConvArgs ca{e->glu + (size_t)r0 * d, e->convz + (size_t)r0 * d, e->cc, L.dw_w, L.dw_b, L.bn_scale, L.bn_shift,
+                slots, d, c.kernel, C, c.layers, l};
     const size_t conv_smem = (size_t)(c.kernel - 1 + C) * 128 * sizeof(float);
     if (c.kernel == 9) k_dwconv<9><<<dim3(n, d / 128), 128, conv_smem, s>>>(ca);
     else k_dwconv<0><<<dim3(n, d / 128), 128, conv_smem, s>>>(ca);
     gemm(kEResid, e->m_convz, L.m_pw2, d, d, L.pw2_b, e->x, d, 1.f);
     mark(2);
-    ln_launch<false>(ln_grid, s, e->x, e->nrm, M, d, L.ln_ff2_g, L.ln_ff2_b);
+    ln_launch<false>(ln_grid, s, x, nrm, M, d, L.ln_ff2_g, L.ln_ff2_b);
     gemm(kESwish, e->m_nrm, L.m_ff2_w1, c.ff, d, L.ff2_b1, e->hid, c.ff, 1.f);
     gemm(kEResid, e->m_hid, L.m_ff2_w2, d, c.ff, L.ff2_b2, e->x, d, 0.5f);
     mark(2);
-    ln_launch<true>(ln_grid, s, e->x, l + 1 == c.layers ? e->outb : nullptr, M, d, L.ln_out_g, L.ln_out_b);
+    ln_launch<true>(ln_grid, s, x, l + 1 == c.layers ? e->outb + (size_t)r0 * d : nullptr, M, d, L.ln_out_g,
+                    L.ln_out_b);
   }
-  mark(2);
+}
+
+// Where the call's streams split into two halves that run as two branches
+// of the graph (rows of different streams never meet until the output, so
+// one half's attention, layer norms and convolution fill the SMs while the
+// other half's GEMMs run).  0: no split.  The split prefers a multiple of
+// the 128-row tile.
+int split_point(int n, int C) {
+  if (n < 2 || n * C < 512) return 0;
+  for (int k = n / 2; k < n; ++k)
+    if (k * C % 128 == 0) return k;
+  return n / 2;
+}
+
+// The whole chunk step on stream s.  With events (the instrumented pass) the
+// kernels run in one sequence so that every kernel boundary is marked;
+// otherwise the two halves of the call run as parallel branches.
+void enqueue(tsd_encoder* e, int n, int C, cudaStream_t s, const std::vector<cudaEvent_t>* ev,
+             std::vector<int8_t>* cls) {
+  int mk = 0;
+  const int n0 = ev ? 0 : split_point(n, C);
+  if (n0 == 0) {
+    enqueue_rows(e, 0, n, C, s, ev, cls, mk);
+  } else {
+    cudaEventRecord(e->fork_ev, s);
+    cudaStreamWaitEvent(e->cap_stream2, e->fork_ev, 0);
+    enqueue_rows(e, 0, n0, C, s, nullptr, nullptr, mk);
+    enqueue_rows(e, n0, n - n0, C, e->cap_stream2, nullptr, nullptr, mk);
+    cudaEventRecord(e->join_ev, e->cap_stream2);
+    cudaStreamWaitEvent(s, e->join_ev, 0);
+  }
+  if (ev) {
+    cudaEventRecordWithFlags((*ev)[(size_t)mk], s, cudaEventRecordExternal);
+    if (cls) (*cls)[(size_t)mk] = 2;
+    ++mk;
+  }
   k_advance<<<1, 256, 0, s>>>(e->seen, e->slots_dev, n, C);
-  mark(-1);
+  if (ev) {
+    cudaEventRecordWithFlags((*ev)[(size_t)mk], s, cudaEventRecordExternal);
+    if (cls) (*cls)[(size_t)mk] = -1;
+  }
 }
 
 void harvest(tsd_encoder* e, tsd_encoder::Graph& g) {
@@ -615,6 +659,9 @@ extern "C" tsd_status tsd_encoder_create(const tsd_encoder_cfg* cfg, const void*
   TSD_CUDA(cudaMallocHost(&e->slots_host, sizeof(int32_t) * (size_t)c.max_streams));
   TSD_CUDA(cudaEventCreateWithFlags(&e->slots_ev, cudaEventDisableTiming));
   TSD_CUDA(cudaStreamCreateWithFlags(&e->cap_stream, cudaStreamNonBlocking));
+  TSD_CUDA(cudaStreamCreateWithFlags(&e->cap_stream2, cudaStreamNonBlocking));
+  TSD_CUDA(cudaEventCreateWithFlags(&e->fork_ev, cudaEventDisableTiming));
+  TSD_CUDA(cudaEventCreateWithFlags(&e->join_ev, cudaEventDisableTiming));
   TSD_CUDA(cudaStreamSynchronize(s));
   TSD_CUDA(cudaGetLastError());
   e->slot_open.assign((size_t)c.max_streams, 0);

@@ -25,10 +25,12 @@ enum EncEpilogue {
 struct EGemm {
   int M, N, K;        // output rows, B rows (GLU: twice the outputs), inner size (multiple of 64)
   const float* bias;  // [N], in B's row order
-  void* out;          // kEInit / kEResid: float [M][ld]; otherwise bf16 [M][ld]
+  void* out;          // kEInit / kEResid: float [rows][ld]; otherwise bf16 [rows][ld]
   int ld;             // output row stride (elements)
   float alpha;        // kEResid
   unsigned int* err;  // device status word
+  int m0;             // first output row (rows m0 .. m0+M-1 of A and out; tiles past m0+M
+                      // may read further rows of A, but write nothing there)
 };
 
 constexpr int kEgBN = 128;  // output-tile width (B rows per tile)
@@ -75,6 +77,8 @@ struct tsd_encoder {
   int32_t* slots_host = nullptr;  // pinned staging for the slot list
   cudaEvent_t slots_ev = nullptr;
   cudaStream_t last_stream = nullptr, cap_stream = nullptr;
+  cudaStream_t cap_stream2 = nullptr;              // second branch of a captured chunk step
+  cudaEvent_t fork_ev = nullptr, join_ev = nullptr;  // its fork and join inside the capture
   // captured graphs per (n, C, timing)
   struct Graph {
     cudaGraphExec_t exec = nullptr;
@@ -96,6 +100,9 @@ struct tsd_encoder {
     if (slots_host) cudaFreeHost(slots_host);
     if (slots_ev) cudaEventDestroy(slots_ev);
     if (cap_stream) cudaStreamDestroy(cap_stream);
+    if (cap_stream2) cudaStreamDestroy(cap_stream2);
+    if (fork_ev) cudaEventDestroy(fork_ev);
+    if (join_ev) cudaEventDestroy(join_ev);
     arena.release();
     cudaGetLastError();
   }

@@ -88,7 +88,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       int it = 0;
       bool ok = true;
       for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x) {
-        const int m0 = (t % Mt) * kBM, n0 = (t / Mt) * kBN;
+        const int m0 = g.m0 + (t % Mt) * kBM, n0 = (t / Mt) * kBN;
         for (int kb = 0; kb < KB; ++kb, ++it) {
           const int s = it % kStages;
           const uint32_t ph = (uint32_t)(it / kStages) & 1u;
@@ -140,9 +140,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     bool ok = true;
     for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x, ++tl) {
       const int buf = tl & 1, use = tl >> 1;
-      const int m0 = (t % Mt) * kBM, n0 = (t / Mt) * kBN;
+      const int m0 = g.m0 + (t % Mt) * kBM, n0 = (t / Mt) * kBN;
       const int gr = m0 + q * 32 + lane;
-      const bool live = gr < g.M;
+      const bool live = gr < g.m0 + g.M;
       // each epilogue warp keeps its own copy of the tile's bias (no
       // cross-warp barrier: a warp that gives up cannot stall the others)
       float* bias = s_bias + ((warp - 2) * 2 + buf) * kBN;

@@ -149,6 +149,30 @@ def test_streams_do_not_interact():
         assert np.array_equal(a[2], b[0])
 
 
+def test_two_branch_split_inside_a_tile():
+    """A call of 40 streams x 13 frames (520 rows) runs as two parallel
+    halves of 20 streams whose boundary, row 260, falls inside a 128-row
+    tile: every stream's output is bit-identical to the same stream encoded
+    alone (a single-branch call), and two streams match the oracle."""
+    cfg = synth.EncoderCfg("split", d=256, layers=2, heads=4, ff=512, kernel=5, left=12, chunk=13, feat=16, stack=4)
+    w = synth.encoder_weights(cfg)
+    n = 40
+    many, one = _gpu(w, max_streams=n), _gpu(w, max_streams=n)
+    m_slots = [many.open() for _ in range(n)]
+    o_slots = [one.open() for _ in range(n)]
+    got = []
+    for c in range(3):
+        a = many.encode_chunk(m_slots, _feats(cfg, range(n), c * 13, 13)).cpu().numpy()
+        for i in (0, 19, 20, 21, 39):
+            b = one.encode_chunk([o_slots[i]], _feats(cfg, [i], c * 13, 13)).cpu().numpy()
+            assert np.array_equal(a[i], b[0]), (c, i)
+        got.append(a)
+    many.check()
+    got = np.stack(got, axis=1)
+    for s in (19, 20):
+        _close(got[s].view(np.uint16), _oracle_stream(w, s, 3, 13), 0.0095, 0.032)
+
+
 def test_reopened_slot_starts_fresh():
     cfg = SMALL
     w = synth.encoder_weights(cfg)
