@@ -470,34 +470,49 @@ void enqueue_rows(tsd_encoder* e, int off, int n, int C, cudaStream_t s, const s
   }
 }
 
-// Where the call's streams split into two halves that run as two branches
-// of the graph (rows of different streams never meet until the output, so
-// one half's attention, layer norms and convolution fill the SMs while the
-// other half's GEMMs run).  0: no split.  The split prefers a multiple of
-// the 128-row tile.
-int split_point(int n, int C) {
-  if (n < 2 || n * C < 512) return 0;
-  for (int k = n / 2; k < n; ++k)
-    if (k * C % 128 == 0) return k;
-  return n / 2;
+// How the call's streams split into parallel branches of the graph (rows of
+// different streams never meet until the output, so one branch's attention,
+// layer norms and convolution fill the SMs while another's GEMMs run):
+// branch i takes streams at[i] .. at[i+1]-1.  Up to kEncBranches branches
+// of at least 256 rows each; a boundary moves up to a multiple of the
+// 128-row tile where one lies within its share.  Returns the branch count.
+int branch_points(int n, int C, int* at) {
+  int P = std::min(kEncBranches, n * C / 256);
+  P = std::min(P, n);
+  at[0] = 0;
+  if (P < 2) {
+    at[1] = n;
+    return 1;
+  }
+  for (int i = 1; i < P; ++i) {
+    const int lo = i * n / P, hi = (i + 1) * n / P;
+    int k = lo;
+    while (k < hi && k * C % 128) ++k;
+    at[i] = k < hi ? k : lo;
+  }
+  at[P] = n;
+  return P;
 }
 
 // The whole chunk step on stream s.  With events (the instrumented pass) the
 // kernels run in one sequence so that every kernel boundary is marked;
-// otherwise the two halves of the call run as parallel branches.
+// otherwise the call's streams run as parallel branches.
 void enqueue(tsd_encoder* e, int n, int C, cudaStream_t s, const std::vector<cudaEvent_t>* ev,
              std::vector<int8_t>* cls) {
   int mk = 0;
-  const int n0 = ev ? 0 : split_point(n, C);
-  if (n0 == 0) {
+  int at[kEncBranches + 1];
+  const int P = ev ? 1 : branch_points(n, C, at);
+  if (P == 1) {
     enqueue_rows(e, 0, n, C, s, ev, cls, mk);
   } else {
     cudaEventRecord(e->fork_ev, s);
-    cudaStreamWaitEvent(e->cap_stream2, e->fork_ev, 0);
-    enqueue_rows(e, 0, n0, C, s, nullptr, nullptr, mk);
-    enqueue_rows(e, n0, n - n0, C, e->cap_stream2, nullptr, nullptr, mk);
-    cudaEventRecord(e->join_ev, e->cap_stream2);
-    cudaStreamWaitEvent(s, e->join_ev, 0);
+    for (int i = 1; i < P; ++i) cudaStreamWaitEvent(e->branch[i - 1], e->fork_ev, 0);
+    for (int i = 0; i < P; ++i)
+      enqueue_rows(e, at[i], at[i + 1] - at[i], C, i ? e->branch[i - 1] : s, nullptr, nullptr, mk);
+    for (int i = 1; i < P; ++i) {
+      cudaEventRecord(e->join_ev[i - 1], e->branch[i - 1]);
+      cudaStreamWaitEvent(s, e->join_ev[i - 1], 0);
+    }
   }
   if (ev) {
     cudaEventRecordWithFlags((*ev)[(size_t)mk], s, cudaEventRecordExternal);
@@ -659,9 +674,11 @@ extern "C" tsd_status tsd_encoder_create(const tsd_encoder_cfg* cfg, const void*
   TSD_CUDA(cudaMallocHost(&e->slots_host, sizeof(int32_t) * (size_t)c.max_streams));
   TSD_CUDA(cudaEventCreateWithFlags(&e->slots_ev, cudaEventDisableTiming));
   TSD_CUDA(cudaStreamCreateWithFlags(&e->cap_stream, cudaStreamNonBlocking));
-  TSD_CUDA(cudaStreamCreateWithFlags(&e->cap_stream2, cudaStreamNonBlocking));
   TSD_CUDA(cudaEventCreateWithFlags(&e->fork_ev, cudaEventDisableTiming));
-  TSD_CUDA(cudaEventCreateWithFlags(&e->join_ev, cudaEventDisableTiming));
+  for (int i = 0; i < kEncBranches - 1; ++i) {
+    TSD_CUDA(cudaStreamCreateWithFlags(&e->branch[i], cudaStreamNonBlocking));
+    TSD_CUDA(cudaEventCreateWithFlags(&e->join_ev[i], cudaEventDisableTiming));
+  }
   TSD_CUDA(cudaStreamSynchronize(s));
   TSD_CUDA(cudaGetLastError());
   e->slot_open.assign((size_t)c.max_streams, 0);

@@ -34,6 +34,7 @@ struct EGemm {
 };
 
 constexpr int kEgBN = 128;  // output-tile width (B rows per tile)
+constexpr int kEncBranches = 2;  // most parallel branches of the encoder's chunk graph
 
 bool egemm_map_a(CUtensorMap* m, const uint16_t* A, int rows, int K);
 bool egemm_map_b(CUtensorMap* m, const uint16_t* B, int rows, int K);
@@ -77,8 +78,9 @@ struct tsd_encoder {
   int32_t* slots_host = nullptr;  // pinned staging for the slot list
   cudaEvent_t slots_ev = nullptr;
   cudaStream_t last_stream = nullptr, cap_stream = nullptr;
-  cudaStream_t cap_stream2 = nullptr;              // second branch of a captured chunk step
-  cudaEvent_t fork_ev = nullptr, join_ev = nullptr;  // its fork and join inside the capture
+  // further branches of a captured chunk step, their fork and joins
+  cudaStream_t branch[tsd::kEncBranches - 1] = {};
+  cudaEvent_t fork_ev = nullptr, join_ev[tsd::kEncBranches - 1] = {};
   // captured graphs per (n, C, timing)
   struct Graph {
     cudaGraphExec_t exec = nullptr;
@@ -100,9 +102,11 @@ struct tsd_encoder {
     if (slots_host) cudaFreeHost(slots_host);
     if (slots_ev) cudaEventDestroy(slots_ev);
     if (cap_stream) cudaStreamDestroy(cap_stream);
-    if (cap_stream2) cudaStreamDestroy(cap_stream2);
+    for (int i = 0; i < tsd::kEncBranches - 1; ++i) {
+      if (branch[i]) cudaStreamDestroy(branch[i]);
+      if (join_ev[i]) cudaEventDestroy(join_ev[i]);
+    }
     if (fork_ev) cudaEventDestroy(fork_ev);
-    if (join_ev) cudaEventDestroy(join_ev);
     arena.release();
     cudaGetLastError();
   }
