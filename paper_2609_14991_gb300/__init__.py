@@ -110,6 +110,7 @@ SIGNATURES = {
     "tsd_encoder_set_timing": ([_vp, _i32], _i32),
     "tsd_encoder_timing": ([_vp, _vp, _vp, _i32, _i32], _i32),
     "tsd_encoder_gemm_flops": ([_vp, _i32, _i32, _P(ctypes.c_double)], _i32),
+    "tsd_encoder_launches_per_chunk": ([_vp, _i32, _i32, _P(_i64)], _i32),
 }
 
 _lib = None
@@ -592,4 +593,10 @@ class Encoder:
     def gemm_flops(self, n: int, C: int) -> float:
         x = ctypes.c_double()
         _check(lib().tsd_encoder_gemm_flops(self.h, n, C, ctypes.byref(x)))
+        return x.value
+
+    def launches_per_chunk(self, n: int, C: int) -> int:
+        """Kernel launches of one encode_chunk(n, C) with timing off."""
+        x = _i64()
+        _check(lib().tsd_encoder_launches_per_chunk(self.h, int(n), int(C), ctypes.byref(x)))
         return x.value

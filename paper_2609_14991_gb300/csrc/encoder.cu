@@ -831,3 +831,14 @@ extern "C" tsd_status tsd_encoder_gemm_flops(const tsd_encoder* e, int32_t n, in
   *flops = 2.0 * M * d * c.stack * c.feat + c.layers * 2.0 * M * (7.0 * d * d + 4.0 * ff * d);
   return TSD_OK;
 }
+
+extern "C" tsd_status tsd_encoder_launches_per_chunk(const tsd_encoder* e, int32_t n, int32_t C, int64_t* launches) {
+  clear_error();
+  if (!e || !launches) return fail(TSD_EINVAL, "tsd_encoder_launches_per_chunk: NULL argument");
+  if (n < 1 || n > e->cfg.max_streams || C < 1 || C > e->cfg.max_chunk)
+    return fail(TSD_EINVAL, "tsd_encoder_launches_per_chunk: n=%d C=%d out of range", n, C);
+  int at[kEncBranches + 1];
+  const int P = branch_points(n, C, at);
+  *launches = (int64_t)P * (1 + 15 * e->cfg.layers) + 1;
+  return TSD_OK;
+}

@@ -60,4 +60,6 @@ def test_null_handles_are_rejected():
     assert tsd.lib().tsd_encode_chunk(None, 1, None, None, 1, None, None) == tsd.TSD_EINVAL
     assert tsd.lib().tsd_encoder_open(None, None) == tsd.TSD_EINVAL
     assert tsd.lib().tsd_encoder_check(None) == tsd.TSD_EINVAL
+    x = ctypes.c_int64()
+    assert tsd.lib().tsd_encoder_launches_per_chunk(None, 1, 1, ctypes.byref(x)) == tsd.TSD_EINVAL
     tsd.lib().tsd_encoder_free(None)  # no-op
