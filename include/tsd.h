@@ -519,9 +519,11 @@ TSD_API tsd_status tsd_encoder_timing(tsd_encoder* enc, double* ms, int64_t* lau
 TSD_API tsd_status tsd_encoder_gemm_flops(const tsd_encoder* enc, int32_t n, int32_t C, double* flops);
 /* Kernel launches of one encode_chunk(n, C) with timing off (for launch
  * accounting): the call's streams run as up to two parallel graph branches
- * of at least 256 frame rows each, each branch the subsampling GEMM and 15
- * kernels per block, then one kernel that advances the frame counts.
- * TSD_EINVAL on n, C outside [1, max_streams] x [1, max_chunk]. */
+ * of at least 256 frame rows each, each branch the subsampling GEMM, the
+ * first block's first layer norm and 14 kernels per block (a block's
+ * closing layer norm also computes the next block's first one), then one
+ * kernel that advances the frame counts.  TSD_EINVAL on n, C outside
+ * [1, max_streams] x [1, max_chunk]. */
 TSD_API tsd_status tsd_encoder_launches_per_chunk(const tsd_encoder* enc, int32_t n, int32_t C, int64_t* launches);
 
 #ifdef __cplusplus

@@ -39,25 +39,15 @@ __device__ __forceinline__ float warp_sum(float v) {
   return v;
 }
 
-// Layer norm of rows of the fp32 stream x [M][d] (one warp per row; the row
-// stays in registers: lane j holds float4 groups j, j + 32, ..):
-// FINAL = false: y = bf16(LN(x)) (a module's input);
-// FINAL = true:  x = LN(x) in place, and y = bf16(LN(x)) when y != nullptr.
-template <bool FINAL, int kMaxQ>  // d <= 128 kMaxQ
-__global__ void __launch_bounds__(256) k_ln(float* x, uint16_t* y, int M, int d, const float* g, const float* b) {
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int r = blockIdx.x * 8 + warp;
-  if (r >= M) return;
-  float* xr = x + (size_t)r * d;
-  const int nq = d / 128;  // float4 groups per lane
-  float4 v[kMaxQ];
+// v := LN(v) * g + b over a row held by one warp (lane j holds the float4
+// groups j, j + 32, ..; nq groups per lane): mean, then the variance about
+// it, in fp32.
+template <int kMaxQ>
+__device__ __forceinline__ void ln_regs(float4 (&v)[kMaxQ], int nq, int d, int lane, const float* g, const float* b) {
   float s = 0.f;
 #pragma unroll
   for (int i = 0; i < kMaxQ; ++i)
-    if (i < nq) {
-      v[i] = *reinterpret_cast<const float4*>(xr + 128 * i + 4 * lane);
-      s += (v[i].x + v[i].y) + (v[i].z + v[i].w);
-    }
+    if (i < nq) s += (v[i].x + v[i].y) + (v[i].z + v[i].w);
   const float mean = warp_sum(s) / (float)d;
   float q = 0.f;
 #pragma unroll
@@ -73,16 +63,50 @@ __global__ void __launch_bounds__(256) k_ln(float* x, uint16_t* y, int M, int d,
       const int c = 128 * i + 4 * lane;
       const float4 gg = *reinterpret_cast<const float4*>(g + c);
       const float4 be = *reinterpret_cast<const float4*>(b + c);
-      const float o0 = (v[i].x - mean) * rstd * gg.x + be.x, o1 = (v[i].y - mean) * rstd * gg.y + be.y;
-      const float o2 = (v[i].z - mean) * rstd * gg.z + be.z, o3 = (v[i].w - mean) * rstd * gg.w + be.w;
-      if (FINAL) *reinterpret_cast<float4*>(xr + c) = make_float4(o0, o1, o2, o3);
-      if (y) {
-        uint2 w;
-        w.x = (uint32_t)f2bf(o0) | ((uint32_t)f2bf(o1) << 16);
-        w.y = (uint32_t)f2bf(o2) | ((uint32_t)f2bf(o3) << 16);
-        *reinterpret_cast<uint2*>(y + (size_t)r * d + c) = w;
-      }
+      v[i] = make_float4((v[i].x - mean) * rstd * gg.x + be.x, (v[i].y - mean) * rstd * gg.y + be.y,
+                         (v[i].z - mean) * rstd * gg.z + be.z, (v[i].w - mean) * rstd * gg.w + be.w);
     }
+}
+
+template <int kMaxQ>
+__device__ __forceinline__ void store_bf16(uint16_t* yr, const float4 (&v)[kMaxQ], int nq, int lane) {
+#pragma unroll
+  for (int i = 0; i < kMaxQ; ++i)
+    if (i < nq) {
+      uint2 w;
+      w.x = (uint32_t)f2bf(v[i].x) | ((uint32_t)f2bf(v[i].y) << 16);
+      w.y = (uint32_t)f2bf(v[i].z) | ((uint32_t)f2bf(v[i].w) << 16);
+      *reinterpret_cast<uint2*>(yr + 128 * i + 4 * lane) = w;
+    }
+}
+
+// Layer norms of rows of the fp32 stream x [M][d], one warp per row, the row
+// in registers:
+// FINAL = false: y = bf16(LN_1(x)) (a module's input);
+// FINAL = true:  x = LN_1(x) in place (a block's closing norm), then, with
+//                g2 != nullptr, y = bf16(LN_2(x)) (the next block's first
+//                module input, from the same registers), else y = bf16(x)
+//                when y != nullptr (the encoder's output).
+template <bool FINAL, int kMaxQ>  // d <= 128 kMaxQ
+__global__ void __launch_bounds__(256) k_ln(float* x, uint16_t* y, int M, int d, const float* g, const float* b,
+                                            const float* g2, const float* b2) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int r = blockIdx.x * 8 + warp;
+  if (r >= M) return;
+  float* xr = x + (size_t)r * d;
+  const int nq = d / 128;  // float4 groups per lane
+  float4 v[kMaxQ];
+#pragma unroll
+  for (int i = 0; i < kMaxQ; ++i)
+    if (i < nq) v[i] = *reinterpret_cast<const float4*>(xr + 128 * i + 4 * lane);
+  ln_regs<kMaxQ>(v, nq, d, lane, g, b);
+  if (FINAL) {
+#pragma unroll
+    for (int i = 0; i < kMaxQ; ++i)
+      if (i < nq) *reinterpret_cast<float4*>(xr + 128 * i + 4 * lane) = v[i];
+    if (g2) ln_regs<kMaxQ>(v, nq, d, lane, g2, b2);
+  }
+  if (y) store_bf16<kMaxQ>(y + (size_t)r * d, v, nq, lane);
 }
 
 struct AttnArgs {
@@ -396,7 +420,7 @@ tsd_status set_device(tsd_encoder* e) {
   return TSD_OK;
 }
 
-int n_marks(const tsd_encoder* e) { return 1 + 15 * e->cfg.layers + 1 + 1; }
+int n_marks(const tsd_encoder* e) { return 2 + 14 * e->cfg.layers + 1 + 1; }
 
 void launch_attn(const tsd_encoder* e, const AttnArgs& a, int n, cudaStream_t s) {
   const size_t sm = attn_smem(e->cfg.d / e->cfg.heads, e->cfg.left, a.C);
@@ -406,10 +430,11 @@ void launch_attn(const tsd_encoder* e, const AttnArgs& a, int n, cudaStream_t s)
 }
 
 template <bool FINAL>
-void ln_launch(dim3 grid, cudaStream_t s, float* x, uint16_t* y, int M, int d, const float* g, const float* b) {
-  if (d <= 512) k_ln<FINAL, 4><<<grid, 256, 0, s>>>(x, y, M, d, g, b);
-  else if (d <= 1024) k_ln<FINAL, 8><<<grid, 256, 0, s>>>(x, y, M, d, g, b);
-  else k_ln<FINAL, 16><<<grid, 256, 0, s>>>(x, y, M, d, g, b);
+void ln_launch(dim3 grid, cudaStream_t s, float* x, uint16_t* y, int M, int d, const float* g, const float* b,
+               const float* g2 = nullptr, const float* b2 = nullptr) {
+  if (d <= 512) k_ln<FINAL, 4><<<grid, 256, 0, s>>>(x, y, M, d, g, b, g2, b2);
+  else if (d <= 1024) k_ln<FINAL, 8><<<grid, 256, 0, s>>>(x, y, M, d, g, b, g2, b2);
+  else k_ln<FINAL, 16><<<grid, 256, 0, s>>>(x, y, M, d, g, b, g2, b2);
 }
 
 // The block sequence for streams [off, off + n) of the call (their rows
@@ -436,10 +461,11 @@ void enqueue_rows(tsd_encoder* e, int off, int n, int C, cudaStream_t s, const s
   uint16_t* nrm = e->nrm + (size_t)r0 * d;
   const int32_t* slots = e->slots_dev + off;
   gemm(kEInit, e->m_feat, e->m_sub, d, c.stack * c.feat, e->sub_b, e->x, d, 1.f);
+  mark(2);
+  ln_launch<false>(ln_grid, s, x, nrm, M, d, e->L[0].ln_ff1_g, e->L[0].ln_ff1_b);
   for (int l = 0; l < c.layers; ++l) {
     EncLayerDev& L = e->L[(size_t)l];
-    mark(2);
-    ln_launch<false>(ln_grid, s, x, nrm, M, d, L.ln_ff1_g, L.ln_ff1_b);
+    // the first module's norm of this block ran with the previous block's closing norm
     gemm(kESwish, e->m_nrm, L.m_ff1_w1, c.ff, d, L.ff1_b1, e->hid, c.ff, 1.f);
     gemm(kEResid, e->m_hid, L.m_ff1_w2, d, c.ff, L.ff1_b2, e->x, d, 0.5f);
     mark(2);
@@ -465,8 +491,11 @@ void enqueue_rows(tsd_encoder* e, int off, int n, int C, cudaStream_t s, const s
     gemm(kESwish, e->m_nrm, L.m_ff2_w1, c.ff, d, L.ff2_b1, e->hid, c.ff, 1.f);
     gemm(kEResid, e->m_hid, L.m_ff2_w2, d, c.ff, L.ff2_b2, e->x, d, 0.5f);
     mark(2);
-    ln_launch<true>(ln_grid, s, x, l + 1 == c.layers ? e->outb + (size_t)r0 * d : nullptr, M, d, L.ln_out_g,
-                    L.ln_out_b);
+    if (l + 1 < c.layers)
+      ln_launch<true>(ln_grid, s, x, nrm, M, d, L.ln_out_g, L.ln_out_b, e->L[(size_t)l + 1].ln_ff1_g,
+                      e->L[(size_t)l + 1].ln_ff1_b);
+    else
+      ln_launch<true>(ln_grid, s, x, e->outb + (size_t)r0 * d, M, d, L.ln_out_g, L.ln_out_b);
   }
 }
 
@@ -839,6 +868,6 @@ extern "C" tsd_status tsd_encoder_launches_per_chunk(const tsd_encoder* e, int32
     return fail(TSD_EINVAL, "tsd_encoder_launches_per_chunk: n=%d C=%d out of range", n, C);
   int at[kEncBranches + 1];
   const int P = branch_points(n, C, at);
-  *launches = (int64_t)P * (1 + 15 * e->cfg.layers) + 1;
+  *launches = (int64_t)P * (2 + 14 * e->cfg.layers) + 1;
   return TSD_OK;
 }

@@ -168,9 +168,9 @@ def test_two_branch_split_inside_a_tile():
             assert np.array_equal(a[i], b[0]), (c, i)
         got.append(a)
     many.check()
-    # two branches of (subsampling + 15 kernels per block), then the frame counts
-    assert many.launches_per_chunk(n, 13) == 2 * (1 + 15 * 2) + 1
-    assert one.launches_per_chunk(1, 13) == 1 + 15 * 2 + 1
+    # two branches of (subsampling, the first layer norm, 14 kernels per block), then the frame counts
+    assert many.launches_per_chunk(n, 13) == 2 * (2 + 14 * 2) + 1
+    assert one.launches_per_chunk(1, 13) == 2 + 14 * 2 + 1
     got = np.stack(got, axis=1)
     for s in (19, 20):
         _close(got[s].view(np.uint16), _oracle_stream(w, s, 3, 13), 0.0095, 0.032)
