@@ -58,6 +58,7 @@ def peaks():
 KERNEL_SOURCES = {
     "joint": ["joint_tc.cu", "joint_tc.h", "tc_common.cuh", "decoder.h", "internal.h"],
     "row": ["row_pass.cu", "row_beam.cu", "row_common.cuh", "decoder.h", "internal.h"],
+    "egemm": ["encoder_gemm.cu", "encoder.cu", "encoder.h", "tc_common.cuh", "internal.h"],
 }
 TRAFFIC = {
     (2, 256, "joint"): (4480879, "c364bfcf57dcdddc"),
@@ -79,8 +80,15 @@ def kernel_source_hash(kernel: str) -> str:
     return h.hexdigest()[:16]
 
 
-def recorded_traffic(w: synth.Workload, kernel: str):
-    rec = TRAFFIC.get((w.cfg, w.B, kernel))
+# The encoder GEMMs' DRAM traffic per chunk (every k_egemm launch of one
+# chunk step, summed), keyed by (encoder shape, streams, frames per chunk).
+ENC_TRAFFIC = {
+    ("0.6b", 256, 13): (5934569801, "7794f5c88b32f9a0"),
+}
+
+
+def recorded_traffic(w: synth.Workload, kernel: str, key=None):
+    rec = (ENC_TRAFFIC if key else TRAFFIC).get(key or (w.cfg, w.B, kernel))
     if rec is None or rec[1] != kernel_source_hash(kernel):
         return None
     return rec[0]
@@ -601,7 +609,9 @@ def run_ours(args, w):
                     "peak": pk["bf16_tflops_sustained"],
                     "peak_kind": f"{pk_kind} bf16 sustained (kernels timed inside the step)",
                     "algorithmic": f"{enc_flop:.4g} FLOP per chunk (M={w.B * w.T} frame rows, 2 M N K per GEMM)",
-                    "ms_per_chunk": gemm_chunk_ms, "launches": enc_n["gemm"], "traffic": None,
+                    "ms_per_chunk": gemm_chunk_ms, "launches": enc_n["gemm"],
+                    "traffic": recorded_traffic(w, "egemm", (args.encoder, w.B, w.T)),
+                    "traffic_unit": "DRAM bytes per chunk (all encoder GEMM launches of one chunk step)",
                     "share_of_device_time": share_enc,
                     "encoder_other_kernels": {
                         "attention_ms_per_chunk": enc_ms["attention"] / args.steps,
