@@ -178,12 +178,13 @@ tsd_status create_impl(const tsd_decoder_cfg* cfg, const void* W_out_bf16, const
 
   DevArena& A = d->arena;
   DecView& v = d->view;
-  uint16_t *Wt, *E, *Abuf;
-  float* bias;
-  float4* part;
-  int32_t *rt, *rs, *rc, *sl, *sll, *slc, *stl, *stc, *err;
+  uint16_t *Wt = nullptr, *E = nullptr, *Abuf = nullptr;
+  float* bias = nullptr;
+  float4* part = nullptr;
+  int32_t *rt = nullptr, *rs = nullptr, *rc = nullptr, *sl = nullptr, *sll = nullptr, *slc = nullptr, *stl = nullptr,
+          *stc = nullptr, *err = nullptr;
   int4 *slr = nullptr, *strc = nullptr;
-  unsigned long long* ctr;
+  unsigned long long* ctr = nullptr;
   float2* bpart = nullptr;
   float* dflt = nullptr;
   uint32_t* droot = nullptr;
