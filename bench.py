@@ -5,11 +5,14 @@ A step is one decode_chunk call: a 13-frame encoder chunk (the paper's
 path -- joint GEMM, log-softmax, LM and phrase-boost fusion, greedy
 selection and state advance, T*max_symbols label steps.
 
-Workload (default): B=256 streams, H=1024, V=1024+blank (0.6B-model-sized
-joint), 6-gram LM with ~20M n-grams, 5,000 boost phrases, lambda=0.5,
-beta=1.5, greedy with at most 5 labels per frame; synthetic seeded data.
+Workload (default, the largest configuration that fits one GPU): B=1024
+streams, H=1024, V=4096+blank, a 10-gram LM with ~100M n-grams over Zipf(1.05)
+unigrams, 50,000 boost phrases, lambda=0.6, beta=1.5, greedy with at most 5
+labels per frame; synthetic seeded data.  The same run also times the
+workload at B = 1, 16 and 128 streams (latency against throughput).
+--config 0..3 selects the smaller workloads.
 
-  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference] [--config C]
 
 The reference arm (--impl reference) times the CPU oracle on this host's
 cores on a bounded sample of the same workload and reports the same metric.
@@ -328,6 +331,43 @@ def run_reference(args, w):
     print(json.dumps(line), flush=True)
 
 
+def stream_sweep(args, w, tsd, dev, stream, W, E, lm, lms, bo, pw, flush):
+    """Frames/s and chunk latency of the same workload at the stream counts in
+    args.sweep (one decoder each, same tables), K timed chunks after W
+    warm-up chunks, L2 flushed before every timed chunk."""
+    import torch
+
+    out = []
+    for B in args.sweep:
+        if B == w.B or B < 1:
+            continue
+        d = tsd.Decoder(w.V, w.H, torch.from_numpy(W.view(np.int16)).to(dev),
+                        torch.from_numpy(E.view(np.int16)).to(dev), lm=None if lms else lm, lms=lms, boost=bo,
+                        max_symbols=w.max_sym, beam_k=w.beam, max_streams=B, max_T=w.T, prune_k=args.prune_k,
+                        pred=pw)
+        sl = np.array([d.open() for _ in range(B)], dtype=np.int32)
+        encs = [torch.from_numpy(synth.enc_chunk(w, range(B), c % w.chunks).view(np.int16)).to(dev)
+                for c in range(args.warmup + args.steps)]
+        o = d.alloc_out(B, w.T)
+        op = (o.tokens.data_ptr(), o.frames.data_ptr(), o.scores.data_ptr(), o.counts.data_ptr())
+        for c in range(args.warmup):
+            d.decode_chunk_raw(sl, encs[c].data_ptr(), w.T, w.lam, w.beta, op, stream.cuda_stream)
+        torch.cuda.synchronize()
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+        for k, (a, b) in enumerate(ev):
+            flush.zero_()
+            a.record(stream)
+            d.decode_chunk_raw(sl, encs[args.warmup + k].data_ptr(), w.T, w.lam, w.beta, op, stream.cuda_stream)
+            b.record(stream)
+        torch.cuda.synchronize()
+        d.check()
+        per = [a.elapsed_time(b) for a, b in ev]
+        out.append({"B": B, "value": B * w.T * args.steps / (sum(per) / 1000.0), "ms_per_chunk": sum(per) / len(per),
+                    **{k: v for k, v in latency_stats(per).items() if k != "steps"}})
+        del d
+    return out
+
+
 def run_ours(args, w):
     import torch
 
@@ -451,7 +491,7 @@ def run_ours(args, w):
     dev_enc = [torch.empty_like(encs[0]) for _ in range(2)]
     host_out = [torch.empty(t.shape, dtype=t.dtype, pin_memory=True) for t in
                 (out.tokens, out.frames, out.scores, out.counts)]
-    e2e_steps = min(args.steps, 8)
+    e2e_steps = args.steps  # the same K steps as the headline
     copy_stream = torch.cuda.Stream()
     copied = [torch.cuda.Event() for _ in range(2)]
     consumed = [torch.cuda.Event() for _ in range(2)]
@@ -507,6 +547,13 @@ def run_ours(args, w):
     joint_cold, joint_warm = replay_times(1)
     row_bytes = dec.replay(0, 1, count_bytes=True)
     joint_bytes = dec.replay(1, 1, count_bytes=True)
+
+    sweep = None
+    if args.sweep and ws == 1:
+        sweep = stream_sweep(args, w, tsd, dev, stream, W, E, lm, lms, bo, pw, flush)
+        sweep.append({"B": w.B, "value": value, "ms_per_chunk": t_ms / args.steps,
+                      **{k: v for k, v in latency_stats(step_ms).items() if k != "steps"}})
+        sweep.sort(key=lambda x: x["B"])
 
     if rank != 0:
         return
@@ -650,6 +697,10 @@ def run_ours(args, w):
             "roofline_other_kernel": other,
             **({"roofline_third_kernel": ranked[2][1]} if len(ranked) > 2 else {}),
             "latency_per_chunk": latency_stats(step_ms),
+            **({"stream_sweep": {"what": "the same workload (tables, weights, lambda, beta) decoded at other stream "
+                                         "counts B in this run: frames/s over K timed chunks (L2 flushed before "
+                                         "each) and chunk latency; 1 chunk = T x 80 ms of audio",
+                                 "points": sweep}} if sweep else {}),
             **({"first_token_latency_s": {
                 "value": w.T * 0.080 + float(np.median(step_ms)) / 1000.0,
                 "what": "a chunk's audio (T x 80 ms) arrives before it is encoded, then the chunk's encoder and "
@@ -665,8 +716,14 @@ def run_ours(args, w):
         n_cpu = min(args.cpu_streams, 16) if enc_o is not None else args.cpu_streams
         v, cores, sample, dt = oracle_baseline(w, models, list(range(n_cpu)), 1 if enc_o else args.cpu_chunks,
                                                prune_k=args.prune_k, encoder=enc_o)
+        # the same oracle on one host thread, on a smaller sample of the same streams
+        n_one = max(1, min(n_cpu, args.cpu_streams_single))
+        v1, _, sample1, dt1 = oracle_baseline(w, models, list(range(n_one)), 1, threads=1, prune_k=args.prune_k,
+                                              encoder=enc_o)
         line["cpu_baseline"] = {"value": v, "unit": UNIT, "cores": cores, "kind": "oracle",
-                                "sample": sample, "seconds": dt}
+                                "sample": sample, "seconds": dt,
+                                "single_thread": {"value": v1, "unit": UNIT, "cores": 1, "sample": sample1,
+                                                  "seconds": dt1}}
     print(json.dumps(line), flush=True)
 
 
@@ -676,11 +733,13 @@ def main():
     ap.add_argument("--steps", type=int, default=20)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    ap.add_argument("--config", type=int, default=2)
+    ap.add_argument("--config", type=int, default=4)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-streams", type=int, default=None)
     ap.add_argument("--cpu-chunks", type=int, default=None)
-    ap.add_argument("--ref-streams", type=int, default=64)
+    ap.add_argument("--ref-streams", type=int, default=None, help="streams per step of the reference arm")
+    ap.add_argument("--sweep", default=None,
+                    help="comma-separated stream counts also timed in this run (config 4 default: 1,16,128)")
     ap.add_argument("--streams", type=int, default=None, help="streams B per GPU (default: the config's)")
     ap.add_argument("--extra-lms", type=int, default=0, help="fuse this many further LMs (several-LM workload)")
     ap.add_argument("--prune-k", type=int, default=0,
@@ -696,9 +755,14 @@ def main():
         ap.error("--warmup must be >= 3")
     w = workload(args.config, args.streams)
     # bounded CPU samples (about 10-30 s of oracle work on 16 cores)
-    cpu_default = {0: (4, 1), 1: (64, 12), 2: (256, 6), 3: (64, 2), 4: (32, 1)}[args.config]
+    cpu_default = {0: (4, 1), 1: (64, 12), 2: (256, 6), 3: (64, 2), 4: (64, 1)}[args.config]
     args.cpu_streams = args.cpu_streams or min(cpu_default[0], w.B)
     args.cpu_chunks = args.cpu_chunks or cpu_default[1]
+    args.cpu_streams_single = {0: 4, 1: 8, 2: 8, 3: 4, 4: 4}[args.config]
+    args.ref_streams = args.ref_streams or {4: 32}.get(args.config, 64)
+    if args.sweep is None:
+        args.sweep = "1,16,128" if args.config == 4 and not args.streams else ""
+    args.sweep = [int(x) for x in args.sweep.split(",") if x.strip()]
     if args.impl == "reference":
         run_reference(args, w)
     else:

@@ -399,7 +399,10 @@ TSD_API tsd_status tsd_decoder_replay(tsd_decoder* dec, int32_t kernel, int32_t 
  * memory is a 1 MiB array compiled into the library, which every GPU that
  * loads the library keeps until the process exits.  The first call on a
  * device looks up that array's device address (cudaGetSymbolAddress); make
- * that first call before any stream capture.  All calls share the array:
+ * that first call before any stream capture.  The address is cached per
+ * device for the life of the process: after cudaDeviceReset on a device the
+ * cached address is stale, so do not call this entry point again on that
+ * device in the same process.  All calls share the array:
  * calls that overlap on the GPU (different streams, or host threads on one
  * device without ordering) race and must be serialized by the caller.
  * Asynchronous on cuda_stream. */

@@ -253,8 +253,32 @@ def joint_select_noalloc(A, Wt, bias, out_label, out_score, stream=None):
     that cannot allocate device memory.  A: cuda bf16 [n, H]; Wt: cuda bf16
     [V+1, H]; bias: cuda fp32 [n, V] or None; out_label: cuda int32 [n];
     out_score: cuda fp32 [n].  Nothing is allocated by this call."""
+    import torch
+
+    named = {"A": A, "Wt": Wt, "out_label": out_label, "out_score": out_score}
+    if bias is not None:
+        named["bias"] = bias
+    for name, t in named.items():
+        if not isinstance(t, torch.Tensor):
+            raise TypeError(f"joint_select_noalloc: {name} must be a torch tensor")
+    if A.dim() != 2 or A.dtype != torch.bfloat16:
+        raise ValueError("joint_select_noalloc: A must be bf16 [n, H]")
     n, H = A.shape
+    if Wt.dim() != 2 or Wt.element_size() != 2 or Wt.shape[1] != H:
+        raise ValueError(f"joint_select_noalloc: Wt must be 2-byte [V+1, H] with H = {H}")
     V = Wt.shape[0] - 1
+    if bias is not None and (bias.dtype != torch.float32 or tuple(bias.shape) != (n, V)):
+        raise ValueError(f"joint_select_noalloc: bias must be float32 [{n}, {V}]")
+    if out_label.dtype != torch.int32 or out_label.numel() < n:
+        raise ValueError(f"joint_select_noalloc: out_label must be int32 with at least {n} elements")
+    if out_score.dtype != torch.float32 or out_score.numel() < n:
+        raise ValueError(f"joint_select_noalloc: out_score must be float32 with at least {n} elements")
+    dev = torch.cuda.current_device() if torch.cuda.is_available() else None
+    for name, t in named.items():
+        if not t.is_cuda or t.device.index != dev:
+            raise ValueError(f"joint_select_noalloc: {name} must be a CUDA tensor on the current device")
+        if not t.is_contiguous():
+            raise ValueError(f"joint_select_noalloc: {name} must be contiguous")
     _check(lib().tsd_joint_select_noalloc(n, H, V, _ptr(A), _ptr(Wt), _ptr(bias) if bias is not None else None,
                                           _ptr(out_label), _ptr(out_score), _stream(stream)))
 

@@ -44,7 +44,7 @@ def _stale(target: str, deps: List[str]) -> bool:
 
 def build(force: bool = False, verbose: bool = False, extra: List[str] = ()) -> str:
     os.makedirs(BUILD_DIR, exist_ok=True)
-    headers = [os.path.join(CSRC, f) for f in os.listdir(CSRC) if f.endswith(".h")] + [os.path.join(INCLUDE, "tsd.h")]
+    headers = [os.path.join(CSRC, f) for f in os.listdir(CSRC) if f.endswith((".h", ".cuh"))] + [os.path.join(INCLUDE, "tsd.h")]
     objs, jobs = [], []
     for src in SOURCES:
         path = os.path.join(CSRC, src)

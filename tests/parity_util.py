@@ -116,13 +116,14 @@ class GpuRun:
         return d["tok"][i, :k], d["frame"][i, :k], d["score"][i, :k]
 
 
-def replay_stream(inp: Inputs, run: GpuRun, i: int, olm, obo, model) -> Dict:
-    """Oracle replay of the i-th stream of a GPU run over all its chunks."""
+def replay_stream(inp: Inputs, run: GpuRun, i: int, olm, obo, model, chunks: Optional[int] = None) -> Dict:
+    """Oracle replay of the i-th stream of a GPU run over its first `chunks`
+    chunks (all by default)."""
     w = inp.w
     st = oracle.Stream(w.V)
     rep_all = {"steps": 0, "mismatch": 0, "near_tie": 0, "max_score_diff": 0.0, "min_gap": np.inf,
                "inconsistent": 0, "state_errors": []}
-    for c in range(len(run.chunks)):
+    for c in range(len(run.chunks) if chunks is None else min(chunks, len(run.chunks))):
         tok, fr, sc = run.emitted(i, c)
         _, _, _, rep = oracle.decode_chunk(st, model, olm, obo, run.enc[c][i], inp.lam, inp.beta, w.max_sym,
                                            follow=(tok, fr, sc), gap_tol=GAP_TOL)
@@ -158,11 +159,35 @@ def oracle_models(inp: Inputs):
     return olm, obo, model
 
 
-def replay(inp: Inputs, run: GpuRun, sample: Sequence[int], threads: Optional[int] = None) -> List[Dict]:
-    olm, obo, model = oracle_models(inp)
+def replay(inp: Inputs, run: GpuRun, sample: Sequence[int], threads: Optional[int] = None,
+           chunks: Optional[int] = None, models=None) -> List[Dict]:
+    olm, obo, model = models or oracle_models(inp)
     threads = threads or min(len(sample), os.cpu_count() or 4)
     with concurrent.futures.ThreadPoolExecutor(max_workers=threads) as ex:
-        return list(ex.map(lambda i: replay_stream(inp, run, i, olm, obo, model), sample))
+        return list(ex.map(lambda i: replay_stream(inp, run, i, olm, obo, model, chunks), sample))
+
+
+def captured_logit_error(run: GpuRun, model, steps: int, rows: Sequence[int], threads: Optional[int] = None):
+    """Largest |GPU logit - oracle logit| over the captured steps and rows of
+    the run's last chunk (capture keeps the last decode call's steps): every
+    label of every (step, row) the row was evaluated at, against the oracle's
+    double product of the same bf16 inputs (joint_logits of the captured
+    frame and previous label).  Returns (max error, rows checked)."""
+    caps = run.cap_rows.cpu().numpy()
+    logits = run.cap_logits.cpu().numpy()
+    K = run.K
+    jobs = [(s, r) for s in range(min(steps, caps.shape[0])) for r in rows if caps[s, r, 0] >= 0]
+
+    def one(job):
+        s, r = job
+        t, last = int(caps[s, r, 0]), int(caps[s, r, 1])
+        want = model.joint_logits(run.enc[-1][r // K][t], last)
+        return float(np.abs(logits[s, r] - want).max())
+
+    threads = threads or (os.cpu_count() or 4)
+    with concurrent.futures.ThreadPoolExecutor(max_workers=threads) as ex:
+        errs = list(ex.map(one, jobs))
+    return (max(errs) if errs else 0.0), len(jobs)
 
 
 def assert_reports(reps: List[Dict]):

@@ -110,3 +110,26 @@ def test_null_handles(L):
     L.tsd_ngram_free(None)
     L.tsd_boost_free(None)
     L.tsd_decoder_free(None)
+
+
+def test_noalloc_binding_rejects_bad_tensors_before_the_call(L):
+    """The allocation-free entry point's binding checks its tensors (types,
+    shapes, dtypes, device) before anything reaches the library: a mismatched
+    hidden size and host tensors both raise."""
+    torch = pytest.importorskip("torch")
+    A = torch.zeros((4, 64), dtype=torch.bfloat16)
+    Wt = torch.zeros((17, 64), dtype=torch.int16)
+    lab = torch.zeros(4, dtype=torch.int32)
+    sc = torch.zeros(4, dtype=torch.float32)
+    with pytest.raises(ValueError, match="H = 64"):
+        tsd.joint_select_noalloc(A, torch.zeros((17, 128), dtype=torch.int16), None, lab, sc)
+    with pytest.raises(ValueError, match="bias"):
+        tsd.joint_select_noalloc(A, Wt, torch.zeros((4, 15), dtype=torch.float32), lab, sc)
+    with pytest.raises(ValueError, match="out_label"):
+        tsd.joint_select_noalloc(A, Wt, None, torch.zeros(3, dtype=torch.int32), sc)
+    with pytest.raises(ValueError, match="A must be bf16"):
+        tsd.joint_select_noalloc(A.float(), Wt, None, lab, sc)
+    with pytest.raises(ValueError, match="CUDA tensor"):
+        tsd.joint_select_noalloc(A, Wt, None, lab, sc)
+    with pytest.raises(TypeError):
+        tsd.joint_select_noalloc(np.zeros((4, 64)), Wt, None, lab, sc)

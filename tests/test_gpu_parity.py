@@ -99,16 +99,43 @@ def test_cfg2_sampled_parity_full_size():
     assert any(run.states[c][i][1] != 0 for c in range(w.chunks) for i in range(w.B))
 
 
-def test_cfg4_sampled_parity_full_size():
+def test_cfg4_full_size_parity():
     """The stress configuration at full size: V+1 = 4097, 1024 streams, a
-    10-gram LM with ~100M n-grams, 50,000 phrases; 3 streams replayed over all
-    20 chunks."""
+    10-gram LM with ~100M n-grams, 50,000 phrases.  Every one of the 1024
+    streams is replayed by the oracle over chunk 0 (LM and trie states of all
+    streams compared), 64 streams over all 20 chunks; the last chunk's first
+    label steps are captured and the joint logits of 32 rows compared label
+    by label with the oracle's product."""
     w = synth.WORKLOADS[4]
     inp = pu.Inputs(w)
-    run = pu.GpuRun(inp, range(w.B), w.chunks)
-    reps = pu.replay(inp, run, [0, 511, 1023])
-    pu.assert_reports(reps)
+    run = pu.GpuRun(inp, range(w.B), w.chunks, capture_steps=3)
+    models = pu.oracle_models(inp)
+    long_sample = list(range(0, w.B, 16))
+    pu.assert_reports(pu.replay(inp, run, long_sample, models=models))
+    rest = [i for i in range(w.B) if i % 16]
+    pu.assert_reports(pu.replay(inp, run, rest, chunks=1, models=models))
     assert max(len(run.lm.state_tuple(run.states[-1][i][0])) for i in range(w.B)) >= 3
+    err, n = pu.captured_logit_error(run, models[2], 3, list(range(0, w.B, 32)))
+    assert n >= 32 and err < pu.LOGIT_TOL, (err, n)
+
+
+@pytest.mark.parametrize("shape", ["cfg2", "cfg4"])
+@pytest.mark.parametrize("bn", [64, 128, 256])
+def test_joint_logits_elementwise(shape, bn):
+    """Joint logits label by label against the oracle's double product of the
+    same bf16 inputs, at the 0.6B-sized joint (H = 1024, V+1 = 1025) and the
+    stress vocabulary (V+1 = 4097), for every tensor-core tile width: 200
+    streams (the second 128-row tile is partial), every label including the
+    last partial label tile and blank, the first 4 label steps of 2 chunks."""
+    base = synth.WORKLOADS[2] if shape == "cfg2" else synth.WORKLOADS[4]
+    w = synth.scaled(base, B=200, chunks=2, lm_order=4, lm_total=150_000, n_phr=400)
+    inp = pu.Inputs(w)
+    run = pu.GpuRun(inp, range(w.B), 2, capture_steps=4, options={"joint_bn": bn})
+    models = pu.oracle_models(inp)
+    err, n = pu.captured_logit_error(run, models[2], 4, range(w.B))
+    assert n >= 4 * 190 and err < pu.LOGIT_TOL, (err, n)
+    pu.assert_reports(pu.replay(inp, run, [0, 127, 128, 199], models=models))
+    print(f"{shape} bn={bn}: max |logit - oracle| = {err:.2e} over {n} rows")
 
 
 def test_cfg3_beam_parity():

@@ -1,12 +1,16 @@
 """Stream state export and import: a stream exported after one chunk and
 imported into another decoder (other slot ids) continues exactly as it
-would have in the first."""
+would have in the first, and the oracle, following the first decoder's
+chunk and then the second's, finds every decision, fused score and state
+of the migrated stream correct."""
 from __future__ import annotations
 
 import numpy as np
 import pytest
 
+import oracle
 import synth
+from tests import parity_util as pu
 
 pytestmark = pytest.mark.gpu
 
@@ -48,12 +52,34 @@ def test_greedy_stream_moves_between_decoders(n_lm):
     sa = [a.open() for _ in range(w.B)]
     _ = [b.open() for _ in range(w.B)]  # occupy other slot ids first
     sb = [b.open() for _ in range(w.B)]
-    _chunk(a, sa, w, 0)
+    first = _chunk(a, sa, w, 0)
     for x, y in zip(sa, sb):
         b.import_state(y, a.export_state(x))
-    assert _chunk(a, sa, w, 1) == _chunk(b, sb, w, 1)
+    second = _chunk(b, sb, w, 1)
+    assert _chunk(a, sa, w, 1) == second
     for x, y in zip(sa, sb):
         assert a.state(x) == b.state(y)
+    # the oracle follows chunk 0 as decoded by a, then chunk 1 as decoded by b
+    olms = [(oracle.LM.from_arrays(x), wt) for x, wt in lms]
+    obo = oracle.Boost.from_phrases(w.V, ph, w.bonus)
+    model = oracle.Model(w.V, w.H, E, W)
+    gl = b.lm if isinstance(b.lm, list) else [b.lm]
+    for i in range(w.B):
+        st = oracle.Stream(w.V)
+        for c, res in ((0, first), (1, second)):
+            tok, fr, sc = res[i]
+            _, _, _, rep = oracle.decode_chunk(st, model, olms if n_lm > 1 else olms[0][0], obo,
+                                               synth.enc_chunk(w, [i], c)[0], w.lam, w.beta, w.max_sym,
+                                               follow=(tok, fr, sc), gap_tol=pu.GAP_TOL)
+            assert rep[oracle.REP_INCONSISTENT] == 0 and rep[oracle.REP_MISMATCH] == 0, (i, c, rep)
+            assert rep[oracle.REP_MAX_SCORE_DIFF] <= pu.SCORE_TOL, (i, c, rep)
+        hist = st.history()
+        lm_state, node, last = b.state(sb[i])
+        assert last == (hist[-1] if hist else w.V)
+        for m, g in enumerate(gl):
+            got = b.lm_state(sb[i], m) if n_lm > 1 else lm_state
+            assert g.state_tuple(got) == olms[m][0].state(hist), (i, m)
+        assert b.boost.node_tuple(node) == pu.trie_tuple(obo, hist, st.rho()), i
 
 
 def test_beam_stream_moves_between_decoders():
@@ -65,13 +91,42 @@ def test_beam_stream_moves_between_decoders():
     sa = [a.open() for _ in range(w.B)]
     _ = [b.open() for _ in range(2)]
     sb = [b.open() for _ in range(w.B)]
+    import torch
+
+    caps = []
+    for d in (a, b):
+        rows = torch.full((w.T, w.B * 3, 4), -7, dtype=torch.int32, device="cuda")
+        logits = torch.zeros((w.T, w.B * 3, w.N), dtype=torch.float32, device="cuda")
+        d.debug_capture(logits, rows, w.T)
+        caps.append(rows)
     _chunk(a, sa, w, 0)
+    sel0 = caps[0].cpu().numpy().copy()
     for x, y in zip(sa, sb):
         b.import_state(y, a.export_state(x))
     _chunk(a, sa, w, 1)
     _chunk(b, sb, w, 1)
+    sel1 = caps[1].cpu().numpy().copy()
     for x, y in zip(sa, sb):
         assert a.hyps(x) == b.hyps(y)
+    # the oracle follows a's kept candidates over chunk 0 and b's over chunk 1
+    olm = oracle.LM.from_arrays(lms[0][0])
+    obo = oracle.Boost.from_phrases(w.V, ph, w.bonus)
+    model = oracle.Model(w.V, w.H, E, W)
+    K = 3
+    for i in range(w.B):
+        st = oracle.Stream(w.V)
+        for c, sel in ((0, sel0), (1, sel1)):
+            s_i = sel[:, i * K:(i + 1) * K, :]
+            rep = oracle.beam_chunk_follow(st, model, olm, obo, synth.enc_chunk(w, [i], c)[0], w.lam, w.beta, K,
+                                           s_i[:, :, 0], s_i[:, :, 1], s_i[:, :, 2].view(np.float32), pu.GAP_TOL,
+                                           S=w.max_sym)
+            assert rep[oracle.REP_INCONSISTENT] == 0 and rep[oracle.REP_MISMATCH] == 0, (i, c, rep)
+            assert rep[oracle.REP_MAX_SCORE_DIFF] <= pu.SCORE_TOL, (i, c, rep)
+        want = st.beam_hyps()
+        got = b.hyps(sb[i])
+        assert [g[0] for g in got] == [h[0] for h in want], i
+        for (_, gs), h in zip(got, want):
+            assert abs(gs - h[1]) <= pu.SCORE_TOL * 2 * w.T, i
 
 
 def test_import_rejects_mismatched_or_damaged_blobs():

@@ -9,7 +9,9 @@ The check: one label step from the start of a stream, computed two ways --
 by the ordinary decoder (tsd_decode_chunk with one frame and one symbol per
 frame, fresh streams) and by two consecutive calls of the allocation-free
 entry point on the same joint input, weights and fusion bias -- must agree
-within the tolerances of the parity tests.  This file is collected last.
+within the tolerances of the parity tests; the selection is also checked
+against the oracle's fused row for a fresh stream.  This file is collected
+last.
 """
 import numpy as np
 import pytest
@@ -81,6 +83,25 @@ def test_noalloc_selection_matches_decoder_two_calls():
             first = (lab, score)
         else:
             assert np.array_equal(first[0], lab) and np.array_equal(first[1], score)
+
+    # and against the oracle: the fused row of a fresh stream (empty history,
+    # previous label = blank) in double precision, for a sample of rows
+    import oracle
+
+    olm = oracle.LM.from_arrays(lmA)
+    obo = oracle.Boost.from_phrases(w.V, ph, w.bonus)
+    model = oracle.Model(w.V, w.H, E, W)
+    lab, score = first
+    checked = 0
+    for r in range(0, w.B, 7):
+        f = oracle.fused_row(oracle.Stream(w.V), model, olm, obo, enc[r, 0], w.lam, w.beta)
+        best = int(np.argmax(f))
+        top2 = np.sort(f)[-2:]
+        if top2[1] - top2[0] > pu.GAP_TOL:
+            assert lab[r] == best, r
+            checked += 1
+        assert abs(float(score[r]) - f[lab[r]]) <= pu.SCORE_TOL, r
+    assert checked > 20
 
 
 def test_noalloc_rejects_sizes_beyond_its_array():
