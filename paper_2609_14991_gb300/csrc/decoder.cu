@@ -70,6 +70,7 @@ void enqueue_chunk(tsd_decoder* d, int M, int T, cudaStream_t s, const std::vect
     mark(0);
     if (d->cfg.beam_k > 1) launch_row_beam(v, M / d->cfg.beam_k, step, step == S ? 1 : 0, d->row_smem, s, pdl);
     else if (d->cfg.prune_k > 0) launch_row_pruned(v, M, step, step == S ? 1 : 0, s, pdl);
+    else if (v.fused) launch_row_fused(v, M, step, step == S ? 1 : 0, d->row_smem, s, pdl);
     else launch_row(v, M, step, step == S ? 1 : 0, d->row_smem, s, pdl);
     if (pr.D) {
       // the prediction network reads the labels just emitted; after the last
@@ -173,7 +174,10 @@ tsd_status create_impl(const tsd_decoder_cfg* cfg, const void* W_out_bf16, const
   d->M_pad = round_up(d->M_max, kMPad);
   d->n_ptiles = d->N_pad / kPartialCols;
   d->V4 = round_up(c.V, 16);
-  d->row_smem = row_smem_bytes(d->V4, n_lms);
+  // greedy decoding with at most one LM: the joint kernel writes logits and
+  // the row pass fuses; several LMs and beam search keep the dense bias row
+  const bool fused = c.beam_k == 1 && c.prune_k == 0 && n_lms <= 1;
+  d->row_smem = fused ? row_fused_smem_bytes(d->V4) : row_smem_bytes(d->V4, n_lms);
   if (d->row_smem > 200 * 1024) return fail(TSD_EINVAL, "tsd_decoder_create: V too large for the row pass");
 
   DevArena& A = d->arena;
@@ -206,6 +210,15 @@ tsd_status create_impl(const tsd_decoder_cfg* cfg, const void* W_out_bf16, const
     A.release();
     return st;
   }
+  if (fused) {
+    if ((st = A.alloc(&v.logits, (size_t)d->M_pad * d->N_pad)) || (st = A.alloc(&v.dvec, (size_t)d->N_pad))) {
+      A.release();
+      return st;
+    }
+    TSD_CUDA(cudaMemsetAsync(v.dvec, 0, sizeof(float) * (size_t)d->N_pad, s));
+    TSD_CUDA(cudaMemsetAsync(v.logits, 0, sizeof(float) * (size_t)d->M_pad * d->N_pad, s));
+  }
+  v.fused = fused ? 1 : 0;
   const int topk = c.beam_k > 1 ? c.beam_k : c.prune_k;
   if (c.beam_k == 1 && c.prune_k > 0) {
     if ((st = A.alloc(&bpart, (size_t)d->M_pad * (d->N_pad / 64) * (1 + topk)))) {
@@ -307,7 +320,10 @@ tsd_status create_impl(const tsd_decoder_cfg* cfg, const void* W_out_bf16, const
       return cleanup(fail(TSD_ECUDA, "tsd_decoder_create_pred: TMA descriptors"));
     if ((ce = gemm_tc_prepare()) != cudaSuccess) return cleanup(cuda_fail(ce, "tsd_decoder_create_pred: kernel attributes"));
   }
-  if ((ce = prepare_kernels(d->row_smem)) != cudaSuccess) return cleanup(cuda_fail(ce, "tsd_decoder_create: kernel attributes"));
+  if ((ce = prepare_kernels(row_smem_bytes(d->V4, n_lms))) != cudaSuccess)
+    return cleanup(cuda_fail(ce, "tsd_decoder_create: kernel attributes"));
+  if (fused && (ce = prepare_fused_kernels(d->row_smem)) != cudaSuccess)
+    return cleanup(cuda_fail(ce, "tsd_decoder_create: kernel attributes"));
   if ((ce = prepare_beam_kernels(d->row_smem)) != cudaSuccess) return cleanup(cuda_fail(ce, "tsd_decoder_create: kernel attributes"));
   if (hlive && (ce = cudaMemsetAsync(hlive, 0, sizeof(int32_t) * SK, s)) != cudaSuccess)
     return cleanup(cuda_fail(ce, "tsd_decoder_create: initial copies"));
@@ -320,7 +336,7 @@ tsd_status create_impl(const tsd_decoder_cfg* cfg, const void* W_out_bf16, const
     d->sms = sms;
     d->view.sms = sms;
     const int bn = joint_tc_pick_bn(d->M_max, d->N_pad, sms);
-    if ((ce = joint_tc_prepare(d->jtc, Abuf, d->M_pad, Wt, d->N_pad, c.H, bn, bias)) != cudaSuccess)
+    if ((ce = joint_tc_prepare(d->jtc, Abuf, d->M_pad, Wt, d->N_pad, c.H, bn, bias, v.logits)) != cudaSuccess)
       return cleanup(cuda_fail(ce, "tsd_decoder_create: tensor-core GEMM setup (TMA descriptors)"));
   }
   for (int i = 0; i < tsd_decoder::kRing; ++i) {
@@ -981,7 +997,7 @@ extern "C" tsd_status tsd_decoder_set_option(tsd_decoder* d, const char* name, i
     tsd_status st = drop_graphs(d);
     if (st) return st;
     cudaError_t ce = joint_tc_prepare(d->jtc, d->view.A, d->M_pad, d->view.Wt, d->N_pad, d->cfg.H, (int)value,
-                                      d->view.bias);
+                                      d->view.bias, d->view.logits);
     if (ce != cudaSuccess) return cuda_fail(ce, "tsd_decoder_set_option: joint_bn");
     if (d->joint_kind == 0) {
       d->n_ptiles = d->N_pad / d->jtc->bn;
@@ -1008,6 +1024,7 @@ extern "C" tsd_status tsd_decoder_replay(tsd_decoder* d, int32_t kernel, int32_t
   for (int i = 0; i < reps; ++i) {
     if (kernel == 0 && d->cfg.beam_k > 1) launch_row_beam(d->view, d->last_n, S - 1, 2, d->row_smem, s, false);
     else if (kernel == 0 && d->cfg.prune_k > 0) launch_row_pruned(d->view, M, S - 1, 2, s, false);
+    else if (kernel == 0 && d->view.fused) launch_row_fused(d->view, M, S - 1, 2, d->row_smem, s, false);
     else if (kernel == 0) launch_row(d->view, M, S - 1, 2, d->row_smem, s, false);
     else if (d->joint_kind == 0) launch_joint_tc(*d->jtc, d->view, M, 1 << 30, s, false);
     else launch_joint(d->view, M, 1 << 30, s);
@@ -1021,6 +1038,11 @@ extern "C" tsd_status tsd_decoder_replay(tsd_decoder* d, int32_t kernel, int32_t
       // per launch, plus the dense unigram and root rows every launch reads once
       const int64_t shared = (int64_t)d->cfg.V * ((d->lm ? 4 : 0) + (d->boost ? 4 : 0));
       *algo_bytes = (int64_t)(b / (unsigned long long)reps) + shared;
+    } else if (d->view.fused) {
+      // joint, logits out: the operands once (A rows, W_out), the logits
+      // and the softmax partials written
+      *algo_bytes = (int64_t)M * d->cfg.H * 2 + (int64_t)d->N * d->cfg.H * 2 + (int64_t)M * d->N * 4 +
+                    (int64_t)M * d->n_ptiles * 8;
     } else {
       // joint: the operands once (A rows, W_out) and the bias rows read by the epilogue
       *algo_bytes = (int64_t)M * d->cfg.H * 2 + (int64_t)d->N * d->cfg.H * 2 + (int64_t)M * d->N * 4 +

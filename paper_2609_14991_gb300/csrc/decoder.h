@@ -94,6 +94,14 @@ struct DecView {
   float lm_w[kMaxLm]; // relative weights: LM i enters Eq. 1 with lambda * lm_w[i]
   float* dflt;        // [V4] per-call LM bias default lambda*log p(v) (0 past V)
   uint32_t* droot;    // [ceil(V4/32)] bit v: the trie root has a child labelled v
+  // Greedy decoding with at most one LM (fused = 1): the joint kernel
+  // writes logit + dvec and the per-tile softmax partials of the logits, and
+  // the row pass after it finishes Eq. 1 (its per-row LM and trie terms
+  // computed in shared memory before it waits for the joint kernel) and
+  // takes the argmax; no bias row.
+  int32_t fused;
+  float* logits;        // [M_pad][N_pad] fp32 joint logits of the current step, plus dvec
+  float* dvec;          // [N_pad] per call: lambda*log p(v) + beta*bonus*[the root has a child v]; 0 from V on
   int32_t* err;  // device status word: nonzero after a bounded wait expired
   unsigned long long* ctr;  // algorithmic bytes counted by row passes (replayed or timed)
   int32_t count;            // 1: every row pass adds its algorithmic bytes to *ctr
@@ -107,9 +115,12 @@ void launch_fix_records(const DecView& d, int slot, cudaStream_t s);
 void launch_open_pred(const DecView& d, int slot, cudaStream_t s);
 void launch_copy_enc(const DecView& d, int64_t elems, cudaStream_t s, bool pdl);
 void launch_row(const DecView& d, int M, int step, int mode, size_t smem, cudaStream_t s, bool pdl);
+void launch_row_fused(const DecView& d, int M, int step, int mode, size_t smem, cudaStream_t s, bool pdl);
+cudaError_t prepare_fused_kernels(size_t smem);
 void launch_joint(const DecView& d, int M, int step, cudaStream_t s);
 void launch_defaults(const DecView& d, cudaStream_t s);
 size_t row_smem_bytes(int V4, int n_lm);
+size_t row_fused_smem_bytes(int V4);
 cudaError_t prepare_kernels(size_t row_smem);
 void launch_row_beam(const DecView& d, int n, int step, int mode, size_t smem, cudaStream_t s, bool pdl);
 void launch_row_pruned(const DecView& d, int M, int step, int mode, cudaStream_t s, bool pdl);

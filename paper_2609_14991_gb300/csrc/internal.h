@@ -81,6 +81,18 @@ struct LmView {
   const int32_t* arc_tgt = nullptr;   // [A] state of (state . label), -1 at the top order
   const float* uni_logp = nullptr;    // [V] log p(v)
   const int32_t* uni_tgt = nullptr;   // [V] state of the unigram v (0 if order == 1)
+  // target records, so that finding a label's arc also yields the next
+  // state's table record in the same load: (state, first arc, arcs,
+  // cumulative backoff bits), state -1 at the top order
+  const int4* arc_rec = nullptr;      // [A] record of arc_tgt
+  // [V] the unigram state of v: (its dense row or -1, first arc, arcs,
+  // cumulative backoff bits); the state id itself is 1 + v
+  const int4* uni_rec = nullptr;
+  // Unigram states with many continuations (at least V/8) also have a dense
+  // row: per label log p(v | u) - log p(v), NaN where u has no arc v.
+  const float* dense0 = nullptr;      // [rows][V4]
+  const int32_t* uni_dense = nullptr; // [V] dense row of the unigram state of v, or -1
+  int32_t V4 = 0;                     // row stride of dense0
 };
 
 // Device view of the phrase trie.  Node 0 is the root.
@@ -96,6 +108,10 @@ struct TrieView {
   const int32_t* ch_next = nullptr;     // [C] node after the label: child, or 0 if it ends a phrase
   const int32_t* root_child = nullptr;  // [V] child of the root by label (0 = none)
   const int32_t* root_next = nullptr;   // [V] node after the label from the root
+  // child records: (child node, node after the label, child's first child,
+  // child's children); a root entry with child 0 means no child
+  const int4* ch_rec = nullptr;         // [C]
+  const int4* root_rec = nullptr;       // [V]
 };
 
 }  // namespace tsd

@@ -4,7 +4,9 @@
 // the joint network's output projection), then per row and 128-label tile:
 // the softmax partial (max logit, sum exp(logit - max)) over the V+1 real
 // labels and the best fused value logit + bias (bias = lambda*LM +
-// beta*boost, 0 for blank), ties to the lowest label.  Logits stay on chip.
+// beta*boost, 0 for blank), ties to the lowest label.  With DecView::fused
+// the row's logits plus the call's defaults are written out instead and the
+// row pass fuses.
 // This is the simple reference-grade kernel for small row counts; the
 // tensor-core kernel in joint_tc.cu does the same contraction with tcgen05.
 #include "decoder.h"
@@ -101,7 +103,7 @@ __global__ void __launch_bounds__(256) k_joint_simt(DecView d, int step) {
       l[q] = tile[row * (kJN + 4) + c];
       if (gc < N) {
         mx = fmaxf(mx, l[q]);
-        float f = l[q] + (gc < V ? brow[gc] : 0.f);
+        float f = l[q] + (gc < V && !d.fused ? brow[gc] : 0.f);
         if (f > bv) { bv = f; bi = gc; }
       }
     }
@@ -122,6 +124,13 @@ __global__ void __launch_bounds__(256) k_joint_simt(DecView d, int step) {
     for (int o = 16; o > 0; o >>= 1) se += __shfl_xor_sync(0xffffffffu, se, o);
     if (lane == 0)
       d.part[(size_t)gr * d.n_ptiles + blockIdx.x] = make_float4(mx, se, bv, __int_as_float(bi));
+    if (d.fused) {  // the row pass applies Eq. 1 to the logits
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const int gc = n0 + lane * 4 + q;
+        d.logits[(size_t)gr * d.N_pad + gc] = l[q] + __ldcg(d.dvec + gc);
+      }
+    }
     if (d.cap_logits && step < d.cap_steps) {
 #pragma unroll
       for (int q = 0; q < 4; ++q) {

@@ -30,35 +30,45 @@ using namespace tc;  // kBM, kBK and the tcgen05 / TMA helpers
 constexpr int kThreads = 320;
 constexpr int kEpiThreads = 256;  // warps 2-9
 constexpr float kNegInf = -__builtin_huge_valf();
-// Shared memory: [operand stages][bias boxes][barriers].  The fusion bias of
-// the tile (128 rows x BN fp32) arrives by TMA in 128 x 32 boxes with the
-// 128-byte swizzle while the mainloop runs; at BN = 256 only the first half
-// has its own buffer and the second half lands in the drained stages.
-template <int BN>
+// Shared memory: [operand stages][bias boxes][barriers].  With a fusion
+// bias (several LMs), the bias of the tile (128 rows x BN fp32) arrives by
+// TMA in 128 x 32 boxes with the 128-byte swizzle while the mainloop runs;
+// at BN = 256 only the first half has its own buffer and the second half
+// lands in the drained stages.  LOGITS (greedy decoding with at most one
+// LM) takes no bias: the fusion is applied by the row pass after it.
+constexpr int kStageOff = 16384;  // logits staging buffers: past the halves' exchange, in the drained stages
+template <int BN, bool LOGITS = false>
 struct Smem {
   static constexpr int kStages = (BN == 256) ? 3 : (BN == 128 ? 4 : 8);
   static constexpr int kABytes = kBM * kBK * 2;
   static constexpr int kBBytes = BN * kBK * 2;
   static constexpr int kStageBytes = kABytes + kBBytes;
   static constexpr int kBoxBytes = kBM * 32 * 4;
-  static constexpr int kBoxes = BN / 32;
-  static constexpr int kEarly = (BN == 256) ? 4 : kBoxes;
-  static constexpr int kBiasBytes = kEarly * kBoxBytes;
+  static constexpr int kBoxes = LOGITS ? 0 : BN / 32;
+  static constexpr int kEarly = LOGITS ? 0 : ((BN == 256) ? 4 : kBoxes);
+  static constexpr int kBiasBytes = kEarly * kBoxBytes + (LOGITS ? BN * 4 : 0);  // LOGITS: the tile's defaults D
   static constexpr int kBytes = kStages * kStageBytes + kBiasBytes + 1024 /*align*/ + 256 /*barriers*/;
   static_assert((kBoxes - kEarly) * kBoxBytes <= kStages * kStageBytes, "late bias boxes fit the stages");
   // the epilogue halves' exchange (per row 18 floats, 4 flags) after the late boxes
   static_assert((kBoxes - kEarly) * kBoxBytes + kBM * 18 * 4 + 16 <= kStages * kStageBytes, "exchange fits");
+  static_assert(!LOGITS || (kBM * 18 * 4 + 16 <= kStageOff && kStageOff + 8 * 8192 <= kStages * kStageBytes),
+                "logits staging fits the drained stages");
 };
 
 // BEAM: instead of the single best fused label, each row keeps the top-K
 // (K = d.topk <= 8: the beam width, or the pruned-fusion candidate count)
 // values of the tile, ties to the lower label.  With pruned fusion (d.prune)
 // the values are the plain logits: no bias tile is loaded.
-template <int BN, bool BEAM>
+// LOGITS: no bias and no selection here: the epilogue writes the tile's
+// logits plus the call's shared defaults D[v] (d.dvec; fp32, row-major
+// [M_pad][N_pad], d.logits) and the per-row softmax partial (max, sum exp)
+// of the logits; the row pass finishes Eq. 1 and picks.
+template <int BN, bool BEAM, bool LOGITS>
 __global__ void __launch_bounds__(kThreads, 1)
     k_joint_tc(DecView d, int step, const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-               const __grid_constant__ CUtensorMap tmBias) {
-  using S = Smem<BN>;
+               const __grid_constant__ CUtensorMap tmBias, const __grid_constant__ CUtensorMap tmLogits) {
+  using S = Smem<BN, LOGITS>;
+  static_assert(!(LOGITS && BEAM), "the logits output serves greedy decoding");
   extern __shared__ __align__(1024) unsigned char smem_raw[];
   unsigned char* smem = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   unsigned char* bias_early = smem + S::kStages * S::kStageBytes;
@@ -70,7 +80,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int n0 = blockIdx.x * BN, m0 = blockIdx.y * kBM;
-  const bool use_bias = !(BEAM && d.prune);
+  const bool use_bias = !LOGITS && !(BEAM && d.prune);
   const int M = d.params->n * d.K;
   const int KB = d.H / kBK;
 
@@ -180,6 +190,12 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
     for (int j = 0; j < 8; ++j) { tv[j] = kNegInf; ti[j] = INT_MAX; }
     float tmin = kNegInf;  // tv[K-1]
+    float* sD = reinterpret_cast<float*>(bias_early);  // LOGITS: the tile's defaults D (kEarly is 0)
+    if (LOGITS) {
+      // while the MMAs run: the call's defaults of the tile's labels
+      for (int i = (int)threadIdx.x - 64; i < BN; i += kEpiThreads) sD[i] = __ldcg(d.dvec + n0 + i);
+      asm volatile("bar.sync 2, %0;" ::"n"(kEpiThreads) : "memory");
+    }
     ok = __all_sync(0xffffffffu, mbar_wait(accum, 0));  // warp-uniform: tcgen05.ld is .sync.aligned
     if (!ok && lane == 0) atomicOr(d.err, 4);
     fence_after();
@@ -209,6 +225,66 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (lane == 0) atomicOr(d.err, 32);
             break;
           }
+        }
+        if constexpr (LOGITS) {
+          // the chunk's 32 logits of this row: the softmax partial, then the
+          // warp's 32 x 32 block goes out by one TMA store from a staging
+          // buffer in the drained stages (two per warp, alternating; the
+          // 128-byte swizzle keeps the row-per-thread writes conflict-free)
+          float l[32];
+          tmem_ld32(tbase + (uint32_t)(c * 32), l);
+          const int c0 = n0 + c * 32;
+          if (c0 + 32 > N) {
+#pragma unroll
+            for (int i = 0; i < 32; ++i)
+              if (c0 + i >= N) l[i] = kNegInf;
+          }
+          float t[16];
+#pragma unroll
+          for (int i = 0; i < 16; ++i) t[i] = fmaxf(l[i], l[i + 16]);
+#pragma unroll
+          for (int w = 8; w > 0; w >>= 1)
+#pragma unroll
+            for (int i = 0; i < w; ++i) t[i] = fmaxf(t[i], t[i + w]);
+          const float cm = t[0];
+          if (cm != kNegInf) {
+            const float m2 = fmaxf(mx, cm);
+            const float s2 = m2 * kLog2e;
+            float acc = (mx == kNegInf) ? 0.f : se * ex2_approx(mx * kLog2e - s2);
+#pragma unroll
+            for (int i = 0; i < 32; ++i) acc += ex2_approx(fmaf(l[i], kLog2e, -s2));
+            se = acc;
+            mx = m2;
+          }
+          if (d.cap_logits && step < d.cap_steps && live) {
+            float* cl = d.cap_logits + ((size_t)step * M + gr) * N;
+#pragma unroll
+            for (int i = 0; i < 32; ++i)
+              if (c0 + i < N) cl[c0 + i] = l[i];
+          }
+          {
+            // out go logit + D (the call's defaults, the same for every row)
+            const float4* dv4 = reinterpret_cast<const float4*>(sD + 32 * c);
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+              const float4 dq = dv4[j];
+              l[4 * j] += dq.x; l[4 * j + 1] += dq.y; l[4 * j + 2] += dq.z; l[4 * j + 3] += dq.w;
+            }
+            unsigned char* stg = smem + kStageOff + (warp - 2) * 8192 + ((c >> 1) & 1) * 4096;
+            if (lane == 0) tma_store_wait_read1();  // this buffer's store of two chunks ago has read it
+            __syncwarp();
+#pragma unroll
+            for (int j = 0; j < 8; ++j)
+              *reinterpret_cast<float4*>(stg + lane * 128 + ((j ^ (lane & 7)) << 4)) =
+                  make_float4(l[4 * j], l[4 * j + 1], l[4 * j + 2], l[4 * j + 3]);
+            fence_async_smem();
+            __syncwarp();
+            if (lane == 0) {
+              tma_store_2d(&tmLogits, stg, c0, m0 + q * 32);
+              tma_store_commit();
+            }
+          }
+          continue;
         }
         const unsigned char* box = (c < S::kEarly) ? bias_early + c * S::kBoxBytes : smem + (c - S::kEarly) * S::kBoxBytes;
         float b[32];
@@ -309,8 +385,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
     }
-    // never leave with bias boxes still landing in shared memory
+    // never leave with bias boxes still landing in shared memory, nor with
+    // logits stores still reading the staging buffers
     if (!late_done && warp == 2 && lane == 0) mbar_wait(biasbar + 1, 0);
+    if (LOGITS && lane == 0) tma_store_wait_all();
+    __syncwarp();
     // Merge the two halves' partials of each row: the second half leaves its
     // partial in shared memory past the late bias boxes (the stages are
     // drained: every MMA has completed), the first half combines and stores.
@@ -342,7 +421,9 @@ __global__ void __launch_bounds__(kThreads, 1)
           mx = m2;
         }
       }
-      if (!BEAM) {
+      if (LOGITS) {
+        d.part[(size_t)gr * d.n_ptiles + blockIdx.x] = make_float4(mx, se, 0.f, 0.f);
+      } else if (!BEAM) {
         const float v1 = xch[2];
         const int i1 = __float_as_int(xch[3]);
         if (v1 > bv || (v1 == bv && i1 < bi)) { bv = v1; bi = i1; }
@@ -396,28 +477,48 @@ int joint_tc_pick_bn(int M_max, int N_pad, int sms) {
 }
 
 cudaError_t joint_tc_prepare(JointTc* jt, const uint16_t* A, int M_pad, const uint16_t* Wt, int N_pad, int H, int bn,
-                             const float* bias) {
+                             const float* bias, const float* logits) {
   jt->bn = bn;
   if (!make_map(&jt->mapA, A, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, H, M_pad, kBK, kBM)) return cudaErrorInvalidValue;
   if (!make_map(&jt->mapB, Wt, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, H, N_pad, kBK, bn)) return cudaErrorInvalidValue;
   if (!make_map(&jt->mapBias, bias, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, N_pad, M_pad, 32, kBM))
     return cudaErrorInvalidValue;
+  if (!make_map(&jt->mapLogits, logits ? logits : bias, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, N_pad, M_pad, 32, 32))
+    return cudaErrorInvalidValue;
+  const auto attr = cudaFuncAttributeMaxDynamicSharedMemorySize;
   cudaError_t e = cudaSuccess;
   if (bn == 256) {
-    e = cudaFuncSetAttribute(k_joint_tc<256, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, Smem<256>::kBytes);
-    if (e == cudaSuccess)
-      e = cudaFuncSetAttribute(k_joint_tc<256, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, Smem<256>::kBytes);
+    e = cudaFuncSetAttribute(k_joint_tc<256, false, false>, attr, Smem<256>::kBytes);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(k_joint_tc<256, true, false>, attr, Smem<256>::kBytes);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(k_joint_tc<256, false, true>, attr, Smem<256, true>::kBytes);
   } else if (bn == 128) {
-    e = cudaFuncSetAttribute(k_joint_tc<128, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, Smem<128>::kBytes);
-    if (e == cudaSuccess)
-      e = cudaFuncSetAttribute(k_joint_tc<128, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, Smem<128>::kBytes);
+    e = cudaFuncSetAttribute(k_joint_tc<128, false, false>, attr, Smem<128>::kBytes);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(k_joint_tc<128, true, false>, attr, Smem<128>::kBytes);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(k_joint_tc<128, false, true>, attr, Smem<128, true>::kBytes);
   } else {
-    e = cudaFuncSetAttribute(k_joint_tc<64, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, Smem<64>::kBytes);
-    if (e == cudaSuccess)
-      e = cudaFuncSetAttribute(k_joint_tc<64, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, Smem<64>::kBytes);
+    e = cudaFuncSetAttribute(k_joint_tc<64, false, false>, attr, Smem<64>::kBytes);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(k_joint_tc<64, true, false>, attr, Smem<64>::kBytes);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(k_joint_tc<64, false, true>, attr, Smem<64, true>::kBytes);
   }
   return e;
 }
+
+namespace {
+template <int BN>
+void launch_bn(cudaLaunchConfig_t& cfg, const JointTc& jt, const DecView& d, int step) {
+  const bool beam = d.topk > 1 || d.prune > 0;  // the top-K epilogue
+  if (beam) {
+    cfg.dynamicSmemBytes = Smem<BN>::kBytes;
+    cudaLaunchKernelEx(&cfg, k_joint_tc<BN, true, false>, d, step, jt.mapA, jt.mapB, jt.mapBias, jt.mapLogits);
+  } else if (d.fused) {
+    cfg.dynamicSmemBytes = Smem<BN, true>::kBytes;
+    cudaLaunchKernelEx(&cfg, k_joint_tc<BN, false, true>, d, step, jt.mapA, jt.mapB, jt.mapBias, jt.mapLogits);
+  } else {
+    cfg.dynamicSmemBytes = Smem<BN>::kBytes;
+    cudaLaunchKernelEx(&cfg, k_joint_tc<BN, false, false>, d, step, jt.mapA, jt.mapB, jt.mapBias, jt.mapLogits);
+  }
+}
+}  // namespace
 
 void launch_joint_tc(const JointTc& jt, const DecView& d, int M, int step, cudaStream_t s, bool pdl) {
   cudaLaunchConfig_t cfg = {};
@@ -429,20 +530,9 @@ void launch_joint_tc(const JointTc& jt, const DecView& d, int M, int step, cudaS
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = pdl ? 1 : 0;
-  const bool beam = d.topk > 1 || d.prune > 0;  // the top-K epilogue
-  if (jt.bn == 256) {
-    cfg.dynamicSmemBytes = Smem<256>::kBytes;
-    if (beam) cudaLaunchKernelEx(&cfg, k_joint_tc<256, true>, d, step, jt.mapA, jt.mapB, jt.mapBias);
-    else cudaLaunchKernelEx(&cfg, k_joint_tc<256, false>, d, step, jt.mapA, jt.mapB, jt.mapBias);
-  } else if (jt.bn == 128) {
-    cfg.dynamicSmemBytes = Smem<128>::kBytes;
-    if (beam) cudaLaunchKernelEx(&cfg, k_joint_tc<128, true>, d, step, jt.mapA, jt.mapB, jt.mapBias);
-    else cudaLaunchKernelEx(&cfg, k_joint_tc<128, false>, d, step, jt.mapA, jt.mapB, jt.mapBias);
-  } else {
-    cfg.dynamicSmemBytes = Smem<64>::kBytes;
-    if (beam) cudaLaunchKernelEx(&cfg, k_joint_tc<64, true>, d, step, jt.mapA, jt.mapB, jt.mapBias);
-    else cudaLaunchKernelEx(&cfg, k_joint_tc<64, false>, d, step, jt.mapA, jt.mapB, jt.mapBias);
-  }
+  if (jt.bn == 256) launch_bn<256>(cfg, jt, d, step);
+  else if (jt.bn == 128) launch_bn<128>(cfg, jt, d, step);
+  else launch_bn<64>(cfg, jt, d, step);
 }
 
 }  // namespace tsd

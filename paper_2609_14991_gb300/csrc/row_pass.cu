@@ -480,8 +480,10 @@ __global__ void k_fix_records(DecView d, int slot) {
   const int l = threadIdx.x;
   if (d.has_lm && l < kLmChain && l < d.s_lm_len[slot]) {
     const int st = d.s_lm_chain[(size_t)slot * kLmChain + l];
+    // the fourth field of the first (unigram) level: its dense row, if any
+    const int dense = (l == 0 && d.lm.order >= 2 && st >= 1 && st <= d.V) ? d.lm.uni_dense[st - 1] : -1;
     d.s_lm_rec[(size_t)slot * kLmChain + l] =
-        make_int4(d.lm.st_begin[st], d.lm.st_count[st], __float_as_int(d.lm.st_cum[st]), 0);
+        make_int4(d.lm.st_begin[st], d.lm.st_count[st], __float_as_int(d.lm.st_cum[st]), dense);
   }
   if (d.has_tr && l < kTrChain && l < d.s_tr_len[slot]) {
     const int q = d.s_tr_chain[(size_t)slot * kTrChain + l];
@@ -518,6 +520,8 @@ size_t row_smem_bytes(int V4, int n_lm) {
   return (size_t)V4 * ((n_lm > 1 ? 2 : 1) * sizeof(float) + sizeof(uint8_t));
 }
 
+size_t row_fused_smem_bytes(int V4) { return (size_t)V4 * (sizeof(float) + 2 * sizeof(uint8_t)); }
+
 namespace {
 // Per-call defaults of the fusion bias, which the row pass combines with
 // the row's own terms: lambda * log p(v) for every label (0 past V), and a
@@ -528,6 +532,16 @@ __global__ void k_defaults(DecView d) {
   const float lam = P->lambda;
   const int i = blockIdx.x * blockDim.x + threadIdx.x;
   if (i < d.V4) d.dflt[i] = (d.has_lm && i < d.V) ? lam * __ldg(d.lm.uni_logp + i) : 0.f;
+  if (d.fused && i < d.N_pad) {
+    // the defaults the joint kernel adds to its logits (0 from blank on)
+    float x = 0.f;
+    if (i < d.V) {
+      if (d.has_lm) x = lam * __ldg(d.lm.uni_logp + i);
+      if (d.has_tr && __ldg(d.tr.root_child + i) != 0) x += P->beta * d.tr.bonus;
+    }
+    d.dvec[i] = x;
+  }
+
   if (i < (d.V4 + 31) / 32) {
     uint32_t m = 0;
     if (d.has_tr)
@@ -540,7 +554,9 @@ __global__ void k_defaults(DecView d) {
 }
 }  // namespace
 
-void launch_defaults(const DecView& d, cudaStream_t s) { k_defaults<<<(d.V4 + 255) / 256, 256, 0, s>>>(d); }
+void launch_defaults(const DecView& d, cudaStream_t s) {
+  k_defaults<<<(std::max(d.V4, d.N_pad) + 255) / 256, 256, 0, s>>>(d);
+}
 
 cudaError_t prepare_kernels(size_t row_smem) {
   // dynamic scratch plus the kernel's static shared memory may pass the

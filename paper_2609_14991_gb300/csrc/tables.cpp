@@ -252,6 +252,50 @@ extern "C" tsd_status tsd_ngram_build(int32_t V, int32_t order, const int64_t* c
   }
   std::vector<float> st_cum((size_t)S);
   for (int64_t s = 0; s < S; ++s) st_cum[(size_t)s] = (float)cum[(size_t)s];
+  // each arc's target record, and each unigram state's
+  auto rec_of = [&](int64_t s) {
+    int32_t cb;
+    std::memcpy(&cb, &st_cum[(size_t)s], 4);
+    return make_int4((int32_t)s, st_begin[(size_t)s], st_count[(size_t)s], cb);
+  };
+  std::vector<int4> arc_rec((size_t)total_arcs + 1), uni_rec((size_t)V);
+  parallel_for(total_arcs, [&](int64_t b, int64_t e) {
+    for (int64_t a = b; a < e; ++a) {
+      const int32_t t = arc_tgt[(size_t)a];
+      arc_rec[(size_t)a] = t >= 0 ? rec_of(t) : make_int4(-1, 0, 0, 0);
+    }
+  });
+  arc_rec[(size_t)total_arcs] = make_int4(-1, 0, 0, 0);
+  // dense rows for the unigram states with many continuations (at most
+  // 512 MB of them): log p(v | u) - log p(v) per label, NaN for no arc
+  const int64_t V4 = ((int64_t)V + 15) / 16 * 16;
+  std::vector<int32_t> uni_dense((size_t)V, -1);
+  int64_t n_dense = 0;
+  if (order >= 2) {
+    const int64_t thr = std::max<int64_t>(32, V / 8), cap = (512ll << 20) / (4 * V4);
+    for (int64_t u = 0; u < V && n_dense < cap; ++u)
+      if (st_count[(size_t)(base[1] + u)] >= thr) uni_dense[(size_t)u] = (int32_t)n_dense++;
+  }
+  std::vector<float> dense0((size_t)std::max<int64_t>(1, n_dense) * V4, std::nanf(""));
+  parallel_for(order >= 2 ? V : 0, [&](int64_t b, int64_t e) {
+    for (int64_t u = b; u < e; ++u) {
+      const int32_t row = uni_dense[(size_t)u];
+      if (row < 0) continue;
+      const int64_t s = base[1] + u;
+      for (int32_t a = st_begin[(size_t)s]; a < st_begin[(size_t)s] + st_count[(size_t)s]; ++a) {
+        const int32_t t = arc_tok[(size_t)a];
+        dense0[(size_t)row * V4 + t] = (float)((double)arc_logp[(size_t)a] - (double)uni_logp[(size_t)t]);
+      }
+    }
+  });
+  for (int64_t u = 0; u < V; ++u) {
+    if (order >= 2) {
+      uni_rec[(size_t)u] = rec_of(uni_tgt[(size_t)u]);
+      uni_rec[(size_t)u].x = uni_dense[(size_t)u];
+    } else {
+      uni_rec[(size_t)u] = make_int4(-1, 0, 0, 0);
+    }
+  }
 
   LmView& v = lm->view;
   v.V = V;
@@ -260,6 +304,9 @@ extern "C" tsd_status tsd_ngram_build(int32_t V, int32_t order, const int64_t* c
   v.n_arcs = total_arcs;
   int32_t *d_b, *d_c, *d_at, *d_ag, *d_ut;
   float *d_cum, *d_al, *d_ul;
+  int4 *d_ar, *d_ur;
+  float* d_dense;
+  int32_t* d_ud;
   tsd_status st;
   // the row pass reads arcs in aligned groups of four: room for the last group
   arc_tok.resize((size_t)total_arcs + 4, 0);
@@ -267,10 +314,17 @@ extern "C" tsd_status tsd_ngram_build(int32_t V, int32_t order, const int64_t* c
   if ((st = lm->arena.upload(&d_b, st_begin)) || (st = lm->arena.upload(&d_c, st_count)) ||
       (st = lm->arena.upload(&d_cum, st_cum)) || (st = lm->arena.upload(&d_at, arc_tok)) ||
       (st = lm->arena.upload(&d_al, arc_logp)) || (st = lm->arena.upload(&d_ag, arc_tgt)) ||
-      (st = lm->arena.upload(&d_ul, uni_logp)) || (st = lm->arena.upload(&d_ut, uni_tgt))) {
+      (st = lm->arena.upload(&d_ul, uni_logp)) || (st = lm->arena.upload(&d_ut, uni_tgt)) ||
+      (st = lm->arena.upload(&d_ar, arc_rec)) || (st = lm->arena.upload(&d_ur, uni_rec)) ||
+      (st = lm->arena.upload(&d_dense, dense0)) || (st = lm->arena.upload(&d_ud, uni_dense))) {
     lm->arena.release();
     return st;
   }
+  v.arc_rec = d_ar;
+  v.uni_rec = d_ur;
+  v.dense0 = d_dense;
+  v.uni_dense = d_ud;
+  v.V4 = (int32_t)V4;
   v.st_begin = d_b;
   v.st_count = d_c;
   v.st_cum = d_cum;
@@ -405,6 +459,15 @@ extern "C" tsd_status tsd_boost_build(int32_t V, int32_t n_phr, const int32_t* o
   int32_t *a0 = nullptr, *a1 = nullptr, *a2 = nullptr, *a3 = nullptr, *a4 = nullptr, *a5 = nullptr, *a6 = nullptr,
           *a7 = nullptr, *a8 = nullptr;
   tsd_status st;
+  std::vector<int4> ch_rec(ch_tok.size() + 1, make_int4(-1, 0, 0, 0)), root_rec((size_t)V, make_int4(0, 0, 0, 0));
+  for (size_t c = 0; c < ch_tok.size(); ++c) {
+    const int32_t q = ch_node[c];
+    ch_rec[c] = make_int4(q, ch_next[c], nd_begin[(size_t)q], nd_count[(size_t)q]);
+  }
+  for (int32_t u = 0; u < V; ++u) {
+    const int32_t q = root_child[(size_t)u];
+    if (q) root_rec[(size_t)u] = make_int4(q, root_next[(size_t)u], nd_begin[(size_t)q], nd_count[(size_t)q]);
+  }
   ch_tok.resize(ch_tok.size() + 4, 0);  // aligned groups of four in the row pass
   if ((st = b->arena.upload(&a0, nd_begin)) || (st = b->arena.upload(&a1, nd_count)) ||
       (st = b->arena.upload(&a2, depth)) || (st = b->arena.upload(&a3, nd_fail)) ||
@@ -414,6 +477,13 @@ extern "C" tsd_status tsd_boost_build(int32_t V, int32_t n_phr, const int32_t* o
     b->arena.release();
     return st;
   }
+  int4 *r0 = nullptr, *r1 = nullptr;
+  if ((st = b->arena.upload(&r0, ch_rec)) || (st = b->arena.upload(&r1, root_rec))) {
+    b->arena.release();
+    return st;
+  }
+  v.ch_rec = r0;
+  v.root_rec = r1;
   v.nd_begin = a0;
   v.nd_count = a1;
   v.nd_depth = a2;

@@ -130,6 +130,29 @@ class NGramArrays:
 
 
 def ngram_lm(seed: int, V: int, order: int, total: int, zipf_s: float, discount: float = 0.7) -> NGramArrays:
+    """The seeded LM (see _ngram_lm).  If TSD_SYNTH_CACHE names a directory,
+    large models are kept there as .npz files and read back on later calls
+    (the arrays are a pure function of the arguments)."""
+    cache = os.environ.get("TSD_SYNTH_CACHE")
+    if not cache or total < 1_000_000:
+        return _ngram_lm(seed, V, order, total, zipf_s, discount)
+    path = os.path.join(cache, f"lm_{seed}_{V}_{order}_{total}_{zipf_s}_{discount}.npz")
+    if os.path.exists(path):
+        z = np.load(path)
+        return NGramArrays(V, order, [z[f"t{k}"] for k in range(order)], [z[f"l{k}"] for k in range(order)],
+                           [z[f"b{k}"] for k in range(order)], [z[f"c{k}"] for k in range(order)], discount)
+    a = _ngram_lm(seed, V, order, total, zipf_s, discount)
+    os.makedirs(cache, exist_ok=True)
+    tmp = path + f".tmp{os.getpid()}.npz"
+    arrs = {}
+    for k in range(order):
+        arrs.update({f"t{k}": a.tokens[k], f"l{k}": a.logp[k], f"b{k}": a.bow[k], f"c{k}": a.counts[k]})
+    np.savez(tmp, **arrs)
+    os.replace(tmp, path)
+    return a
+
+
+def _ngram_lm(seed: int, V: int, order: int, total: int, zipf_s: float, discount: float = 0.7) -> NGramArrays:
     L = lib()
     h = L.synth_lm_new(seed, V, order, total, zipf_s, discount)
     if not h:
