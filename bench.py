@@ -441,25 +441,28 @@ def run_ours(args, w):
     def timed_loop(first_chunk):
         starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
         ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
-        with Clocks(local) as clk:
-            barrier()
-            t0 = time.perf_counter()
-            for k in range(args.steps):
-                flush.zero_()  # L2 flush, outside the step's events
-                starts[k].record(stream)
-                step(first_chunk + k)
-                ends[k].record(stream)
-            barrier()
-            wall = time.perf_counter() - t0
+        barrier()
+        t0 = time.perf_counter()
+        for k in range(args.steps):
+            flush.zero_()  # L2 flush, outside the step's events
+            starts[k].record(stream)
+            step(first_chunk + k)
+            ends[k].record(stream)
+        barrier()
+        wall = time.perf_counter() - t0
         per = [s.elapsed_time(e) for s, e in zip(starts, ends)]
-        return float(sum(per)), wall, clk, per
+        return float(sum(per)), wall, per
 
+    # clocks and throttle reasons are sampled from here to the end of the GPU
+    # work (the timed steps, their instrumented replay, the end-to-end steps
+    # and the stream sweep), so the sample spans more than the short timed region
+    clk = Clocks(local).__enter__()
     # warm-up (captures the chunk graph)
     for c in range(args.warmup):
         step(c)
     barrier()
     # timed region: K steps through the captured graph, no instrumentation
-    t_ms, wall, clk, step_ms = timed_loop(args.warmup)
+    t_ms, wall, step_ms = timed_loop(args.warmup)
     # the same K steps again with a CUDA event recorded at every kernel
     # boundary inside the graph: per-kernel device time for the roofline
     dec.set_timing(True)
@@ -472,7 +475,7 @@ def run_ours(args, w):
     dec.timed_bytes(reset=True)
     if encoder is not None:
         encoder.timing(reset=True)
-    t_inst_ms, _, _, _ = timed_loop(args.warmup)
+    t_inst_ms, _, _ = timed_loop(args.warmup)
     kernel_ms, kernel_n = dec.timing(reset=True)
     row_timed_bytes = dec.timed_bytes(reset=True)
     dec.set_timing(False)
@@ -555,6 +558,7 @@ def run_ours(args, w):
                       **{k: v for k, v in latency_stats(step_ms).items() if k != "steps"}})
         sweep.sort(key=lambda x: x["B"])
 
+    clk.__exit__(None, None, None)
     if rank != 0:
         return
     pk, pk_kind = peaks()
@@ -615,12 +619,21 @@ def run_ours(args, w):
             (row_roof, share_row, kernel_n["row"] / args.steps,
              row_bytes_graph / max(1, kernel_n["row"]) / 1e9)):
         ms_in_graph = mean_step_ms * share / max(1e-9, n_per_step)
-        roof_k["in_production_graph"] = {
-            "what": "uninstrumented step time x this kernel's share of device time / its launches per step",
-            "avg_launch_ms": ms_in_graph,
-            "achieved": work / (ms_in_graph / 1000.0),
-        }
-        roof_k["in_production_graph"]["frac"] = roof_k["in_production_graph"]["achieved"] / roof_k["peak"]
+        # the headline figures are the production graph's: the timed steps'
+        # CUDA-event time (no instrumentation) apportioned by this kernel's
+        # device-time share; the instrumented pass's own per-launch times stay
+        # beside them (they are upper bounds: events between kernels end the
+        # programmatic overlap and add their own cost)
+        roof_k["serialized_with_kernel_events"] = {
+            "what": "CUDA events at every kernel boundary inside the graph (second pass of the K steps, "
+                    "programmatic launch off): per-launch device time",
+            "avg_launch_ms": roof_k["avg_launch_ms"], "achieved": roof_k["achieved"], "frac": roof_k["frac"]}
+        roof_k["avg_launch_ms"] = ms_in_graph
+        roof_k["achieved"] = work / (ms_in_graph / 1000.0)
+        roof_k["frac"] = roof_k["achieved"] / roof_k["peak"]
+        roof_k["timing"] = ("avg_launch_ms = uninstrumented step time (CUDA events on the launching stream over the "
+                            "K timed steps) x this kernel's share of device time (CUDA events at every kernel "
+                            "boundary over a second pass of the same steps) / its launches per step")
     pred_roof = None
     if args.pred:
         # the stateful form's GEMMs per chunk: the encoder projection, an LSTM
@@ -638,11 +651,13 @@ def run_ours(args, w):
                      "ms_per_chunk": pred_chunk_ms, "launches": kernel_n["pred"],
                      "traffic": None, "share_of_device_time": share_pred}
         pred_roof["frac"] = pred_roof["achieved"] / pred_roof["peak"]
-        pred_roof["in_production_graph"] = {
-            "what": "uninstrumented step time x this class's share of device time",
-            "ms_per_chunk": mean_step_ms * share_pred,
-            "achieved": pred_flop / (mean_step_ms * share_pred / 1000.0) / 1e12}
-        pred_roof["in_production_graph"]["frac"] = pred_roof["in_production_graph"]["achieved"] / pred_roof["peak"]
+        pred_roof["serialized_with_kernel_events"] = {
+            "what": "CUDA events at every kernel boundary inside the graph (second pass, programmatic launch off)",
+            "ms_per_chunk": pred_roof["ms_per_chunk"], "achieved": pred_roof["achieved"], "frac": pred_roof["frac"]}
+        pred_roof["ms_per_chunk"] = mean_step_ms * share_pred
+        pred_roof["achieved"] = pred_flop / (mean_step_ms * share_pred / 1000.0) / 1e12
+        pred_roof["frac"] = pred_roof["achieved"] / pred_roof["peak"]
+        pred_roof["timing"] = "uninstrumented step time x this class's share of device time (CUDA events)"
     enc_roof = None
     if encoder is not None:
         # the encoder's tensor-core GEMMs (subsampling, q/k/v, attention
@@ -666,6 +681,9 @@ def run_ours(args, w):
                         "layer_norm_conv_cache_ms_per_chunk": enc_ms["other"] / args.steps,
                         "layer_norm_conv_cache_share": enc_ms["other"] / total_ms}}
         enc_roof["frac"] = enc_roof["achieved"] / enc_roof["peak"]
+        enc_roof["serialized_with_kernel_events"] = {
+            "what": "CUDA events at every kernel boundary (second pass, one sequence of kernels)",
+            "ms_per_chunk": enc_roof["ms_per_chunk"], "achieved": enc_roof["achieved"], "frac": enc_roof["frac"]}
         enc_roof["in_production_graph"] = {
             "what": "uninstrumented step time x this class's share of device time (the instrumented pass runs "
                     "the encoder's kernels in one sequence; the production graph runs two branches of streams "
@@ -673,6 +691,12 @@ def run_ours(args, w):
             "ms_per_chunk": mean_step_ms * share_enc,
             "achieved": enc_flop / (mean_step_ms * share_enc / 1000.0) / 1e12}
         enc_roof["in_production_graph"]["frac"] = enc_roof["in_production_graph"]["achieved"] / enc_roof["peak"]
+        for k in ("ms_per_chunk", "achieved", "frac"):
+            enc_roof[k] = enc_roof["in_production_graph"][k]
+        del enc_roof["in_production_graph"]
+        enc_roof["timing"] = ("uninstrumented step time x this class's share of device time (CUDA events); the "
+                              "production graph runs two branches of streams whose kernels overlap, so this "
+                              "apportions the overlapped step by the serial shares")
     # the dominant kernel is the one with the largest device time in the graph
     ranked = sorted([(share_joint, joint_roof), (share_row, row_roof)] + ([(share_pred, pred_roof)] if pred_roof else [])
                     + ([(share_enc, enc_roof)] if enc_roof else []), key=lambda x: -x[0])

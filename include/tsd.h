@@ -361,9 +361,22 @@ TSD_API tsd_status tsd_decoder_check(tsd_decoder* dec);
  *              row pass and the joint kernel, so each kernel's set-up
  *              overlaps the tail of the one before;
  *   "joint_bn" 64, 128 or 256: labels per tensor-core CTA tile (default:
- *              chosen at create from the row count and the SM count).
+ *              chosen at create from the row count and the SM count);
+ *   "wait_ns"  0 .. 1e10: the limit, in nanoseconds, of the joint kernel's
+ *              waits for its operands and accumulator (default 1e9).  A wait
+ *              that expires ends the kernel early -- after it has waited,
+ *              with the 1 s limit, for every copy and MMA it started -- and
+ *              the next tsd_decoder_check returns TSD_EDEVICE; that chunk's
+ *              results are then undefined (but every index stays in range).
+ *              A test hook for the failure path.
  * Unknown names return TSD_EINVAL. */
 TSD_API tsd_status tsd_decoder_set_option(tsd_decoder* dec, const char* name, int64_t value);
+
+/* Test hook: the n-th device allocation the library makes from now on
+ * (n >= 1) fails as cudaMalloc would, and the call that makes it returns
+ * TSD_ENOMEM after releasing what it had allocated; n = 0 turns the hook
+ * off.  The hook is process-wide and fires once. */
+TSD_API tsd_status tsd_debug_fail_alloc(int32_t n);
 
 /* Measurement hook: launches one kernel of the last decode_chunk's final
  * label step reps times back to back on cuda_stream -- kernel 0 the row

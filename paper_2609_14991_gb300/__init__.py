@@ -24,7 +24,9 @@ from typing import List, Optional, Sequence, Tuple
 import numpy as np
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
-LIB_PATH = os.path.join(_HERE, "libtsd.so")
+# TSD_LIBRARY selects another build of the library (the range-checked
+# libtsd_checks.so); by default the in-tree libtsd.so
+LIB_PATH = os.environ.get("TSD_LIBRARY") or os.path.join(_HERE, "libtsd.so")
 
 TSD_OK, TSD_EINVAL, TSD_ENOMEM, TSD_ECUDA, TSD_ESTATE, TSD_EDEVICE = 0, -1, -2, -3, -4, -5
 _STATUS = {-1: "EINVAL", -2: "ENOMEM", -3: "ECUDA", -4: "ESTATE", -5: "EDEVICE"}
@@ -101,6 +103,7 @@ SIGNATURES = {
     "tsd_decoder_set_option": ([_vp, ctypes.c_char_p, _i64], _i32),
     "tsd_decoder_replay": ([_vp, _i32, _i32, _vp, _P(_i64)], _i32),
     "tsd_joint_select_noalloc": ([_i32, _i32, _i32, _vp, _vp, _vp, _vp, _vp, _vp], _i32),
+    "tsd_debug_fail_alloc": ([_i32], _i32),
     "tsd_encoder_create": ([_P(EncoderCfgC), _vp, _vp, _vp, _vp, _P(_vp)], _i32),
     "tsd_encoder_free": ([_vp], None),
     "tsd_encoder_open": ([_vp, _P(_i32)], _i32),
@@ -246,6 +249,11 @@ class Boost:
         if getattr(self, "h", None):
             lib().tsd_boost_free(self.h)
             self.h = None
+
+
+def debug_fail_alloc(n: int):
+    """Test hook: the n-th device allocation from now on fails (0: off)."""
+    _check(lib().tsd_debug_fail_alloc(int(n)))
 
 
 def joint_select_noalloc(A, Wt, bias, out_label, out_score, stream=None):

@@ -18,6 +18,10 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD_DIR = os.path.join(PKG, "_build")
 LIB_PATH = os.path.join(PKG, "libtsd.so")
+# the range-checked variant (TSD_CHECKS): every index the fused row pass
+# follows is checked, a violation recorded in the decoder's status word
+CHECKS_BUILD_DIR = os.path.join(PKG, "_build_checks")
+CHECKS_LIB_PATH = os.path.join(PKG, "libtsd_checks.so")
 
 SOURCES = ["tables.cpp", "arpa.cpp", "decoder.cu", "row_pass.cu", "row_fused.cu", "joint_simt.cu", "joint_tc.cu", "noalloc.cu", "row_beam.cu", "row_pruned.cu", "gemm_tc.cu", "encoder.cu", "encoder_gemm.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
@@ -42,13 +46,19 @@ def _stale(target: str, deps: List[str]) -> bool:
     return any(os.path.getmtime(p) > t for p in deps)
 
 
-def build(force: bool = False, verbose: bool = False, extra: List[str] = ()) -> str:
-    os.makedirs(BUILD_DIR, exist_ok=True)
+def build(force: bool = False, verbose: bool = False, extra: List[str] = (), checks: bool = False) -> str:
+    """Compiles libtsd.so (or, with checks, libtsd_checks.so built with
+    -DTSD_CHECKS) and returns its path."""
+    build_dir = CHECKS_BUILD_DIR if checks else BUILD_DIR
+    lib_path = CHECKS_LIB_PATH if checks else LIB_PATH
+    if checks:
+        extra = list(extra) + ["-DTSD_CHECKS"]
+    os.makedirs(build_dir, exist_ok=True)
     headers = [os.path.join(CSRC, f) for f in os.listdir(CSRC) if f.endswith((".h", ".cuh"))] + [os.path.join(INCLUDE, "tsd.h")]
     objs, jobs = [], []
     for src in SOURCES:
         path = os.path.join(CSRC, src)
-        obj = os.path.join(BUILD_DIR, src + ".o")
+        obj = os.path.join(build_dir, src + ".o")
         objs.append(obj)
         if force or _stale(obj, [path] + headers):
             x = ["-x", "cu"] if src.endswith(".cu") else []
@@ -64,13 +74,12 @@ def build(force: bool = False, verbose: bool = False, extra: List[str] = ()) -> 
 
     with concurrent.futures.ThreadPoolExecutor(max_workers=max(1, min(len(jobs), os.cpu_count() or 4))) as ex:
         list(ex.map(run, jobs))
-    if force or jobs or _stale(LIB_PATH, objs):
-        tmp = LIB_PATH + f".tmp{os.getpid()}"
+    if force or jobs or _stale(lib_path, objs):
+        tmp = lib_path + f".tmp{os.getpid()}"
         run([nvcc()] + ARCH + ["-shared", "-cudart", "static", "-o", tmp] + objs)
-        os.replace(tmp, LIB_PATH)
-    return LIB_PATH
+        os.replace(tmp, lib_path)
+    return lib_path
 
 
 if __name__ == "__main__":
-    build(force="--force" in sys.argv, verbose=True)
-    print(LIB_PATH)
+    print(build(force="--force" in sys.argv, verbose=True, checks="--checks" in sys.argv))

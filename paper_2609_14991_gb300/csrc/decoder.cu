@@ -67,6 +67,7 @@ void enqueue_chunk(tsd_decoder* d, int M, int T, cudaStream_t s, const std::vect
   }
   for (int step = 0; step <= S; ++step) {
     const bool pdl = d->pdl && !ev && step > 0;  // the first launch follows the parameter copy
+    NvtxRange nvtx_step("label step");  // host-side enqueue (captured once into the chunk's graph)
     mark(0);
     if (d->cfg.beam_k > 1) launch_row_beam(v, M / d->cfg.beam_k, step, step == S ? 1 : 0, d->row_smem, s, pdl);
     else if (d->cfg.prune_k > 0) launch_row_pruned(v, M, step, step == S ? 1 : 0, s, pdl);
@@ -400,6 +401,7 @@ tsd_status create_impl(const tsd_decoder_cfg* cfg, const void* W_out_bf16, const
   v.cap_rows = nullptr;
   v.cap_steps = 0;
   v.err = err;
+  v.wait_ns = tc_wait_ns_default();
   v.ctr = ctr;
   v.count = 0;
   v.dflt = dflt;
@@ -514,6 +516,7 @@ extern "C" tsd_status tsd_decode_chunk(tsd_decoder* d, int32_t n, const int32_t*
                                        int32_t* out_tokens, int32_t* out_frames, float* out_scores,
                                        int32_t* out_counts, void* cuda_stream) {
   clear_error();
+  NvtxRange nvtx("tsd_decode_chunk");
   if (!d || !slots || !enc_bf16 || !out_counts) return fail(TSD_EINVAL, "tsd_decode_chunk: NULL argument");
   if (d->cfg.beam_k == 1 && (!out_tokens || !out_frames || !out_scores))
     return fail(TSD_EINVAL, "tsd_decode_chunk: NULL output array");
@@ -587,6 +590,7 @@ extern "C" tsd_status tsd_decode_chunk(tsd_decoder* d, int32_t n, const int32_t*
         return cuda_fail(ce, "tsd_decode_chunk: graph instantiate");
       }
     }
+    NvtxRange nvtx_launch("chunk graph launch");
     TSD_CUDA(cudaGraphLaunch(es.exec, s));
   } else {
     enqueue_chunk(d, M, T, s, evp, d->timing ? &es.cls : nullptr);
@@ -992,6 +996,14 @@ extern "C" tsd_status tsd_decoder_set_option(tsd_decoder* d, const char* name, i
     d->pdl = value ? 1 : 0;
     return drop_graphs(d);
   }
+  if (n == "wait_ns") {
+    // limit of the joint kernel's progress waits; an expired wait ends the
+    // kernel early (after draining its copies) and tsd_decoder_check reports it
+    if (value < 0 || value > 10000000000ll)
+      return fail(TSD_EINVAL, "tsd_decoder_set_option: wait_ns must be in [0, 1e10]");
+    d->view.wait_ns = (unsigned long long)value;
+    return drop_graphs(d);
+  }
   if (n == "joint_bn") {
     if (value != 64 && value != 128 && value != 256) return fail(TSD_EINVAL, "tsd_decoder_set_option: joint_bn must be 64, 128 or 256");
     tsd_status st = drop_graphs(d);
@@ -1062,7 +1074,8 @@ extern "C" tsd_status tsd_decoder_check(tsd_decoder* d) {
   TSD_CUDA(cudaMemcpy(&e, d->view.err, sizeof(e), cudaMemcpyDeviceToHost));
   if (e) {
     TSD_CUDA(cudaMemset(d->view.err, 0, sizeof(e)));
-    return fail(TSD_EDEVICE, "tsd_decoder_check: a device wait expired (code 0x%x)", e);
+    return fail(TSD_EDEVICE, "tsd_decoder_check: device status 0x%x (%s)", e,
+                e >= 0x100 ? "a range check of the checked build failed" : "a bounded device wait expired");
   }
   return TSD_OK;
 }

@@ -103,6 +103,9 @@ struct DecView {
   float* logits;        // [M_pad][N_pad] fp32 joint logits of the current step, plus dvec
   float* dvec;          // [N_pad] per call: lambda*log p(v) + beta*bonus*[the root has a child v]; 0 from V on
   int32_t* err;  // device status word: nonzero after a bounded wait expired
+  // limit of the joint kernel's progress waits (a wait that drains copies or
+  // MMAs still in flight before an early exit keeps the 1 s limit)
+  unsigned long long wait_ns;
   unsigned long long* ctr;  // algorithmic bytes counted by row passes (replayed or timed)
   int32_t count;            // 1: every row pass adds its algorithmic bytes to *ctr
 };

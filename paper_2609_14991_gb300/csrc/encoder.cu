@@ -756,6 +756,7 @@ extern "C" tsd_status tsd_encoder_close(tsd_encoder* e, int32_t slot) {
 extern "C" tsd_status tsd_encode_chunk(tsd_encoder* e, int32_t n, const int32_t* slots, const void* feats_bf16,
                                        int32_t C, void* out_bf16, void* cuda_stream) {
   clear_error();
+  NvtxRange nvtx("tsd_encode_chunk");
   if (!e || !slots || !feats_bf16 || !out_bf16) return fail(TSD_EINVAL, "tsd_encode_chunk: NULL argument");
   const tsd_encoder_cfg& c = e->cfg;
   if (n < 1 || n > c.max_streams) return fail(TSD_EINVAL, "tsd_encode_chunk: n=%d out of [1, %d]", n, c.max_streams);

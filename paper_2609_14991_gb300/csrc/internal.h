@@ -22,6 +22,13 @@ constexpr int kNPad = 256;         // the vocabulary axis is padded to this mult
 constexpr int kMPad = 128;         // the row axis is padded to this multiple
 constexpr int kMaxLm = 4;          // n-gram LMs fused at once (Eq. 1, sum over i)
 
+// An NVTX range for the lifetime of the object (header-only NVTX 3: the
+// calls do nothing unless a profiler is attached).
+struct NvtxRange {
+  explicit NvtxRange(const char* name);
+  ~NvtxRange();
+};
+
 // Records a message for tsd_last_error() and returns st.
 tsd_status fail(tsd_status st, const char* fmt, ...);
 void clear_error();
@@ -33,6 +40,9 @@ tsd_status cuda_fail(cudaError_t e, const char* what);
     if (_e != cudaSuccess) return ::tsd::cuda_fail(_e, #call); \
   } while (0)
 
+// True if the test hook (tsd_debug_fail_alloc) makes this allocation fail.
+bool alloc_hook_fires();
+
 // Device allocations owned by one object; freed together.
 struct DevArena {
   std::vector<void*> ptrs;
@@ -41,6 +51,7 @@ struct DevArena {
   tsd_status alloc(T** p, size_t count) {
     void* q = nullptr;
     size_t nb = sizeof(T) * (count ? count : 1);
+    if (alloc_hook_fires()) return fail(TSD_ENOMEM, "cudaMalloc(%zu bytes) failed: injected by the test hook", nb);
     cudaError_t e = cudaMalloc(&q, nb);
     if (e != cudaSuccess) {
       cudaGetLastError();
@@ -93,11 +104,12 @@ struct LmView {
   const float* dense0 = nullptr;      // [rows][V4]
   const int32_t* uni_dense = nullptr; // [V] dense row of the unigram state of v, or -1
   int32_t V4 = 0;                     // row stride of dense0
+  int32_t n_dense = 0;                // rows of dense0
 };
 
 // Device view of the phrase trie.  Node 0 is the root.
 struct TrieView {
-  int32_t V = 0, n_nodes = 0, max_depth = 0;
+  int32_t V = 0, n_nodes = 0, max_depth = 0, n_children = 0;
   float bonus = 0.f;
   const int32_t* nd_begin = nullptr;    // [Q] first child
   const int32_t* nd_count = nullptr;    // [Q] children

@@ -138,18 +138,18 @@ __global__ void __launch_bounds__(kThreads, 1)
           ++issued;
           continue;
         }
-        if (!mbar_wait(empty + s, ph ^ 1u)) { ok = false; break; }
+        if (!mbar_wait(empty + s, ph ^ 1u, d.wait_ns)) { ok = false; break; }
         mbar_expect_tx(full + s, S::kStageBytes);
         tma_load_2d(sa, &tmA, full + s, kb * kBK, m0);
         tma_load_2d(sa + S::kABytes, &tmB, full + s, kb * kBK, n0);
         ++issued;
       }
-      if (!ok) {
-        // drain the copies this CTA still has in flight before it exits
-        for (int kb = max(0, issued - S::kStages); kb < issued; ++kb)
-          mbar_wait(full + kb % S::kStages, (uint32_t)(kb / S::kStages) & 1u);
-        atomicOr(d.err, 1);
-      }
+      // Never exit with copies in flight: wait for the last use of every
+      // stage (its final phase; complete already when the MMAs consumed it,
+      // as they do unless a wait expired), with the long limit.
+      for (int kb = max(0, issued - S::kStages); kb < issued; ++kb)
+        mbar_wait(full + kb % S::kStages, (uint32_t)(kb / S::kStages) & 1u);
+      if (!ok) atomicOr(d.err, 1);
     }
     __syncwarp();  // reconverge before the CTA barrier below (bar.sync is warp-aligned)
   } else if (warp == 1) {
@@ -158,7 +158,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int kb = 0; kb < KB; ++kb) {
         const int s = kb % S::kStages;
         const uint32_t ph = (uint32_t)(kb / S::kStages) & 1u;
-        if (!mbar_wait(full + s, ph)) { ok = false; break; }
+        if (!mbar_wait(full + s, ph, d.wait_ns)) { ok = false; break; }
         fence_after();
         const uint32_t sa = smem_u32(smem + s * S::kStageBytes);
         const uint64_t ad = sw128_desc(sa), bd = sw128_desc(sa + S::kABytes);
@@ -196,7 +196,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int i = (int)threadIdx.x - 64; i < BN; i += kEpiThreads) sD[i] = __ldcg(d.dvec + n0 + i);
       asm volatile("bar.sync 2, %0;" ::"n"(kEpiThreads) : "memory");
     }
-    ok = __all_sync(0xffffffffu, mbar_wait(accum, 0));  // warp-uniform: tcgen05.ld is .sync.aligned
+    ok = __all_sync(0xffffffffu, mbar_wait(accum, 0, d.wait_ns));  // warp-uniform: tcgen05.ld is .sync.aligned
     if (!ok && lane == 0) atomicOr(d.err, 4);
     fence_after();
     // the second half of a 256-wide bias tile goes into the drained stages
@@ -207,7 +207,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int c = S::kEarly; c < S::kBoxes; ++c)
         tma_load_2d(smem + (c - S::kEarly) * S::kBoxBytes, &tmBias, biasbar + 1, n0 + 32 * c, m0);
     }
-    const bool have_early = use_bias ? __all_sync(0xffffffffu, mbar_wait(biasbar, 0)) : true;
+    const bool have_early = use_bias ? __all_sync(0xffffffffu, mbar_wait(biasbar, 0, d.wait_ns)) : true;
     if (!have_early) {
       ok = false;
       if (lane == 0) atomicOr(d.err, 16);
@@ -221,7 +221,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         __syncwarp();  // the per-chunk selection branches; tcgen05.ld wants the warp whole
         if (use_bias && c >= S::kEarly && !late_done) {
           late_done = true;
-          if (!__all_sync(0xffffffffu, mbar_wait(biasbar + 1, 0))) {
+          if (!__all_sync(0xffffffffu, mbar_wait(biasbar + 1, 0, d.wait_ns))) {
             if (lane == 0) atomicOr(d.err, 32);
             break;
           }
@@ -385,9 +385,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
     }
-    // never leave with bias boxes still landing in shared memory, nor with
-    // logits stores still reading the staging buffers
+    // never leave with bias boxes still landing in shared memory, MMAs still
+    // writing the accumulator, nor logits stores still reading the staging
+    // buffers (these drains keep the long limit whatever wait_ns is)
     if (!late_done && warp == 2 && lane == 0) mbar_wait(biasbar + 1, 0);
+    if (!have_early && warp == 2 && lane == 0) mbar_wait(biasbar, 0);
+    if (warp == 2 && lane == 0) mbar_wait(accum, 0);
     if (LOGITS && lane == 0) tma_store_wait_all();
     __syncwarp();
     // Merge the two halves' partials of each row: the second half leaves its
@@ -466,6 +469,8 @@ __global__ void __launch_bounds__(kThreads, 1)
 }
 
 }  // namespace
+
+unsigned long long tc_wait_ns_default() { return kWaitNs; }
 
 int joint_tc_pick_bn(int M_max, int N_pad, int sms) {
   // wider tiles re-read fewer operands; take the widest whose tiles still

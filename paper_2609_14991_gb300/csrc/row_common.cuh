@@ -8,6 +8,19 @@ namespace row {
 
 constexpr float kNegInf = -__builtin_huge_valf();
 
+// Range checks of the TSD_CHECKS build: a failed check records its code in
+// the decoder's status word (the first one wins; tsd_decoder_check reports
+// TSD_EDEVICE) and the caller skips the access.  In the ordinary build the
+// condition is not evaluated.
+#ifdef TSD_CHECKS
+__device__ __forceinline__ bool checked(bool cond, int32_t* err, int code) {
+  if (!cond) atomicCAS(err, 0, 0x100 + code);
+  return cond;
+}
+#else
+__device__ __forceinline__ constexpr bool checked(bool, int32_t*, int) { return true; }
+#endif
+
 // After divergent code (a single-thread section, a lane-strided loop) the
 // lanes of a warp can keep running apart past the point where they could
 // rejoin, and every warp-synchronous step after it (shuffle, ballot) then

@@ -46,6 +46,7 @@ namespace tsd {
 namespace {
 
 using row::best_merge;
+using row::checked;
 using row::kNegInf;
 using row::lse_merge;
 using row::warp_find;
@@ -99,6 +100,7 @@ __global__ void __launch_bounds__(kFzThreads) __maxnreg__((VAR & 4) ? 128 : 72) 
   __shared__ float s_bv[kFzWarps];
   __shared__ int s_bi[kFzWarps];
   __shared__ unsigned long long s_bytes;  // algorithmic bytes of the row-step (when counting)
+  __shared__ int s_bad;                   // TSD_CHECKS: a range check failed; the row stops
 
   // 1. Row state.  It was written by the previous row pass; under
   // programmatic launch this grid may start before its own wait, so these
@@ -116,6 +118,7 @@ __global__ void __launch_bounds__(kFzThreads) __maxnreg__((VAR & 4) ? 128 : 72) 
     s_beta = P->beta;
     s_n = P->n;
     s_bytes = 0;
+    s_bad = !checked(slot >= 0 && slot < d.lm_stride, d.err, 1);
   }
   {  // per-label scratch reset
     uint4* k4 = reinterpret_cast<uint4*>(key);
@@ -128,6 +131,7 @@ __global__ void __launch_bounds__(kFzThreads) __maxnreg__((VAR & 4) ? 128 : 72) 
     }
   }
   row::block_sync();
+  if (s_bad) return;
   const int slot = s_slot, T = s_T;
   // the chains are read whole (their arrays have room for the longest), so
   // their lengths need not be known first
@@ -154,6 +158,26 @@ __global__ void __launch_bounds__(kFzThreads) __maxnreg__((VAR & 4) ? 128 : 72) 
     }
   }
   row::block_sync();
+#ifdef TSD_CHECKS
+  if (tid == 0) {  // every index the row will follow is inside its table
+    bool ok = checked(s_nl >= 0 && s_nl <= kLmChain && s_nt >= 0 && s_nt <= kTrChain, d.err, 2) &&
+              checked(s_last >= 0 && s_last <= V, d.err, 3);
+    for (int l = 0; ok && l < s_nl; ++l) {
+      const int4 c = s_lmr[l];
+      ok = checked(s_lm[l] >= 0 && s_lm[l] < d.lm.n_states, d.err, 4) &&
+           checked(c.x >= 0 && c.y >= 0 && (int64_t)c.x + c.y <= d.lm.n_arcs, d.err, 5) &&
+           checked(l > 0 || (c.w >= -1 && c.w < d.lm.n_dense), d.err, 6);
+    }
+    for (int k = 0; ok && k < s_nt; ++k) {
+      const int4 c = s_trr[k];
+      ok = checked(s_tr[k] > 0 && s_tr[k] < d.tr.n_nodes, d.err, 7) &&
+           checked(c.x >= 0 && c.y >= 0 && c.x + c.y <= d.tr.n_children && c.z >= 1 && c.z <= 63, d.err, 8);
+    }
+    s_bad = !ok;
+  }
+  row::block_sync();
+  if (s_bad) return;
+#endif
   // the encoder frames this step can use (t, or t+1 after a frame advance)
   // go to L1: no kernel of the chunk writes them
   if (!PRED && s_t < T) {
@@ -221,10 +245,11 @@ __global__ void __launch_bounds__(kFzThreads) __maxnreg__((VAR & 4) ? 128 : 72) 
     auto offer = [&](int l, int i0, int4 tk) {
       const int b = s_lmr[l].x, c = s_lmr[l].y;
       const uint32_t tag = (uint32_t)(l + 1) << 24;
-      if (i0 >= b && i0 < b + c) atomicMax(key + tk.x, tag | (uint32_t)(i0 - b));
-      if (i0 + 1 >= b && i0 + 1 < b + c) atomicMax(key + tk.y, tag | (uint32_t)(i0 + 1 - b));
-      if (i0 + 2 >= b && i0 + 2 < b + c) atomicMax(key + tk.z, tag | (uint32_t)(i0 + 2 - b));
-      if (i0 + 3 >= b && i0 + 3 < b + c) atomicMax(key + tk.w, tag | (uint32_t)(i0 + 3 - b));
+      const int tv[4] = {tk.x, tk.y, tk.z, tk.w};
+#pragma unroll
+      for (int j = 0; j < 4; ++j)
+        if (i0 + j >= b && i0 + j < b + c && checked(tv[j] >= 0 && tv[j] < V, d.err, 9))
+          atomicMax(key + tv[j], tag | (uint32_t)(i0 + j - b));
     };
 #pragma unroll
     for (int u = 0; u < kHeld; ++u)
@@ -299,7 +324,8 @@ __global__ void __launch_bounds__(kFzThreads) __maxnreg__((VAR & 4) ? 128 : 72) 
             const float pv[4] = {lp[u].x, lp[u].y, lp[u].z, lp[u].w};
 #pragma unroll
             for (int j = 0; j < 4; ++j)
-              if (i0 + j >= b0 && i0 + j < b0 + c0 && key[tv[j]] == 0u) {
+              if (i0 + j >= b0 && i0 + j < b0 + c0 && checked(tv[j] >= 0 && tv[j] < V, d.err, 9) &&
+                  key[tv[j]] == 0u) {
                 key[tv[j]] = __float_as_uint(delta_of(0, pv[j], tv[j]));
                 lmf[tv[j]] = 1;
               }
@@ -322,7 +348,8 @@ __global__ void __launch_bounds__(kFzThreads) __maxnreg__((VAR & 4) ? 128 : 72) 
         for (int j = 0; j < 4; ++j) {
           const int i = hi[u] + j;
           wv[u][j] = 0.f;
-          if (i >= b && i < b + c && key[tv[j]] == (tag | (uint32_t)(i - b))) {
+          if (i >= b && i < b + c && checked(tv[j] >= 0 && tv[j] < V, d.err, 9) &&
+              key[tv[j]] == (tag | (uint32_t)(i - b))) {
             won |= 1u << (4 * u + j);
             wv[u][j] = delta_of(l, pv[j], tv[j]);
           }
@@ -364,7 +391,8 @@ __global__ void __launch_bounds__(kFzThreads) __maxnreg__((VAR & 4) ? 128 : 72) 
         const float pv[4] = {lq.x, lq.y, lq.z, lq.w};
 #pragma unroll
         for (int j = 0; j < 4; ++j)
-          if (i0 + j >= b && i0 + j < b + c && lmf[tv[j]] == 0 && key[tv[j]] == (tag | (uint32_t)(i0 + j - b))) {
+          if (i0 + j >= b && i0 + j < b + c && checked(tv[j] >= 0 && tv[j] < V, d.err, 9) && lmf[tv[j]] == 0 &&
+              key[tv[j]] == (tag | (uint32_t)(i0 + j - b))) {
             xw |= 1u << j;
             xv[j] = delta_of(l, pv[j], tv[j]);
           }
@@ -514,6 +542,8 @@ __global__ void __launch_bounds__(kFzThreads) __maxnreg__((VAR & 4) ? 128 : 72) 
           for (int l = 0; l < nl_old && ln < kLmChain; ++l) {
             const int4 h = s_lm_hit[l];
             if (h.x < 0) break;  // no arc at this level (-2) or the top order (-1)
+            if (!checked(h.x < d.lm.n_states && h.y >= 0 && h.z >= 0 && (int64_t)h.y + h.z <= d.lm.n_arcs, d.err, 10))
+              break;
             s_lm[ln] = h.x;
             s_lmr[ln] = make_int4(h.y, h.z, h.w, 0);
             ++ln;
@@ -527,6 +557,7 @@ __global__ void __launch_bounds__(kFzThreads) __maxnreg__((VAR & 4) ? 128 : 72) 
         for (int i = 0; i < nt_old; ++i) {
           const int4 h = s_tr_hit[i];
           if (h.x < 0) continue;
+          if (!checked(h.x > 0 && h.x < d.tr.n_nodes && h.w >= 0 && h.z + h.w <= d.tr.n_children, d.err, 11)) continue;
           if (tn == 0 && h.y == 0) reset = true;
           const int dd = s_trr[i].z + 1;  // the child's children sit one deeper
           if (tn < kTrChain) {

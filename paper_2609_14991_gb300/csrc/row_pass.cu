@@ -1,4 +1,6 @@
-// Row pass of the fused decode step: one CTA per hypothesis row.
+// Row pass of the fused decode step with several n-gram LMs (Eq. 1, the sum
+// over LMs): one CTA per hypothesis row.  (Greedy decoding with at most one
+// LM runs row_fused.cu instead.)
 //
 // For row r at label step s it
 //   1. combines the joint kernel's per-tile partials of step s-1 into the
@@ -561,12 +563,7 @@ void launch_defaults(const DecView& d, cudaStream_t s) {
 cudaError_t prepare_kernels(size_t row_smem) {
   // dynamic scratch plus the kernel's static shared memory may pass the
   // 48 KB default even when the scratch alone does not
-  cudaError_t e = cudaFuncSetAttribute(k_row<0>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)row_smem);
-  if (e == cudaSuccess) e = cudaFuncSetAttribute(k_row<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)row_smem);
-  if (e == cudaSuccess) e = cudaFuncSetAttribute(k_row<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)row_smem);
-  if (e == cudaSuccess) e = cudaFuncSetAttribute(k_row<3>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)row_smem);
-  if (e == cudaSuccess) e = cudaFuncSetAttribute(k_row<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)row_smem);
-  return e;
+  return cudaFuncSetAttribute(k_row<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)row_smem);
 }
 
 void launch_repack(const uint16_t* W, uint16_t* Wt, int H, int N, int N_pad, cudaStream_t s) {
@@ -628,12 +625,9 @@ void launch_row(const DecView& d, int M, int step, int mode, size_t smem, cudaSt
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = pdl ? 1 : 0;
-  const int var = (d.pred_D ? 1 : 0) | (d.n_lm > 1 ? 2 : 0);
-  if (var == 0 && M <= 2 * d.sms) cudaLaunchKernelEx(&cfg, k_row<4>, d, step, mode);
-  else if (var == 0) cudaLaunchKernelEx(&cfg, k_row<0>, d, step, mode);
-  else if (var == 1) cudaLaunchKernelEx(&cfg, k_row<1>, d, step, mode);
-  else if (var == 2) cudaLaunchKernelEx(&cfg, k_row<2>, d, step, mode);
-  else cudaLaunchKernelEx(&cfg, k_row<3>, d, step, mode);
+  // greedy decoding with at most one LM runs k_row_fz (row_fused.cu); this
+  // pass serves several LMs (the stateful form takes one LM)
+  cudaLaunchKernelEx(&cfg, k_row<2>, d, step, mode);
 }
 
 }  // namespace tsd

@@ -11,9 +11,14 @@
 #include <numeric>
 #include <thread>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include "internal.h"
 
 namespace tsd {
+
+NvtxRange::NvtxRange(const char* name) { nvtxRangePushA(name); }
+NvtxRange::~NvtxRange() { nvtxRangePop(); }
 
 namespace {
 thread_local std::string g_err;
@@ -56,6 +61,18 @@ tsd_status cuda_fail(cudaError_t e, const char* what) {
 
 const char* last_error() { return g_err.c_str(); }
 
+namespace {
+std::atomic<int32_t> g_fail_alloc{0};  // allocations left before the injected failure (0: off)
+}  // namespace
+
+bool alloc_hook_fires() {
+  int32_t n = g_fail_alloc.load();
+  while (n > 0) {
+    if (g_fail_alloc.compare_exchange_weak(n, n - 1)) return n == 1;
+  }
+  return false;
+}
+
 }  // namespace tsd
 
 using namespace tsd;
@@ -63,6 +80,13 @@ using namespace tsd;
 extern "C" const char* tsd_last_error(void) { return tsd::last_error(); }
 
 extern "C" const char* tsd_version(void) { return "tsd 0.1 sm_103a"; }
+
+extern "C" tsd_status tsd_debug_fail_alloc(int32_t n) {
+  clear_error();
+  if (n < 0) return fail(TSD_EINVAL, "tsd_debug_fail_alloc: n=%d < 0", n);
+  g_fail_alloc.store(n);
+  return TSD_OK;
+}
 
 // ---------------------------------------------------------------------------
 // n-gram tables
@@ -325,6 +349,7 @@ extern "C" tsd_status tsd_ngram_build(int32_t V, int32_t order, const int64_t* c
   v.dense0 = d_dense;
   v.uni_dense = d_ud;
   v.V4 = (int32_t)V4;
+  v.n_dense = (int32_t)n_dense;
   v.st_begin = d_b;
   v.st_count = d_c;
   v.st_cum = d_cum;
@@ -484,6 +509,7 @@ extern "C" tsd_status tsd_boost_build(int32_t V, int32_t n_phr, const int32_t* o
   }
   v.ch_rec = r0;
   v.root_rec = r1;
+  v.n_children = (int32_t)ch_node.size();
   v.nd_begin = a0;
   v.nd_count = a1;
   v.nd_depth = a2;

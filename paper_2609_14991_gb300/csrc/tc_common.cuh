@@ -55,12 +55,12 @@ __device__ __forceinline__ bool mbar_try(uint64_t* b, uint32_t parity) {
 }
 
 // Waits for the phase of the given parity; false if it did not complete
-// within kWaitNs.
-__device__ __forceinline__ bool mbar_wait(uint64_t* b, uint32_t parity) {
+// within limit_ns nanoseconds.
+__device__ __forceinline__ bool mbar_wait(uint64_t* b, uint32_t parity, unsigned long long limit_ns = kWaitNs) {
   if (mbar_try(b, parity)) return true;
   const unsigned long long t0 = global_ns();
   while (!mbar_try(b, parity)) {
-    if (global_ns() - t0 > kWaitNs) return false;
+    if (global_ns() - t0 > limit_ns) return false;
   }
   return true;
 }

@@ -133,3 +133,21 @@ def test_noalloc_binding_rejects_bad_tensors_before_the_call(L):
         tsd.joint_select_noalloc(A, Wt, None, lab, sc)
     with pytest.raises(TypeError):
         tsd.joint_select_noalloc(np.zeros((4, 64)), Wt, None, lab, sc)
+
+
+def test_checked_build_compiles():
+    """The range-checked variant (-DTSD_CHECKS) of the fused row pass builds."""
+    import subprocess
+
+    src = os.path.join(ROOT, "paper_2609_14991_gb300", "csrc", "row_fused.cu")
+    out = os.path.join(ROOT, "paper_2609_14991_gb300", "_build_checks")
+    os.makedirs(out, exist_ok=True)
+    cmd = [_build.nvcc()] + _build._flags() + ["-DTSD_CHECKS", "-x", "cu", "-c", src, "-o",
+                                                os.path.join(out, "row_fused_check_probe.o")]
+    r = subprocess.run(cmd, capture_output=True, text=True)
+    assert r.returncode == 0, r.stderr[-2000:]
+
+
+def test_debug_fail_alloc_rejects_negative(L):
+    assert L.tsd_debug_fail_alloc(-1) == tsd.TSD_EINVAL
+    assert L.tsd_debug_fail_alloc(0) == tsd.TSD_OK
