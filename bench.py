@@ -60,16 +60,12 @@ def peaks():
 # their commands are summarised under profiles/.
 KERNEL_SOURCES = {
     "joint": ["joint_tc.cu", "joint_tc.h", "tc_common.cuh", "decoder.h", "internal.h"],
-    "row": ["row_pass.cu", "row_beam.cu", "row_common.cuh", "decoder.h", "internal.h"],
+    "row": ["row_fused.cu", "row_pass.cu", "row_beam.cu", "row_common.cuh", "decoder.h", "internal.h"],
     "egemm": ["encoder_gemm.cu", "encoder.cu", "encoder.h", "tc_common.cuh", "internal.h"],
 }
 TRAFFIC = {
-    (2, 256, "joint"): (4480879, "c364bfcf57dcdddc"),
-    (2, 256, "row"): (2176478, "4cb5e8bf2d6d8afb"),
-    (4, 1024, "joint"): (28863138, "c364bfcf57dcdddc"),
-    (4, 1024, "row"): (12059614, "4cb5e8bf2d6d8afb"),
-    (3, 128, "joint"): (6346155, "c364bfcf57dcdddc"),
-    (3, 128, "row"): (1901841, "4cb5e8bf2d6d8afb"),
+    (4, 1024, "joint"): (11050496, "3508e66f2646fc6a"),
+    (4, 1024, "row"): (29144576, "d3e65c4743c47a4d"),
 }
 
 
