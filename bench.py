@@ -569,10 +569,15 @@ def run_ours(args, w):
     # inside a long step takes the sustained bf16 peak.
     joint_ms = kernel_ms["joint"] / max(1, kernel_n["joint"])
     row_ms = kernel_ms["row"] / max(1, kernel_n["row"])
-    shared_rows = w.V * ((4 * (1 + len(extra)) if lmA is not None else 0) + (4 if ph is not None else 0))
+    # the greedy one-LM pass (k_row_ep) reads no shared V-wide row; the others
+    # read the call's unigram and root rows once per launch
+    ep = w.beam == 1 and not args.prune_k and not extra
+    shared_rows = 0 if ep else w.V * ((4 * (1 + len(extra)) if lmA is not None else 0) + (4 if ph is not None else 0))
     row_launches_with_bias = kernel_n["row"] - args.steps  # the final row pass of a chunk builds no bias
     row_bytes_graph = row_timed_bytes + shared_rows * max(0, row_launches_with_bias)
-    joint_roof = {"kernel": "k_joint_tc: joint GEMM (tcgen05) + fused log-softmax/selection epilogue",
+    joint_roof = {"kernel": ("k_joint_tc: joint GEMM (tcgen05) + epilogue applying Eq. 1 with the dense LM row, "
+                             "log-softmax and selection partials") if ep else
+                            "k_joint_tc: joint GEMM (tcgen05) + fused log-softmax/selection epilogue",
                   "bound": "tensor", "unit": "TFLOP/s",
                   "achieved": flop_per_launch / (joint_ms / 1000.0) / 1e12,
                   "peak": pk["bf16_tflops_sustained"],
@@ -587,12 +592,18 @@ def run_ours(args, w):
                                "achieved_warm": flop_per_launch / (joint_warm / 1000.0) / 1e12,
                                "peak": pk["bf16_tflops"], "peak_kind": f"{pk_kind} bf16 burst"}}
     joint_roof["frac"] = joint_roof["achieved"] / joint_roof["peak"]
-    row_roof = {"kernel": "k_row_beam" if w.beam > 1 else "k_row",
-                "what": "selection merge, LM/trie state advance, joint input, fusion bias",
+    row_roof = {"kernel": "k_row_beam" if w.beam > 1 else ("k_row_ep" if ep else "k_row"),
+                "what": ("decision from the tile partials and the correction list, LM/trie state advance, "
+                         "the new state's correction list and mask, joint input") if ep else
+                        "selection merge, LM/trie state advance, joint input, fusion bias",
                 "bound": "hbm", "unit": "GB/s",
                 "achieved": row_bytes_graph / (kernel_ms["row"] / 1000.0) / 1e9,
                 "peak": pk["hbm_gbs"], "peak_kind": f"{pk_kind} HBM copy",
                 "algorithmic": (f"{row_bytes_graph / max(1, kernel_n['row']):.0f} B per launch on average, "
+                                f"counted by the kernel per row (partials, the correction list read with its "
+                                f"logits and written, the mask, row state, label searches, every arc of the LM "
+                                f"chain levels 1.. and every child of the trie chain nodes, joint input)") if ep else
+                               (f"{row_bytes_graph / max(1, kernel_n['row']):.0f} B per launch on average, "
                                 f"counted by the kernel per evaluated row (partials, row state, label searches, "
                                 f"joint input, every arc of the LM chain levels and trie chain nodes) plus the "
                                 f"shared unigram/root rows once per launch; the dense bias row is not counted"),

@@ -175,10 +175,13 @@ tsd_status create_impl(const tsd_decoder_cfg* cfg, const void* W_out_bf16, const
   d->M_pad = round_up(d->M_max, kMPad);
   d->n_ptiles = d->N_pad / kPartialCols;
   d->V4 = round_up(c.V, 16);
-  // greedy decoding with at most one LM: the joint kernel writes logits and
-  // the row pass fuses; several LMs and beam search keep the dense bias row
-  const bool fused = c.beam_k == 1 && c.prune_k == 0 && n_lms <= 1;
-  d->row_smem = fused ? row_fused_smem_bytes(d->V4) : row_smem_bytes(d->V4, n_lms);
+  // greedy decoding with at most one LM (whose unigram states have their
+  // dense rows): the joint kernel's epilogue applies Eq. 1 up to the row's
+  // correction list; several LMs and beam search keep the dense bias row
+  const bool fused = c.beam_k == 1 && c.prune_k == 0 && n_lms <= 1 &&
+                     (n_lms == 0 || !lm_weights || lm_weights[0] == 1.f) &&
+                     (!lm || lm->view.order < 2 || lm->view.n_dense == lm->view.V);
+  d->row_smem = fused ? row_fused_smem_bytes(d->V4, d->N_pad) : row_smem_bytes(d->V4, n_lms);
   if (d->row_smem > 200 * 1024) return fail(TSD_EINVAL, "tsd_decoder_create: V too large for the row pass");
 
   DevArena& A = d->arena;
@@ -212,12 +215,19 @@ tsd_status create_impl(const tsd_decoder_cfg* cfg, const void* W_out_bf16, const
     return st;
   }
   if (fused) {
-    if ((st = A.alloc(&v.logits, (size_t)d->M_pad * d->N_pad)) || (st = A.alloc(&v.dvec, (size_t)d->N_pad))) {
+    v.mask_words = d->N_pad / 32;
+    if ((st = A.alloc(&v.logits, (size_t)d->M_pad * d->N_pad)) || (st = A.alloc(&v.dvec, (size_t)d->N_pad)) ||
+        (st = A.alloc(&v.c_lab, (size_t)d->M_pad * d->V4)) || (st = A.alloc(&v.c_add, (size_t)d->M_pad * d->V4)) ||
+        (st = A.alloc(&v.c_info, (size_t)d->M_pad)) ||
+        (st = A.alloc(&v.c_mask, (size_t)d->M_pad * v.mask_words))) {
       A.release();
       return st;
     }
     TSD_CUDA(cudaMemsetAsync(v.dvec, 0, sizeof(float) * (size_t)d->N_pad, s));
     TSD_CUDA(cudaMemsetAsync(v.logits, 0, sizeof(float) * (size_t)d->M_pad * d->N_pad, s));
+    // no dense row and an empty list until a row pass has written the row's
+    TSD_CUDA(cudaMemsetAsync(v.c_info, 0xff, sizeof(int4) * (size_t)d->M_pad, s));
+    TSD_CUDA(cudaMemsetAsync(v.c_mask, 0, sizeof(uint32_t) * (size_t)d->M_pad * v.mask_words, s));
   }
   v.fused = fused ? 1 : 0;
   const int topk = c.beam_k > 1 ? c.beam_k : c.prune_k;
@@ -337,7 +347,7 @@ tsd_status create_impl(const tsd_decoder_cfg* cfg, const void* W_out_bf16, const
     d->sms = sms;
     d->view.sms = sms;
     const int bn = joint_tc_pick_bn(d->M_max, d->N_pad, sms);
-    if ((ce = joint_tc_prepare(d->jtc, Abuf, d->M_pad, Wt, d->N_pad, c.H, bn, bias, v.logits)) != cudaSuccess)
+    if ((ce = joint_tc_prepare(d->jtc, Abuf, d->M_pad, Wt, d->N_pad, c.H, bn, bias)) != cudaSuccess)
       return cleanup(cuda_fail(ce, "tsd_decoder_create: tensor-core GEMM setup (TMA descriptors)"));
   }
   for (int i = 0; i < tsd_decoder::kRing; ++i) {
@@ -1009,7 +1019,7 @@ extern "C" tsd_status tsd_decoder_set_option(tsd_decoder* d, const char* name, i
     tsd_status st = drop_graphs(d);
     if (st) return st;
     cudaError_t ce = joint_tc_prepare(d->jtc, d->view.A, d->M_pad, d->view.Wt, d->N_pad, d->cfg.H, (int)value,
-                                      d->view.bias, d->view.logits);
+                                      d->view.bias);
     if (ce != cudaSuccess) return cuda_fail(ce, "tsd_decoder_set_option: joint_bn");
     if (d->joint_kind == 0) {
       d->n_ptiles = d->N_pad / d->jtc->bn;
@@ -1051,10 +1061,11 @@ extern "C" tsd_status tsd_decoder_replay(tsd_decoder* d, int32_t kernel, int32_t
       const int64_t shared = (int64_t)d->cfg.V * ((d->lm ? 4 : 0) + (d->boost ? 4 : 0));
       *algo_bytes = (int64_t)(b / (unsigned long long)reps) + shared;
     } else if (d->view.fused) {
-      // joint, logits out: the operands once (A rows, W_out), the logits
-      // and the softmax partials written
-      *algo_bytes = (int64_t)M * d->cfg.H * 2 + (int64_t)d->N * d->cfg.H * 2 + (int64_t)M * d->N * 4 +
-                    (int64_t)M * d->n_ptiles * 8;
+      // joint, dense epilogue: the operands once (A rows, W_out), each row's
+      // dense LM row and mask, the defaults, the partials written (the
+      // listed labels' logits are not counted)
+      *algo_bytes = (int64_t)M * d->cfg.H * 2 + (int64_t)d->N * d->cfg.H * 2 + (int64_t)M * d->V4 * 4 +
+                    (int64_t)M * d->view.mask_words * 4 + (int64_t)d->N_pad * 4 + (int64_t)M * d->n_ptiles * 16;
     } else {
       // joint: the operands once (A rows, W_out) and the bias rows read by the epilogue
       *algo_bytes = (int64_t)M * d->cfg.H * 2 + (int64_t)d->N * d->cfg.H * 2 + (int64_t)M * d->N * 4 +

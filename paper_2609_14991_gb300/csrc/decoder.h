@@ -94,14 +94,23 @@ struct DecView {
   float lm_w[kMaxLm]; // relative weights: LM i enters Eq. 1 with lambda * lm_w[i]
   float* dflt;        // [V4] per-call LM bias default lambda*log p(v) (0 past V)
   uint32_t* droot;    // [ceil(V4/32)] bit v: the trie root has a child labelled v
-  // Greedy decoding with at most one LM (fused = 1): the joint kernel
-  // writes logit + dvec and the per-tile softmax partials of the logits, and
-  // the row pass after it finishes Eq. 1 (its per-row LM and trie terms
-  // computed in shared memory before it waits for the joint kernel) and
-  // takes the argmax; no bias row.
+  // Greedy decoding with at most one LM (fused = 1).  Per row the joint
+  // kernel's epilogue evaluates Eq. 1 for every label up to the row's
+  // constant c_r, from the call's defaults dvec and the dense LM row of the
+  // row's unigram state (LmView::dense0): F[v] = logit[v] + dvec[v] +
+  // lambda * dense0[u][v].  The labels whose term differs from that (those
+  // that a deeper LM state or a trie node below the root continues with, and
+  // blank) are the row's correction list, written by the row pass before
+  // the joint runs: the joint leaves them out of its per-tile best and
+  // stores their raw logits; the next row pass evaluates them from the list.
   int32_t fused;
-  float* logits;        // [M_pad][N_pad] fp32 joint logits of the current step, plus dvec
+  float* logits;        // [M_pad][N_pad] fp32 raw logits of the listed labels (other entries unused)
   float* dvec;          // [N_pad] per call: lambda*log p(v) + beta*bonus*[the root has a child v]; 0 from V on
+  int32_t* c_lab;       // [M_pad][V4] the row's listed labels
+  float* c_add;         // [M_pad][V4] their term: F[v] = logit[v] + c_add
+  int4* c_info;         // [M_pad] (dense row of the row's unigram state or -1, list length, c_r bits, -)
+  uint32_t* c_mask;     // [M_pad][mask_words] bit v: label v is listed (blank always)
+  int32_t mask_words;   // N_pad / 32
   int32_t* err;  // device status word: nonzero after a bounded wait expired
   // limit of the joint kernel's progress waits (a wait that drains copies or
   // MMAs still in flight before an early exit keeps the 1 s limit)
@@ -123,7 +132,7 @@ cudaError_t prepare_fused_kernels(size_t smem);
 void launch_joint(const DecView& d, int M, int step, cudaStream_t s);
 void launch_defaults(const DecView& d, cudaStream_t s);
 size_t row_smem_bytes(int V4, int n_lm);
-size_t row_fused_smem_bytes(int V4);
+size_t row_fused_smem_bytes(int V4, int N_pad);
 cudaError_t prepare_kernels(size_t row_smem);
 void launch_row_beam(const DecView& d, int n, int step, int mode, size_t smem, cudaStream_t s, bool pdl);
 void launch_row_pruned(const DecView& d, int M, int step, int mode, cudaStream_t s, bool pdl);

@@ -99,8 +99,10 @@ struct LmView {
   // [V] the unigram state of v: (its dense row or -1, first arc, arcs,
   // cumulative backoff bits); the state id itself is 1 + v
   const int4* uni_rec = nullptr;
-  // Unigram states with many continuations (at least V/8) also have a dense
-  // row: per label log p(v | u) - log p(v), NaN where u has no arc v.
+  // Every unigram state u (order >= 2, V x V4 floats at most 1 GiB) also
+  // has a dense row: per label log p(v | u) - log p(v) - cum(u), 0 where u
+  // has no arc v (the LM term of a label whose deepest arc is u's, relative
+  // to lambda*log p(v) and the row's summed backoff).
   const float* dense0 = nullptr;      // [rows][V4]
   const int32_t* uni_dense = nullptr; // [V] dense row of the unigram state of v, or -1
   int32_t V4 = 0;                     // row stride of dense0

@@ -5,8 +5,10 @@
 // the softmax partial (max logit, sum exp(logit - max)) over the V+1 real
 // labels and the best fused value logit + bias (bias = lambda*LM +
 // beta*boost, 0 for blank), ties to the lowest label.  With DecView::fused
-// the row's logits plus the call's defaults are written out instead and the
-// row pass fuses.
+// the fused value is logit + D[v] + lambda*dense0[u][v] (the call's defaults
+// and the dense LM row of the row's unigram state u), and the labels on the
+// row's correction list are no candidates: their raw logits are stored for
+// the row pass.
 // This is the simple reference-grade kernel for small row counts; the
 // tensor-core kernel in joint_tc.cu does the same contraction with tcgen05.
 #include "decoder.h"
@@ -94,6 +96,14 @@ __global__ void __launch_bounds__(256) k_joint_simt(DecView d, int step) {
     const int gr = m0 + row;
     if (gr >= M) break;
     const float* brow = d.bias + (size_t)gr * d.N_pad;
+    const float* urow = nullptr;
+    const uint32_t* mrow = nullptr;
+    const float lam = d.params->lambda;
+    if (d.fused) {
+      const int u = __ldcg(&d.c_info[gr].x);
+      if (u >= 0 && u < d.lm.n_dense) urow = d.lm.dense0 + (size_t)u * d.V4;
+      mrow = d.c_mask + (size_t)gr * d.mask_words;
+    }
     float l[4];
     float mx = kNegInf, bv = kNegInf;
     int bi = INT_MAX;
@@ -103,7 +113,16 @@ __global__ void __launch_bounds__(256) k_joint_simt(DecView d, int step) {
       l[q] = tile[row * (kJN + 4) + c];
       if (gc < N) {
         mx = fmaxf(mx, l[q]);
-        float f = l[q] + (gc < V && !d.fused ? brow[gc] : 0.f);
+        float f;
+        if (d.fused) {
+          if ((__ldcg(mrow + (gc >> 5)) >> (gc & 31)) & 1u) {  // listed: the row pass evaluates it
+            d.logits[(size_t)gr * d.N_pad + gc] = l[q];
+            continue;
+          }
+          f = l[q] + fmaf(lam, (urow && gc < V) ? __ldg(urow + gc) : 0.f, __ldcg(d.dvec + gc));
+        } else {
+          f = l[q] + (gc < V ? brow[gc] : 0.f);
+        }
         if (f > bv) { bv = f; bi = gc; }
       }
     }
@@ -124,13 +143,6 @@ __global__ void __launch_bounds__(256) k_joint_simt(DecView d, int step) {
     for (int o = 16; o > 0; o >>= 1) se += __shfl_xor_sync(0xffffffffu, se, o);
     if (lane == 0)
       d.part[(size_t)gr * d.n_ptiles + blockIdx.x] = make_float4(mx, se, bv, __int_as_float(bi));
-    if (d.fused) {  // the row pass applies Eq. 1 to the logits
-#pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        const int gc = n0 + lane * 4 + q;
-        d.logits[(size_t)gr * d.N_pad + gc] = l[q] + __ldcg(d.dvec + gc);
-      }
-    }
     if (d.cap_logits && step < d.cap_steps) {
 #pragma unroll
       for (int q = 0; q < 4; ++q) {

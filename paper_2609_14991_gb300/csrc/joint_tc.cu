@@ -9,8 +9,12 @@
 // tcgen05.ld (thread = row; two warps per 32-lane quadrant take alternate
 // 32-column chunks) and reduce it on chip to the row's selection partial for
 // this tile: softmax max and sum over the real labels, and the best fused
-// value logit + bias (lambda*LM + beta*boost; blank gets 0), ties to the
-// lowest label.  Logits never leave the SM.
+// value, ties to the lowest label.  The fused value is logit + bias with a
+// dense fusion bias row per row (several LMs), or, for greedy decoding with
+// at most one LM (DENSE), logit + D[v] + lambda * dense0[u][v]: the call's
+// defaults plus the dense LM row of the row's unigram state u, leaving out
+// the labels on the row's correction list, whose raw logits are stored for
+// the row pass instead.  No other logit leaves the SM.
 //
 // Warp roles (320 threads): warp 0 TMA producer, warp 1 TMEM allocator and
 // MMA issuer, warps 2-9 epilogue.  Every wait on an mbarrier is bounded in
@@ -34,41 +38,57 @@ constexpr float kNegInf = -__builtin_huge_valf();
 // bias (several LMs), the bias of the tile (128 rows x BN fp32) arrives by
 // TMA in 128 x 32 boxes with the 128-byte swizzle while the mainloop runs;
 // at BN = 256 only the first half has its own buffer and the second half
-// lands in the drained stages.  LOGITS (greedy decoding with at most one
-// LM) takes no bias: the fusion is applied by the row pass after it.
-constexpr int kStageOff = 16384;  // logits staging buffers: past the halves' exchange, in the drained stages
-template <int BN, bool LOGITS = false>
+// lands in the drained stages.  DENSE takes the tile's BN defaults instead.
+template <int BN, bool DENSE = false>
 struct Smem {
   static constexpr int kStages = (BN == 256) ? 3 : (BN == 128 ? 4 : 8);
   static constexpr int kABytes = kBM * kBK * 2;
   static constexpr int kBBytes = BN * kBK * 2;
   static constexpr int kStageBytes = kABytes + kBBytes;
   static constexpr int kBoxBytes = kBM * 32 * 4;
-  static constexpr int kBoxes = LOGITS ? 0 : BN / 32;
-  static constexpr int kEarly = LOGITS ? 0 : ((BN == 256) ? 4 : kBoxes);
-  static constexpr int kBiasBytes = kEarly * kBoxBytes + (LOGITS ? BN * 4 : 0);  // LOGITS: the tile's defaults D
+  static constexpr int kBoxes = DENSE ? 0 : BN / 32;
+  static constexpr int kEarly = DENSE ? 0 : ((BN == 256) ? 4 : kBoxes);
+  static constexpr int kBiasBytes = kEarly * kBoxBytes + (DENSE ? BN * 4 : 0);  // DENSE: the tile's defaults D
   static constexpr int kBytes = kStages * kStageBytes + kBiasBytes + 1024 /*align*/ + 256 /*barriers*/;
   static_assert((kBoxes - kEarly) * kBoxBytes <= kStages * kStageBytes, "late bias boxes fit the stages");
   // the epilogue halves' exchange (per row 18 floats, 4 flags) after the late boxes
   static_assert((kBoxes - kEarly) * kBoxBytes + kBM * 18 * 4 + 16 <= kStages * kStageBytes, "exchange fits");
-  static_assert(!LOGITS || (kBM * 18 * 4 + 16 <= kStageOff && kStageOff + 8 * 8192 <= kStages * kStageBytes),
-                "logits staging fits the drained stages");
 };
+
+// Sum over a chunk of 2^(l[i] * log2 e - s2) in four independent
+// accumulators (a single running sum would chain 32 dependent adds).
+__device__ __forceinline__ float sum_exp2_32(const float* l, float s2) {
+  float a[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+  for (int i = 0; i < 32; ++i) a[i & 3] += ex2_approx(fmaf(l[i], kLog2e, -s2));
+  return (a[0] + a[1]) + (a[2] + a[3]);
+}
+
+// The dense LM row segment of one row for one 32-label chunk (0 past the
+// table's row width V4, which is a multiple of 16; no row: all 0).
+__device__ __forceinline__ void load_dense_chunk(const float* __restrict__ row, int c0, int V4, float* x) {
+#pragma unroll
+  for (int j = 0; j < 8; ++j) {
+    float4 q = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (row && c0 + 4 * j < V4) q = __ldg(reinterpret_cast<const float4*>(row + c0) + j);
+    x[4 * j] = q.x; x[4 * j + 1] = q.y; x[4 * j + 2] = q.z; x[4 * j + 3] = q.w;
+  }
+}
 
 // BEAM: instead of the single best fused label, each row keeps the top-K
 // (K = d.topk <= 8: the beam width, or the pruned-fusion candidate count)
 // values of the tile, ties to the lower label.  With pruned fusion (d.prune)
 // the values are the plain logits: no bias tile is loaded.
-// LOGITS: no bias and no selection here: the epilogue writes the tile's
-// logits plus the call's shared defaults D[v] (d.dvec; fp32, row-major
-// [M_pad][N_pad], d.logits) and the per-row softmax partial (max, sum exp)
-// of the logits; the row pass finishes Eq. 1 and picks.
-template <int BN, bool BEAM, bool LOGITS>
+// DENSE: no bias tile; the fused value is logit + D[v] (d.dvec, the call's
+// defaults) + lambda * dense0[u][v] (u: the row's dense LM row, d.c_info),
+// and the labels whose bit is set in the row's mask (d.c_mask) are no
+// candidates here: their raw logits go to d.logits for the row pass.
+template <int BN, bool BEAM, bool DENSE>
 __global__ void __launch_bounds__(kThreads, 1)
     k_joint_tc(DecView d, int step, const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-               const __grid_constant__ CUtensorMap tmBias, const __grid_constant__ CUtensorMap tmLogits) {
-  using S = Smem<BN, LOGITS>;
-  static_assert(!(LOGITS && BEAM), "the logits output serves greedy decoding");
+               const __grid_constant__ CUtensorMap tmBias) {
+  using S = Smem<BN, DENSE>;
+  static_assert(!(DENSE && BEAM), "the dense epilogue serves greedy decoding");
   extern __shared__ __align__(1024) unsigned char smem_raw[];
   unsigned char* smem = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   unsigned char* bias_early = smem + S::kStages * S::kStageBytes;
@@ -80,7 +100,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int n0 = blockIdx.x * BN, m0 = blockIdx.y * kBM;
-  const bool use_bias = !LOGITS && !(BEAM && d.prune);
+  const bool use_bias = !DENSE && !(BEAM && d.prune);
   const int M = d.params->n * d.K;
   const int KB = d.H / kBK;
 
@@ -190,11 +210,34 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
     for (int j = 0; j < 8; ++j) { tv[j] = kNegInf; ti[j] = INT_MAX; }
     float tmin = kNegInf;  // tv[K-1]
-    float* sD = reinterpret_cast<float*>(bias_early);  // LOGITS: the tile's defaults D (kEarly is 0)
-    if (LOGITS) {
-      // while the MMAs run: the call's defaults of the tile's labels
+    float* sD = reinterpret_cast<float*>(bias_early);  // DENSE: the tile's defaults D (kEarly is 0)
+    const float* urow = nullptr;      // DENSE: the row's dense LM row
+    const uint32_t* mrow = nullptr;   // DENSE: the row's mask words of this tile
+    float lam = 0.f;
+    if (DENSE) {
+      // while the MMAs run: the call's defaults of the tile's labels, the
+      // row's dense LM row (its segment requested into L2 now) and mask
+      // (both written by the row pass before this grid's wait)
       for (int i = (int)threadIdx.x - 64; i < BN; i += kEpiThreads) sD[i] = __ldcg(d.dvec + n0 + i);
+      lam = d.params->lambda;
+      if (live) {
+        const int u = __ldcg(&d.c_info[gr].x);
+        if (u >= 0 && u < d.lm.n_dense) urow = d.lm.dense0 + (size_t)u * d.V4;
+        mrow = d.c_mask + (size_t)gr * d.mask_words + n0 / 32;
+        if (urow && half == 0 && n0 < d.V4) {
+          const uint32_t bytes = (uint32_t)min(BN, d.V4 - n0) * 4u;
+          asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(urow + n0), "r"(bytes) : "memory");
+        }
+      }
       asm volatile("bar.sync 2, %0;" ::"n"(kEpiThreads) : "memory");
+    }
+    // DENSE: the mask word and dense LM values of the next chunk this warp
+    // takes, loaded one chunk ahead (the first while the MMAs run)
+    float xn[32];
+    uint32_t mkn = 0u;
+    if (DENSE) {
+      load_dense_chunk(urow, n0 + half * 32, d.V4, xn);
+      mkn = mrow ? __ldcg(mrow + half) : 0u;
     }
     ok = __all_sync(0xffffffffu, mbar_wait(accum, 0, d.wait_ns));  // warp-uniform: tcgen05.ld is .sync.aligned
     if (!ok && lane == 0) atomicOr(d.err, 4);
@@ -226,14 +269,18 @@ __global__ void __launch_bounds__(kThreads, 1)
             break;
           }
         }
-        if constexpr (LOGITS) {
-          // the chunk's 32 logits of this row: the softmax partial, then the
-          // warp's 32 x 32 block goes out by one TMA store from a staging
-          // buffer in the drained stages (two per warp, alternating; the
-          // 128-byte swizzle keeps the row-per-thread writes conflict-free)
+        if constexpr (DENSE) {
+          const int c0 = n0 + c * 32;
+          const uint32_t mk = mkn;
+          float x[32];
+#pragma unroll
+          for (int i = 0; i < 32; ++i) x[i] = xn[i];
+          if (c + 2 < BN / 32) {
+            load_dense_chunk(urow, c0 + 64, d.V4, xn);
+            mkn = mrow ? __ldcg(mrow + c + 2) : 0u;
+          }
           float l[32];
           tmem_ld32(tbase + (uint32_t)(c * 32), l);
-          const int c0 = n0 + c * 32;
           if (c0 + 32 > N) {
 #pragma unroll
             for (int i = 0; i < 32; ++i)
@@ -251,8 +298,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             const float m2 = fmaxf(mx, cm);
             const float s2 = m2 * kLog2e;
             float acc = (mx == kNegInf) ? 0.f : se * ex2_approx(mx * kLog2e - s2);
-#pragma unroll
-            for (int i = 0; i < 32; ++i) acc += ex2_approx(fmaf(l[i], kLog2e, -s2));
+            acc += sum_exp2_32(l, s2);
             se = acc;
             mx = m2;
           }
@@ -262,27 +308,40 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int i = 0; i < 32; ++i)
               if (c0 + i < N) cl[c0 + i] = l[i];
           }
-          {
-            // out go logit + D (the call's defaults, the same for every row)
-            const float4* dv4 = reinterpret_cast<const float4*>(sD + 32 * c);
+          // fused values (reuse x); listed labels are stored, not candidates
+          const float4* dv4 = reinterpret_cast<const float4*>(sD + 32 * c);
 #pragma unroll
-            for (int j = 0; j < 8; ++j) {
-              const float4 dq = dv4[j];
-              l[4 * j] += dq.x; l[4 * j + 1] += dq.y; l[4 * j + 2] += dq.z; l[4 * j + 3] += dq.w;
-            }
-            unsigned char* stg = smem + kStageOff + (warp - 2) * 8192 + ((c >> 1) & 1) * 4096;
-            if (lane == 0) tma_store_wait_read1();  // this buffer's store of two chunks ago has read it
-            __syncwarp();
+          for (int j = 0; j < 8; ++j) {
+            const float4 dq = dv4[j];
+            x[4 * j] = l[4 * j] + fmaf(lam, x[4 * j], dq.x);
+            x[4 * j + 1] = l[4 * j + 1] + fmaf(lam, x[4 * j + 1], dq.y);
+            x[4 * j + 2] = l[4 * j + 2] + fmaf(lam, x[4 * j + 2], dq.z);
+            x[4 * j + 3] = l[4 * j + 3] + fmaf(lam, x[4 * j + 3], dq.w);
+          }
+          if (mk) {
+            float* lo = d.logits + (size_t)gr * d.N_pad + c0;
 #pragma unroll
-            for (int j = 0; j < 8; ++j)
-              *reinterpret_cast<float4*>(stg + lane * 128 + ((j ^ (lane & 7)) << 4)) =
-                  make_float4(l[4 * j], l[4 * j + 1], l[4 * j + 2], l[4 * j + 3]);
-            fence_async_smem();
-            __syncwarp();
-            if (lane == 0) {
-              tma_store_2d(&tmLogits, stg, c0, m0 + q * 32);
-              tma_store_commit();
-            }
+            for (int i = 0; i < 32; ++i)
+              if ((mk >> i) & 1u) {
+                lo[i] = l[i];
+                x[i] = kNegInf;
+              }
+          }
+          float u[16];
+#pragma unroll
+          for (int i = 0; i < 16; ++i) u[i] = fmaxf(x[i], x[i + 16]);
+#pragma unroll
+          for (int w = 8; w > 0; w >>= 1)
+#pragma unroll
+            for (int i = 0; i < w; ++i) u[i] = fmaxf(u[i], u[i + w]);
+          const float fm = u[0];
+          if (fm > bv) {
+            int j = 31;
+#pragma unroll
+            for (int i = 31; i >= 0; --i)
+              if (x[i] == fm) j = i;
+            bv = fm;
+            bi = c0 + j;
           }
           continue;
         }
@@ -372,8 +431,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           const float m2 = fmaxf(mx, cm);
           const float s2 = m2 * kLog2e;
           float acc = (mx == kNegInf) ? 0.f : se * ex2_approx(mx * kLog2e - s2);
-#pragma unroll
-          for (int i = 0; i < 32; ++i) acc += ex2_approx(fmaf(l[i], kLog2e, -s2));
+          acc += sum_exp2_32(l, s2);
           se = acc;
           mx = m2;
         }
@@ -385,13 +443,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
     }
-    // never leave with bias boxes still landing in shared memory, MMAs still
-    // writing the accumulator, nor logits stores still reading the staging
-    // buffers (these drains keep the long limit whatever wait_ns is)
+    // never leave with bias boxes still landing in shared memory or MMAs
+    // still writing the accumulator (these drains keep the long limit
+    // whatever wait_ns is)
     if (!late_done && warp == 2 && lane == 0) mbar_wait(biasbar + 1, 0);
     if (!have_early && warp == 2 && lane == 0) mbar_wait(biasbar, 0);
     if (warp == 2 && lane == 0) mbar_wait(accum, 0);
-    if (LOGITS && lane == 0) tma_store_wait_all();
     __syncwarp();
     // Merge the two halves' partials of each row: the second half leaves its
     // partial in shared memory past the late bias boxes (the stages are
@@ -424,9 +481,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           mx = m2;
         }
       }
-      if (LOGITS) {
-        d.part[(size_t)gr * d.n_ptiles + blockIdx.x] = make_float4(mx, se, 0.f, 0.f);
-      } else if (!BEAM) {
+      if (!BEAM) {
         const float v1 = xch[2];
         const int i1 = __float_as_int(xch[3]);
         if (v1 > bv || (v1 == bv && i1 < bi)) { bv = v1; bi = i1; }
@@ -482,13 +537,11 @@ int joint_tc_pick_bn(int M_max, int N_pad, int sms) {
 }
 
 cudaError_t joint_tc_prepare(JointTc* jt, const uint16_t* A, int M_pad, const uint16_t* Wt, int N_pad, int H, int bn,
-                             const float* bias, const float* logits) {
+                             const float* bias) {
   jt->bn = bn;
   if (!make_map(&jt->mapA, A, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, H, M_pad, kBK, kBM)) return cudaErrorInvalidValue;
   if (!make_map(&jt->mapB, Wt, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, H, N_pad, kBK, bn)) return cudaErrorInvalidValue;
   if (!make_map(&jt->mapBias, bias, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, N_pad, M_pad, 32, kBM))
-    return cudaErrorInvalidValue;
-  if (!make_map(&jt->mapLogits, logits ? logits : bias, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, N_pad, M_pad, 32, 32))
     return cudaErrorInvalidValue;
   const auto attr = cudaFuncAttributeMaxDynamicSharedMemorySize;
   cudaError_t e = cudaSuccess;
@@ -514,13 +567,13 @@ void launch_bn(cudaLaunchConfig_t& cfg, const JointTc& jt, const DecView& d, int
   const bool beam = d.topk > 1 || d.prune > 0;  // the top-K epilogue
   if (beam) {
     cfg.dynamicSmemBytes = Smem<BN>::kBytes;
-    cudaLaunchKernelEx(&cfg, k_joint_tc<BN, true, false>, d, step, jt.mapA, jt.mapB, jt.mapBias, jt.mapLogits);
+    cudaLaunchKernelEx(&cfg, k_joint_tc<BN, true, false>, d, step, jt.mapA, jt.mapB, jt.mapBias);
   } else if (d.fused) {
     cfg.dynamicSmemBytes = Smem<BN, true>::kBytes;
-    cudaLaunchKernelEx(&cfg, k_joint_tc<BN, false, true>, d, step, jt.mapA, jt.mapB, jt.mapBias, jt.mapLogits);
+    cudaLaunchKernelEx(&cfg, k_joint_tc<BN, false, true>, d, step, jt.mapA, jt.mapB, jt.mapBias);
   } else {
     cfg.dynamicSmemBytes = Smem<BN>::kBytes;
-    cudaLaunchKernelEx(&cfg, k_joint_tc<BN, false, false>, d, step, jt.mapA, jt.mapB, jt.mapBias, jt.mapLogits);
+    cudaLaunchKernelEx(&cfg, k_joint_tc<BN, false, false>, d, step, jt.mapA, jt.mapB, jt.mapBias);
   }
 }
 }  // namespace

@@ -1,42 +1,52 @@
 // Row pass of the fused decode step (greedy decoding, at most one n-gram
-// LM): one CTA per hypothesis row.  The joint kernel before it wrote, for
-// every label v of the row, logit[v] + D[v] with the call's shared defaults
-// D[v] = lambda*log p(v) + beta*bonus*[the trie root has a child v] (0 for
-// blank), and per-tile softmax partials of the raw logits; this pass finishes
-// Eq. 1 for the row, takes the greedy decision and advances the state.
+// LM): one CTA per hypothesis row.
 //
 // Eq. 1 for label v < V at the row's state is
 //   fused[v] = logit[v] - lse + lambda*log p_LM(v | h) + beta*bonus*(g(v) - depth)
-// where the LM state is kept as its whole suffix chain (one state per order):
+// where the LM state is kept as its whole suffix chain s_0 (the unigram state
+// of the previous label u), s_1, ..., s_{L-1} (one state per order):
 // log p_LM(v | h) is the arc v of the deepest chain state s_l that has one
 // plus the backoff weights of the deeper states, or log p(v) plus all of
 // them; g(v) is the depth of v's goto node from the deepest trie chain node
 // with a child v (the trie chain holds every trie node that is a suffix of
-// the current match), else [the root has a child v].  So
-//   fused[v] + lse = (logit[v] + D[v]) + c_r + delta[v],
-//   c_r = lambda*(summed backoff of the state) - beta*bonus*depth,
-//   delta[v] = lambda*(log p(v | s_l) - summed backoff of s_l - log p(v))
-//            + beta*bonus*(g(v) - [the root has a child v]),
-// delta[v] = 0 for a label no chain element continues with.  For row r at
-// label step s the pass
-//   1. (before waiting for the joint kernel) loads the row's state and chains
-//      and finds each label's deepest LM chain level: a deeper level's labels
-//      are a subset of a shallower one's (the model is suffix-closed).  The
-//      levels above 0 (few arcs) offer ((l + 1) << 24 | position) to their
-//      labels' words by a shared-memory atomicMax, so the deepest wins; then
-//      level 0 (the previous label's continuations, up to every label) is
-//      streamed once and writes the delta of every label no level above
-//      offered, and the offers' winners (held in registers) write theirs.
-//      The trie chain nodes are scattered shallowest first (the deepest
-//      overwrites);
-//   2. (after the wait) the log-sum-exp from the tile partials and the argmax
-//      of logit + D + c_r + delta over the labels (blank: its logit alone;
-//      ties to the lowest label), i.e. the greedy decision and its fused score;
+// the current match), else [the root has a child v].  With cum_l the summed
+// backoff of s_0..s_l and
+//   c_r = lambda*cum_{L-1} - beta*bonus*depth   (one constant per row),
+//   F[v] = fused[v] + lse - c_r
+//        = logit[v] + lambda*(log p(v | s_l) - cum_l) + beta*bonus*g(v),
+// with log p(v) and cum_{-1} = 0 when no chain state has an arc v.  Blank
+// (label V) has F = logit[V] - c_r.
+//
+// The deeper chain states' labels are nested: s_{l+1} has an arc v only if
+// s_l has one (the model is suffix-closed), so every label whose deepest arc
+// is not s_0's is a label of s_1, which has few arcs (a context of two
+// labels).  The joint kernel therefore evaluates, for every label,
+//   F0[v] = logit[v] + D[v] + lambda*dense0[u][v],
+//   D[v] = lambda*log p(v) + beta*bonus*[the root has a child v],
+//   dense0[u][v] = log p(v | u) - log p(v) - cum_0 (0 if u has no arc v),
+// which is F[v] for every label except those of s_1's arcs, the children of
+// the trie chain nodes, and blank: this pass lists those for the row (label
+// and its term F[v] - logit[v]) and marks them in a bitmask; the joint
+// leaves them out of its per-tile best and stores their raw logits.
+//
+// For row r at label step s the pass
+//   1. loads the row's state, both chains with their table records, and the
+//      length of the list its previous step wrote (for the state the joint
+//      just evaluated);
+//   2. after waiting for the joint kernel: the log-sum-exp and the best
+//      unlisted label from the tile partials, every listed label's F from its
+//      stored logit, blank's, and the argmax of them all (ties to the lowest
+//      label): the greedy decision and its fused score;
 //   3. blank (or the per-frame label limit) advances the frame; a label y is
 //      emitted and advances the chains, assembled from independent searches
 //      of y in every chain element, each hit carrying the next state's table
 //      record (first arc, arcs, summed backoff) in the same 16-byte load;
-//   4. writes the joint input of step s, bf16(ReLU(enc_t + E[last])).
+//   4. lists the labels of the new state: s_1's arcs, each with the term of
+//      its deepest chain level (found by a shared-memory atomicMax of
+//      ((level + 1) << 24 | position) over levels 1..L-1) plus the trie
+//      term; then the trie chain nodes' children that are not s_1 labels,
+//      with the level-0 LM term; the bitmask; c_r;
+//   5. writes the joint input of step s, bf16(ReLU(enc_t + E[last])).
 #include <algorithm>
 
 #include "row_common.cuh"
@@ -52,9 +62,9 @@ using row::lse_merge;
 using row::warp_find;
 
 constexpr int kFzThreads = 128;  // 4 warps: seven CTAs per SM at 72 registers
-constexpr int kStream = 4;       // level-0 arc groups of four per thread whose loads are issued together
-constexpr int kDense = 8;        // dense level-0 quads per thread whose loads are issued together
 constexpr int kFzWarps = kFzThreads / 32;
+constexpr int kHeld = 2;      // arc groups of four of levels 1.. a thread keeps in registers
+constexpr int kListHeld = 2;  // list entries a thread loads before waiting for the joint kernel
 
 // Aligned groups of four arcs a chain level's arcs [b, b + c) span.
 __device__ __forceinline__ int level_groups(int b, int c) { return c > 0 ? (b + c - (b & ~3) + 3) >> 2 : 0; }
@@ -65,10 +75,8 @@ __device__ __forceinline__ int level_groups(int b, int c) { return c > 0 ? (b + 
 // VAR bit 0: the stateful form (LSTM input rows instead of the joint input);
 // bit 2: few rows (at most two CTAs per SM are needed, registers are free).
 template <int VAR>
-__global__ void __launch_bounds__(kFzThreads) __maxnreg__((VAR & 4) ? 128 : 72) k_row_fz(DecView d, int step, int mode) {
+__global__ void __launch_bounds__(kFzThreads) __maxnreg__((VAR & 4) ? 128 : 72) k_row_ep(DecView d, int step, int mode) {
   constexpr bool PRED = (VAR & 1) != 0;
-  constexpr int QB = 8;     // label quads per thread whose loads are issued together
-  constexpr int kHeld = 2;  // arc groups of four of the levels above 0 a thread keeps in registers
   const Params* __restrict__ P = d.params;
   const int r = blockIdx.x;
   const int V = d.V;
@@ -76,27 +84,29 @@ __global__ void __launch_bounds__(kFzThreads) __maxnreg__((VAR & 4) ? 128 : 72) 
   const bool commit = (mode != 2);
   const bool counting = (mode == 2 || d.count);
   extern __shared__ __align__(16) unsigned char smem[];
-  // per label: the LM tag, then (for the winners) the LM delta's bits; 1 if
-  // the label has an LM delta; the trie goto depth (0: none)
-  uint32_t* key = reinterpret_cast<uint32_t*>(smem);      // [V4]
-  uint8_t* lmf = reinterpret_cast<uint8_t*>(key + d.V4);   // [V4]
-  uint8_t* dep = lmf + d.V4;                               // [V4]
+  // per label: the offer tag, then (for the winners) the LM term's bits; the
+  // list bitmask; 1 if the label has its LM term; the trie goto depth (0: none)
+  uint32_t* key = reinterpret_cast<uint32_t*>(smem);              // [V4]
+  uint32_t* msk = key + d.V4;                                      // [mask_words]
+  uint8_t* lmf = reinterpret_cast<uint8_t*>(msk + d.mask_words);  // [V4]
+  uint8_t* dep = lmf + d.V4;                                       // [V4]
 
   __shared__ int s_t, s_sym, s_cnt, s_y, s_last, s_slot, s_T, s_n;
-  __shared__ int s_nl, s_nt;
+  __shared__ int s_nl, s_nt, s_ext;
   __shared__ int32_t* s_out_tok;
   __shared__ int32_t* s_out_frame;
   __shared__ float* s_out_score;
   __shared__ int32_t* s_out_count;
   __shared__ const uint16_t* s_enc;
   __shared__ float s_lam, s_beta, s_score, s_lse, s_cr;
+  __shared__ int4 s_ci;               // the list the joint evaluated: (dense row, length, c_r bits, -)
   __shared__ int s_lm[kLmChain], s_tr[kTrChain];
-  __shared__ int4 s_lmr[kLmChain];    // LM chain records: (first arc, arcs, summed backoff bits, -)
+  __shared__ int4 s_lmr[kLmChain];    // LM chain records: (first arc, arcs, summed backoff bits, dense row at level 0)
   __shared__ int4 s_trr[kTrChain];    // trie chain records: (first child, children, depth of the children, -)
   __shared__ int4 s_lm_hit[kLmChain]; // target record of y's arc at each old level (x = -2: none)
   __shared__ int4 s_tr_hit[kTrChain]; // child record of y at each old trie node (x = -1: none)
   __shared__ int4 s_uni_hit, s_root_hit;
-  __shared__ int s_gbeg[kLmChain + 1];  // arc groups of the LM levels before level l
+  __shared__ int s_gbeg[kLmChain + 1];  // arc groups of the LM levels 1.. before level l
   __shared__ float s_bv[kFzWarps];
   __shared__ int s_bi[kFzWarps];
   __shared__ unsigned long long s_bytes;  // algorithmic bytes of the row-step (when counting)
@@ -118,6 +128,8 @@ __global__ void __launch_bounds__(kFzThreads) __maxnreg__((VAR & 4) ? 128 : 72) 
     s_beta = P->beta;
     s_n = P->n;
     s_bytes = 0;
+    s_ext = 0;
+    s_ci = step > 0 ? __ldcg(d.c_info + r) : make_int4(-1, 0, 0, 0);
     s_bad = !checked(slot >= 0 && slot < d.lm_stride, d.err, 1);
   }
   {  // per-label scratch reset
@@ -129,10 +141,25 @@ __global__ void __launch_bounds__(kFzThreads) __maxnreg__((VAR & 4) ? 128 : 72) 
       f4[q] = 0u;
       e4[q] = 0u;
     }
+    for (int q = tid; q < d.mask_words; q += blockDim.x) msk[q] = 0u;
   }
   row::block_sync();
   if (s_bad) return;
   const int slot = s_slot, T = s_T;
+  // the list of the state the joint evaluated (its first kListHeld entries
+  // per thread in registers)
+  int hv[kListHeld];
+  float ha[kListHeld];
+#pragma unroll
+  for (int u = 0; u < kListHeld; ++u) {
+    const int k = tid + u * kFzThreads;
+    hv[u] = -1;
+    ha[u] = 0.f;
+    if (k < s_ci.y) {  // step > 0 (the list of a finished row is loaded but not used)
+      hv[u] = __ldcg(d.c_lab + (size_t)r * d.V4 + k);
+      ha[u] = __ldcg(d.c_add + (size_t)r * d.V4 + k);
+    }
+  }
   // the chains are read whole (their arrays have room for the longest), so
   // their lengths need not be known first
   if (tid == 0) {
@@ -173,6 +200,7 @@ __global__ void __launch_bounds__(kFzThreads) __maxnreg__((VAR & 4) ? 128 : 72) 
       ok = checked(s_tr[k] > 0 && s_tr[k] < d.tr.n_nodes, d.err, 7) &&
            checked(c.x >= 0 && c.y >= 0 && c.x + c.y <= d.tr.n_children && c.z >= 1 && c.z <= 63, d.err, 8);
     }
+    if (ok && step > 0 && s_t < T) ok = checked(s_ci.y >= 0 && s_ci.y <= d.V4, d.err, 12);
     s_bad = !ok;
   }
   row::block_sync();
@@ -191,243 +219,28 @@ __global__ void __launch_bounds__(kFzThreads) __maxnreg__((VAR & 4) ? 128 : 72) 
   const float lam = s_lam;
   const float bscale = s_beta * (d.has_tr ? d.tr.bonus : 0.f);
 
-  if (evaluated) {
-    if (tid == 0) {
-      // arc groups of the levels above level 0 (level 0 is streamed apart)
-      int g = 0;
-      unsigned long long ab = 0;
-      for (int l = 0; l < nl_old; ++l) {
-        s_gbeg[l] = g;
-        if (l > 0) g += level_groups(s_lmr[l].x, s_lmr[l].y);
-        ab += 16 + 8ull * s_lmr[l].y;
-      }
-      s_gbeg[nl_old] = g;
-      for (int k = 0; k < nt_old; ++k) ab += 16 + 4ull * s_trr[k].y;
-      const float cum_top = nl_old ? __int_as_float(s_lmr[nl_old - 1].z) : 0.f;
-      const int depth_cur = nt_old ? s_trr[0].z - 1 : 0;
-      s_cr = lam * cum_top - bscale * (float)depth_cur;
-      // Algorithmic bytes (when counting): the row's logits and partials
-      // read, the row state read and written, every arc of every LM chain
-      // level (label + log-probability) and every child of every trie chain
-      // node (label) with its record; searches and the joint input are added
-      // where they happen; the call's shared rows once per launch by the host.
-      s_bytes = ab + 4ull * (V + 1) + 16ull * d.n_ptiles + 2ull * (24 + 4 * (nl_old + nt_old));
-    }
-    row::block_sync();
-    const int4* t4 = reinterpret_cast<const int4*>(d.lm.arc_tok);
-    const float4* p4 = reinterpret_cast<const float4*>(d.lm.arc_logp);
-    // the group g of the levels above 0: its level and first arc
-    auto locate = [&](int g, int& l) {
-      l = 1;
-      while (g >= s_gbeg[l + 1]) ++l;
-      return (s_lmr[l].x & ~3) + 4 * (g - s_gbeg[l]);
-    };
-    // 1a. the levels above 0 (few arcs: they continue longer contexts) offer
-    //     ((l + 1) << 24 | position) to their labels by atomicMax, so the
-    //     deepest wins; their labels and log-probabilities stay in registers
-    const int G = s_gbeg[nl_old];
-    int4 ht[kHeld];
-    float4 hp[kHeld];
-    int hl[kHeld], hi[kHeld];
-#pragma unroll
-    for (int u = 0; u < kHeld; ++u) {
-      const int g = tid + u * kFzThreads;
-      hl[u] = -1;
-      hi[u] = 0;
-      if (g < G) {
-        int l;
-        hi[u] = locate(g, l);
-        ht[u] = __ldg(t4 + (hi[u] >> 2));
-        hp[u] = __ldg(p4 + (hi[u] >> 2));
-        hl[u] = l;
-      }
-    }
-    auto offer = [&](int l, int i0, int4 tk) {
-      const int b = s_lmr[l].x, c = s_lmr[l].y;
-      const uint32_t tag = (uint32_t)(l + 1) << 24;
-      const int tv[4] = {tk.x, tk.y, tk.z, tk.w};
-#pragma unroll
-      for (int j = 0; j < 4; ++j)
-        if (i0 + j >= b && i0 + j < b + c && checked(tv[j] >= 0 && tv[j] < V, d.err, 9))
-          atomicMax(key + tv[j], tag | (uint32_t)(i0 + j - b));
-    };
-#pragma unroll
-    for (int u = 0; u < kHeld; ++u)
-      if (hl[u] >= 0) offer(hl[u], hi[u], ht[u]);
-    for (int g = tid + kHeld * kFzThreads; g < G; g += kFzThreads) {  // past what registers hold
-      int l;
-      const int i0 = locate(g, l);
-      offer(l, i0, __ldg(t4 + (i0 >> 2)));
-    }
-    if (nt_old > 0) {
-      const int k = nt_old - 1;
-      row::scatter_trie_node(d.tr.ch_tok, s_trr[k].x, s_trr[k].x + s_trr[k].y, (uint8_t)s_trr[k].z, dep);
-    }
-    row::block_sync();
-    // 1b. level 0 (the previous label's continuations, up to all V labels)
-    //     streamed once, labels and log-probabilities together: its arc is
-    //     the deepest for v exactly when no level above offered v (their
-    //     labels are a subset of level 0's), and then it writes v's delta at
-    //     once -- no level above ever looks at such a label.  The levels
-    //     above judge their offers meanwhile.
-    auto delta_of = [&](int l, float lp, int v) {
-      return lam * (lp - __int_as_float(s_lmr[l].z)) - lam * __ldg(d.lm.uni_logp + v);
-    };
-    if (nl_old > 0 && s_lmr[0].w >= 0) {
-      // a dense row: per label log p(v | u) - log p(v) or NaN, contiguous
-      const float4* R = reinterpret_cast<const float4*>(d.lm.dense0 + (size_t)s_lmr[0].w * d.lm.V4);
-      const float cum0 = __int_as_float(s_lmr[0].z);
-      const int nq4 = d.lm.V4 / 4;
-      for (int q0 = tid; q0 < nq4; q0 += kDense * kFzThreads) {
-        float4 rq[kDense];
-#pragma unroll
-        for (int u = 0; u < kDense; ++u) {
-          const int q = q0 + u * kFzThreads;
-          if (q < nq4) rq[u] = __ldg(R + q);
-        }
-#pragma unroll
-        for (int u = 0; u < kDense; ++u) {
-          const int q = q0 + u * kFzThreads;
-          if (q < nq4) {
-            const uint4 kq = reinterpret_cast<const uint4*>(key)[q];
-            const float rv[4] = {rq[u].x, rq[u].y, rq[u].z, rq[u].w};
-            const uint32_t kv[4] = {kq.x, kq.y, kq.z, kq.w};
-#pragma unroll
-            for (int j = 0; j < 4; ++j)
-              if (!isnan(rv[j]) && kv[j] == 0u) {
-                key[4 * q + j] = __float_as_uint(lam * (rv[j] - cum0));
-                lmf[4 * q + j] = 1;
-              }
-          }
-        }
-      }
-    } else if (nl_old > 0) {
-      const int b0 = s_lmr[0].x, c0 = s_lmr[0].y;
-      const int a0 = b0 & ~3, G0 = level_groups(b0, c0);
-      for (int gb = 0; gb < G0; gb += kStream * kFzThreads) {
-        int4 tk[kStream];
-        float4 lp[kStream];
-#pragma unroll
-        for (int u = 0; u < kStream; ++u) {
-          const int g = gb + u * kFzThreads + tid;
-          if (g < G0) {
-            tk[u] = __ldg(t4 + (a0 >> 2) + g);
-            lp[u] = __ldg(p4 + (a0 >> 2) + g);
-          }
-        }
-#pragma unroll
-        for (int u = 0; u < kStream; ++u) {
-          const int g = gb + u * kFzThreads + tid;
-          if (g < G0) {
-            const int i0 = a0 + 4 * g;
-            const int tv[4] = {tk[u].x, tk[u].y, tk[u].z, tk[u].w};
-            const float pv[4] = {lp[u].x, lp[u].y, lp[u].z, lp[u].w};
-#pragma unroll
-            for (int j = 0; j < 4; ++j)
-              if (i0 + j >= b0 && i0 + j < b0 + c0 && checked(tv[j] >= 0 && tv[j] < V, d.err, 9) &&
-                  key[tv[j]] == 0u) {
-                key[tv[j]] = __float_as_uint(delta_of(0, pv[j], tv[j]));
-                lmf[tv[j]] = 1;
-              }
-          }
-        }
-      }
-    }
-    // the winners among the offers (one per label), deltas kept until every
-    // offer is judged
-    uint32_t won = 0;  // bit 4u + j: arc j of held group u won
-    float wv[kHeld][4];
-#pragma unroll
-    for (int u = 0; u < kHeld; ++u) {
-      if (hl[u] >= 0) {
-        const int l = hl[u], b = s_lmr[l].x, c = s_lmr[l].y;
-        const uint32_t tag = (uint32_t)(l + 1) << 24;
-        const int tv[4] = {ht[u].x, ht[u].y, ht[u].z, ht[u].w};
-        const float pv[4] = {hp[u].x, hp[u].y, hp[u].z, hp[u].w};
-#pragma unroll
-        for (int j = 0; j < 4; ++j) {
-          const int i = hi[u] + j;
-          wv[u][j] = 0.f;
-          if (i >= b && i < b + c && checked(tv[j] >= 0 && tv[j] < V, d.err, 9) &&
-              key[tv[j]] == (tag | (uint32_t)(i - b))) {
-            won |= 1u << (4 * u + j);
-            wv[u][j] = delta_of(l, pv[j], tv[j]);
-          }
-        }
-      }
-    }
-    if (nt_old > 1) {
-      const int k = nt_old - 2;
-      row::scatter_trie_node(d.tr.ch_tok, s_trr[k].x, s_trr[k].x + s_trr[k].y, (uint8_t)s_trr[k].z, dep);
-    }
-    row::block_sync();
-#pragma unroll
-    for (int u = 0; u < kHeld; ++u) {
-      const int tv[4] = {ht[u].x, ht[u].y, ht[u].z, ht[u].w};
-#pragma unroll
-      for (int j = 0; j < 4; ++j)
-        if ((won >> (4 * u + j)) & 1u) {
-          key[tv[j]] = __float_as_uint(wv[u][j]);
-          lmf[tv[j]] = 1;
-        }
-    }
-    // offers past what registers hold (rows whose longer contexts have very
-    // many continuations): judged a round at a time, a barrier between the
-    // judging and the writing; a label already written is skipped by its flag
-    for (int g0 = kHeld * kFzThreads; g0 < G; g0 += kFzThreads) {
-      row::block_sync();
-      const int g = g0 + tid;
-      int4 tk = make_int4(0, 0, 0, 0);
-      float xv[4] = {0.f, 0.f, 0.f, 0.f};
-      uint32_t xw = 0;
-      if (g < G) {
-        int l;
-        const int i0 = locate(g, l);
-        tk = __ldg(t4 + (i0 >> 2));
-        const float4 lq = __ldg(p4 + (i0 >> 2));
-        const int b = s_lmr[l].x, c = s_lmr[l].y;
-        const uint32_t tag = (uint32_t)(l + 1) << 24;
-        const int tv[4] = {tk.x, tk.y, tk.z, tk.w};
-        const float pv[4] = {lq.x, lq.y, lq.z, lq.w};
-#pragma unroll
-        for (int j = 0; j < 4; ++j)
-          if (i0 + j >= b && i0 + j < b + c && checked(tv[j] >= 0 && tv[j] < V, d.err, 9) && lmf[tv[j]] == 0 &&
-              key[tv[j]] == (tag | (uint32_t)(i0 + j - b))) {
-            xw |= 1u << j;
-            xv[j] = delta_of(l, pv[j], tv[j]);
-          }
-      }
-      row::block_sync();
-      const int tv[4] = {tk.x, tk.y, tk.z, tk.w};
-#pragma unroll
-      for (int j = 0; j < 4; ++j)
-        if ((xw >> j) & 1u) {
-          key[tv[j]] = __float_as_uint(xv[j]);
-          lmf[tv[j]] = 1;
-        }
-    }
-    for (int k = nt_old - 3; k >= 0; --k) {
-      row::block_sync();
-      row::scatter_trie_node(d.tr.ch_tok, s_trr[k].x, s_trr[k].x + s_trr[k].y, (uint8_t)s_trr[k].z, dep);
-    }
-    row::block_sync();
-  }
   // Programmatic dependent launch: everything above reads only state the
   // previous row pass wrote (complete before the joint kernel in between let
-  // this grid launch) and constant tables; the logits need the wait.
+  // this grid launch) and constant tables; the partials and logits need the
+  // wait.
   asm volatile("griddepcontrol.wait;" ::: "memory");
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
   if (evaluated) {
-    // 2. log-sum-exp (warp 0, from the tile partials) and the argmax of
-    //    logit + D + c_r + delta over the labels; blank takes its logit
+    // 2. the decision: the log-sum-exp and the best unlisted label from the
+    //    tile partials (warp 0), every listed label from its stored logit
     const float* lg = d.logits + (size_t)r * d.N_pad;
+    const int4 ci = s_ci;
+    const float cr_prev = __int_as_float(ci.z);
+    float bv = kNegInf;
+    int bi = INT_MAX;
     if (warp == 0) {
       float m = kNegInf, s = 0.f;
       const float4* pr = d.part + (size_t)r * d.n_ptiles;
       for (int j = lane; j < d.n_ptiles; j += 32) {
         const float4 p = __ldcg(pr + j);  // written by the joint kernel just before
         lse_merge(m, s, p.x, p.y);
+        best_merge(bv, bi, p.z, __float_as_int(p.w));
       }
       row::reconverge();
       for (int o = 16; o > 0; o >>= 1) {
@@ -437,52 +250,41 @@ __global__ void __launch_bounds__(kFzThreads) __maxnreg__((VAR & 4) ? 128 : 72) 
       }
       if (lane == 0) s_lse = m + logf(s);
     }
-    float bv = kNegInf;
-    int bi = INT_MAX;
     {
-      const float cr = s_cr;
-      const int nq = (V + 3) >> 2;  // quads holding labels < V
-      const float4* l4 = reinterpret_cast<const float4*>(lg);
-      const uint4* k4 = reinterpret_cast<const uint4*>(key);
-      const uint32_t* f4 = reinterpret_cast<const uint32_t*>(lmf);
-      const uint32_t* e4 = reinterpret_cast<const uint32_t*>(dep);
-      for (int q0 = tid; q0 < nq; q0 += QB * kFzThreads) {
-        float4 lq[QB];
+      float x[kListHeld];
 #pragma unroll
-        for (int u = 0; u < QB; ++u) {
-          const int q = q0 + u * kFzThreads;
-          if (q < nq) lq[u] = __ldcg(l4 + q);
-        }
+      for (int u = 0; u < kListHeld; ++u)
+        if (hv[u] >= 0 && checked(hv[u] < V, d.err, 13)) x[u] = __ldcg(lg + hv[u]);
 #pragma unroll
-        for (int u = 0; u < QB; ++u) {
-          const int q = q0 + u * kFzThreads;
-          if (q < nq) {
-            const uint32_t fq = f4[q], eq = e4[q];
-            const float lv[4] = {lq[u].x, lq[u].y, lq[u].z, lq[u].w};
-            float dl[4] = {0.f, 0.f, 0.f, 0.f};
-            if (fq | eq) {  // a label of this quad has an LM or trie delta
-              const uint4 kq = k4[q];
-              const uint32_t kv[4] = {kq.x, kq.y, kq.z, kq.w};
-              const uint32_t rb = __ldg(d.droot + (q >> 3)) >> ((4 * q) & 31);
+      for (int u = 0; u < kListHeld; ++u)
+        if (hv[u] >= 0 && hv[u] < V) best_merge(bv, bi, x[u] + ha[u], hv[u]);
+      const int32_t* cl = d.c_lab + (size_t)r * d.V4;
+      const float* ca = d.c_add + (size_t)r * d.V4;
+      for (int k0 = tid + kListHeld * kFzThreads; k0 < ci.y; k0 += 4 * kFzThreads) {
+        int v[4];
+        float a[4], x[4];
 #pragma unroll
-              for (int j = 0; j < 4; ++j) {
-                if ((fq >> (8 * j)) & 0xffu) dl[j] = __uint_as_float(kv[j]);
-                const uint32_t e = (eq >> (8 * j)) & 0xffu;
-                if (e) dl[j] += bscale * (float)e - (((rb >> j) & 1u) ? bscale : 0.f);
-              }
-            }
-#pragma unroll
-            for (int j = 0; j < 4; ++j) {
-              const float fv = lv[j] + (cr + dl[j]);
-              if (4 * q + j < V && fv > bv) { bv = fv; bi = 4 * q + j; }
-            }
+        for (int u = 0; u < 4; ++u) {
+          const int k = k0 + u * kFzThreads;
+          v[u] = -1;
+          a[u] = 0.f;
+          x[u] = kNegInf;
+          if (k < ci.y) {
+            v[u] = __ldcg(cl + k);
+            a[u] = __ldcg(ca + k);
           }
         }
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+          if (v[u] >= 0 && checked(v[u] < V, d.err, 13)) x[u] = __ldcg(lg + v[u]);
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+          if (v[u] >= 0 && v[u] < V) best_merge(bv, bi, x[u] + a[u], v[u]);
       }
-      if (tid == 0) {
-        const float fb = __ldcg(lg + V);  // blank: D[V] = 0, no fusion terms
-        if (fb > bv) { bv = fb; bi = V; }
-      }
+    }
+    if (tid == 0) {
+      const float fb = __ldcg(lg + V) - cr_prev;  // blank: no fusion terms
+      if (fb > bv) { bv = fb; bi = V; }
     }
     row::reconverge();
     for (int o = 16; o > 0; o >>= 1) {
@@ -501,7 +303,15 @@ __global__ void __launch_bounds__(kFzThreads) __maxnreg__((VAR & 4) ? 128 : 72) 
 #pragma unroll
       for (int w = 1; w < kFzWarps; ++w) best_merge(b, i, s_bv[w], s_bi[w]);
       s_y = (i >= 0 && i <= V) ? i : V;
-      s_score = b - s_lse;
+      s_score = (b + cr_prev) - s_lse;
+      if (counting) {
+        // algorithmic bytes of the decision: partials, the list and its
+        // logits, blank's logit, the row state read and written, the chain
+        // records read
+        unsigned long long ab = 16ull * d.n_ptiles + 12ull * ci.y + 4 + 16;
+        ab += 2ull * (24 + 4 * (nl_old + nt_old)) + 16ull * (nl_old + nt_old);
+        s_bytes = ab;
+      }
     }
     row::block_sync();
     const int y = s_y;
@@ -529,57 +339,78 @@ __global__ void __launch_bounds__(kFzThreads) __maxnreg__((VAR & 4) ? 128 : 72) 
         }
       }
       row::block_sync();
-      // 3b. assemble the new chains in place (shared memory) and emit
-      if (tid == 0) {
-        // LM: y's unigram state, then the target of y's arc at every level
-        // of the old chain up to the first level without one
+      // 3b. assemble the new chains in place (shared memory) and commit them:
+      //     warp 0 the LM chain (y's unigram state, then the targets of y's
+      //     arcs at the old levels up to the first level without one), warp 1
+      //     the trie chain (y's children of the old chain nodes, deepest
+      //     first, then the root's; a completed phrase resets it), warp 2
+      //     the outputs
+      if (warp == 0) {
         int ln = 0;
-        const int4 u = s_uni_hit;
         if (d.has_lm && d.lm.order >= 2) {
-          s_lm[0] = 1 + y;  // the unigram state of y; u.x is its dense row
-          s_lmr[0] = make_int4(u.y, u.z, u.w, u.x);
-          ln = 1;
-          for (int l = 0; l < nl_old && ln < kLmChain; ++l) {
-            const int4 h = s_lm_hit[l];
-            if (h.x < 0) break;  // no arc at this level (-2) or the top order (-1)
-            if (!checked(h.x < d.lm.n_states && h.y >= 0 && h.z >= 0 && (int64_t)h.y + h.z <= d.lm.n_arcs, d.err, 10))
-              break;
-            s_lm[ln] = h.x;
-            s_lmr[ln] = make_int4(h.y, h.z, h.w, 0);
-            ++ln;
+          const int4 h = lane < nl_old ? s_lm_hit[lane] : make_int4(-2, 0, 0, 0);
+          const bool cont =
+              h.x >= 0 && checked(h.x < d.lm.n_states && h.y >= 0 && h.z >= 0 && (int64_t)h.y + h.z <= d.lm.n_arcs,
+                                  d.err, 10);
+          const unsigned miss = __ballot_sync(0xffffffffu, !cont);
+          ln = 1 + min(miss ? __ffs((int)miss) - 1 : 32, kLmChain - 1);
+          const int4 u = s_uni_hit;
+          const int st = lane == 0 ? 1 + y : h.x;  // new level `lane`: y's unigram state, then targets
+          const int4 rec = lane == 0 ? make_int4(u.y, u.z, u.w, u.x) : make_int4(0, 0, 0, 0);
+          // lane l >= 1 takes the hit of old level l - 1
+          const int px = __shfl_up_sync(0xffffffffu, h.x, 1), py = __shfl_up_sync(0xffffffffu, h.y, 1);
+          const int pz = __shfl_up_sync(0xffffffffu, h.z, 1), pw = __shfl_up_sync(0xffffffffu, h.w, 1);
+          const int4 nrec = lane == 0 ? rec : make_int4(py, pz, pw, 0);
+          const int nst = lane == 0 ? st : px;
+          __syncwarp();
+          if (lane < ln) {
+            s_lm[lane] = nst;
+            s_lmr[lane] = nrec;
+            if (commit) {
+              d.s_lm_chain[(size_t)slot * kLmChain + lane] = nst;
+              d.s_lm_rec[(size_t)slot * kLmChain + lane] = nrec;
+            }
           }
         }
-        s_nl = ln;
-        // trie: y's children of the old chain nodes (deepest first), then the
-        // root's; completing a phrase (the deepest match's next is 0) resets
-        int tn = 0;
-        bool reset = false;
-        for (int i = 0; i < nt_old; ++i) {
-          const int4 h = s_tr_hit[i];
-          if (h.x < 0) continue;
-          if (!checked(h.x > 0 && h.x < d.tr.n_nodes && h.w >= 0 && h.z + h.w <= d.tr.n_children, d.err, 11)) continue;
-          if (tn == 0 && h.y == 0) reset = true;
-          const int dd = s_trr[i].z + 1;  // the child's children sit one deeper
-          if (tn < kTrChain) {
-            s_tr[tn] = h.x;
-            s_trr[tn] = make_int4(h.z, h.w, dd, 0);
-            ++tn;
-          }
+        if (lane == 0) {
+          s_nl = ln;
+          if (commit && d.has_lm) d.s_lm_len[slot] = ln;
         }
+      } else if (warp == 1) {
+        const int4 h = lane < nt_old ? s_tr_hit[lane] : make_int4(-1, 0, 0, 0);
+        const int dd = lane < nt_old ? s_trr[lane].z + 1 : 0;  // the child's children sit one deeper
+        const bool ok = h.x >= 0 && checked(h.x > 0 && h.x < d.tr.n_nodes && h.w >= 0 && h.z + h.w <= d.tr.n_children,
+                                            d.err, 11);
+        const unsigned vm = __ballot_sync(0xffffffffu, ok);
+        const int nv = __popc(vm);
         const int4 rh = s_root_hit;
-        if (rh.x != 0) {
-          if (tn == 0 && rh.y == 0) reset = true;
-          if (tn < kTrChain) {
-            s_tr[tn] = rh.x;
-            s_trr[tn] = make_int4(rh.z, rh.w, 2, 0);
-            ++tn;
-          }
+        const bool root = rh.x != 0;
+        // the first element of the new chain ends a phrase: the chain resets
+        const int f = __ffs((int)vm) - 1;
+        const int fy = __shfl_sync(0xffffffffu, h.y, f < 0 ? 0 : f);
+        const bool reset = nv > 0 ? fy == 0 : (root && rh.y == 0);
+        const int tn = reset ? 0 : min(nv + (root ? 1 : 0), kTrChain);
+        __syncwarp();
+        const int pos = __popc(vm & ((1u << lane) - 1u));
+        if (ok && pos < tn) {
+          s_tr[pos] = h.x;
+          s_trr[pos] = make_int4(h.z, h.w, dd, 0);
         }
-        if (reset) tn = 0;
-        s_nt = tn;
+        if (lane == 0 && root && nv < tn) {
+          s_tr[nv] = rh.x;
+          s_trr[nv] = make_int4(rh.z, rh.w, 2, 0);
+        }
+        __syncwarp();
+        if (commit && lane < tn) {
+          d.s_tr_chain[slot * kTrChain + lane] = s_tr[lane];
+          d.s_tr_rec[(size_t)slot * kTrChain + lane] = s_trr[lane];
+        }
+        if (lane == 0) {
+          s_nt = tn;
+          if (commit && d.has_tr) d.s_tr_len[slot] = tn;
+        }
+      } else if (tid == 64) {
         if (commit) {
-          if (d.has_lm) d.s_lm_len[slot] = ln;
-          if (d.has_tr) d.s_tr_len[slot] = tn;
           const int cap = T * d.max_sym;
           const int o = r * cap + s_cnt;
           s_out_tok[o] = y;
@@ -591,18 +422,6 @@ __global__ void __launch_bounds__(kFzThreads) __maxnreg__((VAR & 4) ? 128 : 72) 
         s_last = y;
         s_sym += 1;
         if (s_sym >= d.max_sym) { s_t += 1; s_sym = 0; }
-      }
-      row::block_sync();
-      if (commit) {  // the new chains and their records, for the next step
-        if (tid < s_nl) {
-          d.s_lm_chain[(size_t)slot * kLmChain + tid] = s_lm[tid];
-          d.s_lm_rec[(size_t)slot * kLmChain + tid] = s_lmr[tid];
-        }
-        if (tid >= 64 && tid - 64 < s_nt) {
-          const int k = tid - 64;
-          d.s_tr_chain[slot * kTrChain + k] = s_tr[k];
-          d.s_tr_rec[(size_t)slot * kTrChain + k] = s_trr[k];
-        }
       }
     } else if (tid == 0) {
       s_t += 1;
@@ -630,8 +449,8 @@ __global__ void __launch_bounds__(kFzThreads) __maxnreg__((VAR & 4) ? 128 : 72) 
       for (int i = tid; i < D / 4; i += blockDim.x) dst[i] = (i < D / 8) ? __ldg(src_x + i) : __ldcg(src_h + i - D / 8);
     }
   }
-  if (counting && tid == 0 && evaluated) atomicAdd(d.ctr, s_bytes);
   if (mode == 1) {
+    if (counting && tid == 0 && evaluated) atomicAdd(d.ctr, s_bytes);
     if (tid == 0) s_out_count[r] = s_cnt;
     return;
   }
@@ -653,20 +472,226 @@ __global__ void __launch_bounds__(kFzThreads) __maxnreg__((VAR & 4) ? 128 : 72) 
       c[0] = -1; c[1] = -1; c[2] = -1; c[3] = -1;
     }
   }
-  if (t >= T) return;
+  if (t >= T) {  // no joint input this step: the row's list is not read
+    if (counting && tid == 0 && evaluated) atomicAdd(d.ctr, s_bytes);
+    return;
+  }
 
-  // 4. joint input of this step
+  // 4. the correction list of the row's (new) state, for the joint kernel
+  //    of this step and the decision of the next.  Warp 0: the arc groups
+  //    of levels 1.. before each level (a prefix sum over its lanes), c_r
+  if (warp == 0) {
+    const int l = lane + 1;
+    const int4 rc = l < nl ? s_lmr[l] : make_int4(0, 0, 0, 0);
+    const int g = l < nl ? level_groups(rc.x, rc.y) : 0;
+    int incl = g;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int v = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += v;
+    }
+    if (l <= max(nl, 1)) s_gbeg[l] = incl - g;
+    if (counting) {  // every arc of levels 1.. (label + log-probability), every child label of the trie chain
+      unsigned long long ab = (l < nl ? 8ull * rc.y : 0ull) + (lane < nt ? 4ull * s_trr[lane].y : 0ull);
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) ab += __shfl_xor_sync(0xffffffffu, ab, o);
+      if (lane == 0) s_bytes += ab;
+    }
+    if (lane == 0) {
+      const float cum_top = nl ? __int_as_float(s_lmr[nl - 1].z) : 0.f;
+      const int depth_cur = nt ? s_trr[0].z - 1 : 0;
+      s_cr = lam * cum_top - bscale * (float)depth_cur;
+    }
+  }
+  row::block_sync();
+  const int4* t4 = reinterpret_cast<const int4*>(d.lm.arc_tok);
+  const float4* p4 = reinterpret_cast<const float4*>(d.lm.arc_logp);
+  // the group g of levels 1..: its level and first arc
+  auto locate = [&](int g, int& l) {
+    l = 1;
+    while (g >= s_gbeg[l + 1]) ++l;
+    return (s_lmr[l].x & ~3) + 4 * (g - s_gbeg[l]);
+  };
+  auto lm_term = [&](int l, float lp) { return lam * (lp - __int_as_float(s_lmr[l].z)); };
+  // 4a. levels 1.. offer ((l + 1) << 24 | position) to their labels, so the
+  //     deepest wins; the trie chain nodes scatter their goto depths,
+  //     shallowest first (the deepest overwrites), one node per phase
+  const int G = nl >= 2 ? s_gbeg[nl] : 0;
+  int4 ht[kHeld];
+  float4 hp[kHeld];
+  int hl[kHeld], hi[kHeld];
+#pragma unroll
+  for (int u = 0; u < kHeld; ++u) {
+    const int g = tid + u * kFzThreads;
+    hl[u] = -1;
+    hi[u] = 0;
+    ht[u] = make_int4(0, 0, 0, 0);
+    hp[u] = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (g < G) {
+      int l;
+      hi[u] = locate(g, l);
+      ht[u] = __ldg(t4 + (hi[u] >> 2));
+      hp[u] = __ldg(p4 + (hi[u] >> 2));
+      hl[u] = l;
+    }
+  }
+  auto offer = [&](int l, int i0, int4 tk) {
+    const int b = s_lmr[l].x, c = s_lmr[l].y;
+    const uint32_t tag = (uint32_t)(l + 1) << 24;
+    const int tv[4] = {tk.x, tk.y, tk.z, tk.w};
+#pragma unroll
+    for (int j = 0; j < 4; ++j)
+      if (i0 + j >= b && i0 + j < b + c && checked(tv[j] >= 0 && tv[j] < V, d.err, 9))
+        atomicMax(key + tv[j], tag | (uint32_t)(i0 + j - b));
+  };
+#pragma unroll
+  for (int u = 0; u < kHeld; ++u)
+    if (hl[u] >= 0) offer(hl[u], hi[u], ht[u]);
+  for (int g = tid + kHeld * kFzThreads; g < G; g += kFzThreads) {  // past what registers hold
+    int l;
+    const int i0 = locate(g, l);
+    offer(l, i0, __ldg(t4 + (i0 >> 2)));
+  }
+  if (nt > 0) {
+    const int k = nt - 1;
+    row::scatter_trie_node(d.tr.ch_tok, s_trr[k].x, s_trr[k].x + s_trr[k].y, (uint8_t)s_trr[k].z, dep);
+  }
+  row::block_sync();
+  // 4b. the winners among the held offers (one per label) compute their LM
+  //     term; it is written once every offer is judged
+  uint32_t won = 0;  // bit 4u + j: arc j of held group u won
+  float wv[kHeld][4];
+#pragma unroll
+  for (int u = 0; u < kHeld; ++u) {
+    const int tv[4] = {ht[u].x, ht[u].y, ht[u].z, ht[u].w};
+    const float pv[4] = {hp[u].x, hp[u].y, hp[u].z, hp[u].w};
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      wv[u][j] = 0.f;
+      if (hl[u] >= 0) {
+        const int l = hl[u], b = s_lmr[l].x, c = s_lmr[l].y;
+        const int i = hi[u] + j;
+        if (i >= b && i < b + c && checked(tv[j] >= 0 && tv[j] < V, d.err, 9) &&
+            key[tv[j]] == (((uint32_t)(l + 1) << 24) | (uint32_t)(i - b))) {
+          won |= 1u << (4 * u + j);
+          wv[u][j] = lm_term(l, pv[j]);
+        }
+      }
+    }
+  }
+  if (nt > 1) {
+    const int k = nt - 2;
+    row::scatter_trie_node(d.tr.ch_tok, s_trr[k].x, s_trr[k].x + s_trr[k].y, (uint8_t)s_trr[k].z, dep);
+  }
+  row::block_sync();
+#pragma unroll
+  for (int u = 0; u < kHeld; ++u) {
+    const int tv[4] = {ht[u].x, ht[u].y, ht[u].z, ht[u].w};
+#pragma unroll
+    for (int j = 0; j < 4; ++j)
+      if ((won >> (4 * u + j)) & 1u) {
+        key[tv[j]] = __float_as_uint(wv[u][j]);
+        lmf[tv[j]] = 1;
+      }
+  }
+  // offers past what registers hold (states with very many continuations):
+  // judged a round at a time, a barrier between the judging and the
+  // writing; a label already written is skipped by its flag
+  for (int g0 = kHeld * kFzThreads; g0 < G; g0 += kFzThreads) {
+    row::block_sync();
+    const int g = g0 + tid;
+    int4 tk = make_int4(0, 0, 0, 0);
+    float xv[4] = {0.f, 0.f, 0.f, 0.f};
+    uint32_t xw = 0;
+    if (g < G) {
+      int l;
+      const int i0 = locate(g, l);
+      tk = __ldg(t4 + (i0 >> 2));
+      const float4 lq = __ldg(p4 + (i0 >> 2));
+      const int b = s_lmr[l].x, c = s_lmr[l].y;
+      const uint32_t tag = (uint32_t)(l + 1) << 24;
+      const int tv[4] = {tk.x, tk.y, tk.z, tk.w};
+      const float pv[4] = {lq.x, lq.y, lq.z, lq.w};
+#pragma unroll
+      for (int j = 0; j < 4; ++j)
+        if (i0 + j >= b && i0 + j < b + c && checked(tv[j] >= 0 && tv[j] < V, d.err, 9) && lmf[tv[j]] == 0 &&
+            key[tv[j]] == (tag | (uint32_t)(i0 + j - b))) {
+          xw |= 1u << j;
+          xv[j] = lm_term(l, pv[j]);
+        }
+    }
+    row::block_sync();
+    const int tv[4] = {tk.x, tk.y, tk.z, tk.w};
+#pragma unroll
+    for (int j = 0; j < 4; ++j)
+      if ((xw >> j) & 1u) {
+        key[tv[j]] = __float_as_uint(xv[j]);
+        lmf[tv[j]] = 1;
+      }
+  }
+  for (int k = nt - 3; k >= 0; --k) {
+    row::block_sync();
+    row::scatter_trie_node(d.tr.ch_tok, s_trr[k].x, s_trr[k].x + s_trr[k].y, (uint8_t)s_trr[k].z, dep);
+  }
+  row::block_sync();
+  // 4c. the list: level 1's arcs in order (every label of a deeper level is
+  //     one of them), then the trie chain's children that are not
+  {
+    int32_t* cl = d.c_lab + (size_t)r * d.V4;
+    float* ca = d.c_add + (size_t)r * d.V4;
+    const int b1 = nl >= 2 ? s_lmr[1].x : 0, c1 = nl >= 2 ? s_lmr[1].y : 0;
+    for (int j = tid; j < c1; j += kFzThreads) {
+      const int v = __ldg(d.lm.arc_tok + b1 + j);
+      if (!checked(v >= 0 && v < V && lmf[v] != 0, d.err, 14)) continue;
+      const uint32_t e = dep[v];
+      const float tr = e ? bscale * (float)e : (((__ldg(d.droot + (v >> 5)) >> (v & 31)) & 1u) ? bscale : 0.f);
+      cl[j] = v;
+      ca[j] = __uint_as_float(key[v]) + tr;
+      atomicOr(msk + (v >> 5), 1u << (v & 31));
+    }
+    const int drow = (d.has_lm && nl >= 1) ? s_lmr[0].w : -1;
+    const float* dense = drow >= 0 ? d.lm.dense0 + (size_t)drow * d.V4 : nullptr;
+    for (int k = 0; k < nt; ++k) {
+      const int b = s_trr[k].x, c = s_trr[k].y;
+      const uint32_t dd = (uint32_t)s_trr[k].z;
+      for (int i = tid; i < c; i += kFzThreads) {
+        const int v = __ldg(d.tr.ch_tok + b + i);
+        if (!checked(v >= 0 && v < V, d.err, 15) || dep[v] != dd || lmf[v] != 0) continue;
+        float lmv = 0.f;  // the LM term when the deepest arc is level 0's, or none
+        if (d.has_lm) lmv = lam * ((dense ? __ldg(dense + v) : 0.f) + __ldg(d.lm.uni_logp + v));
+        const int j = c1 + atomicAdd(&s_ext, 1);
+        cl[j] = v;
+        ca[j] = lmv + bscale * (float)dd;
+        atomicOr(msk + (v >> 5), 1u << (v & 31));
+      }
+    }
+    if (tid == 0) atomicOr(msk + (V >> 5), 1u << (V & 31));  // blank is always evaluated by the row pass
+    row::block_sync();
+    uint32_t* mo = d.c_mask + (size_t)r * d.mask_words;
+    for (int q = tid; q < d.mask_words; q += kFzThreads) mo[q] = msk[q];
+    if (tid == 0) {
+      const int n = c1 + s_ext;
+      d.c_info[r] = make_int4(drow, n, __float_as_int(s_cr), 0);
+      if (counting) s_bytes += 8ull * n + 4ull * d.mask_words + 16 + 8ull * s_ext;
+    }
+  }
+
+  // 5. joint input of this step
   if (!PRED) row::build_joint_input(d, s_enc + ((size_t)r * T + t) * d.H, s_last, r);
-  if (counting && tid == 0 && !PRED) atomicAdd(d.ctr, 6ull * d.H);  // encoder frame, embedding row, A row
+  if (counting && tid == 0) atomicAdd(d.ctr, s_bytes + (PRED ? 0ull : 6ull * d.H));  // + frame, embedding row, A row
 }
 
 }  // namespace
 
+size_t row_fused_smem_bytes(int V4, int N_pad) {
+  return (size_t)V4 * (sizeof(uint32_t) + 2 * sizeof(uint8_t)) + sizeof(uint32_t) * (size_t)(N_pad / 32);
+}
+
 cudaError_t prepare_fused_kernels(size_t smem) {
-  cudaError_t e = cudaFuncSetAttribute(k_row_fz<0>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-  if (e == cudaSuccess) e = cudaFuncSetAttribute(k_row_fz<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-  if (e == cudaSuccess) e = cudaFuncSetAttribute(k_row_fz<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-  if (e == cudaSuccess) e = cudaFuncSetAttribute(k_row_fz<5>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  cudaError_t e = cudaFuncSetAttribute(k_row_ep<0>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e == cudaSuccess) e = cudaFuncSetAttribute(k_row_ep<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e == cudaSuccess) e = cudaFuncSetAttribute(k_row_ep<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e == cudaSuccess) e = cudaFuncSetAttribute(k_row_ep<5>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   return e;
 }
 
@@ -683,11 +708,11 @@ void launch_row_fused(const DecView& d, int M, int step, int mode, size_t smem, 
   cfg.numAttrs = pdl ? 1 : 0;
   const bool few = M <= 2 * d.sms;
   if (d.pred_D) {
-    if (few) cudaLaunchKernelEx(&cfg, k_row_fz<5>, d, step, mode);
-    else cudaLaunchKernelEx(&cfg, k_row_fz<1>, d, step, mode);
+    if (few) cudaLaunchKernelEx(&cfg, k_row_ep<5>, d, step, mode);
+    else cudaLaunchKernelEx(&cfg, k_row_ep<1>, d, step, mode);
   } else {
-    if (few) cudaLaunchKernelEx(&cfg, k_row_fz<4>, d, step, mode);
-    else cudaLaunchKernelEx(&cfg, k_row_fz<0>, d, step, mode);
+    if (few) cudaLaunchKernelEx(&cfg, k_row_ep<4>, d, step, mode);
+    else cudaLaunchKernelEx(&cfg, k_row_ep<0>, d, step, mode);
   }
 }
 

@@ -522,7 +522,6 @@ size_t row_smem_bytes(int V4, int n_lm) {
   return (size_t)V4 * ((n_lm > 1 ? 2 : 1) * sizeof(float) + sizeof(uint8_t));
 }
 
-size_t row_fused_smem_bytes(int V4) { return (size_t)V4 * (sizeof(float) + 2 * sizeof(uint8_t)); }
 
 namespace {
 // Per-call defaults of the fusion bias, which the row pass combines with

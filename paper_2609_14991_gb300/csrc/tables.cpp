@@ -290,25 +290,24 @@ extern "C" tsd_status tsd_ngram_build(int32_t V, int32_t order, const int64_t* c
     }
   });
   arc_rec[(size_t)total_arcs] = make_int4(-1, 0, 0, 0);
-  // dense rows for the unigram states with many continuations (at most
-  // 512 MB of them): log p(v | u) - log p(v) per label, NaN for no arc
+  // a dense row for every unigram state u (V x V4 floats; left out above
+  // 1 GiB): per label v the LM term of a row whose deepest state with an arc
+  // v is u, relative to the call's defaults and the row's summed backoff:
+  // log p(v | u) - log p(v) - cum(u), and 0 where u has no arc v
   const int64_t V4 = ((int64_t)V + 15) / 16 * 16;
   std::vector<int32_t> uni_dense((size_t)V, -1);
   int64_t n_dense = 0;
-  if (order >= 2) {
-    const int64_t thr = std::max<int64_t>(32, V / 8), cap = (512ll << 20) / (4 * V4);
-    for (int64_t u = 0; u < V && n_dense < cap; ++u)
-      if (st_count[(size_t)(base[1] + u)] >= thr) uni_dense[(size_t)u] = (int32_t)n_dense++;
-  }
-  std::vector<float> dense0((size_t)std::max<int64_t>(1, n_dense) * V4, std::nanf(""));
-  parallel_for(order >= 2 ? V : 0, [&](int64_t b, int64_t e) {
+  if (order >= 2 && V * V4 * 4 <= (1ll << 30))
+    for (int64_t u = 0; u < V; ++u) uni_dense[(size_t)u] = (int32_t)n_dense++;
+  std::vector<float> dense0((size_t)std::max<int64_t>(1, n_dense) * V4, 0.f);
+  parallel_for(n_dense > 0 ? V : 0, [&](int64_t b, int64_t e) {
     for (int64_t u = b; u < e; ++u) {
       const int32_t row = uni_dense[(size_t)u];
-      if (row < 0) continue;
       const int64_t s = base[1] + u;
       for (int32_t a = st_begin[(size_t)s]; a < st_begin[(size_t)s] + st_count[(size_t)s]; ++a) {
         const int32_t t = arc_tok[(size_t)a];
-        dense0[(size_t)row * V4 + t] = (float)((double)arc_logp[(size_t)a] - (double)uni_logp[(size_t)t]);
+        dense0[(size_t)row * V4 + t] =
+            (float)((double)arc_logp[(size_t)a] - (double)uni_logp[(size_t)t] - cum[(size_t)s]);
       }
     }
   });
