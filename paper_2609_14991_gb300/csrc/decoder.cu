@@ -219,7 +219,10 @@ tsd_status create_impl(const tsd_decoder_cfg* cfg, const void* W_out_bf16, const
     if ((st = A.alloc(&v.logits, (size_t)d->M_pad * d->N_pad)) || (st = A.alloc(&v.dvec, (size_t)d->N_pad)) ||
         (st = A.alloc(&v.c_lab, (size_t)d->M_pad * d->V4)) || (st = A.alloc(&v.c_add, (size_t)d->M_pad * d->V4)) ||
         (st = A.alloc(&v.c_info, (size_t)d->M_pad)) ||
-        (st = A.alloc(&v.c_mask, (size_t)d->M_pad * v.mask_words))) {
+        (st = A.alloc(&v.c_mask, (size_t)d->M_pad * v.mask_words)) || (st = A.alloc(&v.m_last, (size_t)d->M_pad)) ||
+        (st = A.alloc(&v.m_lm_len, (size_t)d->M_pad)) || (st = A.alloc(&v.m_tr_len, (size_t)d->M_pad)) ||
+        (st = A.alloc(&v.m_lm, (size_t)d->M_pad * kLmChain)) || (st = A.alloc(&v.m_lmr, (size_t)d->M_pad * kLmChain)) ||
+        (st = A.alloc(&v.m_tr, (size_t)d->M_pad * kTrChain)) || (st = A.alloc(&v.m_trr, (size_t)d->M_pad * kTrChain))) {
       A.release();
       return st;
     }

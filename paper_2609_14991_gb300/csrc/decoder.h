@@ -111,6 +111,16 @@ struct DecView {
   int4* c_info;         // [M_pad] (dense row of the row's unigram state or -1, list length, c_r bits, -)
   uint32_t* c_mask;     // [M_pad][mask_words] bit v: label v is listed (blank always)
   int32_t mask_words;   // N_pad / 32
+  // the row's copy of its stream's state within a chunk (previous label,
+  // chain lengths, chains and records), so that a label step reads it by
+  // row in one round
+  int32_t* m_last;      // [M_pad]
+  int32_t* m_lm_len;    // [M_pad]
+  int32_t* m_tr_len;    // [M_pad]
+  int32_t* m_lm;        // [M_pad][kLmChain]
+  int4* m_lmr;          // [M_pad][kLmChain]
+  int32_t* m_tr;        // [M_pad][kTrChain]
+  int4* m_trr;          // [M_pad][kTrChain]
   int32_t* err;  // device status word: nonzero after a bounded wait expired
   // limit of the joint kernel's progress waits (a wait that drains copies or
   // MMAs still in flight before an early exit keeps the 1 s limit)

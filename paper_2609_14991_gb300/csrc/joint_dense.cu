@@ -1,0 +1,397 @@
+// Joint GEMM on the tcgen05 tensor cores with the dense-LM epilogue, for
+// greedy decoding with at most one n-gram LM.
+//
+// Per row r and label v of a 128 x BN tile the epilogue evaluates Eq. 1 up
+// to the row's constant c_r (see row_fused.cu):
+//   F0[v] = logit[v] + D[v] + lambda * dense0[u_r][v]
+// with D the call's defaults (d.dvec) and u_r the dense LM row of the row's
+// unigram state (d.c_info), and reduces the tile to one partial per row:
+// softmax max and sum of the raw logits, and the best F0 over the labels not
+// on the row's correction list (d.c_mask), ties to the lowest label.  The
+// listed labels' raw logits are stored (d.logits) for the row pass.
+//
+// The row's segment of its dense LM row is requested into L2 while the MMAs
+// run and copied into the drained operand stages by one bulk copy per row
+// once they have completed; the epilogue takes the softmax partial of the
+// raw logits (pass 1) while the copies land, then the fused values (pass 2).
+//
+// Warp roles (320 threads): warp 0 TMA producer (A tile 128 x 64 and W_out
+// tile BN x 64 per stage, 128-byte swizzle), warp 1 TMEM
+// allocator and MMA issuer, warps 2-9 epilogue (thread = row; the two warps
+// of a TMEM lane quadrant take alternate 32-column chunks).  Every wait on an
+// mbarrier is bounded; on expiry the kernel records an error in the
+// decoder's status word, drains its own copies and MMAs and returns.
+#include <cuda.h>
+
+#include "decoder.h"
+#include "joint_tc.h"
+#include "tc_common.cuh"
+
+namespace tsd {
+
+namespace {
+
+using namespace tc;
+constexpr int kDThreads = 320;
+constexpr int kDEpi = 256;  // warps 2-9
+constexpr float kNegInf = -__builtin_huge_valf();
+
+// Shared memory: [operand stages][defaults D][barriers].  After the
+// mainloop the stages hold the halves' exchange and, past it, the rows'
+// dense LM segments, rows 16 bytes apart beyond their BN floats so that the
+// 16-byte reads of eight consecutive rows fall in different bank groups.
+template <int BN>
+struct DSmem {
+  static constexpr int kABytes = kBM * kBK * 2;
+  static constexpr int kBBytes = BN * kBK * 2;
+  static constexpr int kStageBytes = kABytes + kBBytes;
+  static constexpr int kStages = BN == 256 ? 4 : (BN == 128 ? 5 : 8);
+  static constexpr int kRowStride = BN * 4 + 16;
+  static constexpr int kDenseOff = 10240;  // past the halves' exchange
+  static constexpr int kDOff = kStages * kStageBytes;
+  static constexpr int kBarOff = kDOff + BN * 4;
+  static constexpr int kBytes = kBarOff + 256 + 1024 /*align*/;
+  static_assert(kBM * 18 * 4 + 16 <= kDenseOff, "the halves' exchange stays clear of the dense rows");
+  static_assert(kDenseOff + kBM * kRowStride <= kStages * kStageBytes, "the dense rows fit the drained stages");
+  static_assert(kBytes <= 227 * 1024, "shared memory per CTA");
+};
+
+// Sum over a chunk of 2^(l[i] * log2 e - s2) in four independent accumulators.
+__device__ __forceinline__ float sum_exp2_chunk(const float* l, float s2) {
+  float a[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+  for (int i = 0; i < 32; ++i) a[i & 3] += ex2_approx(fmaf(l[i], kLog2e, -s2));
+  return (a[0] + a[1]) + (a[2] + a[3]);
+}
+
+template <int N>
+__device__ __forceinline__ uint32_t pick(const uint32_t (&a)[N], int k) {
+  uint32_t v = a[0];
+#pragma unroll
+  for (int i = 1; i < N; ++i) v = (k == i) ? a[i] : v;
+  return v;
+}
+
+template <int BN>
+__global__ void __launch_bounds__(kDThreads, 1)
+    k_joint_dense(DecView d, int step, const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB) {
+  using S = DSmem<BN>;
+  extern __shared__ __align__(1024) unsigned char smem_raw[];
+  unsigned char* smem = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  float* sD = reinterpret_cast<float*>(smem + S::kDOff);
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + S::kBarOff);
+  uint64_t* empty = full + S::kStages;
+  uint64_t* accum = empty + S::kStages;  // every MMA has completed
+  uint64_t* dbar = accum + 1;            // the rows' dense segments have landed
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(dbar + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int n0 = blockIdx.x * BN, m0 = blockIdx.y * kBM;
+  const int M = d.params->n * d.K;
+  const int KB = d.H / kBK;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < S::kStages; ++s) {
+      mbar_init(full + s, 1);
+      mbar_init(empty + s, 1);
+    }
+    mbar_init(accum, 1);
+    mbar_init(dbar, kBM);  // one arrival per row
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
+                 "r"(BN)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  fence_before();
+  __syncthreads();
+  fence_after();
+  const uint32_t tmem = *tmem_slot;
+  // W_out is constant: the first stages' tiles are requested before the
+  // dependency wait (each stage's barrier expects its A tile as well)
+  const int pre = min(KB, S::kStages);
+  if (warp == 0 && lane == 0) {
+    for (int kb = 0; kb < pre; ++kb) {
+      mbar_expect_tx(full + kb, S::kStageBytes);
+      tma_load_2d(smem + kb * S::kStageBytes + S::kABytes, &tmB, full + kb, kb * kBK, n0);
+    }
+  }
+  // Programmatic dependent launch: the set-up above overlaps the row pass;
+  // its outputs (joint input, correction list) are read after the wait.
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+
+  if (warp == 0) {
+    if (lane == 0) {
+      bool ok = true;
+      int issued = 0;
+      for (int kb = 0; kb < KB; ++kb) {
+        const int s = kb % S::kStages;
+        const uint32_t ph = (uint32_t)(kb / S::kStages) & 1u;
+        unsigned char* sa = smem + s * S::kStageBytes;
+        if (kb < pre) {  // first use of the stage: W_out already requested
+          tma_load_2d(sa, &tmA, full + s, kb * kBK, m0);
+          ++issued;
+          continue;
+        }
+        if (!mbar_wait(empty + s, ph ^ 1u, d.wait_ns)) { ok = false; break; }
+        mbar_expect_tx(full + s, S::kStageBytes);
+        tma_load_2d(sa, &tmA, full + s, kb * kBK, m0);
+        tma_load_2d(sa + S::kABytes, &tmB, full + s, kb * kBK, n0);
+        ++issued;
+      }
+      // never exit with copies in flight (the long limit)
+      for (int kb = max(0, issued - S::kStages); kb < issued; ++kb)
+        mbar_wait(full + kb % S::kStages, (uint32_t)(kb / S::kStages) & 1u);
+      if (!ok) atomicOr(d.err, 1);
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    if (lane == 0) {
+      bool ok = true;
+      const uint32_t idesc = idesc_bf16(kBM, BN);
+      for (int kb = 0; kb < KB; ++kb) {
+        const int s = kb % S::kStages;
+        const uint32_t ph = (uint32_t)(kb / S::kStages) & 1u;
+        if (!mbar_wait(full + s, ph, d.wait_ns)) { ok = false; break; }
+        fence_after();
+        const uint32_t sa = smem_u32(smem + s * S::kStageBytes);
+        const uint64_t ad = sw128_desc(sa), bd = sw128_desc(sa + S::kABytes);
+#pragma unroll
+        for (int k = 0; k < kBK / 16; ++k)
+          mma_bf16(tmem, ad + (uint64_t)(2 * k), bd + (uint64_t)(2 * k), idesc, (kb | k) ? 1u : 0u);
+        mma_commit(empty + s);
+      }
+      // signals the epilogue once every issued MMA has completed (also after
+      // a timeout, so nothing is in flight when TMEM is released)
+      mma_commit(accum);
+      if (!ok) atomicOr(d.err, 2);
+    }
+    __syncwarp();
+  } else {
+    // epilogue: warps 2..9, thread = row of the tile
+    const int q = warp & 3;  // TMEM lane quadrant this warp may access
+    const int ehalf = (warp - 2) >> 2;
+    const int row = q * 32 + lane;
+    const int gr = m0 + row;
+    const bool live = gr < M;
+    const int N = d.N, V4 = d.V4;
+    float mx = kNegInf, se = 0.f, bv = kNegInf;
+    int bi = INT_MAX;
+    // while the MMAs run: the call's defaults of the tile's labels, lambda,
+    // the row's dense LM row and mask words (written by the row pass before
+    // this grid's wait)
+    for (int i = (int)threadIdx.x - 64; i < BN; i += kDEpi) sD[i] = __ldcg(d.dvec + n0 + i);
+    const float lam = d.params->lambda;
+    constexpr int kMy = BN / 64;  // chunks each epilogue warp takes: c = ehalf + 2k
+    uint32_t mw[kMy];
+#pragma unroll
+    for (int k = 0; k < kMy; ++k) mw[k] = 0u;
+    int uoff = -1;
+    if (live) {
+      const int u = __ldcg(&d.c_info[gr].x);
+      if (u >= 0 && u < d.lm.n_dense) uoff = u * V4;
+      const uint32_t* mrow = d.c_mask + (size_t)gr * d.mask_words + n0 / 32;
+#pragma unroll
+      for (int k = 0; k < kMy; ++k) mw[k] = __ldcg(mrow + ehalf + 2 * k);
+    }
+    unsigned char* drow = smem + S::kDenseOff + row * S::kRowStride;
+    const int seg = min(BN, V4 - n0);  // labels of the tile inside the dense rows
+    if (ehalf == 0 && uoff >= 0 && seg > 0) {  // the row's segment into L2 while the MMAs run
+      asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(d.lm.dense0 + uoff + n0), "r"((uint32_t)seg * 4u)
+                   : "memory");
+    }
+    asm volatile("bar.sync 2, %0;" ::"n"(kDEpi) : "memory");  // sD complete
+    bool ok = __all_sync(0xffffffffu, mbar_wait(accum, 0, d.wait_ns));  // tcgen05.ld wants the warp whole
+    if (!ok && lane == 0) atomicOr(d.err, 4);
+    fence_after();
+    // the row's segment into the drained stages (every MMA has completed) by
+    // one bulk copy, and the row's arrival on dbar (with the copy's bytes)
+    if (ehalf == 0) {
+      if (ok && uoff >= 0 && seg > 0) {
+        mbar_expect_tx(dbar, (uint32_t)seg * 4u);
+        bulk_g2s(drow, d.lm.dense0 + uoff + n0, (uint32_t)seg * 4u, dbar);
+      } else {
+        mbar_arrive(dbar);
+      }
+    }
+    const uint32_t tbase = tmem + ((uint32_t)(q * 32) << 16);
+    if (ok) {
+      // pass 1, while the copies land: the softmax partial of the raw
+      // logits; the listed labels' logits go out for the row pass
+#pragma unroll 1
+      for (int c = ehalf; c < BN / 32; c += 2) {
+        __syncwarp();
+        const int c0 = n0 + c * 32;
+        float l[32];
+        tmem_ld32(tbase + (uint32_t)(c * 32), l);
+        if (c0 + 32 > N) {
+#pragma unroll
+          for (int i = 0; i < 32; ++i)
+            if (c0 + i >= N) l[i] = kNegInf;
+        }
+        float t[16];
+#pragma unroll
+        for (int i = 0; i < 16; ++i) t[i] = fmaxf(l[i], l[i + 16]);
+#pragma unroll
+        for (int w = 8; w > 0; w >>= 1)
+#pragma unroll
+          for (int i = 0; i < w; ++i) t[i] = fmaxf(t[i], t[i + w]);
+        const float cm = t[0];
+        if (cm != kNegInf) {
+          const float m2 = fmaxf(mx, cm);
+          const float s2 = m2 * kLog2e;
+          float acc = (mx == kNegInf) ? 0.f : se * ex2_approx(mx * kLog2e - s2);
+          acc += sum_exp2_chunk(l, s2);
+          se = acc;
+          mx = m2;
+        }
+        if (d.cap_logits && step < d.cap_steps && live) {
+          float* cl = d.cap_logits + ((size_t)step * M + gr) * N;
+#pragma unroll
+          for (int i = 0; i < 32; ++i)
+            if (c0 + i < N) cl[c0 + i] = l[i];
+        }
+        const uint32_t mk = pick(mw, c >> 1);
+        if (mk) {
+          float* lo = d.logits + (size_t)gr * d.N_pad + c0;
+#pragma unroll
+          for (int i = 0; i < 32; ++i)
+            if ((mk >> i) & 1u) lo[i] = l[i];
+        }
+      }
+      ok = __all_sync(0xffffffffu, mbar_wait(dbar, 0, d.wait_ns));
+      if (!ok && lane == 0) atomicOr(d.err, 64);
+    }
+    if (ok) {
+      // pass 2: F0 = logit + D + lambda * dense0[u] of the unlisted labels and
+      // the tile's best of them
+#pragma unroll 1
+      for (int c = ehalf; c < BN / 32; c += 2) {
+        __syncwarp();
+        const int c0 = n0 + c * 32;
+        float l[32];
+        tmem_ld32(tbase + (uint32_t)(c * 32), l);
+        if (c0 + 32 > N) {
+#pragma unroll
+          for (int i = 0; i < 32; ++i)
+            if (c0 + i >= N) l[i] = kNegInf;
+        }
+        const float4* dv4 = reinterpret_cast<const float4*>(sD + 32 * c);
+        float x[32];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          const float4 dq = dv4[j];
+          float4 xq = make_float4(0.f, 0.f, 0.f, 0.f);
+          if (uoff >= 0 && c * 32 + 4 * j < seg) xq = *reinterpret_cast<const float4*>(drow + (c * 32 + 4 * j) * 4);
+          x[4 * j] = l[4 * j] + fmaf(lam, xq.x, dq.x);
+          x[4 * j + 1] = l[4 * j + 1] + fmaf(lam, xq.y, dq.y);
+          x[4 * j + 2] = l[4 * j + 2] + fmaf(lam, xq.z, dq.z);
+          x[4 * j + 3] = l[4 * j + 3] + fmaf(lam, xq.w, dq.w);
+        }
+        const uint32_t mk = pick(mw, c >> 1);
+        if (mk) {
+#pragma unroll
+          for (int i = 0; i < 32; ++i)
+            if ((mk >> i) & 1u) x[i] = kNegInf;
+        }
+        float u[16];
+#pragma unroll
+        for (int i = 0; i < 16; ++i) u[i] = fmaxf(x[i], x[i + 16]);
+#pragma unroll
+        for (int w = 8; w > 0; w >>= 1)
+#pragma unroll
+          for (int i = 0; i < w; ++i) u[i] = fmaxf(u[i], u[i + w]);
+        const float fm = u[0];
+        if (fm > bv) {
+          int j = 31;
+#pragma unroll
+          for (int i = 31; i >= 0; --i)
+            if (x[i] == fm) j = i;
+          bv = fm;
+          bi = c0 + j;
+        }
+      }
+    }
+    // never leave with MMAs still writing the accumulator or row copies still
+    // landing (the long limit whatever wait_ns is)
+    if (warp == 2 && lane == 0) {
+      mbar_wait(accum, 0);
+      mbar_wait(dbar, 0);
+    }
+    __syncwarp();
+    // merge the two epilogue halves' partials of each row: the second leaves
+    // its partial in the drained stages, the first combines and stores
+    float* xbase = reinterpret_cast<float*>(smem);
+    float* xch = xbase + row * 18;
+    int* xok = reinterpret_cast<int*>(xbase + kBM * 18);
+    if (ehalf == 1) {
+      if (ok) {
+        xch[0] = mx;
+        xch[1] = se;
+        xch[2] = bv;
+        xch[3] = __int_as_float(bi);
+      }
+      if (lane == 0) xok[q] = ok ? 1 : 0;
+    }
+    asm volatile("bar.sync 1, %0;" ::"n"(kDEpi) : "memory");
+    if (ehalf == 0 && ok && xok[q] && live) {
+      const float m1 = xch[0], s1 = xch[1];
+      if (m1 != kNegInf) {
+        if (mx == kNegInf) {
+          mx = m1;
+          se = s1;
+        } else {
+          const float m2 = fmaxf(mx, m1);
+          se = se * ex2_approx((mx - m2) * kLog2e) + s1 * ex2_approx((m1 - m2) * kLog2e);
+          mx = m2;
+        }
+      }
+      const float v1 = xch[2];
+      const int i1 = __float_as_int(xch[3]);
+      if (v1 > bv || (v1 == bv && i1 < bi)) { bv = v1; bi = i1; }
+      d.part[(size_t)gr * d.n_ptiles + blockIdx.x] = make_float4(mx, se, bv, __int_as_float(bi));
+    }
+  }
+  fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(BN) : "memory");
+  }
+}
+
+}  // namespace
+
+cudaError_t joint_dense_prepare(int bn) {
+  const auto attr = cudaFuncAttributeMaxDynamicSharedMemorySize;
+  if (bn == 256) return cudaFuncSetAttribute(k_joint_dense<256>, attr, DSmem<256>::kBytes);
+  if (bn == 128) return cudaFuncSetAttribute(k_joint_dense<128>, attr, DSmem<128>::kBytes);
+  return cudaFuncSetAttribute(k_joint_dense<64>, attr, DSmem<64>::kBytes);
+}
+
+void launch_joint_dense(const JointTc& jt, const DecView& d, int M, int step, cudaStream_t s, bool pdl) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(d.N_pad / jt.bn, (M + kBM - 1) / kBM);
+  cfg.blockDim = dim3(kDThreads);
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl ? 1 : 0;
+  if (jt.bn == 256) {
+    cfg.dynamicSmemBytes = DSmem<256>::kBytes;
+    cudaLaunchKernelEx(&cfg, k_joint_dense<256>, d, step, jt.mapA, jt.mapB);
+  } else if (jt.bn == 128) {
+    cfg.dynamicSmemBytes = DSmem<128>::kBytes;
+    cudaLaunchKernelEx(&cfg, k_joint_dense<128>, d, step, jt.mapA, jt.mapB);
+  } else {
+    cfg.dynamicSmemBytes = DSmem<64>::kBytes;
+    cudaLaunchKernelEx(&cfg, k_joint_dense<64>, d, step, jt.mapA, jt.mapB);
+  }
+}
+
+}  // namespace tsd

@@ -9,12 +9,9 @@
 // tcgen05.ld (thread = row; two warps per 32-lane quadrant take alternate
 // 32-column chunks) and reduce it on chip to the row's selection partial for
 // this tile: softmax max and sum over the real labels, and the best fused
-// value, ties to the lowest label.  The fused value is logit + bias with a
-// dense fusion bias row per row (several LMs), or, for greedy decoding with
-// at most one LM (DENSE), logit + D[v] + lambda * dense0[u][v]: the call's
-// defaults plus the dense LM row of the row's unigram state u, leaving out
-// the labels on the row's correction list, whose raw logits are stored for
-// the row pass instead.  No other logit leaves the SM.
+// value logit + bias (the dense fusion bias row of several LMs), ties to the
+// lowest label, or (BEAM) the tile's top K.  Greedy decoding with at most one
+// LM runs joint_dense.cu instead.  Logits never leave the SM.
 //
 // Warp roles (320 threads): warp 0 TMA producer, warp 1 TMEM allocator and
 // MMA issuer, warps 2-9 epilogue.  Every wait on an mbarrier is bounded in
@@ -38,17 +35,17 @@ constexpr float kNegInf = -__builtin_huge_valf();
 // bias (several LMs), the bias of the tile (128 rows x BN fp32) arrives by
 // TMA in 128 x 32 boxes with the 128-byte swizzle while the mainloop runs;
 // at BN = 256 only the first half has its own buffer and the second half
-// lands in the drained stages.  DENSE takes the tile's BN defaults instead.
-template <int BN, bool DENSE = false>
+// lands in the drained stages.
+template <int BN>
 struct Smem {
   static constexpr int kStages = (BN == 256) ? 3 : (BN == 128 ? 4 : 8);
   static constexpr int kABytes = kBM * kBK * 2;
   static constexpr int kBBytes = BN * kBK * 2;
   static constexpr int kStageBytes = kABytes + kBBytes;
   static constexpr int kBoxBytes = kBM * 32 * 4;
-  static constexpr int kBoxes = DENSE ? 0 : BN / 32;
-  static constexpr int kEarly = DENSE ? 0 : ((BN == 256) ? 4 : kBoxes);
-  static constexpr int kBiasBytes = kEarly * kBoxBytes + (DENSE ? BN * 4 : 0);  // DENSE: the tile's defaults D
+  static constexpr int kBoxes = BN / 32;
+  static constexpr int kEarly = (BN == 256) ? 4 : kBoxes;
+  static constexpr int kBiasBytes = kEarly * kBoxBytes;
   static constexpr int kBytes = kStages * kStageBytes + kBiasBytes + 1024 /*align*/ + 256 /*barriers*/;
   static_assert((kBoxes - kEarly) * kBoxBytes <= kStages * kStageBytes, "late bias boxes fit the stages");
   // the epilogue halves' exchange (per row 18 floats, 4 flags) after the late boxes
@@ -64,31 +61,15 @@ __device__ __forceinline__ float sum_exp2_32(const float* l, float s2) {
   return (a[0] + a[1]) + (a[2] + a[3]);
 }
 
-// The dense LM row segment of one row for one 32-label chunk (0 past the
-// table's row width V4, which is a multiple of 16; no row: all 0).
-__device__ __forceinline__ void load_dense_chunk(const float* __restrict__ row, int c0, int V4, float* x) {
-#pragma unroll
-  for (int j = 0; j < 8; ++j) {
-    float4 q = make_float4(0.f, 0.f, 0.f, 0.f);
-    if (row && c0 + 4 * j < V4) q = __ldg(reinterpret_cast<const float4*>(row + c0) + j);
-    x[4 * j] = q.x; x[4 * j + 1] = q.y; x[4 * j + 2] = q.z; x[4 * j + 3] = q.w;
-  }
-}
-
 // BEAM: instead of the single best fused label, each row keeps the top-K
 // (K = d.topk <= 8: the beam width, or the pruned-fusion candidate count)
 // values of the tile, ties to the lower label.  With pruned fusion (d.prune)
 // the values are the plain logits: no bias tile is loaded.
-// DENSE: no bias tile; the fused value is logit + D[v] (d.dvec, the call's
-// defaults) + lambda * dense0[u][v] (u: the row's dense LM row, d.c_info),
-// and the labels whose bit is set in the row's mask (d.c_mask) are no
-// candidates here: their raw logits go to d.logits for the row pass.
-template <int BN, bool BEAM, bool DENSE>
+template <int BN, bool BEAM>
 __global__ void __launch_bounds__(kThreads, 1)
     k_joint_tc(DecView d, int step, const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                const __grid_constant__ CUtensorMap tmBias) {
-  using S = Smem<BN, DENSE>;
-  static_assert(!(DENSE && BEAM), "the dense epilogue serves greedy decoding");
+  using S = Smem<BN>;
   extern __shared__ __align__(1024) unsigned char smem_raw[];
   unsigned char* smem = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   unsigned char* bias_early = smem + S::kStages * S::kStageBytes;
@@ -100,7 +81,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int n0 = blockIdx.x * BN, m0 = blockIdx.y * kBM;
-  const bool use_bias = !DENSE && !(BEAM && d.prune);
+  const bool use_bias = !(BEAM && d.prune);
   const int M = d.params->n * d.K;
   const int KB = d.H / kBK;
 
@@ -210,35 +191,6 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
     for (int j = 0; j < 8; ++j) { tv[j] = kNegInf; ti[j] = INT_MAX; }
     float tmin = kNegInf;  // tv[K-1]
-    float* sD = reinterpret_cast<float*>(bias_early);  // DENSE: the tile's defaults D (kEarly is 0)
-    const float* urow = nullptr;      // DENSE: the row's dense LM row
-    const uint32_t* mrow = nullptr;   // DENSE: the row's mask words of this tile
-    float lam = 0.f;
-    if (DENSE) {
-      // while the MMAs run: the call's defaults of the tile's labels, the
-      // row's dense LM row (its segment requested into L2 now) and mask
-      // (both written by the row pass before this grid's wait)
-      for (int i = (int)threadIdx.x - 64; i < BN; i += kEpiThreads) sD[i] = __ldcg(d.dvec + n0 + i);
-      lam = d.params->lambda;
-      if (live) {
-        const int u = __ldcg(&d.c_info[gr].x);
-        if (u >= 0 && u < d.lm.n_dense) urow = d.lm.dense0 + (size_t)u * d.V4;
-        mrow = d.c_mask + (size_t)gr * d.mask_words + n0 / 32;
-        if (urow && half == 0 && n0 < d.V4) {
-          const uint32_t bytes = (uint32_t)min(BN, d.V4 - n0) * 4u;
-          asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(urow + n0), "r"(bytes) : "memory");
-        }
-      }
-      asm volatile("bar.sync 2, %0;" ::"n"(kEpiThreads) : "memory");
-    }
-    // DENSE: the mask word and dense LM values of the next chunk this warp
-    // takes, loaded one chunk ahead (the first while the MMAs run)
-    float xn[32];
-    uint32_t mkn = 0u;
-    if (DENSE) {
-      load_dense_chunk(urow, n0 + half * 32, d.V4, xn);
-      mkn = mrow ? __ldcg(mrow + half) : 0u;
-    }
     ok = __all_sync(0xffffffffu, mbar_wait(accum, 0, d.wait_ns));  // warp-uniform: tcgen05.ld is .sync.aligned
     if (!ok && lane == 0) atomicOr(d.err, 4);
     fence_after();
@@ -268,82 +220,6 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (lane == 0) atomicOr(d.err, 32);
             break;
           }
-        }
-        if constexpr (DENSE) {
-          const int c0 = n0 + c * 32;
-          const uint32_t mk = mkn;
-          float x[32];
-#pragma unroll
-          for (int i = 0; i < 32; ++i) x[i] = xn[i];
-          if (c + 2 < BN / 32) {
-            load_dense_chunk(urow, c0 + 64, d.V4, xn);
-            mkn = mrow ? __ldcg(mrow + c + 2) : 0u;
-          }
-          float l[32];
-          tmem_ld32(tbase + (uint32_t)(c * 32), l);
-          if (c0 + 32 > N) {
-#pragma unroll
-            for (int i = 0; i < 32; ++i)
-              if (c0 + i >= N) l[i] = kNegInf;
-          }
-          float t[16];
-#pragma unroll
-          for (int i = 0; i < 16; ++i) t[i] = fmaxf(l[i], l[i + 16]);
-#pragma unroll
-          for (int w = 8; w > 0; w >>= 1)
-#pragma unroll
-            for (int i = 0; i < w; ++i) t[i] = fmaxf(t[i], t[i + w]);
-          const float cm = t[0];
-          if (cm != kNegInf) {
-            const float m2 = fmaxf(mx, cm);
-            const float s2 = m2 * kLog2e;
-            float acc = (mx == kNegInf) ? 0.f : se * ex2_approx(mx * kLog2e - s2);
-            acc += sum_exp2_32(l, s2);
-            se = acc;
-            mx = m2;
-          }
-          if (d.cap_logits && step < d.cap_steps && live) {
-            float* cl = d.cap_logits + ((size_t)step * M + gr) * N;
-#pragma unroll
-            for (int i = 0; i < 32; ++i)
-              if (c0 + i < N) cl[c0 + i] = l[i];
-          }
-          // fused values (reuse x); listed labels are stored, not candidates
-          const float4* dv4 = reinterpret_cast<const float4*>(sD + 32 * c);
-#pragma unroll
-          for (int j = 0; j < 8; ++j) {
-            const float4 dq = dv4[j];
-            x[4 * j] = l[4 * j] + fmaf(lam, x[4 * j], dq.x);
-            x[4 * j + 1] = l[4 * j + 1] + fmaf(lam, x[4 * j + 1], dq.y);
-            x[4 * j + 2] = l[4 * j + 2] + fmaf(lam, x[4 * j + 2], dq.z);
-            x[4 * j + 3] = l[4 * j + 3] + fmaf(lam, x[4 * j + 3], dq.w);
-          }
-          if (mk) {
-            float* lo = d.logits + (size_t)gr * d.N_pad + c0;
-#pragma unroll
-            for (int i = 0; i < 32; ++i)
-              if ((mk >> i) & 1u) {
-                lo[i] = l[i];
-                x[i] = kNegInf;
-              }
-          }
-          float u[16];
-#pragma unroll
-          for (int i = 0; i < 16; ++i) u[i] = fmaxf(x[i], x[i + 16]);
-#pragma unroll
-          for (int w = 8; w > 0; w >>= 1)
-#pragma unroll
-            for (int i = 0; i < w; ++i) u[i] = fmaxf(u[i], u[i + w]);
-          const float fm = u[0];
-          if (fm > bv) {
-            int j = 31;
-#pragma unroll
-            for (int i = 31; i >= 0; --i)
-              if (x[i] == fm) j = i;
-            bv = fm;
-            bi = c0 + j;
-          }
-          continue;
         }
         const unsigned char* box = (c < S::kEarly) ? bias_early + c * S::kBoxBytes : smem + (c - S::kEarly) * S::kBoxBytes;
         float b[32];
@@ -546,18 +422,16 @@ cudaError_t joint_tc_prepare(JointTc* jt, const uint16_t* A, int M_pad, const ui
   const auto attr = cudaFuncAttributeMaxDynamicSharedMemorySize;
   cudaError_t e = cudaSuccess;
   if (bn == 256) {
-    e = cudaFuncSetAttribute(k_joint_tc<256, false, false>, attr, Smem<256>::kBytes);
-    if (e == cudaSuccess) e = cudaFuncSetAttribute(k_joint_tc<256, true, false>, attr, Smem<256>::kBytes);
-    if (e == cudaSuccess) e = cudaFuncSetAttribute(k_joint_tc<256, false, true>, attr, Smem<256, true>::kBytes);
+    e = cudaFuncSetAttribute(k_joint_tc<256, false>, attr, Smem<256>::kBytes);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(k_joint_tc<256, true>, attr, Smem<256>::kBytes);
   } else if (bn == 128) {
-    e = cudaFuncSetAttribute(k_joint_tc<128, false, false>, attr, Smem<128>::kBytes);
-    if (e == cudaSuccess) e = cudaFuncSetAttribute(k_joint_tc<128, true, false>, attr, Smem<128>::kBytes);
-    if (e == cudaSuccess) e = cudaFuncSetAttribute(k_joint_tc<128, false, true>, attr, Smem<128, true>::kBytes);
+    e = cudaFuncSetAttribute(k_joint_tc<128, false>, attr, Smem<128>::kBytes);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(k_joint_tc<128, true>, attr, Smem<128>::kBytes);
   } else {
-    e = cudaFuncSetAttribute(k_joint_tc<64, false, false>, attr, Smem<64>::kBytes);
-    if (e == cudaSuccess) e = cudaFuncSetAttribute(k_joint_tc<64, true, false>, attr, Smem<64>::kBytes);
-    if (e == cudaSuccess) e = cudaFuncSetAttribute(k_joint_tc<64, false, true>, attr, Smem<64, true>::kBytes);
+    e = cudaFuncSetAttribute(k_joint_tc<64, false>, attr, Smem<64>::kBytes);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(k_joint_tc<64, true>, attr, Smem<64>::kBytes);
   }
+  if (e == cudaSuccess) e = joint_dense_prepare(bn);
   return e;
 }
 
@@ -565,20 +439,17 @@ namespace {
 template <int BN>
 void launch_bn(cudaLaunchConfig_t& cfg, const JointTc& jt, const DecView& d, int step) {
   const bool beam = d.topk > 1 || d.prune > 0;  // the top-K epilogue
-  if (beam) {
-    cfg.dynamicSmemBytes = Smem<BN>::kBytes;
-    cudaLaunchKernelEx(&cfg, k_joint_tc<BN, true, false>, d, step, jt.mapA, jt.mapB, jt.mapBias);
-  } else if (d.fused) {
-    cfg.dynamicSmemBytes = Smem<BN, true>::kBytes;
-    cudaLaunchKernelEx(&cfg, k_joint_tc<BN, false, true>, d, step, jt.mapA, jt.mapB, jt.mapBias);
-  } else {
-    cfg.dynamicSmemBytes = Smem<BN>::kBytes;
-    cudaLaunchKernelEx(&cfg, k_joint_tc<BN, false, false>, d, step, jt.mapA, jt.mapB, jt.mapBias);
-  }
+  cfg.dynamicSmemBytes = Smem<BN>::kBytes;
+  if (beam) cudaLaunchKernelEx(&cfg, k_joint_tc<BN, true>, d, step, jt.mapA, jt.mapB, jt.mapBias);
+  else cudaLaunchKernelEx(&cfg, k_joint_tc<BN, false>, d, step, jt.mapA, jt.mapB, jt.mapBias);
 }
 }  // namespace
 
 void launch_joint_tc(const JointTc& jt, const DecView& d, int M, int step, cudaStream_t s, bool pdl) {
+  if (d.fused) {
+    launch_joint_dense(jt, d, M, step, s, pdl);
+    return;
+  }
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(d.N_pad / jt.bn, (M + kBM - 1) / kBM);
   cfg.blockDim = dim3(kThreads);

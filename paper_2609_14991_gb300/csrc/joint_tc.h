@@ -20,6 +20,9 @@ int joint_tc_pick_bn(int M_max, int N_pad, int sms);
 cudaError_t joint_tc_prepare(JointTc* jt, const uint16_t* A, int M_pad, const uint16_t* Wt, int N_pad, int H, int bn,
                              const float* bias);
 void launch_joint_tc(const JointTc& jt, const DecView& d, int M, int step, cudaStream_t s, bool pdl);
+// The dense-LM epilogue variant (greedy decoding with at most one LM): joint_dense.cu.
+cudaError_t joint_dense_prepare(int bn);
+void launch_joint_dense(const JointTc& jt, const DecView& d, int M, int step, cudaStream_t s, bool pdl);
 // The default limit of a bounded wait (1 s).
 unsigned long long tc_wait_ns_default();
 

@@ -65,6 +65,7 @@ constexpr int kFzThreads = 128;  // 4 warps: seven CTAs per SM at 72 registers
 constexpr int kFzWarps = kFzThreads / 32;
 constexpr int kHeld = 2;      // arc groups of four of levels 1.. a thread keeps in registers
 constexpr int kListHeld = 2;  // list entries a thread loads before waiting for the joint kernel
+constexpr int kTrHeld = 1;    // trie chain children a thread keeps in registers
 
 // Aligned groups of four arcs a chain level's arcs [b, b + c) span.
 __device__ __forceinline__ int level_groups(int b, int c) { return c > 0 ? (b + c - (b & ~3) + 3) >> 2 : 0; }
@@ -85,10 +86,12 @@ __global__ void __launch_bounds__(kFzThreads) __maxnreg__((VAR & 4) ? 128 : 72) 
   const bool counting = (mode == 2 || d.count);
   extern __shared__ __align__(16) unsigned char smem[];
   // per label: the offer tag, then (for the winners) the LM term's bits; the
-  // list bitmask; 1 if the label has its LM term; the trie goto depth (0: none)
-  uint32_t* key = reinterpret_cast<uint32_t*>(smem);              // [V4]
-  uint32_t* msk = key + d.V4;                                      // [mask_words]
-  uint8_t* lmf = reinterpret_cast<uint8_t*>(msk + d.mask_words);  // [V4]
+  // list bitmask; the root's children bitmask; 1 if the label has its LM
+  // term; the trie goto depth (0: none)
+  uint32_t* key = reinterpret_cast<uint32_t*>(smem);                // [V4]
+  uint32_t* msk = key + d.V4;                                        // [mask_words]
+  uint32_t* rootw = msk + d.mask_words;                              // [mask_words]
+  uint8_t* lmf = reinterpret_cast<uint8_t*>(rootw + d.mask_words);  // [V4]
   uint8_t* dep = lmf + d.V4;                                       // [V4]
 
   __shared__ int s_t, s_sym, s_cnt, s_y, s_last, s_slot, s_T, s_n;
@@ -107,6 +110,7 @@ __global__ void __launch_bounds__(kFzThreads) __maxnreg__((VAR & 4) ? 128 : 72) 
   __shared__ int4 s_tr_hit[kTrChain]; // child record of y at each old trie node (x = -1: none)
   __shared__ int4 s_uni_hit, s_root_hit;
   __shared__ int s_gbeg[kLmChain + 1];  // arc groups of the LM levels 1.. before level l
+  __shared__ int s_tpre[kTrChain + 1];  // children of the trie chain nodes before node k
   __shared__ float s_bv[kFzWarps];
   __shared__ int s_bi[kFzWarps];
   __shared__ unsigned long long s_bytes;  // algorithmic bytes of the row-step (when counting)
@@ -131,6 +135,35 @@ __global__ void __launch_bounds__(kFzThreads) __maxnreg__((VAR & 4) ? 128 : 72) 
     s_ext = 0;
     s_ci = step > 0 ? __ldcg(d.c_info + r) : make_int4(-1, 0, 0, 0);
     s_bad = !checked(slot >= 0 && slot < d.lm_stride, d.err, 1);
+    if (step > 0) {  // the row's copy of its state, written by the previous row pass
+      s_t = __ldcg(d.r_t + r); s_sym = __ldcg(d.r_sym + r); s_cnt = __ldcg(d.r_cnt + r);
+      s_nl = __ldcg(d.m_lm_len + r);
+      s_nt = __ldcg(d.m_tr_len + r);
+      s_last = __ldcg(d.m_last + r);
+    }
+  } else if (step > 0 && tid >= 32 && tid < 32 + kLmChain) {
+    const int l = tid - 32;
+    s_lm[l] = __ldcg(d.m_lm + (size_t)r * kLmChain + l);
+    s_lmr[l] = __ldcg(d.m_lmr + (size_t)r * kLmChain + l);
+  } else if (step > 0 && tid >= 64 && tid < 64 + kTrChain) {
+    const int k = tid - 64;
+    s_tr[k] = __ldcg(d.m_tr + (size_t)r * kTrChain + k);
+    s_trr[k] = __ldcg(d.m_trr + (size_t)r * kTrChain + k);
+  }
+  // the list of the state the joint evaluated: its first kListHeld entries
+  // per thread in registers (loaded whatever its length; entries past it
+  // are dropped once the length is known)
+  int hv[kListHeld];
+  float ha[kListHeld];
+#pragma unroll
+  for (int u = 0; u < kListHeld; ++u) {
+    const int k = tid + u * kFzThreads;
+    hv[u] = -1;
+    ha[u] = 0.f;
+    if (step > 0 && k < d.V4) {
+      hv[u] = __ldcg(d.c_lab + (size_t)r * d.V4 + k);
+      ha[u] = __ldcg(d.c_add + (size_t)r * d.V4 + k);
+    }
   }
   {  // per-label scratch reset
     uint4* k4 = reinterpret_cast<uint4*>(key);
@@ -141,50 +174,53 @@ __global__ void __launch_bounds__(kFzThreads) __maxnreg__((VAR & 4) ? 128 : 72) 
       f4[q] = 0u;
       e4[q] = 0u;
     }
-    for (int q = tid; q < d.mask_words; q += blockDim.x) msk[q] = 0u;
+    for (int q = tid; q < d.mask_words; q += blockDim.x) {
+      msk[q] = 0u;
+      rootw[q] = q < (V + 31) / 32 ? __ldg(d.droot + q) : 0u;
+    }
   }
   row::block_sync();
   if (s_bad) return;
   const int slot = s_slot, T = s_T;
-  // the list of the state the joint evaluated (its first kListHeld entries
-  // per thread in registers)
-  int hv[kListHeld];
-  float ha[kListHeld];
 #pragma unroll
-  for (int u = 0; u < kListHeld; ++u) {
-    const int k = tid + u * kFzThreads;
-    hv[u] = -1;
-    ha[u] = 0.f;
-    if (k < s_ci.y) {  // step > 0 (the list of a finished row is loaded but not used)
-      hv[u] = __ldcg(d.c_lab + (size_t)r * d.V4 + k);
-      ha[u] = __ldcg(d.c_add + (size_t)r * d.V4 + k);
-    }
-  }
-  // the chains are read whole (their arrays have room for the longest), so
-  // their lengths need not be known first
-  if (tid == 0) {
-    if (step == 0) {
+  for (int u = 0; u < kListHeld; ++u)
+    if (tid + u * kFzThreads >= s_ci.y) hv[u] = -1;
+  if (step == 0) {
+    // the chunk's first step: the stream's state by slot (the chains are
+    // read whole: their arrays have room for the longest), and the row's copy
+    if (tid == 0) {
       s_t = 0; s_sym = 0; s_cnt = 0;
-    } else {
-      s_t = __ldcg(d.r_t + r); s_sym = __ldcg(d.r_sym + r); s_cnt = __ldcg(d.r_cnt + r);
+      s_nl = d.has_lm ? __ldcg(d.s_lm_len + slot) : 0;
+      s_nt = d.has_tr ? __ldcg(d.s_tr_len + slot) : 0;
+      s_last = __ldcg(d.s_last + slot);
+      if (commit) {
+        d.m_lm_len[r] = s_nl;
+        d.m_tr_len[r] = s_nt;
+        d.m_last[r] = s_last;
+      }
+    } else if (tid >= 32 && tid < 32 + kLmChain) {
+      const int l = tid - 32;
+      if (d.has_lm) {
+        s_lm[l] = __ldcg(d.s_lm_chain + (size_t)slot * kLmChain + l);
+        s_lmr[l] = __ldcg(d.s_lm_rec + (size_t)slot * kLmChain + l);
+        if (commit) {
+          d.m_lm[(size_t)r * kLmChain + l] = s_lm[l];
+          d.m_lmr[(size_t)r * kLmChain + l] = s_lmr[l];
+        }
+      }
+    } else if (tid >= 64 && tid < 64 + kTrChain) {
+      const int k = tid - 64;
+      if (d.has_tr) {
+        s_tr[k] = __ldcg(d.s_tr_chain + slot * kTrChain + k);
+        s_trr[k] = __ldcg(d.s_tr_rec + (size_t)slot * kTrChain + k);
+        if (commit) {
+          d.m_tr[(size_t)r * kTrChain + k] = s_tr[k];
+          d.m_trr[(size_t)r * kTrChain + k] = s_trr[k];
+        }
+      }
     }
-    s_nl = d.has_lm ? __ldcg(d.s_lm_len + slot) : 0;
-    s_nt = d.has_tr ? __ldcg(d.s_tr_len + slot) : 0;
-    s_last = __ldcg(d.s_last + slot);
-  } else if (tid >= 32 && tid < 32 + kLmChain) {
-    const int l = tid - 32;
-    if (d.has_lm) {
-      s_lm[l] = __ldcg(d.s_lm_chain + (size_t)slot * kLmChain + l);
-      s_lmr[l] = __ldcg(d.s_lm_rec + (size_t)slot * kLmChain + l);
-    }
-  } else if (tid >= 64 && tid < 64 + kTrChain) {
-    const int k = tid - 64;
-    if (d.has_tr) {
-      s_tr[k] = __ldcg(d.s_tr_chain + slot * kTrChain + k);
-      s_trr[k] = __ldcg(d.s_tr_rec + (size_t)slot * kTrChain + k);
-    }
+    row::block_sync();
   }
-  row::block_sync();
 #ifdef TSD_CHECKS
   if (tid == 0) {  // every index the row will follow is inside its table
     bool ok = checked(s_nl >= 0 && s_nl <= kLmChain && s_nt >= 0 && s_nt <= kTrChain, d.err, 2) &&
@@ -297,12 +333,14 @@ __global__ void __launch_bounds__(kFzThreads) __maxnreg__((VAR & 4) ? 128 : 72) 
       s_bi[warp] = bi;
     }
     row::block_sync();
-    if (tid == 0) {
-      float b = s_bv[0];
-      int i = s_bi[0];
+    // every thread merges the warps' bests (no second barrier)
+    float b = s_bv[0];
+    int bix = s_bi[0];
 #pragma unroll
-      for (int w = 1; w < kFzWarps; ++w) best_merge(b, i, s_bv[w], s_bi[w]);
-      s_y = (i >= 0 && i <= V) ? i : V;
+    for (int w = 1; w < kFzWarps; ++w) best_merge(b, bix, s_bv[w], s_bi[w]);
+    const int y = (bix >= 0 && bix <= V) ? bix : V;
+    if (tid == 0) {
+      s_y = y;
       s_score = (b + cr_prev) - s_lse;
       if (counting) {
         // algorithmic bytes of the decision: partials, the list and its
@@ -310,11 +348,9 @@ __global__ void __launch_bounds__(kFzThreads) __maxnreg__((VAR & 4) ? 128 : 72) 
         // records read
         unsigned long long ab = 16ull * d.n_ptiles + 12ull * ci.y + 4 + 16;
         ab += 2ull * (24 + 4 * (nl_old + nt_old)) + 16ull * (nl_old + nt_old);
-        s_bytes = ab;
+        atomicAdd(&s_bytes, ab);
       }
     }
-    row::block_sync();
-    const int y = s_y;
     if (!PRED) row::prefetch_span(d.E + (size_t)(y != V ? y : s_last) * d.H, (size_t)d.H * 2, 32);
     if (y != V) {
       // 3a. independent searches of y in every chain element; each hit's
@@ -369,12 +405,17 @@ __global__ void __launch_bounds__(kFzThreads) __maxnreg__((VAR & 4) ? 128 : 72) 
             if (commit) {
               d.s_lm_chain[(size_t)slot * kLmChain + lane] = nst;
               d.s_lm_rec[(size_t)slot * kLmChain + lane] = nrec;
+              d.m_lm[(size_t)r * kLmChain + lane] = nst;
+              d.m_lmr[(size_t)r * kLmChain + lane] = nrec;
             }
           }
         }
         if (lane == 0) {
           s_nl = ln;
-          if (commit && d.has_lm) d.s_lm_len[slot] = ln;
+          if (commit && d.has_lm) {
+            d.s_lm_len[slot] = ln;
+            d.m_lm_len[r] = ln;
+          }
         }
       } else if (warp == 1) {
         const int4 h = lane < nt_old ? s_tr_hit[lane] : make_int4(-1, 0, 0, 0);
@@ -404,10 +445,15 @@ __global__ void __launch_bounds__(kFzThreads) __maxnreg__((VAR & 4) ? 128 : 72) 
         if (commit && lane < tn) {
           d.s_tr_chain[slot * kTrChain + lane] = s_tr[lane];
           d.s_tr_rec[(size_t)slot * kTrChain + lane] = s_trr[lane];
+          d.m_tr[(size_t)r * kTrChain + lane] = s_tr[lane];
+          d.m_trr[(size_t)r * kTrChain + lane] = s_trr[lane];
         }
         if (lane == 0) {
           s_nt = tn;
-          if (commit && d.has_tr) d.s_tr_len[slot] = tn;
+          if (commit && d.has_tr) {
+            d.s_tr_len[slot] = tn;
+            d.m_tr_len[r] = tn;
+          }
         }
       } else if (tid == 64) {
         if (commit) {
@@ -417,6 +463,7 @@ __global__ void __launch_bounds__(kFzThreads) __maxnreg__((VAR & 4) ? 128 : 72) 
           s_out_frame[o] = s_t;
           s_out_score[o] = s_score;
           d.s_last[slot] = y;
+          d.m_last[r] = y;
         }
         s_cnt += 1;
         s_last = y;
@@ -502,8 +549,49 @@ __global__ void __launch_bounds__(kFzThreads) __maxnreg__((VAR & 4) ? 128 : 72) 
       const int depth_cur = nt ? s_trr[0].z - 1 : 0;
       s_cr = lam * cum_top - bscale * (float)depth_cur;
     }
+  } else if (warp == 1) {  // the trie chain's children before each node
+    const int c = lane < nt ? s_trr[lane].y : 0;
+    int incl = c;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int v = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += v;
+    }
+    s_tpre[lane + 1] = incl;
+    if (lane == 0) s_tpre[0] = 0;
   }
   row::block_sync();
+  // the trie chain's children, one per thread while they fit (label, node,
+  // and later its level-0 LM term); otherwise every phase reads them again
+  const int TC = s_tpre[nt];
+  const bool tr_held = TC <= kTrHeld * kFzThreads;
+  const int drow = (d.has_lm && nl >= 1) ? s_lmr[0].w : -1;
+  const float* dense = drow >= 0 ? d.lm.dense0 + (size_t)drow * d.V4 : nullptr;
+  int trv[kTrHeld], trk[kTrHeld];
+  float trl[kTrHeld];
+#pragma unroll
+  for (int u = 0; u < kTrHeld; ++u) {
+    const int f = tid + u * kFzThreads;
+    trv[u] = -1;
+    trk[u] = -1;
+    trl[u] = 0.f;
+    if (tr_held && f < TC) {
+      int k = 0;
+      while (f >= s_tpre[k + 1]) ++k;
+      trk[u] = k;
+      trv[u] = __ldg(d.tr.ch_tok + s_trr[k].x + (f - s_tpre[k]));
+    }
+  }
+  // node k's children write their goto depth (phases run shallowest first)
+  auto trie_phase = [&](int k) {
+    if (!tr_held) {
+      row::scatter_trie_node(d.tr.ch_tok, s_trr[k].x, s_trr[k].x + s_trr[k].y, (uint8_t)s_trr[k].z, dep);
+      return;
+    }
+#pragma unroll
+    for (int u = 0; u < kTrHeld; ++u)
+      if (trk[u] == k && checked(trv[u] >= 0 && trv[u] < V, d.err, 15)) dep[trv[u]] = (uint8_t)s_trr[k].z;
+  };
   const int4* t4 = reinterpret_cast<const int4*>(d.lm.arc_tok);
   const float4* p4 = reinterpret_cast<const float4*>(d.lm.arc_logp);
   // the group g of levels 1..: its level and first arc
@@ -552,10 +640,12 @@ __global__ void __launch_bounds__(kFzThreads) __maxnreg__((VAR & 4) ? 128 : 72) 
     const int i0 = locate(g, l);
     offer(l, i0, __ldg(t4 + (i0 >> 2)));
   }
-  if (nt > 0) {
-    const int k = nt - 1;
-    row::scatter_trie_node(d.tr.ch_tok, s_trr[k].x, s_trr[k].x + s_trr[k].y, (uint8_t)s_trr[k].z, dep);
-  }
+  if (nt > 0) trie_phase(nt - 1);
+  // the held children's level-0 LM terms (used if a child is not a level-1 label)
+#pragma unroll
+  for (int u = 0; u < kTrHeld; ++u)
+    if (d.has_lm && trv[u] >= 0 && trv[u] < V)
+      trl[u] = lam * ((dense ? __ldg(dense + trv[u]) : 0.f) + __ldg(d.lm.uni_logp + trv[u]));
   row::block_sync();
   // 4b. the winners among the held offers (one per label) compute their LM
   //     term; it is written once every offer is judged
@@ -579,10 +669,7 @@ __global__ void __launch_bounds__(kFzThreads) __maxnreg__((VAR & 4) ? 128 : 72) 
       }
     }
   }
-  if (nt > 1) {
-    const int k = nt - 2;
-    row::scatter_trie_node(d.tr.ch_tok, s_trr[k].x, s_trr[k].x + s_trr[k].y, (uint8_t)s_trr[k].z, dep);
-  }
+  if (nt > 1) trie_phase(nt - 2);
   row::block_sync();
 #pragma unroll
   for (int u = 0; u < kHeld; ++u) {
@@ -631,7 +718,7 @@ __global__ void __launch_bounds__(kFzThreads) __maxnreg__((VAR & 4) ? 128 : 72) 
   }
   for (int k = nt - 3; k >= 0; --k) {
     row::block_sync();
-    row::scatter_trie_node(d.tr.ch_tok, s_trr[k].x, s_trr[k].x + s_trr[k].y, (uint8_t)s_trr[k].z, dep);
+    trie_phase(k);
   }
   row::block_sync();
   // 4c. the list: level 1's arcs in order (every label of a deeper level is
@@ -640,18 +727,50 @@ __global__ void __launch_bounds__(kFzThreads) __maxnreg__((VAR & 4) ? 128 : 72) 
     int32_t* cl = d.c_lab + (size_t)r * d.V4;
     float* ca = d.c_add + (size_t)r * d.V4;
     const int b1 = nl >= 2 ? s_lmr[1].x : 0, c1 = nl >= 2 ? s_lmr[1].y : 0;
-    for (int j = tid; j < c1; j += kFzThreads) {
-      const int v = __ldg(d.lm.arc_tok + b1 + j);
-      if (!checked(v >= 0 && v < V && lmf[v] != 0, d.err, 14)) continue;
+    auto emit1 = [&](int j, int v) {  // level-1 arc j, label v
+      if (!checked(v >= 0 && v < V && lmf[v] != 0, d.err, 14)) return;
       const uint32_t e = dep[v];
-      const float tr = e ? bscale * (float)e : (((__ldg(d.droot + (v >> 5)) >> (v & 31)) & 1u) ? bscale : 0.f);
+      const float tr = e ? bscale * (float)e : (((rootw[v >> 5] >> (v & 31)) & 1u) ? bscale : 0.f);
       cl[j] = v;
       ca[j] = __uint_as_float(key[v]) + tr;
       atomicOr(msk + (v >> 5), 1u << (v & 31));
+    };
+    // level 1's arcs: the groups held in registers since the offers, then
+    // the rest (groups 0 .. G1-1 of levels 1.. are level 1's)
+#pragma unroll
+    for (int u = 0; u < kHeld; ++u) {
+      if (hl[u] == 1) {
+        const int tv[4] = {ht[u].x, ht[u].y, ht[u].z, ht[u].w};
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          const int i = hi[u] + j;
+          if (i >= b1 && i < b1 + c1) emit1(i - b1, tv[j]);
+        }
+      }
     }
-    const int drow = (d.has_lm && nl >= 1) ? s_lmr[0].w : -1;
-    const float* dense = drow >= 0 ? d.lm.dense0 + (size_t)drow * d.V4 : nullptr;
-    for (int k = 0; k < nt; ++k) {
+    const int G1 = nl >= 2 ? s_gbeg[2] : 0;
+    for (int g = tid + kHeld * kFzThreads; g < G1; g += kFzThreads) {
+      const int i0 = (b1 & ~3) + 4 * g;
+      const int4 tk = __ldg(t4 + (i0 >> 2));
+      const int tv[4] = {tk.x, tk.y, tk.z, tk.w};
+#pragma unroll
+      for (int j = 0; j < 4; ++j)
+        if (i0 + j >= b1 && i0 + j < b1 + c1) emit1(i0 + j - b1, tv[j]);
+    }
+    auto emit_tr = [&](int v, uint32_t dd, float lmv) {  // a child that is not a level-1 label
+      const int j = c1 + atomicAdd(&s_ext, 1);
+      cl[j] = v;
+      ca[j] = lmv + bscale * (float)dd;
+      atomicOr(msk + (v >> 5), 1u << (v & 31));
+    };
+#pragma unroll
+    for (int u = 0; u < kTrHeld; ++u) {
+      if (trk[u] >= 0 && trv[u] >= 0 && trv[u] < V) {
+        const uint32_t dd = (uint32_t)s_trr[trk[u]].z;
+        if (dep[trv[u]] == dd && lmf[trv[u]] == 0) emit_tr(trv[u], dd, trl[u]);
+      }
+    }
+    for (int k = 0; !tr_held && k < nt; ++k) {
       const int b = s_trr[k].x, c = s_trr[k].y;
       const uint32_t dd = (uint32_t)s_trr[k].z;
       for (int i = tid; i < c; i += kFzThreads) {
@@ -659,10 +778,7 @@ __global__ void __launch_bounds__(kFzThreads) __maxnreg__((VAR & 4) ? 128 : 72) 
         if (!checked(v >= 0 && v < V, d.err, 15) || dep[v] != dd || lmf[v] != 0) continue;
         float lmv = 0.f;  // the LM term when the deepest arc is level 0's, or none
         if (d.has_lm) lmv = lam * ((dense ? __ldg(dense + v) : 0.f) + __ldg(d.lm.uni_logp + v));
-        const int j = c1 + atomicAdd(&s_ext, 1);
-        cl[j] = v;
-        ca[j] = lmv + bscale * (float)dd;
-        atomicOr(msk + (v >> 5), 1u << (v & 31));
+        emit_tr(v, dd, lmv);
       }
     }
     if (tid == 0) atomicOr(msk + (V >> 5), 1u << (V & 31));  // blank is always evaluated by the row pass
@@ -684,7 +800,7 @@ __global__ void __launch_bounds__(kFzThreads) __maxnreg__((VAR & 4) ? 128 : 72) 
 }  // namespace
 
 size_t row_fused_smem_bytes(int V4, int N_pad) {
-  return (size_t)V4 * (sizeof(uint32_t) + 2 * sizeof(uint8_t)) + sizeof(uint32_t) * (size_t)(N_pad / 32);
+  return (size_t)V4 * (sizeof(uint32_t) + 2 * sizeof(uint8_t)) + 2 * sizeof(uint32_t) * (size_t)(N_pad / 32);
 }
 
 cudaError_t prepare_fused_kernels(size_t smem) {
