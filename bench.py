@@ -220,6 +220,8 @@ def variant_config(args, w, extra):
     if args.prune_k:
         out["prune_k"] = args.prune_k
         names.append(f"fusion pruned to the acoustic top {args.prune_k}")
+    if w.beam == 1 and not args.prune_k and not extra:
+        out["fusion_path"] = 0 if args.fusion_path == 0 else 1
     if args.pred:
         out["prediction_network"] = {"kind": "1-layer LSTM over the previous label", "D": args.pred, "H_enc": w.H}
         names.append(f"stateful form: LSTM prediction network D={args.pred} + joint projections")
@@ -341,6 +343,8 @@ def stream_sweep(args, w, tsd, dev, stream, W, E, lm, lms, bo, pw, flush):
                         torch.from_numpy(E.view(np.int16)).to(dev), lm=None if lms else lm, lms=lms, boost=bo,
                         max_symbols=w.max_sym, beam_k=w.beam, max_streams=B, max_T=w.T, prune_k=args.prune_k,
                         pred=pw)
+        if w.beam == 1 and not args.prune_k and not lms and args.fusion_path is not None:
+            d.set_option("fusion_path", args.fusion_path)
         sl = np.array([d.open() for _ in range(B)], dtype=np.int32)
         encs = [torch.from_numpy(synth.enc_chunk(w, range(B), c % w.chunks).view(np.int16)).to(dev)
                 for c in range(args.warmup + args.steps)]
@@ -390,6 +394,11 @@ def run_ours(args, w):
     dec = tsd.Decoder(w.V, w.H, torch.from_numpy(W.view(np.int16)).to(dev), torch.from_numpy(E.view(np.int16)).to(dev),
                       lm=None if lms else lm, lms=lms, boost=bo, max_symbols=w.max_sym, beam_k=w.beam,
                       max_streams=w.B, max_T=w.T, prune_k=args.prune_k, pred=pw)
+    greedy1 = w.beam == 1 and not args.prune_k and not extra  # greedy decoding with at most one LM
+    if greedy1:
+        if args.fusion_path is None:  # the decoder's default: the dense epilogue from V = 2048 up
+            args.fusion_path = 1 if w.V >= 2048 else 0
+        dec.set_option("fusion_path", args.fusion_path)
     for kv in args.set or []:
         k, v = kv.split("=")
         dec.set_option(k, int(v))
@@ -554,6 +563,50 @@ def run_ours(args, w):
                       **{k: v for k, v in latency_stats(step_ms).items() if k != "steps"}})
         sweep.sort(key=lambda x: x["B"])
 
+    # the other form of the greedy one-LM step on the same decoder and inputs
+    # (fusion_path switched, graphs recaptured): its throughput and its two
+    # kernels' production-graph figures
+    alt = None
+    if greedy1 and ws == 1 and not args.no_alt_path:
+        alt_path = 1 - args.fusion_path
+        dec.set_option("fusion_path", alt_path)
+        for c in range(args.warmup):
+            step(c)
+        barrier()
+        a_ms, _, _ = timed_loop(args.warmup)
+        dec.set_timing(True)
+        for c in range(2):
+            step(args.warmup + c)
+        barrier()
+        dec.timing(reset=True)
+        dec.timed_bytes(reset=True)
+        timed_loop(args.warmup)
+        a_kms, a_kn = dec.timing(reset=True)
+        a_bytes = dec.timed_bytes(reset=True)
+        dec.set_timing(False)
+        a_tot = max(1e-9, sum(a_kms.values()))
+        a_step = a_ms / args.steps
+        a_shared = 0 if alt_path == 1 else w.V * ((4 if lmA is not None else 0) + (4 if ph is not None else 0))
+        a_row_bytes = (a_bytes + a_shared * max(0, a_kn["row"] - args.steps)) / max(1, a_kn["row"])
+        pk_a, pk_a_kind = peaks()
+        a_joint_ms = a_step * (a_kms["joint"] / a_tot) / max(1e-9, a_kn["joint"] / args.steps)
+        a_row_ms = a_step * (a_kms["row"] / a_tot) / max(1e-9, a_kn["row"] / args.steps)
+        a_flop = 2.0 * w.B * w.H * (w.V + 1)
+        alt = {"fusion_path": alt_path,
+               "what": ("the same workload and decoder with the alt_path form of the greedy one-LM step: "
+                        + ("the LM level-0 term in the joint epilogue with a per-row correction list" if alt_path
+                           else "the streaming form (the joint writes every logit + defaults, the row pass "
+                                "applies the LM and trie terms)")),
+               "value": w.B * w.T * args.steps / (a_ms / 1000.0), "unit": "frames/s", "ms_per_step": a_step,
+               "joint": {"kernel": "k_joint_greedy<dense>" if alt_path else "k_joint_greedy<streaming>",
+                         "avg_launch_ms": a_joint_ms, "achieved_tflops": a_flop / (a_joint_ms / 1000.0) / 1e12,
+                         "frac": a_flop / (a_joint_ms / 1000.0) / 1e12 / pk_a["bf16_tflops_sustained"],
+                         "peak_kind": f"{pk_a_kind} bf16 sustained"},
+               "row": {"kernel": "k_row_ep" if alt_path else "k_row_fz", "avg_launch_ms": a_row_ms,
+                       "bytes_per_launch": a_row_bytes, "achieved_gbs": a_row_bytes / (a_row_ms / 1000.0) / 1e9,
+                       "frac": a_row_bytes / (a_row_ms / 1000.0) / 1e9 / pk_a["hbm_gbs"],
+                       "peak_kind": f"{pk_a_kind} HBM copy"},
+               "timing": "as the headline kernels: uninstrumented step time x device-time share / launches per step"}
     clk.__exit__(None, None, None)
     if rank != 0:
         return
@@ -569,14 +622,18 @@ def run_ours(args, w):
     # inside a long step takes the sustained bf16 peak.
     joint_ms = kernel_ms["joint"] / max(1, kernel_n["joint"])
     row_ms = kernel_ms["row"] / max(1, kernel_n["row"])
-    # the greedy one-LM pass (k_row_ep) reads no shared V-wide row; the others
-    # read the call's unigram and root rows once per launch
-    ep = w.beam == 1 and not args.prune_k and not extra
+    # the greedy one-LM pass with the correction list (k_row_ep) reads no
+    # shared V-wide row; the others read the call's unigram and root rows once
+    # per launch
+    ep = greedy1 and args.fusion_path != 0
+    fz_stream = greedy1 and args.fusion_path == 0
     shared_rows = 0 if ep else w.V * ((4 * (1 + len(extra)) if lmA is not None else 0) + (4 if ph is not None else 0))
     row_launches_with_bias = kernel_n["row"] - args.steps  # the final row pass of a chunk builds no bias
     row_bytes_graph = row_timed_bytes + shared_rows * max(0, row_launches_with_bias)
-    joint_roof = {"kernel": ("k_joint_tc: joint GEMM (tcgen05) + epilogue applying Eq. 1 with the dense LM row, "
-                             "log-softmax and selection partials") if ep else
+    joint_roof = {"kernel": ("k_joint_greedy<dense>: joint GEMM (tcgen05) + epilogue applying Eq. 1 with the dense "
+                             "LM row, log-softmax and selection partials") if ep else
+                            ("k_joint_greedy<streaming>: joint GEMM (tcgen05) + epilogue writing logit + defaults "
+                             "(TMA stores) and log-softmax partials") if fz_stream else
                             "k_joint_tc: joint GEMM (tcgen05) + fused log-softmax/selection epilogue",
                   "bound": "tensor", "unit": "TFLOP/s",
                   "achieved": flop_per_launch / (joint_ms / 1000.0) / 1e12,
@@ -592,9 +649,12 @@ def run_ours(args, w):
                                "achieved_warm": flop_per_launch / (joint_warm / 1000.0) / 1e12,
                                "peak": pk["bf16_tflops"], "peak_kind": f"{pk_kind} bf16 burst"}}
     joint_roof["frac"] = joint_roof["achieved"] / joint_roof["peak"]
-    row_roof = {"kernel": "k_row_beam" if w.beam > 1 else ("k_row_ep" if ep else "k_row"),
+    row_roof = {"kernel": "k_row_beam" if w.beam > 1 else ("k_row_ep" if ep else ("k_row_fz" if fz_stream else "k_row")),
                 "what": ("decision from the tile partials and the correction list, LM/trie state advance, "
                          "the new state's correction list and mask, joint input") if ep else
+                        ("the row's LM and trie deltas (every arc of its LM chain levels, its dense level-0 row, "
+                         "the trie chain's children), argmax over the fused logits, state advance, joint input")
+                        if fz_stream else
                         "selection merge, LM/trie state advance, joint input, fusion bias",
                 "bound": "hbm", "unit": "GB/s",
                 "achieved": row_bytes_graph / (kernel_ms["row"] / 1000.0) / 1e9,
@@ -603,6 +663,11 @@ def run_ours(args, w):
                                 f"counted by the kernel per row (partials, the correction list read with its "
                                 f"logits and written, the mask, row state, label searches, every arc of the LM "
                                 f"chain levels 1.. and every child of the trie chain nodes, joint input)") if ep else
+                               (f"{row_bytes_graph / max(1, kernel_n['row']):.0f} B per launch on average, "
+                                f"counted by the kernel per evaluated row (the fused logits read back, partials, "
+                                f"row state, label searches, joint input, every arc of the LM chain levels above "
+                                f"0, the dense level-0 row, every child of the trie chain nodes) plus the shared "
+                                f"unigram/root rows once per launch") if fz_stream else
                                (f"{row_bytes_graph / max(1, kernel_n['row']):.0f} B per launch on average, "
                                 f"counted by the kernel per evaluated row (partials, row state, label searches, "
                                 f"joint input, every arc of the LM chain levels and trie chain nodes) plus the "
@@ -728,6 +793,7 @@ def run_ours(args, w):
             "roofline_other_kernel": other,
             **({"roofline_third_kernel": ranked[2][1]} if len(ranked) > 2 else {}),
             "latency_per_chunk": latency_stats(step_ms),
+            **({"alt_fusion_path": alt} if alt else {}),
             **({"stream_sweep": {"what": "the same workload (tables, weights, lambda, beta) decoded at other stream "
                                          "counts B in this run: frames/s over K timed chunks (L2 flushed before "
                                          "each) and chunk latency; 1 chunk = T x 80 ms of audio",
@@ -777,6 +843,11 @@ def main():
                     help="pruned fusion over the acoustic model's k best outputs (0: every label)")
     ap.add_argument("--pred", type=int, default=0,
                     help="stateful form: an LSTM prediction network of this many units (0: stateless)")
+    ap.add_argument("--fusion-path", type=int, default=None, choices=(0, 1),
+                    help="greedy decoding with at most one LM: 1 = the LM level-0 term in the joint epilogue "
+                         "(the decoder's default), 0 = the streaming form")
+    ap.add_argument("--no-alt-path", action="store_true",
+                    help="skip timing the other form of the greedy one-LM step (fusion_path)")
     ap.add_argument("--set", action="append", metavar="NAME=VALUE",
                     help="a decoder tuning option (tsd_decoder_set_option), e.g. pdl=0 or joint_bn=128")
     ap.add_argument("--encoder", default=None, choices=sorted(synth.ENCODERS),

@@ -362,6 +362,15 @@ TSD_API tsd_status tsd_decoder_check(tsd_decoder* dec);
  *              overlaps the tail of the one before;
  *   "joint_bn" 64, 128 or 256: labels per tensor-core CTA tile (default:
  *              chosen at create from the row count and the SM count);
+ *   "fusion_path" 0 or 1, greedy decoding with at most one LM (default 1
+ *              from V = 2048 up, else 0):
+ *              1 applies Eq. 1's level-0 LM term (a dense row per unigram
+ *              state) in the joint kernel's epilogue and evaluates the other
+ *              labels of the row's state (its longer contexts' continuations,
+ *              the trie chain's children, blank) in the row pass; 0 is the
+ *              streaming form, in which the joint kernel writes every logit
+ *              and the row pass applies the whole LM and trie terms.  Both
+ *              give the same decisions; TSD_EINVAL for other decoders;
  *   "wait_ns"  0 .. 1e10: the limit, in nanoseconds, of the joint kernel's
  *              waits for its operands and accumulator (default 1e9).  A wait
  *              that expires ends the kernel early -- after it has waited,

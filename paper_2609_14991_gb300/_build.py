@@ -23,7 +23,7 @@ LIB_PATH = os.path.join(PKG, "libtsd.so")
 CHECKS_BUILD_DIR = os.path.join(PKG, "_build_checks")
 CHECKS_LIB_PATH = os.path.join(PKG, "libtsd_checks.so")
 
-SOURCES = ["tables.cpp", "arpa.cpp", "decoder.cu", "row_pass.cu", "row_fused.cu", "joint_simt.cu", "joint_tc.cu", "joint_dense.cu", "noalloc.cu", "row_beam.cu", "row_pruned.cu", "gemm_tc.cu", "encoder.cu", "encoder_gemm.cu"]
+SOURCES = ["tables.cpp", "arpa.cpp", "decoder.cu", "row_pass.cu", "row_fused.cu", "row_stream.cu", "joint_simt.cu", "joint_tc.cu", "joint_greedy.cu", "noalloc.cu", "row_beam.cu", "row_pruned.cu", "gemm_tc.cu", "encoder.cu", "encoder_gemm.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

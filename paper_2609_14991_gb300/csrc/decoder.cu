@@ -71,7 +71,8 @@ void enqueue_chunk(tsd_decoder* d, int M, int T, cudaStream_t s, const std::vect
     mark(0);
     if (d->cfg.beam_k > 1) launch_row_beam(v, M / d->cfg.beam_k, step, step == S ? 1 : 0, d->row_smem, s, pdl);
     else if (d->cfg.prune_k > 0) launch_row_pruned(v, M, step, step == S ? 1 : 0, s, pdl);
-    else if (v.fused) launch_row_fused(v, M, step, step == S ? 1 : 0, d->row_smem, s, pdl);
+    else if (v.fused && v.fz_dense) launch_row_fused(v, M, step, step == S ? 1 : 0, d->row_smem, s, pdl);
+    else if (v.fused) launch_row_stream(v, M, step, step == S ? 1 : 0, d->row_smem, s, pdl);
     else launch_row(v, M, step, step == S ? 1 : 0, d->row_smem, s, pdl);
     if (pr.D) {
       // the prediction network reads the labels just emitted; after the last
@@ -181,7 +182,8 @@ tsd_status create_impl(const tsd_decoder_cfg* cfg, const void* W_out_bf16, const
   const bool fused = c.beam_k == 1 && c.prune_k == 0 && n_lms <= 1 &&
                      (n_lms == 0 || !lm_weights || lm_weights[0] == 1.f) &&
                      (!lm || lm->view.order < 2 || lm->view.n_dense == lm->view.V);
-  d->row_smem = fused ? row_fused_smem_bytes(d->V4, d->N_pad) : row_smem_bytes(d->V4, n_lms);
+  d->row_smem = fused ? std::max(row_fused_smem_bytes(d->V4, d->N_pad), row_stream_smem_bytes(d->V4))
+                      : row_smem_bytes(d->V4, n_lms);
   if (d->row_smem > 200 * 1024) return fail(TSD_EINVAL, "tsd_decoder_create: V too large for the row pass");
 
   DevArena& A = d->arena;
@@ -233,6 +235,9 @@ tsd_status create_impl(const tsd_decoder_cfg* cfg, const void* W_out_bf16, const
     TSD_CUDA(cudaMemsetAsync(v.c_mask, 0, sizeof(uint32_t) * (size_t)d->M_pad * v.mask_words, s));
   }
   v.fused = fused ? 1 : 0;
+  // the dense epilogue pays off with a wide vocabulary (its row pass no longer
+  // scans every label); with a narrow one the streaming form is faster
+  v.fz_dense = c.V >= 2048 ? 1 : 0;
   const int topk = c.beam_k > 1 ? c.beam_k : c.prune_k;
   if (c.beam_k == 1 && c.prune_k > 0) {
     if ((st = A.alloc(&bpart, (size_t)d->M_pad * (d->N_pad / 64) * (1 + topk)))) {
@@ -336,7 +341,8 @@ tsd_status create_impl(const tsd_decoder_cfg* cfg, const void* W_out_bf16, const
   }
   if ((ce = prepare_kernels(row_smem_bytes(d->V4, n_lms))) != cudaSuccess)
     return cleanup(cuda_fail(ce, "tsd_decoder_create: kernel attributes"));
-  if (fused && (ce = prepare_fused_kernels(d->row_smem)) != cudaSuccess)
+  if (fused && ((ce = prepare_fused_kernels(d->row_smem)) != cudaSuccess ||
+                (ce = prepare_stream_kernels(d->row_smem)) != cudaSuccess))
     return cleanup(cuda_fail(ce, "tsd_decoder_create: kernel attributes"));
   if ((ce = prepare_beam_kernels(d->row_smem)) != cudaSuccess) return cleanup(cuda_fail(ce, "tsd_decoder_create: kernel attributes"));
   if (hlive && (ce = cudaMemsetAsync(hlive, 0, sizeof(int32_t) * SK, s)) != cudaSuccess)
@@ -350,7 +356,7 @@ tsd_status create_impl(const tsd_decoder_cfg* cfg, const void* W_out_bf16, const
     d->sms = sms;
     d->view.sms = sms;
     const int bn = joint_tc_pick_bn(d->M_max, d->N_pad, sms);
-    if ((ce = joint_tc_prepare(d->jtc, Abuf, d->M_pad, Wt, d->N_pad, c.H, bn, bias)) != cudaSuccess)
+    if ((ce = joint_tc_prepare(d->jtc, Abuf, d->M_pad, Wt, d->N_pad, c.H, bn, bias, v.logits)) != cudaSuccess)
       return cleanup(cuda_fail(ce, "tsd_decoder_create: tensor-core GEMM setup (TMA descriptors)"));
   }
   for (int i = 0; i < tsd_decoder::kRing; ++i) {
@@ -1017,12 +1023,21 @@ extern "C" tsd_status tsd_decoder_set_option(tsd_decoder* d, const char* name, i
     d->view.wait_ns = (unsigned long long)value;
     return drop_graphs(d);
   }
+  if (n == "fusion_path") {
+    // greedy decoding with at most one LM: 1 = Eq. 1's level-0 LM term in the
+    // joint kernel's epilogue with a per-row correction list, 0 = the
+    // streaming form (the row pass applies the LM and trie terms)
+    if (value != 0 && value != 1) return fail(TSD_EINVAL, "tsd_decoder_set_option: fusion_path must be 0 or 1");
+    if (!d->view.fused) return fail(TSD_EINVAL, "tsd_decoder_set_option: fusion_path applies to greedy decoding with at most one LM");
+    d->view.fz_dense = (int32_t)value;
+    return drop_graphs(d);
+  }
   if (n == "joint_bn") {
     if (value != 64 && value != 128 && value != 256) return fail(TSD_EINVAL, "tsd_decoder_set_option: joint_bn must be 64, 128 or 256");
     tsd_status st = drop_graphs(d);
     if (st) return st;
     cudaError_t ce = joint_tc_prepare(d->jtc, d->view.A, d->M_pad, d->view.Wt, d->N_pad, d->cfg.H, (int)value,
-                                      d->view.bias);
+                                      d->view.bias, d->view.logits);
     if (ce != cudaSuccess) return cuda_fail(ce, "tsd_decoder_set_option: joint_bn");
     if (d->joint_kind == 0) {
       d->n_ptiles = d->N_pad / d->jtc->bn;
@@ -1049,7 +1064,8 @@ extern "C" tsd_status tsd_decoder_replay(tsd_decoder* d, int32_t kernel, int32_t
   for (int i = 0; i < reps; ++i) {
     if (kernel == 0 && d->cfg.beam_k > 1) launch_row_beam(d->view, d->last_n, S - 1, 2, d->row_smem, s, false);
     else if (kernel == 0 && d->cfg.prune_k > 0) launch_row_pruned(d->view, M, S - 1, 2, s, false);
-    else if (kernel == 0 && d->view.fused) launch_row_fused(d->view, M, S - 1, 2, d->row_smem, s, false);
+    else if (kernel == 0 && d->view.fused && d->view.fz_dense) launch_row_fused(d->view, M, S - 1, 2, d->row_smem, s, false);
+    else if (kernel == 0 && d->view.fused) launch_row_stream(d->view, M, S - 1, 2, d->row_smem, s, false);
     else if (kernel == 0) launch_row(d->view, M, S - 1, 2, d->row_smem, s, false);
     else if (d->joint_kind == 0) launch_joint_tc(*d->jtc, d->view, M, 1 << 30, s, false);
     else launch_joint(d->view, M, 1 << 30, s);
@@ -1063,6 +1079,11 @@ extern "C" tsd_status tsd_decoder_replay(tsd_decoder* d, int32_t kernel, int32_t
       // per launch, plus the dense unigram and root rows every launch reads once
       const int64_t shared = (int64_t)d->cfg.V * ((d->lm ? 4 : 0) + (d->boost ? 4 : 0));
       *algo_bytes = (int64_t)(b / (unsigned long long)reps) + shared;
+    } else if (d->view.fused && !d->view.fz_dense) {
+      // joint, streaming epilogue: the operands once (A rows, W_out), the
+      // logits written and the softmax partials
+      *algo_bytes = (int64_t)M * d->cfg.H * 2 + (int64_t)d->N * d->cfg.H * 2 + (int64_t)M * d->N * 4 +
+                    (int64_t)M * d->n_ptiles * 8;
     } else if (d->view.fused) {
       // joint, dense epilogue: the operands once (A rows, W_out), each row's
       // dense LM row and mask, the defaults, the partials written (the

@@ -103,8 +103,12 @@ struct DecView {
   // blank) are the row's correction list, written by the row pass before
   // the joint runs: the joint leaves them out of its per-tile best and
   // stores their raw logits; the next row pass evaluates them from the list.
+  // fusion_path 0 (fz_dense = 0): the streaming form: the joint kernel
+  // writes logit + dvec for every label and the row pass (row_stream.cu)
+  // adds the row's LM and trie terms before it takes the argmax.
   int32_t fused;
-  float* logits;        // [M_pad][N_pad] fp32 raw logits of the listed labels (other entries unused)
+  int32_t fz_dense;     // 1: the dense epilogue with the correction list; 0: streaming
+  float* logits;        // [M_pad][N_pad] fp32: the listed labels' raw logits (dense) or every label's logit + dvec
   float* dvec;          // [N_pad] per call: lambda*log p(v) + beta*bonus*[the root has a child v]; 0 from V on
   int32_t* c_lab;       // [M_pad][V4] the row's listed labels
   float* c_add;         // [M_pad][V4] their term: F[v] = logit[v] + c_add
@@ -139,6 +143,9 @@ void launch_copy_enc(const DecView& d, int64_t elems, cudaStream_t s, bool pdl);
 void launch_row(const DecView& d, int M, int step, int mode, size_t smem, cudaStream_t s, bool pdl);
 void launch_row_fused(const DecView& d, int M, int step, int mode, size_t smem, cudaStream_t s, bool pdl);
 cudaError_t prepare_fused_kernels(size_t smem);
+void launch_row_stream(const DecView& d, int M, int step, int mode, size_t smem, cudaStream_t s, bool pdl);
+cudaError_t prepare_stream_kernels(size_t smem);
+size_t row_stream_smem_bytes(int V4);
 void launch_joint(const DecView& d, int M, int step, cudaStream_t s);
 void launch_defaults(const DecView& d, cudaStream_t s);
 size_t row_smem_bytes(int V4, int n_lm);

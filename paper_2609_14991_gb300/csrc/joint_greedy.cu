@@ -1,19 +1,22 @@
-// Joint GEMM on the tcgen05 tensor cores with the dense-LM epilogue, for
-// greedy decoding with at most one n-gram LM.
+// Joint GEMM on the tcgen05 tensor cores for greedy decoding with at most
+// one n-gram LM, with one of two epilogues (the decoder option fusion_path).
 //
-// Per row r and label v of a 128 x BN tile the epilogue evaluates Eq. 1 up
-// to the row's constant c_r (see row_fused.cu):
+// DENSE (fusion_path 1): per row r and label v of a 128 x BN tile the
+// epilogue evaluates Eq. 1 up to the row's constant c_r (see row_fused.cu):
 //   F0[v] = logit[v] + D[v] + lambda * dense0[u_r][v]
 // with D the call's defaults (d.dvec) and u_r the dense LM row of the row's
 // unigram state (d.c_info), and reduces the tile to one partial per row:
 // softmax max and sum of the raw logits, and the best F0 over the labels not
 // on the row's correction list (d.c_mask), ties to the lowest label.  The
-// listed labels' raw logits are stored (d.logits) for the row pass.
+// listed labels' raw logits are stored (d.logits) for the row pass.  The
+// row's segment of its dense LM row is requested into L2 while the MMAs run
+// and copied into the drained operand stages by one bulk copy per row once
+// they have completed; the softmax pass runs while the copies land.
 //
-// The row's segment of its dense LM row is requested into L2 while the MMAs
-// run and copied into the drained operand stages by one bulk copy per row
-// once they have completed; the epilogue takes the softmax partial of the
-// raw logits (pass 1) while the copies land, then the fused values (pass 2).
+// Streaming (fusion_path 0): the epilogue writes logit + D[v] for every
+// label (d.logits, through per-warp swizzled staging buffers and TMA
+// stores) and the softmax partial; the row pass after it (row_stream.cu)
+// adds the row's LM and trie terms and takes the argmax.
 //
 // Warp roles (320 threads): warp 0 TMA producer (A tile 128 x 64 and W_out
 // tile BN x 64 per stage, 128-byte swizzle), warp 1 TMEM
@@ -37,9 +40,11 @@ constexpr int kDEpi = 256;  // warps 2-9
 constexpr float kNegInf = -__builtin_huge_valf();
 
 // Shared memory: [operand stages][defaults D][barriers].  After the
-// mainloop the stages hold the halves' exchange and, past it, the rows'
-// dense LM segments, rows 16 bytes apart beyond their BN floats so that the
-// 16-byte reads of eight consecutive rows fall in different bank groups.
+// mainloop the stages hold the halves' exchange and, past it, either the
+// rows' dense LM segments (rows 16 bytes apart beyond their BN floats, so
+// that the 16-byte reads of eight consecutive rows fall in different bank
+// groups) or the streaming epilogue's staging buffers (two 32 x 32 fp32
+// boxes per warp).
 template <int BN>
 struct DSmem {
   static constexpr int kABytes = kBM * kBK * 2;
@@ -48,11 +53,13 @@ struct DSmem {
   static constexpr int kStages = BN == 256 ? 4 : (BN == 128 ? 5 : 8);
   static constexpr int kRowStride = BN * 4 + 16;
   static constexpr int kDenseOff = 10240;  // past the halves' exchange
+  static constexpr int kStageOff = 16384;  // streaming: staging buffers, 8 KB per epilogue warp
   static constexpr int kDOff = kStages * kStageBytes;
   static constexpr int kBarOff = kDOff + BN * 4;
   static constexpr int kBytes = kBarOff + 256 + 1024 /*align*/;
   static_assert(kBM * 18 * 4 + 16 <= kDenseOff, "the halves' exchange stays clear of the dense rows");
   static_assert(kDenseOff + kBM * kRowStride <= kStages * kStageBytes, "the dense rows fit the drained stages");
+  static_assert(kStageOff + 8 * 8192 <= kStages * kStageBytes, "the staging buffers fit the drained stages");
   static_assert(kBytes <= 227 * 1024, "shared memory per CTA");
 };
 
@@ -72,9 +79,10 @@ __device__ __forceinline__ uint32_t pick(const uint32_t (&a)[N], int k) {
   return v;
 }
 
-template <int BN>
+template <int BN, bool DENSE>
 __global__ void __launch_bounds__(kDThreads, 1)
-    k_joint_dense(DecView d, int step, const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB) {
+    k_joint_greedy(DecView d, int step, const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                   const __grid_constant__ CUtensorMap tmLogits) {
   using S = DSmem<BN>;
   extern __shared__ __align__(1024) unsigned char smem_raw[];
   unsigned char* smem = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -190,7 +198,7 @@ __global__ void __launch_bounds__(kDThreads, 1)
 #pragma unroll
     for (int k = 0; k < kMy; ++k) mw[k] = 0u;
     int uoff = -1;
-    if (live) {
+    if (DENSE && live) {
       const int u = __ldcg(&d.c_info[gr].x);
       if (u >= 0 && u < d.lm.n_dense) uoff = u * V4;
       const uint32_t* mrow = d.c_mask + (size_t)gr * d.mask_words + n0 / 32;
@@ -199,7 +207,7 @@ __global__ void __launch_bounds__(kDThreads, 1)
     }
     unsigned char* drow = smem + S::kDenseOff + row * S::kRowStride;
     const int seg = min(BN, V4 - n0);  // labels of the tile inside the dense rows
-    if (ehalf == 0 && uoff >= 0 && seg > 0) {  // the row's segment into L2 while the MMAs run
+    if (DENSE && ehalf == 0 && uoff >= 0 && seg > 0) {  // the row's segment into L2 while the MMAs run
       asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(d.lm.dense0 + uoff + n0), "r"((uint32_t)seg * 4u)
                    : "memory");
     }
@@ -209,7 +217,7 @@ __global__ void __launch_bounds__(kDThreads, 1)
     fence_after();
     // the row's segment into the drained stages (every MMA has completed) by
     // one bulk copy, and the row's arrival on dbar (with the copy's bytes)
-    if (ehalf == 0) {
+    if (DENSE && ehalf == 0) {
       if (ok && uoff >= 0 && seg > 0) {
         mbar_expect_tx(dbar, (uint32_t)seg * 4u);
         bulk_g2s(drow, d.lm.dense0 + uoff + n0, (uint32_t)seg * 4u, dbar);
@@ -219,8 +227,9 @@ __global__ void __launch_bounds__(kDThreads, 1)
     }
     const uint32_t tbase = tmem + ((uint32_t)(q * 32) << 16);
     if (ok) {
-      // pass 1, while the copies land: the softmax partial of the raw
-      // logits; the listed labels' logits go out for the row pass
+      // pass 1 (DENSE: while the copies land): the softmax partial of the
+      // raw logits; DENSE: the listed labels' logits go out for the row
+      // pass; streaming: logit + D of every label goes out
 #pragma unroll 1
       for (int c = ehalf; c < BN / 32; c += 2) {
         __syncwarp();
@@ -254,18 +263,46 @@ __global__ void __launch_bounds__(kDThreads, 1)
           for (int i = 0; i < 32; ++i)
             if (c0 + i < N) cl[c0 + i] = l[i];
         }
-        const uint32_t mk = pick(mw, c >> 1);
-        if (mk) {
-          float* lo = d.logits + (size_t)gr * d.N_pad + c0;
+        if constexpr (DENSE) {
+          const uint32_t mk = pick(mw, c >> 1);
+          if (mk) {
+            float* lo = d.logits + (size_t)gr * d.N_pad + c0;
 #pragma unroll
-          for (int i = 0; i < 32; ++i)
-            if ((mk >> i) & 1u) lo[i] = l[i];
+            for (int i = 0; i < 32; ++i)
+              if ((mk >> i) & 1u) lo[i] = l[i];
+          }
+        } else {
+          // the warp's 32 x 32 block of logit + D by one TMA store from a
+          // staging buffer in the drained stages (two per warp, alternating;
+          // the 128-byte swizzle keeps the row-per-thread writes
+          // conflict-free)
+          const float4* dv4 = reinterpret_cast<const float4*>(sD + 32 * c);
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            const float4 dq = dv4[j];
+            l[4 * j] += dq.x; l[4 * j + 1] += dq.y; l[4 * j + 2] += dq.z; l[4 * j + 3] += dq.w;
+          }
+          unsigned char* stg = smem + S::kStageOff + (warp - 2) * 8192 + ((c >> 1) & 1) * 4096;
+          if (lane == 0) tma_store_wait_read1();  // this buffer's store of two chunks ago has read it
+          __syncwarp();
+#pragma unroll
+          for (int j = 0; j < 8; ++j)
+            *reinterpret_cast<float4*>(stg + lane * 128 + ((j ^ (lane & 7)) << 4)) =
+                make_float4(l[4 * j], l[4 * j + 1], l[4 * j + 2], l[4 * j + 3]);
+          fence_async_smem();
+          __syncwarp();
+          if (lane == 0) {
+            tma_store_2d(&tmLogits, stg, c0, m0 + q * 32);
+            tma_store_commit();
+          }
         }
       }
-      ok = __all_sync(0xffffffffu, mbar_wait(dbar, 0, d.wait_ns));
-      if (!ok && lane == 0) atomicOr(d.err, 64);
+      if (DENSE) {
+        ok = __all_sync(0xffffffffu, mbar_wait(dbar, 0, d.wait_ns));
+        if (!ok && lane == 0) atomicOr(d.err, 64);
+      }
     }
-    if (ok) {
+    if (DENSE && ok) {
       // pass 2: F0 = logit + D + lambda * dense0[u] of the unlisted labels and
       // the tile's best of them
 #pragma unroll 1
@@ -319,8 +356,9 @@ __global__ void __launch_bounds__(kDThreads, 1)
     // landing (the long limit whatever wait_ns is)
     if (warp == 2 && lane == 0) {
       mbar_wait(accum, 0);
-      mbar_wait(dbar, 0);
+      if (DENSE) mbar_wait(dbar, 0);
     }
+    if (!DENSE && lane == 0) tma_store_wait_all();  // the staging buffers are read
     __syncwarp();
     // merge the two epilogue halves' partials of each row: the second leaves
     // its partial in the drained stages, the first combines and stores
@@ -365,14 +403,32 @@ __global__ void __launch_bounds__(kDThreads, 1)
 
 }  // namespace
 
-cudaError_t joint_dense_prepare(int bn) {
+cudaError_t joint_greedy_prepare(int bn) {
   const auto attr = cudaFuncAttributeMaxDynamicSharedMemorySize;
-  if (bn == 256) return cudaFuncSetAttribute(k_joint_dense<256>, attr, DSmem<256>::kBytes);
-  if (bn == 128) return cudaFuncSetAttribute(k_joint_dense<128>, attr, DSmem<128>::kBytes);
-  return cudaFuncSetAttribute(k_joint_dense<64>, attr, DSmem<64>::kBytes);
+  cudaError_t e = cudaSuccess;
+  if (bn == 256) {
+    e = cudaFuncSetAttribute(k_joint_greedy<256, true>, attr, DSmem<256>::kBytes);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(k_joint_greedy<256, false>, attr, DSmem<256>::kBytes);
+  } else if (bn == 128) {
+    e = cudaFuncSetAttribute(k_joint_greedy<128, true>, attr, DSmem<128>::kBytes);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(k_joint_greedy<128, false>, attr, DSmem<128>::kBytes);
+  } else {
+    e = cudaFuncSetAttribute(k_joint_greedy<64, true>, attr, DSmem<64>::kBytes);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(k_joint_greedy<64, false>, attr, DSmem<64>::kBytes);
+  }
+  return e;
 }
 
-void launch_joint_dense(const JointTc& jt, const DecView& d, int M, int step, cudaStream_t s, bool pdl) {
+namespace {
+template <int BN>
+void launch_greedy_bn(cudaLaunchConfig_t& cfg, const JointTc& jt, const DecView& d, int step) {
+  cfg.dynamicSmemBytes = DSmem<BN>::kBytes;
+  if (d.fz_dense) cudaLaunchKernelEx(&cfg, k_joint_greedy<BN, true>, d, step, jt.mapA, jt.mapB, jt.mapLogits);
+  else cudaLaunchKernelEx(&cfg, k_joint_greedy<BN, false>, d, step, jt.mapA, jt.mapB, jt.mapLogits);
+}
+}  // namespace
+
+void launch_joint_greedy(const JointTc& jt, const DecView& d, int M, int step, cudaStream_t s, bool pdl) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(d.N_pad / jt.bn, (M + kBM - 1) / kBM);
   cfg.blockDim = dim3(kDThreads);
@@ -382,16 +438,9 @@ void launch_joint_dense(const JointTc& jt, const DecView& d, int M, int step, cu
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = pdl ? 1 : 0;
-  if (jt.bn == 256) {
-    cfg.dynamicSmemBytes = DSmem<256>::kBytes;
-    cudaLaunchKernelEx(&cfg, k_joint_dense<256>, d, step, jt.mapA, jt.mapB);
-  } else if (jt.bn == 128) {
-    cfg.dynamicSmemBytes = DSmem<128>::kBytes;
-    cudaLaunchKernelEx(&cfg, k_joint_dense<128>, d, step, jt.mapA, jt.mapB);
-  } else {
-    cfg.dynamicSmemBytes = DSmem<64>::kBytes;
-    cudaLaunchKernelEx(&cfg, k_joint_dense<64>, d, step, jt.mapA, jt.mapB);
-  }
+  if (jt.bn == 256) launch_greedy_bn<256>(cfg, jt, d, step);
+  else if (jt.bn == 128) launch_greedy_bn<128>(cfg, jt, d, step);
+  else launch_greedy_bn<64>(cfg, jt, d, step);
 }
 
 }  // namespace tsd

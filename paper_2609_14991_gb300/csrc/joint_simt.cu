@@ -8,7 +8,8 @@
 // the fused value is logit + D[v] + lambda*dense0[u][v] (the call's defaults
 // and the dense LM row of the row's unigram state u), and the labels on the
 // row's correction list are no candidates: their raw logits are stored for
-// the row pass.
+// the row pass.  With fusion_path 0 (DecView::fz_dense = 0) the row's logits
+// plus the call's defaults are written out instead and the row pass fuses.
 // This is the simple reference-grade kernel for small row counts; the
 // tensor-core kernel in joint_tc.cu does the same contraction with tcgen05.
 #include "decoder.h"
@@ -99,7 +100,8 @@ __global__ void __launch_bounds__(256) k_joint_simt(DecView d, int step) {
     const float* urow = nullptr;
     const uint32_t* mrow = nullptr;
     const float lam = d.params->lambda;
-    if (d.fused) {
+    const bool dense = d.fused && d.fz_dense;
+    if (dense) {
       const int u = __ldcg(&d.c_info[gr].x);
       if (u >= 0 && u < d.lm.n_dense) urow = d.lm.dense0 + (size_t)u * d.V4;
       mrow = d.c_mask + (size_t)gr * d.mask_words;
@@ -114,7 +116,9 @@ __global__ void __launch_bounds__(256) k_joint_simt(DecView d, int step) {
       if (gc < N) {
         mx = fmaxf(mx, l[q]);
         float f;
-        if (d.fused) {
+        if (d.fused && !dense) {
+          f = l[q];  // the streaming form: the row pass takes the argmax
+        } else if (dense) {
           if ((__ldcg(mrow + (gc >> 5)) >> (gc & 31)) & 1u) {  // listed: the row pass evaluates it
             d.logits[(size_t)gr * d.N_pad + gc] = l[q];
             continue;
@@ -143,6 +147,13 @@ __global__ void __launch_bounds__(256) k_joint_simt(DecView d, int step) {
     for (int o = 16; o > 0; o >>= 1) se += __shfl_xor_sync(0xffffffffu, se, o);
     if (lane == 0)
       d.part[(size_t)gr * d.n_ptiles + blockIdx.x] = make_float4(mx, se, bv, __int_as_float(bi));
+    if (d.fused && !dense) {  // the streaming form: logit + D of every label
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const int gc = n0 + lane * 4 + q;
+        d.logits[(size_t)gr * d.N_pad + gc] = l[q] + __ldcg(d.dvec + gc);
+      }
+    }
     if (d.cap_logits && step < d.cap_steps) {
 #pragma unroll
       for (int q = 0; q < 4; ++q) {

@@ -11,7 +11,7 @@
 // this tile: softmax max and sum over the real labels, and the best fused
 // value logit + bias (the dense fusion bias row of several LMs), ties to the
 // lowest label, or (BEAM) the tile's top K.  Greedy decoding with at most one
-// LM runs joint_dense.cu instead.  Logits never leave the SM.
+// LM runs joint_greedy.cu instead.  Logits never leave the SM.
 //
 // Warp roles (320 threads): warp 0 TMA producer, warp 1 TMEM allocator and
 // MMA issuer, warps 2-9 epilogue.  Every wait on an mbarrier is bounded in
@@ -413,11 +413,13 @@ int joint_tc_pick_bn(int M_max, int N_pad, int sms) {
 }
 
 cudaError_t joint_tc_prepare(JointTc* jt, const uint16_t* A, int M_pad, const uint16_t* Wt, int N_pad, int H, int bn,
-                             const float* bias) {
+                             const float* bias, const float* logits) {
   jt->bn = bn;
   if (!make_map(&jt->mapA, A, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, H, M_pad, kBK, kBM)) return cudaErrorInvalidValue;
   if (!make_map(&jt->mapB, Wt, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, H, N_pad, kBK, bn)) return cudaErrorInvalidValue;
   if (!make_map(&jt->mapBias, bias, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, N_pad, M_pad, 32, kBM))
+    return cudaErrorInvalidValue;
+  if (!make_map(&jt->mapLogits, logits ? logits : bias, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, N_pad, M_pad, 32, 32))
     return cudaErrorInvalidValue;
   const auto attr = cudaFuncAttributeMaxDynamicSharedMemorySize;
   cudaError_t e = cudaSuccess;
@@ -431,7 +433,7 @@ cudaError_t joint_tc_prepare(JointTc* jt, const uint16_t* A, int M_pad, const ui
     e = cudaFuncSetAttribute(k_joint_tc<64, false>, attr, Smem<64>::kBytes);
     if (e == cudaSuccess) e = cudaFuncSetAttribute(k_joint_tc<64, true>, attr, Smem<64>::kBytes);
   }
-  if (e == cudaSuccess) e = joint_dense_prepare(bn);
+  if (e == cudaSuccess) e = joint_greedy_prepare(bn);
   return e;
 }
 
@@ -447,7 +449,7 @@ void launch_bn(cudaLaunchConfig_t& cfg, const JointTc& jt, const DecView& d, int
 
 void launch_joint_tc(const JointTc& jt, const DecView& d, int M, int step, cudaStream_t s, bool pdl) {
   if (d.fused) {
-    launch_joint_dense(jt, d, M, step, s, pdl);
+    launch_joint_greedy(jt, d, M, step, s, pdl);
     return;
   }
   cudaLaunchConfig_t cfg = {};

@@ -119,6 +119,25 @@ def test_cfg4_full_size_parity():
     assert n >= 32 and err < pu.LOGIT_TOL, (err, n)
 
 
+@pytest.mark.parametrize("path", [0, 1])
+def test_fusion_paths_match_oracle(path):
+    """Both forms of the greedy one-LM step (fusion_path 1: the level-0 LM
+    term in the joint epilogue with a per-row correction list; 0: the
+    streaming form) against the oracle, at the stress vocabulary (V+1 =
+    4097) with a 6-gram LM and phrases: 48 streams replayed over both chunks,
+    and the tiny workload in full."""
+    w = synth.scaled(synth.WORKLOADS[4], B=160, chunks=2, lm_order=6, lm_total=400_000, n_phr=2000)
+    inp = pu.Inputs(w)
+    run = pu.GpuRun(inp, range(w.B), 2, options={"fusion_path": path})
+    models = pu.oracle_models(inp)
+    pu.assert_reports(pu.replay(inp, run, list(range(0, w.B, 10)) + [127, 128, 159], models=models))
+    assert max(len(run.lm.state_tuple(run.states[-1][i][0])) for i in range(w.B)) >= 3
+    w0 = synth.WORKLOADS[0]
+    inp0 = pu.Inputs(w0)
+    run0 = pu.GpuRun(inp0, range(w0.B), 1, options={"fusion_path": path})
+    pu.assert_reports(pu.replay(inp0, run0, range(w0.B)))
+
+
 @pytest.mark.parametrize("shape", ["cfg2", "cfg4"])
 @pytest.mark.parametrize("bn", [64, 128, 256])
 def test_joint_logits_elementwise(shape, bn):
