@@ -35,12 +35,13 @@ namespace tsd {
 namespace {
 
 using namespace tc;
-constexpr int kDThreads = 320;
-constexpr int kDEpi = 256;  // warps 2-9
+constexpr int kEW = 4;                 // epilogue warps per TMEM lane quadrant
+constexpr int kDEpi = 128 * kEW;       // epilogue threads: warps 2 .. 2 + 4 kEW - 1
+constexpr int kDThreads = 64 + kDEpi;  // and the producer and MMA warps
 constexpr float kNegInf = -__builtin_huge_valf();
 
 // Shared memory: [operand stages][defaults D][barriers].  After the
-// mainloop the stages hold the halves' exchange and, past it, either the
+// mainloop the stages hold the epilogue warps' exchange and, past it, either the
 // rows' dense LM segments (rows 16 bytes apart beyond their BN floats, so
 // that the 16-byte reads of eight consecutive rows fall in different bank
 // groups) or the streaming epilogue's staging buffers (two 32 x 32 fp32
@@ -52,23 +53,39 @@ struct DSmem {
   static constexpr int kStageBytes = kABytes + kBBytes;
   static constexpr int kStages = BN == 256 ? 4 : (BN == 128 ? 5 : 8);
   static constexpr int kRowStride = BN * 4 + 16;
-  static constexpr int kDenseOff = 10240;  // past the halves' exchange
-  static constexpr int kStageOff = 16384;  // streaming: staging buffers, 8 KB per epilogue warp
+  static constexpr int kDenseOff = 10240;  // past the epilogue warps' exchange
+  static constexpr int kCW = 32;            // columns per TMEM load in the epilogue
+  static constexpr int kStageOff = 16384;   // streaming: staging buffers, two 32 x 32 boxes per warp
+  static constexpr int kStageWarp = 2 * (kCW / 32) * 4096;
   static constexpr int kDOff = kStages * kStageBytes;
   static constexpr int kBarOff = kDOff + BN * 4;
   static constexpr int kBytes = kBarOff + 256 + 1024 /*align*/;
-  static_assert(kBM * 18 * 4 + 16 <= kDenseOff, "the halves' exchange stays clear of the dense rows");
+  static_assert(kBM * 4 * (kEW - 1) * 4 + 4 * 4 * kEW <= kDenseOff, "the exchange stays clear of the dense rows");
   static_assert(kDenseOff + kBM * kRowStride <= kStages * kStageBytes, "the dense rows fit the drained stages");
-  static_assert(kStageOff + 8 * 8192 <= kStages * kStageBytes, "the staging buffers fit the drained stages");
+  static_assert(kStageOff + 4 * kEW * kStageWarp <= kStages * kStageBytes, "the staging buffers fit the drained stages");
   static_assert(kBytes <= 227 * 1024, "shared memory per CTA");
 };
 
-// Sum over a chunk of 2^(l[i] * log2 e - s2) in four independent accumulators.
-__device__ __forceinline__ float sum_exp2_chunk(const float* l, float s2) {
+// Sum over a block of 2^(l[i] * log2 e - s2) in four independent accumulators.
+template <int W>
+__device__ __forceinline__ float sum_exp2_block(const float* l, float s2) {
   float a[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-  for (int i = 0; i < 32; ++i) a[i & 3] += ex2_approx(fmaf(l[i], kLog2e, -s2));
+  for (int i = 0; i < W; ++i) a[i & 3] += ex2_approx(fmaf(l[i], kLog2e, -s2));
   return (a[0] + a[1]) + (a[2] + a[3]);
+}
+
+// The maximum of a block by a tree (the block is left unchanged).
+template <int W>
+__device__ __forceinline__ float block_max(const float* v) {
+  float t[W / 2];
+#pragma unroll
+  for (int i = 0; i < W / 2; ++i) t[i] = fmaxf(v[i], v[i + W / 2]);
+#pragma unroll
+  for (int w = W / 4; w > 0; w >>= 1)
+#pragma unroll
+    for (int i = 0; i < w; ++i) t[i] = fmaxf(t[i], t[i + w]);
+  return t[0];
 }
 
 template <int N>
@@ -179,9 +196,14 @@ __global__ void __launch_bounds__(kDThreads, 1)
     }
     __syncwarp();
   } else {
-    // epilogue: warps 2..9, thread = row of the tile
+    // epilogue: thread = row of the tile; the kEW warps of a TMEM lane
+    // quadrant take blocks of kCW columns in turn (one TMEM load each)
+    constexpr int kCW = S::kCW;
+    constexpr int kNB = BN / kCW;              // blocks per tile
+    constexpr int kMyB = (kNB + kEW - 1) / kEW;  // blocks per warp, at most
+    constexpr int kWB = kCW / 32;          // mask words and 32 x 32 store boxes per block
     const int q = warp & 3;  // TMEM lane quadrant this warp may access
-    const int ehalf = (warp - 2) >> 2;
+    const int ehalf = (warp - 2) >> 2;  // this warp's turn among its quadrant's warps
     const int row = q * 32 + lane;
     const int gr = m0 + row;
     const bool live = gr < M;
@@ -193,17 +215,19 @@ __global__ void __launch_bounds__(kDThreads, 1)
     // this grid's wait)
     for (int i = (int)threadIdx.x - 64; i < BN; i += kDEpi) sD[i] = __ldcg(d.dvec + n0 + i);
     const float lam = d.params->lambda;
-    constexpr int kMy = BN / 64;  // chunks each epilogue warp takes: c = ehalf + 2k
-    uint32_t mw[kMy];
+    uint32_t mw[kMyB * kWB];  // [block of this warp][word]
 #pragma unroll
-    for (int k = 0; k < kMy; ++k) mw[k] = 0u;
+    for (int k = 0; k < kMyB * kWB; ++k) mw[k] = 0u;
     int uoff = -1;
     if (DENSE && live) {
       const int u = __ldcg(&d.c_info[gr].x);
       if (u >= 0 && u < d.lm.n_dense) uoff = u * V4;
       const uint32_t* mrow = d.c_mask + (size_t)gr * d.mask_words + n0 / 32;
 #pragma unroll
-      for (int k = 0; k < kMy; ++k) mw[k] = __ldcg(mrow + ehalf + 2 * k);
+      for (int k = 0; k < kMyB; ++k)
+#pragma unroll
+        for (int j = 0; j < kWB; ++j)
+          if (ehalf + kEW * k < kNB) mw[k * kWB + j] = __ldcg(mrow + (ehalf + kEW * k) * kWB + j);
     }
     unsigned char* drow = smem + S::kDenseOff + row * S::kRowStride;
     const int seg = min(BN, V4 - n0);  // labels of the tile inside the dense rows
@@ -231,69 +255,72 @@ __global__ void __launch_bounds__(kDThreads, 1)
       // raw logits; DENSE: the listed labels' logits go out for the row
       // pass; streaming: logit + D of every label goes out
 #pragma unroll 1
-      for (int c = ehalf; c < BN / 32; c += 2) {
+      for (int k = 0; k < kMyB; ++k) {
+        const int b = ehalf + kEW * k;
+        if (b >= kNB) break;
         __syncwarp();
-        const int c0 = n0 + c * 32;
-        float l[32];
-        tmem_ld32(tbase + (uint32_t)(c * 32), l);
-        if (c0 + 32 > N) {
+        const int c0 = n0 + b * kCW;
+        float l[kCW];
+        tmem_ld<kCW>(tbase + (uint32_t)(b * kCW), l);
+        if (c0 + kCW > N) {
 #pragma unroll
-          for (int i = 0; i < 32; ++i)
+          for (int i = 0; i < kCW; ++i)
             if (c0 + i >= N) l[i] = kNegInf;
         }
-        float t[16];
-#pragma unroll
-        for (int i = 0; i < 16; ++i) t[i] = fmaxf(l[i], l[i + 16]);
-#pragma unroll
-        for (int w = 8; w > 0; w >>= 1)
-#pragma unroll
-          for (int i = 0; i < w; ++i) t[i] = fmaxf(t[i], t[i + w]);
-        const float cm = t[0];
+        const float cm = block_max<kCW>(l);
         if (cm != kNegInf) {
           const float m2 = fmaxf(mx, cm);
           const float s2 = m2 * kLog2e;
           float acc = (mx == kNegInf) ? 0.f : se * ex2_approx(mx * kLog2e - s2);
-          acc += sum_exp2_chunk(l, s2);
+          acc += sum_exp2_block<kCW>(l, s2);
           se = acc;
           mx = m2;
         }
         if (d.cap_logits && step < d.cap_steps && live) {
           float* cl = d.cap_logits + ((size_t)step * M + gr) * N;
 #pragma unroll
-          for (int i = 0; i < 32; ++i)
+          for (int i = 0; i < kCW; ++i)
             if (c0 + i < N) cl[c0 + i] = l[i];
         }
         if constexpr (DENSE) {
-          const uint32_t mk = pick(mw, c >> 1);
-          if (mk) {
-            float* lo = d.logits + (size_t)gr * d.N_pad + c0;
 #pragma unroll
-            for (int i = 0; i < 32; ++i)
-              if ((mk >> i) & 1u) lo[i] = l[i];
+          for (int j = 0; j < kWB; ++j) {
+            const uint32_t mk = pick(mw, k * kWB + j);
+            if (mk) {
+              float* lo = d.logits + (size_t)gr * d.N_pad + c0 + 32 * j;
+#pragma unroll
+              for (int i = 0; i < 32; ++i)
+                if ((mk >> i) & 1u) lo[i] = l[32 * j + i];
+            }
           }
         } else {
-          // the warp's 32 x 32 block of logit + D by one TMA store from a
-          // staging buffer in the drained stages (two per warp, alternating;
-          // the 128-byte swizzle keeps the row-per-thread writes
+          // the warp's 32-row boxes of logit + D by TMA stores from staging
+          // buffers in the drained stages (two sets per warp, alternating by
+          // block; the 128-byte swizzle keeps the row-per-thread writes
           // conflict-free)
-          const float4* dv4 = reinterpret_cast<const float4*>(sD + 32 * c);
+          const float4* dv4 = reinterpret_cast<const float4*>(sD + b * kCW);
 #pragma unroll
-          for (int j = 0; j < 8; ++j) {
+          for (int j = 0; j < kCW / 4; ++j) {
             const float4 dq = dv4[j];
             l[4 * j] += dq.x; l[4 * j + 1] += dq.y; l[4 * j + 2] += dq.z; l[4 * j + 3] += dq.w;
           }
-          unsigned char* stg = smem + S::kStageOff + (warp - 2) * 8192 + ((c >> 1) & 1) * 4096;
-          if (lane == 0) tma_store_wait_read1();  // this buffer's store of two chunks ago has read it
+          unsigned char* stg = smem + S::kStageOff + (warp - 2) * S::kStageWarp + (k & 1) * kWB * 4096;
+          if (lane == 0) tma_store_wait_read<kWB>();  // the stores of two blocks ago have read this set
           __syncwarp();
 #pragma unroll
-          for (int j = 0; j < 8; ++j)
-            *reinterpret_cast<float4*>(stg + lane * 128 + ((j ^ (lane & 7)) << 4)) =
-                make_float4(l[4 * j], l[4 * j + 1], l[4 * j + 2], l[4 * j + 3]);
+          for (int j = 0; j < kWB; ++j)
+#pragma unroll
+            for (int e = 0; e < 8; ++e)
+              *reinterpret_cast<float4*>(stg + j * 4096 + lane * 128 + ((e ^ (lane & 7)) << 4)) =
+                  make_float4(l[32 * j + 4 * e], l[32 * j + 4 * e + 1], l[32 * j + 4 * e + 2], l[32 * j + 4 * e + 3]);
           fence_async_smem();
           __syncwarp();
           if (lane == 0) {
-            tma_store_2d(&tmLogits, stg, c0, m0 + q * 32);
-            tma_store_commit();
+#pragma unroll
+            for (int j = 0; j < kWB; ++j) {
+              tma_store_2d(&tmLogits, stg + j * 4096, c0 + 32 * j, m0 + q * 32);
+              tma_store_commit();
+            }
           }
         }
       }
@@ -306,49 +333,46 @@ __global__ void __launch_bounds__(kDThreads, 1)
       // pass 2: F0 = logit + D + lambda * dense0[u] of the unlisted labels and
       // the tile's best of them
 #pragma unroll 1
-      for (int c = ehalf; c < BN / 32; c += 2) {
+      for (int k = 0; k < kMyB; ++k) {
+        const int b = ehalf + kEW * k;
+        if (b >= kNB) break;
         __syncwarp();
-        const int c0 = n0 + c * 32;
-        float l[32];
-        tmem_ld32(tbase + (uint32_t)(c * 32), l);
-        if (c0 + 32 > N) {
+        const int c0 = n0 + b * kCW;
+        float l[kCW];
+        tmem_ld<kCW>(tbase + (uint32_t)(b * kCW), l);
+        if (c0 + kCW > N) {
 #pragma unroll
-          for (int i = 0; i < 32; ++i)
+          for (int i = 0; i < kCW; ++i)
             if (c0 + i >= N) l[i] = kNegInf;
         }
-        const float4* dv4 = reinterpret_cast<const float4*>(sD + 32 * c);
-        float x[32];
+        const float4* dv4 = reinterpret_cast<const float4*>(sD + b * kCW);
 #pragma unroll
-        for (int j = 0; j < 8; ++j) {
+        for (int j = 0; j < kCW / 4; ++j) {
           const float4 dq = dv4[j];
           float4 xq = make_float4(0.f, 0.f, 0.f, 0.f);
-          if (uoff >= 0 && c * 32 + 4 * j < seg) xq = *reinterpret_cast<const float4*>(drow + (c * 32 + 4 * j) * 4);
-          x[4 * j] = l[4 * j] + fmaf(lam, xq.x, dq.x);
-          x[4 * j + 1] = l[4 * j + 1] + fmaf(lam, xq.y, dq.y);
-          x[4 * j + 2] = l[4 * j + 2] + fmaf(lam, xq.z, dq.z);
-          x[4 * j + 3] = l[4 * j + 3] + fmaf(lam, xq.w, dq.w);
+          if (uoff >= 0 && b * kCW + 4 * j < seg) xq = *reinterpret_cast<const float4*>(drow + (b * kCW + 4 * j) * 4);
+          l[4 * j] += fmaf(lam, xq.x, dq.x);
+          l[4 * j + 1] += fmaf(lam, xq.y, dq.y);
+          l[4 * j + 2] += fmaf(lam, xq.z, dq.z);
+          l[4 * j + 3] += fmaf(lam, xq.w, dq.w);
         }
-        const uint32_t mk = pick(mw, c >> 1);
-        if (mk) {
 #pragma unroll
-          for (int i = 0; i < 32; ++i)
-            if ((mk >> i) & 1u) x[i] = kNegInf;
+        for (int j = 0; j < kWB; ++j) {
+          const uint32_t mk = pick(mw, k * kWB + j);
+          if (mk) {
+#pragma unroll
+            for (int i = 0; i < 32; ++i)
+              if ((mk >> i) & 1u) l[32 * j + i] = kNegInf;
+          }
         }
-        float u[16];
-#pragma unroll
-        for (int i = 0; i < 16; ++i) u[i] = fmaxf(x[i], x[i + 16]);
-#pragma unroll
-        for (int w = 8; w > 0; w >>= 1)
-#pragma unroll
-          for (int i = 0; i < w; ++i) u[i] = fmaxf(u[i], u[i + w]);
-        const float fm = u[0];
+        const float fm = block_max<kCW>(l);
         if (fm > bv) {
-          int j = 31;
+          int jx = kCW - 1;
 #pragma unroll
-          for (int i = 31; i >= 0; --i)
-            if (x[i] == fm) j = i;
+          for (int i = kCW - 1; i >= 0; --i)
+            if (l[i] == fm) jx = i;
           bv = fm;
-          bi = c0 + j;
+          bi = c0 + jx;
         }
       }
     }
@@ -360,37 +384,46 @@ __global__ void __launch_bounds__(kDThreads, 1)
     }
     if (!DENSE && lane == 0) tma_store_wait_all();  // the staging buffers are read
     __syncwarp();
-    // merge the two epilogue halves' partials of each row: the second leaves
-    // its partial in the drained stages, the first combines and stores
+    // merge the quadrant's warps' partials of each row: warps 1..kEW-1 of the
+    // quadrant leave theirs in the drained stages, warp 0 combines and stores
     float* xbase = reinterpret_cast<float*>(smem);
-    float* xch = xbase + row * 18;
-    int* xok = reinterpret_cast<int*>(xbase + kBM * 18);
-    if (ehalf == 1) {
+    int* xok = reinterpret_cast<int*>(xbase + kBM * 4 * (kEW - 1));  // [quadrant][warp 1..]
+    if (ehalf > 0) {
+      float* xch = xbase + (row * (kEW - 1) + ehalf - 1) * 4;
       if (ok) {
         xch[0] = mx;
         xch[1] = se;
         xch[2] = bv;
         xch[3] = __int_as_float(bi);
       }
-      if (lane == 0) xok[q] = ok ? 1 : 0;
+      if (lane == 0) xok[q * (kEW - 1) + ehalf - 1] = ok ? 1 : 0;
     }
     asm volatile("bar.sync 1, %0;" ::"n"(kDEpi) : "memory");
-    if (ehalf == 0 && ok && xok[q] && live) {
-      const float m1 = xch[0], s1 = xch[1];
-      if (m1 != kNegInf) {
-        if (mx == kNegInf) {
-          mx = m1;
-          se = s1;
-        } else {
-          const float m2 = fmaxf(mx, m1);
-          se = se * ex2_approx((mx - m2) * kLog2e) + s1 * ex2_approx((m1 - m2) * kLog2e);
-          mx = m2;
+    if (ehalf == 0 && ok && live) {
+      bool all = true;
+#pragma unroll
+      for (int e = 1; e < kEW; ++e) {
+        if (!xok[q * (kEW - 1) + e - 1]) {
+          all = false;
+          continue;
         }
+        const float* xch = xbase + (row * (kEW - 1) + e - 1) * 4;
+        const float m1 = xch[0], s1 = xch[1];
+        if (m1 != kNegInf) {
+          if (mx == kNegInf) {
+            mx = m1;
+            se = s1;
+          } else {
+            const float m2 = fmaxf(mx, m1);
+            se = se * ex2_approx((mx - m2) * kLog2e) + s1 * ex2_approx((m1 - m2) * kLog2e);
+            mx = m2;
+          }
+        }
+        const float v1 = xch[2];
+        const int i1 = __float_as_int(xch[3]);
+        if (v1 > bv || (v1 == bv && i1 < bi)) { bv = v1; bi = i1; }
       }
-      const float v1 = xch[2];
-      const int i1 = __float_as_int(xch[3]);
-      if (v1 > bv || (v1 == bv && i1 < bi)) { bv = v1; bi = i1; }
-      d.part[(size_t)gr * d.n_ptiles + blockIdx.x] = make_float4(mx, se, bv, __int_as_float(bi));
+      if (all) d.part[(size_t)gr * d.n_ptiles + blockIdx.x] = make_float4(mx, se, bv, __int_as_float(bi));
     }
   }
   fence_before();

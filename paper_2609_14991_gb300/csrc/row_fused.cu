@@ -61,10 +61,10 @@ using row::kNegInf;
 using row::lse_merge;
 using row::warp_find;
 
-constexpr int kFzThreads = 128;  // 4 warps: seven CTAs per SM at 72 registers
+constexpr int kFzThreads = 128;  // 4 warps: seven CTAs per SM at 72 registers (1024 rows over 147 SMs)
 constexpr int kFzWarps = kFzThreads / 32;
-constexpr int kHeld = 2;      // arc groups of four of levels 1.. a thread keeps in registers
-constexpr int kListHeld = 2;  // list entries a thread loads before waiting for the joint kernel
+constexpr int kHeld = 1;      // arc groups of four of levels 1.. a thread keeps in registers
+constexpr int kListPre = 32;  // list entries loaded (one per thread) before the list's length is known
 constexpr int kTrHeld = 1;    // trie chain children a thread keeps in registers
 
 // Aligned groups of four arcs a chain level's arcs [b, b + c) span.
@@ -150,20 +150,14 @@ __global__ void __launch_bounds__(kFzThreads) __maxnreg__((VAR & 4) ? 128 : 72) 
     s_tr[k] = __ldcg(d.m_tr + (size_t)r * kTrChain + k);
     s_trr[k] = __ldcg(d.m_trr + (size_t)r * kTrChain + k);
   }
-  // the list of the state the joint evaluated: its first kListHeld entries
-  // per thread in registers (loaded whatever its length; entries past it
-  // are dropped once the length is known)
-  int hv[kListHeld];
-  float ha[kListHeld];
-#pragma unroll
-  for (int u = 0; u < kListHeld; ++u) {
-    const int k = tid + u * kFzThreads;
-    hv[u] = -1;
-    ha[u] = 0.f;
-    if (step > 0 && k < d.V4) {
-      hv[u] = __ldcg(d.c_lab + (size_t)r * d.V4 + k);
-      ha[u] = __ldcg(d.c_add + (size_t)r * d.V4 + k);
-    }
+  // the list of the state the joint evaluated: its first kListPre entries,
+  // one per thread (loaded whatever its length, which lists rarely exceed;
+  // entries past it are dropped once the length is known)
+  int hv = -1;
+  float ha = 0.f;
+  if (step > 0 && tid < kListPre && tid < d.V4) {
+    hv = __ldcg(d.c_lab + (size_t)r * d.V4 + tid);
+    ha = __ldcg(d.c_add + (size_t)r * d.V4 + tid);
   }
   {  // per-label scratch reset
     uint4* k4 = reinterpret_cast<uint4*>(key);
@@ -182,9 +176,7 @@ __global__ void __launch_bounds__(kFzThreads) __maxnreg__((VAR & 4) ? 128 : 72) 
   row::block_sync();
   if (s_bad) return;
   const int slot = s_slot, T = s_T;
-#pragma unroll
-  for (int u = 0; u < kListHeld; ++u)
-    if (tid + u * kFzThreads >= s_ci.y) hv[u] = -1;
+  if (tid >= s_ci.y) hv = -1;
   if (step == 0) {
     // the chunk's first step: the stream's state by slot (the chains are
     // read whole: their arrays have room for the longest), and the row's copy
@@ -287,16 +279,10 @@ __global__ void __launch_bounds__(kFzThreads) __maxnreg__((VAR & 4) ? 128 : 72) 
       if (lane == 0) s_lse = m + logf(s);
     }
     {
-      float x[kListHeld];
-#pragma unroll
-      for (int u = 0; u < kListHeld; ++u)
-        if (hv[u] >= 0 && checked(hv[u] < V, d.err, 13)) x[u] = __ldcg(lg + hv[u]);
-#pragma unroll
-      for (int u = 0; u < kListHeld; ++u)
-        if (hv[u] >= 0 && hv[u] < V) best_merge(bv, bi, x[u] + ha[u], hv[u]);
+      if (hv >= 0 && checked(hv < V, d.err, 13)) best_merge(bv, bi, __ldcg(lg + hv) + ha, hv);
       const int32_t* cl = d.c_lab + (size_t)r * d.V4;
       const float* ca = d.c_add + (size_t)r * d.V4;
-      for (int k0 = tid + kListHeld * kFzThreads; k0 < ci.y; k0 += 4 * kFzThreads) {
+      for (int k0 = kListPre + tid; k0 < ci.y; k0 += 4 * kFzThreads) {
         int v[4];
         float a[4], x[4];
 #pragma unroll
