@@ -59,13 +59,16 @@ def peaks():
 # changed kernel reports null until it is captured again.  The captures and
 # their commands are summarised under profiles/.
 KERNEL_SOURCES = {
-    "joint": ["joint_tc.cu", "joint_tc.h", "tc_common.cuh", "decoder.h", "internal.h"],
-    "row": ["row_fused.cu", "row_pass.cu", "row_beam.cu", "row_common.cuh", "decoder.h", "internal.h"],
+    "joint": ["joint_greedy.cu", "joint_tc.h", "tc_common.cuh", "decoder.h", "internal.h"],
+    "row": ["row_fused.cu", "row_stream.cu", "row_common.cuh", "decoder.h", "internal.h"],
     "egemm": ["encoder_gemm.cu", "encoder.cu", "encoder.h", "tc_common.cuh", "internal.h"],
 }
+# keyed by (config, streams, kernel, fusion_path)
 TRAFFIC = {
-    (4, 1024, "joint"): (11050496, "3508e66f2646fc6a"),
-    (4, 1024, "row"): (29144576, "d3e65c4743c47a4d"),
+    (4, 1024, "joint", 1): (18074880, "826bf2360316aeca"),
+    (4, 1024, "row", 1): (10575616, "05b72ee1ecb1b352"),
+    (4, 1024, "joint", 0): (11051264, "826bf2360316aeca"),
+    (4, 1024, "row", 0): (29286400, "05b72ee1ecb1b352"),
 }
 
 
@@ -86,8 +89,8 @@ ENC_TRAFFIC = {
 }
 
 
-def recorded_traffic(w: synth.Workload, kernel: str, key=None):
-    rec = (ENC_TRAFFIC if key else TRAFFIC).get(key or (w.cfg, w.B, kernel))
+def recorded_traffic(w: synth.Workload, kernel: str, key=None, path=None):
+    rec = (ENC_TRAFFIC if key else TRAFFIC).get(key or (w.cfg, w.B, kernel, path))
     if rec is None or rec[1] != kernel_source_hash(kernel):
         return None
     return rec[0]
@@ -343,8 +346,8 @@ def stream_sweep(args, w, tsd, dev, stream, W, E, lm, lms, bo, pw, flush):
                         torch.from_numpy(E.view(np.int16)).to(dev), lm=None if lms else lm, lms=lms, boost=bo,
                         max_symbols=w.max_sym, beam_k=w.beam, max_streams=B, max_T=w.T, prune_k=args.prune_k,
                         pred=pw)
-        if w.beam == 1 and not args.prune_k and not lms and args.fusion_path is not None:
-            d.set_option("fusion_path", args.fusion_path)
+        if w.beam == 1 and not args.prune_k and not lms and getattr(args, "fusion_path_given", False):
+            d.set_option("fusion_path", args.fusion_path)  # else the decoder's default for B streams
         sl = np.array([d.open() for _ in range(B)], dtype=np.int32)
         encs = [torch.from_numpy(synth.enc_chunk(w, range(B), c % w.chunks).view(np.int16)).to(dev)
                 for c in range(args.warmup + args.steps)]
@@ -396,8 +399,9 @@ def run_ours(args, w):
                       max_streams=w.B, max_T=w.T, prune_k=args.prune_k, pred=pw)
     greedy1 = w.beam == 1 and not args.prune_k and not extra  # greedy decoding with at most one LM
     if greedy1:
-        if args.fusion_path is None:  # the decoder's default: the dense epilogue from V = 2048 up
-            args.fusion_path = 1 if w.V >= 2048 else 0
+        args.fusion_path_given = args.fusion_path is not None
+        if args.fusion_path is None:  # the decoder's default: the dense epilogue from V = 2048 and 512 streams up
+            args.fusion_path = 1 if (w.V >= 2048 and w.B >= 512) else 0
         dec.set_option("fusion_path", args.fusion_path)
     for kv in args.set or []:
         k, v = kv.split("=")
@@ -593,7 +597,7 @@ def run_ours(args, w):
         a_row_ms = a_step * (a_kms["row"] / a_tot) / max(1e-9, a_kn["row"] / args.steps)
         a_flop = 2.0 * w.B * w.H * (w.V + 1)
         alt = {"fusion_path": alt_path,
-               "what": ("the same workload and decoder with the alt_path form of the greedy one-LM step: "
+               "what": ("the same workload and decoder with the other form of the greedy one-LM step: "
                         + ("the LM level-0 term in the joint epilogue with a per-row correction list" if alt_path
                            else "the streaming form (the joint writes every logit + defaults, the row pass "
                                 "applies the LM and trie terms)")),
@@ -641,7 +645,7 @@ def run_ours(args, w):
                   "peak_kind": f"{pk_kind} bf16 sustained (kernel timed inside the decode step)",
                   "algorithmic": f"2*M*H*(V+1) = {flop_per_launch:.4g} FLOP per launch (M={M} rows)",
                   "avg_launch_ms": joint_ms, "launches": kernel_n["joint"],
-                  "traffic": recorded_traffic(w, "joint"),
+                  "traffic": recorded_traffic(w, "joint", path=args.fusion_path if greedy1 else None),
                   "bytes_per_launch": joint_bytes,
                   "share_of_device_time": share_joint,
                   "isolated": {"cold_l2_ms": joint_cold, "warm_l2_ms": joint_warm,
@@ -673,7 +677,7 @@ def run_ours(args, w):
                                 f"joint input, every arc of the LM chain levels and trie chain nodes) plus the "
                                 f"shared unigram/root rows once per launch; the dense bias row is not counted"),
                 "avg_launch_ms": row_ms, "launches": kernel_n["row"],
-                "traffic": recorded_traffic(w, "row"),
+                "traffic": recorded_traffic(w, "row", path=args.fusion_path if greedy1 else None),
                 "share_of_device_time": share_row,
                 "isolated": {"what": "the chunk's last label step replayed with every row evaluated",
                              "bytes_per_launch": row_bytes, "cold_l2_ms": row_cold, "warm_l2_ms": row_warm,
@@ -795,7 +799,8 @@ def run_ours(args, w):
             "latency_per_chunk": latency_stats(step_ms),
             **({"alt_fusion_path": alt} if alt else {}),
             **({"stream_sweep": {"what": "the same workload (tables, weights, lambda, beta) decoded at other stream "
-                                         "counts B in this run: frames/s over K timed chunks (L2 flushed before "
+                                         "counts B in this run (each with the decoder's default fusion_path for "
+                                         "its stream count): frames/s over K timed chunks (L2 flushed before "
                                          "each) and chunk latency; 1 chunk = T x 80 ms of audio",
                                  "points": sweep}} if sweep else {}),
             **({"first_token_latency_s": {
