@@ -69,6 +69,7 @@ TRAFFIC = {
     (4, 1024, "joint", 1): (18074880, "826bf2360316aeca"),
     (4, 1024, "row", 1): (10575616, "673513be0b5541fe"),
     (4, 1024, "joint", 0): (11051264, "826bf2360316aeca"),
+    (4, 1024, "row", 0): (29131776, "2608d2dffbbc0675"),
 }
 
 

@@ -71,8 +71,8 @@ void enqueue_chunk(tsd_decoder* d, int M, int T, cudaStream_t s, const std::vect
     mark(0);
     if (d->cfg.beam_k > 1) launch_row_beam(v, M / d->cfg.beam_k, step, step == S ? 1 : 0, d->row_smem, s, pdl);
     else if (d->cfg.prune_k > 0) launch_row_pruned(v, M, step, step == S ? 1 : 0, s, pdl);
-    else if (v.fused && v.fz_dense) launch_row_fused(v, M, step, step == S ? 1 : 0, d->row_smem, s, pdl);
-    else if (v.fused) launch_row_stream(v, M, step, step == S ? 1 : 0, d->row_smem, s, pdl);
+    else if (v.fused && v.fz_dense) launch_row_fused(v, M, step, step == S ? 1 : 0, row_fused_smem_bytes(d->V4, d->N_pad), s, pdl);
+    else if (v.fused) launch_row_stream(v, M, step, step == S ? 1 : 0, row_stream_smem_bytes(d->V4), s, pdl);
     else launch_row(v, M, step, step == S ? 1 : 0, d->row_smem, s, pdl);
     if (pr.D) {
       // the prediction network reads the labels just emitted; after the last
@@ -1065,8 +1065,8 @@ extern "C" tsd_status tsd_decoder_replay(tsd_decoder* d, int32_t kernel, int32_t
   for (int i = 0; i < reps; ++i) {
     if (kernel == 0 && d->cfg.beam_k > 1) launch_row_beam(d->view, d->last_n, S - 1, 2, d->row_smem, s, false);
     else if (kernel == 0 && d->cfg.prune_k > 0) launch_row_pruned(d->view, M, S - 1, 2, s, false);
-    else if (kernel == 0 && d->view.fused && d->view.fz_dense) launch_row_fused(d->view, M, S - 1, 2, d->row_smem, s, false);
-    else if (kernel == 0 && d->view.fused) launch_row_stream(d->view, M, S - 1, 2, d->row_smem, s, false);
+    else if (kernel == 0 && d->view.fused && d->view.fz_dense) launch_row_fused(d->view, M, S - 1, 2, row_fused_smem_bytes(d->V4, d->N_pad), s, false);
+    else if (kernel == 0 && d->view.fused) launch_row_stream(d->view, M, S - 1, 2, row_stream_smem_bytes(d->V4), s, false);
     else if (kernel == 0) launch_row(d->view, M, S - 1, 2, d->row_smem, s, false);
     else if (d->joint_kind == 0) launch_joint_tc(*d->jtc, d->view, M, 1 << 30, s, false);
     else launch_joint(d->view, M, 1 << 30, s);

@@ -21,20 +21,22 @@
 // delta[v] = 0 for a label no chain element continues with.  For row r at
 // label step s the pass
 //   1. (before waiting for the joint kernel) loads the row's state and chains
-//      and finds each label's deepest LM chain level: a deeper level's labels
-//      are a subset of a shallower one's (the model is suffix-closed).  The
-//      levels above 0 (few arcs) offer ((l + 1) << 24 | position) to their
-//      labels' words by a shared-memory atomicMax, so the deepest wins; then
-//      level 0 (the previous label's continuations, up to every label) is
-//      streamed once (or, for a state with many continuations, read from its
-//      dense row: per label log p(v | u) - log p(v) - cum_0, 0 for no arc)
-//      and writes the delta of every label no level above offered, and the
-//      offers' winners (held in registers) write theirs.
-//      The trie chain nodes are scattered shallowest first (the deepest
-//      overwrites);
-//   2. (after the wait) the log-sum-exp from the tile partials and the argmax
-//      of logit + D + c_r + delta over the labels (blank: its logit alone;
-//      ties to the lowest label), i.e. the greedy decision and its fused score;
+//      (after the chunk's first step from the row's own copy, indexed by
+//      row) and builds delta[v] in shared memory.  Level 0 (the previous
+//      label's continuations, up to every label) is streamed once and writes
+//      every label's level-0 delta (for a state with many continuations from
+//      its dense row: per label log p(v | u) - log p(v) - cum_0, 0 for no
+//      arc); meanwhile every arc of the levels above 0 (few: they continue
+//      longer contexts) sets its level's bit in its label's level mask.  The
+//      model is suffix-closed (a deeper level's labels are a subset of a
+//      shallower one's), so a label's deepest level is its mask's highest bit,
+//      and after a barrier that level's arc (held in registers) overwrites the
+//      label's delta.  The trie chain nodes are scattered shallowest first
+//      (the deepest overwrites);
+//   2. (after the wait) the argmax of logit + D + c_r + delta over the labels
+//      (blank: its logit alone; ties to the lowest label), i.e. the greedy
+//      decision, and (for an emitted label) the log-sum-exp from the tile
+//      partials for its fused score;
 //   3. blank (or the per-frame label limit) advances the frame; a label y is
 //      emitted and advances the chains, assembled from independent searches
 //      of y in every chain element, each hit carrying the next state's table
@@ -71,7 +73,7 @@ template <int VAR>
 __global__ void __launch_bounds__(kFzThreads) __maxnreg__((VAR & 4) ? 128 : 72) k_row_fz(DecView d, int step, int mode) {
   constexpr bool PRED = (VAR & 1) != 0;
   constexpr int QB = 8;     // label quads per thread whose loads are issued together
-  constexpr int kHeld = 2;  // arc groups of four of the levels above 0 a thread keeps in registers
+  constexpr int kHeld = 1;  // arc groups of four of the levels above 0 a thread keeps in registers
   const Params* __restrict__ P = d.params;
   const int r = blockIdx.x;
   const int V = d.V;
@@ -79,11 +81,11 @@ __global__ void __launch_bounds__(kFzThreads) __maxnreg__((VAR & 4) ? 128 : 72) 
   const bool commit = (mode != 2);
   const bool counting = (mode == 2 || d.count);
   extern __shared__ __align__(16) unsigned char smem[];
-  // per label: the LM tag, then (for the winners) the LM delta's bits; 1 if
-  // the label has an LM delta; the trie goto depth (0: none)
-  uint32_t* key = reinterpret_cast<uint32_t*>(smem);      // [V4]
-  uint8_t* lmf = reinterpret_cast<uint8_t*>(key + d.V4);   // [V4]
-  uint8_t* dep = lmf + d.V4;                               // [V4]
+  // per label: its LM delta (0: none); the LM chain levels above 0 with an
+  // arc for it (bit l); its trie goto depth (0: none)
+  float* dlm = reinterpret_cast<float*>(smem);              // [V4]
+  uint16_t* lev = reinterpret_cast<uint16_t*>(dlm + d.V4);  // [V4]
+  uint8_t* dep = reinterpret_cast<uint8_t*>(lev + d.V4);    // [V4]
 
   __shared__ int s_t, s_sym, s_cnt, s_y, s_last, s_slot, s_T, s_n;
   __shared__ int s_nl, s_nt;
@@ -92,14 +94,13 @@ __global__ void __launch_bounds__(kFzThreads) __maxnreg__((VAR & 4) ? 128 : 72) 
   __shared__ float* s_out_score;
   __shared__ int32_t* s_out_count;
   __shared__ const uint16_t* s_enc;
-  __shared__ float s_lam, s_beta, s_score, s_lse, s_cr;
+  __shared__ float s_lam, s_beta, s_score, s_lse;
   __shared__ int s_lm[kLmChain], s_tr[kTrChain];
   __shared__ int4 s_lmr[kLmChain];    // LM chain records: (first arc, arcs, summed backoff bits, -)
   __shared__ int4 s_trr[kTrChain];    // trie chain records: (first child, children, depth of the children, -)
   __shared__ int4 s_lm_hit[kLmChain]; // target record of y's arc at each old level (x = -2: none)
   __shared__ int4 s_tr_hit[kTrChain]; // child record of y at each old trie node (x = -1: none)
   __shared__ int4 s_uni_hit, s_root_hit;
-  __shared__ int s_gbeg[kLmChain + 1];  // arc groups of the LM levels before level l
   __shared__ float s_bv[kFzWarps];
   __shared__ int s_bi[kFzWarps];
   __shared__ unsigned long long s_bytes;  // algorithmic bytes of the row-step (when counting)
@@ -108,6 +109,9 @@ __global__ void __launch_bounds__(kFzThreads) __maxnreg__((VAR & 4) ? 128 : 72) 
   // 1. Row state.  It was written by the previous row pass; under
   // programmatic launch this grid may start before its own wait, so these
   // loads go through L2 only (ld.global.cg), never a possibly stale L1 line.
+  // After the chunk's first step the row's own copy of its state is read,
+  // indexed by row, together with the slot (the chains are read whole: their
+  // arrays have room for the longest).
   if (tid == 0) {
     const int slot = __ldcg(P->slots + r);
     s_slot = slot;
@@ -122,45 +126,67 @@ __global__ void __launch_bounds__(kFzThreads) __maxnreg__((VAR & 4) ? 128 : 72) 
     s_n = P->n;
     s_bytes = 0;
     s_bad = !checked(slot >= 0 && slot < d.lm_stride, d.err, 1);
+    if (step > 0) {
+      s_t = __ldcg(d.r_t + r); s_sym = __ldcg(d.r_sym + r); s_cnt = __ldcg(d.r_cnt + r);
+      s_nl = __ldcg(d.m_lm_len + r);
+      s_nt = __ldcg(d.m_tr_len + r);
+      s_last = __ldcg(d.m_last + r);
+    }
+  } else if (step > 0 && tid >= 32 && tid < 32 + kLmChain) {
+    const int l = tid - 32;
+    s_lm[l] = __ldcg(d.m_lm + (size_t)r * kLmChain + l);
+    s_lmr[l] = __ldcg(d.m_lmr + (size_t)r * kLmChain + l);
+  } else if (step > 0 && tid >= 64 && tid < 64 + kTrChain) {
+    const int k = tid - 64;
+    s_tr[k] = __ldcg(d.m_tr + (size_t)r * kTrChain + k);
+    s_trr[k] = __ldcg(d.m_trr + (size_t)r * kTrChain + k);
   }
-  {  // per-label scratch reset
-    uint4* k4 = reinterpret_cast<uint4*>(key);
-    uint32_t* f4 = reinterpret_cast<uint32_t*>(lmf);
+  {  // per-label scratch reset (the deltas are reset once the state is known)
+    uint2* v4 = reinterpret_cast<uint2*>(lev);
     uint32_t* e4 = reinterpret_cast<uint32_t*>(dep);
     for (int q = tid; q < d.V4 / 4; q += blockDim.x) {
-      k4[q] = make_uint4(0u, 0u, 0u, 0u);
-      f4[q] = 0u;
+      v4[q] = make_uint2(0u, 0u);
       e4[q] = 0u;
     }
   }
   row::block_sync();
   if (s_bad) return;
   const int slot = s_slot, T = s_T;
-  // the chains are read whole (their arrays have room for the longest), so
-  // their lengths need not be known first
-  if (tid == 0) {
-    if (step == 0) {
+  if (step == 0) {
+    // the chunk's first step: the stream's state by slot, and the row's copy
+    if (tid == 0) {
       s_t = 0; s_sym = 0; s_cnt = 0;
-    } else {
-      s_t = __ldcg(d.r_t + r); s_sym = __ldcg(d.r_sym + r); s_cnt = __ldcg(d.r_cnt + r);
+      s_nl = d.has_lm ? __ldcg(d.s_lm_len + slot) : 0;
+      s_nt = d.has_tr ? __ldcg(d.s_tr_len + slot) : 0;
+      s_last = __ldcg(d.s_last + slot);
+      if (commit) {
+        d.m_lm_len[r] = s_nl;
+        d.m_tr_len[r] = s_nt;
+        d.m_last[r] = s_last;
+      }
+    } else if (tid >= 32 && tid < 32 + kLmChain) {
+      const int l = tid - 32;
+      if (d.has_lm) {
+        s_lm[l] = __ldcg(d.s_lm_chain + (size_t)slot * kLmChain + l);
+        s_lmr[l] = __ldcg(d.s_lm_rec + (size_t)slot * kLmChain + l);
+        if (commit) {
+          d.m_lm[(size_t)r * kLmChain + l] = s_lm[l];
+          d.m_lmr[(size_t)r * kLmChain + l] = s_lmr[l];
+        }
+      }
+    } else if (tid >= 64 && tid < 64 + kTrChain) {
+      const int k = tid - 64;
+      if (d.has_tr) {
+        s_tr[k] = __ldcg(d.s_tr_chain + slot * kTrChain + k);
+        s_trr[k] = __ldcg(d.s_tr_rec + (size_t)slot * kTrChain + k);
+        if (commit) {
+          d.m_tr[(size_t)r * kTrChain + k] = s_tr[k];
+          d.m_trr[(size_t)r * kTrChain + k] = s_trr[k];
+        }
+      }
     }
-    s_nl = d.has_lm ? __ldcg(d.s_lm_len + slot) : 0;
-    s_nt = d.has_tr ? __ldcg(d.s_tr_len + slot) : 0;
-    s_last = __ldcg(d.s_last + slot);
-  } else if (tid >= 32 && tid < 32 + kLmChain) {
-    const int l = tid - 32;
-    if (d.has_lm) {
-      s_lm[l] = __ldcg(d.s_lm_chain + (size_t)slot * kLmChain + l);
-      s_lmr[l] = __ldcg(d.s_lm_rec + (size_t)slot * kLmChain + l);
-    }
-  } else if (tid >= 64 && tid < 64 + kTrChain) {
-    const int k = tid - 64;
-    if (d.has_tr) {
-      s_tr[k] = __ldcg(d.s_tr_chain + slot * kTrChain + k);
-      s_trr[k] = __ldcg(d.s_tr_rec + (size_t)slot * kTrChain + k);
-    }
+    row::block_sync();
   }
-  row::block_sync();
 #ifdef TSD_CHECKS
   if (tid == 0) {  // every index the row will follow is inside its table
     bool ok = checked(s_nl >= 0 && s_nl <= kLmChain && s_nt >= 0 && s_nt <= kTrChain, d.err, 2) &&
@@ -195,40 +221,26 @@ __global__ void __launch_bounds__(kFzThreads) __maxnreg__((VAR & 4) ? 128 : 72) 
   const float bscale = s_beta * (d.has_tr ? d.tr.bonus : 0.f);
 
   if (evaluated) {
-    if (tid == 0) {
-      // arc groups of the levels above level 0 (level 0 is streamed apart)
-      int g = 0;
-      unsigned long long ab = 0;
-      for (int l = 0; l < nl_old; ++l) {
-        s_gbeg[l] = g;
-        if (l > 0) g += level_groups(s_lmr[l].x, s_lmr[l].y);
-        ab += 16 + 8ull * s_lmr[l].y;
-      }
-      s_gbeg[nl_old] = g;
-      for (int k = 0; k < nt_old; ++k) ab += 16 + 4ull * s_trr[k].y;
-      const float cum_top = nl_old ? __int_as_float(s_lmr[nl_old - 1].z) : 0.f;
-      const int depth_cur = nt_old ? s_trr[0].z - 1 : 0;
-      s_cr = lam * cum_top - bscale * (float)depth_cur;
-      // Algorithmic bytes (when counting): the row's logits and partials
-      // read, the row state read and written, every arc of every LM chain
-      // level (label + log-probability) and every child of every trie chain
-      // node (label) with its record; searches and the joint input are added
-      // where they happen; the call's shared rows once per launch by the host.
-      s_bytes = ab + 4ull * (V + 1) + 16ull * d.n_ptiles + 2ull * (24 + 4 * (nl_old + nt_old));
-    }
-    row::block_sync();
     const int4* t4 = reinterpret_cast<const int4*>(d.lm.arc_tok);
     const float4* p4 = reinterpret_cast<const float4*>(d.lm.arc_logp);
-    // the group g of the levels above 0: its level and first arc
+    // the aligned arc groups of the levels above 0, in level order: group g's
+    // level and first arc (g below their count G)
+    int G = 0;
+    for (int l = 1; l < nl_old; ++l) G += level_groups(s_lmr[l].x, s_lmr[l].y);
     auto locate = [&](int g, int& l) {
-      l = 1;
-      while (g >= s_gbeg[l + 1]) ++l;
-      return (s_lmr[l].x & ~3) + 4 * (g - s_gbeg[l]);
+      for (l = 1;; ++l) {
+        const int n = level_groups(s_lmr[l].x, s_lmr[l].y);
+        if (g < n) break;
+        g -= n;
+      }
+      return (s_lmr[l].x & ~3) + 4 * g;
     };
-    // 1a. the levels above 0 (few arcs: they continue longer contexts) offer
-    //     ((l + 1) << 24 | position) to their labels by atomicMax, so the
-    //     deepest wins; their labels and log-probabilities stay in registers
-    const int G = s_gbeg[nl_old];
+    auto delta_of = [&](int l, float lp, int v) {
+      return lam * (lp - __int_as_float(s_lmr[l].z)) - lam * __ldg(d.lm.uni_logp + v);
+    };
+    // 1a. the levels above 0 (few arcs: they continue longer contexts): each
+    //     thread loads its first arc groups, labels and log-probabilities,
+    //     and keeps them in registers
     int4 ht[kHeld];
     float4 hp[kHeld];
     int hl[kHeld], hi[kHeld];
@@ -245,41 +257,14 @@ __global__ void __launch_bounds__(kFzThreads) __maxnreg__((VAR & 4) ? 128 : 72) 
         hl[u] = l;
       }
     }
-    auto offer = [&](int l, int i0, int4 tk) {
-      const int b = s_lmr[l].x, c = s_lmr[l].y;
-      const uint32_t tag = (uint32_t)(l + 1) << 24;
-      const int tv[4] = {tk.x, tk.y, tk.z, tk.w};
-#pragma unroll
-      for (int j = 0; j < 4; ++j)
-        if (i0 + j >= b && i0 + j < b + c && checked(tv[j] >= 0 && tv[j] < V, d.err, 9))
-          atomicMax(key + tv[j], tag | (uint32_t)(i0 + j - b));
-    };
-#pragma unroll
-    for (int u = 0; u < kHeld; ++u)
-      if (hl[u] >= 0) offer(hl[u], hi[u], ht[u]);
-    for (int g = tid + kHeld * kFzThreads; g < G; g += kFzThreads) {  // past what registers hold
-      int l;
-      const int i0 = locate(g, l);
-      offer(l, i0, __ldg(t4 + (i0 >> 2)));
-    }
-    if (nt_old > 0) {
-      const int k = nt_old - 1;
-      row::scatter_trie_node(d.tr.ch_tok, s_trr[k].x, s_trr[k].x + s_trr[k].y, (uint8_t)s_trr[k].z, dep);
-    }
-    row::block_sync();
-    // 1b. level 0 (the previous label's continuations, up to all V labels)
-    //     streamed once, labels and log-probabilities together: its arc is
-    //     the deepest for v exactly when no level above offered v (their
-    //     labels are a subset of level 0's), and then it writes v's delta at
-    //     once -- no level above ever looks at such a label.  The levels
-    //     above judge their offers meanwhile.
-    auto delta_of = [&](int l, float lp, int v) {
-      return lam * (lp - __int_as_float(s_lmr[l].z)) - lam * __ldg(d.lm.uni_logp + v);
-    };
+    // 1b. level 0 (the previous label's continuations, up to all V labels),
+    //     streamed once: every label's level-0 delta (0 for no arc), which
+    //     the deepest level above overwrites below
     if (nl_old > 0 && s_lmr[0].w >= 0 && s_lmr[0].y >= max(32, V / 8)) {  // many continuations
       // the state's dense row: per label log p(v | u) - log p(v) - cum_0, 0
       // for no arc (whose delta is 0 as well), contiguous
       const float4* R = reinterpret_cast<const float4*>(d.lm.dense0 + (size_t)s_lmr[0].w * d.lm.V4);
+      float4* k4 = reinterpret_cast<float4*>(dlm);
       const int nq4 = d.lm.V4 / 4;
       for (int q0 = tid; q0 < nq4; q0 += kDense * kFzThreads) {
         float4 rq[kDense];
@@ -291,20 +276,16 @@ __global__ void __launch_bounds__(kFzThreads) __maxnreg__((VAR & 4) ? 128 : 72) 
 #pragma unroll
         for (int u = 0; u < kDense; ++u) {
           const int q = q0 + u * kFzThreads;
-          if (q < nq4) {
-            const uint4 kq = reinterpret_cast<const uint4*>(key)[q];
-            const float rv[4] = {rq[u].x, rq[u].y, rq[u].z, rq[u].w};
-            const uint32_t kv[4] = {kq.x, kq.y, kq.z, kq.w};
-#pragma unroll
-            for (int j = 0; j < 4; ++j)
-              if (rv[j] != 0.f && kv[j] == 0u) {
-                key[4 * q + j] = __float_as_uint(lam * rv[j]);
-                lmf[4 * q + j] = 1;
-              }
-          }
+          if (q < nq4) k4[q] = make_float4(lam * rq[u].x, lam * rq[u].y, lam * rq[u].z, lam * rq[u].w);
         }
       }
-    } else if (nl_old > 0) {
+    } else {
+      // every label's delta starts at 0 (a dense row above writes them all)
+      float4* k4 = reinterpret_cast<float4*>(dlm);
+      for (int q = tid; q < d.V4 / 4; q += blockDim.x) k4[q] = make_float4(0.f, 0.f, 0.f, 0.f);
+      row::block_sync();
+    }
+    if (nl_old > 0 && !(s_lmr[0].w >= 0 && s_lmr[0].y >= max(32, V / 8))) {
       const int b0 = s_lmr[0].x, c0 = s_lmr[0].y;
       const int a0 = b0 & ~3, G0 = level_groups(b0, c0);
       for (int gb = 0; gb < G0; gb += kStream * kFzThreads) {
@@ -327,87 +308,70 @@ __global__ void __launch_bounds__(kFzThreads) __maxnreg__((VAR & 4) ? 128 : 72) 
             const float pv[4] = {lp[u].x, lp[u].y, lp[u].z, lp[u].w};
 #pragma unroll
             for (int j = 0; j < 4; ++j)
-              if (i0 + j >= b0 && i0 + j < b0 + c0 && checked(tv[j] >= 0 && tv[j] < V, d.err, 9) &&
-                  key[tv[j]] == 0u) {
-                key[tv[j]] = __float_as_uint(delta_of(0, pv[j], tv[j]));
-                lmf[tv[j]] = 1;
-              }
+              if (i0 + j >= b0 && i0 + j < b0 + c0 && checked(tv[j] >= 0 && tv[j] < V, d.err, 9))
+                dlm[tv[j]] = delta_of(0, pv[j], tv[j]);
           }
         }
       }
     }
-    // the winners among the offers (one per label), deltas kept until every
-    // offer is judged
-    uint32_t won = 0;  // bit 4u + j: arc j of held group u won
-    float wv[kHeld][4];
+    // 1c. every arc of the levels above 0 sets its level's bit in its
+    //     label's word (two labels per 32-bit word), so a label's deepest
+    //     level with an arc is its highest bit
+    uint32_t* lev2 = reinterpret_cast<uint32_t*>(lev);
+    auto offer = [&](int l, int i0, int4 tk) {
+      const int b = s_lmr[l].x, c = s_lmr[l].y;
+      const int tv[4] = {tk.x, tk.y, tk.z, tk.w};
+#pragma unroll
+      for (int j = 0; j < 4; ++j)
+        if (i0 + j >= b && i0 + j < b + c && checked(tv[j] >= 0 && tv[j] < V, d.err, 9))
+          atomicOr(lev2 + (tv[j] >> 1), 1u << (l + 16 * (tv[j] & 1)));
+    };
+#pragma unroll
+    for (int u = 0; u < kHeld; ++u)
+      if (hl[u] >= 0) offer(hl[u], hi[u], ht[u]);
+    for (int g = tid + kHeld * kFzThreads; g < G; g += kFzThreads) {  // past what registers hold
+      int l;
+      const int i0 = locate(g, l);
+      offer(l, i0, __ldg(t4 + (i0 >> 2)));
+    }
+    if (nt_old > 0) {  // the trie chain nodes, shallowest first (the deepest overwrites)
+      const int k = nt_old - 1;
+      row::scatter_trie_node(d.tr.ch_tok, s_trr[k].x, s_trr[k].x + s_trr[k].y, (uint8_t)s_trr[k].z, dep);
+    }
+    row::block_sync();
+    // 1d. the arc of each label at its deepest level writes the label's delta
+    //     (one writer per label: a level's arcs have distinct labels)
+    auto deepest = [&](int v) { return 31 - __clz((int)lev[v]); };
 #pragma unroll
     for (int u = 0; u < kHeld; ++u) {
       if (hl[u] >= 0) {
         const int l = hl[u], b = s_lmr[l].x, c = s_lmr[l].y;
-        const uint32_t tag = (uint32_t)(l + 1) << 24;
         const int tv[4] = {ht[u].x, ht[u].y, ht[u].z, ht[u].w};
         const float pv[4] = {hp[u].x, hp[u].y, hp[u].z, hp[u].w};
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
           const int i = hi[u] + j;
-          wv[u][j] = 0.f;
-          if (i >= b && i < b + c && checked(tv[j] >= 0 && tv[j] < V, d.err, 9) &&
-              key[tv[j]] == (tag | (uint32_t)(i - b))) {
-            won |= 1u << (4 * u + j);
-            wv[u][j] = delta_of(l, pv[j], tv[j]);
-          }
+          if (i >= b && i < b + c && checked(tv[j] >= 0 && tv[j] < V, d.err, 9) && deepest(tv[j]) == l)
+            dlm[tv[j]] = delta_of(l, pv[j], tv[j]);
         }
       }
+    }
+    for (int g = tid + kHeld * kFzThreads; g < G; g += kFzThreads) {  // past what registers hold
+      int l;
+      const int i0 = locate(g, l);
+      const int4 tk = __ldg(t4 + (i0 >> 2));
+      const float4 lq = __ldg(p4 + (i0 >> 2));
+      const int b = s_lmr[l].x, c = s_lmr[l].y;
+      const int tv[4] = {tk.x, tk.y, tk.z, tk.w};
+      const float pv[4] = {lq.x, lq.y, lq.z, lq.w};
+#pragma unroll
+      for (int j = 0; j < 4; ++j)
+        if (i0 + j >= b && i0 + j < b + c && checked(tv[j] >= 0 && tv[j] < V, d.err, 9) && deepest(tv[j]) == l)
+          dlm[tv[j]] = delta_of(l, pv[j], tv[j]);
     }
     if (nt_old > 1) {
       const int k = nt_old - 2;
       row::scatter_trie_node(d.tr.ch_tok, s_trr[k].x, s_trr[k].x + s_trr[k].y, (uint8_t)s_trr[k].z, dep);
-    }
-    row::block_sync();
-#pragma unroll
-    for (int u = 0; u < kHeld; ++u) {
-      const int tv[4] = {ht[u].x, ht[u].y, ht[u].z, ht[u].w};
-#pragma unroll
-      for (int j = 0; j < 4; ++j)
-        if ((won >> (4 * u + j)) & 1u) {
-          key[tv[j]] = __float_as_uint(wv[u][j]);
-          lmf[tv[j]] = 1;
-        }
-    }
-    // offers past what registers hold (rows whose longer contexts have very
-    // many continuations): judged a round at a time, a barrier between the
-    // judging and the writing; a label already written is skipped by its flag
-    for (int g0 = kHeld * kFzThreads; g0 < G; g0 += kFzThreads) {
-      row::block_sync();
-      const int g = g0 + tid;
-      int4 tk = make_int4(0, 0, 0, 0);
-      float xv[4] = {0.f, 0.f, 0.f, 0.f};
-      uint32_t xw = 0;
-      if (g < G) {
-        int l;
-        const int i0 = locate(g, l);
-        tk = __ldg(t4 + (i0 >> 2));
-        const float4 lq = __ldg(p4 + (i0 >> 2));
-        const int b = s_lmr[l].x, c = s_lmr[l].y;
-        const uint32_t tag = (uint32_t)(l + 1) << 24;
-        const int tv[4] = {tk.x, tk.y, tk.z, tk.w};
-        const float pv[4] = {lq.x, lq.y, lq.z, lq.w};
-#pragma unroll
-        for (int j = 0; j < 4; ++j)
-          if (i0 + j >= b && i0 + j < b + c && checked(tv[j] >= 0 && tv[j] < V, d.err, 9) && lmf[tv[j]] == 0 &&
-              key[tv[j]] == (tag | (uint32_t)(i0 + j - b))) {
-            xw |= 1u << j;
-            xv[j] = delta_of(l, pv[j], tv[j]);
-          }
-      }
-      row::block_sync();
-      const int tv[4] = {tk.x, tk.y, tk.z, tk.w};
-#pragma unroll
-      for (int j = 0; j < 4; ++j)
-        if ((xw >> j) & 1u) {
-          key[tv[j]] = __float_as_uint(xv[j]);
-          lmf[tv[j]] = 1;
-        }
     }
     for (int k = nt_old - 3; k >= 0; --k) {
       row::block_sync();
@@ -422,32 +386,31 @@ __global__ void __launch_bounds__(kFzThreads) __maxnreg__((VAR & 4) ? 128 : 72) 
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
   if (evaluated) {
-    // 2. log-sum-exp (warp 0, from the tile partials) and the argmax of
-    //    logit + D + c_r + delta over the labels; blank takes its logit
+    // 2. the argmax of logit + D + c_r + delta over the labels (blank takes
+    //    its logit alone); the log-sum-exp of the raw logits (from the tile
+    //    partials) is needed only for an emitted label's score
     const float* lg = d.logits + (size_t)r * d.N_pad;
-    if (warp == 0) {
-      float m = kNegInf, s = 0.f;
-      const float4* pr = d.part + (size_t)r * d.n_ptiles;
-      for (int j = lane; j < d.n_ptiles; j += 32) {
-        const float4 p = __ldcg(pr + j);  // written by the joint kernel just before
-        lse_merge(m, s, p.x, p.y);
-      }
-      row::reconverge();
-      for (int o = 16; o > 0; o >>= 1) {
-        const float m2 = __shfl_xor_sync(0xffffffffu, m, o);
-        const float s2 = __shfl_xor_sync(0xffffffffu, s, o);
-        lse_merge(m, s, m2, s2);
-      }
-      if (lane == 0) s_lse = m + logf(s);
+    if (counting && tid == 0) {
+      // Algorithmic bytes: the row's logits and partials read, the row state
+      // read and written, every arc of every LM chain level (label +
+      // log-probability) and every child of every trie chain node (label)
+      // with its record; searches and the joint input are added where they
+      // happen; the call's shared rows once per launch by the host.
+      unsigned long long ab = 0;
+      for (int l = 0; l < nl_old; ++l) ab += 16 + 8ull * s_lmr[l].y;
+      for (int k = 0; k < nt_old; ++k) ab += 16 + 4ull * s_trr[k].y;
+      s_bytes = ab + 4ull * (V + 1) + 16ull * d.n_ptiles + 2ull * (24 + 4 * (nl_old + nt_old));
     }
     float bv = kNegInf;
     int bi = INT_MAX;
     {
-      const float cr = s_cr;
+      // c_r = lambda*(summed backoff of the state) - beta*bonus*depth
+      const float cum_top = nl_old ? __int_as_float(s_lmr[nl_old - 1].z) : 0.f;
+      const int depth_cur = nt_old ? s_trr[0].z - 1 : 0;
+      const float cr = lam * cum_top - bscale * (float)depth_cur;
       const int nq = (V + 3) >> 2;  // quads holding labels < V
       const float4* l4 = reinterpret_cast<const float4*>(lg);
-      const uint4* k4 = reinterpret_cast<const uint4*>(key);
-      const uint32_t* f4 = reinterpret_cast<const uint32_t*>(lmf);
+      const float4* k4 = reinterpret_cast<const float4*>(dlm);
       const uint32_t* e4 = reinterpret_cast<const uint32_t*>(dep);
       for (int q0 = tid; q0 < nq; q0 += QB * kFzThreads) {
         float4 lq[QB];
@@ -460,16 +423,14 @@ __global__ void __launch_bounds__(kFzThreads) __maxnreg__((VAR & 4) ? 128 : 72) 
         for (int u = 0; u < QB; ++u) {
           const int q = q0 + u * kFzThreads;
           if (q < nq) {
-            const uint32_t fq = f4[q], eq = e4[q];
+            const float4 kq = k4[q];
+            const uint32_t eq = e4[q];
             const float lv[4] = {lq[u].x, lq[u].y, lq[u].z, lq[u].w};
-            float dl[4] = {0.f, 0.f, 0.f, 0.f};
-            if (fq | eq) {  // a label of this quad has an LM or trie delta
-              const uint4 kq = k4[q];
-              const uint32_t kv[4] = {kq.x, kq.y, kq.z, kq.w};
+            float dl[4] = {kq.x, kq.y, kq.z, kq.w};
+            if (eq) {  // a label of this quad has a trie goto node
               const uint32_t rb = __ldg(d.droot + (q >> 3)) >> ((4 * q) & 31);
 #pragma unroll
               for (int j = 0; j < 4; ++j) {
-                if ((fq >> (8 * j)) & 0xffu) dl[j] = __uint_as_float(kv[j]);
                 const uint32_t e = (eq >> (8 * j)) & 0xffu;
                 if (e) dl[j] += bscale * (float)e - (((rb >> j) & 1u) ? bscale : 0.f);
               }
@@ -506,7 +467,7 @@ __global__ void __launch_bounds__(kFzThreads) __maxnreg__((VAR & 4) ? 128 : 72) 
     const int y = (bix >= 0 && bix <= V) ? bix : V;
     if (tid == 0) {
       s_y = y;
-      s_score = b - s_lse;
+      s_score = b;  // the fused score less the log-sum-exp
     }
     if (!PRED) row::prefetch_span(d.E + (size_t)(y != V ? y : s_last) * d.H, (size_t)d.H * 2, 32);
     if (y != V) {
@@ -517,6 +478,10 @@ __global__ void __launch_bounds__(kFzThreads) __maxnreg__((VAR & 4) ? 128 : 72) 
       } else if (tid == kFzThreads - 2) {
         s_uni_hit = (d.has_lm && d.lm.order >= 2) ? __ldg(d.lm.uni_rec + y) : make_int4(-1, 0, 0, 0);
       }
+      // the last warp's first tile partials load while it searches
+      const float4* pr = d.part + (size_t)r * d.n_ptiles;
+      float4 p0 = make_float4(kNegInf, 0.f, 0.f, 0.f);
+      if (warp == kFzWarps - 1 && lane < d.n_ptiles) p0 = __ldcg(pr + lane);  // written by the joint kernel
       for (int task = warp; task < nl_old + nt_old; task += kFzWarps) {
         if (task < nl_old) {
           const int b = s_lmr[task].x, c = s_lmr[task].y;
@@ -530,6 +495,21 @@ __global__ void __launch_bounds__(kFzThreads) __maxnreg__((VAR & 4) ? 128 : 72) 
           if (lane == 0) s_tr_hit[k] = (i >= 0) ? __ldg(d.tr.ch_rec + b + i) : make_int4(-1, 0, 0, 0);
           if (counting && lane == 0) atomicAdd(&s_bytes, 4ull * (32 - __clz(c + 1)) + 16);
         }
+      }
+      if (warp == kFzWarps - 1) {  // the log-sum-exp of the raw logits
+        float pm = kNegInf, ps = 0.f;
+        lse_merge(pm, ps, p0.x, p0.y);
+        for (int j = lane + 32; j < d.n_ptiles; j += 32) {
+          const float4 p = __ldcg(pr + j);
+          lse_merge(pm, ps, p.x, p.y);
+        }
+        row::reconverge();
+        for (int o = 16; o > 0; o >>= 1) {
+          const float m2 = __shfl_xor_sync(0xffffffffu, pm, o);
+          const float s2 = __shfl_xor_sync(0xffffffffu, ps, o);
+          lse_merge(pm, ps, m2, s2);
+        }
+        if (lane == 0) s_lse = pm + logf(ps);
       }
       row::block_sync();
       // 3b. assemble the new chains in place (shared memory) and emit
@@ -553,6 +533,7 @@ __global__ void __launch_bounds__(kFzThreads) __maxnreg__((VAR & 4) ? 128 : 72) 
           }
         }
         s_nl = ln;
+        if (commit) d.m_lm_len[r] = ln;
         // trie: y's children of the old chain nodes (deepest first), then the
         // root's; completing a phrase (the deepest match's next is 0) resets
         int tn = 0;
@@ -583,12 +564,14 @@ __global__ void __launch_bounds__(kFzThreads) __maxnreg__((VAR & 4) ? 128 : 72) 
         if (commit) {
           if (d.has_lm) d.s_lm_len[slot] = ln;
           if (d.has_tr) d.s_tr_len[slot] = tn;
+          d.m_tr_len[r] = tn;
           const int cap = T * d.max_sym;
           const int o = r * cap + s_cnt;
           s_out_tok[o] = y;
           s_out_frame[o] = s_t;
-          s_out_score[o] = s_score;
+          s_out_score[o] = s_score - s_lse;
           d.s_last[slot] = y;
+          d.m_last[r] = y;
         }
         s_cnt += 1;
         s_last = y;
@@ -596,15 +579,19 @@ __global__ void __launch_bounds__(kFzThreads) __maxnreg__((VAR & 4) ? 128 : 72) 
         if (s_sym >= d.max_sym) { s_t += 1; s_sym = 0; }
       }
       row::block_sync();
-      if (commit) {  // the new chains and their records, for the next step
+      if (commit) {  // the new chains and their records, for the next step (by slot and by row)
         if (tid < s_nl) {
           d.s_lm_chain[(size_t)slot * kLmChain + tid] = s_lm[tid];
           d.s_lm_rec[(size_t)slot * kLmChain + tid] = s_lmr[tid];
+          d.m_lm[(size_t)r * kLmChain + tid] = s_lm[tid];
+          d.m_lmr[(size_t)r * kLmChain + tid] = s_lmr[tid];
         }
         if (tid >= 64 && tid - 64 < s_nt) {
           const int k = tid - 64;
           d.s_tr_chain[slot * kTrChain + k] = s_tr[k];
           d.s_tr_rec[(size_t)slot * kTrChain + k] = s_trr[k];
+          d.m_tr[(size_t)r * kTrChain + k] = s_tr[k];
+          d.m_trr[(size_t)r * kTrChain + k] = s_trr[k];
         }
       }
     } else if (tid == 0) {
@@ -665,7 +652,7 @@ __global__ void __launch_bounds__(kFzThreads) __maxnreg__((VAR & 4) ? 128 : 72) 
 
 }  // namespace
 
-size_t row_stream_smem_bytes(int V4) { return (size_t)V4 * (sizeof(uint32_t) + 2 * sizeof(uint8_t)); }
+size_t row_stream_smem_bytes(int V4) { return (size_t)V4 * (sizeof(float) + sizeof(uint16_t) + sizeof(uint8_t)); }
 
 cudaError_t prepare_stream_kernels(size_t smem) {
   cudaError_t e = cudaFuncSetAttribute(k_row_fz<0>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
