@@ -512,59 +512,86 @@ __global__ void __launch_bounds__(kFzThreads) __maxnreg__((VAR & 4) ? 128 : 72) 
         if (lane == 0) s_lse = pm + logf(ps);
       }
       row::block_sync();
-      // 3b. assemble the new chains in place (shared memory) and emit
-      if (tid == 0) {
-        // LM: y's unigram state, then the target of y's arc at every level
-        // of the old chain up to the first level without one
+      // 3b. assemble the new chains in place (shared memory) and commit them
+      //     (by slot, and by row for the next step): warp 0 the LM chain
+      //     (y's unigram state, then the targets of y's arcs at the old levels
+      //     up to the first level without one), warp 1 the trie chain (y's
+      //     children of the old chain nodes, deepest first, then the root's;
+      //     completing a phrase resets it), warp 2 the outputs
+      if (warp == 0) {
         int ln = 0;
-        const int4 u = s_uni_hit;
         if (d.has_lm && d.lm.order >= 2) {
-          s_lm[0] = 1 + y;  // the unigram state of y; u.x is its dense row
-          s_lmr[0] = make_int4(u.y, u.z, u.w, u.x);
-          ln = 1;
-          for (int l = 0; l < nl_old && ln < kLmChain; ++l) {
-            const int4 h = s_lm_hit[l];
-            if (h.x < 0) break;  // no arc at this level (-2) or the top order (-1)
-            if (!checked(h.x < d.lm.n_states && h.y >= 0 && h.z >= 0 && (int64_t)h.y + h.z <= d.lm.n_arcs, d.err, 10))
-              break;
-            s_lm[ln] = h.x;
-            s_lmr[ln] = make_int4(h.y, h.z, h.w, 0);
-            ++ln;
+          const int4 h = lane < nl_old ? s_lm_hit[lane] : make_int4(-2, 0, 0, 0);
+          const bool cont =
+              h.x >= 0 && checked(h.x < d.lm.n_states && h.y >= 0 && h.z >= 0 && (int64_t)h.y + h.z <= d.lm.n_arcs,
+                                  d.err, 10);
+          const unsigned miss = __ballot_sync(0xffffffffu, !cont);
+          ln = 1 + min(miss ? __ffs((int)miss) - 1 : 32, kLmChain - 1);
+          const int4 u = s_uni_hit;  // u.x is y's dense row
+          // lane l >= 1 takes the hit of old level l - 1
+          const int px = __shfl_up_sync(0xffffffffu, h.x, 1), py = __shfl_up_sync(0xffffffffu, h.y, 1);
+          const int pz = __shfl_up_sync(0xffffffffu, h.z, 1), pw = __shfl_up_sync(0xffffffffu, h.w, 1);
+          const int nst = lane == 0 ? 1 + y : px;
+          const int4 nrec = lane == 0 ? make_int4(u.y, u.z, u.w, u.x) : make_int4(py, pz, pw, 0);
+          __syncwarp();
+          if (lane < ln) {
+            s_lm[lane] = nst;
+            s_lmr[lane] = nrec;
+            if (commit) {
+              d.s_lm_chain[(size_t)slot * kLmChain + lane] = nst;
+              d.s_lm_rec[(size_t)slot * kLmChain + lane] = nrec;
+              d.m_lm[(size_t)r * kLmChain + lane] = nst;
+              d.m_lmr[(size_t)r * kLmChain + lane] = nrec;
+            }
           }
         }
-        s_nl = ln;
-        if (commit) d.m_lm_len[r] = ln;
-        // trie: y's children of the old chain nodes (deepest first), then the
-        // root's; completing a phrase (the deepest match's next is 0) resets
-        int tn = 0;
-        bool reset = false;
-        for (int i = 0; i < nt_old; ++i) {
-          const int4 h = s_tr_hit[i];
-          if (h.x < 0) continue;
-          if (!checked(h.x > 0 && h.x < d.tr.n_nodes && h.w >= 0 && h.z + h.w <= d.tr.n_children, d.err, 11)) continue;
-          if (tn == 0 && h.y == 0) reset = true;
-          const int dd = s_trr[i].z + 1;  // the child's children sit one deeper
-          if (tn < kTrChain) {
-            s_tr[tn] = h.x;
-            s_trr[tn] = make_int4(h.z, h.w, dd, 0);
-            ++tn;
+        if (lane == 0) {
+          s_nl = ln;
+          if (commit) {
+            if (d.has_lm) d.s_lm_len[slot] = ln;
+            d.m_lm_len[r] = ln;
           }
         }
+      } else if (warp == 1) {
+        const int4 h = lane < nt_old ? s_tr_hit[lane] : make_int4(-1, 0, 0, 0);
+        const int dd = lane < nt_old ? s_trr[lane].z + 1 : 0;  // the child's children sit one deeper
+        const bool ok = h.x >= 0 && checked(h.x > 0 && h.x < d.tr.n_nodes && h.w >= 0 && h.z + h.w <= d.tr.n_children,
+                                            d.err, 11);
+        const unsigned vm = __ballot_sync(0xffffffffu, ok);
+        const int nv = __popc(vm);
         const int4 rh = s_root_hit;
-        if (rh.x != 0) {
-          if (tn == 0 && rh.y == 0) reset = true;
-          if (tn < kTrChain) {
-            s_tr[tn] = rh.x;
-            s_trr[tn] = make_int4(rh.z, rh.w, 2, 0);
-            ++tn;
+        const bool root = rh.x != 0;
+        // the first element of the new chain ends a phrase: the chain resets
+        const int f = __ffs((int)vm) - 1;
+        const int fy = __shfl_sync(0xffffffffu, h.y, f < 0 ? 0 : f);
+        const bool reset = nv > 0 ? fy == 0 : (root && rh.y == 0);
+        const int tn = reset ? 0 : min(nv + (root ? 1 : 0), kTrChain);
+        __syncwarp();
+        const int pos = __popc(vm & ((1u << lane) - 1u));
+        if (ok && pos < tn) {
+          s_tr[pos] = h.x;
+          s_trr[pos] = make_int4(h.z, h.w, dd, 0);
+        }
+        if (lane == 0 && root && nv < tn) {
+          s_tr[nv] = rh.x;
+          s_trr[nv] = make_int4(rh.z, rh.w, 2, 0);
+        }
+        __syncwarp();
+        if (commit && lane < tn) {
+          d.s_tr_chain[slot * kTrChain + lane] = s_tr[lane];
+          d.s_tr_rec[(size_t)slot * kTrChain + lane] = s_trr[lane];
+          d.m_tr[(size_t)r * kTrChain + lane] = s_tr[lane];
+          d.m_trr[(size_t)r * kTrChain + lane] = s_trr[lane];
+        }
+        if (lane == 0) {
+          s_nt = tn;
+          if (commit) {
+            if (d.has_tr) d.s_tr_len[slot] = tn;
+            d.m_tr_len[r] = tn;
           }
         }
-        if (reset) tn = 0;
-        s_nt = tn;
+      } else if (tid == 64) {
         if (commit) {
-          if (d.has_lm) d.s_lm_len[slot] = ln;
-          if (d.has_tr) d.s_tr_len[slot] = tn;
-          d.m_tr_len[r] = tn;
           const int cap = T * d.max_sym;
           const int o = r * cap + s_cnt;
           s_out_tok[o] = y;
@@ -577,22 +604,6 @@ __global__ void __launch_bounds__(kFzThreads) __maxnreg__((VAR & 4) ? 128 : 72) 
         s_last = y;
         s_sym += 1;
         if (s_sym >= d.max_sym) { s_t += 1; s_sym = 0; }
-      }
-      row::block_sync();
-      if (commit) {  // the new chains and their records, for the next step (by slot and by row)
-        if (tid < s_nl) {
-          d.s_lm_chain[(size_t)slot * kLmChain + tid] = s_lm[tid];
-          d.s_lm_rec[(size_t)slot * kLmChain + tid] = s_lmr[tid];
-          d.m_lm[(size_t)r * kLmChain + tid] = s_lm[tid];
-          d.m_lmr[(size_t)r * kLmChain + tid] = s_lmr[tid];
-        }
-        if (tid >= 64 && tid - 64 < s_nt) {
-          const int k = tid - 64;
-          d.s_tr_chain[slot * kTrChain + k] = s_tr[k];
-          d.s_tr_rec[(size_t)slot * kTrChain + k] = s_trr[k];
-          d.m_tr[(size_t)r * kTrChain + k] = s_tr[k];
-          d.m_trr[(size_t)r * kTrChain + k] = s_trr[k];
-        }
       }
     } else if (tid == 0) {
       s_t += 1;
