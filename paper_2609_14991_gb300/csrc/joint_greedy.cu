@@ -382,7 +382,10 @@ __global__ void __launch_bounds__(kDThreads, 1)
       mbar_wait(accum, 0);
       if (DENSE) mbar_wait(dbar, 0);
     }
-    if (!DENSE && lane == 0) tma_store_wait_all();  // the staging buffers are read
+    // the staging buffers must have been read before the CTA's shared memory
+    // goes; the stores' writes complete with the grid (the row pass reads
+    // them after its dependency wait)
+    if (!DENSE && lane == 0) tma_store_wait_read<0>();
     __syncwarp();
     // merge the quadrant's warps' partials of each row: warps 1..kEW-1 of the
     // quadrant leave theirs in the drained stages, warp 0 combines and stores
