@@ -66,10 +66,9 @@ KERNEL_SOURCES = {
 }
 # keyed by (config, streams, kernel, fusion_path)
 TRAFFIC = {
-    (4, 1024, "joint", 1): (18074880, "826bf2360316aeca"),
     (4, 1024, "row", 1): (10575616, "673513be0b5541fe"),
-    (4, 1024, "joint", 0): (11051264, "826bf2360316aeca"),
-    (4, 1024, "row", 0): (29131776, "2608d2dffbbc0675"),
+    (4, 1024, "joint", 0): (11052032, "7c1347e63e44efbb"),
+    (4, 1024, "row", 0): (29131520, "4dc0d9aab66037e8"),
 }
 
 

@@ -363,7 +363,7 @@ TSD_API tsd_status tsd_decoder_check(tsd_decoder* dec);
  *   "joint_bn" 64, 128 or 256: labels per tensor-core CTA tile (default:
  *              chosen at create from the row count and the SM count);
  *   "fusion_path" 0 or 1, greedy decoding with at most one LM (default 0;
- *              1 is the faster form with a wide vocabulary and many streams):
+ *              1 keeps the V-wide logits out of memory):
  *              1 applies Eq. 1's level-0 LM term (a dense row per unigram
  *              state) in the joint kernel's epilogue and evaluates the other
  *              labels of the row's state (its longer contexts' continuations,

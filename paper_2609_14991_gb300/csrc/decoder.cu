@@ -235,9 +235,9 @@ tsd_status create_impl(const tsd_decoder_cfg* cfg, const void* W_out_bf16, const
     TSD_CUDA(cudaMemsetAsync(v.c_mask, 0, sizeof(uint32_t) * (size_t)d->M_pad * v.mask_words, s));
   }
   v.fused = fused ? 1 : 0;
-  // the streaming form by default; the dense epilogue (fusion_path 1) is the
-  // faster one with a wide vocabulary and many rows, its row pass no longer
-  // scanning every label
+  // the streaming form by default; the dense epilogue (fusion_path 1) keeps
+  // the V-wide logits out of memory and runs within a few percent of it with
+  // a wide vocabulary and many rows
   v.fz_dense = 0;
   const int topk = c.beam_k > 1 ? c.beam_k : c.prune_k;
   if (c.beam_k == 1 && c.prune_k > 0) {
