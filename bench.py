@@ -68,7 +68,7 @@ KERNEL_SOURCES = {
 TRAFFIC = {
     (4, 1024, "row", 1): (10575616, "673513be0b5541fe"),
     (4, 1024, "joint", 0): (11052032, "7c1347e63e44efbb"),
-    (4, 1024, "row", 0): (29131520, "4dc0d9aab66037e8"),
+    (4, 1024, "row", 0): (29132544, "9ff8457f4df50d2c"),
 }
 
 

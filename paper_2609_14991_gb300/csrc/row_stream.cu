@@ -54,7 +54,6 @@ using row::best_merge;
 using row::checked;
 using row::kNegInf;
 using row::lse_merge;
-using row::warp_find;
 
 constexpr int kFzThreads = 128;  // 4 warps: seven CTAs per SM at 72 registers
 constexpr int kStream = 4;       // level-0 arc groups of four per thread whose loads are issued together
@@ -63,6 +62,38 @@ constexpr int kFzWarps = kFzThreads / 32;
 
 // Aligned groups of four arcs a chain level's arcs [b, b + c) span.
 __device__ __forceinline__ int level_groups(int b, int c) { return c > 0 ? (b + c - (b & ~3) + 3) >> 2 : 0; }
+
+// Position of y in the sorted arr[0, n), or -1, by one warp: 32-ary probes
+// narrow the range to at most 124 entries, then one 16-byte load per lane
+// covers them (from the 16-byte boundary at or below arr + lo, so a window
+// reads at most three entries past the range: the tables' label arrays are
+// padded by four).  At most two dependent loads for n <= 3968.
+__device__ __forceinline__ int warp_find_wide(const int32_t* __restrict__ arr, int n, int y, int lane) {
+  row::reconverge();
+  int lo = 0, hi = n;
+  while (hi - lo > 124) {
+    const int step = (hi - lo + 31) >> 5;
+    const int idx = lo + lane * step;
+    const int v = (idx < hi) ? __ldg(arr + idx) : INT_MAX;
+    const unsigned m = __ballot_sync(0xffffffffu, v <= y);
+    if (m == 0) return -1;
+    lo = lo + (31 - __clz((int)m)) * step;
+    hi = min(hi, lo + step);
+  }
+  const uintptr_t at = reinterpret_cast<uintptr_t>(arr + lo);
+  const int4* g = reinterpret_cast<const int4*>(at & ~uintptr_t(15));
+  const int first = 4 * lane - (int)((at & 15u) >> 2);  // this lane's first entry, relative to lo
+  int pos = -1;
+  if (first < hi - lo) {
+    const int4 t = __ldg(g + lane);
+    const int tv[4] = {t.x, t.y, t.z, t.w};
+#pragma unroll
+    for (int j = 3; j >= 0; --j)
+      if (first + j >= 0 && first + j < hi - lo && tv[j] == y) pos = lo + first + j;
+  }
+  const unsigned m = __ballot_sync(0xffffffffu, pos >= 0);
+  return m ? __shfl_sync(0xffffffffu, pos, __ffs((int)m) - 1) : -1;
+}
 
 // mode: 0 = label step, 1 = final step (apply the last decision only),
 // 2 = replay (redo the step's work without committing any state or output;
@@ -485,13 +516,13 @@ __global__ void __launch_bounds__(kFzThreads) __maxnreg__((VAR & 4) ? 128 : 72) 
       for (int task = warp; task < nl_old + nt_old; task += kFzWarps) {
         if (task < nl_old) {
           const int b = s_lmr[task].x, c = s_lmr[task].y;
-          const int i = warp_find(d.lm.arc_tok + b, c, y, lane);
+          const int i = warp_find_wide(d.lm.arc_tok + b, c, y, lane);
           if (lane == 0) s_lm_hit[task] = (i >= 0) ? __ldg(d.lm.arc_rec + b + i) : make_int4(-2, 0, 0, 0);
           if (counting && lane == 0) atomicAdd(&s_bytes, 4ull * (32 - __clz(c + 1)) + 16);
         } else {
           const int k = task - nl_old;
           const int b = s_trr[k].x, c = s_trr[k].y;
-          const int i = warp_find(d.tr.ch_tok + b, c, y, lane);
+          const int i = warp_find_wide(d.tr.ch_tok + b, c, y, lane);
           if (lane == 0) s_tr_hit[k] = (i >= 0) ? __ldg(d.tr.ch_rec + b + i) : make_int4(-1, 0, 0, 0);
           if (counting && lane == 0) atomicAdd(&s_bytes, 4ull * (32 - __clz(c + 1)) + 16);
         }
