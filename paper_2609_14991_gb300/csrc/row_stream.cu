@@ -65,9 +65,10 @@ __device__ __forceinline__ int level_groups(int b, int c) { return c > 0 ? (b + 
 
 // Position of y in the sorted arr[0, n), or -1, by one warp: 32-ary probes
 // narrow the range to at most 124 entries, then one 16-byte load per lane
-// covers them (from the 16-byte boundary at or below arr + lo, so a window
-// reads at most three entries past the range: the tables' label arrays are
-// padded by four).  At most two dependent loads for n <= 3968.
+// covers them, from the 16-byte boundary at or below arr + lo.  A window so
+// reads at most three entries before and after the range, inside the table
+// (its label arrays start 16-byte aligned and are padded by four).  At most
+// two dependent loads for n <= 3968.
 __device__ __forceinline__ int warp_find_wide(const int32_t* __restrict__ arr, int n, int y, int lane) {
   row::reconverge();
   int lo = 0, hi = n;
