@@ -231,7 +231,7 @@ def variant_config(args, w, extra):
         out["prune_k"] = args.prune_k
         names.append(f"fusion pruned to the acoustic top {args.prune_k}")
     if w.beam == 1 and not args.prune_k and not extra:
-        out["fusion_path"] = 0 if args.fusion_path == 0 else 1
+        out["fusion_path"] = 1 if args.fusion_path == 1 else 0  # the decoder's default: 0
     if args.pred:
         out["prediction_network"] = {"kind": "1-layer LSTM over the previous label", "D": args.pred, "H_enc": w.H}
         names.append(f"stateful form: LSTM prediction network D={args.pred} + joint projections")
